@@ -1,0 +1,231 @@
+/*
+ * milo.h -- C ABI of libmilo: decode attention over a many-shot prefix whose
+ * KV cache is stored block-wise in low-rank form (MILO, Sec. 4.2-4.4).
+ *
+ * The paper stores, per block i of the prefix and per KV head, the truncated
+ * SVD factors of the block's keys and values (Eq. 3):
+ *     K_i ~ A^k_i S^k_i (B^k_i)^T,   V_i ~ A^v_i S^v_i (B^v_i)^T,
+ * with per-block ranks r^k_i, r^v_i chosen by the entropy-driven allocation
+ * (Eq. 5-7).  At inference (Alg. 1, Stage 2) a query attends (Eq. 1) to the
+ * selected blocks' reconstructed keys and values.  This library computes that
+ * attention exactly (up to floating-point rounding) without reconstructing:
+ *     q . K^_i^T = (q P^k_i^T) (C^k_i)^T,   p V^_i = (p C^v_i) P^v_i,
+ * where C = A S (singular values folded into the coefficients, n_i x r) and
+ * P = B^T (r x d, orthonormal rows in the paper's setting; not required).
+ *
+ * Conventions for every entry point:
+ *  - Return a milo_status_t; no exceptions or aborts cross the ABI.
+ *  - "device" pointers are CUDA global memory of the current device; "host"
+ *    pointers are ordinary CPU memory.  The caller owns every buffer it passes.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *  - bf16 arrays hold IEEE bfloat16 values.
+ */
+#ifndef MILO_H
+#define MILO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MILO_OK = 0,
+    MILO_ERR_INVALID_ARG = 1,   /* null pointer, bad size, unsupported head dim ...  */
+    MILO_ERR_BAD_TABLE = 2,     /* block table inconsistent (lengths, ranks, bounds)  */
+    MILO_ERR_ALIGNMENT = 3,     /* an offset or pointer is not 16-byte aligned        */
+    MILO_ERR_UNSUPPORTED = 4,   /* valid but outside what the kernels implement       */
+    MILO_ERR_CUDA = 5,          /* a CUDA runtime call failed                         */
+    MILO_ERR_TIMEOUT = 6,       /* device: a bounded wait gave up (sticky word)       */
+    MILO_ERR_DEVICE_BOUNDS = 7, /* device: an index check failed (sticky word)        */
+    MILO_ERR_WORKSPACE = 8      /* workspace missing or smaller than required         */
+} milo_status_t;
+
+/* Short English description of a status code (static string). */
+const char *milo_status_string(int32_t status);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int32_t milo_version(void);
+
+/* Human-readable detail of the last error returned on the calling thread
+ * (empty string if none).  Valid until the thread's next libmilo call. */
+const char *milo_last_error_message(void);
+
+/*
+ * Block table of one decoder layer (the paper's low-rank cache LC, Alg. 1).
+ * Entry e = b * num_kv_heads + g describes block b, KV head g.  The table's
+ * block order is the attention order; passing a subset of blocks is the
+ * paper's retrieval selection (Alg. 1, Stage 2).
+ *
+ *   num_blocks    >= 0 (0 = no prefix; only tails are attended).
+ *   num_kv_heads  >= 1.
+ *   head_dim      64 or 128.
+ *   block_len     host [num_blocks]: tokens n_b of block b, 1 <= n_b <= 65536
+ *                 (blocks may differ in length: a block holds m_i examples).
+ *   rank_k/v      host [num_blocks * num_kv_heads]: 0 <= r <= head_dim.
+ *                 A rank of 0 stores an all-zero key (or value) block.
+ *   off_ck/pk/cv/pv host [num_blocks * num_kv_heads]: element offsets into
+ *                 `arena` of C^K (n_b x r^k), P^K (r^k x d), C^V (n_b x r^v),
+ *                 P^V (r^v x d), each row-major and dense; each offset a
+ *                 multiple of 8 elements (16 bytes).  Regions must lie inside
+ *                 [0, arena_elems) and must not overlap.
+ *   arena         device bf16 [arena_elems], 16-byte aligned.  Read only by
+ *                 milo_prefix_create; it may be freed after that call returns.
+ *   arena_elems   size of `arena` in elements.
+ */
+typedef struct {
+    int32_t num_blocks;
+    int32_t num_kv_heads;
+    int32_t head_dim;
+    const int32_t *block_len;
+    const int32_t *rank_k;
+    const int32_t *rank_v;
+    const int64_t *off_ck;
+    const int64_t *off_pk;
+    const int64_t *off_cv;
+    const int64_t *off_pv;
+    const void *arena;
+    int64_t arena_elems;
+} milo_block_table_t;
+
+/* Opaque per-layer plan: packed factors, static work partition, counters. */
+typedef struct milo_prefix milo_prefix_t;
+
+/*
+ * Check a block table on the host (no device access): lengths, ranks,
+ * alignment, bounds, and pairwise overlap of the factor regions.
+ * Returns MILO_OK, MILO_ERR_INVALID_ARG, MILO_ERR_BAD_TABLE or
+ * MILO_ERR_ALIGNMENT.  milo_prefix_create runs the same checks.
+ */
+milo_status_t milo_validate_table(const milo_block_table_t *table);
+
+/*
+ * Packed ("kernel-native") layout of the factors, computed on the host.
+ * Each factor is stored zero-padded to r8 = roundup(r, 8) ranks and, for the
+ * coefficient matrices, n8 = roundup(n_b, 8) tokens, as 8x8 bf16 tiles of 128
+ * contiguous bytes (one tile = 8 rows x 16 bytes):
+ *   C (n_b x r): token tiles of 64 tokens; the token tile k that holds t8
+ *     padded tokens occupies t8 * r8 * 2 bytes starting at k * 64 * r8 * 2;
+ *     inside it, tile (rank group rg, token group tg) sits at
+ *     (rg * t8/8 + tg) * 128 and holds row (t % 8), column (j % 8).
+ *   P (r x d): tile (rank group jg, column group cg) sits at
+ *     (jg * d/8 + cg) * 128 and holds row (j % 8), column (c % 8).
+ * packed_offsets: host [num_blocks * num_kv_heads * 4] byte offsets of
+ * (C^K, P^K, C^V, P^V) for every entry (128-byte aligned); total_bytes: size
+ * of the packed arena.  Either output may be NULL.
+ */
+milo_status_t milo_packed_layout(const milo_block_table_t *table,
+                                 int64_t *packed_offsets, int64_t *total_bytes);
+
+/*
+ * Static prefix work partition the decode kernel uses, computed on the host.
+ * The prefix (every entry's tokens, KV-head-major, then block order) is cut
+ * at 64-token boundaries into segments so that each of `num_ctas` thread
+ * blocks receives a near-equal share of the cost line, where a token costs its
+ * padded coefficient bytes plus 32 (the softmax work), a block's P^K is charged
+ * with its first 64-token tile and its P^V with its last; a tile goes to the
+ * thread block whose share holds the midpoint of the tile's cost.  Consecutive segments
+ * of one thread block with the same KV head form a "run" whose partial result
+ * occupies one slot.
+ *   seg_entry/seg_t0/seg_t1/seg_slot: host arrays of capacity `max_segments`
+ *     (entry index, token range [t0, t1), slot); may be NULL to query count.
+ *   cta_begin: host [num_ctas + 1] first segment of each thread block; may
+ *     be NULL.
+ *   num_segments/num_slots: outputs (either may be NULL).
+ * Returns MILO_ERR_INVALID_ARG if max_segments is too small.
+ */
+milo_status_t milo_partition_prefix(const milo_block_table_t *table,
+                                    int32_t num_ctas, int32_t max_segments,
+                                    int32_t *seg_entry, int32_t *seg_t0,
+                                    int32_t *seg_t1, int32_t *seg_slot,
+                                    int32_t *cta_begin, int32_t *num_segments,
+                                    int32_t *num_slots);
+
+/*
+ * Build a plan for one layer on the current device: validate the table,
+ * allocate and fill the packed arena (a pack kernel on `stream`, then a
+ * stream synchronisation), build the work partition and the device-side
+ * counters.  The logical arena may be freed after this call returns.
+ *   num_q_heads   multiple of num_kv_heads (query head h reads KV head
+ *                 h / (num_q_heads / num_kv_heads)).
+ *   max_batch     largest batch any decode call on this plan will use.
+ *   out_plan      receives the plan; release with milo_prefix_destroy.
+ */
+milo_status_t milo_prefix_create(const milo_block_table_t *table,
+                                 int32_t num_q_heads, int32_t max_batch,
+                                 void *stream, milo_prefix_t **out_plan);
+
+/* Free a plan and its device memory (synchronises the device first). */
+milo_status_t milo_prefix_destroy(milo_prefix_t *plan);
+
+/* Plan facts for accounting and tests. */
+typedef struct {
+    int32_t num_blocks, num_kv_heads, num_q_heads, head_dim, max_batch;
+    int32_t num_ctas;             /* thread blocks of the decode kernel       */
+    int32_t num_segments;         /* prefix segments of the partition         */
+    int32_t num_slots;            /* prefix partial slots (runs)              */
+    int64_t prefix_tokens;        /* sum of block lengths                     */
+    int64_t logical_factor_bytes; /* bytes of C^K,P^K,C^V,P^V at true ranks   */
+    int64_t packed_bytes;         /* bytes of the packed arena (with padding) */
+    const void *packed_arena;     /* device pointer to the packed arena       */
+} milo_prefix_info_t;
+
+milo_status_t milo_prefix_get_info(const milo_prefix_t *plan,
+                                   milo_prefix_info_t *info);
+
+/*
+ * Workspace a decode call needs (device memory the caller provides): the
+ * split-softmax partial results (running max, sum and output per partition
+ * of the tokens, Eq. 1 split over token ranges).  `bytes` receives the size.
+ */
+milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
+                                  int64_t max_tail_tokens, size_t *bytes);
+
+/*
+ * One decode-attention call for one layer (Alg. 1 Stage 2 + Eq. 1):
+ * for every query i and query head h (KV head g = h / G),
+ *   out[i, h] = softmax(scale * q[i,h] . [K^_1 .. K^_N, Ktail_i[:, g]]) [V^ ...].
+ *   q            device bf16 [batch, num_q_heads, head_dim].
+ *   batch        1 <= batch <= plan's max_batch.
+ *   tail_k/v     device bf16 [tail_rows, num_kv_heads, head_dim], 16-byte
+ *                aligned; may be NULL when max_tail_tokens == 0.
+ *   tail_offsets device int64 [batch + 1]: query i's tail is rows
+ *                tail_offsets[i] .. tail_offsets[i+1]-1 (cu_seqlens style;
+ *                nondecreasing, tail_offsets[batch] <= tail_rows).  May be NULL
+ *                when max_tail_tokens == 0.
+ *   tail_rows    rows allocated in tail_k / tail_v.
+ *   max_tail_tokens  host upper bound on every query's tail length; it sets
+ *                how the tails are split, a longer tail is an error recorded
+ *                in the device status word (MILO_ERR_DEVICE_BOUNDS).
+ *   softmax_scale  <= 0 selects 1 / sqrt(head_dim).
+ *   out          device fp32 [batch, num_q_heads, head_dim].
+ *   workspace    device, at least milo_workspace_size bytes, 256-byte aligned.
+ * Asynchronous on `stream`: no host synchronisation and no allocation, so the
+ * call can be captured in a CUDA graph.  Launched with programmatic dependent
+ * launch: the kernel may begin streaming the plan's factors before the
+ * preceding kernel on `stream` finishes, and reads q, the tails and the
+ * workspace only after it has.  A plan must not be used by two calls that can
+ * run concurrently (it holds per-call counters).  A query whose prefix and
+ * tail are both empty yields NaN.
+ */
+milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q,
+                               int32_t batch, const void *tail_k,
+                               const void *tail_v, const int64_t *tail_offsets,
+                               int64_t tail_rows, int64_t max_tail_tokens,
+                               float softmax_scale, float *out, void *workspace,
+                               size_t workspace_bytes, void *stream);
+
+/*
+ * Read (and optionally clear) the plan's sticky device status word, which the
+ * kernels set on a timed-out wait (MILO_ERR_TIMEOUT) or a failed device-side
+ * index check (MILO_ERR_DEVICE_BOUNDS).  Synchronises `stream`.
+ */
+milo_status_t milo_get_device_status(const milo_prefix_t *plan, void *stream,
+                                     int32_t clear, int32_t *code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MILO_H */

@@ -1,0 +1,551 @@
+// milo_host.cpp -- host side of the libmilo C ABI (include/milo.h):
+// table validation, packed layout, static work partition, plan lifecycle and
+// the decode launch.  No exception crosses the ABI.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "milo.h"
+#include "milo_internal.h"
+
+using namespace milo;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+milo_status_t cuda_fail(cudaError_t e, const char *what)
+{
+    g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+    return MILO_ERR_CUDA;
+}
+
+milo_status_t fail(milo_status_t s, const std::string &msg)
+{
+    g_last_error = msg;
+    return s;
+}
+
+inline int r8(int r) { return (r + 7) & ~7; }
+inline int64_t align_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+struct Seg {
+    int32_t entry, t0, t1, slot, flags;
+};
+
+milo_status_t validate(const milo_block_table_t *t)
+{
+    if (!t) return fail(MILO_ERR_INVALID_ARG, "table is null");
+    if (t->num_blocks < 0 || t->num_kv_heads < 1)
+        return fail(MILO_ERR_INVALID_ARG, "num_blocks < 0 or num_kv_heads < 1");
+    if (t->head_dim != 64 && t->head_dim != 128)
+        return fail(MILO_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
+    if (t->num_blocks == 0) return MILO_OK;
+    if (!t->block_len || !t->rank_k || !t->rank_v || !t->off_ck || !t->off_pk || !t->off_cv || !t->off_pv)
+        return fail(MILO_ERR_INVALID_ARG, "null table array");
+    if (t->arena_elems < 0) return fail(MILO_ERR_INVALID_ARG, "arena_elems < 0");
+    if (t->arena_elems > 0 && !t->arena) return fail(MILO_ERR_INVALID_ARG, "arena is null");
+    if (reinterpret_cast<uintptr_t>(t->arena) % 16 != 0)
+        return fail(MILO_ERR_ALIGNMENT, "arena is not 16-byte aligned");
+    const int d = t->head_dim, H = t->num_kv_heads;
+    struct Region { int64_t a, b; };
+    std::vector<Region> regions;
+    regions.reserve((size_t)t->num_blocks * H * 4);
+    for (int b = 0; b < t->num_blocks; ++b) {
+        const int n = t->block_len[b];
+        if (n < 1 || n > 65536) return fail(MILO_ERR_BAD_TABLE, "block length outside [1, 65536]");
+        for (int g = 0; g < H; ++g) {
+            const int64_t e = (int64_t)b * H + g;
+            const int rk = t->rank_k[e], rv = t->rank_v[e];
+            if (rk < 0 || rk > d || rv < 0 || rv > d) return fail(MILO_ERR_BAD_TABLE, "rank outside [0, head_dim]");
+            const int64_t off[4] = {t->off_ck[e], t->off_pk[e], t->off_cv[e], t->off_pv[e]};
+            const int64_t sz[4] = {(int64_t)n * rk, (int64_t)rk * d, (int64_t)n * rv, (int64_t)rv * d};
+            for (int f = 0; f < 4; ++f) {
+                if (off[f] % 8 != 0) return fail(MILO_ERR_ALIGNMENT, "factor offset not a multiple of 8 elements");
+                if (off[f] < 0 || off[f] + sz[f] > t->arena_elems)
+                    return fail(MILO_ERR_BAD_TABLE, "factor region outside the arena");
+                if (sz[f] > 0) regions.push_back({off[f], off[f] + sz[f]});
+            }
+        }
+    }
+    std::sort(regions.begin(), regions.end(), [](const Region &x, const Region &y) { return x.a < y.a; });
+    for (size_t i = 1; i < regions.size(); ++i)
+        if (regions[i].a < regions[i - 1].b) return fail(MILO_ERR_BAD_TABLE, "factor regions overlap");
+    return MILO_OK;
+}
+
+// Packed byte offsets [E][4] (C^K, P^K, C^V, P^V), each 128-byte aligned.
+int64_t packed_layout(const milo_block_table_t *t, std::vector<int64_t> &offs)
+{
+    const int H = t->num_kv_heads, d = t->head_dim;
+    const int64_t E = (int64_t)t->num_blocks * H;
+    offs.assign((size_t)E * 4, 0);
+    int64_t cur = 0;
+    for (int64_t e = 0; e < E; ++e) {
+        const int n8 = (t->block_len[e / H] + 7) & ~7;
+        const int64_t sz[4] = {(int64_t)n8 * r8(t->rank_k[e]) * 2, (int64_t)r8(t->rank_k[e]) * d * 2,
+                               (int64_t)n8 * r8(t->rank_v[e]) * 2, (int64_t)r8(t->rank_v[e]) * d * 2};
+        for (int f = 0; f < 4; ++f) {
+            offs[(size_t)e * 4 + f] = cur;
+            cur = align_up(cur + sz[f], 128);
+        }
+    }
+    return cur;
+}
+
+// Static partition of the prefix over `P` thread blocks (see milo.h).
+void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::vector<int32_t> &cta_begin,
+               int &num_slots, std::vector<int32_t> *g_slot_begin)
+{
+    const int H = t->num_kv_heads, d = t->head_dim, nb = t->num_blocks;
+    constexpr int64_t kTokenOverhead = 32;  // softmax work per token, in byte-equivalents
+    auto tile_cost = [&](int e, int t8) {
+        return (int64_t)t8 * ((r8(t->rank_k[e]) + r8(t->rank_v[e])) * 2 + kTokenOverhead);
+    };
+    auto seg_cost = [&](int e) { return (int64_t)(r8(t->rank_k[e]) + r8(t->rank_v[e])) * d * 2; };
+    int64_t total = 0;
+    for (int g = 0; g < H; ++g)
+        for (int b = 0; b < nb; ++b) {
+            const int e = b * H + g, n = t->block_len[b];
+            total += seg_cost(e);
+            for (int t0 = 0; t0 < n; t0 += kTileTokens) total += tile_cost(e, (std::min(n - t0, kTileTokens) + 7) & ~7);
+        }
+    segs.clear();
+    cta_begin.assign((size_t)P + 1, 0);
+    // Cost line: entries (KV-head-major, then block order), each charged its
+    // 64-token tiles, with P^K charged to the first tile and P^V to the last.  A tile
+    // belongs to the thread block whose share (c total/P, (c+1) total/P]
+    // contains the midpoint of the tile's cost interval.  A block cut between
+    // two thread blocks is read again for its bases by the second (from L2).
+    int cta = 0;
+    int64_t pos = 0;
+    for (int g = 0; g < H; ++g)
+        for (int b = 0; b < nb; ++b) {
+            const int e = b * H + g, n = t->block_len[b];
+            bool open = false;
+            for (int t0 = 0; t0 < n; t0 += kTileTokens) {
+                const int t1 = std::min(n, t0 + kTileTokens);
+                // P^K is charged with the first tile, P^V with the last
+                const int64_t c = tile_cost(e, (t1 - t0 + 7) & ~7) +
+                                  (t0 == 0 ? (int64_t)r8(t->rank_k[e]) * d * 2 : 0) +
+                                  (t1 == n ? (int64_t)r8(t->rank_v[e]) * d * 2 : 0);
+                const double mid = (double)pos + 0.5 * (double)c;
+                int owner = total > 0 ? (int)(mid * P / (double)total) : 0;
+                owner = std::min(std::max(owner, cta), P - 1);
+                if (owner != cta) {
+                    for (int x = cta + 1; x <= owner; ++x) cta_begin[x] = (int32_t)segs.size();
+                    cta = owner;
+                    open = false;
+                }
+                if (!open) {
+                    segs.push_back({e, t0, t0, 0, 0});
+                    open = true;
+                }
+                segs.back().t1 = t1;
+                pos += c;
+            }
+        }
+    for (int c = cta + 1; c <= P; ++c) cta_begin[c] = (int32_t)segs.size();
+    // runs and slots: consecutive segments of one thread block with one KV head
+    num_slots = 0;
+    if (g_slot_begin) g_slot_begin->assign((size_t)H + 1, 0);
+    std::vector<int32_t> first_slot_of_g((size_t)H, -1);
+    for (int c = 0; c < P; ++c) {
+        int prev_g = -1;
+        for (int s = cta_begin[c]; s < cta_begin[c + 1]; ++s) {
+            const int g = segs[s].entry % H;
+            if (g != prev_g) {
+                segs[s].flags |= kSegFirstOfRun;
+                if (s > cta_begin[c]) segs[s - 1].flags |= kSegLastOfRun;
+                if (first_slot_of_g[g] < 0) first_slot_of_g[g] = num_slots;
+                ++num_slots;
+                prev_g = g;
+            }
+            segs[s].slot = num_slots - 1;
+        }
+        if (cta_begin[c + 1] > cta_begin[c]) segs[cta_begin[c + 1] - 1].flags |= kSegLastOfRun;
+    }
+    if (g_slot_begin) {
+        // slots are numbered in KV-head order, so each head's slots are contiguous
+        auto &gs = *g_slot_begin;
+        gs[H] = num_slots;
+        for (int g = H - 1; g >= 0; --g) gs[g] = first_slot_of_g[g] >= 0 ? first_slot_of_g[g] : gs[g + 1];
+    }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+}  // namespace
+
+struct milo_prefix {
+    int device = 0;
+    int nb = 0, hkv = 0, hq = 0, d = 0, G = 0, max_batch = 0;
+    int num_ctas = 0, num_segments = 0, num_slots = 0, max_nrg = 0;
+    int64_t prefix_tokens = 0, logical_bytes = 0, packed_bytes = 0;
+    uint8_t *packed = nullptr;
+    EntryDev *entries = nullptr;
+    SegDev *segs = nullptr;
+    int32_t *cta_seg_begin = nullptr;
+    int32_t *g_slot_begin = nullptr;
+    CountersDev *counters = nullptr;
+    uint32_t *tickets = nullptr;
+    int32_t *status = nullptr;
+};
+
+extern "C" {
+
+const char *milo_status_string(int32_t s)
+{
+    switch (s) {
+    case MILO_OK: return "ok";
+    case MILO_ERR_INVALID_ARG: return "invalid argument";
+    case MILO_ERR_BAD_TABLE: return "inconsistent block table";
+    case MILO_ERR_ALIGNMENT: return "misaligned pointer or offset";
+    case MILO_ERR_UNSUPPORTED: return "unsupported configuration";
+    case MILO_ERR_CUDA: return "CUDA runtime error";
+    case MILO_ERR_TIMEOUT: return "device wait timed out";
+    case MILO_ERR_DEVICE_BOUNDS: return "device-side bounds check failed";
+    case MILO_ERR_WORKSPACE: return "workspace missing or too small";
+    default: return "unknown status";
+    }
+}
+
+int32_t milo_version(void) { return 100; }
+
+const char *milo_last_error_message(void) { return g_last_error.c_str(); }
+
+milo_status_t milo_validate_table(const milo_block_table_t *table) { return validate(table); }
+
+milo_status_t milo_packed_layout(const milo_block_table_t *table, int64_t *packed_offsets, int64_t *total_bytes)
+{
+    milo_status_t s = validate(table);
+    if (s != MILO_OK) return s;
+    std::vector<int64_t> offs;
+    const int64_t total = packed_layout(table, offs);
+    if (packed_offsets) std::memcpy(packed_offsets, offs.data(), offs.size() * sizeof(int64_t));
+    if (total_bytes) *total_bytes = total;
+    return MILO_OK;
+}
+
+milo_status_t milo_partition_prefix(const milo_block_table_t *table, int32_t num_ctas, int32_t max_segments,
+                                    int32_t *seg_entry, int32_t *seg_t0, int32_t *seg_t1, int32_t *seg_slot,
+                                    int32_t *cta_begin, int32_t *num_segments, int32_t *num_slots)
+{
+    milo_status_t s = validate(table);
+    if (s != MILO_OK) return s;
+    if (num_ctas < 1) return fail(MILO_ERR_INVALID_ARG, "num_ctas < 1");
+    std::vector<Seg> segs;
+    std::vector<int32_t> cb;
+    int ns = 0;
+    partition(table, num_ctas, segs, cb, ns, nullptr);
+    if (num_segments) *num_segments = (int32_t)segs.size();
+    if (num_slots) *num_slots = ns;
+    if (cta_begin) std::memcpy(cta_begin, cb.data(), cb.size() * sizeof(int32_t));
+    if (seg_entry || seg_t0 || seg_t1 || seg_slot) {
+        if ((int64_t)segs.size() > max_segments) return fail(MILO_ERR_INVALID_ARG, "max_segments too small");
+        for (size_t i = 0; i < segs.size(); ++i) {
+            if (seg_entry) seg_entry[i] = segs[i].entry;
+            if (seg_t0) seg_t0[i] = segs[i].t0;
+            if (seg_t1) seg_t1[i] = segs[i].t1;
+            if (seg_slot) seg_slot[i] = segs[i].slot;
+        }
+    }
+    return MILO_OK;
+}
+
+milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
+{
+    if (!plan) return MILO_OK;
+    int cur = 0;
+    cudaGetDevice(&cur);
+    cudaSetDevice(plan->device);
+    cudaDeviceSynchronize();
+    cudaFree(plan->packed);
+    cudaFree(plan->entries);
+    cudaFree(plan->segs);
+    cudaFree(plan->cta_seg_begin);
+    cudaFree(plan->g_slot_begin);
+    cudaFree(plan->counters);
+    cudaFree(plan->status);
+    cudaSetDevice(cur);
+    delete plan;
+    return MILO_OK;
+}
+
+milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_heads, int32_t max_batch,
+                                 void *stream_, milo_prefix_t **out_plan)
+{
+    if (!out_plan) return fail(MILO_ERR_INVALID_ARG, "out_plan is null");
+    *out_plan = nullptr;
+    milo_status_t s = validate(table);
+    if (s != MILO_OK) return s;
+    if (num_q_heads < 1 || num_q_heads % table->num_kv_heads != 0)
+        return fail(MILO_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
+    if (max_batch < 1) return fail(MILO_ERR_INVALID_ARG, "max_batch < 1");
+    const int G = num_q_heads / table->num_kv_heads;
+    if (G > 32) return fail(MILO_ERR_UNSUPPORTED, "more than 32 query heads per KV head");
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+
+    milo_prefix *p = new (std::nothrow) milo_prefix;
+    if (!p) return fail(MILO_ERR_INVALID_ARG, "out of host memory");
+    cudaError_t e = cudaGetDevice(&p->device);
+    if (e != cudaSuccess) { delete p; return cuda_fail(e, "cudaGetDevice"); }
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
+    if (e != cudaSuccess) { delete p; return cuda_fail(e, "cudaDeviceGetAttribute"); }
+    const int H = table->num_kv_heads, d = table->head_dim, nb = table->num_blocks;
+    p->nb = nb; p->hkv = H; p->hq = num_q_heads; p->d = d; p->G = G; p->max_batch = max_batch;
+    p->num_ctas = sms;
+    p->max_nrg = (max_batch * G + 7) / 8;
+
+    std::vector<int64_t> poffs;
+    p->packed_bytes = packed_layout(table, poffs);
+    std::vector<Seg> segs;
+    std::vector<int32_t> cta_begin, g_slot;
+    partition(table, p->num_ctas, segs, cta_begin, p->num_slots, &g_slot);
+    p->num_segments = (int)segs.size();
+
+    const int64_t E = (int64_t)nb * H;
+    std::vector<EntryDev> ents((size_t)E);
+    std::vector<int64_t> loffs((size_t)E * 4);
+    for (int64_t x = 0; x < E; ++x) {
+        EntryDev &en = ents[(size_t)x];
+        en.off_ck = poffs[(size_t)x * 4 + 0];
+        en.off_pk = poffs[(size_t)x * 4 + 1];
+        en.off_cv = poffs[(size_t)x * 4 + 2];
+        en.off_pv = poffs[(size_t)x * 4 + 3];
+        en.n = table->block_len[x / H];
+        en.rk = table->rank_k[x];
+        en.rv = table->rank_v[x];
+        en.g = (int)(x % H);
+        loffs[(size_t)x * 4 + 0] = table->off_ck[x];
+        loffs[(size_t)x * 4 + 1] = table->off_pk[x];
+        loffs[(size_t)x * 4 + 2] = table->off_cv[x];
+        loffs[(size_t)x * 4 + 3] = table->off_pv[x];
+        p->prefix_tokens += (x % H == 0) ? en.n : 0;
+        p->logical_bytes += ((int64_t)en.n * (en.rk + en.rv) + (int64_t)(en.rk + en.rv) * d) * 2;
+    }
+    std::vector<SegDev> sd(segs.size());
+    for (size_t i = 0; i < segs.size(); ++i) {
+        sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
+    }
+
+    int64_t *loff_dev = nullptr;
+    auto cleanup = [&](cudaError_t err, const char *what) {
+        cudaFree(loff_dev);
+        milo_prefix_destroy(p);
+        return cuda_fail(err, what);
+    };
+    const size_t cnt_bytes = sizeof(CountersDev) + sizeof(uint32_t) * (size_t)H * p->max_nrg;
+    if ((e = cudaMalloc(&p->packed, (size_t)std::max<int64_t>(p->packed_bytes, 128))) != cudaSuccess)
+        return cleanup(e, "cudaMalloc packed");
+    if ((e = cudaMalloc(&p->entries, sizeof(EntryDev) * std::max<size_t>(ents.size(), 1))) != cudaSuccess)
+        return cleanup(e, "cudaMalloc entries");
+    if ((e = cudaMalloc(&p->segs, sizeof(SegDev) * std::max<size_t>(sd.size(), 1))) != cudaSuccess)
+        return cleanup(e, "cudaMalloc segs");
+    if ((e = cudaMalloc(&p->cta_seg_begin, sizeof(int32_t) * cta_begin.size())) != cudaSuccess)
+        return cleanup(e, "cudaMalloc cta_seg_begin");
+    if ((e = cudaMalloc(&p->g_slot_begin, sizeof(int32_t) * g_slot.size())) != cudaSuccess)
+        return cleanup(e, "cudaMalloc g_slot_begin");
+    if ((e = cudaMalloc(&p->counters, cnt_bytes)) != cudaSuccess) return cleanup(e, "cudaMalloc counters");
+    if ((e = cudaMalloc(&p->status, sizeof(int32_t))) != cudaSuccess) return cleanup(e, "cudaMalloc status");
+    if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
+        return cleanup(e, "cudaMalloc offsets");
+    p->tickets = reinterpret_cast<uint32_t *>(p->counters + 1);
+
+    if (!ents.empty() &&
+        (e = cudaMemcpyAsync(p->entries, ents.data(), sizeof(EntryDev) * ents.size(), cudaMemcpyHostToDevice,
+                             stream)) != cudaSuccess)
+        return cleanup(e, "copy entries");
+    if (!sd.empty() && (e = cudaMemcpyAsync(p->segs, sd.data(), sizeof(SegDev) * sd.size(), cudaMemcpyHostToDevice,
+                                            stream)) != cudaSuccess)
+        return cleanup(e, "copy segs");
+    if ((e = cudaMemcpyAsync(p->cta_seg_begin, cta_begin.data(), sizeof(int32_t) * cta_begin.size(),
+                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+        return cleanup(e, "copy cta_seg_begin");
+    if ((e = cudaMemcpyAsync(p->g_slot_begin, g_slot.data(), sizeof(int32_t) * g_slot.size(),
+                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+        return cleanup(e, "copy g_slot_begin");
+    if (!loffs.empty() && (e = cudaMemcpyAsync(loff_dev, loffs.data(), sizeof(int64_t) * loffs.size(),
+                                               cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+        return cleanup(e, "copy offsets");
+    if ((e = cudaMemsetAsync(p->counters, 0, cnt_bytes, stream)) != cudaSuccess) return cleanup(e, "memset counters");
+    if ((e = cudaMemsetAsync(p->status, 0, sizeof(int32_t), stream)) != cudaSuccess) return cleanup(e, "memset status");
+    if ((e = launch_pack(table->arena, p->entries, loff_dev, (int)E, d, p->packed, p->packed_bytes, stream)) !=
+        cudaSuccess)
+        return cleanup(e, "pack kernel");
+    if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cleanup(e, "synchronize after pack");
+    cudaFree(loff_dev);
+    *out_plan = p;
+    return MILO_OK;
+}
+
+milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t *info)
+{
+    if (!plan || !info) return fail(MILO_ERR_INVALID_ARG, "null argument");
+    info->num_blocks = plan->nb;
+    info->num_kv_heads = plan->hkv;
+    info->num_q_heads = plan->hq;
+    info->head_dim = plan->d;
+    info->max_batch = plan->max_batch;
+    info->num_ctas = plan->num_ctas;
+    info->num_segments = plan->num_segments;
+    info->num_slots = plan->num_slots;
+    info->prefix_tokens = plan->prefix_tokens;
+    info->logical_factor_bytes = plan->logical_bytes;
+    info->packed_bytes = plan->packed_bytes;
+    info->packed_arena = plan->packed;
+    return MILO_OK;
+}
+
+namespace {
+struct CallShape {
+    int rows_g, nrg, nrg_cta, npass, nrg_t, S;
+    int64_t records;
+};
+
+CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
+{
+    CallShape c;
+    c.rows_g = batch * p->G;
+    c.nrg = (c.rows_g + 7) / 8;
+    c.nrg_cta = c.nrg >= 3 ? 4 : (c.nrg == 2 ? 2 : 1);
+    c.npass = (c.nrg + c.nrg_cta - 1) / c.nrg_cta;
+    c.nrg_t = (p->G + 7) / 8;
+    c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
+    c.records = (int64_t)p->num_slots * c.nrg + (int64_t)batch * p->hkv * c.S * c.nrg_t;
+    return c;
+}
+}  // namespace
+
+milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch, int64_t max_tail_tokens, size_t *bytes)
+{
+    if (!plan || !bytes) return fail(MILO_ERR_INVALID_ARG, "null argument");
+    if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
+    if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
+    const CallShape c = call_shape(plan, batch, max_tail_tokens);
+    *bytes = (size_t)std::max<int64_t>(c.records, 1) * (8 * plan->d + kRecFloatsExtra) * sizeof(float);
+    return MILO_OK;
+}
+
+milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t batch, const void *tail_k,
+                               const void *tail_v, const int64_t *tail_offsets, int64_t tail_rows,
+                               int64_t max_tail_tokens, float softmax_scale, float *out, void *workspace,
+                               size_t workspace_bytes, void *stream_)
+{
+    if (!plan || !q || !out) return fail(MILO_ERR_INVALID_ARG, "null plan, q or out");
+    if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
+    if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
+    if (plan->nb == 0 && max_tail_tokens == 0) return fail(MILO_ERR_INVALID_ARG, "no prefix and no tail");
+    if (max_tail_tokens > 0) {
+        if (!tail_k || !tail_v || !tail_offsets) return fail(MILO_ERR_INVALID_ARG, "null tail pointer");
+        if (tail_rows < 1 || tail_rows > 0x7fffffff) return fail(MILO_ERR_INVALID_ARG, "tail_rows outside [1, 2^31)");
+        if (reinterpret_cast<uintptr_t>(tail_k) % 16 || reinterpret_cast<uintptr_t>(tail_v) % 16)
+            return fail(MILO_ERR_ALIGNMENT, "tails must be 16-byte aligned");
+        if (max_tail_tokens > (int64_t)kTailTokens * (1 << 20)) return fail(MILO_ERR_INVALID_ARG, "tail too long");
+    }
+    if (reinterpret_cast<uintptr_t>(q) % 4) return fail(MILO_ERR_ALIGNMENT, "q must be 4-byte aligned");
+    if (reinterpret_cast<uintptr_t>(out) % 16) return fail(MILO_ERR_ALIGNMENT, "out must be 16-byte aligned");
+    size_t need = 0;
+    milo_workspace_size(plan, batch, max_tail_tokens, &need);
+    if (!workspace || workspace_bytes < need) return fail(MILO_ERR_WORKSPACE, "workspace missing or too small");
+    if (reinterpret_cast<uintptr_t>(workspace) % 16) return fail(MILO_ERR_ALIGNMENT, "workspace misaligned");
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
+
+    const CallShape c = call_shape(plan, batch, max_tail_tokens);
+    DecodeParams prm{};
+    prm.packed = plan->packed;
+    prm.entries = plan->entries;
+    prm.segs = plan->segs;
+    prm.cta_seg_begin = plan->cta_seg_begin;
+    prm.g_slot_begin = plan->g_slot_begin;
+    prm.q = static_cast<const uint16_t *>(q);
+    prm.tail_offsets = tail_offsets;
+    prm.out = out;
+    prm.rec = static_cast<float *>(workspace);
+    prm.counters = plan->counters;
+    prm.tickets = plan->tickets;
+    prm.status = plan->status;
+    prm.batch = batch;
+    prm.hq = plan->hq;
+    prm.hkv = plan->hkv;
+    prm.G = plan->G;
+    prm.d = plan->d;
+    prm.rows_g = c.rows_g;
+    prm.nrg = c.nrg;
+    prm.nrg_cta = c.nrg_cta;
+    prm.npass = c.npass;
+    prm.nrg_t = c.nrg_t;
+    prm.num_slots = plan->num_slots;
+    prm.tail_splits = c.S;
+    prm.num_tail_items = batch * plan->hkv * c.S;
+    prm.has_tail = c.S > 0 ? 1 : 0;
+    prm.tail_rec_base = (int64_t)plan->num_slots * c.nrg;
+    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)plan->d);
+    prm.scale_log2 = scale * 1.4426950408889634f;
+    prm.num_ctas = plan->num_ctas;
+
+    alignas(64) CUtensorMap mk, mv;
+    std::memset(&mk, 0, sizeof mk);
+    std::memset(&mv, 0, sizeof mv);
+    if (c.S > 0) {
+        EncodeTiledFn enc = encode_fn();
+        if (!enc) return fail(MILO_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+        const cuuint64_t dims[3] = {(cuuint64_t)plan->d, (cuuint64_t)plan->hkv, (cuuint64_t)tail_rows};
+        const cuuint64_t strides[2] = {(cuuint64_t)plan->d * 2, (cuuint64_t)plan->hkv * plan->d * 2};
+        const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTailTokens};
+        const cuuint32_t estr[3] = {1, 1, 1};
+        CUresult r1 = enc(&mk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(tail_k), dims, strides, box,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        CUresult r2 = enc(&mv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(tail_v), dims, strides, box,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS) return fail(MILO_ERR_CUDA, "tensor map encoding failed");
+    }
+    const int smem = decode_smem_bytes(plan->d, c.nrg_cta);
+    cudaError_t e = launch_decode(prm, &mk, &mv, smem, plan->num_ctas, static_cast<cudaStream_t>(stream_));
+    if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    return MILO_OK;
+}
+
+milo_status_t milo_get_device_status(const milo_prefix_t *plan, void *stream, int32_t clear, int32_t *code)
+{
+    if (!plan || !code) return fail(MILO_ERR_INVALID_ARG, "null argument");
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int32_t v = 0;
+    if ((e = cudaMemcpy(&v, plan->status, sizeof v, cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_fail(e, "read status");
+    *code = v;
+    if (clear && (e = cudaMemset(plan->status, 0, sizeof(int32_t))) != cudaSuccess)
+        return cuda_fail(e, "clear status");
+    return MILO_OK;
+}
+
+}  // extern "C"

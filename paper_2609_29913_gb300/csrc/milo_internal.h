@@ -1,0 +1,85 @@
+// milo_internal.h -- structures shared by the libmilo host code and kernels.
+#pragma once
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace milo {
+
+constexpr int kTileTokens = 64;      // tokens per packed coefficient tile
+constexpr int kConsumerWarps = 8;    // MMA warps per decode thread block
+constexpr int kThreads = 32 * (kConsumerWarps + 1);
+constexpr int kSlots = 4;            // shared-memory ring depth
+constexpr int kSlotBytes = 32768;    // bytes per ring slot
+constexpr int kHdrInts = 16;         // slot header (ints)
+constexpr int kTailTokens = 64;      // tokens per dense-tail work item
+constexpr int kRecFloatsExtra = 16;  // m[8], l[8] after o[8][d] in a record
+
+// Per-(block, KV head) entry of the packed arena.
+struct EntryDev {
+    int64_t off_ck, off_pk, off_cv, off_pv;  // byte offsets (128-aligned)
+    int32_t n;                               // tokens
+    int32_t rk, rv;                          // true ranks
+    int32_t g;                               // KV head
+};
+
+// Prefix segment of the static partition.
+enum : int32_t { kSegFirstOfRun = 1, kSegLastOfRun = 2 };
+struct SegDev {
+    int32_t entry;
+    int32_t t0, t1;    // token range within the block
+    int32_t slot;      // partial slot (run)
+    int32_t flags;
+    int32_t pad[3];
+};
+
+// Device-side counters owned by a plan (zero between calls).
+struct CountersDev {
+    uint32_t tail_next;   // dynamic tail work counter
+    uint32_t ctas_done;   // thread blocks finished (resets tail_next)
+    uint32_t pad[30];
+    // followed by tickets[num_kv_heads * max_row_groups]
+};
+
+struct DecodeParams {
+    const uint8_t *packed;
+    const EntryDev *entries;
+    const SegDev *segs;
+    const int32_t *cta_seg_begin;   // [num_ctas + 1]
+    const int32_t *g_slot_begin;    // [Hkv + 1]
+    const uint16_t *q;              // bf16 [batch, Hq, d]
+    const int64_t *tail_offsets;    // [batch + 1] or null
+    float *out;                     // [batch, Hq, d]
+    float *rec;                     // workspace records
+    CountersDev *counters;
+    uint32_t *tickets;              // [Hkv * nrg]
+    int32_t *status;
+    int batch, hq, hkv, G, d;
+    int rows_g;                     // batch * G
+    int nrg;                        // ceil(rows_g / 8)
+    int nrg_cta;                    // prefix row groups per pass (1, 2 or 4)
+    int npass;                      // ceil(nrg / nrg_cta)
+    int nrg_t;                      // tail row groups per query: ceil(G / 8)
+    int num_slots;                  // prefix record slots
+    int tail_splits;                // S
+    int num_tail_items;             // batch * Hkv * S
+    int has_tail;
+    int64_t tail_rec_base;          // first tail record index
+    float scale_log2;               // softmax scale * log2(e)
+    int num_ctas;
+};
+
+// Launchers implemented in the .cu files.
+cudaError_t launch_pack(const void *arena, const EntryDev *entries_dev,
+                        const int64_t *logical_offsets_dev, int num_entries,
+                        int head_dim, uint8_t *packed, int64_t packed_bytes,
+                        cudaStream_t stream);
+
+cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k,
+                          const void *tmap_v, int smem_bytes, int num_ctas,
+                          cudaStream_t stream);
+
+int decode_smem_bytes(int head_dim, int nrg_cta);
+
+}  // namespace milo

@@ -1,0 +1,273 @@
+"""Python binding of libmilo (include/milo.h): argument marshalling only.
+
+Every computation runs inside libmilo's CUDA kernels; this module converts
+numpy arrays and torch tensors into the pointers and sizes the C ABI takes.
+Importing it does not build anything: call ``paper_2609_29913_gb300.build``
+(or ``__graft_entry__.build()``) first.  A missing library raises
+:class:`MiloError` -- there is no fallback.
+
+Functions carry the C names.  :class:`Prefix` is the convenience wrapper a
+user calls: create once per layer from a block table, then ``decode`` per
+step (torch tensors in, fp32 attention output out).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libmilo.so")
+
+MILO_OK = 0
+STATUS_NAMES = {0: "MILO_OK", 1: "MILO_ERR_INVALID_ARG", 2: "MILO_ERR_BAD_TABLE",
+                3: "MILO_ERR_ALIGNMENT", 4: "MILO_ERR_UNSUPPORTED", 5: "MILO_ERR_CUDA",
+                6: "MILO_ERR_TIMEOUT", 7: "MILO_ERR_DEVICE_BOUNDS", 8: "MILO_ERR_WORKSPACE"}
+
+# every symbol include/milo.h declares
+EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
+           "milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
+           "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
+           "milo_workspace_size", "milo_attn_decode", "milo_get_device_status"]
+
+
+class MiloError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str = ""):
+        self.status = int(status)
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}" + (f" ({detail})" if detail else ""))
+
+
+class BlockTableC(ctypes.Structure):
+    _fields_ = [("num_blocks", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32),
+                ("block_len", ctypes.c_void_p), ("rank_k", ctypes.c_void_p),
+                ("rank_v", ctypes.c_void_p), ("off_ck", ctypes.c_void_p),
+                ("off_pk", ctypes.c_void_p), ("off_cv", ctypes.c_void_p),
+                ("off_pv", ctypes.c_void_p), ("arena", ctypes.c_void_p),
+                ("arena_elems", ctypes.c_int64)]
+
+
+class PrefixInfoC(ctypes.Structure):
+    _fields_ = [("num_blocks", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("num_q_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("max_batch", ctypes.c_int32), ("num_ctas", ctypes.c_int32),
+                ("num_segments", ctypes.c_int32), ("num_slots", ctypes.c_int32),
+                ("prefix_tokens", ctypes.c_int64), ("logical_factor_bytes", ctypes.c_int64),
+                ("packed_bytes", ctypes.c_int64), ("packed_arena", ctypes.c_void_p)]
+
+
+_lib = None
+
+
+def lib():
+    """The loaded libmilo (raises MiloError if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise MiloError(5, "load libmilo", f"{LIB_PATH} missing; build it first")
+        L = ctypes.CDLL(LIB_PATH)
+        P, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+        L.milo_status_string.argtypes = [i32]
+        L.milo_status_string.restype = ctypes.c_char_p
+        L.milo_version.restype = i32
+        L.milo_last_error_message.restype = ctypes.c_char_p
+        L.milo_validate_table.argtypes = [P]
+        L.milo_packed_layout.argtypes = [P, P, P]
+        L.milo_partition_prefix.argtypes = [P, i32, i32, P, P, P, P, P, P, P]
+        L.milo_prefix_create.argtypes = [P, i32, i32, P, P]
+        L.milo_prefix_destroy.argtypes = [P]
+        L.milo_prefix_get_info.argtypes = [P, P]
+        L.milo_workspace_size.argtypes = [P, i32, i64, P]
+        L.milo_attn_decode.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P,
+                                       ctypes.c_size_t, P]
+        L.milo_get_device_status.argtypes = [P, P, i32, P]
+        for name in ("milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
+                     "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
+                     "milo_workspace_size", "milo_attn_decode", "milo_get_device_status"):
+            getattr(L, name).restype = i32
+        _lib = L
+    return _lib
+
+
+def _check(status: int, where: str):
+    if status != MILO_OK:
+        detail = lib().milo_last_error_message().decode(errors="replace")
+        raise MiloError(status, where, detail)
+
+
+def _arr(a, dtype):
+    return np.ascontiguousarray(np.asarray(a), dtype=dtype)
+
+
+class HostTable:
+    """Host-side arrays of a block table plus the device arena pointer, kept
+    alive for as long as the ctypes struct built from them is used."""
+
+    def __init__(self, *, num_kv_heads, head_dim, block_len, rank_k, rank_v, off_ck,
+                 off_pk, off_cv, off_pv, arena_ptr=0, arena_elems=0):
+        self.block_len = _arr(block_len, np.int32)
+        self.rank_k = _arr(rank_k, np.int32)
+        self.rank_v = _arr(rank_v, np.int32)
+        self.off_ck = _arr(off_ck, np.int64)
+        self.off_pk = _arr(off_pk, np.int64)
+        self.off_cv = _arr(off_cv, np.int64)
+        self.off_pv = _arr(off_pv, np.int64)
+        nb = int(self.block_len.shape[0])
+        ptr = lambda a: a.ctypes.data if a.size else None
+        self.c = BlockTableC(nb, int(num_kv_heads), int(head_dim), ptr(self.block_len),
+                             ptr(self.rank_k), ptr(self.rank_v), ptr(self.off_ck),
+                             ptr(self.off_pk), ptr(self.off_cv), ptr(self.off_pv),
+                             int(arena_ptr) or None, int(arena_elems))
+
+    @property
+    def num_entries(self) -> int:
+        return int(self.c.num_blocks) * int(self.c.num_kv_heads)
+
+    @classmethod
+    def from_layer(cls, layer):
+        """From a ``workloads.LayerInputs`` (arena on the GPU)."""
+        return cls(**layer.table_arrays(), arena_ptr=layer.arena.data_ptr(),
+                   arena_elems=int(layer.arena.numel()))
+
+
+def milo_validate_table(table: HostTable) -> int:
+    return int(lib().milo_validate_table(ctypes.byref(table.c)))
+
+
+def milo_packed_layout(table: HostTable):
+    offs = np.zeros(max(table.num_entries * 4, 1), dtype=np.int64)
+    total = ctypes.c_int64(0)
+    _check(lib().milo_packed_layout(ctypes.byref(table.c), offs.ctypes.data, ctypes.byref(total)),
+           "milo_packed_layout")
+    return offs[:table.num_entries * 4].reshape(-1, 4), int(total.value)
+
+
+def milo_partition_prefix(table: HostTable, num_ctas: int) -> dict:
+    nseg, nslot = ctypes.c_int32(0), ctypes.c_int32(0)
+    L = lib()
+    _check(L.milo_partition_prefix(ctypes.byref(table.c), int(num_ctas), 0, None, None, None,
+                                   None, None, ctypes.byref(nseg), ctypes.byref(nslot)),
+           "milo_partition_prefix")
+    n = int(nseg.value)
+    out = {k: np.zeros(max(n, 1), dtype=np.int32) for k in ("entry", "t0", "t1", "slot")}
+    cb = np.zeros(int(num_ctas) + 1, dtype=np.int32)
+    _check(L.milo_partition_prefix(ctypes.byref(table.c), int(num_ctas), n,
+                                   out["entry"].ctypes.data, out["t0"].ctypes.data,
+                                   out["t1"].ctypes.data, out["slot"].ctypes.data,
+                                   cb.ctypes.data, None, None), "milo_partition_prefix")
+    res = {k: v[:n] for k, v in out.items()}
+    res["cta_begin"] = cb
+    res["num_slots"] = int(nslot.value)
+    return res
+
+
+def _stream_ptr(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream or None
+    if isinstance(stream, int):
+        return stream or None
+    return stream.cuda_stream or None
+
+
+def milo_prefix_create(table: HostTable, num_q_heads: int, max_batch: int, stream=None) -> int:
+    plan = ctypes.c_void_p(0)
+    _check(lib().milo_prefix_create(ctypes.byref(table.c), int(num_q_heads), int(max_batch),
+                                    _stream_ptr(stream), ctypes.byref(plan)), "milo_prefix_create")
+    return int(plan.value)
+
+
+def milo_prefix_destroy(plan: int) -> None:
+    _check(lib().milo_prefix_destroy(plan), "milo_prefix_destroy")
+
+
+def milo_prefix_get_info(plan: int) -> dict:
+    info = PrefixInfoC()
+    _check(lib().milo_prefix_get_info(plan, ctypes.byref(info)), "milo_prefix_get_info")
+    return {name: getattr(info, name) for name, _ in PrefixInfoC._fields_}
+
+
+def milo_workspace_size(plan: int, batch: int, max_tail_tokens: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().milo_workspace_size(plan, int(batch), int(max_tail_tokens), ctypes.byref(n)),
+           "milo_workspace_size")
+    return int(n.value)
+
+
+def milo_attn_decode(plan: int, q_ptr: int, batch: int, tail_k_ptr: int, tail_v_ptr: int,
+                     tail_offsets_ptr: int, tail_rows: int, max_tail_tokens: int,
+                     softmax_scale: float, out_ptr: int, workspace_ptr: int,
+                     workspace_bytes: int, stream=None) -> None:
+    _check(lib().milo_attn_decode(plan, q_ptr, int(batch), tail_k_ptr or None, tail_v_ptr or None,
+                                  tail_offsets_ptr or None, int(tail_rows), int(max_tail_tokens),
+                                  float(softmax_scale), out_ptr, workspace_ptr,
+                                  int(workspace_bytes), _stream_ptr(stream)), "milo_attn_decode")
+
+
+def milo_get_device_status(plan: int, stream=None, clear: bool = False) -> int:
+    code = ctypes.c_int32(0)
+    _check(lib().milo_get_device_status(plan, _stream_ptr(stream), int(bool(clear)),
+                                        ctypes.byref(code)), "milo_get_device_status")
+    return int(code.value)
+
+
+class Prefix:
+    """One layer's compressed prefix on the GPU (a libmilo plan).
+
+    ``Prefix(table, num_q_heads, max_batch)`` packs the factors; ``decode``
+    runs one attention call into a preallocated fp32 output."""
+
+    def __init__(self, table: HostTable, num_q_heads: int, max_batch: int, stream=None):
+        self.table = table
+        self.num_q_heads = int(num_q_heads)
+        self.max_batch = int(max_batch)
+        self.head_dim = int(table.c.head_dim)
+        self.num_kv_heads = int(table.c.num_kv_heads)
+        self.plan = milo_prefix_create(table, num_q_heads, max_batch, stream)
+        self.info = milo_prefix_get_info(self.plan)
+
+    @classmethod
+    def from_layer(cls, layer, max_batch=None, stream=None):
+        return cls(HostTable.from_layer(layer), layer.num_q_heads,
+                   max_batch or layer.batch, stream)
+
+    def workspace_size(self, batch: int, max_tail_tokens: int) -> int:
+        return milo_workspace_size(self.plan, batch, max_tail_tokens)
+
+    def decode(self, q, tail_k=None, tail_v=None, tail_offsets=None, max_tail_tokens=0,
+               softmax_scale: float = 0.0, out=None, workspace=None, stream=None):
+        """q: bf16 [batch, Hq, d] cuda tensor; tails bf16 [rows, Hkv, d];
+        tail_offsets int64 cuda tensor [batch + 1].  Returns fp32 out."""
+        import torch
+        batch = int(q.shape[0])
+        if out is None:
+            out = torch.empty((batch, self.num_q_heads, self.head_dim), device=q.device,
+                              dtype=torch.float32)
+        need = self.workspace_size(batch, max_tail_tokens)
+        if workspace is None:
+            workspace = torch.empty(need, device=q.device, dtype=torch.uint8)
+        tail_rows = int(tail_k.shape[0]) if (tail_k is not None and max_tail_tokens > 0) else 0
+        milo_attn_decode(self.plan, q.data_ptr(), batch,
+                         tail_k.data_ptr() if tail_rows else 0,
+                         tail_v.data_ptr() if tail_rows else 0,
+                         tail_offsets.data_ptr() if tail_rows else 0,
+                         tail_rows, max_tail_tokens if tail_rows else 0, softmax_scale,
+                         out.data_ptr(), workspace.data_ptr(), workspace.numel() * workspace.element_size(),
+                         stream)
+        return out
+
+    def status(self, stream=None, clear=False) -> int:
+        return milo_get_device_status(self.plan, stream, clear)
+
+    def close(self):
+        if getattr(self, "plan", None):
+            milo_prefix_destroy(self.plan)
+            self.plan = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

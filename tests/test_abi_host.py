@@ -1,0 +1,177 @@
+"""CPU tests of the C ABI: the library loads without a GPU, exports every
+symbol the header declares, validates tables, computes the packed layout and
+the static work partition -- all host logic, checked bit-exactly."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="session")
+def milo():
+    from paper_2609_29913_gb300 import build, milo
+    build.build()
+    milo.lib()
+    return milo
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "milo.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(milo_[a-z_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(milo):
+    names = declared_functions()
+    assert len(names) >= 10
+    lib = ctypes.CDLL(milo.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    assert sorted(milo.EXPORTS) == names
+
+
+def test_status_strings_and_version(milo):
+    L = milo.lib()
+    assert L.milo_version() >= 100
+    for s in range(9):
+        assert L.milo_status_string(s)
+    assert L.milo_status_string(0) == b"ok"
+
+
+def table(block_len, rk, rv=None, hkv=1, d=64, gap=0, base=0, arena_elems=None):
+    """Logical row-major layout with optional gaps (multiples of 8)."""
+    block_len = list(block_len)
+    rk = np.asarray(rk).reshape(-1)
+    rv = rk if rv is None else np.asarray(rv).reshape(-1)
+    offs = np.zeros((len(rk), 4), np.int64)
+    cur = base
+    for b, n in enumerate(block_len):
+        for g in range(hkv):
+            e = b * hkv + g
+            for f, sz in enumerate((n * rk[e], rk[e] * d, n * rv[e], rv[e] * d)):
+                offs[e, f] = cur
+                cur += int(sz) + ((-int(sz)) % 8) + gap
+    return dict(num_kv_heads=hkv, head_dim=d, block_len=block_len, rank_k=rk, rank_v=rv,
+                off_ck=offs[:, 0], off_pk=offs[:, 1], off_cv=offs[:, 2], off_pv=offs[:, 3],
+                arena_ptr=0x10000, arena_elems=cur if arena_elems is None else arena_elems)
+
+
+def ht(milo, **kw):
+    return milo.HostTable(**kw)
+
+
+def test_validate_accepts_good_tables(milo):
+    assert milo.milo_validate_table(ht(milo, **table([7, 64, 129], [1, 8, 64], [13, 0, 64]))) == 0
+    assert milo.milo_validate_table(ht(milo, **table([512] * 3, [16, 32, 128] * 2, hkv=2, d=128, gap=8))) == 0
+    empty = table([], [])
+    assert milo.milo_validate_table(ht(milo, **empty)) == 0
+
+
+@pytest.mark.parametrize("mutate,code", [
+    (lambda t: t.update(rank_k=np.array([65, 8])), 2),        # rank > head_dim
+    (lambda t: t.update(rank_v=np.array([-1, 8])), 2),        # negative rank
+    (lambda t: t.update(block_len=[0, 9]), 2),                # empty block
+    (lambda t: t.update(block_len=[70000, 9]), 2),            # block too long
+    (lambda t: t["off_pk"].__setitem__(0, t["off_pk"][0] + 4), 3),  # misaligned offset
+    (lambda t: t.update(arena_elems=t["arena_elems"] - 8), 2),      # region outside arena
+    (lambda t: t["off_cv"].__setitem__(1, t["off_ck"][1]), 2),      # overlapping regions
+    (lambda t: t.update(head_dim=96), 4),                     # unsupported head dim
+    (lambda t: t.update(num_kv_heads=0), 1),                  # no heads
+    (lambda t: t.update(arena_ptr=0x10004), 3),               # misaligned arena
+])
+def test_validate_rejects(milo, mutate, code):
+    t = table([5, 9], [4, 8])
+    mutate(t)
+    assert milo.milo_validate_table(ht(milo, **t)) == code
+
+
+def test_packed_layout_sizes_and_alignment(milo):
+    rng = np.random.default_rng(0)
+    bl = list(rng.integers(1, 300, size=6))
+    rk = rng.integers(0, 129, size=12)
+    rv = rng.integers(0, 129, size=12)
+    t = ht(milo, **table(bl, rk, rv, hkv=2, d=128))
+    offs, total = milo.milo_packed_layout(t)
+    r8 = lambda r: (r + 7) // 8 * 8
+    sizes = []
+    for e in range(12):
+        n8 = (bl[e // 2] + 7) // 8 * 8
+        sizes += [n8 * r8(rk[e]) * 2, r8(rk[e]) * 128 * 2, n8 * r8(rv[e]) * 2, r8(rv[e]) * 128 * 2]
+    flat = offs.reshape(-1)
+    assert (flat % 128 == 0).all()
+    assert (np.diff(flat) >= np.array(sizes[:-1])).all()           # in order, no overlap
+    assert total >= flat[-1] + sizes[-1] and total % 128 == 0
+    assert total - (flat[-1] + sizes[-1]) < 128
+
+
+@pytest.mark.parametrize("ctas", [1, 3, 7, 152, 1000])
+@pytest.mark.parametrize("shape", [
+    ([512] * 64, "choice", 4, 128),
+    ([7, 129, 1, 64, 65, 300], "rand", 2, 64),
+    ([512] * 8, "rand", 1, 128),
+])
+def test_partition_covers_every_token_once(milo, ctas, shape):
+    bl, law, hkv, d = shape
+    rng = np.random.default_rng(len(bl) * 7 + ctas)
+    nb = len(bl)
+    if law == "choice":
+        rk = rng.choice([16, 32, 64, 96, 128], size=nb * hkv)
+    else:
+        rk = rng.integers(0, d + 1, size=nb * hkv)
+    rv = rng.integers(0, d + 1, size=nb * hkv)
+    t = ht(milo, **table(bl, rk, rv, hkv=hkv, d=d))
+    part = milo.milo_partition_prefix(t, ctas)
+    cover = {}
+    for e, t0, t1 in zip(part["entry"], part["t0"], part["t1"]):
+        assert t0 % 64 == 0 and t0 < t1 <= bl[e // hkv]
+        assert (t1 % 64 == 0) or t1 == bl[e // hkv]
+        for tok in range(t0, t1):
+            key = (int(e), tok)
+            assert key not in cover
+            cover[key] = 1
+    assert len(cover) == sum(bl) * hkv
+    cb = part["cta_begin"]
+    assert cb[0] == 0 and cb[-1] == len(part["entry"]) and (np.diff(cb) >= 0).all()
+    # slots: one per (thread block, KV-head run), numbered in KV-head order
+    slots = part["slot"]
+    heads_of_slot = {}
+    for c in range(ctas):
+        prev = None
+        for s in range(cb[c], cb[c + 1]):
+            g = int(part["entry"][s]) % hkv
+            heads_of_slot.setdefault(int(slots[s]), set()).add(g)
+            if prev is not None and g == prev[0]:
+                assert slots[s] == prev[1]
+            prev = (g, int(slots[s]))
+    assert all(len(v) == 1 for v in heads_of_slot.values())
+    order = [next(iter(heads_of_slot[s])) for s in sorted(heads_of_slot)]
+    assert order == sorted(order)
+    assert part["num_slots"] == len(heads_of_slot)
+
+
+def test_partition_balances_bytes(milo):
+    rng = np.random.default_rng(5)
+    nb, hkv, d = 64, 4, 128
+    rk = rng.choice([16, 32, 64, 96, 128], size=nb * hkv)
+    t = ht(milo, **table([512] * nb, rk, rk, hkv=hkv, d=d))
+    ctas = 152
+    part = milo.milo_partition_prefix(t, ctas)
+    r8 = lambda r: (r + 7) // 8 * 8
+    cost = np.zeros(ctas)
+    cb = part["cta_begin"]
+    for c in range(ctas):
+        for s in range(cb[c], cb[c + 1]):
+            e = part["entry"][s]
+            tok = part["t1"][s] - part["t0"][s]
+            # the header's cost model: factor bytes + 32 per token for the softmax;
+            # bases count once per block (a cut block's second reader hits L2)
+            cost[c] += tok * (r8(rk[e]) * 4 + 32)
+            cost[c] += r8(rk[e]) * d * 2 if part["t0"][s] == 0 else 0      # P^K
+            cost[c] += r8(rk[e]) * d * 2 if part["t1"][s] == 512 else 0    # P^V
+    mean = cost.mean()
+    assert cost.max() <= mean * 1.15, (cost.max(), mean)
+    assert (cost > 0).all()
