@@ -301,12 +301,14 @@ def main():
         dist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clocks:
+        torch.cuda.nvtx.range_push("milo_timed")
         start.record(stream)
         with torch.cuda.stream(stream):
             for _ in range(args.steps):
                 graph.replay()
         stop.record(stream)
         torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
     if dist:
         dist.barrier()
     ms_total = start.elapsed_time(stop)

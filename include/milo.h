@@ -105,8 +105,8 @@ milo_status_t milo_validate_table(const milo_block_table_t *table);
  * Each factor is stored zero-padded to r8 = roundup(r, 8) ranks and, for the
  * coefficient matrices, n8 = roundup(n_b, 8) tokens, as 8x8 bf16 tiles of 128
  * contiguous bytes (one tile = 8 rows x 16 bytes):
- *   C (n_b x r): token tiles of 64 tokens; the token tile k that holds t8
- *     padded tokens occupies t8 * r8 * 2 bytes starting at k * 64 * r8 * 2;
+ *   C (n_b x r): token tiles of 32 tokens; the token tile k that holds t8
+ *     padded tokens occupies t8 * r8 * 2 bytes starting at k * 32 * r8 * 2;
  *     inside it, tile (rank group rg, token group tg) sits at
  *     (rg * t8/8 + tg) * 128 and holds row (t % 8), column (j % 8).
  *   P (r x d): tile (rank group jg, column group cg) sits at
@@ -121,10 +121,10 @@ milo_status_t milo_packed_layout(const milo_block_table_t *table,
 /*
  * Static prefix work partition the decode kernel uses, computed on the host.
  * The prefix (every entry's tokens, KV-head-major, then block order) is cut
- * at 64-token boundaries into segments so that each of `num_ctas` thread
+ * at 32-token boundaries into segments so that each of `num_ctas` thread
  * blocks receives a near-equal share of the cost line, where a token costs its
  * padded coefficient bytes plus 32 (the softmax work), a block's P^K is charged
- * with its first 64-token tile and its P^V with its last; a tile goes to the
+ * with its first 32-token tile and its P^V with its last; a tile goes to the
  * thread block whose share holds the midpoint of the tile's cost.  Consecutive segments
  * of one thread block with the same KV head form a "run" whose partial result
  * occupies one slot.

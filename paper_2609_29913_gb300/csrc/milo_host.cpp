@@ -423,7 +423,7 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t
 
 namespace {
 struct CallShape {
-    int rows_g, nrg, nrg_cta, npass, nrg_t, S;
+    int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
     int64_t records;
 };
 
@@ -432,9 +432,11 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     CallShape c;
     c.rows_g = batch * p->G;
     c.nrg = (c.rows_g + 7) / 8;
-    c.nrg_cta = c.nrg >= 3 ? 4 : (c.nrg == 2 ? 2 : 1);
+    c.nrg_cta = c.nrg >= 2 ? 2 : 1;
     c.npass = (c.nrg + c.nrg_cta - 1) / c.nrg_cta;
     c.nrg_t = (p->G + 7) / 8;
+    c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
+    c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
     c.records = (int64_t)p->num_slots * c.nrg + (int64_t)batch * p->hkv * c.S * c.nrg_t;
     return c;
@@ -501,6 +503,8 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.nrg_cta = c.nrg_cta;
     prm.npass = c.npass;
     prm.nrg_t = c.nrg_t;
+    prm.ngrp_t = c.ngrp_t;
+    prm.npass_t = c.npass_t;
     prm.num_slots = plan->num_slots;
     prm.tail_splits = c.S;
     prm.num_tail_items = batch * plan->hkv * c.S;

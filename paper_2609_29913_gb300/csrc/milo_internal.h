@@ -7,13 +7,13 @@
 
 namespace milo {
 
-constexpr int kTileTokens = 64;      // tokens per packed coefficient tile
-constexpr int kConsumerWarps = 8;    // MMA warps per decode thread block
-constexpr int kThreads = 32 * (kConsumerWarps + 1);
-constexpr int kSlots = 4;            // shared-memory ring depth
-constexpr int kSlotBytes = 32768;    // bytes per ring slot
+constexpr int kTileTokens = 32;      // tokens per packed coefficient tile
+constexpr int kMmaWarps = 8;         // score/value warps per decode thread block
+constexpr int kThreads = 32 * (3 + kMmaWarps);  // + producer, projection, epilogue
+constexpr int kSlots = 6;            // coefficient ring depth
+constexpr int kSlotBytes = 16384;    // bytes per ring slot
 constexpr int kHdrInts = 16;         // slot header (ints)
-constexpr int kTailTokens = 64;      // tokens per dense-tail work item
+constexpr int kTailTokens = 32;      // tokens per dense-tail work item
 constexpr int kRecFloatsExtra = 16;  // m[8], l[8] after o[8][d] in a record
 
 // Per-(block, KV head) entry of the packed arena.
@@ -58,9 +58,11 @@ struct DecodeParams {
     int batch, hq, hkv, G, d;
     int rows_g;                     // batch * G
     int nrg;                        // ceil(rows_g / 8)
-    int nrg_cta;                    // prefix row groups per pass (1, 2 or 4)
+    int nrg_cta;                    // prefix row groups per pass (1 or 2)
     int npass;                      // ceil(nrg / nrg_cta)
     int nrg_t;                      // tail row groups per query: ceil(G / 8)
+    int ngrp_t;                     // tail row groups per pass (1 or 2)
+    int npass_t;                    // ceil(nrg_t / ngrp_t)
     int num_slots;                  // prefix record slots
     int tail_splits;                // S
     int num_tail_items;             // batch * Hkv * S

@@ -16,7 +16,8 @@ Logical prefix layout (one decoder layer, one arena):
 
 Recipe (stands in for the paper's Qwen2.5 many-shot KV caches, which need
 model weights and datasets that are not available here):
-  P = (Q of the reduced QR of a d x r standard Gaussian)^T, rounded to bf16;
+  P = (Q of the reduced QR of a d x r standard Gaussian)^T, rounded to bf16
+      (drawn and factorised on the host, so identical on every device);
   C[:, j] ~ N(0, 1/j) for j = 1..r (1/j is the variance), rounded to bf16;
   q, tail K, tail V ~ N(0, 1) in bf16; ``q_scale`` multiplies q (e.g. 30 for
   a peaked softmax).  Integer draws (ranks, tail lengths) use numpy's PCG64
@@ -176,11 +177,12 @@ def _torch_gen(device, seed: int, layer: int) -> torch.Generator:
     return g
 
 
-def _orthonormal_rows(m: int, r: int, d: int, gen, device) -> torch.Tensor:
-    """m independent r x d matrices with orthonormal rows (fp32)."""
-    a = torch.randn((m, d, r), generator=gen, device=device, dtype=torch.float32)
+def _orthonormal_rows(m: int, r: int, d: int, gen_cpu, device) -> torch.Tensor:
+    """m independent r x d matrices with orthonormal rows (fp32), drawn and
+    factorised on the host (identical on every device), then moved."""
+    a = torch.randn((m, d, r), generator=gen_cpu, dtype=torch.float32)
     qm, _ = torch.linalg.qr(a, mode="reduced")    # [m, d, r]
-    return qm.transpose(1, 2).contiguous()          # [m, r, d]
+    return qm.transpose(1, 2).contiguous().to(device)  # [m, r, d]
 
 
 def build_layer(num_q_heads: int, num_kv_heads: int, head_dim: int,
@@ -198,6 +200,7 @@ def build_layer(num_q_heads: int, num_kv_heads: int, head_dim: int,
     rk = np.asarray(rank_k, dtype=np.int32).reshape(nb * hk)
     rv = rk.copy() if rank_v is None else np.asarray(rank_v, dtype=np.int32).reshape(nb * hk)
     gen = _torch_gen(device, seed, layer)
+    gen_cpu = _torch_gen("cpu", seed + 104_729, layer)
 
     # element offsets, every factor 8-aligned, entries in (b, g) order
     offs = np.zeros((4, nb * hk), dtype=np.int64)
@@ -238,7 +241,7 @@ def build_layer(num_q_heads: int, num_kv_heads: int, head_dim: int,
                 if basis == "identity":
                     x = torch.eye(d, device=device, dtype=torch.float32)[:r].expand(m, r, d)
                 elif r:
-                    x = _orthonormal_rows(m, r, d, gen, device)
+                    x = _orthonormal_rows(m, r, d, gen_cpu, device)
                 else:
                     x = torch.zeros((m, 0, d), device=device)
             x = x.to(torch.bfloat16)

@@ -127,8 +127,8 @@ def test_partition_covers_every_token_once(milo, ctas, shape):
     part = milo.milo_partition_prefix(t, ctas)
     cover = {}
     for e, t0, t1 in zip(part["entry"], part["t0"], part["t1"]):
-        assert t0 % 64 == 0 and t0 < t1 <= bl[e // hkv]
-        assert (t1 % 64 == 0) or t1 == bl[e // hkv]
+        assert t0 % 32 == 0 and t0 < t1 <= bl[e // hkv]
+        assert (t1 % 32 == 0) or t1 == bl[e // hkv]
         for tok in range(t0, t1):
             key = (int(e), tok)
             assert key not in cover

