@@ -16,14 +16,15 @@
 //               tail items from a counter and streams them with 3-D TMA.
 //   projection  (warp 1): q~ = scale * log2(e) * P^K q for every segment, as
 //               bf16 hi + lo mma fragments, into a double buffer.
-//   MMA warps   (warps 3..10): 16-token sub-tiles round-robin: scores (mma
+//   MMA warps   (warps 4..11): 16-token sub-tiles round-robin: scores (mma
 //               m16n8k16; A rows 0-7 = q~ hi, 8-15 = q~ lo), online softmax
 //               in registers, rank-space values (A rows = p hi / p lo).  At a
 //               segment's end each warp dumps (max, sum, v~) into its own
 //               shared-memory region and continues with the next segment.
-//   epilogue    (warp 2): merges the 8 dumps of a segment, back-projects v~
-//               through P^V into the head dimension, folds the result into
-//               the run's output, writes partial records and counts tickets.
+//   epilogue    (warps 2-3): both merge the 8 dumps of a segment; each
+//               back-projects v~ through P^V into half of the head dimension,
+//               folds it into its half of the run's output and writes it to
+//               the partial record; the first counts the tickets.
 // The thread block that brings the last record of a (KV head, row group)
 // merges all of that row group's records at the end of the kernel (no
 // thread block ever waits for another).  Every wait is bounded (~2 s); on
@@ -48,7 +49,7 @@ enum : int { F_FIRST_C = 1, F_LAST_C = 2, F_RUN_FIRST = 4, F_RUN_LAST = 8 };
 enum : int { H_KIND, H_E, H_G, H_T0, H_T1, H_RK8, H_RV8, H_TOK8, H_NSUB, H_FLAGS, H_REC, H_PASS, H_QI, H_ITEM };
 // barrier indices (after the ring's full[kSlots], empty[kSlots])
 enum : int {
-    B_PKF = 2 * kSlots, B_PKE, B_PVF, B_PVE, B_QR0, B_QR1, B_QF0, B_QF1, B_MF, B_ME, B_FIN, B_COUNT
+    B_PKF = 2 * kSlots, B_PKE, B_PVF, B_PVE, B_QR0, B_QR1, B_QF0, B_QF1, B_MF, B_ME, B_EPS, B_FIN, B_COUNT
 };
 
 // ------------------------------------------------------------------ PTX ----
@@ -217,6 +218,7 @@ struct Lay {
 template <int D>
 __device__ void combine_rows(const DecodeParams &p, int g, int rg, int tid, int nthr)
 {
+    constexpr int kChunk = 12;  // records whose loads are in flight together
     const int recf = 8 * D + kRecFloatsExtra;
     const int gs0 = p.g_slot_begin[g], gs1 = p.g_slot_begin[g + 1];
     const int nprefix = gs1 - gs0;
@@ -227,37 +229,45 @@ __device__ void combine_rows(const DecodeParams &p, int g, int rg, int tid, int 
         const int rho = 8 * rg + k;
         if (rho >= p.rows_g) continue;
         const int i = rho / p.G, hh = rho % p.G;
-        auto rec_of = [&](int s, int &row) -> const float * {
-            if (s < nprefix) {
-                row = k;
-                return p.rec + (int64_t)((gs0 + s) * p.nrg + rg) * recf;
-            }
-            const int t = s - nprefix;
-            row = hh % 8;
-            return p.rec + (p.tail_rec_base + ((int64_t)(i * p.hkv + g) * S + t) * p.nrg_t + hh / 8) * recf;
-        };
-        float M = -INFINITY;
-#pragma unroll 8
-        for (int s = 0; s < nsrc; ++s) {
-            int row;
-            const float *r = rec_of(s, row);
-            M = fmaxf(M, __ldcg(r + 8 * D + row));
-        }
-        float Lsum = 0.f;
+        const float *tail0 = p.rec + (p.tail_rec_base + (int64_t)(i * p.hkv + g) * S * p.nrg_t + hh / 8) * recf;
+        float M = -INFINITY, Lsum = 0.f;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-        for (int s = 0; s < nsrc; ++s) {
-            int row;
-            const float *r = rec_of(s, row);
-            const float m = __ldcg(r + 8 * D + row);
-            const float l = __ldcg(r + 8 * D + 8 + row);
-            const float4 o = __ldcg(reinterpret_cast<const float4 *>(r + row * D) + c4);
-            const float w8 = exp2_diff(m, M);
-            Lsum += w8 * l;
-            acc.x += w8 * o.x;
-            acc.y += w8 * o.y;
-            acc.z += w8 * o.z;
-            acc.w += w8 * o.w;
+        for (int s0 = 0; s0 < nsrc; s0 += kChunk) {
+            float mm[kChunk], ll[kChunk];
+            float4 oo[kChunk];
+#pragma unroll
+            for (int j = 0; j < kChunk; ++j) {
+                const int s = s0 + j;
+                if (s < nsrc) {
+                    const bool pre = s < nprefix;
+                    const int row = pre ? k : hh % 8;
+                    const float *r = pre ? p.rec + (int64_t)((gs0 + s) * p.nrg + rg) * recf
+                                         : tail0 + (int64_t)(s - nprefix) * p.nrg_t * recf;
+                    mm[j] = __ldcg(r + 8 * D + row);
+                    ll[j] = __ldcg(r + 8 * D + 8 + row);
+                    oo[j] = __ldcg(reinterpret_cast<const float4 *>(r + row * D) + c4);
+                } else {
+                    mm[j] = -INFINITY;
+                    ll[j] = 0.f;
+                    oo[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+            }
+            float Mc = M;
+#pragma unroll
+            for (int j = 0; j < kChunk; ++j) Mc = fmaxf(Mc, mm[j]);
+            const float a = exp2_diff(M, Mc);
+            Lsum *= a;
+            acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
+#pragma unroll
+            for (int j = 0; j < kChunk; ++j) {
+                const float w8 = exp2_diff(mm[j], Mc);
+                Lsum += w8 * ll[j];
+                acc.x += w8 * oo[j].x;
+                acc.y += w8 * oo[j].y;
+                acc.z += w8 * oo[j].z;
+                acc.w += w8 * oo[j].w;
+            }
+            M = Mc;
         }
         const float inv = 1.f / Lsum;
         float *dst = p.out + ((int64_t)i * p.hq + g * p.G + hh) * D;
@@ -785,24 +795,37 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
 // ================================================================ epilogue
 template <int D>
 __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t *dsc, uint64_t *bars,
-                             int32_t *list, uint32_t zero_addr, int lane)
+                             int32_t *list, uint32_t zero_addr, int ep, int lane)
 {
     using L = Lay<D>;
     constexpr int kMaxNt = D / 8;
     constexpr int kMaxKs = D / 16;
+    constexpr int kHalf = kMaxNt / 2;      // column tiles of this warp's half of the head dimension
+    const int ct0 = ep * kHalf;            // first column tile of this warp
+    int neps = 0;                          // record hand-offs between the two epilogue warps
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
     const int quad = lane / 4, qlane = lane % 4;
     const uint32_t pv = smem_u32(smem + L::kPv);
     const int recf = 8 * D + kRecFloatsExtra;
     auto region = [&](int w) { return reinterpret_cast<const float2 *>(smem + L::kMerge + w * L::kMergeWarp); };
 
-    float orun[2][kMaxNt][2];
+    float orun[2][kHalf][2];
     float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
     int ndump = 0, npv = 0;
 #pragma unroll
     for (int a = 0; a < 2; ++a)
 #pragma unroll
-        for (int x = 0; x < kMaxNt; ++x) orun[a][x][0] = orun[a][x][1] = 0.f;
+        for (int x = 0; x < kHalf; ++x) orun[a][x][0] = orun[a][x][1] = 0.f;
+    // Both epilogue warps meet once their halves of a record are written (a
+    // two-warp barrier: neither can run a phase ahead of the other); the
+    // first one then counts the tickets.
+    auto await_partner = [&]() -> bool {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(B_EPS));
+        const bool ok = warp_wait(bar(B_EPS), neps & 1, p.status);
+        ++neps;
+        return ok;
+    };
 
     pdl_wait();  // records and tickets belong to the preceding grid until here
 
@@ -884,7 +907,7 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
                     m_run[grp] = -INFINITY;
                     l_run[grp] = 0.f;
 #pragma unroll
-                    for (int x = 0; x < kMaxNt; ++x) orun[grp][x][0] = orun[grp][x][1] = 0.f;
+                    for (int x = 0; x < kHalf; ++x) orun[grp][x][0] = orun[grp][x][1] = 0.f;
                 }
                 const float m_new = fmaxf(m_run[grp], M);
                 const float a_run = exp2_diff(m_run[grp], m_new), a_seg = exp2_diff(M, m_new);
@@ -900,13 +923,13 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
                         split_hi_lo(y.x, y.y, af[kj][2], af[kj][3]);
                     }
                 }
-                // back-projection through P^V into the run's output
+                // back-projection through P^V into this warp's half of the run's output
                 const int mi = lane / 8;
 #pragma unroll
-                for (int cp = 0; cp < kMaxNt / 2; ++cp) {
+                for (int cp = 0; cp < kHalf / 2; ++cp) {
                     float oa[4] = {0.f, 0.f, 0.f, 0.f}, ob[4] = {0.f, 0.f, 0.f, 0.f};
-                    // tiles (2kj, 2cp), (2kj+1, 2cp), (2kj, 2cp+1), (2kj+1, 2cp+1) of P^V
-                    const int ct = 2 * cp + (mi >> 1);
+                    // tiles (2kj, c), (2kj+1, c), (2kj, c+1), (2kj+1, c+1) of P^V, c = ct0 + 2cp
+                    const int ct = ct0 + 2 * cp + (mi >> 1);
 #pragma unroll
                     for (int kj = 0; kj < kMaxKs; ++kj) {
                         if (kj < nkj) {
@@ -941,16 +964,16 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
                     if (rg >= p.nrg) continue;
                     float *rec = p.rec + ((int64_t)recslot * p.nrg + rg) * recf;
 #pragma unroll
-                    for (int x = 0; x < kMaxNt; ++x)
-                        __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * x + 2 * qlane),
+                    for (int x = 0; x < kHalf; ++x)
+                        __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * (ct0 + x) + 2 * qlane),
                                make_float2(orun[grp][x][0], orun[grp][x][1]));
-                    if (qlane == 0) {
+                    if (ep == 0 && qlane == 0) {
                         __stcg(rec + 8 * D + quad, m_run[grp]);
                         __stcg(rec + 8 * D + 8 + quad, l_run[grp]);
                     }
                     __threadfence();
-                    __syncwarp();
-                    ticket(g, rg);
+                    if (!await_partner()) return false;
+                    if (ep == 0) ticket(g, rg);
                 }
             }
         } else {  // tail item: the merged accumulator is already the output
@@ -962,9 +985,10 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
                 merge_scales(ngrp, grp, sc, M, Lsum);
                 float *rec = p.rec + (p.tail_rec_base + (int64_t)item * p.nrg_t + rgt) * recf;
 #pragma unroll
-                for (int x = 0; x < kMaxNt; ++x)
-                    __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * x + 2 * qlane), merged_pair(sc, x));
-                if (qlane == 0) {
+                for (int x = 0; x < kHalf; ++x)
+                    __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * (ct0 + x) + 2 * qlane),
+                           merged_pair(sc, ct0 + x));
+                if (ep == 0 && qlane == 0) {
                     __stcg(rec + 8 * D + quad, M);
                     __stcg(rec + 8 * D + 8 + quad, Lsum);
                 }
@@ -972,7 +996,11 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(B_ME));
             __threadfence();
-            __syncwarp();
+            if (!await_partner()) return false;
+            if (ep == 1) {
+                ++ndump;
+                continue;
+            }
             // tickets of the prefix row groups these query rows belong to
             for (int grp = 0; grp < ngrp; ++grp) {
                 const int rgt = pass * ngrp + grp;
@@ -1011,14 +1039,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(smem_u32(&bars[B_PKF]), 1);
         mbar_init(smem_u32(&bars[B_PKE]), 1);
         mbar_init(smem_u32(&bars[B_PVF]), 1);
-        mbar_init(smem_u32(&bars[B_PVE]), 1);
+        mbar_init(smem_u32(&bars[B_PVE]), 2);  // both epilogue warps
         mbar_init(smem_u32(&bars[B_QR0]), 1);
         mbar_init(smem_u32(&bars[B_QR1]), 1);
         mbar_init(smem_u32(&bars[B_QF0]), kMmaWarps);
         mbar_init(smem_u32(&bars[B_QF1]), kMmaWarps);
         mbar_init(smem_u32(&bars[B_MF]), kMmaWarps);
-        mbar_init(smem_u32(&bars[B_ME]), 1);
-        mbar_init(smem_u32(&bars[B_FIN]), 2 + kMmaWarps);
+        mbar_init(smem_u32(&bars[B_ME]), 2);   // both epilogue warps
+        mbar_init(smem_u32(&bars[B_EPS]), 2);
+        mbar_init(smem_u32(&bars[B_FIN]), 3 + kMmaWarps);
         list[0] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -1032,10 +1061,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok;
     if (warp == 1)
         ok = run_projection<D>(p, smem, pkh, bars, lane);
-    else if (warp == 2)
-        ok = run_epilogue<D>(p, smem, dsc, bars, list, zero_addr, lane);
+    else if (warp <= 3)
+        ok = run_epilogue<D>(p, smem, dsc, bars, list, zero_addr, warp - 2, lane);
     else
-        ok = run_mma<D>(p, smem, hdr, dsc, bars, zero_addr, warp - 3, lane);
+        ok = run_mma<D>(p, smem, hdr, dsc, bars, zero_addr, warp - 4, lane);
     if (!ok) return;
     // every role done: merge the row groups this thread block completed
     __syncwarp();

@@ -30,10 +30,10 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint16_t *__restrict__ 
     uint8_t *dst = packed + dst0;
     if (r8 == 0) return;
     if ((f & 1) == 0) {
-        // coefficients C (n x r): tiles of 64 tokens, inside [rank group][token group]
+        // coefficients C (n x r): tiles of kTileTokens tokens, inside [rank group][token group]
         const int n = ent.n, n8 = (n + 7) & ~7;
         const int64_t chunks = (int64_t)n8 * r8 / 8;
-        const int per_full_tile = 8 * r8;  // 16-byte lines in a 64-token tile
+        const int per_full_tile = kTileTokens * r8 / 8;  // 16-byte lines in a full tile
         for (int64_t qi = threadIdx.x; qi < chunks; qi += blockDim.x) {
             const int kt = (int)(qi / per_full_tile);
             const int qq = (int)(qi % per_full_tile);
