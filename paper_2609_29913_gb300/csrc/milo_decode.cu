@@ -11,11 +11,11 @@
 // One persistent thread block per SM with four warp roles:
 //   producer    (warp 0, one lane): walks the block's static list of prefix
 //               segments, bulk-copies each segment's P^K and P^V into their
-//               own buffers and its packed coefficient tiles into a ring of
+//               own buffers (P^V double-buffered) and its packed coefficient tiles into a ring of
 //               slots (1-D cp.async.bulk, mbarrier completion); grabs dense
 //               tail items from a counter and streams them with 3-D TMA.
 //   projection  (warp 1): q~ = scale * log2(e) * P^K q for every segment, as
-//               bf16 hi + lo mma fragments, into a double buffer.
+//               bf16 hi + lo mma fragments, into a shared buffer.
 //   MMA warps   (warps 4..11): 16-token sub-tiles round-robin: scores (mma
 //               m16n8k16; A rows 0-7 = q~ hi, 8-15 = q~ lo), online softmax
 //               in registers, rank-space values (A rows = p hi / p lo).  At a
@@ -49,7 +49,7 @@ enum : int { F_FIRST_C = 1, F_LAST_C = 2, F_RUN_FIRST = 4, F_RUN_LAST = 8 };
 enum : int { H_KIND, H_E, H_G, H_T0, H_T1, H_RK8, H_RV8, H_TOK8, H_NSUB, H_FLAGS, H_REC, H_PASS, H_QI, H_ITEM };
 // barrier indices (after the ring's full[kSlots], empty[kSlots])
 enum : int {
-    B_PKF = 2 * kSlots, B_PKE, B_PVF, B_PVE, B_QR0, B_QR1, B_QF0, B_QF1, B_MF, B_ME, B_EPS, B_FIN, B_COUNT
+    B_PKF = 2 * kSlots, B_PKE, B_PVF0, B_PVF1, B_PVE0, B_PVE1, B_QR, B_QF, B_MF, B_ME, B_EPS, B_FIN, B_COUNT
 };
 
 // ------------------------------------------------------------------ PTX ----
@@ -196,12 +196,12 @@ struct Lay {
     static constexpr int al(int x, int a) { return (x + a - 1) / a * a; }
     static constexpr int kPBytes = D * D * 2;                   // largest P (r <= d)
     static constexpr int kPk = kSlots * kSlotBytes;             // ring at 0
-    static constexpr int kPv = kPk + kPBytes;
-    static constexpr int kMerge = kPv + kPBytes;
+    static constexpr int kPv = kPk + kPBytes;                   // two P^V buffers
+    static constexpr int kMerge = kPv + 2 * kPBytes;
     static constexpr int kMergeWarp = 32 * D + 256;             // v~ [d/8][32 lanes] float2 + (m,l) [32] float2
-    static constexpr int kQsPart = (D / 16) * 32 * 16;          // q~ fragments of one (parity, row group)
+    static constexpr int kQsPart = (D / 16) * 32 * 16;          // q~ fragments of one row group
     static constexpr int kQs = kMerge + kMmaWarps * kMergeWarp;
-    static constexpr int kHdr = kQs + 4 * kQsPart;              // ring headers, P^K header, dump descriptor
+    static constexpr int kHdr = kQs + 2 * kQsPart;              // ring headers, P^K header, dump descriptor
     static constexpr int kBar = al(kHdr + (kSlots + 2) * 64, 128);
     static constexpr int kZero = al(kBar + B_COUNT * 8, 128);
     static constexpr int kList = kZero + 128;                   // deferred combines: count, (g, rg) pairs
@@ -360,13 +360,14 @@ __device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr,
         return true;
     };
     auto emit_pv = [&](int rv8, int64_t off) -> bool {
-        if (npv >= 1 && !mbar_wait(bar(B_PVE), (npv - 1) & 1, p.status)) return false;
+        const int b = npv & 1;  // double-buffered: the epilogue may still hold the other one
+        if (npv >= 2 && !mbar_wait(bar(B_PVE0 + b), ((npv / 2) - 1) & 1, p.status)) return false;
         const uint32_t bytes = (uint32_t)rv8 * D * 2;
         if (bytes) {
-            mbar_arrive_tx(bar(B_PVF), bytes);
-            bulk_g2s(smem_u32(smem + L::kPv), p.packed + off, bytes, bar(B_PVF));
+            mbar_arrive_tx(bar(B_PVF0 + b), bytes);
+            bulk_g2s(smem_u32(smem + L::kPv + b * L::kPBytes), p.packed + off, bytes, bar(B_PVF0 + b));
         } else {
-            mbar_arrive(bar(B_PVF));
+            mbar_arrive(bar(B_PVF0 + b));
         }
         ++npv;
         return true;
@@ -518,7 +519,7 @@ __device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr,
     for (int j = max(0, seq - kSlots); j < seq; ++j)
         if (!mbar_wait(bar(j % kSlots), (j / kSlots) & 1, p.status)) break;
     if (npk > 0) mbar_wait(bar(B_PKF), (npk - 1) & 1, p.status);
-    if (npv > 0) mbar_wait(bar(B_PVF), (npv - 1) & 1, p.status);
+    for (int j = max(0, npv - 2); j < npv; ++j) mbar_wait(bar(B_PVF0 + (j & 1)), (j / 2) & 1, p.status);
 }
 
 // ================================================================ projection
@@ -536,8 +537,9 @@ __device__ bool run_projection(const DecodeParams &p, uint8_t *smem, const int32
         const int kind = pkh[0];
         if (kind == kPkEnd) return true;
         const int g = pkh[1], rk8 = pkh[2], pass = pkh[3];
-        const int par = k & 1;
-        if (k >= 2 && !warp_wait(bar(B_QF0 + par), ((k / 2) - 1) & 1, p.status)) return false;
+        // the MMA warps load segment k-1's q~ when they start it, long before
+        // segment k's basis arrives: one buffer suffices
+        if (k >= 1 && !warp_wait(bar(B_QF), (k - 1) & 1, p.status)) return false;
         for (int grp = 0; grp < p.nrg_cta; ++grp) {
             const int rg = pass * p.nrg_cta + grp;
             const int rho = 8 * rg + quad;
@@ -552,7 +554,7 @@ __device__ bool run_projection(const DecodeParams &p, uint8_t *smem, const int32
                 qlo[kc] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 2 * qlane) : 0u;
                 qhi[kc] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 8 + 2 * qlane) : 0u;
             }
-            uint4 *qs = reinterpret_cast<uint4 *>(smem + L::kQs + (par * 2 + grp) * L::kQsPart);
+            uint4 *qs = reinterpret_cast<uint4 *>(smem + L::kQs + grp * L::kQsPart);
             const int njt = 2 * ((rk8 + 15) / 16);
             for (int jt = 0; jt < njt; ++jt) {
                 float acc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -579,7 +581,7 @@ __device__ bool run_projection(const DecodeParams &p, uint8_t *smem, const int32
         __syncwarp();
         if (lane == 0) {
             mbar_arrive(bar(B_PKE));
-            mbar_arrive(bar(B_QR0 + par));
+            mbar_arrive(bar(B_QR));
         }
     }
 }
@@ -706,11 +708,10 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
             const int flags = h[H_FLAGS], rk8 = h[H_RK8], rv8 = h[H_RV8];
             const int nks = (rk8 + 15) / 16, njp = (rv8 + 15) / 16;
             if (flags & F_FIRST_C) {
-                const int par = nseg & 1;
-                if (!warp_wait(bar(B_QR0 + par), (nseg / 2) & 1, p.status)) return false;
+                if (!warp_wait(bar(B_QR), nseg & 1, p.status)) return false;
                 active = rg < p.nrg;
                 if (active) {
-                    const uint4 *qs = reinterpret_cast<const uint4 *>(smem + L::kQs + (par * 2 + grp) * L::kQsPart);
+                    const uint4 *qs = reinterpret_cast<const uint4 *>(smem + L::kQs + grp * L::kQsPart);
 #pragma unroll
                     for (int kk = 0; kk < kMaxKs; ++kk)
                         if (kk < nks) {
@@ -719,7 +720,7 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
                         }
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(bar(B_QF0 + par));
+                if (lane == 0) mbar_arrive(bar(B_QF));
                 reset_state();
                 ++nseg;
             }
@@ -805,7 +806,7 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
     int neps = 0;                          // record hand-offs between the two epilogue warps
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
     const int quad = lane / 4, qlane = lane % 4;
-    const uint32_t pv = smem_u32(smem + L::kPv);
+    const uint32_t pv_base = smem_u32(smem + L::kPv);
     const int recf = 8 * D + kRecFloatsExtra;
     auto region = [&](int w) { return reinterpret_cast<const float2 *>(smem + L::kMerge + w * L::kMergeWarp); };
 
@@ -893,9 +894,16 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
         const int g = dsc[1], rv8 = dsc[2], flags = dsc[3], recslot = dsc[4], pass = dsc[5];
         const int item = dsc[6], qi = dsc[7];
         if (kind == kDumpSeg) {
-            if (!warp_wait(bar(B_PVF), npv & 1, p.status)) return false;
+            const int pb = npv & 1;
+            if (!warp_wait(bar(B_PVF0 + pb), (npv / 2) & 1, p.status)) return false;
+            const uint32_t pv = pv_base + pb * L::kPBytes;
             const int nkj = (rv8 + 15) / 16, nvt = rv8 / 8;
             const int ngrp = p.nrg_cta;
+            // the dump regions are free once the last row group is merged
+            int last_grp = 0;
+            for (int x = 0; x < ngrp; ++x)
+                if (pass * ngrp + x < p.nrg) last_grp = x;
+            bool me_done = false;
 #pragma unroll
             for (int grp = 0; grp < 2; ++grp) {
                 if (grp >= ngrp) break;
@@ -922,6 +930,11 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
                         split_hi_lo(x.x, x.y, af[kj][0], af[kj][1]);
                         split_hi_lo(y.x, y.y, af[kj][2], af[kj][3]);
                     }
+                }
+                if (grp == last_grp) {
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar(B_ME));
+                    me_done = true;
                 }
                 // back-projection through P^V into this warp's half of the run's output
                 const int mi = lane / 8;
@@ -952,8 +965,8 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
             }
             __syncwarp();
             if (lane == 0) {
-                mbar_arrive(bar(B_ME));
-                mbar_arrive(bar(B_PVE));
+                if (!me_done) mbar_arrive(bar(B_ME));
+                mbar_arrive(bar(B_PVE0 + pb));
             }
             ++npv;
             if (flags & F_RUN_LAST) {
@@ -1038,12 +1051,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(smem_u32(&bars[B_PKF]), 1);
         mbar_init(smem_u32(&bars[B_PKE]), 1);
-        mbar_init(smem_u32(&bars[B_PVF]), 1);
-        mbar_init(smem_u32(&bars[B_PVE]), 2);  // both epilogue warps
-        mbar_init(smem_u32(&bars[B_QR0]), 1);
-        mbar_init(smem_u32(&bars[B_QR1]), 1);
-        mbar_init(smem_u32(&bars[B_QF0]), kMmaWarps);
-        mbar_init(smem_u32(&bars[B_QF1]), kMmaWarps);
+        mbar_init(smem_u32(&bars[B_PVF0]), 1);
+        mbar_init(smem_u32(&bars[B_PVF1]), 1);
+        mbar_init(smem_u32(&bars[B_PVE0]), 2);  // both epilogue warps
+        mbar_init(smem_u32(&bars[B_PVE1]), 2);
+        mbar_init(smem_u32(&bars[B_QR]), 1);
+        mbar_init(smem_u32(&bars[B_QF]), kMmaWarps);
         mbar_init(smem_u32(&bars[B_MF]), kMmaWarps);
         mbar_init(smem_u32(&bars[B_ME]), 2);   // both epilogue warps
         mbar_init(smem_u32(&bars[B_EPS]), 2);

@@ -10,7 +10,7 @@ namespace milo {
 constexpr int kTileTokens = 32;      // tokens per packed coefficient tile
 constexpr int kMmaWarps = 8;         // score/value warps per decode thread block
 constexpr int kThreads = 32 * (4 + kMmaWarps);  // + producer, projection, 2 epilogue
-constexpr int kSlots = 6;            // coefficient ring depth
+constexpr int kSlots = 5;            // coefficient ring depth
 constexpr int kSlotBytes = 16384;    // bytes per ring slot
 constexpr int kHdrInts = 16;         // slot header (ints)
 constexpr int kTailTokens = 32;      // tokens per dense-tail work item
