@@ -217,6 +217,33 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q,
                                size_t workspace_bytes, void *stream);
 
 /*
+ * milo_attn_decode without a workspace argument: the same computation, with
+ * the partial results kept in a fixed scratch array built into the library
+ * (8 MiB per GPU, held by every GPU that loads the library until the process
+ * exits).  The paper has no counterpart; this exists for callers that cannot
+ * allocate device memory on the decode path -- a plug-in that receives only
+ * its inputs and outputs from a host runtime owning all device memory, or a
+ * caller that must not call cudaMalloc there because it can synchronise the
+ * device and stall other work.
+ *   Arguments are those of milo_attn_decode minus workspace/workspace_bytes.
+ *   Returns MILO_ERR_WORKSPACE if the call needs more scratch than the array
+ *   holds (milo_workspace_size tells), without launching anything.
+ *   The call allocates nothing.  Its first call on a device looks up the
+ *   array's device address (once per device, with that device current); make
+ *   that first call before any stream capture.  The scratch needs no
+ *   clearing (every partial result is written before it is read in the same
+ *   call) and keeps the last call's contents; all calls on a device share it,
+ *   so calls that can overlap on the GPU (different streams) race.
+ */
+milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q,
+                                      int32_t batch, const void *tail_k,
+                                      const void *tail_v,
+                                      const int64_t *tail_offsets,
+                                      int64_t tail_rows, int64_t max_tail_tokens,
+                                      float softmax_scale, float *out,
+                                      void *stream);
+
+/*
  * Read (and optionally clear) the plan's sticky device status word, which the
  * kernels set on a timed-out wait (MILO_ERR_TIMEOUT) or a failed device-side
  * index check (MILO_ERR_DEVICE_BOUNDS).  Synchronises `stream`.

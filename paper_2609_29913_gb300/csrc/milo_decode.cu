@@ -33,6 +33,8 @@
 #include <cuda.h>
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "milo.h"
 #include "milo_internal.h"
 
@@ -1089,6 +1091,33 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 }  // namespace
+
+// Scratch of milo_attn_decode_static: the split-softmax partial records of
+// one call live here instead of in a caller-provided workspace.  Every GPU
+// that loads the library holds this array until the process exits.
+static __device__ __align__(256) unsigned char g_static_workspace[kStaticWorkspaceBytes];
+
+cudaError_t static_workspace(void **ptr)
+{
+    // Host code cannot use the array's name as a device address: look the
+    // address up once per device, with that device current, and keep it.
+    constexpr int kMaxDevices = 64;
+    static std::mutex mu;
+    static void *addr[kMaxDevices] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_workspace);
+        if (e != cudaSuccess) return e;
+        addr[dev] = p;
+    }
+    *ptr = addr[dev];
+    return cudaSuccess;
+}
 
 int decode_smem_bytes(int head_dim, int /*nrg_cta*/)
 {

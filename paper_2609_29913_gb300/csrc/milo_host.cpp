@@ -538,6 +538,26 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     return MILO_OK;
 }
 
+milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q, int32_t batch,
+                                      const void *tail_k, const void *tail_v, const int64_t *tail_offsets,
+                                      int64_t tail_rows, int64_t max_tail_tokens, float softmax_scale, float *out,
+                                      void *stream)
+{
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    size_t need = 0;
+    milo_status_t s = milo_workspace_size(plan, batch, max_tail_tokens, &need);
+    if (s != MILO_OK) return s;
+    if (need > kStaticWorkspaceBytes)
+        return fail(MILO_ERR_WORKSPACE, "call needs " + std::to_string(need) +
+                                            " bytes of scratch; the built-in scratch holds " +
+                                            std::to_string(kStaticWorkspaceBytes) + " (use milo_attn_decode)");
+    void *ws = nullptr;
+    cudaError_t e = static_workspace(&ws);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the built-in scratch");
+    return milo_attn_decode(plan, q, batch, tail_k, tail_v, tail_offsets, tail_rows, max_tail_tokens,
+                            softmax_scale, out, ws, kStaticWorkspaceBytes, stream);
+}
+
 milo_status_t milo_get_device_status(const milo_prefix_t *plan, void *stream, int32_t clear, int32_t *code)
 {
     if (!plan || !code) return fail(MILO_ERR_INVALID_ARG, "null argument");

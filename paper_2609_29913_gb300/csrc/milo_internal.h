@@ -84,4 +84,10 @@ cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k,
 
 int decode_smem_bytes(int head_dim, int nrg_cta);
 
+// Fixed scratch of milo_attn_decode_static (a file-scope device array).
+constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;
+// Device address of that array on the current device (looked up once per
+// device).
+cudaError_t static_workspace(void **ptr);
+
 }  // namespace milo

@@ -30,7 +30,8 @@ STATUS_NAMES = {0: "MILO_OK", 1: "MILO_ERR_INVALID_ARG", 2: "MILO_ERR_BAD_TABLE"
 EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
            "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
-           "milo_workspace_size", "milo_attn_decode", "milo_get_device_status"]
+           "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
+           "milo_get_device_status"]
 
 
 class MiloError(RuntimeError):
@@ -82,10 +83,12 @@ def lib():
         L.milo_workspace_size.argtypes = [P, i32, i64, P]
         L.milo_attn_decode.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P,
                                        ctypes.c_size_t, P]
+        L.milo_attn_decode_static.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         for name in ("milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
                      "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
-                     "milo_workspace_size", "milo_attn_decode", "milo_get_device_status"):
+                     "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
+                     "milo_get_device_status"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -204,6 +207,16 @@ def milo_attn_decode(plan: int, q_ptr: int, batch: int, tail_k_ptr: int, tail_v_
                                   tail_offsets_ptr or None, int(tail_rows), int(max_tail_tokens),
                                   float(softmax_scale), out_ptr, workspace_ptr,
                                   int(workspace_bytes), _stream_ptr(stream)), "milo_attn_decode")
+
+
+def milo_attn_decode_static(plan: int, q_ptr: int, batch: int, tail_k_ptr: int, tail_v_ptr: int,
+                            tail_offsets_ptr: int, tail_rows: int, max_tail_tokens: int,
+                            softmax_scale: float, out_ptr: int, stream=None) -> None:
+    """milo_attn_decode with the library's built-in scratch (no workspace)."""
+    _check(lib().milo_attn_decode_static(plan, q_ptr, int(batch), tail_k_ptr or None,
+                                         tail_v_ptr or None, tail_offsets_ptr or None,
+                                         int(tail_rows), int(max_tail_tokens), float(softmax_scale),
+                                         out_ptr, _stream_ptr(stream)), "milo_attn_decode_static")
 
 
 def milo_get_device_status(plan: int, stream=None, clear: bool = False) -> int:
