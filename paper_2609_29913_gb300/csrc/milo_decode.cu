@@ -8,32 +8,34 @@
 // split softmax (Eq. 1 is associative over token partitions once each part
 // carries its running max and sum).
 //
-// One persistent thread block per SM with four warp roles:
-//   producer    (warp 0, one lane): walks the block's static list of prefix
-//               segments, bulk-copies each segment's P^K and P^V into their
-//               own buffers (P^V double-buffered) and its packed coefficient tiles into a ring of
-//               slots (1-D cp.async.bulk, mbarrier completion); grabs dense
-//               tail items from a counter and streams them with 3-D TMA.
-//   projection  (warp 1): q~ = scale * log2(e) * P^K q for every segment, as
-//               bf16 hi + lo mma fragments, into a shared buffer.
-//   MMA warps   (warps 4..11): 16-token sub-tiles round-robin: scores (mma
-//               m16n8k16; A rows 0-7 = q~ hi, 8-15 = q~ lo), online softmax
-//               in registers, rank-space values (A rows = p hi / p lo).  At a
-//               segment's end each warp dumps (max, sum, v~) into its own
-//               shared-memory region and continues with the next segment.
-//   epilogue    (warps 2-3): both merge the 8 dumps of a segment; each
-//               back-projects v~ through P^V into half of the head dimension,
-//               folds it into its half of the run's output and writes it to
-//               the partial record; the first counts the tickets.
+// One persistent thread block per SM, two roles:
+//   producer   (warp 0, one lane): turns the block's static list of prefix
+//              segments, then dynamically claimed dense-tail items, into an
+//              in-order stream of "fills" of at most kSlotBytes.  A fill packs
+//              the previous segment's P^V, the next segment's P^K and as many
+//              whole coefficient tiles of that segment as fit; a tail fill
+//              holds one tail item's K and V (3-D TMA, 128-byte swizzle).  Each
+//              fill is one ring slot, one mbarrier, up to four bulk copies.
+//   MMA warps  (warps 1..7): consume every fill in order.  P^K part: each warp
+//              projects q~ = scale * log2(e) * P^K q for a slice of the rank
+//              tiles (mma m16n8k16, result split into bf16 hi + lo rows).
+//              Coefficient part: 16-token sub-tiles round-robin over the
+//              warps -- scores (A rows 0-7 q~ hi, rows 8-15 q~ lo), online
+//              softmax in registers, rank-space values (A rows = p hi, p lo).
+//              P^V part (segment end): the warps pool their (max, sum, v~),
+//              each merges a slice of v~, then each back-projects a slice of
+//              the head dimension through P^V into its running output; at the
+//              end of a run the slices are written as one partial record.
+//              Tail fills go whole to one warp each (no pooling needed).
 // The thread block that brings the last record of a (KV head, row group)
-// merges all of that row group's records at the end of the kernel (no
-// thread block ever waits for another).  Every wait is bounded (~2 s); on
-// expiry the thread records MILO_ERR_TIMEOUT in the sticky status word and
-// leaves.
+// merges that row group's records at the end of the kernel; no thread block
+// waits for another.  Every wait is bounded (~2 s); on expiry the thread
+// records MILO_ERR_TIMEOUT in the sticky status word and leaves.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
 #include <mutex>
+#include <type_traits>
 
 #include "milo.h"
 #include "milo_internal.h"
@@ -43,15 +45,34 @@ namespace {
 
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 
-enum : int { kEnd = 0, kC = 2, kTail = 4 };             // ring slot kinds
-enum : int { kPkEnd = 0, kPkSeg = 1 };                  // P^K buffer kinds
-enum : int { kDumpEnd = 0, kDumpSeg = 1, kDumpTail = 2 };
-enum : int { F_FIRST_C = 1, F_LAST_C = 2, F_RUN_FIRST = 4, F_RUN_LAST = 8 };
-// ring slot header words
-enum : int { H_KIND, H_E, H_G, H_T0, H_T1, H_RK8, H_RV8, H_TOK8, H_NSUB, H_FLAGS, H_REC, H_PASS, H_QI, H_ITEM };
-// barrier indices (after the ring's full[kSlots], empty[kSlots])
+// fill flags: a fill carries, in processing order, the previous segment's
+// P^V, up to two bases P^K of coming segments, the start of a segment, its
+// coefficient tiles, a tail item, the end marker
+enum : int { kHasPv = 1, kHasPk0 = 2, kHasPk1 = 4, kSegStart = 8, kHasC = 16, kTailFill = 32, kEndFill = 64 };
+// run flags of a segment end
+enum : int { F_RUN_FIRST = 1, F_RUN_LAST = 2 };
+// fill header words
 enum : int {
-    B_PKF = 2 * kSlots, B_PKE, B_PVF0, B_PVF1, B_PVE0, B_PVE1, B_QR, B_QF, B_MF, B_ME, B_EPS, B_FIN, B_COUNT
+    H_FLAGS,
+    H_PV_G, H_PV_RV8, H_PV_REC, H_PV_RUN, H_PV_PASS, H_PV_OFF,
+    H_PK_J, H_PK_G, H_PK_RK8, H_PK_PASS, H_PK_OFF,  // P^K part 0; part 1 follows with the same layout
+    H_PK1_J = H_PK_J + 5,
+    H_SS_J = H_PK1_J + 5, H_SS_PASS, H_SS_RK8,
+    H_C_OFF, H_T0, H_T1, H_RK8, H_RV8, H_TOK8,
+    H_QI, H_G, H_ITEM,
+    H_WORDS
+};
+static_assert(H_WORDS <= kHdrInts, "fill header size");
+// barrier indices: full[kSlots], empty[kSlots], then the MMA warps' own
+enum : int {
+    B_GS = 2 * kSlots,  // group sync of the MMA warps
+    B_FIN,              // final meeting of all warps
+    B_QREADY,           // [2] q~ buffer written by every MMA warp
+    B_QFREE = B_QREADY + 2,  // [2] q~ buffer loaded by every MMA warp
+    B_DUMPED = B_QFREE + 2,  // every MMA warp dumped its state of a segment
+    B_MERGED,           // every MMA warp merged its slice of the pooled v~
+    B_BPDONE,           // every MMA warp back-projected (merged v~ buffer free)
+    B_COUNT
 };
 
 // ------------------------------------------------------------------ PTX ----
@@ -80,6 +101,19 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t tx)
 __device__ __forceinline__ void mbar_arrive(uint32_t bar)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
 }
 
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
@@ -196,22 +230,26 @@ __device__ __forceinline__ float exp2_diff(float a, float b)
 template <int D>
 struct Lay {
     static constexpr int al(int x, int a) { return (x + a - 1) / a * a; }
-    static constexpr int kPBytes = D * D * 2;                   // largest P (r <= d)
-    static constexpr int kPk = kSlots * kSlotBytes;             // ring at 0
-    static constexpr int kPv = kPk + kPBytes;                   // two P^V buffers
-    static constexpr int kMerge = kPv + 2 * kPBytes;
-    static constexpr int kMergeWarp = 32 * D + 256;             // v~ [d/8][32 lanes] float2 + (m,l) [32] float2
-    static constexpr int kQsPart = (D / 16) * 32 * 16;          // q~ fragments of one row group
-    static constexpr int kQs = kMerge + kMmaWarps * kMergeWarp;
-    static constexpr int kHdr = kQs + 2 * kQsPart;              // ring headers, P^K header, dump descriptor
-    static constexpr int kBar = al(kHdr + (kSlots + 2) * 64, 128);
+    static constexpr int kRing = 0;                               // kSlots fills
+    static constexpr int kMerge = kRing + kSlots * kSlotBytes;    // per-warp (max, sum, v~) dumps
+    static constexpr int kMergeWarp = 32 * D + 256;               // v~ [d/8][32 lanes] float2 + (m,l) [32] float2
+    static constexpr int kFragPart = (D / 16) * 32 * 16;          // A fragments (hi/lo) of one row group
+    static constexpr int kQs = kMerge + kMmaWarps * kMergeWarp;   // q~ [2 buffers][2 row groups]
+    static constexpr int kAf = kQs + 4 * kFragPart;               // merged v~ of two row groups
+    static constexpr int kHdr = kAf + 2 * kFragPart;
+    static constexpr int kQc = al(kHdr + kSlots * kHdrInts * 4, 128);  // copy of q when it is small
+    static constexpr int kQcBytes = 8192;
+    static constexpr int kBar = kQc + kQcBytes;
     static constexpr int kZero = al(kBar + B_COUNT * 8, 128);
-    static constexpr int kList = kZero + 128;                   // deferred combines: count, (g, rg) pairs
-    static constexpr int kListCap = 255;
-    static constexpr int kTotal = kList + 8 * (kListCap + 1);
-    static_assert(kPk % 1024 == 0 && kSlotBytes % 1024 == 0, "ring alignment (128B-swizzled TMA boxes)");
-    static_assert(kPv % 128 == 0 && kMerge % 128 == 0 && kQs % 128 == 0 && kHdr % 128 == 0, "alignment");
-    static_assert(kZero % 128 == 0, "zero line alignment");
+    static constexpr int kList = kZero + 128;                     // count of row groups to merge (list in the workspace)
+    static constexpr int kTkCap = 255;                            // tail records to count at the end
+    static constexpr int kTkT = kList + 128;                      //   count, (g, rg) pairs
+    static constexpr int kTotal = kTkT + 8 * (kTkCap + 1);
+    static_assert(kSlotBytes % 1024 == 0, "ring slots must keep 1024-byte alignment (128B-swizzled TMA boxes)");
+    static_assert(kMerge % 128 == 0 && kQs % 128 == 0 && kAf % 128 == 0 && kHdr % 128 == 0, "alignment");
+    static_assert(kQc % 128 == 0 && kBar % 128 == 0, "alignment");
+    static_assert(2 * D * kTailTokens * 2 <= kSlotBytes, "a tail item must fit one fill");
+    static_assert(D * D * 2 <= kSlotBytes, "a full-rank basis must fit one fill");
     static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
 
@@ -220,7 +258,7 @@ struct Lay {
 template <int D>
 __device__ void combine_rows(const DecodeParams &p, int g, int rg, int tid, int nthr)
 {
-    constexpr int kChunk = 12;  // records whose loads are in flight together
+    constexpr int kChunk = 8;  // records whose loads are in flight together
     const int recf = 8 * D + kRecFloatsExtra;
     const int gs0 = p.g_slot_begin[g], gs1 = p.g_slot_begin[g + 1];
     const int nprefix = gs1 - gs0;
@@ -332,89 +370,198 @@ struct SegIter {
 
 // ================================================================ producer
 template <int D>
-__device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr, int32_t *pkh, uint64_t *bars,
+__device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr, uint64_t *bars,
                              const CUtensorMap *tmap_k, const CUtensorMap *tmap_v)
 {
-    using L = Lay<D>;
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
-    int seq = 0, npk = 0, npv = 0;
-    bool ok = true, waited = false;
+    // a tail item lands as cores [column group][token group] (one 16-byte column
+    // chunk per box), the layout of a packed coefficient tile
+    constexpr uint32_t kTailChunk = kTailTokens * 16;             // one box: kTailTokens rows x 8 columns
+    constexpr uint32_t kTailBytes = 2 * (D / 8) * kTailChunk;
+    int seq = 0;
+    bool ok = true;
 
-    auto ring_acquire = [&]() -> int {
-        const int slot = seq % kSlots;
-        if (seq >= kSlots && !mbar_wait(bar(kSlots + slot), ((seq / kSlots) - 1) & 1, p.status)) return -1;
-        return slot;
-    };
-    auto emit_pk = [&](int kind, int g, int rk8, int pass, int64_t off) -> bool {
-        if (npk >= 1 && !mbar_wait(bar(B_PKE), (npk - 1) & 1, p.status)) return false;
-        pkh[0] = kind;
-        pkh[1] = g;
-        pkh[2] = rk8;
-        pkh[3] = pass;
-        const uint32_t bytes = kind == kPkSeg ? (uint32_t)rk8 * D * 2 : 0u;
-        if (bytes) {
-            mbar_arrive_tx(bar(B_PKF), bytes);
-            bulk_g2s(smem_u32(smem + L::kPk), p.packed + off, bytes, bar(B_PKF));
-        } else {
-            mbar_arrive(bar(B_PKF));
-        }
-        ++npk;
+    // the fill under construction
+    int slot = 0, flags = 0, ncp = 0;
+    uint32_t used = 0;
+    int32_t *h = nullptr;
+    uint32_t cp_off[6], cp_bytes[6];
+    const uint8_t *cp_src[6];
+    int tail_row = -1, tail_g = 0;
+
+    auto open_fill = [&]() -> bool {
+        slot = seq % kSlots;
+        if (seq >= kSlots && !mbar_wait(bar(kSlots + slot), ((seq / kSlots) - 1) & 1, p.status)) return false;
+        h = hdr + slot * kHdrInts;
+        used = 0;
+        flags = 0;
+        ncp = 0;
+        tail_row = -1;
         return true;
     };
-    auto emit_pv = [&](int rv8, int64_t off) -> bool {
-        const int b = npv & 1;  // double-buffered: the epilogue may still hold the other one
-        if (npv >= 2 && !mbar_wait(bar(B_PVE0 + b), ((npv / 2) - 1) & 1, p.status)) return false;
-        const uint32_t bytes = (uint32_t)rv8 * D * 2;
-        if (bytes) {
-            mbar_arrive_tx(bar(B_PVF0 + b), bytes);
-            bulk_g2s(smem_u32(smem + L::kPv + b * L::kPBytes), p.packed + off, bytes, bar(B_PVF0 + b));
+    auto add_copy = [&](uint32_t off, const uint8_t *src, uint32_t bytes) {
+        if (bytes == 0) return;
+        cp_off[ncp] = off;
+        cp_src[ncp] = src;
+        cp_bytes[ncp] = bytes;
+        ++ncp;
+    };
+    auto close_fill = [&]() {
+        h[H_FLAGS] = flags;
+        const uint32_t fb = bar(slot);
+        uint32_t tx = tail_row >= 0 ? kTailBytes : 0u;
+        for (int c = 0; c < ncp; ++c) tx += cp_bytes[c];
+        const uint32_t base = smem_u32(smem + Lay<D>::kRing + slot * kSlotBytes);
+        if (tx) {
+            mbar_arrive_tx(fb, tx);
+            for (int c = 0; c < ncp; ++c) bulk_g2s(base + cp_off[c], cp_src[c], cp_bytes[c], fb);
+            if (tail_row >= 0) {
+#pragma unroll 1
+                for (int c = 0; c < D / 8; ++c) {
+                    tma_load_3d(base + c * kTailChunk, tmap_k, 8 * c, tail_g, tail_row, fb);
+                    tma_load_3d(base + (D / 8 + c) * kTailChunk, tmap_v, 8 * c, tail_g, tail_row, fb);
+                }
+            }
         } else {
-            mbar_arrive(bar(B_PVF0 + b));
+            mbar_arrive(fb);
         }
-        ++npv;
+        ++seq;
+    };
+
+    // P^V of the last finished segment, attached to the next fill
+    bool pv_pending = false;
+    int pv_g = 0, pv_rv8 = 0, pv_rec = 0, pv_run = 0, pv_pass = 0;
+    int64_t pv_off = 0;
+    auto put_pv = [&]() {
+        const uint32_t bytes = (uint32_t)pv_rv8 * D * 2;
+        h[H_PV_G] = pv_g;
+        h[H_PV_RV8] = pv_rv8;
+        h[H_PV_REC] = pv_rec;
+        h[H_PV_RUN] = pv_run;
+        h[H_PV_PASS] = pv_pass;
+        h[H_PV_OFF] = (int)used;
+        add_copy(used, p.packed + pv_off, bytes);
+        used += bytes;
+        flags |= kHasPv;
+        pv_pending = false;
+    };
+    auto flush_pv = [&]() -> bool {
+        if (!pv_pending) return true;
+        if (!open_fill()) return false;
+        put_pv();
+        close_fill();
         return true;
     };
+
+    // P^K goes out one segment early (the MMA warps project while the previous
+    // segment streams); pk_it walks the (segment, pass) sequence ahead of it
+    SegIter pk_it;
+    int pk_j = 0;
+    auto put_pks = [&](int j) {
+        for (int part = 0; part < 2 && !pk_it.done && pk_j <= j + 1; ++part) {
+            const EntryDev e = p.entries[p.segs[pk_it.sg].entry];
+            const int rk8 = (e.rk + 7) & ~7;
+            const uint32_t bytes = (uint32_t)rk8 * D * 2;
+            if (used + bytes > (uint32_t)kSlotBytes) return;
+            int32_t *f = h + H_PK_J + 5 * part;
+            f[0] = pk_j;
+            f[1] = e.g;
+            f[2] = rk8;
+            f[3] = pk_it.pass;
+            f[4] = (int)used;
+            add_copy(used, p.packed + e.off_pk, bytes);
+            used += bytes;
+            flags |= part == 0 ? kHasPk0 : kHasPk1;
+            ++pk_j;
+            pk_it.advance(p);
+        }
+    };
+
+    auto emit_segment = [&](const SegIter &it, int j) -> bool {
+        const SegDev seg = p.segs[it.sg];
+        const EntryDev ent = p.entries[seg.entry];
+        const int rk8 = (ent.rk + 7) & ~7, rv8 = (ent.rv + 7) & ~7;
+        const int n8 = (ent.n + 7) & ~7;
+        bool started = false;
+        int t = seg.t0;
+        while (!started || t < seg.t1) {
+            if (!open_fill()) return false;
+            if (pv_pending) put_pv();
+            put_pks(j);
+            if (!started) {
+                if (pk_j <= j) {  // this segment's basis has not gone out yet
+                    close_fill();
+                    continue;
+                }
+                h[H_SS_J] = j;
+                h[H_SS_PASS] = it.pass;
+                h[H_SS_RK8] = rk8;
+                flags |= kSegStart;
+                started = true;
+            }
+            if (t < seg.t1) {
+                // whole coefficient tiles (the entry's last one may be short)
+                const uint32_t cap = (uint32_t)kSlotBytes - used;
+                int tt1 = t;
+                uint32_t cbytes = 0;
+                while (tt1 < seg.t1) {
+                    const int te = min(tt1 + kTileTokens, seg.t1);
+                    const int tok = min((te + 7) & ~7, n8) - tt1;
+                    const uint32_t b = (uint32_t)tok * (rk8 + rv8) * 2;
+                    if (cbytes + b > cap) break;
+                    cbytes += b;
+                    tt1 = te;
+                }
+                if (tt1 > t) {
+                    const int tok8 = min((tt1 + 7) & ~7, n8) - t;
+                    const uint32_t kb = (uint32_t)tok8 * rk8 * 2, vb = (uint32_t)tok8 * rv8 * 2;
+                    h[H_C_OFF] = (int)used;
+                    h[H_T0] = t;
+                    h[H_T1] = tt1;
+                    h[H_RK8] = rk8;
+                    h[H_RV8] = rv8;
+                    h[H_TOK8] = tok8;
+                    add_copy(used, p.packed + ent.off_ck + (int64_t)t * rk8 * 2, kb);
+                    add_copy(used + kb, p.packed + ent.off_cv + (int64_t)t * rv8 * 2, vb);
+                    used += kb + vb;
+                    flags |= kHasC;
+                    t = tt1;
+                }
+            }
+            close_fill();
+        }
+        pv_pending = true;
+        pv_g = ent.g;
+        pv_rv8 = rv8;
+        pv_rec = seg.slot;
+        pv_run = (it.sg == it.r0 ? F_RUN_FIRST : 0) | (it.sg == it.r1 ? F_RUN_LAST : 0);
+        pv_pass = it.pass;
+        pv_off = ent.off_pv;
+        return true;
+    };
+
     auto emit_tail = [&](uint32_t item) -> bool {
+        if (!flush_pv()) return false;
         const int S = p.tail_splits;
         const int i = item / (p.hkv * S), g = (item / S) % p.hkv, sp = item % S;
         const int64_t o0 = p.tail_offsets[i], o1 = p.tail_offsets[i + 1];
         const int T = (int)(o1 - o0);
         if (sp == S - 1 && T > S * kTailTokens) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
         const int t0 = sp * kTailTokens, t1 = min(t0 + kTailTokens, T);
-        for (int pass = 0; pass < p.npass_t; ++pass) {
-            const int slot = ring_acquire();
-            if (slot < 0) return false;
-            int32_t *h = hdr + slot * kHdrInts;
-            h[H_KIND] = kTail;
-            h[H_G] = g;
-            h[H_QI] = i;
-            h[H_ITEM] = (int)item;
-            h[H_T0] = t0;
-            h[H_T1] = t1;
-            h[H_PASS] = pass;
-            h[H_RV8] = D;
-            h[H_FLAGS] = 0;
-            const uint32_t fb = bar(slot);
-            if (t1 > t0) {
-                constexpr uint32_t half = kTailTokens * 128;  // one box: kTailTokens rows x 64 columns
-                constexpr uint32_t bytes = 2 * (D / 64) * half;
-                mbar_arrive_tx(fb, bytes);
-                const uint32_t dst = smem_u32(smem + slot * kSlotBytes);
-                const int row = (int)(o0 + t0);
-#pragma unroll
-                for (int hb = 0; hb < D / 64; ++hb) {
-                    tma_load_3d(dst + hb * half, tmap_k, 64 * hb, g, row, fb);
-                    tma_load_3d(dst + (D / 64) * half + hb * half, tmap_v, 64 * hb, g, row, fb);
-                }
-            } else {
-                mbar_arrive(fb);
-            }
-            ++seq;
+        if (!open_fill()) return false;
+        h[H_QI] = i;
+        h[H_G] = g;
+        h[H_ITEM] = (int)item;
+        h[H_T0] = t0;
+        h[H_T1] = t1;
+        flags |= kTailFill;
+        if (t1 > t0) {
+            tail_row = (int)(o0 + t0);
+            tail_g = g;
         }
+        close_fill();
         return true;
     };
-    const uint32_t tail_quota =
-        p.has_tail ? (uint32_t)((p.num_tail_items + p.num_ctas - 1) / p.num_ctas) : 0u;
     auto grab_tails = [&](uint32_t max_items) -> bool {
         if (!p.has_tail) return true;
         for (uint32_t n = 0; n < max_items; ++n) {
@@ -428,89 +575,19 @@ __device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr,
     const int cta = blockIdx.x;
     SegIter it;
     it.begin(p, p.cta_seg_begin[cta], p.cta_seg_begin[cta + 1]);
-    bool first_segment = true;
-    if (!it.done) {
-        const SegDev s0 = p.segs[it.sg];
-        const EntryDev e0 = p.entries[s0.entry];
-        ok = emit_pk(kPkSeg, e0.g, (e0.rk + 7) & ~7, it.pass, e0.off_pk);
+    pk_it = it;
+    for (int j = 0; ok && !it.done; ++j) {
+        ok = emit_segment(it, j);
+        it.advance(p);
     }
-    while (ok && !it.done) {
-        const SegDev seg = p.segs[it.sg];
-        const EntryDev ent = p.entries[seg.entry];
-        const int rk8 = (ent.rk + 7) & ~7, rv8 = (ent.rv + 7) & ~7;
-        int runfl = 0;
-        if (it.sg == it.r0) runfl |= F_RUN_FIRST;
-        if (it.sg == it.r1) runfl |= F_RUN_LAST;
-        SegIter nx = it;
-        nx.advance(p);
-        bool pk_next = nx.done;
-        const int per_tile = kTileTokens * (rk8 + rv8) * 2;
-        int tps = per_tile > 0 ? kSlotBytes / per_tile : 16;
-        tps = max(1, min(tps, 16));
-        const int n8 = (ent.n + 7) & ~7;
-        const int nsl = (seg.t1 - seg.t0 + tps * kTileTokens - 1) / (tps * kTileTokens);
-        const int pk_at = first_segment ? min(kSlots - 1, nsl - 1) : min(1, nsl - 1);
-        for (int si = 0; si < nsl && ok; ++si) {
-            const int tt0 = seg.t0 + si * tps * kTileTokens;
-            const int tt1 = min(seg.t1, tt0 + tps * kTileTokens);
-            const int tok8 = min((tt1 + 7) & ~7, n8) - tt0;
-            const int ntl = (tt1 - tt0 + kTileTokens - 1) / kTileTokens;
-            const int last8 = tok8 - (ntl - 1) * kTileTokens;
-            const int nsub = 2 * (ntl - 1) + (last8 + 15) / 16;
-            const int slot = ring_acquire();
-            if (slot < 0) { ok = false; break; }
-            int32_t *h = hdr + slot * kHdrInts;
-            h[H_KIND] = kC;
-            h[H_E] = seg.entry;
-            h[H_G] = ent.g;
-            h[H_T0] = tt0;
-            h[H_T1] = tt1;
-            h[H_RK8] = rk8;
-            h[H_RV8] = rv8;
-            h[H_TOK8] = tok8;
-            h[H_NSUB] = nsub;
-            h[H_FLAGS] = runfl | (si == 0 ? F_FIRST_C : 0) | (si == nsl - 1 ? F_LAST_C : 0);
-            h[H_REC] = seg.slot;
-            h[H_PASS] = it.pass;
-            const uint32_t kb = (uint32_t)tok8 * rk8 * 2, vb = (uint32_t)tok8 * rv8 * 2;
-            const uint32_t fb = bar(slot);
-            if (kb + vb) {
-                mbar_arrive_tx(fb, kb + vb);
-                const uint32_t dst = smem_u32(smem + slot * kSlotBytes);
-                if (kb) bulk_g2s(dst, p.packed + ent.off_ck + (int64_t)tt0 * rk8 * 2, kb, fb);
-                if (vb) bulk_g2s(dst + kb, p.packed + ent.off_cv + (int64_t)tt0 * rv8 * 2, vb, fb);
-            } else {
-                mbar_arrive(fb);
-            }
-            ++seq;
-            if (!pk_next && si == pk_at) {
-                // the next segment's basis, early, so its q~ is ready in time
-                const SegDev ns = p.segs[nx.sg];
-                const EntryDev ne = p.entries[ns.entry];
-                ok = emit_pk(kPkSeg, ne.g, (ne.rk + 7) & ~7, nx.pass, ne.off_pk);
-                pk_next = true;
-            }
-        }
-        if (!ok) break;
-        ok = emit_pv(rv8, ent.off_pv);
-        if (ok && first_segment) {
-            pdl_wait();
-            waited = true;
-            ok = grab_tails(tail_quota);
-        }
-        first_segment = false;
-        it = nx;
-    }
-    if (!waited) pdl_wait();
+    // tail items go after the prefix (any block that finishes early takes more);
+    // the tail counter and the tails belong to the preceding grid until here
+    pdl_wait();
     if (ok) ok = grab_tails(0xffffffffu);
-    if (ok) {
-        const int slot = ring_acquire();
-        if (slot >= 0) {
-            hdr[slot * kHdrInts + H_KIND] = kEnd;
-            mbar_arrive(bar(slot));
-            ++seq;
-        }
-        emit_pk(kPkEnd, 0, 0, 0, 0);
+    if (ok && open_fill()) {
+        if (pv_pending) put_pv();
+        flags |= kEndFill;
+        close_fill();
     }
     // the last thread block to finish grabbing resets the tail counter
     if (atomicAdd(&p.counters->ctas_done, 1u) == (uint32_t)p.num_ctas - 1) {
@@ -520,322 +597,81 @@ __device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr,
     // do not leave while a copy this thread started may still be landing
     for (int j = max(0, seq - kSlots); j < seq; ++j)
         if (!mbar_wait(bar(j % kSlots), (j / kSlots) & 1, p.status)) break;
-    if (npk > 0) mbar_wait(bar(B_PKF), (npk - 1) & 1, p.status);
-    for (int j = max(0, npv - 2); j < npv; ++j) mbar_wait(bar(B_PVF0 + (j & 1)), (j / 2) & 1, p.status);
-}
-
-// ================================================================ projection
-template <int D>
-__device__ bool run_projection(const DecodeParams &p, uint8_t *smem, const int32_t *pkh, uint64_t *bars, int lane)
-{
-    using L = Lay<D>;
-    constexpr int kMaxKs = D / 16;
-    auto bar = [&](int i) { return smem_u32(&bars[i]); };
-    const int quad = lane / 4, qlane = lane % 4;
-    const uint32_t pk = smem_u32(smem + L::kPk);
-    pdl_wait();
-    for (int k = 0;; ++k) {
-        if (!warp_wait(bar(B_PKF), k & 1, p.status)) return false;
-        const int kind = pkh[0];
-        if (kind == kPkEnd) return true;
-        const int g = pkh[1], rk8 = pkh[2], pass = pkh[3];
-        // the MMA warps load segment k-1's q~ when they start it, long before
-        // segment k's basis arrives: one buffer suffices
-        if (k >= 1 && !warp_wait(bar(B_QF), (k - 1) & 1, p.status)) return false;
-        for (int grp = 0; grp < p.nrg_cta; ++grp) {
-            const int rg = pass * p.nrg_cta + grp;
-            const int rho = 8 * rg + quad;
-            const uint16_t *qrow = nullptr;
-            if (rg < p.nrg && rho < p.rows_g) {
-                const int i = rho / p.G, hh = rho % p.G;
-                qrow = p.q + ((int64_t)i * p.hq + g * p.G + hh) * D;
-            }
-            uint32_t qlo[kMaxKs], qhi[kMaxKs];
-#pragma unroll
-            for (int kc = 0; kc < kMaxKs; ++kc) {
-                qlo[kc] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 2 * qlane) : 0u;
-                qhi[kc] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 8 + 2 * qlane) : 0u;
-            }
-            uint4 *qs = reinterpret_cast<uint4 *>(smem + L::kQs + grp * L::kQsPart);
-            const int njt = 2 * ((rk8 + 15) / 16);
-            for (int jt = 0; jt < njt; ++jt) {
-                float acc[4] = {0.f, 0.f, 0.f, 0.f};
-                if (jt < rk8 / 8) {
-#pragma unroll
-                    for (int kc = 0; kc < kMaxKs; kc += 2) {
-                        uint32_t b0, b1, b2, b3;
-                        // tiles (jt, 2kc), (jt, 2kc+1), (jt, 2kc+2), (jt, 2kc+3) of P^K
-                        const int cg = 2 * kc + (lane / 8);
-                        ldsm_x4(pk + (jt * (D / 8) + cg) * 128 + (lane % 8) * 16, b0, b1, b2, b3);
-                        const uint32_t a0[4] = {qlo[kc], 0u, qhi[kc], 0u};
-                        const uint32_t a1[4] = {qlo[kc + 1], 0u, qhi[kc + 1], 0u};
-                        mma16816(acc, a0, b0, b1);
-                        mma16816(acc, a1, b2, b3);
-                    }
-                }
-                uint32_t hi, lo;
-                split_hi_lo(acc[0] * p.scale_log2, acc[1] * p.scale_log2, hi, lo);
-                uint32_t *dst = reinterpret_cast<uint32_t *>(qs + (jt / 2) * 32 + lane);
-                dst[(jt & 1) * 2 + 0] = hi;
-                dst[(jt & 1) * 2 + 1] = lo;
-            }
-        }
-        __syncwarp();
-        if (lane == 0) {
-            mbar_arrive(bar(B_PKE));
-            mbar_arrive(bar(B_QR));
-        }
-    }
 }
 
 // ================================================================ MMA warps
+template <int N>
+using IC = std::integral_constant<int, N>;
+
 template <int D>
-__device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr, int32_t *dsc, uint64_t *bars,
-                        uint32_t zero_addr, int mw, int lane)
+__device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr, uint64_t *bars, int32_t *list,
+                        int32_t *tkt, uint32_t zero_addr, int mw, int lane)
 {
     using L = Lay<D>;
     constexpr int kMaxNt = D / 8;   // max rank (or column) 8-tiles
     constexpr int kMaxKs = D / 16;  // max 16-wide k-steps
+    // column tiles one warp back-projects (a row group has at least kMmaWarps / 2
+    // warps), rounded up to even: the back-projection takes them in pairs
+    constexpr int kMaxCt = ((kMaxNt + kMmaWarps / 2 - 1) / (kMmaWarps / 2) + 1) & ~1;
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
-    const int quad = lane / 4, qlane = lane % 4;
-    float2 *region = reinterpret_cast<float2 *>(smem + L::kMerge + mw * L::kMergeWarp);
+    const int quad = lane / 4, qlane = lane % 4, mi = lane / 8;
+    const int recf = 8 * D + kRecFloatsExtra;
+    // prefix row groups: warp mw serves group mw % ngrp as member wi of nwg
+    const int ngrp = p.nrg_cta, grp = mw % ngrp, wi = mw / ngrp;
+    const int nwg = (kMmaWarps - grp + ngrp - 1) / ngrp;
+    float2 *myregion = reinterpret_cast<float2 *>(smem + L::kMerge + mw * L::kMergeWarp);
+    auto region = [&](int w) { return reinterpret_cast<const float2 *>(smem + L::kMerge + w * L::kMergeWarp); };
+    auto qs_part = [&](int b) { return reinterpret_cast<uint32_t *>(smem + L::kQs + (2 * b + grp) * L::kFragPart); };
+    uint32_t *af = reinterpret_cast<uint32_t *>(smem + L::kAf + grp * L::kFragPart);
+    const bool qcached = (int64_t)p.batch * p.hq * D * 2 <= L::kQcBytes;
+    const uint16_t *qsrc = qcached ? reinterpret_cast<const uint16_t *>(smem + L::kQc) : p.q;
 
-    uint32_t qf[kMaxKs][4];
+    // A operand of the scores, read per tile: hi/lo fragments of q~ (a q~ buffer)
+    // or of scale * log2(e) * q for a tail item (this warp's dump area)
+    uint32_t a_frag = 0;
+    int cur_b = 0;      // q~ buffer of the current segment
     float vacc[kMaxNt][4];
     float m_w = -INFINITY, l_w = 0.f;
-    int nseg = 0, ndump = 0, sub_base = 0;
-    bool active = false;
+    float orun[kMaxCt][2];
+    float m_run = -INFINITY, l_run = 0.f;
+    bool act = false;   // this warp's row group exists in the current pass
+    int ngs = 0;        // group syncs passed
+    int tile_base = 0;  // round-robin position of prefix tiles
+    int tail_ctr = 0;   // tail row-group jobs seen
+    int nends = 0;      // segment ends so far (the same count in every MMA warp)
+    // the pending segment end: 0 none, 1 merge next, 2 back-projection next
+    int pend = 0, pe_e = 0, pe_seq = 0, pe_g = 0, pe_rg = 0, pe_rv8 = 0, pe_run = 0, pe_rec = 0;
+    uint32_t pe_pv = 0;
+    float pe_M = -INFINITY, pe_arun = 0.f, pe_Ls = 0.f;
+#pragma unroll
+    for (int c = 0; c < kMaxCt; ++c) orun[c][0] = orun[c][1] = 0.f;
 
-    pdl_wait();
-
+    auto gsync = [&]() -> bool {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(B_GS));
+        const bool ok = warp_wait(bar(B_GS), ngs & 1, p.status);
+        ++ngs;
+        return ok;
+    };
+    auto arrive = [&](int b) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(b));
+    };
+    auto test_bar = [&](int b, int parity) -> bool {
+        int ok = 0;
+        if (lane == 0) ok = mbar_test(bar(b), parity) ? 1 : 0;
+        return __shfl_sync(0xffffffffu, ok, 0) != 0;
+    };
     auto reset_state = [&]() {
         m_w = -INFINITY;
         l_w = 0.f;
 #pragma unroll
         for (int x = 0; x < kMaxNt; ++x) vacc[x][0] = vacc[x][1] = vacc[x][2] = vacc[x][3] = 0.f;
     };
-
-    // One 16-token sub-tile: scores, online softmax, rank-space values.
-    // Keys/values are read through `kaddr(mi, kk)` / `vaddr(mi, jp)`.
-    auto subtile = [&](int nks, int njp, float sc_mul, int tok_base, int t1, bool tgb_ok, auto kaddr, auto vaddr) {
-        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
-        const int mi = lane / 8;
-#pragma unroll
-        for (int kk = 0; kk < kMaxKs; ++kk) {
-            if (kk < nks) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4(kaddr(mi, kk), b0, b1, b2, b3);
-                mma16816(sa, qf[kk], b0, b1);
-                mma16816(sb, qf[kk], b2, b3);
-            }
-        }
-        const int tokA = tok_base + 2 * qlane;
-        float s0 = (sa[0] + sa[2]) * sc_mul, s1 = (sa[1] + sa[3]) * sc_mul;
-        float s2 = (sb[0] + sb[2]) * sc_mul, s3 = (sb[1] + sb[3]) * sc_mul;
-        if (tokA >= t1) s0 = -INFINITY;
-        if (tokA + 1 >= t1) s1 = -INFINITY;
-        if (!tgb_ok || tokA + 8 >= t1) s2 = -INFINITY;
-        if (!tgb_ok || tokA + 9 >= t1) s3 = -INFINITY;
-        const float mx = quad_max(fmaxf(fmaxf(s0, s1), fmaxf(s2, s3)));
-        if (mx > m_w + 8.f) {  // lazy rescale: p stays <= 2^8
-            const float alpha = exp2_diff(m_w, mx);
-            l_w *= alpha;
-#pragma unroll
-            for (int x = 0; x < kMaxNt; ++x) {
-                vacc[x][0] *= alpha; vacc[x][1] *= alpha; vacc[x][2] *= alpha; vacc[x][3] *= alpha;
-            }
-            m_w = mx;
-        }
-        const float p0 = exp2f(s0 - m_w), p1 = exp2f(s1 - m_w);
-        const float p2 = exp2f(s2 - m_w), p3 = exp2f(s3 - m_w);
-        l_w += (p0 + p1) + (p2 + p3);
-        uint32_t pa[4];
-        split_hi_lo(p0, p1, pa[0], pa[1]);
-        split_hi_lo(p2, p3, pa[2], pa[3]);
-#pragma unroll
-        for (int jp = 0; jp < kMaxKs; ++jp) {
-            if (jp < njp) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(vaddr(mi, jp), b0, b1, b2, b3);
-                mma16816(vacc[2 * jp], pa, b0, b1);
-                mma16816(vacc[2 * jp + 1], pa, b2, b3);
-            }
-        }
-    };
-
-    // Hand this warp's (max, sum, v~) to the epilogue warp.
-    auto dump = [&](int kind, const int32_t *h, int nvt) -> bool {
-        if (ndump >= 1 && !warp_wait(bar(B_ME), (ndump - 1) & 1, p.status)) return false;
-        const float lq = quad_sum(l_w);
-        if (active) {
-#pragma unroll
-            for (int x = 0; x < kMaxNt; ++x)
-                if (x < nvt) region[x * 32 + lane] = make_float2(vacc[x][0] + vacc[x][2], vacc[x][1] + vacc[x][3]);
-        }
-        region[kMaxNt * 32 + lane] = make_float2(active ? m_w : -INFINITY, active ? lq : 0.f);
-        if (mw == 0 && lane == 0) {
-            dsc[0] = kind;
-            if (h) {
-                dsc[1] = h[H_G];
-                dsc[2] = h[H_RV8];
-                dsc[3] = h[H_FLAGS];
-                dsc[4] = h[H_REC];
-                dsc[5] = h[H_PASS];
-                dsc[6] = h[H_ITEM];
-                dsc[7] = h[H_QI];
-            }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(B_MF));
-        ++ndump;
-        return true;
-    };
-
-    for (int seq = 0;; ++seq) {
-        const int slot = seq % kSlots;
-        if (!warp_wait(bar(slot), (seq / kSlots) & 1, p.status)) return false;
-        const int32_t *h = hdr + slot * kHdrInts;
-        const int kind = h[H_KIND];
-        const uint32_t sbase = smem_u32(smem + slot * kSlotBytes);
-        if (kind == kEnd) {
-            active = false;
-            if (!dump(kDumpEnd, nullptr, 0)) return false;
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kSlots + slot));
-            return true;
-        }
-        if (kind == kC) {
-            const int ngrp = p.nrg_cta, grp = mw % ngrp, phase = mw / ngrp, ts = kMmaWarps / ngrp;
-            const int rg = h[H_PASS] * ngrp + grp;
-            const int flags = h[H_FLAGS], rk8 = h[H_RK8], rv8 = h[H_RV8];
-            const int nks = (rk8 + 15) / 16, njp = (rv8 + 15) / 16;
-            if (flags & F_FIRST_C) {
-                if (!warp_wait(bar(B_QR), nseg & 1, p.status)) return false;
-                active = rg < p.nrg;
-                if (active) {
-                    const uint4 *qs = reinterpret_cast<const uint4 *>(smem + L::kQs + grp * L::kQsPart);
-#pragma unroll
-                    for (int kk = 0; kk < kMaxKs; ++kk)
-                        if (kk < nks) {
-                            const uint4 v = qs[kk * 32 + lane];
-                            qf[kk][0] = v.x; qf[kk][1] = v.y; qf[kk][2] = v.z; qf[kk][3] = v.w;
-                        }
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(bar(B_QF));
-                reset_state();
-                ++nseg;
-            }
-            if (active) {
-                const int t0 = h[H_T0], t1 = h[H_T1], tok8 = h[H_TOK8], nsub = h[H_NSUB];
-                const uint32_t kbase = sbase, vbase = sbase + tok8 * rk8 * 2;
-                const int ntl = (t1 - t0 + kTileTokens - 1) / kTileTokens;
-                for (int u = 0; u < nsub; ++u) {
-                    if ((sub_base + u) % ts != phase) continue;
-                    const int kt = u / 2, su = u % 2;
-                    const int t8 = (kt == ntl - 1) ? tok8 - kt * kTileTokens : kTileTokens;
-                    const int ntg = t8 / 8;
-                    const int tga = 2 * su, tgb = tga + 1;
-                    const uint32_t ktile = kbase + kt * kTileTokens * rk8 * 2;
-                    const uint32_t vtile = vbase + kt * kTileTokens * rv8 * 2;
-                    auto kaddr = [&](int mi, int kk) -> uint32_t {
-                        const int tg = (mi < 2) ? tga : tgb, rgk = 2 * kk + (mi & 1);
-                        return (tg < ntg && rgk < rk8 / 8) ? ktile + (rgk * ntg + tg) * 128 + (lane % 8) * 16
-                                                           : zero_addr;
-                    };
-                    auto vaddr = [&](int mi, int jp) -> uint32_t {
-                        const int tg = (mi & 1) ? tgb : tga, rgv = 2 * jp + (mi >> 1);
-                        return (tg < ntg && rgv < rv8 / 8) ? vtile + (rgv * ntg + tg) * 128 + (lane % 8) * 16
-                                                           : zero_addr;
-                    };
-                    subtile(nks, njp, 1.f, t0 + kt * kTileTokens + 8 * tga, t1, tgb < ntg, kaddr, vaddr);
-                }
-                sub_base += nsub;
-            }
-            if (flags & F_LAST_C)
-                if (!dump(kDumpSeg, h, rv8 / 8)) return false;
-        } else if (kind == kTail) {
-            const int ngrp = p.ngrp_t, grp = mw % ngrp, phase = mw / ngrp, ts = kMmaWarps / ngrp;
-            const int rgt = h[H_PASS] * ngrp + grp;
-            active = rgt < p.nrg_t;
-            reset_state();
-            if (active) {
-                const int i = h[H_QI], g = h[H_G], t0 = h[H_T0], t1 = h[H_T1];
-                const int rloc = 8 * rgt + quad;  // query head within the KV group
-                const uint16_t *qrow = (rloc < p.G) ? p.q + ((int64_t)i * p.hq + g * p.G + rloc) * D : nullptr;
-#pragma unroll
-                for (int kc = 0; kc < kMaxKs; ++kc) {
-                    qf[kc][0] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 2 * qlane) : 0u;
-                    qf[kc][1] = 0u;
-                    qf[kc][2] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 8 + 2 * qlane) : 0u;
-                    qf[kc][3] = 0u;
-                }
-                constexpr uint32_t half = kTailTokens * 128;
-                const uint32_t kb = sbase, vb = sbase + (D / 64) * half;
-                const int ntok = t1 - t0;
-                const int nsub = (ntok + 15) / 16;
-                for (int u = phase; u < nsub; u += ts) {
-                    const int tga = 2 * u, tgb = tga + 1;
-                    // 128B-swizzled boxes: row tr, 16-byte chunk ch at ((ch % 8) ^ (tr % 8))
-                    auto kaddr = [&](int mi, int kc) -> uint32_t {
-                        const int tr = 8 * ((mi < 2) ? tga : tgb) + (lane % 8), ch = 2 * kc + (mi & 1);
-                        return kb + (ch / 8) * half + tr * 128 + (((ch % 8) ^ (tr % 8)) * 16);
-                    };
-                    auto vaddr = [&](int mi, int cp) -> uint32_t {
-                        const int tr = 8 * ((mi & 1) ? tgb : tga) + (lane % 8), ch = 2 * cp + (mi >> 1);
-                        return vb + (ch / 8) * half + tr * 128 + (((ch % 8) ^ (tr % 8)) * 16);
-                    };
-                    subtile(kMaxKs, kMaxKs, p.scale_log2, 8 * tga, ntok, true, kaddr, vaddr);
-                }
-            }
-            if (!dump(kDumpTail, h, kMaxNt)) return false;
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(kSlots + slot));
-    }
-}
-
-// ================================================================ epilogue
-template <int D>
-__device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t *dsc, uint64_t *bars,
-                             int32_t *list, uint32_t zero_addr, int ep, int lane)
-{
-    using L = Lay<D>;
-    constexpr int kMaxNt = D / 8;
-    constexpr int kMaxKs = D / 16;
-    constexpr int kHalf = kMaxNt / 2;      // column tiles of this warp's half of the head dimension
-    const int ct0 = ep * kHalf;            // first column tile of this warp
-    int neps = 0;                          // record hand-offs between the two epilogue warps
-    auto bar = [&](int i) { return smem_u32(&bars[i]); };
-    const int quad = lane / 4, qlane = lane % 4;
-    const uint32_t pv_base = smem_u32(smem + L::kPv);
-    const int recf = 8 * D + kRecFloatsExtra;
-    auto region = [&](int w) { return reinterpret_cast<const float2 *>(smem + L::kMerge + w * L::kMergeWarp); };
-
-    float orun[2][kHalf][2];
-    float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-    int ndump = 0, npv = 0;
-#pragma unroll
-    for (int a = 0; a < 2; ++a)
-#pragma unroll
-        for (int x = 0; x < kHalf; ++x) orun[a][x][0] = orun[a][x][1] = 0.f;
-    // Both epilogue warps meet once their halves of a record are written (a
-    // two-warp barrier: neither can run a phase ahead of the other); the
-    // first one then counts the tickets.
-    auto await_partner = [&]() -> bool {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(B_EPS));
-        const bool ok = warp_wait(bar(B_EPS), neps & 1, p.status);
-        ++neps;
-        return ok;
-    };
-
-    pdl_wait();  // records and tickets belong to the preceding grid until here
-
-    // Count one record of (g, rg).  The thread block bringing the last one
-    // merges that row group: at the end of the kernel with every thread, or
-    // right away with this warp when the deferral list is full.
-    auto ticket = [&](int g, int rg) {
+    // Count one record of (g, rg) now (its writers' stores are already ordered
+    // before this point); the block that brings the last one merges the row group.
+    auto ticket_now = [&](int g, int rg) {
+        __threadfence();
         int last = 0;
         if (lane == 0) {
             const uint32_t old = atomicAdd(&p.tickets[g * p.nrg + rg], 1u);
@@ -845,187 +681,497 @@ __device__ bool run_epilogue(const DecodeParams &p, uint8_t *smem, const int32_t
                 __threadfence();
             }
         }
-        last = __shfl_sync(0xffffffffu, last, 0);
-        if (!last) return;
-        if (list[0] < L::kListCap) {
+        if (lane == 0 && last) {
+            const int pos = atomicAdd(&list[0], 1);
+            p.clist[2 * (blockIdx.x * p.clist_cap + pos)] = g;
+            p.clist[2 * (blockIdx.x * p.clist_cap + pos) + 1] = rg;
+        }
+        __syncwarp();
+    };
+    // A tail record is written by one warp: note it for the end of the block,
+    // or count it right away when the list is full.
+    auto note_tail = [&](int g, int rg) {
+        int pos = 0;
+        if (lane == 0) pos = atomicAdd(&tkt[0], 1);
+        pos = __shfl_sync(0xffffffffu, pos, 0);
+        if (pos < L::kTkCap) {
             if (lane == 0) {
-                const int n = list[0];
-                list[1 + 2 * n] = g;
-                list[2 + 2 * n] = rg;
-                list[0] = n + 1;
+                tkt[1 + 2 * pos] = g;
+                tkt[2 + 2 * pos] = rg;
             }
             __syncwarp();
         } else {
-            combine_rows<D>(p, g, rg, lane, 32);
+            ticket_now(g, rg);
+        }
+    };
+    // The tile code comes in four widths (1, 2, 4 and D/16 k-steps of 16 ranks;
+    // rank groups past a factor's rank read a zero line): close to the exact
+    // work for every rank, while the hot code stays small enough for the
+    // instruction cache (which a variant per rank overflows).
+    auto full_width = [&](int /*nk*/, auto body) { body(IC<kMaxKs>{}); };
+    auto by_width = [&](int nk, auto body) {
+        if (nk <= 1) body(IC<1>{});
+        else if (nk <= 2) body(IC<2>{});
+        else if (nk <= 4) body(IC<4>{});
+        else body(IC<kMaxKs>{});
+    };
+
+    // One 32-token tile (token groups 0-3) with NK 16-wide k-steps: scores,
+    // online softmax, rank-space values.  Keys/values are read through
+    // kaddr(h, m, kk) / vaddr(h, m, jp), h = half of the tile (token groups 2h, 2h+1).
+    auto tile32 = [&](auto nkc, float sc_mul, int tok_base, int t1, int ntg, auto kaddr, auto vaddr) {
+        constexpr int NK = decltype(nkc)::value;
+        float sc4[4][4];
+#pragma unroll
+        for (int n = 0; n < 4; ++n) sc4[n][0] = sc4[n][1] = sc4[n][2] = sc4[n][3] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < NK; ++kk) {
+            uint32_t qa[4];
+            asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                         : "=r"(qa[0]), "=r"(qa[1]), "=r"(qa[2]), "=r"(qa[3])
+                         : "r"(a_frag + (kk * 32 + lane) * 16));
+            uint32_t b0, b1, b2, b3, c0, c1, c2, c3;
+            ldsm_x4(kaddr(0, mi, kk), b0, b1, b2, b3);
+            ldsm_x4(kaddr(1, mi, kk), c0, c1, c2, c3);
+            mma16816(sc4[0], qa, b0, b1);
+            mma16816(sc4[1], qa, b2, b3);
+            mma16816(sc4[2], qa, c0, c1);
+            mma16816(sc4[3], qa, c2, c3);
+        }
+        // score of token tok_base + 8n + 2 qlane + j (rows: hi part + lo part)
+        float sv[8];
+#pragma unroll
+        for (int n = 0; n < 4; ++n) {
+            const int tok = tok_base + 8 * n + 2 * qlane;
+            sv[2 * n] = (n < ntg && tok < t1) ? (sc4[n][0] + sc4[n][2]) * sc_mul : -INFINITY;
+            sv[2 * n + 1] = (n < ntg && tok + 1 < t1) ? (sc4[n][1] + sc4[n][3]) * sc_mul : -INFINITY;
+        }
+        float mx = sv[0];
+#pragma unroll
+        for (int j = 1; j < 8; ++j) mx = fmaxf(mx, sv[j]);
+        mx = quad_max(mx);
+        if (mx > m_w + 8.f) {  // lazy rescale: p stays <= 2^8
+            const float alpha = exp2_diff(m_w, mx);
+            l_w *= alpha;
+#pragma unroll
+            for (int x = 0; x < 2 * NK; ++x) {
+                vacc[x][0] *= alpha; vacc[x][1] *= alpha; vacc[x][2] *= alpha; vacc[x][3] *= alpha;
+            }
+            m_w = mx;
+        }
+        float pv[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) pv[j] = exp2f(sv[j] - m_w);
+        l_w += ((pv[0] + pv[1]) + (pv[2] + pv[3])) + ((pv[4] + pv[5]) + (pv[6] + pv[7]));
+        uint32_t pa0[4], pa1[4];
+        split_hi_lo(pv[0], pv[1], pa0[0], pa0[1]);
+        split_hi_lo(pv[2], pv[3], pa0[2], pa0[3]);
+        split_hi_lo(pv[4], pv[5], pa1[0], pa1[1]);
+        split_hi_lo(pv[6], pv[7], pa1[2], pa1[3]);
+#pragma unroll
+        for (int jp = 0; jp < NK; ++jp) {
+            uint32_t b0, b1, b2, b3, c0, c1, c2, c3;
+            ldsm_x4_t(vaddr(0, mi, jp), b0, b1, b2, b3);
+            ldsm_x4_t(vaddr(1, mi, jp), c0, c1, c2, c3);
+            mma16816(vacc[2 * jp], pa0, b0, b1);
+            mma16816(vacc[2 * jp + 1], pa0, b2, b3);
+            mma16816(vacc[2 * jp], pa1, c0, c1);
+            mma16816(vacc[2 * jp + 1], pa1, c2, c3);
         }
     };
 
-    // Merge weights of the warps of one row group: sc[w] = 2^(m_w - M).
-    auto merge_scales = [&](int ngrp, int grp, float (&sc)[kMmaWarps], float &M, float &Lsum) {
-        M = -INFINITY;
+    // ---- segment end, deferred in three steps: dump (at the P^V part), merge
+    // slice (once every warp dumped), back-projection (once every warp merged).
+    // The fill carrying P^V stays held until this warp's back-projection.
+    auto do_merge = [&]() -> bool {
+        // the merged v~ buffer is free once every warp back-projected the previous end
+        if (pe_e >= 1 && !warp_wait(bar(B_BPDONE), (pe_e - 1) & 1, p.status)) return false;
+        const bool pact = pe_rg < p.nrg;
+        const int nvt = pe_rv8 / 8, nkj = (pe_rv8 + 15) / 16;
+        if (pe_run & F_RUN_FIRST) {
+            m_run = -INFINITY;
+            l_run = 0.f;
+#pragma unroll
+            for (int c = 0; c < kMaxCt; ++c) orun[c][0] = orun[c][1] = 0.f;
+        }
+        // merge weights relative to the run's new maximum (row = quad); another row
+        // group's dumps may hold anything: select, never multiply by zero
+        float2 ml[kMmaWarps];
+#pragma unroll
+        for (int w = 0; w < kMmaWarps; ++w) ml[w] = region(w)[kMaxNt * 32 + lane];
+        float M = m_run;
 #pragma unroll
         for (int w = 0; w < kMmaWarps; ++w)
-            if (w % ngrp == grp) M = fmaxf(M, region(w)[kMaxNt * 32 + lane].x);
-        Lsum = 0.f;
+            if ((w & (ngrp - 1)) == grp) M = fmaxf(M, ml[w].x);
+        float sc[kMmaWarps];
+        float Ls = 0.f;
 #pragma unroll
         for (int w = 0; w < kMmaWarps; ++w) {
-            sc[w] = 0.f;
-            if (w % ngrp == grp) {
-                const float2 ml = region(w)[kMaxNt * 32 + lane];
-                sc[w] = exp2_diff(ml.x, M);
-                Lsum += sc[w] * ml.y;
+            const bool mine = (w & (ngrp - 1)) == grp;
+            sc[w] = mine ? exp2_diff(ml[w].x, M) : 0.f;
+            Ls += mine ? sc[w] * ml[w].y : 0.f;
+        }
+        // this warp's slice of the merged v~ (tiles wi, wi + nwg, ...), as bf16 hi/lo A fragments
+#pragma unroll 1
+        for (int x = wi; x < 2 * nkj; x += nwg) {
+            {
+                float2 t[kMmaWarps];
+#pragma unroll
+                for (int w = 0; w < kMmaWarps; ++w) t[w] = region(w)[x * 32 + lane];
+                float2 v = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int w = 0; w < kMmaWarps; ++w) {
+                    const bool mine = (w & (ngrp - 1)) == grp;
+                    v.x = mine ? fmaf(sc[w], t[w].x, v.x) : v.x;
+                    v.y = mine ? fmaf(sc[w], t[w].y, v.y) : v.y;
+                }
+                if (!(pact && x < nvt)) v = make_float2(0.f, 0.f);
+                uint32_t hi, lo;
+                split_hi_lo(v.x, v.y, hi, lo);
+                af[((x / 2) * 32 + lane) * 4 + (x & 1) * 2 + 0] = hi;
+                af[((x / 2) * 32 + lane) * 4 + (x & 1) * 2 + 1] = lo;
             }
         }
+        pe_M = M;
+        pe_arun = exp2_diff(m_run, M);
+        pe_Ls = Ls;
+        arrive(B_MERGED);
+        pend = 2;
+        return true;
     };
-    auto merged_pair = [&](const float (&sc)[kMmaWarps], int x) -> float2 {
-        float2 v = make_float2(0.f, 0.f);
+    auto do_backproj = [&]() {
+        const bool pact = pe_rg < p.nrg;
+        const int nvt = pe_rv8 / 8;
+        if (pact) {
+            full_width((pe_rv8 + 15) / 16, [&](auto nkc) {
+                float o[kMaxCt][4];
 #pragma unroll
-        for (int w = 0; w < kMmaWarps; ++w)
-            if (sc[w] != 0.f) {
-                const float2 t = region(w)[x * 32 + lane];
-                v.x += sc[w] * t.x;
-                v.y += sc[w] * t.y;
-            }
-        return v;
-    };
-
-    for (;;) {
-        if (!warp_wait(bar(B_MF), ndump & 1, p.status)) return false;
-        const int kind = dsc[0];
-        if (kind == kDumpEnd) return true;
-        const int g = dsc[1], rv8 = dsc[2], flags = dsc[3], recslot = dsc[4], pass = dsc[5];
-        const int item = dsc[6], qi = dsc[7];
-        if (kind == kDumpSeg) {
-            const int pb = npv & 1;
-            if (!warp_wait(bar(B_PVF0 + pb), (npv / 2) & 1, p.status)) return false;
-            const uint32_t pv = pv_base + pb * L::kPBytes;
-            const int nkj = (rv8 + 15) / 16, nvt = rv8 / 8;
-            const int ngrp = p.nrg_cta;
-            // the dump regions are free once the last row group is merged
-            int last_grp = 0;
-            for (int x = 0; x < ngrp; ++x)
-                if (pass * ngrp + x < p.nrg) last_grp = x;
-            bool me_done = false;
+                for (int c = 0; c < kMaxCt; ++c) o[c][0] = o[c][1] = o[c][2] = o[c][3] = 0.f;
+#pragma unroll 1
+                for (int kj = 0; kj < (pe_rv8 + 15) / 16; ++kj) {
+                    const uint4 a4 = reinterpret_cast<const uint4 *>(af)[kj * 32 + lane];
+                    const uint32_t a[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
-            for (int grp = 0; grp < 2; ++grp) {
-                if (grp >= ngrp) break;
-                const int rg = pass * ngrp + grp;
-                if (rg >= p.nrg) continue;
-                float sc[kMmaWarps], M, Lsum;
-                merge_scales(ngrp, grp, sc, M, Lsum);
-                if (flags & F_RUN_FIRST) {
-                    m_run[grp] = -INFINITY;
-                    l_run[grp] = 0.f;
-#pragma unroll
-                    for (int x = 0; x < kHalf; ++x) orun[grp][x][0] = orun[grp][x][1] = 0.f;
-                }
-                const float m_new = fmaxf(m_run[grp], M);
-                const float a_run = exp2_diff(m_run[grp], m_new), a_seg = exp2_diff(M, m_new);
-#pragma unroll
-                for (int w = 0; w < kMmaWarps; ++w) sc[w] *= a_seg;
-                uint32_t af[kMaxKs][4];
-#pragma unroll
-                for (int kj = 0; kj < kMaxKs; ++kj) {
-                    if (kj < nkj) {
-                        const float2 x = (2 * kj < nvt) ? merged_pair(sc, 2 * kj) : make_float2(0.f, 0.f);
-                        const float2 y = (2 * kj + 1 < nvt) ? merged_pair(sc, 2 * kj + 1) : make_float2(0.f, 0.f);
-                        split_hi_lo(x.x, x.y, af[kj][0], af[kj][1]);
-                        split_hi_lo(y.x, y.y, af[kj][2], af[kj][3]);
-                    }
-                }
-                if (grp == last_grp) {
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(bar(B_ME));
-                    me_done = true;
-                }
-                // back-projection through P^V into this warp's half of the run's output
-                const int mi = lane / 8;
-#pragma unroll
-                for (int cp = 0; cp < kHalf / 2; ++cp) {
-                    float oa[4] = {0.f, 0.f, 0.f, 0.f}, ob[4] = {0.f, 0.f, 0.f, 0.f};
-                    // tiles (2kj, c), (2kj+1, c), (2kj, c+1), (2kj+1, c+1) of P^V, c = ct0 + 2cp
-                    const int ct = ct0 + 2 * cp + (mi >> 1);
-#pragma unroll
-                    for (int kj = 0; kj < kMaxKs; ++kj) {
-                        if (kj < nkj) {
+                    for (int cp = 0; cp < kMaxCt; cp += 2) {
+                        if (wi + cp * nwg < kMaxNt) {
+                            const int ct = wi + (cp + (mi >> 1)) * nwg;  // matrices 2,3: the pair's second tile
                             const int jg = 2 * kj + (mi & 1);
-                            const uint32_t addr =
-                                (jg < rv8 / 8) ? pv + (jg * (D / 8) + ct) * 128 + (lane % 8) * 16 : zero_addr;
+                            const uint32_t addr = (ct < kMaxNt && jg < nvt)
+                                                      ? pe_pv + (jg * (D / 8) + ct) * 128 + (lane % 8) * 16
+                                                      : zero_addr;
                             uint32_t b0, b1, b2, b3;
                             ldsm_x4_t(addr, b0, b1, b2, b3);
-                            mma16816(oa, af[kj], b0, b1);
-                            mma16816(ob, af[kj], b2, b3);
+                            mma16816(o[cp], a, b0, b1);
+                            mma16816(o[cp + 1], a, b2, b3);
                         }
                     }
-                    orun[grp][2 * cp][0] = orun[grp][2 * cp][0] * a_run + (oa[0] + oa[2]);
-                    orun[grp][2 * cp][1] = orun[grp][2 * cp][1] * a_run + (oa[1] + oa[3]);
-                    orun[grp][2 * cp + 1][0] = orun[grp][2 * cp + 1][0] * a_run + (ob[0] + ob[2]);
-                    orun[grp][2 * cp + 1][1] = orun[grp][2 * cp + 1][1] * a_run + (ob[1] + ob[3]);
                 }
-                l_run[grp] = l_run[grp] * a_run + Lsum * a_seg;
-                m_run[grp] = m_new;
-            }
-            __syncwarp();
-            if (lane == 0) {
-                if (!me_done) mbar_arrive(bar(B_ME));
-                mbar_arrive(bar(B_PVE0 + pb));
-            }
-            ++npv;
-            if (flags & F_RUN_LAST) {
 #pragma unroll
-                for (int grp = 0; grp < 2; ++grp) {
-                    if (grp >= ngrp) break;
-                    const int rg = pass * ngrp + grp;
-                    if (rg >= p.nrg) continue;
-                    float *rec = p.rec + ((int64_t)recslot * p.nrg + rg) * recf;
-#pragma unroll
-                    for (int x = 0; x < kHalf; ++x)
-                        __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * (ct0 + x) + 2 * qlane),
-                               make_float2(orun[grp][x][0], orun[grp][x][1]));
-                    if (ep == 0 && qlane == 0) {
-                        __stcg(rec + 8 * D + quad, m_run[grp]);
-                        __stcg(rec + 8 * D + 8 + quad, l_run[grp]);
-                    }
-                    __threadfence();
-                    if (!await_partner()) return false;
-                    if (ep == 0) ticket(g, rg);
+                for (int c = 0; c < kMaxCt; ++c) {
+                    orun[c][0] = orun[c][0] * pe_arun + (o[c][0] + o[c][2]);
+                    orun[c][1] = orun[c][1] * pe_arun + (o[c][1] + o[c][3]);
                 }
-            }
-        } else {  // tail item: the merged accumulator is already the output
-            const int ngrp = p.ngrp_t;
-            for (int grp = 0; grp < ngrp; ++grp) {
-                const int rgt = pass * ngrp + grp;
-                if (rgt >= p.nrg_t) continue;
-                float sc[kMmaWarps], M, Lsum;
-                merge_scales(ngrp, grp, sc, M, Lsum);
-                float *rec = p.rec + (p.tail_rec_base + (int64_t)item * p.nrg_t + rgt) * recf;
+            });
+            l_run = l_run * pe_arun + pe_Ls;
+            m_run = pe_M;
+            if (pe_run & F_RUN_LAST) {
+                float *rec = p.rec + ((int64_t)pe_rec * p.nrg + pe_rg) * recf;
 #pragma unroll
-                for (int x = 0; x < kHalf; ++x)
-                    __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * (ct0 + x) + 2 * qlane),
-                           merged_pair(sc, ct0 + x));
-                if (ep == 0 && qlane == 0) {
-                    __stcg(rec + 8 * D + quad, M);
-                    __stcg(rec + 8 * D + 8 + quad, Lsum);
+                for (int c = 0; c < kMaxCt; ++c)
+                    if (wi + c * nwg < kMaxNt)
+                        __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * (wi + c * nwg) + 2 * qlane),
+                               make_float2(orun[c][0], orun[c][1]));
+                if (wi == 0 && qlane == 0) {
+                    __stcg(rec + 8 * D + quad, m_run);
+                    __stcg(rec + 8 * D + 8 + quad, l_run);
                 }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(B_ME));
-            __threadfence();
-            if (!await_partner()) return false;
-            if (ep == 1) {
-                ++ndump;
-                continue;
-            }
-            // tickets of the prefix row groups these query rows belong to
-            for (int grp = 0; grp < ngrp; ++grp) {
-                const int rgt = pass * ngrp + grp;
-                if (rgt >= p.nrg_t) continue;
-                const int ra = qi * p.G + 8 * rgt, rb = qi * p.G + min(8 * rgt + 8, p.G);  // [ra, rb)
-                for (int rg = ra / 8; rg <= (rb - 1) / 8; ++rg) ticket(g, rg);
             }
         }
-        ++ndump;
+        arrive(kSlots + pe_seq % kSlots);  // the fill that carried P^V
+        arrive(B_BPDONE);
+        pend = 0;
+    };
+    // Advance the pending segment end as far as the other warps allow
+    // (force: wait for them).
+    auto poll = [&](bool force) -> bool {
+        if (pend == 1) {
+            if (force) {
+                if (!warp_wait(bar(B_DUMPED), pe_e & 1, p.status)) return false;
+            } else if (!test_bar(B_DUMPED, pe_e & 1)) {
+                return true;
+            }
+            if (!do_merge()) return false;
+        }
+        if (pend == 2) {
+            if (force) {
+                if (!warp_wait(bar(B_MERGED), pe_e & 1, p.status)) return false;
+            } else if (!test_bar(B_MERGED, pe_e & 1)) {
+                return true;
+            }
+            do_backproj();
+        }
+        return true;
+    };
+    auto segment_end = [&](const int32_t *h, uint32_t sbase, int seq) -> bool {
+        // the previous end is complete for this warp, and every merge of it has
+        // read the dumps: the dump area is free
+        if (!poll(true)) return false;
+        const int nvt = h[H_PV_RV8] / 8;
+        const float lq = quad_sum(l_w);
+        if (act) {
+#pragma unroll
+            for (int x = 0; x < kMaxNt; ++x)
+                if (x < nvt) myregion[x * 32 + lane] = make_float2(vacc[x][0] + vacc[x][2], vacc[x][1] + vacc[x][3]);
+        }
+        myregion[kMaxNt * 32 + lane] = make_float2(act ? m_w : -INFINITY, act ? lq : 0.f);
+        reset_state();
+        arrive(B_QFREE + cur_b);  // the segment's q~ buffer is no longer read by this warp
+        arrive(B_DUMPED);
+        pend = 1;
+        pe_e = nends++;
+        pe_seq = seq;
+        pe_pv = sbase + h[H_PV_OFF];
+        pe_g = h[H_PV_G];
+        pe_rg = h[H_PV_PASS] * ngrp + grp;
+        pe_rv8 = h[H_PV_RV8];
+        pe_run = h[H_PV_RUN];
+        pe_rec = h[H_PV_REC];
+        return true;
+    };
+
+    // ---- P^K part: this warp's slice of q~ for a coming segment
+    auto project = [&](const int32_t *f, uint32_t sbase) -> bool {
+        const int j = f[0], g = f[1], rk8 = f[2];
+        const int rg = f[3] * ngrp + grp;
+        const uint32_t pk = sbase + f[4];
+        const int b = j & 1, u = j >> 1;
+        // the buffer is free once every warp has ended segment j - 2
+        if (u >= 1 && !warp_wait(bar(B_QFREE + b), (u - 1) & 1, p.status)) return false;
+        if (rg < p.nrg) {
+            uint32_t *qs = qs_part(b);
+            const int rho = 8 * rg + quad;
+            const uint16_t *qrow = nullptr;
+            if (rho < p.rows_g) qrow = qsrc + ((int64_t)(rho / p.G) * p.hq + g * p.G + rho % p.G) * D;
+            uint32_t qa[kMaxKs], qb[kMaxKs];
+#pragma unroll
+            for (int kc = 0; kc < kMaxKs; ++kc) {
+                qa[kc] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 2 * qlane) : 0u;
+                qb[kc] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + 16 * kc + 8 + 2 * qlane) : 0u;
+            }
+            const int njt = 2 * ((rk8 + 15) / 16);
+            // rank tiles wi, wi + nwg, ... with two accumulators each (even / odd k-steps);
+            // a rolled loop: this code runs a few times per launch, mostly from a cold
+            // instruction cache, so its size matters more than its ILP
+#pragma unroll 1
+            for (int jt = wi; jt < njt; jt += nwg) {
+                {
+                    float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
+                    if (jt < rk8 / 8) {
+#pragma unroll
+                        for (int kc = 0; kc < kMaxKs; kc += 2) {
+                            // cores (jt, 2kc .. 2kc+3) of P^K: k-steps kc and kc+1
+                            uint32_t b0, b1, b2, b3;
+                            ldsm_x4(pk + (jt * (D / 8) + 2 * kc + mi) * 128 + (lane % 8) * 16, b0, b1, b2, b3);
+                            const uint32_t a0[4] = {qa[kc], 0u, qb[kc], 0u};
+                            const uint32_t a1[4] = {qa[kc + 1], 0u, qb[kc + 1], 0u};
+                            mma16816(acc0, a0, b0, b1);
+                            mma16816(acc1, a1, b2, b3);
+                        }
+                    }
+                    uint32_t hi, lo;
+                    split_hi_lo((acc0[0] + acc1[0]) * p.scale_log2, (acc0[1] + acc1[1]) * p.scale_log2, hi, lo);
+                    qs[((jt / 2) * 32 + lane) * 4 + (jt & 1) * 2 + 0] = hi;
+                    qs[((jt / 2) * 32 + lane) * 4 + (jt & 1) * 2 + 1] = lo;
+                }
+            }
+        }
+        arrive(B_QREADY + b);
+        return true;
+    };
+
+    // ---- start of a segment (one row-group pass of it): its q~ is in buffer j & 1
+    auto segment_start = [&](const int32_t *h) -> bool {
+        const int j = h[H_SS_J];
+        const int b = j & 1, u = j >> 1;
+        if (!warp_wait(bar(B_QREADY + b), u & 1, p.status)) return false;
+        act = h[H_SS_PASS] * ngrp + grp < p.nrg;
+        cur_b = b;
+        reset_state();
+        return true;
+    };
+
+    // Tile addressing shared by coefficient tiles and tail items (one copy of the
+    // tile code): cores [rank group][token group] of 128 bytes from t_k / t_v,
+    // t_stride token groups per rank group, t_ntg of them valid.
+    uint32_t t_k = 0, t_v = 0;
+    int t_stride = 4, t_ntg = 4, t_nrk = 0, t_nrv = 0;
+    auto kaddr = [&](int hf, int m4, int kk) -> uint32_t {
+        const int tg = 2 * hf + (m4 >> 1), rgk = 2 * kk + (m4 & 1);
+        return (tg < t_ntg && rgk < t_nrk) ? t_k + (rgk * t_stride + tg) * 128 + (lane % 8) * 16 : zero_addr;
+    };
+    auto vaddr = [&](int hf, int m4, int jp) -> uint32_t {
+        const int tg = 2 * hf + (m4 & 1), rgv = 2 * jp + (m4 >> 1);
+        return (tg < t_ntg && rgv < t_nrv) ? t_v + (rgv * t_stride + tg) * 128 + (lane % 8) * 16 : zero_addr;
+    };
+    auto run_tile = [&](float sc_mul, int tok_base, int t1) {
+        by_width(max((t_nrk + 1) / 2, (t_nrv + 1) / 2),
+                 [&](auto nkc) { tile32(nkc, sc_mul, tok_base, t1, t_ntg, kaddr, vaddr); });
+    };
+
+    // ---- tiles of one fill: the coefficient tiles this warp takes, or the whole
+    // tail item when this warp owns one of its row groups.  One call site of the
+    // tile code for both.
+    auto fill_tiles = [&](const int32_t *h, uint32_t sbase, int flags) -> bool {
+        int njobs = 0, kt0 = 0, ntl = 0, last8 = 0, t0 = 0, t1 = 0, rk8 = 0, rv8 = 0, rgt = -1;
+        uint32_t kbase = 0, vbase = 0;
+        float sc_mul = 1.f;
+        if (flags & kHasC) {
+            t0 = h[H_T0];
+            t1 = h[H_T1];
+            const int tok8 = h[H_TOK8];
+            rk8 = h[H_RK8];
+            rv8 = h[H_RV8];
+            ntl = (t1 - t0 + kTileTokens - 1) / kTileTokens;
+            if (act) {
+                last8 = tok8 - (ntl - 1) * kTileTokens;
+                kbase = sbase + h[H_C_OFF];
+                vbase = kbase + tok8 * rk8 * 2;
+                kt0 = (wi - tile_base % nwg + nwg) % nwg;  // this warp's first tile in the fill
+                a_frag = smem_u32(qs_part(cur_b));
+                njobs = kt0 < ntl ? (ntl - kt0 + nwg - 1) / nwg : 0;
+                t_nrk = rk8 / 8;
+                t_nrv = rv8 / 8;
+            }
+            tile_base += ntl;
+        } else if (flags & kTailFill) {
+            for (int r = 0; r < p.nrg_t; ++r)
+                if ((tail_ctr + r) % kMmaWarps == mw) rgt = r;
+            tail_ctr += p.nrg_t;
+            if (rgt >= 0) {
+                const int i = h[H_QI], g = h[H_G];
+                t1 = h[H_T1] - h[H_T0];  // tokens of the item
+                reset_state();
+                // tails come after the prefix: once the last segment end is through, no
+                // warp reads this warp's dump area again; stage the item's A fragments there
+                if (!poll(true)) return false;
+                const int rloc = 8 * rgt + quad;  // query head within the KV group
+                const uint16_t *qrow = (rloc < p.G) ? qsrc + ((int64_t)i * p.hq + g * p.G + rloc) * D : nullptr;
+                uint32_t *fr = reinterpret_cast<uint32_t *>(myregion);
+#pragma unroll 1
+                for (int kk = 0; kk < kMaxKs; ++kk) {
+                    float2 x0 = make_float2(0.f, 0.f), x1 = make_float2(0.f, 0.f);
+                    if (qrow) {
+                        x0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(qrow + 16 * kk + 2 * qlane));
+                        x1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(qrow + 16 * kk + 8 + 2 * qlane));
+                    }
+                    uint32_t h0, l0, h1, l1;
+                    split_hi_lo(x0.x * p.scale_log2, x0.y * p.scale_log2, h0, l0);
+                    split_hi_lo(x1.x * p.scale_log2, x1.y * p.scale_log2, h1, l1);
+                    *reinterpret_cast<uint4 *>(fr + (kk * 32 + lane) * 4) = make_uint4(h0, l0, h1, l1);
+                }
+                __syncwarp();
+                a_frag = smem_u32(myregion);
+                // the item arrives as one coefficient-style tile of kTailTokens tokens and rank d
+                kbase = sbase;
+                vbase = sbase + (D / 8) * kTailTokens * 16;
+                njobs = (t1 + kTileTokens - 1) / kTileTokens;
+                t_nrk = t_nrv = kMaxNt;
+            }
+        }
+        for (int jb = 0; jb < njobs; ++jb) {
+            int tok_base;
+            if (rgt < 0) {
+                const int kt = kt0 + jb * nwg;
+                t_ntg = ((kt == ntl - 1) ? last8 : kTileTokens) / 8;
+                t_stride = t_ntg;
+                t_k = kbase + kt * kTileTokens * rk8 * 2;
+                t_v = vbase + kt * kTileTokens * rv8 * 2;
+                tok_base = t0 + kt * kTileTokens;
+            } else {
+                t_ntg = 4;
+                t_stride = kTailTokens / 8;
+                t_k = kbase + 4 * jb * 128;
+                t_v = vbase + 4 * jb * 128;
+                tok_base = kTileTokens * jb;
+            }
+            run_tile(sc_mul, tok_base, t1);
+        }
+        if (rgt >= 0) {
+            const int i = h[H_QI], g = h[H_G], item = h[H_ITEM];
+            float *rec = p.rec + (p.tail_rec_base + (int64_t)item * p.nrg_t + rgt) * recf;
+#pragma unroll
+            for (int x = 0; x < kMaxNt; ++x)
+                __stcg(reinterpret_cast<float2 *>(rec + quad * D + 8 * x + 2 * qlane),
+                       make_float2(vacc[x][0] + vacc[x][2], vacc[x][1] + vacc[x][3]));
+            const float lq = quad_sum(l_w);
+            if (qlane == 0) {
+                __stcg(rec + 8 * D + quad, m_w);
+                __stcg(rec + 8 * D + 8 + quad, lq);
+            }
+            // the prefix row groups these query rows belong to
+            const int ra = i * p.G + 8 * rgt, rb = i * p.G + min(8 * rgt + 8, p.G);  // [ra, rb)
+            for (int rg = ra / 8; rg <= (rb - 1) / 8; ++rg) note_tail(g, rg);
+        }
+        return true;
+    };
+
+    pdl_wait();  // q, records and tickets belong to the preceding grid until here
+    if (qcached) {  // q is 4-byte aligned (checked on the host)
+        const int n4 = (int)((int64_t)p.batch * p.hq * D * 2 / 4);
+        const uint32_t *src = reinterpret_cast<const uint32_t *>(p.q);
+        uint32_t *dst = reinterpret_cast<uint32_t *>(smem + L::kQc);
+        for (int k = mw * 32 + lane; k < n4; k += kMmaWarps * 32) dst[k] = src[k];
+        if (!gsync()) return false;
     }
+    for (int seq = 0;; ++seq) {
+        const int slot = seq % kSlots;
+        // the ring is about to come back to the fill still held for a back-projection
+        if (pend != 0 && pe_seq % kSlots == slot && !poll(true)) return false;
+        if (!warp_wait(bar(slot), (seq / kSlots) & 1, p.status)) return false;
+        const int32_t *h = hdr + slot * kHdrInts;
+        const int flags = h[H_FLAGS];
+        const uint32_t sbase = smem_u32(smem + L::kRing + slot * kSlotBytes);
+        if ((flags & kHasPv) && !segment_end(h, sbase, seq)) return false;
+        if ((flags & kHasPk0) && !project(h + H_PK_J, sbase)) return false;
+        if ((flags & kHasPk1) && !project(h + H_PK1_J, sbase)) return false;
+        if ((flags & kSegStart) && !segment_start(h)) return false;
+        if ((flags & (kHasC | kTailFill)) && !fill_tiles(h, sbase, flags)) return false;
+        if (!(flags & kHasPv)) arrive(kSlots + slot);  // a fill with P^V is released by its back-projection
+        if (flags & kEndFill) {
+            if (!poll(true)) return false;
+            break;
+        }
+        if (!poll(false)) return false;
+    }
+    // every record of this block is written: count them (one fence for all).  The
+    // prefix records follow from the static partition: one per run and row group.
+    if (!gsync()) return false;
+    if (mw == 0) {
+        __threadfence();
+        const int s0 = p.cta_seg_begin[blockIdx.x], s1 = p.cta_seg_begin[blockIdx.x + 1];
+        const int np = (s1 - s0) * p.nrg, nt = min(tkt[0], L::kTkCap);
+        for (int k = lane; k < np + nt; k += 32) {
+            int g, rg;
+            if (k < np) {
+                const SegDev sg = p.segs[s0 + k / p.nrg];
+                if (!(sg.flags & kSegLastOfRun)) continue;
+                g = p.entries[sg.entry].g;
+                rg = k % p.nrg;
+            } else {
+                g = tkt[1 + 2 * (k - np)];
+                rg = tkt[2 + 2 * (k - np)];
+            }
+            const uint32_t old = atomicAdd(&p.tickets[g * p.nrg + rg], 1u);
+            if (old == (uint32_t)expected_arrivals(p, g, rg) - 1) {
+                p.tickets[g * p.nrg + rg] = 0u;
+                const int pos = atomicAdd(&list[0], 1);  // at most clist_cap: one per (g, rg)
+                p.clist[2 * (blockIdx.x * p.clist_cap + pos)] = g;
+                p.clist[2 * (blockIdx.x * p.clist_cap + pos) + 1] = rg;
+            }
+        }
+        __threadfence();
+    }
+    return true;
 }
 
 // ================================================================ kernel
@@ -1035,13 +1181,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                   const __grid_constant__ CUtensorMap tmap_v)
 {
     using L = Lay<D>;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     int32_t *hdr = reinterpret_cast<int32_t *>(smem + L::kHdr);
-    int32_t *pkh = hdr + kSlots * kHdrInts;
-    int32_t *dsc = hdr + (kSlots + 1) * kHdrInts;
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L::kBar);
     int32_t *list = reinterpret_cast<int32_t *>(smem + L::kList);
+    int32_t *tkt = reinterpret_cast<int32_t *>(smem + L::kTkT);
     const uint32_t zero_addr = smem_u32(smem + L::kZero);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
@@ -1051,43 +1196,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(smem_u32(&bars[s]), 1);                    // full: producer + bytes
             mbar_init(smem_u32(&bars[kSlots + s]), kMmaWarps);   // empty: every MMA warp
         }
-        mbar_init(smem_u32(&bars[B_PKF]), 1);
-        mbar_init(smem_u32(&bars[B_PKE]), 1);
-        mbar_init(smem_u32(&bars[B_PVF0]), 1);
-        mbar_init(smem_u32(&bars[B_PVF1]), 1);
-        mbar_init(smem_u32(&bars[B_PVE0]), 2);  // both epilogue warps
-        mbar_init(smem_u32(&bars[B_PVE1]), 2);
-        mbar_init(smem_u32(&bars[B_QR]), 1);
-        mbar_init(smem_u32(&bars[B_QF]), kMmaWarps);
-        mbar_init(smem_u32(&bars[B_MF]), kMmaWarps);
-        mbar_init(smem_u32(&bars[B_ME]), 2);   // both epilogue warps
-        mbar_init(smem_u32(&bars[B_EPS]), 2);
-        mbar_init(smem_u32(&bars[B_FIN]), 3 + kMmaWarps);
+        mbar_init(smem_u32(&bars[B_GS]), kMmaWarps);
+        mbar_init(smem_u32(&bars[B_FIN]), kMmaWarps + 1);
+        for (int b = B_QREADY; b < B_COUNT; ++b) mbar_init(smem_u32(&bars[b]), kMmaWarps);
         list[0] = 0;
+        tkt[0] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (threadIdx.x < 32) reinterpret_cast<uint32_t *>(smem + L::kZero)[threadIdx.x] = 0u;
+    // dumps, q~ and merged v~ fragments: padding entries are read (times zero) before
+    // they are first written, so they start as zeros
+    for (int k = threadIdx.x; k < (L::kHdr - L::kMerge) / 4; k += kThreads)
+        reinterpret_cast<uint32_t *>(smem + L::kMerge)[k] = 0u;
     __syncthreads();
 
+    bool ok = true;
     if (warp == 0) {
-        if (lane == 0) run_producer<D>(p, smem, hdr, pkh, bars, &tmap_k, &tmap_v);
-        return;
+        if (lane == 0) run_producer<D>(p, smem, hdr, bars, &tmap_k, &tmap_v);
+        __syncwarp();
+    } else {
+        ok = run_mma<D>(p, smem, hdr, bars, list, tkt, zero_addr, warp - 1, lane);
     }
-    bool ok;
-    if (warp == 1)
-        ok = run_projection<D>(p, smem, pkh, bars, lane);
-    else if (warp <= 3)
-        ok = run_epilogue<D>(p, smem, dsc, bars, list, zero_addr, warp - 2, lane);
-    else
-        ok = run_mma<D>(p, smem, hdr, dsc, bars, zero_addr, warp - 4, lane);
-    if (!ok) return;
-    // every role done: merge the row groups this thread block completed
+    if (!__all_sync(0xffffffffu, ok)) return;
+    // all warps: merge the row groups whose last record this block brought
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(&bars[B_FIN]));
     if (!warp_wait(smem_u32(&bars[B_FIN]), 0, p.status)) return;
-    const int n = min(list[0], L::kListCap);
-    for (int k = 0; k < n; ++k)
-        combine_rows<D>(p, list[1 + 2 * k], list[2 + 2 * k], threadIdx.x - 32, kThreads - 32);
+    const int n = list[0];
+    const int32_t *cl = p.clist + 2 * blockIdx.x * p.clist_cap;
+    for (int k = 0; k < n; ++k) combine_rows<D>(p, cl[2 * k], cl[2 * k + 1], threadIdx.x, kThreads);
 }
 
 }  // namespace

@@ -425,6 +425,8 @@ namespace {
 struct CallShape {
     int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
     int64_t records;
+    int64_t rec_bytes;    // partial records, at the start of the workspace
+    int64_t clist_bytes;  // per-block lists of row groups to merge, after the records
 };
 
 CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
@@ -439,6 +441,9 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
     c.records = (int64_t)p->num_slots * c.nrg + (int64_t)batch * p->hkv * c.S * c.nrg_t;
+    c.rec_bytes = (std::max<int64_t>(c.records, 1) * (8 * p->d + kRecFloatsExtra) * (int64_t)sizeof(float) + 255) / 256 * 256;
+    // a block may have to merge every (KV head, row group)
+    c.clist_bytes = (int64_t)p->num_ctas * p->hkv * c.nrg * 2 * (int64_t)sizeof(int32_t);
     return c;
 }
 }  // namespace
@@ -449,7 +454,7 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch, int6
     if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
     if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
-    *bytes = (size_t)std::max<int64_t>(c.records, 1) * (8 * plan->d + kRecFloatsExtra) * sizeof(float);
+    *bytes = (size_t)(c.rec_bytes + c.clist_bytes);
     return MILO_OK;
 }
 
@@ -490,6 +495,8 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.tail_offsets = tail_offsets;
     prm.out = out;
     prm.rec = static_cast<float *>(workspace);
+    prm.clist = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) + c.rec_bytes);
+    prm.clist_cap = plan->hkv * c.nrg;
     prm.counters = plan->counters;
     prm.tickets = plan->tickets;
     prm.status = plan->status;
@@ -522,13 +529,15 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
         if (!enc) return fail(MILO_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
         const cuuint64_t dims[3] = {(cuuint64_t)plan->d, (cuuint64_t)plan->hkv, (cuuint64_t)tail_rows};
         const cuuint64_t strides[2] = {(cuuint64_t)plan->d * 2, (cuuint64_t)plan->hkv * plan->d * 2};
-        const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTailTokens};
+        // boxes of one 16-byte column chunk: a tail item lands in shared memory as
+        // 8x8 cores [column group][token group], like a packed coefficient tile
+        const cuuint32_t box[3] = {8, 1, (cuuint32_t)kTailTokens};
         const cuuint32_t estr[3] = {1, 1, 1};
         CUresult r1 = enc(&mk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(tail_k), dims, strides, box,
-                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         CUresult r2 = enc(&mv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(tail_v), dims, strides, box,
-                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS) return fail(MILO_ERR_CUDA, "tensor map encoding failed");
     }

@@ -8,12 +8,13 @@
 namespace milo {
 
 constexpr int kTileTokens = 32;      // tokens per packed coefficient tile
-constexpr int kMmaWarps = 8;         // score/value warps per decode thread block
-constexpr int kThreads = 32 * (4 + kMmaWarps);  // + producer, projection, 2 epilogue
-constexpr int kSlots = 5;            // coefficient ring depth
-constexpr int kSlotBytes = 16384;    // bytes per ring slot
-constexpr int kHdrInts = 16;         // slot header (ints)
-constexpr int kTailTokens = 32;      // tokens per dense-tail work item
+constexpr int kMmaWarps = 7;         // compute warps per decode thread block (8 warps in all:
+                                     // at most two per SM sub-partition, 255 registers each)
+constexpr int kThreads = 32 * (1 + kMmaWarps);  // + one producer warp
+constexpr int kSlots = 5;            // ring depth (fills in flight)
+constexpr int kSlotBytes = 32768;    // bytes per ring slot (one fill)
+constexpr int kHdrInts = 32;         // fill header (ints)
+constexpr int kTailTokens = 64;      // tokens per dense-tail work item
 constexpr int kRecFloatsExtra = 16;  // m[8], l[8] after o[8][d] in a record
 
 // Per-(block, KV head) entry of the packed arena.
@@ -52,6 +53,8 @@ struct DecodeParams {
     const int64_t *tail_offsets;    // [batch + 1] or null
     float *out;                     // [batch, Hq, d]
     float *rec;                     // workspace records
+    int32_t *clist;                 // workspace: per-block (g, rg) pairs to merge
+    int clist_cap;                  // pairs per block (Hkv * nrg)
     CountersDev *counters;
     uint32_t *tickets;              // [Hkv * nrg]
     int32_t *status;
