@@ -387,7 +387,8 @@ def main():
                    "tokens_per_step": tokens, "algorithmic_bytes_per_step": alg_bytes,
                    "l2": "inputs larger than L2 (step reads %.2f GB > 129 MB); no flush" % (alg_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "launch": "one CUDA graph of %d per-layer calls (programmatic dependent launch)" % cfg.layers},
+                   "launch": "one CUDA graph of %d per-layer calls, each a decode and a merge kernel "
+                             "(programmatic dependent launch)" % cfg.layers},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": f"{peak_kind} copy bandwidth",
@@ -397,7 +398,7 @@ def main():
         "cpu_baseline": cpu,
         "e2e": {"value": world * tokens / (e_ms * 1e-3), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms},
-        "gpu_launches": cfg.layers * args.steps,
+        "gpu_launches": 2 * cfg.layers * args.steps,  # decode + merge kernel per layer
         "clocks": clocks.summary(),
         "parity_check": check,
         "setup_s": t_gen,

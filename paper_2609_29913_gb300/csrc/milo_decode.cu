@@ -66,7 +66,6 @@ static_assert(H_WORDS <= kHdrInts, "fill header size");
 // barrier indices: full[kSlots], empty[kSlots], then the MMA warps' own
 enum : int {
     B_GS = 2 * kSlots,  // group sync of the MMA warps
-    B_FIN,              // final meeting of all warps
     B_QREADY,           // [2] q~ buffer written by every MMA warp
     B_QFREE = B_QREADY + 2,  // [2] q~ buffer loaded by every MMA warp
     B_DUMPED = B_QFREE + 2,  // every MMA warp dumped its state of a segment
@@ -241,10 +240,7 @@ struct Lay {
     static constexpr int kQcBytes = 8192;
     static constexpr int kBar = kQc + kQcBytes;
     static constexpr int kZero = al(kBar + B_COUNT * 8, 128);
-    static constexpr int kList = kZero + 128;                     // count of row groups to merge (list in the workspace)
-    static constexpr int kTkCap = 255;                            // tail records to count at the end
-    static constexpr int kTkT = kList + 128;                      //   count, (g, rg) pairs
-    static constexpr int kTotal = kTkT + 8 * (kTkCap + 1);
+    static constexpr int kTotal = kZero + 128;
     static_assert(kSlotBytes % 1024 == 0, "ring slots must keep 1024-byte alignment (128B-swizzled TMA boxes)");
     static_assert(kMerge % 128 == 0 && kQs % 128 == 0 && kAf % 128 == 0 && kHdr % 128 == 0, "alignment");
     static_assert(kQc % 128 == 0 && kBar % 128 == 0, "alignment");
@@ -252,85 +248,6 @@ struct Lay {
     static_assert(D * D * 2 <= kSlotBytes, "a full-rank basis must fit one fill");
     static_assert(kTotal + 1024 <= 232448, "shared memory budget");
 };
-
-// ------------------------------------------------------- combine ----------
-// Merge every partial record of (KV head g, row group rg) and write out.
-template <int D>
-__device__ void combine_rows(const DecodeParams &p, int g, int rg, int tid, int nthr)
-{
-    constexpr int kChunk = 8;  // records whose loads are in flight together
-    const int recf = 8 * D + kRecFloatsExtra;
-    const int gs0 = p.g_slot_begin[g], gs1 = p.g_slot_begin[g + 1];
-    const int nprefix = gs1 - gs0;
-    const int S = p.tail_splits;
-    const int nsrc = nprefix + S;
-    for (int w = tid; w < 8 * (D / 4); w += nthr) {
-        const int k = w / (D / 4), c4 = w % (D / 4);
-        const int rho = 8 * rg + k;
-        if (rho >= p.rows_g) continue;
-        const int i = rho / p.G, hh = rho % p.G;
-        const float *tail0 = p.rec + (p.tail_rec_base + (int64_t)(i * p.hkv + g) * S * p.nrg_t + hh / 8) * recf;
-        float M = -INFINITY, Lsum = 0.f;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int s0 = 0; s0 < nsrc; s0 += kChunk) {
-            float mm[kChunk], ll[kChunk];
-            float4 oo[kChunk];
-#pragma unroll
-            for (int j = 0; j < kChunk; ++j) {
-                const int s = s0 + j;
-                if (s < nsrc) {
-                    const bool pre = s < nprefix;
-                    const int row = pre ? k : hh % 8;
-                    const float *r = pre ? p.rec + (int64_t)((gs0 + s) * p.nrg + rg) * recf
-                                         : tail0 + (int64_t)(s - nprefix) * p.nrg_t * recf;
-                    mm[j] = __ldcg(r + 8 * D + row);
-                    ll[j] = __ldcg(r + 8 * D + 8 + row);
-                    oo[j] = __ldcg(reinterpret_cast<const float4 *>(r + row * D) + c4);
-                } else {
-                    mm[j] = -INFINITY;
-                    ll[j] = 0.f;
-                    oo[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-            }
-            float Mc = M;
-#pragma unroll
-            for (int j = 0; j < kChunk; ++j) Mc = fmaxf(Mc, mm[j]);
-            const float a = exp2_diff(M, Mc);
-            Lsum *= a;
-            acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
-#pragma unroll
-            for (int j = 0; j < kChunk; ++j) {
-                const float w8 = exp2_diff(mm[j], Mc);
-                Lsum += w8 * ll[j];
-                acc.x += w8 * oo[j].x;
-                acc.y += w8 * oo[j].y;
-                acc.z += w8 * oo[j].z;
-                acc.w += w8 * oo[j].w;
-            }
-            M = Mc;
-        }
-        const float inv = 1.f / Lsum;
-        float *dst = p.out + ((int64_t)i * p.hq + g * p.G + hh) * D;
-        reinterpret_cast<float4 *>(dst)[c4] = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-    }
-}
-
-// Expected number of records for (g, rg): prefix runs of g plus tail items
-// whose query rows meet the row group.
-__device__ __forceinline__ int expected_arrivals(const DecodeParams &p, int g, int rg)
-{
-    int cnt = p.g_slot_begin[g + 1] - p.g_slot_begin[g];
-    if (p.tail_splits > 0) {
-        const int r0 = 8 * rg, r1 = min(8 * rg + 8, p.rows_g);  // [r0, r1)
-        const int i0 = r0 / p.G, i1 = (r1 - 1) / p.G;
-        for (int i = i0; i <= i1; ++i)
-            for (int t = 0; t < p.nrg_t; ++t) {
-                const int a = i * p.G + 8 * t, b = i * p.G + min(8 * t + 8, p.G);
-                if (a < r1 && b > r0) cnt += p.tail_splits;
-            }
-    }
-    return cnt;
-}
 
 // Iterator over a thread block's prefix work in emission order:
 // run (consecutive segments of one KV head) -> row-group pass -> segment.
@@ -604,8 +521,8 @@ template <int N>
 using IC = std::integral_constant<int, N>;
 
 template <int D>
-__device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr, uint64_t *bars, int32_t *list,
-                        int32_t *tkt, uint32_t zero_addr, int mw, int lane)
+__device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr, uint64_t *bars, uint32_t zero_addr,
+                        int mw, int lane)
 {
     using L = Lay<D>;
     constexpr int kMaxNt = D / 8;   // max rank (or column) 8-tiles
@@ -667,42 +584,6 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
         l_w = 0.f;
 #pragma unroll
         for (int x = 0; x < kMaxNt; ++x) vacc[x][0] = vacc[x][1] = vacc[x][2] = vacc[x][3] = 0.f;
-    };
-    // Count one record of (g, rg) now (its writers' stores are already ordered
-    // before this point); the block that brings the last one merges the row group.
-    auto ticket_now = [&](int g, int rg) {
-        __threadfence();
-        int last = 0;
-        if (lane == 0) {
-            const uint32_t old = atomicAdd(&p.tickets[g * p.nrg + rg], 1u);
-            last = (old == (uint32_t)expected_arrivals(p, g, rg) - 1) ? 1 : 0;
-            if (last) {
-                p.tickets[g * p.nrg + rg] = 0u;
-                __threadfence();
-            }
-        }
-        if (lane == 0 && last) {
-            const int pos = atomicAdd(&list[0], 1);
-            p.clist[2 * (blockIdx.x * p.clist_cap + pos)] = g;
-            p.clist[2 * (blockIdx.x * p.clist_cap + pos) + 1] = rg;
-        }
-        __syncwarp();
-    };
-    // A tail record is written by one warp: note it for the end of the block,
-    // or count it right away when the list is full.
-    auto note_tail = [&](int g, int rg) {
-        int pos = 0;
-        if (lane == 0) pos = atomicAdd(&tkt[0], 1);
-        pos = __shfl_sync(0xffffffffu, pos, 0);
-        if (pos < L::kTkCap) {
-            if (lane == 0) {
-                tkt[1 + 2 * pos] = g;
-                tkt[2 + 2 * pos] = rg;
-            }
-            __syncwarp();
-        } else {
-            ticket_now(g, rg);
-        }
     };
     // The tile code comes in four widths (1, 2, 4 and D/16 k-steps of 16 ranks;
     // rank groups past a factor's rank read a zero line): close to the exact
@@ -1097,7 +978,7 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
             run_tile(sc_mul, tok_base, t1);
         }
         if (rgt >= 0) {
-            const int i = h[H_QI], g = h[H_G], item = h[H_ITEM];
+            const int item = h[H_ITEM];
             float *rec = p.rec + (p.tail_rec_base + (int64_t)item * p.nrg_t + rgt) * recf;
 #pragma unroll
             for (int x = 0; x < kMaxNt; ++x)
@@ -1108,14 +989,11 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
                 __stcg(rec + 8 * D + quad, m_w);
                 __stcg(rec + 8 * D + 8 + quad, lq);
             }
-            // the prefix row groups these query rows belong to
-            const int ra = i * p.G + 8 * rgt, rb = i * p.G + min(8 * rgt + 8, p.G);  // [ra, rb)
-            for (int rg = ra / 8; rg <= (rb - 1) / 8; ++rg) note_tail(g, rg);
         }
         return true;
     };
 
-    pdl_wait();  // q, records and tickets belong to the preceding grid until here
+    pdl_wait();  // q and the records belong to the preceding grids until here
     if (qcached) {  // q is 4-byte aligned (checked on the host)
         const int n4 = (int)((int64_t)p.batch * p.hq * D * 2 / 4);
         const uint32_t *src = reinterpret_cast<const uint32_t *>(p.q);
@@ -1143,34 +1021,6 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
         }
         if (!poll(false)) return false;
     }
-    // every record of this block is written: count them (one fence for all).  The
-    // prefix records follow from the static partition: one per run and row group.
-    if (!gsync()) return false;
-    if (mw == 0) {
-        __threadfence();
-        const int s0 = p.cta_seg_begin[blockIdx.x], s1 = p.cta_seg_begin[blockIdx.x + 1];
-        const int np = (s1 - s0) * p.nrg, nt = min(tkt[0], L::kTkCap);
-        for (int k = lane; k < np + nt; k += 32) {
-            int g, rg;
-            if (k < np) {
-                const SegDev sg = p.segs[s0 + k / p.nrg];
-                if (!(sg.flags & kSegLastOfRun)) continue;
-                g = p.entries[sg.entry].g;
-                rg = k % p.nrg;
-            } else {
-                g = tkt[1 + 2 * (k - np)];
-                rg = tkt[2 + 2 * (k - np)];
-            }
-            const uint32_t old = atomicAdd(&p.tickets[g * p.nrg + rg], 1u);
-            if (old == (uint32_t)expected_arrivals(p, g, rg) - 1) {
-                p.tickets[g * p.nrg + rg] = 0u;
-                const int pos = atomicAdd(&list[0], 1);  // at most clist_cap: one per (g, rg)
-                p.clist[2 * (blockIdx.x * p.clist_cap + pos)] = g;
-                p.clist[2 * (blockIdx.x * p.clist_cap + pos) + 1] = rg;
-            }
-        }
-        __threadfence();
-    }
     return true;
 }
 
@@ -1185,8 +1035,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     int32_t *hdr = reinterpret_cast<int32_t *>(smem + L::kHdr);
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L::kBar);
-    int32_t *list = reinterpret_cast<int32_t *>(smem + L::kList);
-    int32_t *tkt = reinterpret_cast<int32_t *>(smem + L::kTkT);
     const uint32_t zero_addr = smem_u32(smem + L::kZero);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
@@ -1197,10 +1045,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(smem_u32(&bars[kSlots + s]), kMmaWarps);   // empty: every MMA warp
         }
         mbar_init(smem_u32(&bars[B_GS]), kMmaWarps);
-        mbar_init(smem_u32(&bars[B_FIN]), kMmaWarps + 1);
         for (int b = B_QREADY; b < B_COUNT; ++b) mbar_init(smem_u32(&bars[b]), kMmaWarps);
-        list[0] = 0;
-        tkt[0] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (threadIdx.x < 32) reinterpret_cast<uint32_t *>(smem + L::kZero)[threadIdx.x] = 0u;
@@ -1210,21 +1055,91 @@ __global__ void __launch_bounds__(kThreads, 1)
         reinterpret_cast<uint32_t *>(smem + L::kMerge)[k] = 0u;
     __syncthreads();
 
-    bool ok = true;
     if (warp == 0) {
         if (lane == 0) run_producer<D>(p, smem, hdr, bars, &tmap_k, &tmap_v);
-        __syncwarp();
     } else {
-        ok = run_mma<D>(p, smem, hdr, bars, list, tkt, zero_addr, warp - 1, lane);
+        run_mma<D>(p, smem, hdr, bars, zero_addr, warp - 1, lane);
     }
-    if (!__all_sync(0xffffffffu, ok)) return;
-    // all warps: merge the row groups whose last record this block brought
-    __syncwarp();
-    if (lane == 0) mbar_arrive(smem_u32(&bars[B_FIN]));
-    if (!warp_wait(smem_u32(&bars[B_FIN]), 0, p.status)) return;
-    const int n = list[0];
-    const int32_t *cl = p.clist + 2 * blockIdx.x * p.clist_cap;
-    for (int k = 0; k < n; ++k) combine_rows<D>(p, cl[2 * k], cl[2 * k + 1], threadIdx.x, kThreads);
+}
+
+
+// ================================================================ combine
+// The log-sum-exp merge of the split softmax (Eq. 1 over a partition of the
+// tokens): one thread block per (KV head g, row group rg, quarter of the head
+// dimension).  A thread owns one row, one float4 column and every kNs-th
+// source record; its loads are all in flight at once, and the kNs partial
+// merges of a (row, column) meet through warp shuffles.
+template <int D>
+__global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ DecodeParams p)
+{
+    constexpr int kC4 = D / 16;              // float4 columns in a quarter
+    constexpr int kNs = 256 / (8 * kC4);     // source groups: 4 (D = 128) or 8 (D = 64)
+    constexpr int kChunk = 12;               // loads in flight per thread and round
+    pdl_trigger();
+    pdl_wait();  // every record of the decode grid is written
+    const int q4 = blockIdx.x % 4, rg = (blockIdx.x / 4) % p.nrg, g = blockIdx.x / (4 * p.nrg);
+    const int t = threadIdx.x;
+    const int sg = t % kNs, k = t / (kNs * kC4), c4 = q4 * kC4 + (t / kNs) % kC4;
+    const int recf = 8 * D + kRecFloatsExtra;
+    const int rho = 8 * rg + k;
+    const bool row_ok = rho < p.rows_g;
+    const int i = row_ok ? rho / p.G : 0, hh = row_ok ? rho % p.G : 0;
+    const int gs0 = p.g_slot_begin[g], nprefix = p.g_slot_begin[g + 1] - gs0;
+    const int S = p.tail_splits, nsrc = nprefix + S;
+    const float *tail0 = p.rec + (p.tail_rec_base + (int64_t)(i * p.hkv + g) * S * p.nrg_t + hh / 8) * recf;
+    float M = -INFINITY, Lsum = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s0 = sg; s0 < nsrc; s0 += kChunk * kNs) {
+        float mm[kChunk], ll[kChunk];
+        float4 oo[kChunk];
+#pragma unroll
+        for (int j = 0; j < kChunk; ++j) {
+            const int s = s0 + j * kNs;
+            mm[j] = -INFINITY;
+            ll[j] = 0.f;
+            oo[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (row_ok && s < nsrc) {
+                const bool pre = s < nprefix;
+                const int row = pre ? k : hh % 8;
+                const float *r = pre ? p.rec + (int64_t)((gs0 + s) * p.nrg + rg) * recf
+                                     : tail0 + (int64_t)(s - nprefix) * p.nrg_t * recf;
+                mm[j] = __ldcg(r + 8 * D + row);
+                ll[j] = __ldcg(r + 8 * D + 8 + row);
+                oo[j] = __ldcg(reinterpret_cast<const float4 *>(r + row * D) + c4);
+            }
+        }
+        float Mc = M;
+#pragma unroll
+        for (int j = 0; j < kChunk; ++j) Mc = fmaxf(Mc, mm[j]);
+        const float a = exp2_diff(M, Mc);
+        Lsum *= a;
+        acc.x *= a; acc.y *= a; acc.z *= a; acc.w *= a;
+#pragma unroll
+        for (int j = 0; j < kChunk; ++j) {
+            const float w = exp2_diff(mm[j], Mc);
+            Lsum += w * ll[j];
+            acc.x += w * oo[j].x; acc.y += w * oo[j].y; acc.z += w * oo[j].z; acc.w += w * oo[j].w;
+        }
+        M = Mc;
+    }
+    // the kNs source groups of this (row, column) are adjacent lanes
+#pragma unroll
+    for (int off = 1; off < kNs; off <<= 1) {
+        const float Mo = __shfl_xor_sync(0xffffffffu, M, off);
+        const float Lo = __shfl_xor_sync(0xffffffffu, Lsum, off);
+        const float4 ao = make_float4(__shfl_xor_sync(0xffffffffu, acc.x, off), __shfl_xor_sync(0xffffffffu, acc.y, off),
+                                      __shfl_xor_sync(0xffffffffu, acc.z, off), __shfl_xor_sync(0xffffffffu, acc.w, off));
+        const float Mn = fmaxf(M, Mo);
+        const float a = exp2_diff(M, Mn), b = exp2_diff(Mo, Mn);
+        Lsum = Lsum * a + Lo * b;
+        acc = make_float4(acc.x * a + ao.x * b, acc.y * a + ao.y * b, acc.z * a + ao.z * b, acc.w * a + ao.w * b);
+        M = Mn;
+    }
+    if (row_ok && sg == 0) {
+        const float inv = 1.f / Lsum;
+        float *dst = p.out + ((int64_t)i * p.hq + g * p.G + hh) * D;
+        reinterpret_cast<float4 *>(dst)[c4] = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    }
 }
 
 }  // namespace
@@ -1286,8 +1201,15 @@ cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k, const void 
         if (e != cudaSuccess) return e;
         configured[which] = smem_bytes;
     }
-    if (which == 0) return cudaLaunchKernelEx(&cfg, decode_kernel<64>, p, mk, mv);
-    return cudaLaunchKernelEx(&cfg, decode_kernel<128>, p, mk, mv);
+    cudaError_t e = which == 0 ? cudaLaunchKernelEx(&cfg, decode_kernel<64>, p, mk, mv)
+                               : cudaLaunchKernelEx(&cfg, decode_kernel<128>, p, mk, mv);
+    if (e != cudaSuccess) return e;
+    // the merge of the partial records, overlapping the decode grid's tail
+    cudaLaunchConfig_t cc = cfg;
+    cc.gridDim = dim3(p.hkv * p.nrg * 4);
+    cc.blockDim = dim3(256);
+    cc.dynamicSmemBytes = 0;
+    return which == 0 ? cudaLaunchKernelEx(&cc, combine_kernel<64>, p) : cudaLaunchKernelEx(&cc, combine_kernel<128>, p);
 }
 
 }  // namespace milo

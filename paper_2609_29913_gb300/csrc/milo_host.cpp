@@ -211,7 +211,6 @@ struct milo_prefix {
     int32_t *cta_seg_begin = nullptr;
     int32_t *g_slot_begin = nullptr;
     CountersDev *counters = nullptr;
-    uint32_t *tickets = nullptr;
     int32_t *status = nullptr;
 };
 
@@ -359,7 +358,7 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         milo_prefix_destroy(p);
         return cuda_fail(err, what);
     };
-    const size_t cnt_bytes = sizeof(CountersDev) + sizeof(uint32_t) * (size_t)H * p->max_nrg;
+    const size_t cnt_bytes = sizeof(CountersDev);
     if ((e = cudaMalloc(&p->packed, (size_t)std::max<int64_t>(p->packed_bytes, 128))) != cudaSuccess)
         return cleanup(e, "cudaMalloc packed");
     if ((e = cudaMalloc(&p->entries, sizeof(EntryDev) * std::max<size_t>(ents.size(), 1))) != cudaSuccess)
@@ -374,7 +373,6 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     if ((e = cudaMalloc(&p->status, sizeof(int32_t))) != cudaSuccess) return cleanup(e, "cudaMalloc status");
     if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
         return cleanup(e, "cudaMalloc offsets");
-    p->tickets = reinterpret_cast<uint32_t *>(p->counters + 1);
 
     if (!ents.empty() &&
         (e = cudaMemcpyAsync(p->entries, ents.data(), sizeof(EntryDev) * ents.size(), cudaMemcpyHostToDevice,
@@ -425,8 +423,6 @@ namespace {
 struct CallShape {
     int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
     int64_t records;
-    int64_t rec_bytes;    // partial records, at the start of the workspace
-    int64_t clist_bytes;  // per-block lists of row groups to merge, after the records
 };
 
 CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
@@ -441,9 +437,7 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
     c.records = (int64_t)p->num_slots * c.nrg + (int64_t)batch * p->hkv * c.S * c.nrg_t;
-    c.rec_bytes = (std::max<int64_t>(c.records, 1) * (8 * p->d + kRecFloatsExtra) * (int64_t)sizeof(float) + 255) / 256 * 256;
-    // a block may have to merge every (KV head, row group)
-    c.clist_bytes = (int64_t)p->num_ctas * p->hkv * c.nrg * 2 * (int64_t)sizeof(int32_t);
+
     return c;
 }
 }  // namespace
@@ -454,7 +448,7 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch, int6
     if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
     if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
-    *bytes = (size_t)(c.rec_bytes + c.clist_bytes);
+    *bytes = (size_t)std::max<int64_t>(c.records, 1) * (8 * plan->d + kRecFloatsExtra) * sizeof(float);
     return MILO_OK;
 }
 
@@ -495,10 +489,8 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.tail_offsets = tail_offsets;
     prm.out = out;
     prm.rec = static_cast<float *>(workspace);
-    prm.clist = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) + c.rec_bytes);
-    prm.clist_cap = plan->hkv * c.nrg;
+
     prm.counters = plan->counters;
-    prm.tickets = plan->tickets;
     prm.status = plan->status;
     prm.batch = batch;
     prm.hq = plan->hq;

@@ -40,7 +40,6 @@ struct CountersDev {
     uint32_t tail_next;   // dynamic tail work counter
     uint32_t ctas_done;   // thread blocks finished (resets tail_next)
     uint32_t pad[30];
-    // followed by tickets[num_kv_heads * max_row_groups]
 };
 
 struct DecodeParams {
@@ -53,10 +52,7 @@ struct DecodeParams {
     const int64_t *tail_offsets;    // [batch + 1] or null
     float *out;                     // [batch, Hq, d]
     float *rec;                     // workspace records
-    int32_t *clist;                 // workspace: per-block (g, rg) pairs to merge
-    int clist_cap;                  // pairs per block (Hkv * nrg)
     CountersDev *counters;
-    uint32_t *tickets;              // [Hkv * nrg]
     int32_t *status;
     int batch, hq, hkv, G, d;
     int rows_g;                     // batch * G
