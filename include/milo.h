@@ -105,10 +105,10 @@ milo_status_t milo_validate_table(const milo_block_table_t *table);
  * Each factor is stored zero-padded to r8 = roundup(r, 8) ranks and, for the
  * coefficient matrices, n8 = roundup(n_b, 8) tokens, as 8x8 bf16 tiles of 128
  * contiguous bytes (one tile = 8 rows x 16 bytes):
- *   C (n_b x r): token tiles of 32 tokens; the token tile k that holds t8
- *     padded tokens occupies t8 * r8 * 2 bytes starting at k * 32 * r8 * 2;
- *     inside it, tile (rank group rg, token group tg) sits at
- *     (rg * t8/8 + tg) * 128 and holds row (t % 8), column (j % 8).
+ *   C (n_b x r): tile (token group tg, rank group rg) sits at
+ *     (tg * r8/8 + rg) * 128 and holds row (t % 8), column (j % 8); tokens
+ *     [t0, t1) with t0 % 8 == 0 are the contiguous bytes
+ *     [t0 * r8 * 2, roundup(t1, 8) * r8 * 2).
  *   P (r x d): tile (rank group jg, column group cg) sits at
  *     (jg * d/8 + cg) * 128 and holds row (j % 8), column (c % 8).
  * packed_offsets: host [num_blocks * num_kv_heads * 4] byte offsets of

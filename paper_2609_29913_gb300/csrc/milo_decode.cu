@@ -882,17 +882,18 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
     };
 
     // Tile addressing shared by coefficient tiles and tail items (one copy of the
-    // tile code): cores [rank group][token group] of 128 bytes from t_k / t_v,
-    // t_stride token groups per rank group, t_ntg of them valid.
+    // tile code): 128-byte cores from t_k / t_v, core (token group tg, rank
+    // group rg) at tg * t_tgs + rg * t_rgs cores (coefficients: token-group
+    // major; tail items: column-group major), t_ntg token groups valid.
     uint32_t t_k = 0, t_v = 0;
-    int t_stride = 4, t_ntg = 4, t_nrk = 0, t_nrv = 0;
+    int t_tgk = 1, t_rgk = 1, t_tgv = 1, t_rgv = 1, t_ntg = 4, t_nrk = 0, t_nrv = 0;
     auto kaddr = [&](int hf, int m4, int kk) -> uint32_t {
         const int tg = 2 * hf + (m4 >> 1), rgk = 2 * kk + (m4 & 1);
-        return (tg < t_ntg && rgk < t_nrk) ? t_k + (rgk * t_stride + tg) * 128 + (lane % 8) * 16 : zero_addr;
+        return (tg < t_ntg && rgk < t_nrk) ? t_k + (tg * t_tgk + rgk * t_rgk) * 128 + (lane % 8) * 16 : zero_addr;
     };
     auto vaddr = [&](int hf, int m4, int jp) -> uint32_t {
         const int tg = 2 * hf + (m4 & 1), rgv = 2 * jp + (m4 >> 1);
-        return (tg < t_ntg && rgv < t_nrv) ? t_v + (rgv * t_stride + tg) * 128 + (lane % 8) * 16 : zero_addr;
+        return (tg < t_ntg && rgv < t_nrv) ? t_v + (tg * t_tgv + rgv * t_rgv) * 128 + (lane % 8) * 16 : zero_addr;
     };
     auto run_tile = [&](float sc_mul, int tok_base, int t1) {
         by_width(max((t_nrk + 1) / 2, (t_nrv + 1) / 2),
@@ -922,6 +923,9 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
                 njobs = kt0 < ntl ? (ntl - kt0 + nwg - 1) / nwg : 0;
                 t_nrk = rk8 / 8;
                 t_nrv = rv8 / 8;
+                t_tgk = t_nrk;
+                t_tgv = t_nrv;
+                t_rgk = t_rgv = 1;
             }
             tile_base += ntl;
         } else if (flags & kTailFill) {
@@ -957,6 +961,8 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
                 vbase = sbase + (D / 8) * kTailTokens * 16;
                 njobs = (t1 + kTileTokens - 1) / kTileTokens;
                 t_nrk = t_nrv = kMaxNt;
+                t_tgk = t_tgv = 1;
+                t_rgk = t_rgv = kTailTokens / 8;
             }
         }
         for (int jb = 0; jb < njobs; ++jb) {
@@ -964,13 +970,11 @@ __device__ bool run_mma(const DecodeParams &p, uint8_t *smem, const int32_t *hdr
             if (rgt < 0) {
                 const int kt = kt0 + jb * nwg;
                 t_ntg = ((kt == ntl - 1) ? last8 : kTileTokens) / 8;
-                t_stride = t_ntg;
                 t_k = kbase + kt * kTileTokens * rk8 * 2;
                 t_v = vbase + kt * kTileTokens * rv8 * 2;
                 tok_base = t0 + kt * kTileTokens;
             } else {
                 t_ntg = 4;
-                t_stride = kTailTokens / 8;
                 t_k = kbase + 4 * jb * 128;
                 t_v = vbase + 4 * jb * 128;
                 tok_base = kTileTokens * jb;

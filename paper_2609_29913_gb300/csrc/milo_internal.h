@@ -7,7 +7,7 @@
 
 namespace milo {
 
-constexpr int kTileTokens = 32;      // tokens per packed coefficient tile
+constexpr int kTileTokens = 32;      // tokens per coefficient tile (and partition cut granularity)
 constexpr int kMmaWarps = 7;         // compute warps per decode thread block (8 warps in all:
                                      // at most two per SM sub-partition, 255 registers each)
 constexpr int kThreads = 32 * (1 + kMmaWarps);  // + one producer warp

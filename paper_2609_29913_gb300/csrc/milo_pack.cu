@@ -3,9 +3,10 @@
 // table into the packed layout the decode kernel streams:
 //   * ranks zero-padded to a multiple of 8, coefficient tokens to a multiple
 //     of 8;
-//   * 8x8 bf16 tiles of 128 contiguous bytes, so that a 1-D bulk copy of a
-//     token range lands in shared memory in an ldmatrix-ready, bank-conflict
-//     free order (each tile row is one 16-byte line).
+//   * 8x8 bf16 cores of 128 contiguous bytes (each core row is one 16-byte
+//     line): for C, [token group][rank group] over the whole entry, so a 1-D
+//     bulk copy of any token range lands in shared memory as evenly strided
+//     cores (what ldmatrix and tensor-core shared-memory descriptors read).
 // The copy is bit-exact; padding is zero, so NaN-filled gaps between the
 // caller's factors never reach the packed arena.
 #include <cuda_bf16.h>
@@ -30,18 +31,14 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint16_t *__restrict__ 
     uint8_t *dst = packed + dst0;
     if (r8 == 0) return;
     if ((f & 1) == 0) {
-        // coefficients C (n x r): tiles of kTileTokens tokens, inside [rank group][token group]
-        const int n = ent.n, n8 = (n + 7) & ~7;
+        // coefficients C (n x r): 8x8 cores [token group][rank group] over the whole
+        // entry, so token groups are evenly spaced (r8/8 cores apart)
+        const int n = ent.n, n8 = (n + 7) & ~7, nrg = r8 / 8;
         const int64_t chunks = (int64_t)n8 * r8 / 8;
-        const int per_full_tile = kTileTokens * r8 / 8;  // 16-byte lines in a full tile
         for (int64_t qi = threadIdx.x; qi < chunks; qi += blockDim.x) {
-            const int kt = (int)(qi / per_full_tile);
-            const int qq = (int)(qi % per_full_tile);
-            const int t8 = min(kTileTokens, n8 - kTileTokens * kt);
-            const int ntg = t8 / 8;
-            const int core = qq / 8, row = qq % 8;
-            const int rg = core / ntg, tg = core % ntg;
-            const int t = kTileTokens * kt + 8 * tg + row;
+            const int core = (int)(qi / 8), row = (int)(qi % 8);
+            const int tg = core / nrg, rg = core % nrg;
+            const int t = 8 * tg + row;
             const int j0 = 8 * rg;
             alignas(16) uint16_t v[8];
 #pragma unroll

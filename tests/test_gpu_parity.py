@@ -159,19 +159,15 @@ def test_packed_arena_is_bit_exact(env):
             r = int(r)
             r8 = (r + 7) // 8 * 8
             base = int(offs[e, f]) // 2
-            if f % 2 == 0:   # C: tiles of 32 tokens, [rank group][token group] 8x8 tiles
+            if f % 2 == 0:   # C: [token group][rank group] 8x8 tiles over the whole entry
                 n8 = (n + 7) // 8 * 8
                 full = np.zeros((n8, r8), np.uint16)
                 full[:n, :r] = logical[loff:loff + n * r].reshape(n, r)
                 got = np.zeros_like(full)
-                for kt in range((n8 + 31) // 32):
-                    t8 = min(32, n8 - 32 * kt)
-                    ntg = t8 // 8
-                    tb = base + kt * 32 * r8
+                for tg in range(n8 // 8):
                     for rg in range(r8 // 8):
-                        for tg in range(ntg):
-                            blk = pk[tb + (rg * ntg + tg) * 64: tb + (rg * ntg + tg) * 64 + 64].reshape(8, 8)
-                            got[32 * kt + 8 * tg: 32 * kt + 8 * tg + 8, 8 * rg: 8 * rg + 8] = blk
+                        o = base + (tg * (r8 // 8) + rg) * 64
+                        got[8 * tg: 8 * tg + 8, 8 * rg: 8 * rg + 8] = pk[o:o + 64].reshape(8, 8)
             else:            # P: [rank group][column group] 8x8 tiles
                 full = np.zeros((r8, d), np.uint16)
                 full[:r] = logical[loff:loff + r * d].reshape(r, d)
