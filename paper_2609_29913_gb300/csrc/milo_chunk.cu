@@ -1,0 +1,421 @@
+// milo_chunk.cu -- the split-K decode of milo_decode.cu for up to 8 query rows
+// per KV head (batch x heads of one KV head <= 8): one warp per chunk, many
+// chunks per SM, each chunk streamed through two shared-memory slots.
+//
+// A chunk is a token range of one prefix entry (block b, KV head g).  Its warp
+// walks a fixed sequence of pieces, each at most kPieceBytes and brought by
+// bulk copies into one of two slots while the warp works on the other:
+//
+//   P^K pieces   q~ = scale * log2(e) * P^K q for up to 64 ranks per piece
+//                (Eq. 3 folded into Eq. 1); q~ is kept as bf16 hi + lo rows of
+//                the score A operand.
+//   C pieces     whole 32-token tiles (C^K rows, then C^V rows of the same
+//                tokens): scores s = C^K q~, an online softmax with a lazily
+//                raised reference max, rank-space values v~ += C^V^T p.
+//   P^V pieces   o += P^V^T v~ over up to 64 ranks per piece (Alg. 1 Stage
+//                2's back-projection), v~ taken straight from the registers.
+//
+// The chunk's record is (o, max, sum) per query row.  A dense-tail item (one
+// query's tail split for one KV head, kTailTokens tokens) brings its K and V
+// rows with 3-D TMA boxes (8 head dimensions x kTailTokens rows each, landing
+// as cores [column group][token group]) and runs the C steps on them with
+// q~ = scale * log2(e) * q; its values are already o.  The
+// merge kernel combines every record of a KV head with the log-sum-exp rule
+// (Eq. 1 over a partition of the tokens).
+//
+// Shared-memory cores are 8 rows x 16 bytes (rows = tokens or ranks); a core
+// past the data reads a zero line, so no product meets stale memory.  Every
+// wait is bounded (~2 s) and sets MILO_ERR_TIMEOUT.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include "milo.h"
+#include "milo_internal.h"
+#include "milo_ptx.cuh"
+
+namespace milo {
+namespace {
+
+constexpr int kPieceBytes = 16384;  // one slot
+constexpr int kTile = 32;           // tokens per tile
+
+template <int D>
+struct CLay {
+    static constexpr int kQ = 2 * kPieceBytes;                  // q~ A fragments [D/16][32 lanes][4]
+    static constexpr int kZero = kQ + (D / 16) * 32 * 16;       // a zero core line
+    static constexpr int kBar = kZero + 128;                    // 2 mbarriers
+    static constexpr int kTotal = kBar + 16;
+    static constexpr int kRanksPerPiece = kPieceBytes / (D * 2);  // P^K / P^V rows per piece
+};
+
+// The pieces of a prefix chunk, in order: P^K, C, P^V.
+struct Pieces {
+    int npk, nc, npv;   // pieces of each kind
+    int tpp;            // tiles per C piece
+    int rpp;            // rank 8-groups per P piece
+    __device__ int total() const { return npk + nc + npv; }
+};
+
+template <int D>
+__device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
+{
+    Pieces s;
+    s.rpp = CLay<D>::kRanksPerPiece / 8;
+    s.npk = (c.nrk + s.rpp - 1) / s.rpp;
+    s.npv = (c.nrv + s.rpp - 1) / s.rpp;
+    s.tpp = max(1, kPieceBytes / (kTile * (c.nrk + c.nrv) * 16));
+    s.nc = (c.ntok + s.tpp * kTile - 1) / (s.tpp * kTile);
+    return s;
+}
+
+template <int D>
+__global__ void __launch_bounds__(32)
+    chunk_kernel(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tmap_k,
+                 const __grid_constant__ CUtensorMap tmap_v)
+{
+    static_assert(2 * (D / 8) * kTailTokens * 16 <= 2 * kPieceBytes, "a tail item fits the two slots");
+    using L = CLay<D>;
+    constexpr int KD = D / 16;  // 16-wide k-steps over the head dimension
+    constexpr int NT = D / 8;   // 8-wide tiles over the head dimension (and the largest rank)
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int lane = threadIdx.x;
+    const int r4 = lane >> 2, c4 = lane & 3;  // mma fragment row and column pair
+    const int mi = lane >> 3, mr = lane & 7;  // ldmatrix: matrix and row this lane addresses
+    uint4 *sq = reinterpret_cast<uint4 *>(smem + L::kQ);
+    const uint32_t zline = smem_u32(smem + L::kZero) + mr * 16;
+    const uint32_t bar0 = smem_u32(smem + L::kBar);
+    const int recf = 8 * D + kRecFloatsExtra;
+    const bool is_tail = (int)blockIdx.x >= p.num_chunks;
+
+    pdl_trigger();
+    for (int i = lane; i < (L::kBar - L::kQ) / 16; i += 32)
+        reinterpret_cast<uint4 *>(smem + L::kQ)[i] = make_uint4(0u, 0u, 0u, 0u);
+
+    ChunkDev ch = {};
+    Pieces ps = {};
+    int g = 0, ntok = 0, nrk = 0, nrv = 0;
+    if (!is_tail) {
+        ch = p.chunks[blockIdx.x];
+        ps = pieces_of<D>(ch);
+        g = ch.g;
+        ntok = ch.ntok;
+        nrk = ch.nrk;
+        nrv = ch.nrv;
+    }
+    // piece k into slot k & 1 (lane 0)
+    auto issue = [&](int k) {
+        const uint32_t bar = bar0 + 8 * (k & 1), dst = smem_u32(smem) + (k & 1) * kPieceBytes;
+        if (k < ps.npk) {
+            const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, ch.nrk);
+            const uint32_t b = (uint32_t)(r1 - r0) * D * 16;
+            mbar_arrive_tx(bar, b);
+            bulk_g2s(dst, p.packed + ch.pk + (int64_t)r0 * D * 16, b, bar);
+        } else if (k < ps.npk + ps.nc) {
+            const int t0 = (k - ps.npk) * ps.tpp * kTile;
+            const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;  // rows (a multiple of 8)
+            const uint32_t kb = (uint32_t)r8 * ch.nrk * 16, vb = (uint32_t)r8 * ch.nrv * 16;
+            mbar_arrive_tx(bar, kb + vb);
+            bulk_g2s(dst, p.packed + ch.ck + (int64_t)t0 * ch.nrk * 16, kb, bar);
+            bulk_g2s(dst + kb, p.packed + ch.cv + (int64_t)t0 * ch.nrv * 16, vb, bar);
+        } else {
+            const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, ch.nrv);
+            const uint32_t b = (uint32_t)(r1 - r0) * D * 16;
+            mbar_arrive_tx(bar, b);
+            bulk_g2s(dst, p.packed + ch.pv + (int64_t)r0 * D * 16, b, bar);
+        }
+    };
+    if (lane == 0) {
+        mbar_init(bar0, 1);
+        mbar_init(bar0 + 8, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        if (!is_tail) {
+            issue(0);
+            if (ps.total() > 1) issue(1);
+        }
+    }
+    __syncwarp();
+    pdl_wait();  // q, the tails and the records belong to the preceding grids until here
+
+    // the warp's online-softmax state and rank-space values
+    float m_w = -INFINITY, l_w = 0.f;
+    float vacc[NT][4];
+#pragma unroll
+    for (int n = 0; n < NT; ++n) vacc[n][0] = vacc[n][1] = vacc[n][2] = vacc[n][3] = 0.f;
+
+    // One 32-token tile at token tb of the tile data: C^K core (tg, rg) at
+    // kb + tg * ktg + rg * krg, C^V core at vb + tg * vtg + rg * vrg; tg8 token
+    // groups present, tokens < nv valid.
+    auto tile = [&](uint32_t kb, uint32_t ktg, uint32_t krg, uint32_t vb, uint32_t vtg, uint32_t vrg, int tb, int tg8,
+                    int nv) {
+        const int nks = (nrk + 1) / 2;
+        float s4[4][4];
+#pragma unroll
+        for (int n = 0; n < 4; ++n) s4[n][0] = s4[n][1] = s4[n][2] = s4[n][3] = 0.f;
+#pragma unroll
+        for (int ks = 0; ks < KD; ++ks) {
+            if (ks < nks) {
+                const uint4 q4 = sq[ks * 32 + lane];
+                const uint32_t qa[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    // matrices: (tg0, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks), (tg0 + 1, 2ks + 1)
+                    const int tg = tb / 8 + 2 * h + (mi >> 1), rg = 2 * ks + (mi & 1);
+                    const uint32_t addr = (tg < tg8 && rg < nrk) ? kb + tg * ktg + rg * krg + mr * 16 : zline;
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4(addr, b0, b1, b2, b3);
+                    mma16816(s4[2 * h], qa, b0, b1);
+                    mma16816(s4[2 * h + 1], qa, b2, b3);
+                }
+            }
+        }
+        // score of token tb + 8n + 2 c4 + j: hi rows + lo rows
+        float sv8[8];
+#pragma unroll
+        for (int n = 0; n < 4; ++n) {
+            const int tok = tb + 8 * n + 2 * c4;
+            sv8[2 * n] = tok < nv ? s4[n][0] + s4[n][2] : -INFINITY;
+            sv8[2 * n + 1] = tok + 1 < nv ? s4[n][1] + s4[n][3] : -INFINITY;
+        }
+        float mx = sv8[0];
+#pragma unroll
+        for (int j = 1; j < 8; ++j) mx = fmaxf(mx, sv8[j]);
+        mx = quad_max(mx);
+        if (mx > m_w + 8.f) {  // lazy rescale: p stays <= 2^8
+            const float alpha = exp2_diff(m_w, mx);
+            l_w *= alpha;
+#pragma unroll
+            for (int n = 0; n < NT; ++n) {
+                vacc[n][0] *= alpha;
+                vacc[n][1] *= alpha;
+                vacc[n][2] *= alpha;
+                vacc[n][3] *= alpha;
+            }
+            m_w = mx;
+        }
+        float pr[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            pr[j] = exp2_diff(sv8[j], m_w);
+            l_w += pr[j];
+        }
+        // A fragments of p for the two 16-token halves (rows 0-7 hi, 8-15 lo)
+        uint32_t pa[2][4];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            split_hi_lo(pr[4 * h], pr[4 * h + 1], pa[h][0], pa[h][1]);
+            split_hi_lo(pr[4 * h + 2], pr[4 * h + 3], pa[h][2], pa[h][3]);
+        }
+#pragma unroll
+        for (int jp = 0; jp < NT / 2; ++jp) {
+            if (2 * jp < nrv) {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    if (tb + 16 * h < nv) {
+                        // matrices (transposed): (tg0, 2jp), (tg0 + 1, 2jp), (tg0, 2jp + 1), (tg0 + 1, 2jp + 1)
+                        const int tg = tb / 8 + 2 * h + (mi & 1), rg = 2 * jp + (mi >> 1);
+                        const uint32_t addr = (tg < tg8 && rg < nrv) ? vb + tg * vtg + rg * vrg + mr * 16 : zline;
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4_t(addr, b0, b1, b2, b3);
+                        mma16816(vacc[2 * jp], pa[h], b0, b1);
+                        mma16816(vacc[2 * jp + 1], pa[h], b2, b3);
+                    }
+                }
+            }
+        }
+    };
+
+    const int64_t rec_idx = is_tail ? p.tail_rec_base + ((int)blockIdx.x - p.num_chunks) : (int64_t)blockIdx.x;
+    float *rec = p.rec + rec_idx * recf;
+    if (is_tail) {
+        // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense tail
+        const int item = (int)blockIdx.x - p.num_chunks, S = p.tail_splits;
+        const int qi = item / (p.hkv * S), sp = item % S;
+        g = (item / S) % p.hkv;
+        const int64_t o0 = p.tail_offsets[qi], o1 = p.tail_offsets[qi + 1];
+        const int T = (int)(o1 - o0);
+        if (sp == S - 1 && T > S * kTailTokens && lane == 0) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
+        const int t0 = sp * kTailTokens;
+        ntok = max(0, min(t0 + kTailTokens, T) - t0);
+        nrk = nrv = NT;
+        // q~ = scale * log2(e) * q of the G heads of query qi, as score A fragments
+#pragma unroll 1
+        for (int ks = 0; ks < KD; ++ks) {
+            float x[4] = {0.f, 0.f, 0.f, 0.f};
+            if (r4 < p.G) {
+                const uint16_t *qr = p.q + ((int64_t)qi * p.hq + g * p.G + r4) * D + 16 * ks + 2 * c4;
+                const __nv_bfloat162 a2 = *reinterpret_cast<const __nv_bfloat162 *>(qr);
+                const __nv_bfloat162 b2 = *reinterpret_cast<const __nv_bfloat162 *>(qr + 8);
+                x[0] = __low2float(a2) * p.scale_log2;
+                x[1] = __high2float(a2) * p.scale_log2;
+                x[2] = __low2float(b2) * p.scale_log2;
+                x[3] = __high2float(b2) * p.scale_log2;
+            }
+            uint4 f;
+            split_hi_lo(x[0], x[1], f.x, f.y);
+            split_hi_lo(x[2], x[3], f.z, f.w);
+            sq[ks * 32 + lane] = f;
+        }
+        // K then V: one box of kTailTokens rows x 8 columns per column group
+        constexpr uint32_t kBox = kTailTokens * 16, kHalf = NT * kBox;
+        if (ntok > 0) {
+            if (lane == 0) {
+                mbar_arrive_tx(bar0, 2 * kHalf);
+#pragma unroll 1
+                for (int c = 0; c < NT; ++c) {
+                    tma_load_3d(smem_u32(smem) + c * kBox, &tmap_k, 8 * c, g, (int)(o0 + t0), bar0);
+                    tma_load_3d(smem_u32(smem) + kHalf + c * kBox, &tmap_v, 8 * c, g, (int)(o0 + t0), bar0);
+                }
+            }
+            __syncwarp();
+            mbar_wait(bar0, 0, p.status);
+        }
+#pragma unroll 1
+        for (int tb = 0; tb < ntok; tb += kTile)
+            tile(smem_u32(smem), 128, kBox, smem_u32(smem) + kHalf, 128, kBox, tb, kTailTokens / 8, ntok);
+        // the values are already in the head dimension: o = v~
+        l_w = quad_sum(l_w);
+#pragma unroll
+        for (int n = 0; n < NT; ++n)
+            __stcg(reinterpret_cast<float2 *>(rec + r4 * D + 8 * n + 2 * c4),
+                   make_float2(vacc[n][0] + vacc[n][2], vacc[n][1] + vacc[n][3]));
+        if (c4 == 0) {
+            __stcg(rec + 8 * D + r4, ntok > 0 ? m_w : -INFINITY);
+            __stcg(rec + 8 * D + 8 + r4, ntok > 0 ? l_w : 0.f);
+        }
+        return;
+    }
+
+    // q rows of KV head g as projection A fragments (rows 0-7; rows 8-15 zero)
+    uint32_t qa[KD][2];
+    {
+        const bool row_ok = r4 < p.rows_g;
+        const uint16_t *qr = p.q + ((int64_t)(r4 / p.G) * p.hq + g * p.G + r4 % p.G) * D + 2 * c4;
+#pragma unroll
+        for (int ks = 0; ks < KD; ++ks) {
+            qa[ks][0] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks) : 0u;
+            qa[ks][1] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks + 8) : 0u;
+        }
+    }
+    float o[NT][4];
+#pragma unroll
+    for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+    const int np = ps.total();
+#pragma unroll 1
+    for (int k = 0; k < np; ++k) {
+        mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
+        const uint32_t slot = smem_u32(smem) + (k & 1) * kPieceBytes;
+        if (k < ps.npk) {
+            // projection of rank 8-tiles [r0, r1): cores (nt - r0, cg) of this piece
+            const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, nrk);
+#pragma unroll 1
+            for (int nt = r0; nt < r1; nt += 2) {
+                float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll
+                for (int ks = 0; ks < KD; ks += 2) {
+                    const uint32_t a0[4] = {qa[ks][0], 0u, qa[ks][1], 0u};
+                    const uint32_t a1[4] = {qa[ks + 1][0], 0u, qa[ks + 1][1], 0u};
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        if (nt + j < r1) {
+                            // matrices: cores (nt + j, 2ks .. 2ks + 3) -> b0, b1 of k-steps ks, ks + 1
+                            uint32_t b0, b1, b2, b3;
+                            ldsm_x4(slot + ((nt + j - r0) * NT + 2 * ks + mi) * 128 + mr * 16, b0, b1, b2, b3);
+                            mma16816(acc[j], a0, b0, b1);
+                            mma16816(acc[j], a1, b2, b3);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 2; ++j) {
+                    if (nt + j < r1) {
+                        uint32_t hi, lo;
+                        split_hi_lo(acc[j][0] * p.scale_log2, acc[j][1] * p.scale_log2, hi, lo);
+                        uint32_t *f = reinterpret_cast<uint32_t *>(&sq[((nt + j) / 2) * 32 + lane]);
+                        f[((nt + j) & 1) * 2] = hi;
+                        f[((nt + j) & 1) * 2 + 1] = lo;
+                    }
+                }
+            }
+            __syncwarp();
+        } else if (k < ps.npk + ps.nc) {
+            const int t0 = (k - ps.npk) * ps.tpp * kTile;
+            const int nv = min(ps.tpp * kTile, ntok - t0);  // valid tokens of this piece
+            const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;
+            const uint32_t vb = slot + (uint32_t)r8 * nrk * 16;
+#pragma unroll 1
+            for (int tb = 0; tb < nv; tb += kTile) tile(slot, nrk * 128, 128, vb, nrv * 128, 128, tb, r8 / 8, nv);
+        } else {
+            // back-projection over rank 8-groups [r0, r1): 16-rank k-steps of v~
+            const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, nrv);
+#pragma unroll
+            for (int ks = 0; ks < NT / 2; ++ks) {
+                if (2 * ks >= r0 && 2 * ks < r1) {
+                    uint32_t a[4];
+                    split_hi_lo(vacc[2 * ks][0] + vacc[2 * ks][2], vacc[2 * ks][1] + vacc[2 * ks][3], a[0], a[1]);
+                    split_hi_lo(vacc[2 * ks + 1][0] + vacc[2 * ks + 1][2], vacc[2 * ks + 1][1] + vacc[2 * ks + 1][3],
+                                a[2], a[3]);
+#pragma unroll
+                    for (int cp = 0; cp < NT / 2; ++cp) {
+                        // matrices (transposed): (2ks, 2cp), (2ks + 1, 2cp), (2ks, 2cp + 1), (2ks + 1, 2cp + 1)
+                        const int jg = 2 * ks + (mi & 1), cg = 2 * cp + (mi >> 1);
+                        const uint32_t addr = jg < r1 ? slot + ((jg - r0) * NT + cg) * 128 + mr * 16 : zline;
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4_t(addr, b0, b1, b2, b3);
+                        mma16816(o[2 * cp], a, b0, b1);
+                        mma16816(o[2 * cp + 1], a, b2, b3);
+                    }
+                }
+            }
+        }
+        // the slot is free again (its reads ordered before the async-proxy
+        // write): bring piece k + 2 into it
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0 && k + 2 < np) issue(k + 2);
+    }
+    l_w = quad_sum(l_w);
+#pragma unroll
+    for (int n = 0; n < NT; ++n)
+        __stcg(reinterpret_cast<float2 *>(rec + r4 * D + 8 * n + 2 * c4),
+               make_float2(o[n][0] + o[n][2], o[n][1] + o[n][3]));
+    if (c4 == 0) {
+        __stcg(rec + 8 * D + r4, m_w);
+        __stcg(rec + 8 * D + 8 + r4, l_w);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void *tmap_v, cudaStream_t stream)
+{
+    const CUtensorMap &mk = *static_cast<const CUtensorMap *>(tmap_k);
+    const CUtensorMap &mv = *static_cast<const CUtensorMap *>(tmap_v);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.num_chunks + (p.has_tail ? p.num_tail_items : 0));
+    cfg.blockDim = dim3(32);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cfg.gridDim.x == 0) return cudaSuccess;
+    static int configured[2] = {0, 0};
+    const int w = p.d == 64 ? 0 : 1;
+    const void *fn = w == 0 ? reinterpret_cast<const void *>(chunk_kernel<64>)
+                            : reinterpret_cast<const void *>(chunk_kernel<128>);
+    const int smem = w == 0 ? CLay<64>::kTotal : CLay<128>::kTotal;
+    if (!configured[w]) {
+        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        // several thread blocks per SM need the largest shared-memory carveout
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        if (e != cudaSuccess) return e;
+        configured[w] = 1;
+    }
+    cfg.dynamicSmemBytes = (size_t)smem;
+    return w == 0 ? cudaLaunchKernelEx(&cfg, chunk_kernel<64>, p, mk, mv)
+                  : cudaLaunchKernelEx(&cfg, chunk_kernel<128>, p, mk, mv);
+}
+
+}  // namespace milo

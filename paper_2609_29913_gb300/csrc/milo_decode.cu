@@ -8,29 +8,34 @@
 // split softmax (Eq. 1 is associative over token partitions once each part
 // carries its running max and sum).
 //
-// One persistent thread block per SM, two roles:
+// This file holds the persistent kernel, used when a KV head has more than 8
+// query rows (several row groups share every coefficient tile read), and the
+// merge kernel.  Up to 8 rows per KV head take the short-block kernel of
+// milo_chunk.cu.
+//
+// Persistent kernel, one thread block per SM, two roles:
 //   producer   (warp 0, one lane): turns the block's static list of prefix
 //              segments, then dynamically claimed dense-tail items, into an
 //              in-order stream of "fills" of at most kSlotBytes.  A fill packs
 //              the previous segment's P^V, the next segment's P^K and as many
 //              whole coefficient tiles of that segment as fit; a tail fill
-//              holds one tail item's K and V (3-D TMA, 128-byte swizzle).  Each
-//              fill is one ring slot, one mbarrier, up to four bulk copies.
+//              holds one tail item's K and V (3-D TMA).  Each fill is one ring
+//              slot, one mbarrier, up to six bulk copies.
 //   MMA warps  (warps 1..7): consume every fill in order.  P^K part: each warp
 //              projects q~ = scale * log2(e) * P^K q for a slice of the rank
 //              tiles (mma m16n8k16, result split into bf16 hi + lo rows).
-//              Coefficient part: 16-token sub-tiles round-robin over the
-//              warps -- scores (A rows 0-7 q~ hi, rows 8-15 q~ lo), online
-//              softmax in registers, rank-space values (A rows = p hi, p lo).
-//              P^V part (segment end): the warps pool their (max, sum, v~),
-//              each merges a slice of v~, then each back-projects a slice of
-//              the head dimension through P^V into its running output; at the
-//              end of a run the slices are written as one partial record.
-//              Tail fills go whole to one warp each (no pooling needed).
-// The thread block that brings the last record of a (KV head, row group)
-// merges that row group's records at the end of the kernel; no thread block
-// waits for another.  Every wait is bounded (~2 s); on expiry the thread
-// records MILO_ERR_TIMEOUT in the sticky status word and leaves.
+//              Coefficient part: 32-token tiles round-robin over the warps --
+//              scores (A rows 0-7 q~ hi, rows 8-15 q~ lo), online softmax in
+//              registers, rank-space values (A rows = p hi, p lo).  P^V part
+//              (segment end): the warps pool their (max, sum, v~), each merges
+//              a slice of v~, then each back-projects a slice of the head
+//              dimension through P^V into its running output; at the end of a
+//              run the slices are written as one partial record.  Tail fills
+//              go whole to one warp each.
+// The merge kernel (launched next, with programmatic dependent launch)
+// combines the partial records of every (KV head, row group).  Every wait is
+// bounded (~2 s); on expiry the thread records MILO_ERR_TIMEOUT in the sticky
+// status word and leaves.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -39,30 +44,13 @@
 
 #include "milo.h"
 #include "milo_internal.h"
+#include "milo_ptx.cuh"
 
 namespace milo {
 namespace {
 
-constexpr uint64_t kTimeoutNs = 2000000000ull;
-
-// fill flags: a fill carries, in processing order, the previous segment's
-// P^V, up to two bases P^K of coming segments, the start of a segment, its
-// coefficient tiles, a tail item, the end marker
-enum : int { kHasPv = 1, kHasPk0 = 2, kHasPk1 = 4, kSegStart = 8, kHasC = 16, kTailFill = 32, kEndFill = 64 };
 // run flags of a segment end
 enum : int { F_RUN_FIRST = 1, F_RUN_LAST = 2 };
-// fill header words
-enum : int {
-    H_FLAGS,
-    H_PV_G, H_PV_RV8, H_PV_REC, H_PV_RUN, H_PV_PASS, H_PV_OFF,
-    H_PK_J, H_PK_G, H_PK_RK8, H_PK_PASS, H_PK_OFF,  // P^K part 0; part 1 follows with the same layout
-    H_PK1_J = H_PK_J + 5,
-    H_SS_J = H_PK1_J + 5, H_SS_PASS, H_SS_RK8,
-    H_C_OFF, H_T0, H_T1, H_RK8, H_RV8, H_TOK8,
-    H_QI, H_G, H_ITEM,
-    H_WORDS
-};
-static_assert(H_WORDS <= kHdrInts, "fill header size");
 // barrier indices: full[kSlots], empty[kSlots], then the MMA warps' own
 enum : int {
     B_GS = 2 * kSlots,  // group sync of the MMA warps
@@ -74,161 +62,10 @@ enum : int {
     B_COUNT
 };
 
-// ------------------------------------------------------------------ PTX ----
-__device__ __forceinline__ uint32_t smem_u32(const void *p)
-{
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ uint64_t globaltimer()
-{
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t tx)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(tx) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar)
-{
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Bounded wait: false (and the status word set) once kTimeoutNs has passed.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status)
-{
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer();
-    for (;;) {
-#pragma unroll 1
-        for (int i = 0; i < 32; ++i)
-            if (mbar_try_wait(bar, parity)) return true;
-        if (globaltimer() - t0 > kTimeoutNs) {
-            atomicCAS(status, 0, (int32_t)MILO_ERR_TIMEOUT);
-            return false;
-        }
-    }
-}
-
-// Warp-uniform bounded wait: every lane waits; all agree on the outcome.
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, int32_t *status)
-{
-    const bool ok = mbar_wait(bar, parity, status);
-    return __all_sync(0xffffffffu, ok);
-}
-
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar)
-{
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-        "l"(src), "r"(bytes), "r"(bar)
-        : "memory");
-}
-
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, int c0, int c1, int c2,
-                                            uint32_t bar)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
-        "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-        "l"(map), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
-        : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3)
-{
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
-}
-
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3)
-{
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
-}
-
-// D(16x8 f32) += A(16x16 bf16, row) * B(16x8 bf16, col)
-__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1)
-{
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
-        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" :::); }
-
-// Two floats -> bf16x2 (low half = first) rounded to nearest, and the
-// bf16x2 of their rounding residuals: x = hi + lo to ~16 significant bits.
-__device__ __forceinline__ void split_hi_lo(float x0, float x1, uint32_t &hi, uint32_t &lo)
-{
-    const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
-    const float2 hf = __bfloat1622float2(h);
-    const __nv_bfloat162 l = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
-    hi = *reinterpret_cast<const uint32_t *>(&h);
-    lo = *reinterpret_cast<const uint32_t *>(&l);
-}
-
-__device__ __forceinline__ float quad_max(float v)
-{
-    v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
-    return fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
-}
-
-__device__ __forceinline__ float quad_sum(float v)
-{
-    v += __shfl_xor_sync(0xffffffffu, v, 1);
-    return v + __shfl_xor_sync(0xffffffffu, v, 2);
-}
-
-// exp2(a - b) with the convention that a = -inf gives 0 (and b = -inf too).
-__device__ __forceinline__ float exp2_diff(float a, float b)
-{
-    return (a == -INFINITY) ? 0.f : exp2f(a - b);
-}
-
 // ------------------------------------------------------- shared memory ----
+constexpr int al(int x, int a) { return (x + a - 1) / a * a; }
 template <int D>
 struct Lay {
-    static constexpr int al(int x, int a) { return (x + a - 1) / a * a; }
     static constexpr int kRing = 0;                               // kSlots fills
     static constexpr int kMerge = kRing + kSlots * kSlotBytes;    // per-warp (max, sum, v~) dumps
     static constexpr int kMergeWarp = 32 * D + 256;               // v~ [d/8][32 lanes] float2 + (m,l) [32] float2
@@ -347,13 +184,14 @@ __device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr,
 
     // P^V of the last finished segment, attached to the next fill
     bool pv_pending = false;
-    int pv_g = 0, pv_rv8 = 0, pv_rec = 0, pv_run = 0, pv_pass = 0;
+    int pv_g = 0, pv_rv8 = 0, pv_rec = 0, pv_run = 0, pv_pass = 0, pv_seg = 0;
     int64_t pv_off = 0;
     auto put_pv = [&]() {
         const uint32_t bytes = (uint32_t)pv_rv8 * D * 2;
         h[H_PV_G] = pv_g;
         h[H_PV_RV8] = pv_rv8;
         h[H_PV_REC] = pv_rec;
+        h[H_PV_SEG] = pv_seg;
         h[H_PV_RUN] = pv_run;
         h[H_PV_PASS] = pv_pass;
         h[H_PV_OFF] = (int)used;
@@ -451,6 +289,7 @@ __device__ void run_producer(const DecodeParams &p, uint8_t *smem, int32_t *hdr,
         pv_g = ent.g;
         pv_rv8 = rv8;
         pv_rec = seg.slot;
+        pv_seg = it.sg;
         pv_run = (it.sg == it.r0 ? F_RUN_FIRST : 0) | (it.sg == it.r1 ? F_RUN_LAST : 0);
         pv_pass = it.pass;
         pv_off = ent.off_pv;
@@ -1069,40 +908,38 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ================================================================ combine
 // The log-sum-exp merge of the split softmax (Eq. 1 over a partition of the
-// tokens): one thread block per (KV head g, row group rg, quarter of the head
-// dimension).  A thread owns one row, one float4 column and every kNs-th
-// source record; its loads are all in flight at once, and the kNs partial
-// merges of a (row, column) meet through warp shuffles.
+// tokens): one thread block per (KV head g, row group rg, float4 column c of
+// the head dimension), one warp per row.  Lane l of a warp takes source
+// records l, l + 32, ...; its loads are all in flight at once, and the 32
+// partial merges meet through a shuffle butterfly.
 template <int D>
 __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ DecodeParams p)
 {
-    constexpr int kC4 = D / 16;              // float4 columns in a quarter
-    constexpr int kNs = 256 / (8 * kC4);     // source groups: 4 (D = 128) or 8 (D = 64)
-    constexpr int kChunk = 12;               // loads in flight per thread and round
+    constexpr int kC4 = D / 4;    // float4 columns of a row
+    constexpr int kChunk = 8;     // records in flight per lane and round
     pdl_trigger();
     pdl_wait();  // every record of the decode grid is written
-    const int q4 = blockIdx.x % 4, rg = (blockIdx.x / 4) % p.nrg, g = blockIdx.x / (4 * p.nrg);
-    const int t = threadIdx.x;
-    const int sg = t % kNs, k = t / (kNs * kC4), c4 = q4 * kC4 + (t / kNs) % kC4;
+    const int c4 = blockIdx.x % kC4, rg = (blockIdx.x / kC4) % p.nrg, g = blockIdx.x / (kC4 * p.nrg);
+    const int k = threadIdx.x / 32, sl = threadIdx.x % 32;
     const int recf = 8 * D + kRecFloatsExtra;
     const int rho = 8 * rg + k;
     const bool row_ok = rho < p.rows_g;
     const int i = row_ok ? rho / p.G : 0, hh = row_ok ? rho % p.G : 0;
     const int gs0 = p.g_slot_begin[g], nprefix = p.g_slot_begin[g + 1] - gs0;
-    const int S = p.tail_splits, nsrc = nprefix + S;
+    const int S = p.tail_splits, nsrc = row_ok ? nprefix + S : 0;
     const float *tail0 = p.rec + (p.tail_rec_base + (int64_t)(i * p.hkv + g) * S * p.nrg_t + hh / 8) * recf;
     float M = -INFINITY, Lsum = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s0 = sg; s0 < nsrc; s0 += kChunk * kNs) {
+    for (int s0 = sl; s0 < nsrc; s0 += kChunk * 32) {
         float mm[kChunk], ll[kChunk];
         float4 oo[kChunk];
 #pragma unroll
         for (int j = 0; j < kChunk; ++j) {
-            const int s = s0 + j * kNs;
+            const int s = s0 + j * 32;
             mm[j] = -INFINITY;
             ll[j] = 0.f;
             oo[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (row_ok && s < nsrc) {
+            if (s < nsrc) {
                 const bool pre = s < nprefix;
                 const int row = pre ? k : hh % 8;
                 const float *r = pre ? p.rec + (int64_t)((gs0 + s) * p.nrg + rg) * recf
@@ -1126,9 +963,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ De
         }
         M = Mc;
     }
-    // the kNs source groups of this (row, column) are adjacent lanes
 #pragma unroll
-    for (int off = 1; off < kNs; off <<= 1) {
+    for (int off = 1; off < 32; off <<= 1) {
         const float Mo = __shfl_xor_sync(0xffffffffu, M, off);
         const float Lo = __shfl_xor_sync(0xffffffffu, Lsum, off);
         const float4 ao = make_float4(__shfl_xor_sync(0xffffffffu, acc.x, off), __shfl_xor_sync(0xffffffffu, acc.y, off),
@@ -1139,7 +975,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ De
         acc = make_float4(acc.x * a + ao.x * b, acc.y * a + ao.y * b, acc.z * a + ao.z * b, acc.w * a + ao.w * b);
         M = Mn;
     }
-    if (row_ok && sg == 0) {
+    if (row_ok && sl == 0) {
         const float inv = 1.f / Lsum;
         float *dst = p.out + ((int64_t)i * p.hq + g * p.G + hh) * D;
         reinterpret_cast<float4 *>(dst)[c4] = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
@@ -1205,12 +1041,13 @@ cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k, const void 
         if (e != cudaSuccess) return e;
         configured[which] = smem_bytes;
     }
-    cudaError_t e = which == 0 ? cudaLaunchKernelEx(&cfg, decode_kernel<64>, p, mk, mv)
-                               : cudaLaunchKernelEx(&cfg, decode_kernel<128>, p, mk, mv);
+    cudaError_t e = p.num_chunks > 0 ? launch_chunks(p, tmap_k, tmap_v, stream)
+                    : which == 0 ? cudaLaunchKernelEx(&cfg, decode_kernel<64>, p, mk, mv)
+                                      : cudaLaunchKernelEx(&cfg, decode_kernel<128>, p, mk, mv);
     if (e != cudaSuccess) return e;
     // the merge of the partial records, overlapping the decode grid's tail
     cudaLaunchConfig_t cc = cfg;
-    cc.gridDim = dim3(p.hkv * p.nrg * 4);
+    cc.gridDim = dim3(p.hkv * p.nrg * (p.d / 4));
     cc.blockDim = dim3(256);
     cc.dynamicSmemBytes = 0;
     return which == 0 ? cudaLaunchKernelEx(&cc, combine_kernel<64>, p) : cudaLaunchKernelEx(&cc, combine_kernel<128>, p);

@@ -180,6 +180,41 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
     }
 }
 
+// Chunks of the short-block decode: every prefix entry, KV-head-major then in
+// block order, cut into token ranges of at most kChunkMaxTok tokens whose
+// coefficient rows (C^K and C^V, rounded up to 8 tokens) fit kChunkBytes; a
+// range starts at a multiple of 32 tokens.
+void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs, std::vector<ChunkDev> &chunks,
+                  std::vector<int32_t> &g_begin)
+{
+    const int H = t->num_kv_heads, nb = t->num_blocks;
+    chunks.clear();
+    g_begin.assign((size_t)H + 1, 0);
+    for (int g = 0; g < H; ++g) {
+        g_begin[(size_t)g] = (int32_t)chunks.size();
+        for (int b = 0; b < nb; ++b) {
+            const int e = b * H + g, n = t->block_len[b];
+            const int rk8 = r8(t->rank_k[e]), rv8 = r8(t->rank_v[e]), n8 = r8(n);
+            const int tok = std::max(32, std::min(kChunkMaxTok, kChunkBytes / ((rk8 + rv8) * 2) / 32 * 32));
+            for (int t0 = 0; t0 < n; t0 += tok) {
+                ChunkDev c = {};
+                const int t1 = std::min(n, t0 + tok);
+                c.ck = poffs[(size_t)e * 4 + 0] + (int64_t)t0 * rk8 * 2;
+                c.pk = poffs[(size_t)e * 4 + 1];
+                c.cv = poffs[(size_t)e * 4 + 2] + (int64_t)t0 * rv8 * 2;
+                c.pv = poffs[(size_t)e * 4 + 3];
+                c.ntok = t1 - t0;
+                c.tok8 = std::min(r8(t1), n8) - t0;
+                c.nrk = rk8 / 8;
+                c.nrv = rv8 / 8;
+                c.g = g;
+                chunks.push_back(c);
+            }
+        }
+    }
+    g_begin[(size_t)H] = (int32_t)chunks.size();
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -210,6 +245,9 @@ struct milo_prefix {
     SegDev *segs = nullptr;
     int32_t *cta_seg_begin = nullptr;
     int32_t *g_slot_begin = nullptr;
+    ChunkDev *chunks = nullptr;       // short-block decode: prefix chunks, KV-head-major
+    int32_t *g_chunk_begin = nullptr; // first chunk of each KV head
+    int num_chunks = 0;
     CountersDev *counters = nullptr;
     int32_t *status = nullptr;
 };
@@ -287,6 +325,8 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaFree(plan->segs);
     cudaFree(plan->cta_seg_begin);
     cudaFree(plan->g_slot_begin);
+    cudaFree(plan->chunks);
+    cudaFree(plan->g_chunk_begin);
     cudaFree(plan->counters);
     cudaFree(plan->status);
     cudaSetDevice(cur);
@@ -347,6 +387,10 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         p->prefix_tokens += (x % H == 0) ? en.n : 0;
         p->logical_bytes += ((int64_t)en.n * (en.rk + en.rv) + (int64_t)(en.rk + en.rv) * d) * 2;
     }
+    std::vector<ChunkDev> chunks;
+    std::vector<int32_t> g_chunk;
+    build_chunks(table, poffs, chunks, g_chunk);
+    p->num_chunks = (int)chunks.size();
     std::vector<SegDev> sd(segs.size());
     for (size_t i = 0; i < segs.size(); ++i) {
         sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
@@ -369,6 +413,16 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         return cleanup(e, "cudaMalloc cta_seg_begin");
     if ((e = cudaMalloc(&p->g_slot_begin, sizeof(int32_t) * g_slot.size())) != cudaSuccess)
         return cleanup(e, "cudaMalloc g_slot_begin");
+    if ((e = cudaMalloc(&p->chunks, sizeof(ChunkDev) * std::max<size_t>(chunks.size(), 1))) != cudaSuccess)
+        return cleanup(e, "cudaMalloc chunks");
+    if ((e = cudaMalloc(&p->g_chunk_begin, sizeof(int32_t) * g_chunk.size())) != cudaSuccess)
+        return cleanup(e, "cudaMalloc g_chunk_begin");
+    if (!chunks.empty() && (e = cudaMemcpyAsync(p->chunks, chunks.data(), sizeof(ChunkDev) * chunks.size(),
+                                                cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+        return cleanup(e, "copy chunks");
+    if ((e = cudaMemcpyAsync(p->g_chunk_begin, g_chunk.data(), sizeof(int32_t) * g_chunk.size(),
+                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+        return cleanup(e, "copy g_chunk_begin");
     if ((e = cudaMalloc(&p->counters, cnt_bytes)) != cudaSuccess) return cleanup(e, "cudaMalloc counters");
     if ((e = cudaMalloc(&p->status, sizeof(int32_t))) != cudaSuccess) return cleanup(e, "cudaMalloc status");
     if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
@@ -436,7 +490,10 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
-    c.records = (int64_t)p->num_slots * c.nrg + (int64_t)batch * p->hkv * c.S * c.nrg_t;
+    // one record per prefix chunk (one row group: the short-block decode) or
+    // per run and row group (the persistent kernel); then the tail items
+    const int64_t prefix = c.nrg == 1 ? (int64_t)p->num_chunks : (int64_t)p->num_slots * c.nrg;
+    c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
 
     return c;
 }
@@ -509,6 +566,16 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.num_tail_items = batch * plan->hkv * c.S;
     prm.has_tail = c.S > 0 ? 1 : 0;
     prm.tail_rec_base = (int64_t)plan->num_slots * c.nrg;
+    // one row group: the short-block decode
+    prm.tail_k = static_cast<const uint16_t *>(tail_k);
+    prm.tail_v = static_cast<const uint16_t *>(tail_v);
+    prm.chunks = plan->chunks;
+    prm.num_chunks = c.nrg == 1 ? plan->num_chunks : 0;
+    if (prm.num_chunks > 0) {
+        prm.g_slot_begin = plan->g_chunk_begin;
+        prm.num_slots = plan->num_chunks;
+        prm.tail_rec_base = plan->num_chunks;
+    }
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)plan->d);
     prm.scale_log2 = scale * 1.4426950408889634f;
     prm.num_ctas = plan->num_ctas;

@@ -17,6 +17,24 @@ constexpr int kHdrInts = 32;         // fill header (ints)
 constexpr int kTailTokens = 64;      // tokens per dense-tail work item
 constexpr int kRecFloatsExtra = 16;  // m[8], l[8] after o[8][d] in a record
 
+// fill flags: a fill carries, in processing order, the previous segment's
+// P^V, up to two bases P^K of coming segments, the start of a segment, its
+// coefficient tiles, a tail item, the end marker
+enum : int { kHasPv = 1, kHasPk0 = 2, kHasPk1 = 4, kSegStart = 8, kHasC = 16, kTailFill = 32, kEndFill = 64 };
+// fill header words
+enum : int {
+    H_FLAGS,
+    H_PV_G, H_PV_RV8, H_PV_REC, H_PV_RUN, H_PV_PASS, H_PV_OFF,
+    H_PK_J, H_PK_G, H_PK_RK8, H_PK_PASS, H_PK_OFF,  // P^K part 0; part 1 follows with the same layout
+    H_PK1_J = H_PK_J + 5,
+    H_SS_J = H_PK1_J + 5, H_SS_PASS, H_SS_RK8,
+    H_C_OFF, H_T0, H_T1, H_RK8, H_RV8, H_TOK8,
+    H_QI, H_G, H_ITEM,
+    H_PV_SEG,
+    H_WORDS
+};
+static_assert(H_WORDS <= kHdrInts, "fill header size");
+
 // Per-(block, KV head) entry of the packed arena.
 struct EntryDev {
     int64_t off_ck, off_pk, off_cv, off_pv;  // byte offsets (128-aligned)
@@ -34,6 +52,18 @@ struct SegDev {
     int32_t flags;
     int32_t pad[3];
 };
+
+// One chunk of the short-block decode: tokens [t0, t1) of a prefix entry.
+constexpr int kChunkBytes = 49152;   // coefficient bytes (C^K + C^V rows) per chunk
+constexpr int kChunkMaxTok = 1024;   // tokens per chunk
+struct ChunkDev {
+    int64_t ck, cv, pk, pv;     // byte offsets in the packed arena (C^K, C^V at the chunk's first token)
+    int32_t ntok, tok8;         // tokens, and rows copied (rounded up to 8 within the entry)
+    int32_t nrk, nrv;           // rank 8-groups of K and V
+    int32_t g;                  // KV head
+    int32_t pad[3];
+};
+static_assert(sizeof(ChunkDev) == 64, "chunk descriptor size");
 
 // Device-side counters owned by a plan (zero between calls).
 struct CountersDev {
@@ -69,6 +99,9 @@ struct DecodeParams {
     int64_t tail_rec_base;          // first tail record index
     float scale_log2;               // softmax scale * log2(e)
     int num_ctas;
+    const ChunkDev *chunks;         // short-block decode: the prefix chunks (KV-head-major)
+    int num_chunks;                 // 0: the persistent kernels run
+    const uint16_t *tail_k, *tail_v;  // bf16 [rows, Hkv, d] dense tails (or null)
 };
 
 // Launchers implemented in the .cu files.
@@ -82,6 +115,11 @@ cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k,
                           cudaStream_t stream);
 
 int decode_smem_bytes(int head_dim, int nrg_cta);
+
+// The short-block decode grid alone (one thread block per prefix chunk and
+// per tail item); launch_decode calls it and then launches the merge.
+cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void *tmap_v, cudaStream_t stream);
+
 
 // Fixed scratch of milo_attn_decode_static (a file-scope device array).
 constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;
