@@ -15,13 +15,20 @@
 //   P^V pieces   o += P^V^T v~ over up to 64 ranks per piece (Alg. 1 Stage
 //                2's back-projection), v~ taken straight from the registers.
 //
-// The chunk's record is (o, max, sum) per query row.  A dense-tail item (one
+// The chunk's record is (o, max, sum) per query row.  The last chunk block
+// of a prefix entry (a per-entry counter) merges the entry's chunk records
+// into one entry record; an entry of one chunk writes its entry record
+// directly.  Entry and tail records are counted per KV head.  A dense-tail item (one
 // query's tail split for one KV head, kTailTokens tokens) brings its K and V
 // rows with 3-D TMA boxes (8 head dimensions x kTailTokens rows each, landing
 // as cores [column group][token group]) and runs the C steps on them with
 // q~ = scale * log2(e) * q; its values are already o.  The
-// merge kernel combines every record of a KV head with the log-sum-exp rule
-// (Eq. 1 over a partition of the tokens).
+// last thread blocks of the grid merge: one warp per (KV head, row, quarter
+// of the head dimension) waits (bounded) until every entry and tail record
+// of its KV head is counted, then combines them with the log-sum-exp rule (Eq. 1 over a
+// partition of the tokens) and writes the output; the last of a KV head's
+// merge blocks resets its counters for the next call.  Chunk and tail blocks
+// never wait on other blocks, and they come first in the grid.
 //
 // Shared-memory cores are 8 rows x 16 bytes (rows = tokens or ranks); a core
 // past the data reads a zero line, so no product meets stale memory.  Every
@@ -68,6 +75,194 @@ __device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
     return s;
 }
 
+constexpr int kMergeWarpsPerHead = 32;  // 8 rows x 4 quarters of the head dimension
+
+// This block's record is written: count it for KV head g (lane 0 after a fence).
+__device__ __forceinline__ void count_record(const DecodeParams &p, int g, int lane)
+{
+    __threadfence();
+    __syncwarp();
+    if (lane == 0) atomicAdd(&p.head_cnt[g], 1u);
+}
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t *ptr)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
+    return v;
+}
+
+// The last chunk of a prefix entry: merge the entry's nch chunk records
+// (c0 ...) into its entry record.  Lane l: row l / 4, quarter l % 4.
+template <int D>
+__device__ void merge_entry(const DecodeParams &p, int c0, int nch, float *dst, int lane)
+{
+    constexpr int kF4 = D / 16;
+    constexpr int kLoads = 4;
+    const int recf = 8 * D + kRecFloatsExtra;
+    const int row = lane >> 2, qq = lane & 3;
+    float M = -INFINITY, Lsum = 0.f;
+    float4 acc[kF4];
+#pragma unroll
+    for (int f = 0; f < kF4; ++f) acc[f] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s0 = 0; s0 < nch; s0 += kLoads) {
+        float mm[kLoads], ll[kLoads];
+        float4 oo[kLoads][kF4];
+#pragma unroll
+        for (int j = 0; j < kLoads; ++j) {
+            mm[j] = -INFINITY;
+            ll[j] = 0.f;
+#pragma unroll
+            for (int f = 0; f < kF4; ++f) oo[j][f] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (s0 + j < nch) {
+                const float *r = p.rec + (int64_t)(c0 + s0 + j) * recf;
+                mm[j] = __ldcg(r + 8 * D + row);
+                ll[j] = __ldcg(r + 8 * D + 8 + row);
+#pragma unroll
+                for (int f = 0; f < kF4; ++f)
+                    oo[j][f] = __ldcg(reinterpret_cast<const float4 *>(r + row * D + qq * (D / 4)) + f);
+            }
+        }
+        float Mc = M;
+#pragma unroll
+        for (int j = 0; j < kLoads; ++j) Mc = fmaxf(Mc, mm[j]);
+        const float a = exp2_diff(M, Mc);
+        Lsum *= a;
+#pragma unroll
+        for (int f = 0; f < kF4; ++f) {
+            acc[f].x *= a; acc[f].y *= a; acc[f].z *= a; acc[f].w *= a;
+        }
+#pragma unroll
+        for (int j = 0; j < kLoads; ++j) {
+            const float w = exp2_diff(mm[j], Mc);
+            Lsum += w * ll[j];
+#pragma unroll
+            for (int f = 0; f < kF4; ++f) {
+                acc[f].x += w * oo[j][f].x; acc[f].y += w * oo[j][f].y;
+                acc[f].z += w * oo[j][f].z; acc[f].w += w * oo[j][f].w;
+            }
+        }
+        M = Mc;
+    }
+#pragma unroll
+    for (int f = 0; f < kF4; ++f) __stcg(reinterpret_cast<float4 *>(dst + row * D + qq * (D / 4)) + f, acc[f]);
+    if (qq == 0) {
+        __stcg(dst + 8 * D + row, M);
+        __stcg(dst + 8 * D + 8 + row, Lsum);
+    }
+}
+
+// One merge warp: KV head g, row k of the row group, quarter qq of the head
+// dimension.  Lane l takes records l, l + 32, ...; the 32 partial merges meet
+// through a shuffle butterfly.
+template <int D>
+__device__ void merge_warp(const DecodeParams &p, int mb, int lane)
+{
+    constexpr int kF4 = D / 16;  // float4 columns per quarter
+    constexpr int kChunkLoads = 4;
+    const int g = mb / kMergeWarpsPerHead, k = (mb / 4) % 8, qq = mb % 4;
+    const int recf = 8 * D + kRecFloatsExtra;
+    const int gs0 = p.g_entry_begin[g], nprefix = p.g_entry_begin[g + 1] - gs0;
+    const int S = p.tail_splits, nsrc = nprefix + p.batch * S;
+    pdl_wait();  // the output belongs to the preceding grids until here
+    // every record of KV head g: its chunks and the tail items of every query
+    if (lane == 0) {
+        const uint64_t t0 = globaltimer();
+        while (ld_acquire(&p.head_cnt[g]) < (uint32_t)nsrc) {
+            __nanosleep(200);
+            if (globaltimer() - t0 > kTimeoutNs) {
+                atomicCAS(p.status, 0, (int32_t)MILO_ERR_TIMEOUT);
+                break;
+            }
+        }
+    }
+    __syncwarp();
+    const bool row_ok = k < p.rows_g;
+    if (row_ok) {
+        const int i = k / p.G, hh = k % p.G;
+        const float *tail0 = p.rec + (p.tail_rec_base + (int64_t)(i * p.hkv + g) * S) * recf;
+        const int ns = nprefix + S;  // this row: the prefix chunks and query i's tail splits
+        float M = -INFINITY, Lsum = 0.f;
+        float4 acc[kF4];
+#pragma unroll
+        for (int j = 0; j < kF4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int s0 = lane; s0 < ns; s0 += 32 * kChunkLoads) {
+            float mm[kChunkLoads], ll[kChunkLoads];
+            float4 oo[kChunkLoads][kF4];
+#pragma unroll
+            for (int j = 0; j < kChunkLoads; ++j) {
+                const int s = s0 + 32 * j;
+                mm[j] = -INFINITY;
+                ll[j] = 0.f;
+#pragma unroll
+                for (int f = 0; f < kF4; ++f) oo[j][f] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (s < ns) {
+                    const bool pre = s < nprefix;
+                    const int row = pre ? k : hh;
+                    const float *r = pre ? p.rec + (int64_t)(gs0 + s) * recf : tail0 + (int64_t)(s - nprefix) * recf;
+                    mm[j] = __ldcg(r + 8 * D + row);
+                    ll[j] = __ldcg(r + 8 * D + 8 + row);
+#pragma unroll
+                    for (int f = 0; f < kF4; ++f)
+                        oo[j][f] = __ldcg(reinterpret_cast<const float4 *>(r + row * D + qq * (D / 4)) + f);
+                }
+            }
+            float Mc = M;
+#pragma unroll
+            for (int j = 0; j < kChunkLoads; ++j) Mc = fmaxf(Mc, mm[j]);
+            const float a = exp2_diff(M, Mc);
+            Lsum *= a;
+#pragma unroll
+            for (int f = 0; f < kF4; ++f) {
+                acc[f].x *= a; acc[f].y *= a; acc[f].z *= a; acc[f].w *= a;
+            }
+#pragma unroll
+            for (int j = 0; j < kChunkLoads; ++j) {
+                const float w = exp2_diff(mm[j], Mc);
+                Lsum += w * ll[j];
+#pragma unroll
+                for (int f = 0; f < kF4; ++f) {
+                    acc[f].x += w * oo[j][f].x; acc[f].y += w * oo[j][f].y;
+                    acc[f].z += w * oo[j][f].z; acc[f].w += w * oo[j][f].w;
+                }
+            }
+            M = Mc;
+        }
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const float Mo = __shfl_xor_sync(0xffffffffu, M, off);
+            const float Lo = __shfl_xor_sync(0xffffffffu, Lsum, off);
+            const float Mn = fmaxf(M, Mo);
+            const float a = exp2_diff(M, Mn), b = exp2_diff(Mo, Mn);
+            Lsum = Lsum * a + Lo * b;
+#pragma unroll
+            for (int f = 0; f < kF4; ++f) {
+                const float4 o2 = make_float4(__shfl_xor_sync(0xffffffffu, acc[f].x, off),
+                                              __shfl_xor_sync(0xffffffffu, acc[f].y, off),
+                                              __shfl_xor_sync(0xffffffffu, acc[f].z, off),
+                                              __shfl_xor_sync(0xffffffffu, acc[f].w, off));
+                acc[f] = make_float4(acc[f].x * a + o2.x * b, acc[f].y * a + o2.y * b, acc[f].z * a + o2.z * b,
+                                     acc[f].w * a + o2.w * b);
+            }
+            M = Mn;
+        }
+        const float inv = 1.f / Lsum;
+        float *dst = p.out + ((int64_t)i * p.hq + g * p.G + hh) * D + qq * (D / 4);
+#pragma unroll
+        for (int f = 0; f < kF4; ++f)
+            if (lane == f)
+                reinterpret_cast<float4 *>(dst)[f] =
+                    make_float4(acc[f].x * inv, acc[f].y * inv, acc[f].z * inv, acc[f].w * inv);
+    }
+    // the last merge warp of KV head g resets its counters for the next call
+    __syncwarp();
+    if (lane == 0 && atomicAdd(&p.head_cnt[p.hkv + g], 1u) == kMergeWarpsPerHead - 1) {
+        p.head_cnt[g] = 0u;
+        p.head_cnt[p.hkv + g] = 0u;
+        __threadfence();
+    }
+}
+
 template <int D>
 __global__ void __launch_bounds__(32)
     chunk_kernel(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tmap_k,
@@ -88,6 +283,11 @@ __global__ void __launch_bounds__(32)
     const bool is_tail = (int)blockIdx.x >= p.num_chunks;
 
     pdl_trigger();
+    const int first_merge = p.num_chunks + (p.has_tail ? p.num_tail_items : 0);
+    if ((int)blockIdx.x >= first_merge) {
+        merge_warp<D>(p, (int)blockIdx.x - first_merge, lane);
+        return;
+    }
     for (int i = lane; i < (L::kBar - L::kQ) / 16; i += 32)
         reinterpret_cast<uint4 *>(smem + L::kQ)[i] = make_uint4(0u, 0u, 0u, 0u);
 
@@ -224,7 +424,9 @@ __global__ void __launch_bounds__(32)
         }
     };
 
-    const int64_t rec_idx = is_tail ? p.tail_rec_base + ((int)blockIdx.x - p.num_chunks) : (int64_t)blockIdx.x;
+    const int64_t rec_idx = is_tail      ? p.tail_rec_base + ((int)blockIdx.x - p.num_chunks)
+                            : ch.nch == 1 ? (int64_t)p.num_chunks + ch.erec  // the entry record itself
+                                          : (int64_t)blockIdx.x;
     float *rec = p.rec + rec_idx * recf;
     if (is_tail) {
         // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense tail
@@ -282,6 +484,7 @@ __global__ void __launch_bounds__(32)
             __stcg(rec + 8 * D + r4, ntok > 0 ? m_w : -INFINITY);
             __stcg(rec + 8 * D + 8 + r4, ntok > 0 ? l_w : 0.f);
         }
+        count_record(p, g, lane);
         return;
     }
 
@@ -382,6 +585,19 @@ __global__ void __launch_bounds__(32)
         __stcg(rec + 8 * D + r4, m_w);
         __stcg(rec + 8 * D + 8 + r4, l_w);
     }
+    if (ch.nch > 1) {
+        // the entry's last chunk to finish merges its chunk records
+        __threadfence();
+        __syncwarp();
+        uint32_t old = 0;
+        if (lane == 0) old = atomicAdd(&p.entry_cnt[ch.erec], 1u);
+        old = __shfl_sync(0xffffffffu, old, 0);
+        if (old != (uint32_t)ch.nch - 1) return;
+        if (lane == 0) p.entry_cnt[ch.erec] = 0u;  // ready for the next call
+        __threadfence();
+        merge_entry<D>(p, ch.c0, ch.nch, p.rec + ((int64_t)p.num_chunks + ch.erec) * recf, lane);
+    }
+    count_record(p, g, lane);
 }
 
 }  // namespace
@@ -391,7 +607,7 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     const CUtensorMap &mk = *static_cast<const CUtensorMap *>(tmap_k);
     const CUtensorMap &mv = *static_cast<const CUtensorMap *>(tmap_v);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.num_chunks + (p.has_tail ? p.num_tail_items : 0));
+    cfg.gridDim = dim3(p.num_chunks + (p.has_tail ? p.num_tail_items : 0) + p.hkv * kMergeWarpsPerHead);
     cfg.blockDim = dim3(32);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -399,7 +615,6 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (cfg.gridDim.x == 0) return cudaSuccess;
     static int configured[2] = {0, 0};
     const int w = p.d == 64 ? 0 : 1;
     const void *fn = w == 0 ? reinterpret_cast<const void *>(chunk_kernel<64>)

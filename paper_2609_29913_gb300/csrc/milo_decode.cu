@@ -1044,7 +1044,7 @@ cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k, const void 
     cudaError_t e = p.num_chunks > 0 ? launch_chunks(p, tmap_k, tmap_v, stream)
                     : which == 0 ? cudaLaunchKernelEx(&cfg, decode_kernel<64>, p, mk, mv)
                                       : cudaLaunchKernelEx(&cfg, decode_kernel<128>, p, mk, mv);
-    if (e != cudaSuccess) return e;
+    if (e != cudaSuccess || p.num_chunks > 0) return e;  // the short-block grid merges itself
     // the merge of the partial records, overlapping the decode grid's tail
     cudaLaunchConfig_t cc = cfg;
     cc.gridDim = dim3(p.hkv * p.nrg * (p.d / 4));

@@ -185,14 +185,17 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
 // coefficient rows (C^K and C^V, rounded up to 8 tokens) fit kChunkBytes; a
 // range starts at a multiple of 32 tokens.
 void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs, std::vector<ChunkDev> &chunks,
-                  std::vector<int32_t> &g_begin)
+                  std::vector<int32_t> &g_begin, std::vector<int32_t> &g_entry)
 {
     const int H = t->num_kv_heads, nb = t->num_blocks;
     chunks.clear();
     g_begin.assign((size_t)H + 1, 0);
+    g_entry.assign((size_t)H + 1, 0);
     for (int g = 0; g < H; ++g) {
         g_begin[(size_t)g] = (int32_t)chunks.size();
+        g_entry[(size_t)g] = g * nb;
         for (int b = 0; b < nb; ++b) {
+            const int c0 = (int)chunks.size();
             const int e = b * H + g, n = t->block_len[b];
             const int rk8 = r8(t->rank_k[e]), rv8 = r8(t->rank_v[e]), n8 = r8(n);
             const int tok = std::max(32, std::min(kChunkMaxTok, kChunkBytes / ((rk8 + rv8) * 2) / 32 * 32));
@@ -208,11 +211,15 @@ void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs
                 c.nrk = rk8 / 8;
                 c.nrv = rv8 / 8;
                 c.g = g;
+                c.erec = g * nb + b;
+                c.c0 = c0;
                 chunks.push_back(c);
             }
+            for (size_t x = (size_t)c0; x < chunks.size(); ++x) chunks[x].nch = (int32_t)chunks.size() - c0;
         }
     }
     g_begin[(size_t)H] = (int32_t)chunks.size();
+    g_entry[(size_t)H] = H * nb;
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -247,6 +254,7 @@ struct milo_prefix {
     int32_t *g_slot_begin = nullptr;
     ChunkDev *chunks = nullptr;       // short-block decode: prefix chunks, KV-head-major
     int32_t *g_chunk_begin = nullptr; // first chunk of each KV head
+    int32_t *g_entry_begin = nullptr; // first entry record of each KV head (after the chunk records)
     int num_chunks = 0;
     CountersDev *counters = nullptr;
     int32_t *status = nullptr;
@@ -327,6 +335,7 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaFree(plan->g_slot_begin);
     cudaFree(plan->chunks);
     cudaFree(plan->g_chunk_begin);
+    cudaFree(plan->g_entry_begin);
     cudaFree(plan->counters);
     cudaFree(plan->status);
     cudaSetDevice(cur);
@@ -388,9 +397,10 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         p->logical_bytes += ((int64_t)en.n * (en.rk + en.rv) + (int64_t)(en.rk + en.rv) * d) * 2;
     }
     std::vector<ChunkDev> chunks;
-    std::vector<int32_t> g_chunk;
-    build_chunks(table, poffs, chunks, g_chunk);
+    std::vector<int32_t> g_chunk, g_entry;
+    build_chunks(table, poffs, chunks, g_chunk, g_entry);
     p->num_chunks = (int)chunks.size();
+    for (auto &x : g_entry) x += p->num_chunks;  // entry records follow the chunk records
     std::vector<SegDev> sd(segs.size());
     for (size_t i = 0; i < segs.size(); ++i) {
         sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
@@ -402,7 +412,8 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         milo_prefix_destroy(p);
         return cuda_fail(err, what);
     };
-    const size_t cnt_bytes = sizeof(CountersDev);
+    // + per-KV-head and per-entry counters of the short-block decode
+    const size_t cnt_bytes = sizeof(CountersDev) + sizeof(uint32_t) * (2 * (size_t)H + (size_t)E);
     if ((e = cudaMalloc(&p->packed, (size_t)std::max<int64_t>(p->packed_bytes, 128))) != cudaSuccess)
         return cleanup(e, "cudaMalloc packed");
     if ((e = cudaMalloc(&p->entries, sizeof(EntryDev) * std::max<size_t>(ents.size(), 1))) != cudaSuccess)
@@ -417,6 +428,11 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         return cleanup(e, "cudaMalloc chunks");
     if ((e = cudaMalloc(&p->g_chunk_begin, sizeof(int32_t) * g_chunk.size())) != cudaSuccess)
         return cleanup(e, "cudaMalloc g_chunk_begin");
+    if ((e = cudaMalloc(&p->g_entry_begin, sizeof(int32_t) * g_entry.size())) != cudaSuccess)
+        return cleanup(e, "cudaMalloc g_entry_begin");
+    if ((e = cudaMemcpyAsync(p->g_entry_begin, g_entry.data(), sizeof(int32_t) * g_entry.size(),
+                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+        return cleanup(e, "copy g_entry_begin");
     if (!chunks.empty() && (e = cudaMemcpyAsync(p->chunks, chunks.data(), sizeof(ChunkDev) * chunks.size(),
                                                 cudaMemcpyHostToDevice, stream)) != cudaSuccess)
         return cleanup(e, "copy chunks");
@@ -490,9 +506,11 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
-    // one record per prefix chunk (one row group: the short-block decode) or
-    // per run and row group (the persistent kernel); then the tail items
-    const int64_t prefix = c.nrg == 1 ? (int64_t)p->num_chunks : (int64_t)p->num_slots * c.nrg;
+    // one record per prefix chunk and one per prefix entry (one row group: the
+    // short-block decode), or one per run and row group (the persistent
+    // kernel); then the tail items
+    const int64_t prefix = c.nrg == 1 ? (int64_t)p->num_chunks + (int64_t)p->nb * p->hkv
+                                      : (int64_t)p->num_slots * c.nrg;
     c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
 
     return c;
@@ -548,6 +566,9 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.rec = static_cast<float *>(workspace);
 
     prm.counters = plan->counters;
+    prm.head_cnt = reinterpret_cast<uint32_t *>(plan->counters + 1);
+    prm.entry_cnt = prm.head_cnt + 2 * plan->hkv;
+    prm.g_entry_begin = plan->g_entry_begin;
     prm.status = plan->status;
     prm.batch = batch;
     prm.hq = plan->hq;
@@ -574,7 +595,7 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     if (prm.num_chunks > 0) {
         prm.g_slot_begin = plan->g_chunk_begin;
         prm.num_slots = plan->num_chunks;
-        prm.tail_rec_base = plan->num_chunks;
+        prm.tail_rec_base = (int64_t)plan->num_chunks + (int64_t)plan->nb * plan->hkv;
     }
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)plan->d);
     prm.scale_log2 = scale * 1.4426950408889634f;

@@ -61,7 +61,8 @@ struct ChunkDev {
     int32_t ntok, tok8;         // tokens, and rows copied (rounded up to 8 within the entry)
     int32_t nrk, nrv;           // rank 8-groups of K and V
     int32_t g;                  // KV head
-    int32_t pad[3];
+    int32_t erec;               // the entry's record slot (KV-head-major entry order)
+    int32_t c0, nch;            // the entry's first chunk and its number of chunks
 };
 static_assert(sizeof(ChunkDev) == 64, "chunk descriptor size");
 
@@ -102,6 +103,9 @@ struct DecodeParams {
     const ChunkDev *chunks;         // short-block decode: the prefix chunks (KV-head-major)
     int num_chunks;                 // 0: the persistent kernels run
     const uint16_t *tail_k, *tail_v;  // bf16 [rows, Hkv, d] dense tails (or null)
+    uint32_t *head_cnt;             // [2 Hkv]: records done per KV head, merge blocks done per KV head
+    uint32_t *entry_cnt;            // [entries]: chunk records done per prefix entry
+    const int32_t *g_entry_begin;   // [Hkv + 1]: first entry record of each KV head
 };
 
 // Launchers implemented in the .cu files.
