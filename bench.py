@@ -370,13 +370,18 @@ def main():
             tr = json.load(f)
         from paper_2609_29913_gb300 import build as b
         import hashlib
-        h = hashlib.sha256(open(os.path.join(b.CSRC, "milo_decode.cu"), "rb").read()).hexdigest()[:16]
         entry = tr.get(cfg.name)
+        src = entry.get("kernel_source", "milo_decode.cu") if entry else "milo_decode.cu"
+        h = hashlib.sha256(open(os.path.join(b.CSRC, src), "rb").read()).hexdigest()[:16]
         if entry and entry.get("kernel_sha") == h:
             traffic = entry["dram_bytes_per_launch"]
     except Exception:
         traffic = None
     value = world * tokens / (ms_step * 1e-3)
+    # up to 8 query rows per KV head: one short-block grid per layer (chunks,
+    # tail items and the merge); more: the persistent kernel and the merge kernel
+    short = cfg.batch * (cfg.num_q_heads // cfg.num_kv_heads) <= 8
+    kernels_per_layer = 1 if short else 2
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
@@ -387,18 +392,22 @@ def main():
                    "tokens_per_step": tokens, "algorithmic_bytes_per_step": alg_bytes,
                    "l2": "inputs larger than L2 (step reads %.2f GB > 129 MB); no flush" % (alg_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "launch": "one CUDA graph of %d per-layer calls, each a decode and a merge kernel "
-                             "(programmatic dependent launch)" % cfg.layers},
+                   "launch": ("one CUDA graph of %d per-layer calls, each one grid of one-warp blocks: "
+                              "prefix chunks, dense-tail items, merge warps (programmatic dependent launch)"
+                              if short else
+                              "one CUDA graph of %d per-layer calls, each a persistent decode and a merge "
+                              "kernel (programmatic dependent launch)") % cfg.layers},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": f"{peak_kind} copy bandwidth",
-                     "kernel": "decode_kernel (rank-space split-K decode, fused combine)",
+                     "kernel": ("chunk_kernel (one warp per prefix chunk, fused merge)" if short
+                                else "decode_kernel (persistent rank-space split-K decode)"),
                      "per_launch_bytes": alg_bytes // cfg.layers,
                      "per_launch_us": ms_step * 1e3 / cfg.layers},
         "cpu_baseline": cpu,
         "e2e": {"value": world * tokens / (e_ms * 1e-3), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms},
-        "gpu_launches": 2 * cfg.layers * args.steps,  # decode + merge kernel per layer
+        "gpu_launches": kernels_per_layer * cfg.layers * args.steps,
         "clocks": clocks.summary(),
         "parity_check": check,
         "setup_s": t_gen,
