@@ -36,6 +36,8 @@
 #include <cuda.h>
 #include <cuda_bf16.h>
 
+#include <type_traits>
+
 #include "milo.h"
 #include "milo_internal.h"
 #include "milo_ptx.cuh"
@@ -344,28 +346,29 @@ __global__ void __launch_bounds__(32)
 
     // One 32-token tile at token tb of the tile data: C^K core (tg, rg) at
     // kb + tg * ktg + rg * krg, C^V core at vb + tg * vtg + rg * vrg; tg8 token
-    // groups present, tokens < nv valid.
-    auto tile = [&](uint32_t kb, uint32_t ktg, uint32_t krg, uint32_t vb, uint32_t vtg, uint32_t vrg, int tb, int tg8,
-                    int nv) {
-        const int nks = (nrk + 1) / 2;
+    // groups present, tokens < nv valid.  R16 (a compile-time constant, at
+    // least both ranks / 16) fixes the 16-rank steps, so that the body is one
+    // straight block; rank groups past a rank and token groups past the data
+    // read the zero line.
+    auto tile = [&](auto r16c, uint32_t kb, uint32_t ktg, uint32_t krg, uint32_t vb, uint32_t vtg, uint32_t vrg,
+                    int tb, int tg8, int nv) {
+        constexpr int R16 = decltype(r16c)::value;
         float s4[4][4];
 #pragma unroll
         for (int n = 0; n < 4; ++n) s4[n][0] = s4[n][1] = s4[n][2] = s4[n][3] = 0.f;
 #pragma unroll
-        for (int ks = 0; ks < KD; ++ks) {
-            if (ks < nks) {
-                const uint4 q4 = sq[ks * 32 + lane];
-                const uint32_t qa[4] = {q4.x, q4.y, q4.z, q4.w};
+        for (int ks = 0; ks < R16; ++ks) {
+            const uint4 q4 = sq[ks * 32 + lane];
+            const uint32_t qa[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    // matrices: (tg0, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks), (tg0 + 1, 2ks + 1)
-                    const int tg = tb / 8 + 2 * h + (mi >> 1), rg = 2 * ks + (mi & 1);
-                    const uint32_t addr = (tg < tg8 && rg < nrk) ? kb + tg * ktg + rg * krg + mr * 16 : zline;
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4(addr, b0, b1, b2, b3);
-                    mma16816(s4[2 * h], qa, b0, b1);
-                    mma16816(s4[2 * h + 1], qa, b2, b3);
-                }
+            for (int h = 0; h < 2; ++h) {
+                // matrices: (tg0, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks), (tg0 + 1, 2ks + 1)
+                const int tg = tb / 8 + 2 * h + (mi >> 1), rg = 2 * ks + (mi & 1);
+                const uint32_t addr = (tg < tg8 && rg < nrk) ? kb + tg * ktg + rg * krg + mr * 16 : zline;
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4(addr, b0, b1, b2, b3);
+                mma16816(s4[2 * h], qa, b0, b1);
+                mma16816(s4[2 * h + 1], qa, b2, b3);
             }
         }
         // score of token tb + 8n + 2 c4 + j: hi rows + lo rows
@@ -376,28 +379,29 @@ __global__ void __launch_bounds__(32)
             sv8[2 * n] = tok < nv ? s4[n][0] + s4[n][2] : -INFINITY;
             sv8[2 * n + 1] = tok + 1 < nv ? s4[n][1] + s4[n][3] : -INFINITY;
         }
-        float mx = sv8[0];
+        const float lm = fmaxf(fmaxf(fmaxf(sv8[0], sv8[1]), fmaxf(sv8[2], sv8[3])),
+                               fmaxf(fmaxf(sv8[4], sv8[5]), fmaxf(sv8[6], sv8[7])));
+        // lazy rescale (p stays <= 2^8): the row maximum is formed only when
+        // some score passes the reference by more than 8
+        if (__any_sync(0xffffffffu, lm > m_w + 8.f)) {
+            const float mx = quad_max(lm);
+            if (mx > m_w + 8.f) {
+                const float alpha = exp2_diff(m_w, mx);
+                l_w *= alpha;
 #pragma unroll
-        for (int j = 1; j < 8; ++j) mx = fmaxf(mx, sv8[j]);
-        mx = quad_max(mx);
-        if (mx > m_w + 8.f) {  // lazy rescale: p stays <= 2^8
-            const float alpha = exp2_diff(m_w, mx);
-            l_w *= alpha;
-#pragma unroll
-            for (int n = 0; n < NT; ++n) {
-                vacc[n][0] *= alpha;
-                vacc[n][1] *= alpha;
-                vacc[n][2] *= alpha;
-                vacc[n][3] *= alpha;
+                for (int n = 0; n < NT; ++n) {
+                    vacc[n][0] *= alpha;
+                    vacc[n][1] *= alpha;
+                    vacc[n][2] *= alpha;
+                    vacc[n][3] *= alpha;
+                }
+                m_w = mx;
             }
-            m_w = mx;
         }
         float pr[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            pr[j] = exp2_diff(sv8[j], m_w);
-            l_w += pr[j];
-        }
+        for (int j = 0; j < 8; ++j) pr[j] = exp2_diff(sv8[j], m_w);
+        l_w += ((pr[0] + pr[1]) + (pr[2] + pr[3])) + ((pr[4] + pr[5]) + (pr[6] + pr[7]));
         // A fragments of p for the two 16-token halves (rows 0-7 hi, 8-15 lo)
         uint32_t pa[2][4];
 #pragma unroll
@@ -406,23 +410,36 @@ __global__ void __launch_bounds__(32)
             split_hi_lo(pr[4 * h + 2], pr[4 * h + 3], pa[h][2], pa[h][3]);
         }
 #pragma unroll
-        for (int jp = 0; jp < NT / 2; ++jp) {
-            if (2 * jp < nrv) {
+        for (int jp = 0; jp < R16; ++jp) {
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    if (tb + 16 * h < nv) {
-                        // matrices (transposed): (tg0, 2jp), (tg0 + 1, 2jp), (tg0, 2jp + 1), (tg0 + 1, 2jp + 1)
-                        const int tg = tb / 8 + 2 * h + (mi & 1), rg = 2 * jp + (mi >> 1);
-                        const uint32_t addr = (tg < tg8 && rg < nrv) ? vb + tg * vtg + rg * vrg + mr * 16 : zline;
-                        uint32_t b0, b1, b2, b3;
-                        ldsm_x4_t(addr, b0, b1, b2, b3);
-                        mma16816(vacc[2 * jp], pa[h], b0, b1);
-                        mma16816(vacc[2 * jp + 1], pa[h], b2, b3);
-                    }
-                }
+            for (int h = 0; h < 2; ++h) {
+                // matrices (transposed): (tg0, 2jp), (tg0 + 1, 2jp), (tg0, 2jp + 1), (tg0 + 1, 2jp + 1)
+                const int tg = tb / 8 + 2 * h + (mi & 1), rg = 2 * jp + (mi >> 1);
+                const uint32_t addr = (tg < tg8 && rg < nrv) ? vb + tg * vtg + rg * vrg + mr * 16 : zline;
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_t(addr, b0, b1, b2, b3);
+                mma16816(vacc[2 * jp], pa[h], b0, b1);
+                mma16816(vacc[2 * jp + 1], pa[h], b2, b3);
             }
         }
     };
+    // f(integral_constant<int, v>) for v the least of 1, 2, 4, 8 that is >= n
+    // (at most N): few variants, so that the instruction cache holds them
+    auto dispatch = [&](auto nc, int n, auto &&f) {
+        using std::integral_constant;
+        constexpr int N = decltype(nc)::value;
+        static_assert(N == 4 || N == 8, "4 or 8 cases");
+        if (n <= 1) {
+            f(integral_constant<int, 1>{});
+        } else if (n <= 2) {
+            f(integral_constant<int, 2>{});
+        } else if (n <= 4 || N == 4) {
+            f(integral_constant<int, 4>{});
+        } else {
+            f(integral_constant<int, N>{});
+        }
+    };
+    auto by_r16 = [&](int r, auto &&f) { dispatch(std::integral_constant<int, NT / 2>{}, r, f); };
 
     const int64_t rec_idx = is_tail      ? p.tail_rec_base + ((int)blockIdx.x - p.num_chunks)
                             : ch.nch == 1 ? (int64_t)p.num_chunks + ch.erec  // the entry record itself
@@ -473,7 +490,8 @@ __global__ void __launch_bounds__(32)
         }
 #pragma unroll 1
         for (int tb = 0; tb < ntok; tb += kTile)
-            tile(smem_u32(smem), 128, kBox, smem_u32(smem) + kHalf, 128, kBox, tb, kTailTokens / 8, ntok);
+            tile(std::integral_constant<int, NT / 2>{}, smem_u32(smem), 128, kBox, smem_u32(smem) + kHalf, 128, kBox,
+                 tb, kTailTokens / 8, ntok);
         // the values are already in the head dimension: o = v~
         l_w = quad_sum(l_w);
 #pragma unroll
@@ -488,9 +506,24 @@ __global__ void __launch_bounds__(32)
         return;
     }
 
-    // q rows of KV head g as projection A fragments (rows 0-7; rows 8-15 zero)
-    uint32_t qa[KD][2];
+    const int np = ps.total();
+    const int r16 = (max(nrk, nrv) + 1) / 2;
+    // wait for piece k; afterwards release its slot and bring piece k + 2 into it
+    auto wait_piece = [&](int k) {
+        mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
+        return smem_u32(smem) + (k & 1) * kPieceBytes;
+    };
+    auto release_piece = [&](int k) {
+        // the slot's reads are ordered before the async-proxy write
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0 && k + 2 < np) issue(k + 2);
+    };
+    // P^K pieces (three loops over the piece kinds keep each kind's registers
+    // local to its loop)
     {
+        // q rows of KV head g as the projection's B fragments (q^T)
+        uint32_t qa[KD][2];
         const bool row_ok = r4 < p.rows_g;
         const uint16_t *qr = p.q + ((int64_t)(r4 / p.G) * p.hq + g * p.G + r4 % p.G) * D + 2 * c4;
 #pragma unroll
@@ -498,83 +531,91 @@ __global__ void __launch_bounds__(32)
             qa[ks][0] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks) : 0u;
             qa[ks][1] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks + 8) : 0u;
         }
+#pragma unroll 1
+        for (int k = 0; k < ps.npk; ++k) {
+            const uint32_t slot = wait_piece(k);
+            // q~ for the 16-rank steps of rank groups [r0, r1): A = P^K (16 ranks x
+            // 16 columns, cores (rg - r0, cg) of this piece), B = q^T, so that one
+            // product covers 16 ranks; the accumulator [rank][row] is split into
+            // bf16 hi + lo and transposed (movmatrix) into the score A layout.
+            const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, nrk);
+            dispatch(std::integral_constant<int, L::kRanksPerPiece / 16>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
+                constexpr int NK = decltype(nkc)::value;
+                float acc[NK][2][4];
+#pragma unroll
+                for (int j = 0; j < NK; ++j)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) acc[j][0][e] = acc[j][1][e] = 0.f;
+#pragma unroll
+                for (int ks = 0; ks < KD; ++ks) {
+#pragma unroll
+                    for (int j = 0; j < NK; ++j) {
+                        // matrices: (2j, 2ks), (2j + 1, 2ks), (2j, 2ks + 1), (2j + 1, 2ks + 1)
+                        const int rl = 2 * j + (mi & 1);
+                        const uint32_t addr =
+                            r0 + rl < r1 ? slot + (rl * NT + 2 * ks + (mi >> 1)) * 128 + mr * 16 : zline;
+                        uint32_t a[4];
+                        ldsm_x4(addr, a[0], a[1], a[2], a[3]);
+                        mma16816(acc[j][ks & 1], a, qa[ks][0], qa[ks][1]);
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < NK; ++j) {
+                    // acc: ranks 16 kk + r4 (regs 0, 1) and + 8 (regs 2, 3) for rows 2 c4, 2 c4 + 1
+                    uint32_t hi0, lo0, hi1, lo1;
+                    split_hi_lo((acc[j][0][0] + acc[j][1][0]) * p.scale_log2,
+                                (acc[j][0][1] + acc[j][1][1]) * p.scale_log2, hi0, lo0);
+                    split_hi_lo((acc[j][0][2] + acc[j][1][2]) * p.scale_log2,
+                                (acc[j][0][3] + acc[j][1][3]) * p.scale_log2, hi1, lo1);
+                    sq[(r0 / 2 + j) * 32 + lane] = make_uint4(movm_t(hi0), movm_t(lo0), movm_t(hi1), movm_t(lo1));
+                }
+            });
+            __syncwarp();
+            release_piece(k);
+        }
+    }
+#pragma unroll 1
+    for (int k = ps.npk; k < ps.npk + ps.nc; ++k) {
+        const uint32_t slot = wait_piece(k);
+        const int t0 = (k - ps.npk) * ps.tpp * kTile;
+        const int nv = min(ps.tpp * kTile, ntok - t0);  // valid tokens of this piece
+        const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;
+        const uint32_t vb = slot + (uint32_t)r8 * nrk * 16;
+        by_r16(r16, [&](auto r16c) {
+#pragma unroll 1
+            for (int tb = 0; tb < nv; tb += kTile)
+                tile(r16c, slot, nrk * 128, 128, vb, nrv * 128, 128, tb, r8 / 8, nv);
+        });
+        release_piece(k);
     }
     float o[NT][4];
 #pragma unroll
     for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
-    const int np = ps.total();
 #pragma unroll 1
-    for (int k = 0; k < np; ++k) {
-        mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
-        const uint32_t slot = smem_u32(smem) + (k & 1) * kPieceBytes;
-        if (k < ps.npk) {
-            // projection of rank 8-tiles [r0, r1): cores (nt - r0, cg) of this piece
-            const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, nrk);
-#pragma unroll 1
-            for (int nt = r0; nt < r1; nt += 2) {
-                float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    for (int k = ps.npk + ps.nc; k < np; ++k) {
+        const uint32_t slot = wait_piece(k);
+        // back-projection over rank 8-groups [r0, r1): 16-rank k-steps of v~
+        const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, nrv);
 #pragma unroll
-                for (int ks = 0; ks < KD; ks += 2) {
-                    const uint32_t a0[4] = {qa[ks][0], 0u, qa[ks][1], 0u};
-                    const uint32_t a1[4] = {qa[ks + 1][0], 0u, qa[ks + 1][1], 0u};
+        for (int ks = 0; ks < NT / 2; ++ks) {
+            if (2 * ks >= r0 && 2 * ks < r1) {
+                uint32_t a[4];
+                split_hi_lo(vacc[2 * ks][0] + vacc[2 * ks][2], vacc[2 * ks][1] + vacc[2 * ks][3], a[0], a[1]);
+                split_hi_lo(vacc[2 * ks + 1][0] + vacc[2 * ks + 1][2], vacc[2 * ks + 1][1] + vacc[2 * ks + 1][3],
+                            a[2], a[3]);
 #pragma unroll
-                    for (int j = 0; j < 2; ++j) {
-                        if (nt + j < r1) {
-                            // matrices: cores (nt + j, 2ks .. 2ks + 3) -> b0, b1 of k-steps ks, ks + 1
-                            uint32_t b0, b1, b2, b3;
-                            ldsm_x4(slot + ((nt + j - r0) * NT + 2 * ks + mi) * 128 + mr * 16, b0, b1, b2, b3);
-                            mma16816(acc[j], a0, b0, b1);
-                            mma16816(acc[j], a1, b2, b3);
-                        }
-                    }
-                }
-#pragma unroll
-                for (int j = 0; j < 2; ++j) {
-                    if (nt + j < r1) {
-                        uint32_t hi, lo;
-                        split_hi_lo(acc[j][0] * p.scale_log2, acc[j][1] * p.scale_log2, hi, lo);
-                        uint32_t *f = reinterpret_cast<uint32_t *>(&sq[((nt + j) / 2) * 32 + lane]);
-                        f[((nt + j) & 1) * 2] = hi;
-                        f[((nt + j) & 1) * 2 + 1] = lo;
-                    }
-                }
-            }
-            __syncwarp();
-        } else if (k < ps.npk + ps.nc) {
-            const int t0 = (k - ps.npk) * ps.tpp * kTile;
-            const int nv = min(ps.tpp * kTile, ntok - t0);  // valid tokens of this piece
-            const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;
-            const uint32_t vb = slot + (uint32_t)r8 * nrk * 16;
-#pragma unroll 1
-            for (int tb = 0; tb < nv; tb += kTile) tile(slot, nrk * 128, 128, vb, nrv * 128, 128, tb, r8 / 8, nv);
-        } else {
-            // back-projection over rank 8-groups [r0, r1): 16-rank k-steps of v~
-            const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, nrv);
-#pragma unroll
-            for (int ks = 0; ks < NT / 2; ++ks) {
-                if (2 * ks >= r0 && 2 * ks < r1) {
-                    uint32_t a[4];
-                    split_hi_lo(vacc[2 * ks][0] + vacc[2 * ks][2], vacc[2 * ks][1] + vacc[2 * ks][3], a[0], a[1]);
-                    split_hi_lo(vacc[2 * ks + 1][0] + vacc[2 * ks + 1][2], vacc[2 * ks + 1][1] + vacc[2 * ks + 1][3],
-                                a[2], a[3]);
-#pragma unroll
-                    for (int cp = 0; cp < NT / 2; ++cp) {
-                        // matrices (transposed): (2ks, 2cp), (2ks + 1, 2cp), (2ks, 2cp + 1), (2ks + 1, 2cp + 1)
-                        const int jg = 2 * ks + (mi & 1), cg = 2 * cp + (mi >> 1);
-                        const uint32_t addr = jg < r1 ? slot + ((jg - r0) * NT + cg) * 128 + mr * 16 : zline;
-                        uint32_t b0, b1, b2, b3;
-                        ldsm_x4_t(addr, b0, b1, b2, b3);
-                        mma16816(o[2 * cp], a, b0, b1);
-                        mma16816(o[2 * cp + 1], a, b2, b3);
-                    }
+                for (int cp = 0; cp < NT / 2; ++cp) {
+                    // matrices (transposed): (2ks, 2cp), (2ks + 1, 2cp), (2ks, 2cp + 1), (2ks + 1, 2cp + 1)
+                    const int jg = 2 * ks + (mi & 1), cg = 2 * cp + (mi >> 1);
+                    const uint32_t addr = jg < r1 ? slot + ((jg - r0) * NT + cg) * 128 + mr * 16 : zline;
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4_t(addr, b0, b1, b2, b3);
+                    mma16816(o[2 * cp], a, b0, b1);
+                    mma16816(o[2 * cp + 1], a, b2, b3);
                 }
             }
         }
-        // the slot is free again (its reads ordered before the async-proxy
-        // write): bring piece k + 2 into it
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        __syncwarp();
-        if (lane == 0 && k + 2 < np) issue(k + 2);
+        release_piece(k);
     }
     l_w = quad_sum(l_w);
 #pragma unroll

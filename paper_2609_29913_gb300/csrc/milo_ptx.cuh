@@ -146,6 +146,15 @@ __device__ __forceinline__ void split_hi_lo(float x0, float x1, uint32_t &hi, ui
     lo = *reinterpret_cast<const uint32_t *>(&l);
 }
 
+// Transpose of an 8x8 b16 matrix held one row pair per lane (the mma
+// accumulator / A-fragment layout): lane l gets row l / 4, columns 2 (l % 4) ..
+__device__ __forceinline__ uint32_t movm_t(uint32_t x)
+{
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+
 __device__ __forceinline__ float quad_max(float v)
 {
     v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
