@@ -77,191 +77,148 @@ __device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
     return s;
 }
 
-constexpr int kMergeWarpsPerHead = 32;  // 8 rows x 4 quarters of the head dimension
+// The per-KV-head merge.  Every chunk and tail item ends with (o, m, l) per
+// query row: o = sum 2^(s - m) v over its tokens, l = sum 2^(s - m) (Eq. 1 on
+// a partition of the tokens).  Rather than storing these and merging them
+// afterwards, each item adds 2^(m - M) o and 2^(m - M) l into fp32
+// accumulators of its KV head with vector reductions, for one reference M per
+// row: the first item to finish a tile sets M = its running maximum +
+// kRefMargin (compare-and-swap), and every other item reads it back.  With M
+// within kDirectMax below an item's maximum nothing overflows; an item whose
+// maximum lies further above M (a rare outlier) writes its record instead and
+// lists it.  The item that brings the count of its KV head to the total
+// divides the accumulators by the sum, folds in the listed records by the
+// log-sum-exp rule, writes the output and clears the accumulators.
+constexpr float kRefMargin = 40.f;  // M = first tile maximum + this
+constexpr float kDirectMax = 60.f;  // items with m - M above this keep a record
 
-// This block's record is written: count it for KV head g (lane 0 after a fence).
-__device__ __forceinline__ void count_record(const DecodeParams &p, int g, int lane)
-{
-    __threadfence();
-    __syncwarp();
-    if (lane == 0) atomicAdd(&p.head_cnt[g], 1u);
-}
+// A reference maximum is stored as its float bits with the sign flipped, so
+// that 0 means "not set" (x + kRefMargin is never -0).
+__device__ __forceinline__ uint32_t ref_enc(float x) { return __float_as_uint(x) ^ 0x80000000u; }
+__device__ __forceinline__ float ref_dec(uint32_t u) { return __uint_as_float(u ^ 0x80000000u); }
 
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t *ptr)
+// Lane c4 == 0 of each valid row sets or reads the row's reference; the
+// result arrives later (it is used only at the end of the item).
+__device__ __forceinline__ uint32_t publish_ref(const DecodeParams &p, int g, int arow, bool row_ok, int c4, float m)
 {
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
-    return v;
-}
-
-// The last chunk of a prefix entry: merge the entry's nch chunk records
-// (c0 ...) into its entry record.  Lane l: row l / 4, quarter l % 4.
-template <int D>
-__device__ void merge_entry(const DecodeParams &p, int c0, int nch, float *dst, int lane)
-{
-    constexpr int kF4 = D / 16;
-    constexpr int kLoads = 4;
-    const int recf = 8 * D + kRecFloatsExtra;
-    const int row = lane >> 2, qq = lane & 3;
-    float M = -INFINITY, Lsum = 0.f;
-    float4 acc[kF4];
-#pragma unroll
-    for (int f = 0; f < kF4; ++f) acc[f] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s0 = 0; s0 < nch; s0 += kLoads) {
-        float mm[kLoads], ll[kLoads];
-        float4 oo[kLoads][kF4];
-#pragma unroll
-        for (int j = 0; j < kLoads; ++j) {
-            mm[j] = -INFINITY;
-            ll[j] = 0.f;
-#pragma unroll
-            for (int f = 0; f < kF4; ++f) oo[j][f] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (s0 + j < nch) {
-                const float *r = p.rec + (int64_t)(c0 + s0 + j) * recf;
-                mm[j] = __ldcg(r + 8 * D + row);
-                ll[j] = __ldcg(r + 8 * D + 8 + row);
-#pragma unroll
-                for (int f = 0; f < kF4; ++f)
-                    oo[j][f] = __ldcg(reinterpret_cast<const float4 *>(r + row * D + qq * (D / 4)) + f);
-            }
-        }
-        float Mc = M;
-#pragma unroll
-        for (int j = 0; j < kLoads; ++j) Mc = fmaxf(Mc, mm[j]);
-        const float a = exp2_diff(M, Mc);
-        Lsum *= a;
-#pragma unroll
-        for (int f = 0; f < kF4; ++f) {
-            acc[f].x *= a; acc[f].y *= a; acc[f].z *= a; acc[f].w *= a;
-        }
-#pragma unroll
-        for (int j = 0; j < kLoads; ++j) {
-            const float w = exp2_diff(mm[j], Mc);
-            Lsum += w * ll[j];
-#pragma unroll
-            for (int f = 0; f < kF4; ++f) {
-                acc[f].x += w * oo[j][f].x; acc[f].y += w * oo[j][f].y;
-                acc[f].z += w * oo[j][f].z; acc[f].w += w * oo[j][f].w;
-            }
-        }
-        M = Mc;
+    uint32_t got = 0u;
+    if (c4 == 0 && row_ok) {
+        const uint32_t mine = ref_enc(m + kRefMargin);
+        const uint32_t old = atomicCAS(p.acc_m + g * 8 + arow, 0u, mine);
+        got = old ? old : mine;
     }
-#pragma unroll
-    for (int f = 0; f < kF4; ++f) __stcg(reinterpret_cast<float4 *>(dst + row * D + qq * (D / 4)) + f, acc[f]);
-    if (qq == 0) {
-        __stcg(dst + 8 * D + row, M);
-        __stcg(dst + 8 * D + 8 + row, Lsum);
-    }
+    return got;
 }
 
-// One merge warp: KV head g, row k of the row group, quarter qq of the head
-// dimension.  Lane l takes records l, l + 32, ...; the 32 partial merges meet
-// through a shuffle butterfly.
+// The last item of KV head g: fold the listed records into the accumulators,
+// write the output rows, clear the accumulators.  Lane l: row l / 4, quarter
+// l % 4 of the head dimension.
 template <int D>
-__device__ void merge_warp(const DecodeParams &p, int mb, int lane)
+__device__ void finish_head(const DecodeParams &p, int g, int list_base, int lane)
 {
     constexpr int kF4 = D / 16;  // float4 columns per quarter
-    constexpr int kChunkLoads = 4;
-    const int g = mb / kMergeWarpsPerHead, k = (mb / 4) % 8, qq = mb % 4;
     const int recf = 8 * D + kRecFloatsExtra;
-    const int gs0 = p.g_entry_begin[g], nprefix = p.g_entry_begin[g + 1] - gs0;
-    const int S = p.tail_splits, nsrc = nprefix + p.batch * S;
-    pdl_wait();  // the output belongs to the preceding grids until here
-    // every record of KV head g: its chunks and the tail items of every query
-    if (lane == 0) {
-        const uint64_t t0 = globaltimer();
-        while (ld_acquire(&p.head_cnt[g]) < (uint32_t)nsrc) {
-            __nanosleep(200);
-            if (globaltimer() - t0 > kTimeoutNs) {
-                atomicCAS(p.status, 0, (int32_t)MILO_ERR_TIMEOUT);
-                break;
-            }
+    const int row = lane >> 2, qq = lane & 3;
+    const int64_t ai = (int64_t)g * 8 + row;
+    float4 *Oq = reinterpret_cast<float4 *>(p.acc_o + ai * D + qq * (D / 4));
+    const uint32_t mb = __ldcg(p.acc_m + ai);
+    float M = mb ? ref_dec(mb) : -INFINITY;
+    float Lsum = __ldcg(p.acc_l + ai);
+    float4 acc[kF4];
+#pragma unroll
+    for (int f = 0; f < kF4; ++f) acc[f] = __ldcg(Oq + f);
+    const uint32_t nov = __ldcg(p.ovf_cnt + g);
+#pragma unroll 1
+    for (uint32_t k = 0; k < nov; ++k) {
+        const int4 e = __ldcg(reinterpret_cast<const int4 *>(p.ovf_list) + list_base + k);
+        const int rr = row - e.y;  // this row's row in the record
+        if (rr < 0 || rr >= e.z) continue;
+        const float *r = p.rec + (int64_t)e.x * recf;
+        const float mr = __ldcg(r + 8 * D + rr), lr = __ldcg(r + 8 * D + 8 + rr);
+        const float Mn = fmaxf(M, mr);
+        const float a = exp2_diff(M, Mn), b = exp2_diff(mr, Mn);
+        Lsum = Lsum * a + lr * b;
+#pragma unroll
+        for (int f = 0; f < kF4; ++f) {
+            const float4 o = __ldcg(reinterpret_cast<const float4 *>(r + rr * D + qq * (D / 4)) + f);
+            acc[f] = make_float4(acc[f].x * a + o.x * b, acc[f].y * a + o.y * b, acc[f].z * a + o.z * b,
+                                 acc[f].w * a + o.w * b);
         }
+        M = Mn;
     }
-    __syncwarp();
-    const bool row_ok = k < p.rows_g;
-    if (row_ok) {
-        const int i = k / p.G, hh = k % p.G;
-        const float *tail0 = p.rec + (p.tail_rec_base + (int64_t)(i * p.hkv + g) * S) * recf;
-        const int ns = nprefix + S;  // this row: the prefix chunks and query i's tail splits
-        float M = -INFINITY, Lsum = 0.f;
-        float4 acc[kF4];
-#pragma unroll
-        for (int j = 0; j < kF4; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int s0 = lane; s0 < ns; s0 += 32 * kChunkLoads) {
-            float mm[kChunkLoads], ll[kChunkLoads];
-            float4 oo[kChunkLoads][kF4];
-#pragma unroll
-            for (int j = 0; j < kChunkLoads; ++j) {
-                const int s = s0 + 32 * j;
-                mm[j] = -INFINITY;
-                ll[j] = 0.f;
-#pragma unroll
-                for (int f = 0; f < kF4; ++f) oo[j][f] = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (s < ns) {
-                    const bool pre = s < nprefix;
-                    const int row = pre ? k : hh;
-                    const float *r = pre ? p.rec + (int64_t)(gs0 + s) * recf : tail0 + (int64_t)(s - nprefix) * recf;
-                    mm[j] = __ldcg(r + 8 * D + row);
-                    ll[j] = __ldcg(r + 8 * D + 8 + row);
-#pragma unroll
-                    for (int f = 0; f < kF4; ++f)
-                        oo[j][f] = __ldcg(reinterpret_cast<const float4 *>(r + row * D + qq * (D / 4)) + f);
-                }
-            }
-            float Mc = M;
-#pragma unroll
-            for (int j = 0; j < kChunkLoads; ++j) Mc = fmaxf(Mc, mm[j]);
-            const float a = exp2_diff(M, Mc);
-            Lsum *= a;
-#pragma unroll
-            for (int f = 0; f < kF4; ++f) {
-                acc[f].x *= a; acc[f].y *= a; acc[f].z *= a; acc[f].w *= a;
-            }
-#pragma unroll
-            for (int j = 0; j < kChunkLoads; ++j) {
-                const float w = exp2_diff(mm[j], Mc);
-                Lsum += w * ll[j];
-#pragma unroll
-                for (int f = 0; f < kF4; ++f) {
-                    acc[f].x += w * oo[j][f].x; acc[f].y += w * oo[j][f].y;
-                    acc[f].z += w * oo[j][f].z; acc[f].w += w * oo[j][f].w;
-                }
-            }
-            M = Mc;
-        }
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            const float Mo = __shfl_xor_sync(0xffffffffu, M, off);
-            const float Lo = __shfl_xor_sync(0xffffffffu, Lsum, off);
-            const float Mn = fmaxf(M, Mo);
-            const float a = exp2_diff(M, Mn), b = exp2_diff(Mo, Mn);
-            Lsum = Lsum * a + Lo * b;
-#pragma unroll
-            for (int f = 0; f < kF4; ++f) {
-                const float4 o2 = make_float4(__shfl_xor_sync(0xffffffffu, acc[f].x, off),
-                                              __shfl_xor_sync(0xffffffffu, acc[f].y, off),
-                                              __shfl_xor_sync(0xffffffffu, acc[f].z, off),
-                                              __shfl_xor_sync(0xffffffffu, acc[f].w, off));
-                acc[f] = make_float4(acc[f].x * a + o2.x * b, acc[f].y * a + o2.y * b, acc[f].z * a + o2.z * b,
-                                     acc[f].w * a + o2.w * b);
-            }
-            M = Mn;
-        }
+    if (row < p.rows_g) {
         const float inv = 1.f / Lsum;
-        float *dst = p.out + ((int64_t)i * p.hq + g * p.G + hh) * D + qq * (D / 4);
+        const int i = row / p.G, hh = row % p.G;
+        float4 *dst = reinterpret_cast<float4 *>(p.out + ((int64_t)i * p.hq + g * p.G + hh) * D + qq * (D / 4));
 #pragma unroll
         for (int f = 0; f < kF4; ++f)
-            if (lane == f)
-                reinterpret_cast<float4 *>(dst)[f] =
-                    make_float4(acc[f].x * inv, acc[f].y * inv, acc[f].z * inv, acc[f].w * inv);
+            dst[f] = make_float4(acc[f].x * inv, acc[f].y * inv, acc[f].z * inv, acc[f].w * inv);
     }
-    // the last merge warp of KV head g resets its counters for the next call
-    __syncwarp();
-    if (lane == 0 && atomicAdd(&p.head_cnt[p.hkv + g], 1u) == kMergeWarpsPerHead - 1) {
-        p.head_cnt[g] = 0u;
-        p.head_cnt[p.hkv + g] = 0u;
+    // clear for the next call
+#pragma unroll
+    for (int f = 0; f < kF4; ++f) __stcg(Oq + f, make_float4(0.f, 0.f, 0.f, 0.f));
+    if (qq == 0) {
+        __stcg(p.acc_l + ai, 0.f);
+        __stcg(p.acc_m + ai, 0u);
+    }
+    if (lane == 0) {
+        __stcg(p.ovf_cnt + g, 0u);
+        __stcg(p.head_cnt + g, 0u);
+    }
+}
+
+// An item's contribution to KV head g (rows arow = row0 + r4 of the head's
+// row group for r4 < nrows; ov = o of row r4 at columns 8n + 2 c4, + 1) and
+// its count; the item that completes the count finishes the head.
+template <int D>
+__device__ void contribute(const DecodeParams &p, int g, int lane, const float (&ov)[D / 8][2], float m_w,
+                           float l_r, uint32_t ref_lane0, int row0, int nrows, int64_t rec_idx)
+{
+    constexpr int NT = D / 8;
+    const int r4 = lane >> 2, c4 = lane & 3;
+    const int S = p.tail_splits;
+    const int list_base = p.g_slot_begin[g] + g * p.batch * S;
+    const bool row_ok = r4 < nrows;
+    const uint32_t rb = __shfl_sync(0xffffffffu, ref_lane0, lane & ~3);
+    const float M = rb ? ref_dec(rb) : m_w;  // unset only when the row saw no token
+    const bool direct = !row_ok || !(m_w - M > kDirectMax);
+    if (__all_sync(0xffffffffu, direct)) {
+        if (row_ok && m_w != -INFINITY) {
+            const float f = ex2_approx(m_w - M);
+            float *orow = p.acc_o + ((int64_t)g * 8 + row0 + r4) * D + 2 * c4;
+#pragma unroll
+            for (int n = 0; n < NT; ++n)
+                atomicAdd(reinterpret_cast<float2 *>(orow + 8 * n), make_float2(f * ov[n][0], f * ov[n][1]));
+            if (c4 == 0) atomicAdd(p.acc_l + g * 8 + row0 + r4, f * l_r);
+        }
+    } else {
+        // an outlier maximum: the whole record goes to the list
+        const int recf = 8 * D + kRecFloatsExtra;
+        float *rec = p.rec + rec_idx * recf;
+#pragma unroll
+        for (int n = 0; n < NT; ++n)
+            __stcg(reinterpret_cast<float2 *>(rec + r4 * D + 8 * n + 2 * c4), make_float2(ov[n][0], ov[n][1]));
+        if (c4 == 0) {
+            __stcg(rec + 8 * D + r4, m_w);
+            __stcg(rec + 8 * D + 8 + r4, l_r);
+        }
         __threadfence();
+        __syncwarp();
+        if (lane == 0) {
+            const uint32_t k = atomicAdd(p.ovf_cnt + g, 1u);
+            __stcg(reinterpret_cast<int4 *>(p.ovf_list) + list_base + k, make_int4((int)rec_idx, row0, nrows, 0));
+        }
+    }
+    // count the item (its reductions and stores ordered before the count)
+    __threadfence();
+    __syncwarp();
+    uint32_t old = 0u;
+    if (lane == 0) old = atomicAdd(p.head_cnt + g, 1u);
+    old = __shfl_sync(0xffffffffu, old, 0);
+    const uint32_t total = (uint32_t)(p.g_slot_begin[g + 1] - p.g_slot_begin[g] + p.batch * S);
+    if (old == total - 1) {
+        __threadfence();  // every other item's contribution is visible from here
+        finish_head<D>(p, g, list_base, lane);
     }
 }
 
@@ -281,17 +238,14 @@ __global__ void __launch_bounds__(32)
     uint4 *sq = reinterpret_cast<uint4 *>(smem + L::kQ);
     const uint32_t zline = smem_u32(smem + L::kZero) + mr * 16;
     const uint32_t bar0 = smem_u32(smem + L::kBar);
-    const int recf = 8 * D + kRecFloatsExtra;
     const bool is_tail = (int)blockIdx.x >= p.num_chunks;
 
     pdl_trigger();
-    const int first_merge = p.num_chunks + (p.has_tail ? p.num_tail_items : 0);
-    if ((int)blockIdx.x >= first_merge) {
-        merge_warp<D>(p, (int)blockIdx.x - first_merge, lane);
-        return;
-    }
-    for (int i = lane; i < (L::kBar - L::kQ) / 16; i += 32)
-        reinterpret_cast<uint4 *>(smem + L::kQ)[i] = make_uint4(0u, 0u, 0u, 0u);
+    // zero the slots, q~ and the zero line: reads past a piece's data then
+    // see finite values (the copies below are ordered after these stores)
+    for (int i = lane; i < L::kBar / 16; i += 32) reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    __syncwarp();
 
     ChunkDev ch = {};
     Pieces ps = {};
@@ -345,14 +299,30 @@ __global__ void __launch_bounds__(32)
     for (int n = 0; n < NT; ++n) vacc[n][0] = vacc[n][1] = vacc[n][2] = vacc[n][3] = 0.f;
 
     // One 32-token tile at token tb of the tile data: C^K core (tg, rg) at
-    // kb + tg * ktg + rg * krg, C^V core at vb + tg * vtg + rg * vrg; tg8 token
-    // groups present, tokens < nv valid.  R16 (a compile-time constant, at
-    // least both ranks / 16) fixes the 16-rank steps, so that the body is one
-    // straight block; rank groups past a rank and token groups past the data
-    // read the zero line.
-    auto tile = [&](auto r16c, uint32_t kb, uint32_t ktg, uint32_t krg, uint32_t vb, uint32_t vtg, uint32_t vrg,
-                    int tb, int tg8, int nv) {
+    // kb + tg * ktg + rg * KRG, C^V core at vb + tg * vtg + rg * VRG; tg8 token
+    // groups present, tokens < nv valid.  R16 (at least both ranks / 16) fixes
+    // the 16-rank steps; R16, KRG and VRG are compile-time constants, so that
+    // the body is one straight block whose loads take immediate offsets.
+    // Token groups past the data read the last one (their scores are masked
+    // and their p is 0).  Rank groups past a rank read whatever follows in
+    // shared memory (finite: the slots are zeroed at start, and the furthest
+    // such read ends inside the q~ area): for scores their q~ is 0, and the
+    // rank-space values they give are never back-projected.
+    auto tile = [&](auto r16c, auto krgc, auto vrgc, uint32_t kb, uint32_t ktg, uint32_t vb, uint32_t vtg, int tb,
+                    int tg8, int nv) {
         constexpr int R16 = decltype(r16c)::value;
+        constexpr uint32_t KRG = decltype(krgc)::value, VRG = decltype(vrgc)::value;
+        // per 16-token half h: this lane's ldmatrix row address at rank step 0
+        uint32_t kh[2], vh[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            // scores, matrices (tg0, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks), (tg0 + 1, 2ks + 1)
+            const int tgk = min(tb / 8 + 2 * h + (mi >> 1), tg8 - 1);
+            kh[h] = kb + tgk * ktg + (mi & 1) * KRG + mr * 16;
+            // values (transposed), matrices (tg0, 2jp), (tg0 + 1, 2jp), (tg0, 2jp + 1), (tg0 + 1, 2jp + 1)
+            const int tgv = min(tb / 8 + 2 * h + (mi & 1), tg8 - 1);
+            vh[h] = vb + tgv * vtg + (mi >> 1) * VRG + mr * 16;
+        }
         float s4[4][4];
 #pragma unroll
         for (int n = 0; n < 4; ++n) s4[n][0] = s4[n][1] = s4[n][2] = s4[n][3] = 0.f;
@@ -362,27 +332,25 @@ __global__ void __launch_bounds__(32)
             const uint32_t qa[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                // matrices: (tg0, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks), (tg0 + 1, 2ks + 1)
-                const int tg = tb / 8 + 2 * h + (mi >> 1), rg = 2 * ks + (mi & 1);
-                const uint32_t addr = (tg < tg8 && rg < nrk) ? kb + tg * ktg + rg * krg + mr * 16 : zline;
                 uint32_t b0, b1, b2, b3;
-                ldsm_x4(addr, b0, b1, b2, b3);
+                ldsm_x4(kh[h] + 2 * ks * KRG, b0, b1, b2, b3);
                 mma16816(s4[2 * h], qa, b0, b1);
                 mma16816(s4[2 * h + 1], qa, b2, b3);
             }
         }
         // score of token tb + 8n + 2 c4 + j: hi rows + lo rows
+        const int nl = nv - tb - 2 * c4;  // this lane's tokens 8n + j are valid while 8n + j < nl
         float sv8[8];
 #pragma unroll
         for (int n = 0; n < 4; ++n) {
-            const int tok = tb + 8 * n + 2 * c4;
-            sv8[2 * n] = tok < nv ? s4[n][0] + s4[n][2] : -INFINITY;
-            sv8[2 * n + 1] = tok + 1 < nv ? s4[n][1] + s4[n][3] : -INFINITY;
+            sv8[2 * n] = 8 * n < nl ? s4[n][0] + s4[n][2] : -INFINITY;
+            sv8[2 * n + 1] = 8 * n + 1 < nl ? s4[n][1] + s4[n][3] : -INFINITY;
         }
         const float lm = fmaxf(fmaxf(fmaxf(sv8[0], sv8[1]), fmaxf(sv8[2], sv8[3])),
                                fmaxf(fmaxf(sv8[4], sv8[5]), fmaxf(sv8[6], sv8[7])));
         // lazy rescale (p stays <= 2^8): the row maximum is formed only when
-        // some score passes the reference by more than 8
+        // some score passes the reference by more than 8.  Every row has a
+        // valid score in the first tile, so m_w is finite from then on.
         if (__any_sync(0xffffffffu, lm > m_w + 8.f)) {
             const float mx = quad_max(lm);
             if (mx > m_w + 8.f) {
@@ -400,7 +368,7 @@ __global__ void __launch_bounds__(32)
         }
         float pr[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) pr[j] = exp2_diff(sv8[j], m_w);
+        for (int j = 0; j < 8; ++j) pr[j] = ex2_approx(sv8[j] - m_w);  // a masked score gives 0
         l_w += ((pr[0] + pr[1]) + (pr[2] + pr[3])) + ((pr[4] + pr[5]) + (pr[6] + pr[7]));
         // A fragments of p for the two 16-token halves (rows 0-7 hi, 8-15 lo)
         uint32_t pa[2][4];
@@ -413,11 +381,8 @@ __global__ void __launch_bounds__(32)
         for (int jp = 0; jp < R16; ++jp) {
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                // matrices (transposed): (tg0, 2jp), (tg0 + 1, 2jp), (tg0, 2jp + 1), (tg0 + 1, 2jp + 1)
-                const int tg = tb / 8 + 2 * h + (mi & 1), rg = 2 * jp + (mi >> 1);
-                const uint32_t addr = (tg < tg8 && rg < nrv) ? vb + tg * vtg + rg * vrg + mr * 16 : zline;
                 uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(addr, b0, b1, b2, b3);
+                ldsm_x4_t(vh[h] + 2 * jp * VRG, b0, b1, b2, b3);
                 mma16816(vacc[2 * jp], pa[h], b0, b1);
                 mma16816(vacc[2 * jp + 1], pa[h], b2, b3);
             }
@@ -441,10 +406,7 @@ __global__ void __launch_bounds__(32)
     };
     auto by_r16 = [&](int r, auto &&f) { dispatch(std::integral_constant<int, NT / 2>{}, r, f); };
 
-    const int64_t rec_idx = is_tail      ? p.tail_rec_base + ((int)blockIdx.x - p.num_chunks)
-                            : ch.nch == 1 ? (int64_t)p.num_chunks + ch.erec  // the entry record itself
-                                          : (int64_t)blockIdx.x;
-    float *rec = p.rec + rec_idx * recf;
+    uint32_t ref = 0u;  // this row's reference maximum (lane c4 == 0), see publish_ref
     if (is_tail) {
         // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense tail
         const int item = (int)blockIdx.x - p.num_chunks, S = p.tail_splits;
@@ -489,20 +451,20 @@ __global__ void __launch_bounds__(32)
             mbar_wait(bar0, 0, p.status);
         }
 #pragma unroll 1
-        for (int tb = 0; tb < ntok; tb += kTile)
-            tile(std::integral_constant<int, NT / 2>{}, smem_u32(smem), 128, kBox, smem_u32(smem) + kHalf, 128, kBox,
-                 tb, kTailTokens / 8, ntok);
-        // the values are already in the head dimension: o = v~
-        l_w = quad_sum(l_w);
-#pragma unroll
-        for (int n = 0; n < NT; ++n)
-            __stcg(reinterpret_cast<float2 *>(rec + r4 * D + 8 * n + 2 * c4),
-                   make_float2(vacc[n][0] + vacc[n][2], vacc[n][1] + vacc[n][3]));
-        if (c4 == 0) {
-            __stcg(rec + 8 * D + r4, ntok > 0 ? m_w : -INFINITY);
-            __stcg(rec + 8 * D + 8 + r4, ntok > 0 ? l_w : 0.f);
+        for (int tb = 0; tb < ntok; tb += kTile) {
+            tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<uint32_t, kBox>{},
+                 std::integral_constant<uint32_t, kBox>{}, smem_u32(smem), 128, smem_u32(smem) + kHalf, 128, tb,
+                 kTailTokens / 8, ntok);
+            if (tb == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
         }
-        count_record(p, g, lane);
+        // the values are already in the head dimension: o = v~
+        float ov[NT][2];
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+            ov[n][0] = vacc[n][0] + vacc[n][2];
+            ov[n][1] = vacc[n][1] + vacc[n][3];
+        }
+        contribute<D>(p, g, lane, ov, m_w, quad_sum(l_w), ref, qi * p.G, p.G, p.tail_rec_base + item);
         return;
     }
 
@@ -539,7 +501,9 @@ __global__ void __launch_bounds__(32)
             // product covers 16 ranks; the accumulator [rank][row] is split into
             // bf16 hi + lo and transposed (movmatrix) into the score A layout.
             const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, nrk);
-            dispatch(std::integral_constant<int, L::kRanksPerPiece / 16>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
+            // (a piece never holds more 16-rank steps than q~ has: ranks <= D)
+            constexpr int kNKMax = L::kRanksPerPiece / 16 < KD ? L::kRanksPerPiece / 16 : KD;
+            dispatch(std::integral_constant<int, kNKMax>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
                 constexpr int NK = decltype(nkc)::value;
                 float acc[NK][2][4];
 #pragma unroll
@@ -567,7 +531,8 @@ __global__ void __launch_bounds__(32)
                                 (acc[j][0][1] + acc[j][1][1]) * p.scale_log2, hi0, lo0);
                     split_hi_lo((acc[j][0][2] + acc[j][1][2]) * p.scale_log2,
                                 (acc[j][0][3] + acc[j][1][3]) * p.scale_log2, hi1, lo1);
-                    sq[(r0 / 2 + j) * 32 + lane] = make_uint4(movm_t(hi0), movm_t(lo0), movm_t(hi1), movm_t(lo1));
+                    if (r0 / 2 + j < KD)
+                        sq[(r0 / 2 + j) * 32 + lane] = make_uint4(movm_t(hi0), movm_t(lo0), movm_t(hi1), movm_t(lo1));
                 }
             });
             __syncwarp();
@@ -584,8 +549,10 @@ __global__ void __launch_bounds__(32)
         by_r16(r16, [&](auto r16c) {
 #pragma unroll 1
             for (int tb = 0; tb < nv; tb += kTile)
-                tile(r16c, slot, nrk * 128, 128, vb, nrv * 128, 128, tb, r8 / 8, nv);
+                tile(r16c, std::integral_constant<uint32_t, 128>{}, std::integral_constant<uint32_t, 128>{}, slot,
+                     nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
         });
+        if (k == ps.npk) ref = publish_ref(p, g, r4, r4 < p.rows_g, c4, m_w);
         release_piece(k);
     }
     float o[NT][4];
@@ -617,28 +584,13 @@ __global__ void __launch_bounds__(32)
         }
         release_piece(k);
     }
-    l_w = quad_sum(l_w);
+    float ov[NT][2];
 #pragma unroll
-    for (int n = 0; n < NT; ++n)
-        __stcg(reinterpret_cast<float2 *>(rec + r4 * D + 8 * n + 2 * c4),
-               make_float2(o[n][0] + o[n][2], o[n][1] + o[n][3]));
-    if (c4 == 0) {
-        __stcg(rec + 8 * D + r4, m_w);
-        __stcg(rec + 8 * D + 8 + r4, l_w);
+    for (int n = 0; n < NT; ++n) {
+        ov[n][0] = o[n][0] + o[n][2];
+        ov[n][1] = o[n][1] + o[n][3];
     }
-    if (ch.nch > 1) {
-        // the entry's last chunk to finish merges its chunk records
-        __threadfence();
-        __syncwarp();
-        uint32_t old = 0;
-        if (lane == 0) old = atomicAdd(&p.entry_cnt[ch.erec], 1u);
-        old = __shfl_sync(0xffffffffu, old, 0);
-        if (old != (uint32_t)ch.nch - 1) return;
-        if (lane == 0) p.entry_cnt[ch.erec] = 0u;  // ready for the next call
-        __threadfence();
-        merge_entry<D>(p, ch.c0, ch.nch, p.rec + ((int64_t)p.num_chunks + ch.erec) * recf, lane);
-    }
-    count_record(p, g, lane);
+    contribute<D>(p, g, lane, ov, m_w, quad_sum(l_w), ref, 0, p.rows_g, (int64_t)blockIdx.x);
 }
 
 }  // namespace
@@ -648,7 +600,7 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     const CUtensorMap &mk = *static_cast<const CUtensorMap *>(tmap_k);
     const CUtensorMap &mv = *static_cast<const CUtensorMap *>(tmap_v);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.num_chunks + (p.has_tail ? p.num_tail_items : 0) + p.hkv * kMergeWarpsPerHead);
+    cfg.gridDim = dim3(p.num_chunks + (p.has_tail ? p.num_tail_items : 0));
     cfg.blockDim = dim3(32);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];

@@ -185,17 +185,14 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
 // coefficient rows (C^K and C^V, rounded up to 8 tokens) fit kChunkBytes; a
 // range starts at a multiple of 32 tokens.
 void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs, std::vector<ChunkDev> &chunks,
-                  std::vector<int32_t> &g_begin, std::vector<int32_t> &g_entry)
+                  std::vector<int32_t> &g_begin)
 {
     const int H = t->num_kv_heads, nb = t->num_blocks;
     chunks.clear();
     g_begin.assign((size_t)H + 1, 0);
-    g_entry.assign((size_t)H + 1, 0);
     for (int g = 0; g < H; ++g) {
         g_begin[(size_t)g] = (int32_t)chunks.size();
-        g_entry[(size_t)g] = g * nb;
         for (int b = 0; b < nb; ++b) {
-            const int c0 = (int)chunks.size();
             const int e = b * H + g, n = t->block_len[b];
             const int rk8 = r8(t->rank_k[e]), rv8 = r8(t->rank_v[e]), n8 = r8(n);
             const int tok = std::max(32, std::min(kChunkMaxTok, kChunkBytes / ((rk8 + rv8) * 2) / 32 * 32));
@@ -211,16 +208,18 @@ void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs
                 c.nrk = rk8 / 8;
                 c.nrv = rv8 / 8;
                 c.g = g;
-                c.erec = g * nb + b;
-                c.c0 = c0;
                 chunks.push_back(c);
             }
-            for (size_t x = (size_t)c0; x < chunks.size(); ++x) chunks[x].nch = (int32_t)chunks.size() - c0;
         }
     }
     g_begin[(size_t)H] = (int32_t)chunks.size();
-    g_entry[(size_t)H] = H * nb;
 }
+
+// The plan's counter buffer: CountersDev, then for the short-block decode the
+// per-KV-head item counts [H], reference maxima [8 H], list counts [H], and at
+// a 16-byte boundary the row sums [8 H] and output accumulators [8 H d].
+size_t acc_l_offset(int H) { return (sizeof(CountersDev) + sizeof(uint32_t) * 10 * (size_t)H + 15) / 16 * 16; }
+size_t counters_bytes(int H, int d) { return acc_l_offset(H) + sizeof(float) * 8 * (size_t)H * (1 + (size_t)d); }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
@@ -254,7 +253,6 @@ struct milo_prefix {
     int32_t *g_slot_begin = nullptr;
     ChunkDev *chunks = nullptr;       // short-block decode: prefix chunks, KV-head-major
     int32_t *g_chunk_begin = nullptr; // first chunk of each KV head
-    int32_t *g_entry_begin = nullptr; // first entry record of each KV head (after the chunk records)
     int num_chunks = 0;
     CountersDev *counters = nullptr;
     int32_t *status = nullptr;
@@ -335,7 +333,6 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaFree(plan->g_slot_begin);
     cudaFree(plan->chunks);
     cudaFree(plan->g_chunk_begin);
-    cudaFree(plan->g_entry_begin);
     cudaFree(plan->counters);
     cudaFree(plan->status);
     cudaSetDevice(cur);
@@ -397,10 +394,9 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         p->logical_bytes += ((int64_t)en.n * (en.rk + en.rv) + (int64_t)(en.rk + en.rv) * d) * 2;
     }
     std::vector<ChunkDev> chunks;
-    std::vector<int32_t> g_chunk, g_entry;
-    build_chunks(table, poffs, chunks, g_chunk, g_entry);
+    std::vector<int32_t> g_chunk;
+    build_chunks(table, poffs, chunks, g_chunk);
     p->num_chunks = (int)chunks.size();
-    for (auto &x : g_entry) x += p->num_chunks;  // entry records follow the chunk records
     std::vector<SegDev> sd(segs.size());
     for (size_t i = 0; i < segs.size(); ++i) {
         sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
@@ -413,7 +409,7 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         return cuda_fail(err, what);
     };
     // + per-KV-head and per-entry counters of the short-block decode
-    const size_t cnt_bytes = sizeof(CountersDev) + sizeof(uint32_t) * (2 * (size_t)H + (size_t)E);
+    const size_t cnt_bytes = counters_bytes(H, d);
     if ((e = cudaMalloc(&p->packed, (size_t)std::max<int64_t>(p->packed_bytes, 128))) != cudaSuccess)
         return cleanup(e, "cudaMalloc packed");
     if ((e = cudaMalloc(&p->entries, sizeof(EntryDev) * std::max<size_t>(ents.size(), 1))) != cudaSuccess)
@@ -428,11 +424,6 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         return cleanup(e, "cudaMalloc chunks");
     if ((e = cudaMalloc(&p->g_chunk_begin, sizeof(int32_t) * g_chunk.size())) != cudaSuccess)
         return cleanup(e, "cudaMalloc g_chunk_begin");
-    if ((e = cudaMalloc(&p->g_entry_begin, sizeof(int32_t) * g_entry.size())) != cudaSuccess)
-        return cleanup(e, "cudaMalloc g_entry_begin");
-    if ((e = cudaMemcpyAsync(p->g_entry_begin, g_entry.data(), sizeof(int32_t) * g_entry.size(),
-                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
-        return cleanup(e, "copy g_entry_begin");
     if (!chunks.empty() && (e = cudaMemcpyAsync(p->chunks, chunks.data(), sizeof(ChunkDev) * chunks.size(),
                                                 cudaMemcpyHostToDevice, stream)) != cudaSuccess)
         return cleanup(e, "copy chunks");
@@ -493,6 +484,7 @@ namespace {
 struct CallShape {
     int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
     int64_t records;
+    int64_t list_bytes;
 };
 
 CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
@@ -506,12 +498,12 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
-    // one record per prefix chunk and one per prefix entry (one row group: the
-    // short-block decode), or one per run and row group (the persistent
-    // kernel); then the tail items
-    const int64_t prefix = c.nrg == 1 ? (int64_t)p->num_chunks + (int64_t)p->nb * p->hkv
-                                      : (int64_t)p->num_slots * c.nrg;
+    // one record per prefix chunk (one row group: the short-block decode),
+    // or one per run and row group (the persistent kernel); then the tail
+    // items.  The short-block decode also lists records (an int4 per item).
+    const int64_t prefix = c.nrg == 1 ? (int64_t)p->num_chunks : (int64_t)p->num_slots * c.nrg;
     c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
+    c.list_bytes = c.nrg == 1 ? 16 * c.records : 0;
 
     return c;
 }
@@ -523,7 +515,8 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch, int6
     if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
     if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
-    *bytes = (size_t)std::max<int64_t>(c.records, 1) * (8 * plan->d + kRecFloatsExtra) * sizeof(float);
+    *bytes = (size_t)std::max<int64_t>(c.records, 1) * (8 * plan->d + kRecFloatsExtra) * sizeof(float) +
+             (size_t)c.list_bytes;
     return MILO_OK;
 }
 
@@ -567,8 +560,16 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
 
     prm.counters = plan->counters;
     prm.head_cnt = reinterpret_cast<uint32_t *>(plan->counters + 1);
-    prm.entry_cnt = prm.head_cnt + 2 * plan->hkv;
-    prm.g_entry_begin = plan->g_entry_begin;
+    {
+        // after the head counters: reference maxima, list counts, then the
+        // 16-byte aligned sums and output accumulators
+        const int H = plan->hkv;
+        prm.acc_m = prm.head_cnt + H;
+        prm.ovf_cnt = prm.acc_m + 8 * H;
+        uint8_t *base = reinterpret_cast<uint8_t *>(plan->counters);
+        prm.acc_l = reinterpret_cast<float *>(base + acc_l_offset(H));
+        prm.acc_o = prm.acc_l + 8 * H;
+    }
     prm.status = plan->status;
     prm.batch = batch;
     prm.hq = plan->hq;
@@ -595,7 +596,10 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     if (prm.num_chunks > 0) {
         prm.g_slot_begin = plan->g_chunk_begin;
         prm.num_slots = plan->num_chunks;
-        prm.tail_rec_base = (int64_t)plan->num_chunks + (int64_t)plan->nb * plan->hkv;
+        prm.tail_rec_base = plan->num_chunks;
+        // the record list follows the records
+        prm.ovf_list = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) +
+                                                   (size_t)c.records * (8 * plan->d + kRecFloatsExtra) * sizeof(float));
     }
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)plan->d);
     prm.scale_log2 = scale * 1.4426950408889634f;

@@ -61,8 +61,7 @@ struct ChunkDev {
     int32_t ntok, tok8;         // tokens, and rows copied (rounded up to 8 within the entry)
     int32_t nrk, nrv;           // rank 8-groups of K and V
     int32_t g;                  // KV head
-    int32_t erec;               // the entry's record slot (KV-head-major entry order)
-    int32_t c0, nch;            // the entry's first chunk and its number of chunks
+    int32_t pad[3];
 };
 static_assert(sizeof(ChunkDev) == 64, "chunk descriptor size");
 
@@ -103,9 +102,12 @@ struct DecodeParams {
     const ChunkDev *chunks;         // short-block decode: the prefix chunks (KV-head-major)
     int num_chunks;                 // 0: the persistent kernels run
     const uint16_t *tail_k, *tail_v;  // bf16 [rows, Hkv, d] dense tails (or null)
-    uint32_t *head_cnt;             // [2 Hkv]: records done per KV head, merge blocks done per KV head
-    uint32_t *entry_cnt;            // [entries]: chunk records done per prefix entry
-    const int32_t *g_entry_begin;   // [Hkv + 1]: first entry record of each KV head
+    uint32_t *head_cnt;             // [Hkv]: chunks and tail items done per KV head
+    float *acc_o;                   // [Hkv][8][d]: per-row accumulators of the short-block decode
+    float *acc_l;                   // [Hkv][8]
+    uint32_t *acc_m;                // [Hkv][8]: reference maxima (sign-flipped float bits; 0 = unset)
+    uint32_t *ovf_cnt;              // [Hkv]: records listed for the final merge
+    int32_t *ovf_list;              // int4 [chunks + tail items]: listed records (workspace)
 };
 
 // Launchers implemented in the .cu files.

@@ -167,6 +167,15 @@ __device__ __forceinline__ float quad_sum(float v)
     return v + __shfl_xor_sync(0xffffffffu, v, 2);
 }
 
+// 2^x by the hardware approximation (ex2.approx.ftz: relative error ~2^-22;
+// -inf gives +0).
+__device__ __forceinline__ float ex2_approx(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // exp2(a - b) with the convention that a = -inf gives 0 (and b = -inf too).
 __device__ __forceinline__ float exp2_diff(float a, float b)
 {

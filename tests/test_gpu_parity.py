@@ -89,6 +89,29 @@ def test_peaked_softmax(env):
     compare(out.cpu().numpy(), ref, "peaked")
 
 
+def test_outlier_maximum_takes_the_record_path(env):
+    """Scores of a few late tokens 256 times larger than the rest.  Every
+    prefix chunk fixes its KV head's shared reference maximum (if it is the
+    first) from the scores of its first piece, which here are ordinary
+    (tokens 0-255 at rank 16), so the chunk holding tokens 300-309 ends with a
+    maximum hundreds above the reference whichever item set it: its result
+    must go through the listed-record merge rather than the accumulators."""
+    W = env["W"]
+    layer = W.build_layer(14, 2, 128, [1024, 512], [[16, 16], [64, 32]], batch=1, tail_lengths=[70],
+                          seed=8, device="cuda")
+    A = layer.arena
+    for e in range(2):  # block 0, both KV heads
+        r = int(layer.rank_k[e])
+        off = int(layer.off_ck[e])
+        A[off + 300 * r:off + 310 * r] *= 256.0
+    out, pre = decode(env, layer)
+    ref = env["oracle"].attention(**layer.to_numpy_bits())
+    compare(out.cpu().numpy(), ref, "outlier")
+    out2, _ = decode(env, layer, plan=pre)  # the accumulators were cleared
+    compare(out2.cpu().numpy(), ref, "outlier again")
+    pre.close()
+
+
 def test_explicit_scale(env):
     layer = env["W"].make_random_case(num_q_heads=7, num_kv_heads=1, head_dim=64,
                                       block_lens=[128, 64], rank_choices=(16, 40),
