@@ -1,37 +1,36 @@
 // milo_chunk.cu -- the split-K decode of milo_decode.cu for up to 8 query rows
-// per KV head (batch x heads of one KV head <= 8): one warp per chunk, many
-// chunks per SM, each chunk streamed through two shared-memory slots.
+// per KV head (batch x heads of one KV head <= 8): one two-warp thread block
+// per chunk, six blocks per SM, each chunk streamed through two
+// shared-memory slots that both warps read.
 //
-// A chunk is a token range of one prefix entry (block b, KV head g).  Its warp
-// walks a fixed sequence of pieces, each at most kPieceBytes and brought by
-// bulk copies into one of two slots while the warp works on the other:
+// A chunk is a token range of one prefix entry (block b, KV head g).  Its
+// block walks a fixed sequence of pieces, each at most kPieceBytes and
+// brought by bulk copies into one of two slots while the warps work on the
+// other:
 //
 //   P^K pieces   q~ = scale * log2(e) * P^K q for up to 64 ranks per piece
-//                (Eq. 3 folded into Eq. 1); q~ is kept as bf16 hi + lo rows of
-//                the score A operand.
+//                (Eq. 3 folded into Eq. 1), the 16-rank steps shared between
+//                the warps; q~ is kept as bf16 hi + lo rows of the score A
+//                operand.
 //   C pieces     whole 32-token tiles (C^K rows, then C^V rows of the same
 //                tokens): scores s = C^K q~, an online softmax with a lazily
-//                raised reference max, rank-space values v~ += C^V^T p.
+//                raised reference max, rank-space values v~ += C^V^T p.  Up
+//                to 64 ranks the warps take alternate tiles, above that the
+//                two 16-token halves of each tile; each warp keeps its own
+//                softmax state.
 //   P^V pieces   o += P^V^T v~ over up to 64 ranks per piece (Alg. 1 Stage
-//                2's back-projection), v~ taken straight from the registers.
+//                2's back-projection), after the warps' v~ are merged; each
+//                warp produces half of the head dimension.
 //
-// The chunk's record is (o, max, sum) per query row.  The last chunk block
-// of a prefix entry (a per-entry counter) merges the entry's chunk records
-// into one entry record; an entry of one chunk writes its entry record
-// directly.  Entry and tail records are counted per KV head.  A dense-tail item (one
-// query's tail split for one KV head, kTailTokens tokens) brings its K and V
-// rows with 3-D TMA boxes (8 head dimensions x kTailTokens rows each, landing
-// as cores [column group][token group]) and runs the C steps on them with
-// q~ = scale * log2(e) * q; its values are already o.  The
-// last thread blocks of the grid merge: one warp per (KV head, row, quarter
-// of the head dimension) waits (bounded) until every entry and tail record
-// of its KV head is counted, then combines them with the log-sum-exp rule (Eq. 1 over a
-// partition of the tokens) and writes the output; the last of a KV head's
-// merge blocks resets its counters for the next call.  Chunk and tail blocks
-// never wait on other blocks, and they come first in the grid.
+// A dense-tail item (one query's tail split for one KV head, kTailTokens
+// tokens) brings its K and V rows with 3-D TMA boxes (8 head dimensions x
+// kTailTokens rows each, landing as cores [column group][token group]) and
+// runs the C steps on them with q~ = scale * log2(e) * q, one tile per warp;
+// its values are already o.  Every item then adds its result into fp32
+// accumulators of its KV head (see contribute), and the item that completes a
+// KV head writes the normalised output.  No block waits on another.
 //
-// Shared-memory cores are 8 rows x 16 bytes (rows = tokens or ranks); a core
-// past the data reads a zero line, so no product meets stale memory.  Every
+// Shared-memory cores are 8 rows x 16 bytes (rows = tokens or ranks).  Every
 // wait is bounded (~2 s) and sets MILO_ERR_TIMEOUT.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -47,13 +46,15 @@ namespace {
 
 constexpr int kPieceBytes = 16384;  // one slot
 constexpr int kTile = 32;           // tokens per tile
+constexpr int kChunkThreads = 64;        // two warps per chunk
 
 template <int D>
 struct CLay {
-    static constexpr int kQ = 2 * kPieceBytes;                  // q~ A fragments [D/16][32 lanes][4]
+    static constexpr int kQ = 2 * kPieceBytes;                  // q~ (then v~) A fragments [D/16][32 lanes][4]
     static constexpr int kZero = kQ + (D / 16) * 32 * 16;       // a zero core line
     static constexpr int kBar = kZero + 128;                    // 2 mbarriers
-    static constexpr int kTotal = kBar + 16;
+    static constexpr int kX = kBar + 16;                        // warp exchange: m [2][8], l [2][8], ref [8], count
+    static constexpr int kTotal = kX + 256;
     static constexpr int kRanksPerPiece = kPieceBytes / (D * 2);  // P^K / P^V rows per piece
 };
 
@@ -167,63 +168,45 @@ __device__ void finish_head(const DecodeParams &p, int g, int list_base, int lan
     }
 }
 
-// An item's contribution to KV head g (rows arow = row0 + r4 of the head's
-// row group for r4 < nrows; ov = o of row r4 at columns 8n + 2 c4, + 1) and
-// its count; the item that completes the count finishes the head.
-template <int D>
-__device__ void contribute(const DecodeParams &p, int g, int lane, const float (&ov)[D / 8][2], float m_w,
-                           float l_r, uint32_t ref_lane0, int row0, int nrows, int64_t rec_idx)
+// This warp's share of an item's contribution to KV head g: head-dimension
+// columns 8 (n0 + n) + 2 c4, + 1 of row r4 (ov[n]), for rows arow = row0 + r4
+// with r4 < nrows.  M is the item's row maximum, lsum its row sum (used when
+// with_l), refb the row's reference (encoded; 0 = unset).  Returns whether the
+// item went to the accumulators (the same in both warps: their inputs agree);
+// otherwise the warp wrote its columns of the item's record.
+template <int D, int NC>
+__device__ bool add_part(const DecodeParams &p, int g, int lane, int n0, const float (&ov)[NC][2], float M,
+                         float lsum, uint32_t refb, bool with_l, int row0, int nrows, int64_t rec_idx)
 {
-    constexpr int NT = D / 8;
     const int r4 = lane >> 2, c4 = lane & 3;
-    const int S = p.tail_splits;
-    const int list_base = p.g_slot_begin[g] + g * p.batch * S;
     const bool row_ok = r4 < nrows;
-    const uint32_t rb = __shfl_sync(0xffffffffu, ref_lane0, lane & ~3);
-    const float M = rb ? ref_dec(rb) : m_w;  // unset only when the row saw no token
-    const bool direct = !row_ok || !(m_w - M > kDirectMax);
-    if (__all_sync(0xffffffffu, direct)) {
-        if (row_ok && m_w != -INFINITY) {
-            const float f = ex2_approx(m_w - M);
-            float *orow = p.acc_o + ((int64_t)g * 8 + row0 + r4) * D + 2 * c4;
+    const float Mref = refb ? ref_dec(refb) : M;  // unset only when the row saw no token
+    const bool direct = __all_sync(0xffffffffu, !row_ok || !(M - Mref > kDirectMax));
+    if (direct) {
+        if (row_ok && M != -INFINITY) {
+            const float f = ex2_approx(M - Mref);
+            float *orow = p.acc_o + ((int64_t)g * 8 + row0 + r4) * D + 8 * n0 + 2 * c4;
 #pragma unroll
-            for (int n = 0; n < NT; ++n)
+            for (int n = 0; n < NC; ++n)
                 atomicAdd(reinterpret_cast<float2 *>(orow + 8 * n), make_float2(f * ov[n][0], f * ov[n][1]));
-            if (c4 == 0) atomicAdd(p.acc_l + g * 8 + row0 + r4, f * l_r);
+            if (with_l && c4 == 0) atomicAdd(p.acc_l + g * 8 + row0 + r4, f * lsum);
         }
     } else {
-        // an outlier maximum: the whole record goes to the list
-        const int recf = 8 * D + kRecFloatsExtra;
-        float *rec = p.rec + rec_idx * recf;
+        // an outlier maximum: the item keeps a record for the final merge
+        float *rec = p.rec + rec_idx * (8 * D + kRecFloatsExtra);
 #pragma unroll
-        for (int n = 0; n < NT; ++n)
-            __stcg(reinterpret_cast<float2 *>(rec + r4 * D + 8 * n + 2 * c4), make_float2(ov[n][0], ov[n][1]));
-        if (c4 == 0) {
-            __stcg(rec + 8 * D + r4, m_w);
-            __stcg(rec + 8 * D + 8 + r4, l_r);
-        }
-        __threadfence();
-        __syncwarp();
-        if (lane == 0) {
-            const uint32_t k = atomicAdd(p.ovf_cnt + g, 1u);
-            __stcg(reinterpret_cast<int4 *>(p.ovf_list) + list_base + k, make_int4((int)rec_idx, row0, nrows, 0));
+        for (int n = 0; n < NC; ++n)
+            __stcg(reinterpret_cast<float2 *>(rec + r4 * D + 8 * (n0 + n) + 2 * c4), make_float2(ov[n][0], ov[n][1]));
+        if (with_l && c4 == 0) {
+            __stcg(rec + 8 * D + r4, M);
+            __stcg(rec + 8 * D + 8 + r4, lsum);
         }
     }
-    // count the item (its reductions and stores ordered before the count)
-    __threadfence();
-    __syncwarp();
-    uint32_t old = 0u;
-    if (lane == 0) old = atomicAdd(p.head_cnt + g, 1u);
-    old = __shfl_sync(0xffffffffu, old, 0);
-    const uint32_t total = (uint32_t)(p.g_slot_begin[g + 1] - p.g_slot_begin[g] + p.batch * S);
-    if (old == total - 1) {
-        __threadfence();  // every other item's contribution is visible from here
-        finish_head<D>(p, g, list_base, lane);
-    }
+    return direct;
 }
 
 template <int D>
-__global__ void __launch_bounds__(32)
+__global__ void __launch_bounds__(kChunkThreads)
     chunk_kernel(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tmap_k,
                  const __grid_constant__ CUtensorMap tmap_v)
 {
@@ -232,10 +215,14 @@ __global__ void __launch_bounds__(32)
     constexpr int KD = D / 16;  // 16-wide k-steps over the head dimension
     constexpr int NT = D / 8;   // 8-wide tiles over the head dimension (and the largest rank)
     extern __shared__ __align__(128) uint8_t smem[];
-    const int lane = threadIdx.x;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int r4 = lane >> 2, c4 = lane & 3;  // mma fragment row and column pair
     const int mi = lane >> 3, mr = lane & 7;  // ldmatrix: matrix and row this lane addresses
     uint4 *sq = reinterpret_cast<uint4 *>(smem + L::kQ);
+    float *sx_m = reinterpret_cast<float *>(smem + L::kX);       // [warp][row]
+    float *sx_l = sx_m + 16;                                     // [warp][row]
+    uint32_t *sx_ref = reinterpret_cast<uint32_t *>(sx_l + 16);  // [row]
+    uint32_t *sx_cnt = sx_ref + 8;
     const uint32_t zline = smem_u32(smem + L::kZero) + mr * 16;
     const uint32_t bar0 = smem_u32(smem + L::kBar);
     const bool is_tail = (int)blockIdx.x >= p.num_chunks;
@@ -243,9 +230,8 @@ __global__ void __launch_bounds__(32)
     pdl_trigger();
     // zero the slots, q~ and the zero line: reads past a piece's data then
     // see finite values (the copies below are ordered after these stores)
-    for (int i = lane; i < L::kBar / 16; i += 32) reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
+    for (int i = tid; i < L::kBar / 16; i += kChunkThreads) reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    __syncwarp();
 
     ChunkDev ch = {};
     Pieces ps = {};
@@ -258,7 +244,7 @@ __global__ void __launch_bounds__(32)
         nrk = ch.nrk;
         nrv = ch.nrv;
     }
-    // piece k into slot k & 1 (lane 0)
+    // piece k into slot k & 1 (thread 0)
     auto issue = [&](int k) {
         const uint32_t bar = bar0 + 8 * (k & 1), dst = smem_u32(smem) + (k & 1) * kPieceBytes;
         if (k < ps.npk) {
@@ -280,7 +266,7 @@ __global__ void __launch_bounds__(32)
             bulk_g2s(dst, p.packed + ch.pv + (int64_t)r0 * D * 16, b, bar);
         }
     };
-    if (lane == 0) {
+    if (tid == 0) {
         mbar_init(bar0, 1);
         mbar_init(bar0 + 8, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -289,8 +275,8 @@ __global__ void __launch_bounds__(32)
             if (ps.total() > 1) issue(1);
         }
     }
-    __syncwarp();
-    pdl_wait();  // q, the tails and the records belong to the preceding grids until here
+    __syncthreads();
+    pdl_wait();  // q, the tails and the accumulators belong to the preceding grids until here
 
     // the warp's online-softmax state and rank-space values
     float m_w = -INFINITY, l_w = 0.f;
@@ -298,24 +284,26 @@ __global__ void __launch_bounds__(32)
 #pragma unroll
     for (int n = 0; n < NT; ++n) vacc[n][0] = vacc[n][1] = vacc[n][2] = vacc[n][3] = 0.f;
 
-    // One 32-token tile at token tb of the tile data: C^K core (tg, rg) at
-    // kb + tg * ktg + rg * KRG, C^V core at vb + tg * vtg + rg * VRG; tg8 token
-    // groups present, tokens < nv valid.  R16 (at least both ranks / 16) fixes
-    // the 16-rank steps; R16, KRG and VRG are compile-time constants, so that
-    // the body is one straight block whose loads take immediate offsets.
-    // Token groups past the data read the last one (their scores are masked
-    // and their p is 0).  Rank groups past a rank read whatever follows in
-    // shared memory (finite: the slots are zeroed at start, and the furthest
-    // such read ends inside the q~ area): for scores their q~ is 0, and the
-    // rank-space values they give are never back-projected.
-    auto tile = [&](auto r16c, auto krgc, auto vrgc, uint32_t kb, uint32_t ktg, uint32_t vb, uint32_t vtg, int tb,
-                    int tg8, int nv) {
+    // One tile of TT (16 or 32) tokens at token tb of the tile data: C^K core
+    // (tg, rg) at kb + tg * ktg + rg * KRG, C^V core at vb + tg * vtg + rg * VRG;
+    // tg8 token groups present, tokens < nv valid, at least one of them in
+    // this tile.  R16 (at least both ranks / 16) fixes the 16-rank steps;
+    // R16, TT, KRG and VRG are compile-time constants, so that the body is one
+    // straight block whose loads take immediate offsets.  Token groups past
+    // the data read the last one (their scores are masked and their p is 0).
+    // Rank groups past a rank read whatever follows in shared memory (finite:
+    // the slots are zeroed at start, and the furthest such read ends inside
+    // the q~ area): for scores their q~ is 0, and the rank-space values they
+    // give are never back-projected.
+    auto tile = [&](auto r16c, auto ttc, auto krgc, auto vrgc, uint32_t kb, uint32_t ktg, uint32_t vb,
+                    uint32_t vtg, int tb, int tg8, int nv) {
         constexpr int R16 = decltype(r16c)::value;
+        constexpr int NH = decltype(ttc)::value / 16;  // 16-token halves
         constexpr uint32_t KRG = decltype(krgc)::value, VRG = decltype(vrgc)::value;
-        // per 16-token half h: this lane's ldmatrix row address at rank step 0
-        uint32_t kh[2], vh[2];
+        // per half h: this lane's ldmatrix row address at rank step 0
+        uint32_t kh[NH], vh[NH];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
+        for (int h = 0; h < NH; ++h) {
             // scores, matrices (tg0, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks), (tg0 + 1, 2ks + 1)
             const int tgk = min(tb / 8 + 2 * h + (mi >> 1), tg8 - 1);
             kh[h] = kb + tgk * ktg + (mi & 1) * KRG + mr * 16;
@@ -323,15 +311,15 @@ __global__ void __launch_bounds__(32)
             const int tgv = min(tb / 8 + 2 * h + (mi & 1), tg8 - 1);
             vh[h] = vb + tgv * vtg + (mi >> 1) * VRG + mr * 16;
         }
-        float s4[4][4];
+        float s4[2 * NH][4];
 #pragma unroll
-        for (int n = 0; n < 4; ++n) s4[n][0] = s4[n][1] = s4[n][2] = s4[n][3] = 0.f;
+        for (int n = 0; n < 2 * NH; ++n) s4[n][0] = s4[n][1] = s4[n][2] = s4[n][3] = 0.f;
 #pragma unroll
         for (int ks = 0; ks < R16; ++ks) {
             const uint4 q4 = sq[ks * 32 + lane];
             const uint32_t qa[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < NH; ++h) {
                 uint32_t b0, b1, b2, b3;
                 ldsm_x4(kh[h] + 2 * ks * KRG, b0, b1, b2, b3);
                 mma16816(s4[2 * h], qa, b0, b1);
@@ -340,19 +328,24 @@ __global__ void __launch_bounds__(32)
         }
         // score of token tb + 8n + 2 c4 + j: hi rows + lo rows
         const int nl = nv - tb - 2 * c4;  // this lane's tokens 8n + j are valid while 8n + j < nl
-        float sv8[8];
+        float sv[4 * NH];
 #pragma unroll
-        for (int n = 0; n < 4; ++n) {
-            sv8[2 * n] = 8 * n < nl ? s4[n][0] + s4[n][2] : -INFINITY;
-            sv8[2 * n + 1] = 8 * n + 1 < nl ? s4[n][1] + s4[n][3] : -INFINITY;
+        for (int n = 0; n < 2 * NH; ++n) {
+            sv[2 * n] = 8 * n < nl ? s4[n][0] + s4[n][2] : -INFINITY;
+            sv[2 * n + 1] = 8 * n + 1 < nl ? s4[n][1] + s4[n][3] : -INFINITY;
         }
-        const float lm = fmaxf(fmaxf(fmaxf(sv8[0], sv8[1]), fmaxf(sv8[2], sv8[3])),
-                               fmaxf(fmaxf(sv8[4], sv8[5]), fmaxf(sv8[6], sv8[7])));
+        float lm[4 * NH];
+#pragma unroll
+        for (int j = 0; j < 4 * NH; ++j) lm[j] = sv[j];
+#pragma unroll
+        for (int w = 2 * NH; w >= 1; w /= 2)
+#pragma unroll
+            for (int j = 0; j < w; ++j) lm[j] = fmaxf(lm[j], lm[j + w]);
         // lazy rescale (p stays <= 2^8): the row maximum is formed only when
         // some score passes the reference by more than 8.  Every row has a
-        // valid score in the first tile, so m_w is finite from then on.
-        if (__any_sync(0xffffffffu, lm > m_w + 8.f)) {
-            const float mx = quad_max(lm);
+        // valid score in the warp's first tile, so m_w is finite from then on.
+        if (__any_sync(0xffffffffu, lm[0] > m_w + 8.f)) {
+            const float mx = quad_max(lm[0]);
             if (mx > m_w + 8.f) {
                 const float alpha = exp2_diff(m_w, mx);
                 l_w *= alpha;
@@ -366,21 +359,28 @@ __global__ void __launch_bounds__(32)
                 m_w = mx;
             }
         }
-        float pr[8];
+        float pr[4 * NH];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) pr[j] = ex2_approx(sv8[j] - m_w);  // a masked score gives 0
-        l_w += ((pr[0] + pr[1]) + (pr[2] + pr[3])) + ((pr[4] + pr[5]) + (pr[6] + pr[7]));
-        // A fragments of p for the two 16-token halves (rows 0-7 hi, 8-15 lo)
-        uint32_t pa[2][4];
+        for (int j = 0; j < 4 * NH; ++j) pr[j] = ex2_approx(sv[j] - m_w);  // a masked score gives 0
+        float ls[4 * NH];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
+        for (int j = 0; j < 4 * NH; ++j) ls[j] = pr[j];
+#pragma unroll
+        for (int w = 2 * NH; w >= 1; w /= 2)
+#pragma unroll
+            for (int j = 0; j < w; ++j) ls[j] += ls[j + w];
+        l_w += ls[0];
+        // A fragments of p for the 16-token halves (rows 0-7 hi, 8-15 lo)
+        uint32_t pa[NH][4];
+#pragma unroll
+        for (int h = 0; h < NH; ++h) {
             split_hi_lo(pr[4 * h], pr[4 * h + 1], pa[h][0], pa[h][1]);
             split_hi_lo(pr[4 * h + 2], pr[4 * h + 3], pa[h][2], pa[h][3]);
         }
 #pragma unroll
         for (int jp = 0; jp < R16; ++jp) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < NH; ++h) {
                 uint32_t b0, b1, b2, b3;
                 ldsm_x4_t(vh[h] + 2 * jp * VRG, b0, b1, b2, b3);
                 mma16816(vacc[2 * jp], pa[h], b0, b1);
@@ -404,23 +404,50 @@ __global__ void __launch_bounds__(32)
             f(integral_constant<int, N>{});
         }
     };
-    auto by_r16 = [&](int r, auto &&f) { dispatch(std::integral_constant<int, NT / 2>{}, r, f); };
 
-    uint32_t ref = 0u;  // this row's reference maximum (lane c4 == 0), see publish_ref
+    const int np = ps.total();
+    // wait for piece k (both warps); afterwards release its slot and bring
+    // piece k + 2 into it
+    auto wait_piece = [&](int k) {
+        mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
+        return smem_u32(smem) + (k & 1) * kPieceBytes;
+    };
+    auto release_piece = [&](int k) {
+        // the slot's reads are ordered before the async-proxy write
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncthreads();
+        if (tid == 0 && k + 2 < np) issue(k + 2);
+    };
+
+    uint32_t ref = 0u;  // this row's reference maximum (warp 0, lane c4 == 0), see publish_ref
+    int qi = 0, item = 0;
     if (is_tail) {
         // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense tail
-        const int item = (int)blockIdx.x - p.num_chunks, S = p.tail_splits;
-        const int qi = item / (p.hkv * S), sp = item % S;
+        item = (int)blockIdx.x - p.num_chunks;
+        const int S = p.tail_splits;
+        qi = item / (p.hkv * S);
+        const int sp = item % S;
         g = (item / S) % p.hkv;
         const int64_t o0 = p.tail_offsets[qi], o1 = p.tail_offsets[qi + 1];
         const int T = (int)(o1 - o0);
-        if (sp == S - 1 && T > S * kTailTokens && lane == 0) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
+        if (sp == S - 1 && T > S * kTailTokens && tid == 0) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
         const int t0 = sp * kTailTokens;
         ntok = max(0, min(t0 + kTailTokens, T) - t0);
         nrk = nrv = NT;
-        // q~ = scale * log2(e) * q of the G heads of query qi, as score A fragments
+        // K then V: one box of kTailTokens rows x 8 columns per column group
+        constexpr uint32_t kBox = kTailTokens * 16, kHalf = NT * kBox;
+        if (ntok > 0 && tid == 0) {
+            mbar_arrive_tx(bar0, 2 * kHalf);
 #pragma unroll 1
-        for (int ks = 0; ks < KD; ++ks) {
+            for (int c = 0; c < NT; ++c) {
+                tma_load_3d(smem_u32(smem) + c * kBox, &tmap_k, 8 * c, g, (int)(o0 + t0), bar0);
+                tma_load_3d(smem_u32(smem) + kHalf + c * kBox, &tmap_v, 8 * c, g, (int)(o0 + t0), bar0);
+            }
+        }
+        // q~ = scale * log2(e) * q of the G heads of query qi, as score A fragments
+        // (k-steps split between the warps)
+#pragma unroll 1
+        for (int ks = warp; ks < KD; ks += 2) {
             float x[4] = {0.f, 0.f, 0.f, 0.f};
             if (r4 < p.G) {
                 const uint16_t *qr = p.q + ((int64_t)qi * p.hq + g * p.G + r4) * D + 16 * ks + 2 * c4;
@@ -436,144 +463,199 @@ __global__ void __launch_bounds__(32)
             split_hi_lo(x[2], x[3], f.z, f.w);
             sq[ks * 32 + lane] = f;
         }
-        // K then V: one box of kTailTokens rows x 8 columns per column group
-        constexpr uint32_t kBox = kTailTokens * 16, kHalf = NT * kBox;
-        if (ntok > 0) {
-            if (lane == 0) {
-                mbar_arrive_tx(bar0, 2 * kHalf);
+        __syncthreads();
+        if (ntok > 0) mbar_wait(bar0, 0, p.status);
+        // one 32-token tile per warp
+        const int tb = kTile * warp;
+        if (tb < ntok) {
+            tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTile>{},
+                 std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{}, smem_u32(smem),
+                 128, smem_u32(smem) + kHalf, 128, tb, kTailTokens / 8, ntok);
+            if (warp == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
+        }
+    } else {
+        // P^K pieces (the loops over the piece kinds keep each kind's
+        // registers local to its loop)
+        {
+            // q rows of KV head g as the projection's B fragments (q^T)
+            uint32_t qa[KD][2];
+            const bool row_ok = r4 < p.rows_g;
+            const uint16_t *qr = p.q + ((int64_t)(r4 / p.G) * p.hq + g * p.G + r4 % p.G) * D + 2 * c4;
+#pragma unroll
+            for (int ks = 0; ks < KD; ++ks) {
+                qa[ks][0] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks) : 0u;
+                qa[ks][1] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks + 8) : 0u;
+            }
 #pragma unroll 1
-                for (int c = 0; c < NT; ++c) {
-                    tma_load_3d(smem_u32(smem) + c * kBox, &tmap_k, 8 * c, g, (int)(o0 + t0), bar0);
-                    tma_load_3d(smem_u32(smem) + kHalf + c * kBox, &tmap_v, 8 * c, g, (int)(o0 + t0), bar0);
+            for (int k = 0; k < ps.npk; ++k) {
+                const uint32_t slot = wait_piece(k);
+                // q~ for the 16-rank steps j of rank groups [r0, r1), j of this
+                // warp's parity: A = P^K (16 ranks x 16 columns, cores (rg - r0,
+                // cg) of this piece), B = q^T, so that one product covers 16
+                // ranks; the accumulator [rank][row] is split into bf16 hi + lo
+                // and transposed (movmatrix) into the score A layout.
+                const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, nrk);
+                // (a piece never holds more 16-rank steps than q~ has: ranks <= D)
+                constexpr int kNKMax = L::kRanksPerPiece / 16 < KD ? L::kRanksPerPiece / 16 : KD;
+                dispatch(std::integral_constant<int, kNKMax>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
+                    constexpr int NJ = (decltype(nkc)::value + 1) / 2;  // steps per warp
+                    float acc[NJ][2][4];
+#pragma unroll
+                    for (int jj = 0; jj < NJ; ++jj)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) acc[jj][0][e] = acc[jj][1][e] = 0.f;
+#pragma unroll
+                    for (int ks = 0; ks < KD; ++ks) {
+#pragma unroll
+                        for (int jj = 0; jj < NJ; ++jj) {
+                            // matrices: (2j, 2ks), (2j + 1, 2ks), (2j, 2ks + 1), (2j + 1, 2ks + 1)
+                            const int rl = 2 * (2 * jj + warp) + (mi & 1);
+                            const uint32_t addr =
+                                r0 + rl < r1 ? slot + (rl * NT + 2 * ks + (mi >> 1)) * 128 + mr * 16 : zline;
+                            uint32_t a[4];
+                            ldsm_x4(addr, a[0], a[1], a[2], a[3]);
+                            mma16816(acc[jj][ks & 1], a, qa[ks][0], qa[ks][1]);
+                        }
+                    }
+#pragma unroll
+                    for (int jj = 0; jj < NJ; ++jj) {
+                        // acc: ranks 16 j + r4 (regs 0, 1) and + 8 (regs 2, 3) for rows 2 c4, 2 c4 + 1
+                        const int j = r0 / 2 + 2 * jj + warp;
+                        uint32_t hi0, lo0, hi1, lo1;
+                        split_hi_lo((acc[jj][0][0] + acc[jj][1][0]) * p.scale_log2,
+                                    (acc[jj][0][1] + acc[jj][1][1]) * p.scale_log2, hi0, lo0);
+                        split_hi_lo((acc[jj][0][2] + acc[jj][1][2]) * p.scale_log2,
+                                    (acc[jj][0][3] + acc[jj][1][3]) * p.scale_log2, hi1, lo1);
+                        if (2 * j < r1 && j < KD)
+                            sq[j * 32 + lane] = make_uint4(movm_t(hi0), movm_t(lo0), movm_t(hi1), movm_t(lo1));
+                    }
+                });
+                release_piece(k);
+            }
+        }
+        const int r16 = (max(nrk, nrv) + 1) / 2;
+#pragma unroll 1
+        for (int k = ps.npk; k < ps.npk + ps.nc; ++k) {
+            const uint32_t slot = wait_piece(k);
+            const int t0 = (k - ps.npk) * ps.tpp * kTile;
+            const int nv = min(ps.tpp * kTile, ntok - t0);  // valid tokens of this piece
+            const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;
+            const uint32_t vb = slot + (uint32_t)r8 * nrk * 16;
+            dispatch(std::integral_constant<int, NT / 2>{}, r16, [&](auto r16c) {
+                using std::integral_constant;
+                if constexpr (decltype(r16c)::value <= 4) {
+                    // up to 64 ranks a piece holds at least two tiles: alternate tiles
+#pragma unroll 1
+                    for (int tb = kTile * warp; tb < nv; tb += 2 * kTile)
+                        tile(r16c, integral_constant<int, kTile>{}, integral_constant<uint32_t, 128>{},
+                             integral_constant<uint32_t, 128>{}, slot, nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
+                } else {
+                    // the two 16-token halves of each tile
+#pragma unroll 1
+                    for (int tb = 16 * warp; tb < nv; tb += kTile)
+                        tile(r16c, integral_constant<int, 16>{}, integral_constant<uint32_t, 128>{},
+                             integral_constant<uint32_t, 128>{}, slot, nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
+                }
+            });
+            if (k == ps.npk && warp == 0) ref = publish_ref(p, g, r4, r4 < p.rows_g, c4, m_w);
+            release_piece(k);
+        }
+    }
+
+    // ---- merge the two warps' softmax states: M = max(m0, m1) per row
+    {
+        const float lq = quad_sum(l_w);
+        if (c4 == 0) {
+            sx_m[8 * warp + r4] = m_w;
+            sx_l[8 * warp + r4] = lq;
+            if (warp == 0) sx_ref[r4] = ref;
+        }
+    }
+    __syncthreads();
+    const float m0 = sx_m[r4], m1 = sx_m[8 + r4];
+    const float M = fmaxf(m0, m1);  // -inf only for an item without tokens
+    const float lsum = sx_l[r4] * exp2_diff(m0, M) + sx_l[8 + r4] * exp2_diff(m1, M);
+    const uint32_t refb = sx_ref[r4];
+    {
+        // v~ = 2^(m0 - M) v~0 + 2^(m1 - M) v~1, gathered in warp 0: warp 1's
+        // scaled values pass through the q~ area, half of them at a time
+        const float sc = exp2_diff(m_w, M);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            if (warp == 1) {
+#pragma unroll
+                for (int n = 0; n < NT / 2; ++n) {
+                    const float *v = vacc[half * (NT / 2) + n];
+                    reinterpret_cast<float4 *>(sq)[n * 32 + lane] = make_float4(sc * v[0], sc * v[1], sc * v[2], sc * v[3]);
                 }
             }
-            __syncwarp();
-            mbar_wait(bar0, 0, p.status);
+            __syncthreads();
+            if (warp == 0) {
+#pragma unroll
+                for (int n = 0; n < NT / 2; ++n) {
+                    float *v = vacc[half * (NT / 2) + n];
+                    const float4 o = reinterpret_cast<const float4 *>(sq)[n * 32 + lane];
+                    v[0] = sc * v[0] + o.x;
+                    v[1] = sc * v[1] + o.y;
+                    v[2] = sc * v[2] + o.z;
+                    v[3] = sc * v[3] + o.w;
+                }
+            }
+            __syncthreads();
         }
-#pragma unroll 1
-        for (int tb = 0; tb < ntok; tb += kTile) {
-            tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<uint32_t, kBox>{},
-                 std::integral_constant<uint32_t, kBox>{}, smem_u32(smem), 128, smem_u32(smem) + kHalf, 128, tb,
-                 kTailTokens / 8, ntok);
-            if (tb == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
-        }
-        // the values are already in the head dimension: o = v~
+    }
+
+    bool direct;
+    int64_t rec_idx;
+    int row0, nrows;
+    if (is_tail) {
+        // the values are already in the head dimension: o = v~ (warp 0 adds all of it)
+        rec_idx = p.tail_rec_base + item;
+        row0 = qi * p.G;
+        nrows = p.G;
         float ov[NT][2];
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
             ov[n][0] = vacc[n][0] + vacc[n][2];
             ov[n][1] = vacc[n][1] + vacc[n][3];
         }
-        contribute<D>(p, g, lane, ov, m_w, quad_sum(l_w), ref, qi * p.G, p.G, p.tail_rec_base + item);
-        return;
-    }
-
-    const int np = ps.total();
-    const int r16 = (max(nrk, nrv) + 1) / 2;
-    // wait for piece k; afterwards release its slot and bring piece k + 2 into it
-    auto wait_piece = [&](int k) {
-        mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
-        return smem_u32(smem) + (k & 1) * kPieceBytes;
-    };
-    auto release_piece = [&](int k) {
-        // the slot's reads are ordered before the async-proxy write
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        __syncwarp();
-        if (lane == 0 && k + 2 < np) issue(k + 2);
-    };
-    // P^K pieces (three loops over the piece kinds keep each kind's registers
-    // local to its loop)
-    {
-        // q rows of KV head g as the projection's B fragments (q^T)
-        uint32_t qa[KD][2];
-        const bool row_ok = r4 < p.rows_g;
-        const uint16_t *qr = p.q + ((int64_t)(r4 / p.G) * p.hq + g * p.G + r4 % p.G) * D + 2 * c4;
+        direct = warp == 0 ? add_part<D, NT>(p, g, lane, 0, ov, M, lsum, refb, true, row0, nrows, rec_idx)
+                           : __all_sync(0xffffffffu, r4 >= nrows || !(M - (refb ? ref_dec(refb) : M) > kDirectMax));
+    } else {
+        rec_idx = (int64_t)blockIdx.x;
+        row0 = 0;
+        nrows = p.rows_g;
+        // warp 0 stages the merged v~ as the back-projection's A fragments (rows
+        // 0-7 hi, 8-15 lo) in the q~ area, so that the rank loop below stays rolled
+        if (warp == 0) {
 #pragma unroll
-        for (int ks = 0; ks < KD; ++ks) {
-            qa[ks][0] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks) : 0u;
-            qa[ks][1] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks + 8) : 0u;
-        }
-#pragma unroll 1
-        for (int k = 0; k < ps.npk; ++k) {
-            const uint32_t slot = wait_piece(k);
-            // q~ for the 16-rank steps of rank groups [r0, r1): A = P^K (16 ranks x
-            // 16 columns, cores (rg - r0, cg) of this piece), B = q^T, so that one
-            // product covers 16 ranks; the accumulator [rank][row] is split into
-            // bf16 hi + lo and transposed (movmatrix) into the score A layout.
-            const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, nrk);
-            // (a piece never holds more 16-rank steps than q~ has: ranks <= D)
-            constexpr int kNKMax = L::kRanksPerPiece / 16 < KD ? L::kRanksPerPiece / 16 : KD;
-            dispatch(std::integral_constant<int, kNKMax>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
-                constexpr int NK = decltype(nkc)::value;
-                float acc[NK][2][4];
-#pragma unroll
-                for (int j = 0; j < NK; ++j)
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) acc[j][0][e] = acc[j][1][e] = 0.f;
-#pragma unroll
-                for (int ks = 0; ks < KD; ++ks) {
-#pragma unroll
-                    for (int j = 0; j < NK; ++j) {
-                        // matrices: (2j, 2ks), (2j + 1, 2ks), (2j, 2ks + 1), (2j + 1, 2ks + 1)
-                        const int rl = 2 * j + (mi & 1);
-                        const uint32_t addr =
-                            r0 + rl < r1 ? slot + (rl * NT + 2 * ks + (mi >> 1)) * 128 + mr * 16 : zline;
-                        uint32_t a[4];
-                        ldsm_x4(addr, a[0], a[1], a[2], a[3]);
-                        mma16816(acc[j][ks & 1], a, qa[ks][0], qa[ks][1]);
-                    }
-                }
-#pragma unroll
-                for (int j = 0; j < NK; ++j) {
-                    // acc: ranks 16 kk + r4 (regs 0, 1) and + 8 (regs 2, 3) for rows 2 c4, 2 c4 + 1
-                    uint32_t hi0, lo0, hi1, lo1;
-                    split_hi_lo((acc[j][0][0] + acc[j][1][0]) * p.scale_log2,
-                                (acc[j][0][1] + acc[j][1][1]) * p.scale_log2, hi0, lo0);
-                    split_hi_lo((acc[j][0][2] + acc[j][1][2]) * p.scale_log2,
-                                (acc[j][0][3] + acc[j][1][3]) * p.scale_log2, hi1, lo1);
-                    if (r0 / 2 + j < KD)
-                        sq[(r0 / 2 + j) * 32 + lane] = make_uint4(movm_t(hi0), movm_t(lo0), movm_t(hi1), movm_t(lo1));
-                }
-            });
-            __syncwarp();
-            release_piece(k);
-        }
-    }
-#pragma unroll 1
-    for (int k = ps.npk; k < ps.npk + ps.nc; ++k) {
-        const uint32_t slot = wait_piece(k);
-        const int t0 = (k - ps.npk) * ps.tpp * kTile;
-        const int nv = min(ps.tpp * kTile, ntok - t0);  // valid tokens of this piece
-        const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;
-        const uint32_t vb = slot + (uint32_t)r8 * nrk * 16;
-        by_r16(r16, [&](auto r16c) {
-#pragma unroll 1
-            for (int tb = 0; tb < nv; tb += kTile)
-                tile(r16c, std::integral_constant<uint32_t, 128>{}, std::integral_constant<uint32_t, 128>{}, slot,
-                     nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
-        });
-        if (k == ps.npk) ref = publish_ref(p, g, r4, r4 < p.rows_g, c4, m_w);
-        release_piece(k);
-    }
-    float o[NT][4];
-#pragma unroll
-    for (int n = 0; n < NT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
-#pragma unroll 1
-    for (int k = ps.npk + ps.nc; k < np; ++k) {
-        const uint32_t slot = wait_piece(k);
-        // back-projection over rank 8-groups [r0, r1): 16-rank k-steps of v~
-        const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, nrv);
-#pragma unroll
-        for (int ks = 0; ks < NT / 2; ++ks) {
-            if (2 * ks >= r0 && 2 * ks < r1) {
-                uint32_t a[4];
-                split_hi_lo(vacc[2 * ks][0] + vacc[2 * ks][2], vacc[2 * ks][1] + vacc[2 * ks][3], a[0], a[1]);
+            for (int ks = 0; ks < NT / 2; ++ks) {
+                uint4 f;
+                split_hi_lo(vacc[2 * ks][0] + vacc[2 * ks][2], vacc[2 * ks][1] + vacc[2 * ks][3], f.x, f.y);
                 split_hi_lo(vacc[2 * ks + 1][0] + vacc[2 * ks + 1][2], vacc[2 * ks + 1][1] + vacc[2 * ks + 1][3],
-                            a[2], a[3]);
+                            f.z, f.w);
+                sq[ks * 32 + lane] = f;
+            }
+        }
+        __syncthreads();
+        // back-projection: warp w produces head-dimension columns [w D / 2, (w + 1) D / 2)
+        constexpr int NO = NT / 2;  // 8-column tiles per warp
+        float o[NO][4];
 #pragma unroll
-                for (int cp = 0; cp < NT / 2; ++cp) {
-                    // matrices (transposed): (2ks, 2cp), (2ks + 1, 2cp), (2ks, 2cp + 1), (2ks + 1, 2cp + 1)
-                    const int jg = 2 * ks + (mi & 1), cg = 2 * cp + (mi >> 1);
+        for (int n = 0; n < NO; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+#pragma unroll 1
+        for (int k = ps.npk + ps.nc; k < np; ++k) {
+            const uint32_t slot = wait_piece(k);
+            // rank 8-groups [r0, r1) of this piece: 16-rank k-steps of v~
+            const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, nrv);
+#pragma unroll 1
+            for (int ks = r0 / 2; 2 * ks < r1; ++ks) {
+                const uint4 a4 = sq[ks * 32 + lane];
+                const uint32_t a[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+                for (int cp = 0; cp < NO / 2; ++cp) {
+                    // matrices (transposed): (2ks, 2c), (2ks + 1, 2c), (2ks, 2c + 1), (2ks + 1, 2c + 1)
+                    const int jg = 2 * ks + (mi & 1), cg = warp * NO + 2 * cp + (mi >> 1);
                     const uint32_t addr = jg < r1 ? slot + ((jg - r0) * NT + cg) * 128 + mr * 16 : zline;
                     uint32_t b0, b1, b2, b3;
                     ldsm_x4_t(addr, b0, b1, b2, b3);
@@ -581,16 +663,37 @@ __global__ void __launch_bounds__(32)
                     mma16816(o[2 * cp + 1], a, b2, b3);
                 }
             }
+            release_piece(k);
         }
-        release_piece(k);
-    }
-    float ov[NT][2];
+        float ov[NO][2];
 #pragma unroll
-    for (int n = 0; n < NT; ++n) {
-        ov[n][0] = o[n][0] + o[n][2];
-        ov[n][1] = o[n][1] + o[n][3];
+        for (int n = 0; n < NO; ++n) {
+            ov[n][0] = o[n][0] + o[n][2];
+            ov[n][1] = o[n][1] + o[n][3];
+        }
+        direct = add_part<D, NO>(p, g, lane, warp * NO, ov, M, lsum, refb, warp == 0, row0, nrows, rec_idx);
     }
-    contribute<D>(p, g, lane, ov, m_w, quad_sum(l_w), ref, 0, p.rows_g, (int64_t)blockIdx.x);
+
+    // ---- count the item (its reductions and stores ordered before the
+    // count); the item that completes its KV head finishes it
+    const int S = p.tail_splits;
+    const int list_base = p.g_slot_begin[g] + g * p.batch * S;
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+        if (!direct) {
+            const uint32_t k = atomicAdd(p.ovf_cnt + g, 1u);
+            __stcg(reinterpret_cast<int4 *>(p.ovf_list) + list_base + k, make_int4((int)rec_idx, row0, nrows, 0));
+            __threadfence();
+        }
+        *sx_cnt = atomicAdd(p.head_cnt + g, 1u);
+    }
+    __syncthreads();
+    const uint32_t total = (uint32_t)(p.g_slot_begin[g + 1] - p.g_slot_begin[g] + p.batch * S);
+    if (*sx_cnt == total - 1 && warp == 0) {
+        __threadfence();  // every other item's contribution is visible from here
+        finish_head<D>(p, g, list_base, lane);
+    }
 }
 
 }  // namespace
@@ -601,7 +704,7 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     const CUtensorMap &mv = *static_cast<const CUtensorMap *>(tmap_v);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(p.num_chunks + (p.has_tail ? p.num_tail_items : 0));
-    cfg.blockDim = dim3(32);
+    cfg.blockDim = dim3(kChunkThreads);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
