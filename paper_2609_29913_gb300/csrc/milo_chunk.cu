@@ -44,17 +44,18 @@
 namespace milo {
 namespace {
 
-constexpr int kPieceBytes = 16384;  // one slot
+constexpr int kPieceBytes = 32768;  // one slot
 constexpr int kTile = 32;           // tokens per tile
-constexpr int kChunkThreads = 64;        // two warps per chunk
+constexpr int kWarps = 2;           // warps per chunk block
+constexpr int kChunkThreads = 32 * kWarps;
 
 template <int D>
 struct CLay {
     static constexpr int kQ = 2 * kPieceBytes;                  // q~ (then v~) A fragments [D/16][32 lanes][4]
     static constexpr int kZero = kQ + (D / 16) * 32 * 16;       // a zero core line
     static constexpr int kBar = kZero + 128;                    // 2 mbarriers
-    static constexpr int kX = kBar + 16;                        // warp exchange: m [2][8], l [2][8], ref [8], count
-    static constexpr int kTotal = kX + 256;
+    static constexpr int kX = kBar + 16;                        // warp exchange: m, l [kWarps][8], ref [8], count
+    static constexpr int kTotal = kX + ((16 * kWarps + 9) * 4 + 15) / 16 * 16;
     static constexpr int kRanksPerPiece = kPieceBytes / (D * 2);  // P^K / P^V rows per piece
 };
 
@@ -220,8 +221,8 @@ __global__ void __launch_bounds__(kChunkThreads)
     const int mi = lane >> 3, mr = lane & 7;  // ldmatrix: matrix and row this lane addresses
     uint4 *sq = reinterpret_cast<uint4 *>(smem + L::kQ);
     float *sx_m = reinterpret_cast<float *>(smem + L::kX);       // [warp][row]
-    float *sx_l = sx_m + 16;                                     // [warp][row]
-    uint32_t *sx_ref = reinterpret_cast<uint32_t *>(sx_l + 16);  // [row]
+    float *sx_l = sx_m + 8 * kWarps;                             // [warp][row]
+    uint32_t *sx_ref = reinterpret_cast<uint32_t *>(sx_l + 8 * kWarps);  // [row]
     uint32_t *sx_cnt = sx_ref + 8;
     const uint32_t zline = smem_u32(smem + L::kZero) + mr * 16;
     const uint32_t bar0 = smem_u32(smem + L::kBar);
@@ -447,7 +448,7 @@ __global__ void __launch_bounds__(kChunkThreads)
         // q~ = scale * log2(e) * q of the G heads of query qi, as score A fragments
         // (k-steps split between the warps)
 #pragma unroll 1
-        for (int ks = warp; ks < KD; ks += 2) {
+        for (int ks = warp; ks < KD; ks += kWarps) {
             float x[4] = {0.f, 0.f, 0.f, 0.f};
             if (r4 < p.G) {
                 const uint16_t *qr = p.q + ((int64_t)qi * p.hq + g * p.G + r4) * D + 16 * ks + 2 * c4;
@@ -465,10 +466,12 @@ __global__ void __launch_bounds__(kChunkThreads)
         }
         __syncthreads();
         if (ntok > 0) mbar_wait(bar0, 0, p.status);
-        // one 32-token tile per warp
-        const int tb = kTile * warp;
+        // the item's tokens in units of kTailTokens / kWarps, one per warp
+        constexpr int kTU = kTailTokens / kWarps;
+        static_assert(kTU == 16 || kTU == 32, "tail units of 16 or 32 tokens");
+        const int tb = kTU * warp;
         if (tb < ntok) {
-            tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTile>{},
+            tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTU>{},
                  std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{}, smem_u32(smem),
                  128, smem_u32(smem) + kHalf, 128, tb, kTailTokens / 8, ntok);
             if (warp == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
@@ -498,7 +501,7 @@ __global__ void __launch_bounds__(kChunkThreads)
                 // (a piece never holds more 16-rank steps than q~ has: ranks <= D)
                 constexpr int kNKMax = L::kRanksPerPiece / 16 < KD ? L::kRanksPerPiece / 16 : KD;
                 dispatch(std::integral_constant<int, kNKMax>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
-                    constexpr int NJ = (decltype(nkc)::value + 1) / 2;  // steps per warp
+                    constexpr int NJ = (decltype(nkc)::value + kWarps - 1) / kWarps;  // steps per warp
                     float acc[NJ][2][4];
 #pragma unroll
                     for (int jj = 0; jj < NJ; ++jj)
@@ -509,7 +512,7 @@ __global__ void __launch_bounds__(kChunkThreads)
 #pragma unroll
                         for (int jj = 0; jj < NJ; ++jj) {
                             // matrices: (2j, 2ks), (2j + 1, 2ks), (2j, 2ks + 1), (2j + 1, 2ks + 1)
-                            const int rl = 2 * (2 * jj + warp) + (mi & 1);
+                            const int rl = 2 * (kWarps * jj + warp) + (mi & 1);
                             const uint32_t addr =
                                 r0 + rl < r1 ? slot + (rl * NT + 2 * ks + (mi >> 1)) * 128 + mr * 16 : zline;
                             uint32_t a[4];
@@ -520,7 +523,7 @@ __global__ void __launch_bounds__(kChunkThreads)
 #pragma unroll
                     for (int jj = 0; jj < NJ; ++jj) {
                         // acc: ranks 16 j + r4 (regs 0, 1) and + 8 (regs 2, 3) for rows 2 c4, 2 c4 + 1
-                        const int j = r0 / 2 + 2 * jj + warp;
+                        const int j = r0 / 2 + kWarps * jj + warp;
                         uint32_t hi0, lo0, hi1, lo1;
                         split_hi_lo((acc[jj][0][0] + acc[jj][1][0]) * p.scale_log2,
                                     (acc[jj][0][1] + acc[jj][1][1]) * p.scale_log2, hi0, lo0);
@@ -544,15 +547,15 @@ __global__ void __launch_bounds__(kChunkThreads)
             dispatch(std::integral_constant<int, NT / 2>{}, r16, [&](auto r16c) {
                 using std::integral_constant;
                 if constexpr (decltype(r16c)::value <= 4) {
-                    // up to 64 ranks a piece holds at least two tiles: alternate tiles
+                    // up to 64 ranks: whole tiles round-robin over the warps
 #pragma unroll 1
-                    for (int tb = kTile * warp; tb < nv; tb += 2 * kTile)
+                    for (int tb = kTile * warp; tb < nv; tb += kWarps * kTile)
                         tile(r16c, integral_constant<int, kTile>{}, integral_constant<uint32_t, 128>{},
                              integral_constant<uint32_t, 128>{}, slot, nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
                 } else {
-                    // the two 16-token halves of each tile
+                    // above: 16-token halves of the tiles round-robin over the warps
 #pragma unroll 1
-                    for (int tb = 16 * warp; tb < nv; tb += kTile)
+                    for (int tb = 16 * warp; tb < nv; tb += kWarps * 16)
                         tile(r16c, integral_constant<int, 16>{}, integral_constant<uint32_t, 128>{},
                              integral_constant<uint32_t, 128>{}, slot, nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
                 }
@@ -562,7 +565,7 @@ __global__ void __launch_bounds__(kChunkThreads)
         }
     }
 
-    // ---- merge the two warps' softmax states: M = max(m0, m1) per row
+    // ---- merge the warps' softmax states: M = max over the warps per row
     {
         const float lq = quad_sum(l_w);
         if (c4 == 0) {
@@ -572,36 +575,53 @@ __global__ void __launch_bounds__(kChunkThreads)
         }
     }
     __syncthreads();
-    const float m0 = sx_m[r4], m1 = sx_m[8 + r4];
-    const float M = fmaxf(m0, m1);  // -inf only for an item without tokens
-    const float lsum = sx_l[r4] * exp2_diff(m0, M) + sx_l[8 + r4] * exp2_diff(m1, M);
+    float M = -INFINITY;  // -inf only for an item without tokens
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, sx_m[8 * w + r4]);
+    float lsum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) lsum += sx_l[8 * w + r4] * exp2_diff(sx_m[8 * w + r4], M);
     const uint32_t refb = sx_ref[r4];
     {
-        // v~ = 2^(m0 - M) v~0 + 2^(m1 - M) v~1, gathered in warp 0: warp 1's
-        // scaled values pass through the q~ area, half of them at a time
+        // v~ = sum over warps of 2^(m_w - M) v~_w, gathered in warp 0: the
+        // other warps' scaled values pass through the q~ area in turn, half
+        // of them at a time
         const float sc = exp2_diff(m_w, M);
+        float4 *xv = reinterpret_cast<float4 *>(sq);
+        if (warp == 0) {
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            if (warp == 1) {
-#pragma unroll
-                for (int n = 0; n < NT / 2; ++n) {
-                    const float *v = vacc[half * (NT / 2) + n];
-                    reinterpret_cast<float4 *>(sq)[n * 32 + lane] = make_float4(sc * v[0], sc * v[1], sc * v[2], sc * v[3]);
-                }
+            for (int n = 0; n < NT; ++n) {
+                vacc[n][0] *= sc;
+                vacc[n][1] *= sc;
+                vacc[n][2] *= sc;
+                vacc[n][3] *= sc;
             }
-            __syncthreads();
-            if (warp == 0) {
+        }
+#pragma unroll 1
+        for (int w = 1; w < kWarps; ++w) {
 #pragma unroll
-                for (int n = 0; n < NT / 2; ++n) {
-                    float *v = vacc[half * (NT / 2) + n];
-                    const float4 o = reinterpret_cast<const float4 *>(sq)[n * 32 + lane];
-                    v[0] = sc * v[0] + o.x;
-                    v[1] = sc * v[1] + o.y;
-                    v[2] = sc * v[2] + o.z;
-                    v[3] = sc * v[3] + o.w;
+            for (int half = 0; half < 2; ++half) {
+                if (warp == w) {
+#pragma unroll
+                    for (int n = 0; n < NT / 2; ++n) {
+                        const float *v = vacc[half * (NT / 2) + n];
+                        xv[n * 32 + lane] = make_float4(sc * v[0], sc * v[1], sc * v[2], sc * v[3]);
+                    }
                 }
+                __syncthreads();
+                if (warp == 0) {
+#pragma unroll
+                    for (int n = 0; n < NT / 2; ++n) {
+                        float *v = vacc[half * (NT / 2) + n];
+                        const float4 o = xv[n * 32 + lane];
+                        v[0] += o.x;
+                        v[1] += o.y;
+                        v[2] += o.z;
+                        v[3] += o.w;
+                    }
+                }
+                __syncthreads();
             }
-            __syncthreads();
         }
     }
 
@@ -638,8 +658,9 @@ __global__ void __launch_bounds__(kChunkThreads)
             }
         }
         __syncthreads();
-        // back-projection: warp w produces head-dimension columns [w D / 2, (w + 1) D / 2)
-        constexpr int NO = NT / 2;  // 8-column tiles per warp
+        // back-projection: warp w produces head-dimension columns [w D / kWarps, (w + 1) D / kWarps)
+        constexpr int NO = NT / kWarps;  // 8-column tiles per warp
+        static_assert(NO % 2 == 0, "column pairs per warp");
         float o[NO][4];
 #pragma unroll
         for (int n = 0; n < NO; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;

@@ -54,7 +54,7 @@ struct SegDev {
 };
 
 // One chunk of the short-block decode: tokens [t0, t1) of a prefix entry.
-constexpr int kChunkBytes = 49152;   // coefficient bytes (C^K + C^V rows) per chunk
+constexpr int kChunkBytes = 131072;   // coefficient bytes (C^K + C^V rows) per chunk
 constexpr int kChunkMaxTok = 1024;   // tokens per chunk
 struct ChunkDev {
     int64_t ck, cv, pk, pv;     // byte offsets in the packed arena (C^K, C^V at the chunk's first token)
