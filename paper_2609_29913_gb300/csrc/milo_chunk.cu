@@ -1,34 +1,34 @@
 // milo_chunk.cu -- the split-K decode of milo_decode.cu for up to 8 query rows
-// per KV head (batch x heads of one KV head <= 8): one two-warp thread block
-// per chunk, six blocks per SM, each chunk streamed through two
-// shared-memory slots that both warps read.
+// per KV head (batch x heads of one KV head <= 8): one thread block of kWarps
+// warps per chunk (three blocks per SM at head dimension 128), each chunk
+// streamed through two shared-memory slots that all its warps read.
 //
 // A chunk is a token range of one prefix entry (block b, KV head g).  Its
 // block walks a fixed sequence of pieces, each at most kPieceBytes and
 // brought by bulk copies into one of two slots while the warps work on the
 // other:
 //
-//   P^K pieces   q~ = scale * log2(e) * P^K q for up to 64 ranks per piece
-//                (Eq. 3 folded into Eq. 1), the 16-rank steps shared between
-//                the warps; q~ is kept as bf16 hi + lo rows of the score A
-//                operand.
+//   P^K pieces   q~ = scale * log2(e) * P^K q for up to kPieceBytes / (2 d)
+//                ranks per piece (Eq. 3 folded into Eq. 1), the 16-rank steps
+//                dealt round-robin to the warps; q~ is kept as bf16 hi + lo
+//                rows of the score A operand.
 //   C pieces     whole 32-token tiles (C^K rows, then C^V rows of the same
 //                tokens): scores s = C^K q~, an online softmax with a lazily
 //                raised reference max, rank-space values v~ += C^V^T p.  Up
-//                to 64 ranks the warps take alternate tiles, above that the
-//                two 16-token halves of each tile; each warp keeps its own
-//                softmax state.
-//   P^V pieces   o += P^V^T v~ over up to 64 ranks per piece (Alg. 1 Stage
-//                2's back-projection), after the warps' v~ are merged; each
-//                warp produces half of the head dimension.
+//                to 64 ranks the warps take whole tiles round-robin, above
+//                that 16-token halves; each warp keeps its own softmax state.
+//   P^V pieces   o += P^V^T v~ over up to kPieceBytes / (2 d) ranks per piece
+//                (Alg. 1 Stage 2's back-projection), after the warps' v~ are
+//                merged; each warp produces a share of the head dimension.
 //
 // A dense-tail item (one query's tail split for one KV head, kTailTokens
 // tokens) brings its K and V rows with 3-D TMA boxes (8 head dimensions x
 // kTailTokens rows each, landing as cores [column group][token group]) and
-// runs the C steps on them with q~ = scale * log2(e) * q, one tile per warp;
-// its values are already o.  Every item then adds its result into fp32
-// accumulators of its KV head (see contribute), and the item that completes a
-// KV head writes the normalised output.  No block waits on another.
+// runs the C steps on them with q~ = scale * log2(e) * q, a share of the
+// tokens per warp; its values are already o.  Every item then adds its result
+// into fp32 accumulators of its KV head (see add_part), and the item that
+// completes a KV head writes the normalised output.  No block waits on
+// another.
 //
 // Shared-memory cores are 8 rows x 16 bytes (rows = tokens or ranks).  Every
 // wait is bounded (~2 s) and sets MILO_ERR_TIMEOUT.

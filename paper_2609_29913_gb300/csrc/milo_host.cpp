@@ -181,9 +181,10 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
 }
 
 // Chunks of the short-block decode: every prefix entry, KV-head-major then in
-// block order, cut into token ranges of at most kChunkMaxTok tokens whose
-// coefficient rows (C^K and C^V, rounded up to 8 tokens) fit kChunkBytes; a
-// range starts at a multiple of 32 tokens.
+// block order, cut into the fewest token ranges of at most kChunkMaxTok tokens
+// whose coefficient rows (C^K and C^V, rounded up to 8 tokens) fit
+// kChunkBytes, of about equal length; a range starts at a multiple of 32
+// tokens.
 void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs, std::vector<ChunkDev> &chunks,
                   std::vector<int32_t> &g_begin)
 {
@@ -195,7 +196,12 @@ void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs
         for (int b = 0; b < nb; ++b) {
             const int e = b * H + g, n = t->block_len[b];
             const int rk8 = r8(t->rank_k[e]), rv8 = r8(t->rank_v[e]), n8 = r8(n);
-            const int tok = std::max(32, std::min(kChunkMaxTok, kChunkBytes / ((rk8 + rv8) * 2) / 32 * 32));
+            // the fewest chunks within the byte budget, then equal token
+            // ranges (multiples of 32), so that an entry's chunks take
+            // about equally long
+            const int most = std::max(32, std::min(kChunkMaxTok, kChunkBytes / ((rk8 + rv8) * 2) / 32 * 32));
+            const int nch = std::max(1, (n + most - 1) / most);
+            const int tok = ((n + nch - 1) / nch + 31) / 32 * 32;
             for (int t0 = 0; t0 < n; t0 += tok) {
                 ChunkDev c = {};
                 const int t1 = std::min(n, t0 + tok);
