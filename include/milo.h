@@ -143,6 +143,26 @@ milo_status_t milo_partition_prefix(const milo_block_table_t *table,
                                     int32_t *num_slots);
 
 /*
+ * Host-only: the work list of the short-block decode (calls with at most 8
+ * query rows per KV head).  Every prefix entry, KV-head-major then in block
+ * order, is cut into the fewest token ranges of at most 1024 tokens whose
+ * coefficient rows (C^K and C^V at ranks rounded up to 8, tokens rounded up
+ * to 8, bf16) fit 128 KB, of equal length in multiples of 32 tokens (the
+ * last range takes the remainder); each range is one thread block of the
+ * decode grid.
+ *   chunk_entry/chunk_t0/chunk_t1: host arrays of capacity `max_chunks`
+ *     (entry index b * num_kv_heads + g, token range [t0, t1)); all may be
+ *     NULL to query the count.
+ *   num_chunks: output (may be NULL).
+ * Returns MILO_ERR_INVALID_ARG (after setting num_chunks) if max_chunks is
+ * too small, or the table's validation status.
+ */
+milo_status_t milo_chunk_prefix(const milo_block_table_t *table,
+                                int32_t max_chunks, int32_t *chunk_entry,
+                                int32_t *chunk_t0, int32_t *chunk_t1,
+                                int32_t *num_chunks);
+
+/*
  * Build a plan for one layer on the current device: validate the table,
  * allocate and fill the packed arena (a pack kernel on `stream`, then a
  * stream synchronisation), build the work partition and the device-side

@@ -184,41 +184,50 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
 // block order, cut into the fewest token ranges of at most kChunkMaxTok tokens
 // whose coefficient rows (C^K and C^V, rounded up to 8 tokens) fit
 // kChunkBytes, of about equal length; a range starts at a multiple of 32
-// tokens.
-void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs, std::vector<ChunkDev> &chunks,
-                  std::vector<int32_t> &g_begin)
+// tokens.  f(entry, KV head, t0, t1) for each range in that order.
+template <class F>
+void for_each_chunk(const milo_block_table_t *t, F &&f)
 {
     const int H = t->num_kv_heads, nb = t->num_blocks;
-    chunks.clear();
-    g_begin.assign((size_t)H + 1, 0);
     for (int g = 0; g < H; ++g) {
-        g_begin[(size_t)g] = (int32_t)chunks.size();
         for (int b = 0; b < nb; ++b) {
             const int e = b * H + g, n = t->block_len[b];
-            const int rk8 = r8(t->rank_k[e]), rv8 = r8(t->rank_v[e]), n8 = r8(n);
+            const int rk8 = r8(t->rank_k[e]), rv8 = r8(t->rank_v[e]);
             // the fewest chunks within the byte budget, then equal token
             // ranges (multiples of 32), so that an entry's chunks take
             // about equally long
             const int most = std::max(32, std::min(kChunkMaxTok, kChunkBytes / ((rk8 + rv8) * 2) / 32 * 32));
             const int nch = std::max(1, (n + most - 1) / most);
             const int tok = ((n + nch - 1) / nch + 31) / 32 * 32;
-            for (int t0 = 0; t0 < n; t0 += tok) {
-                ChunkDev c = {};
-                const int t1 = std::min(n, t0 + tok);
-                c.ck = poffs[(size_t)e * 4 + 0] + (int64_t)t0 * rk8 * 2;
-                c.pk = poffs[(size_t)e * 4 + 1];
-                c.cv = poffs[(size_t)e * 4 + 2] + (int64_t)t0 * rv8 * 2;
-                c.pv = poffs[(size_t)e * 4 + 3];
-                c.ntok = t1 - t0;
-                c.tok8 = std::min(r8(t1), n8) - t0;
-                c.nrk = rk8 / 8;
-                c.nrv = rv8 / 8;
-                c.g = g;
-                chunks.push_back(c);
-            }
+            for (int t0 = 0; t0 < n; t0 += tok) f(e, g, t0, std::min(n, t0 + tok));
         }
     }
-    g_begin[(size_t)H] = (int32_t)chunks.size();
+}
+
+void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs, std::vector<ChunkDev> &chunks,
+                  std::vector<int32_t> &g_begin)
+{
+    const int H = t->num_kv_heads;
+    chunks.clear();
+    g_begin.assign((size_t)H + 1, 0);
+    for_each_chunk(t, [&](int e, int g, int t0, int t1) {
+        const int n = t->block_len[e / H];
+        const int rk8 = r8(t->rank_k[e]), rv8 = r8(t->rank_v[e]), n8 = r8(n);
+        ChunkDev c = {};
+        c.ck = poffs[(size_t)e * 4 + 0] + (int64_t)t0 * rk8 * 2;
+        c.pk = poffs[(size_t)e * 4 + 1];
+        c.cv = poffs[(size_t)e * 4 + 2] + (int64_t)t0 * rv8 * 2;
+        c.pv = poffs[(size_t)e * 4 + 3];
+        c.ntok = t1 - t0;
+        c.tok8 = std::min(r8(t1), n8) - t0;
+        c.nrk = rk8 / 8;
+        c.nrv = rv8 / 8;
+        c.g = g;
+        chunks.push_back(c);
+        g_begin[(size_t)g + 1] = (int32_t)chunks.size();
+    });
+    // a KV head without chunks starts where the previous one ended
+    for (int g = 1; g <= H; ++g) g_begin[(size_t)g] = std::max(g_begin[(size_t)g], g_begin[(size_t)g - 1]);
 }
 
 // The plan's counter buffer: CountersDev, then for the short-block decode the
@@ -322,6 +331,29 @@ milo_status_t milo_partition_prefix(const milo_block_table_t *table, int32_t num
             if (seg_slot) seg_slot[i] = segs[i].slot;
         }
     }
+    return MILO_OK;
+}
+
+milo_status_t milo_chunk_prefix(const milo_block_table_t *table, int32_t max_chunks, int32_t *chunk_entry,
+                                int32_t *chunk_t0, int32_t *chunk_t1, int32_t *num_chunks)
+{
+    milo_status_t s = validate(table);
+    if (s != MILO_OK) return s;
+    int32_t n = 0;
+    const bool fill = chunk_entry || chunk_t0 || chunk_t1;
+    bool overflow = false;
+    for_each_chunk(table, [&](int e, int, int t0, int t1) {
+        if (fill && n < max_chunks) {
+            if (chunk_entry) chunk_entry[n] = e;
+            if (chunk_t0) chunk_t0[n] = t0;
+            if (chunk_t1) chunk_t1[n] = t1;
+        } else if (fill) {
+            overflow = true;
+        }
+        ++n;
+    });
+    if (num_chunks) *num_chunks = n;
+    if (overflow) return fail(MILO_ERR_INVALID_ARG, "max_chunks too small");
     return MILO_OK;
 }
 

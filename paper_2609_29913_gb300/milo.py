@@ -29,7 +29,7 @@ STATUS_NAMES = {0: "MILO_OK", 1: "MILO_ERR_INVALID_ARG", 2: "MILO_ERR_BAD_TABLE"
 # every symbol include/milo.h declares
 EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
-           "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
+           "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
            "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
            "milo_get_device_status"]
 
@@ -77,6 +77,7 @@ def lib():
         L.milo_validate_table.argtypes = [P]
         L.milo_packed_layout.argtypes = [P, P, P]
         L.milo_partition_prefix.argtypes = [P, i32, i32, P, P, P, P, P, P, P]
+        L.milo_chunk_prefix.argtypes = [P, i32, P, P, P, P]
         L.milo_prefix_create.argtypes = [P, i32, i32, P, P]
         L.milo_prefix_destroy.argtypes = [P]
         L.milo_prefix_get_info.argtypes = [P, P]
@@ -86,7 +87,7 @@ def lib():
         L.milo_attn_decode_static.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         for name in ("milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
-                     "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
+                     "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
                      "milo_get_device_status"):
             getattr(L, name).restype = i32
@@ -164,6 +165,19 @@ def milo_partition_prefix(table: HostTable, num_ctas: int) -> dict:
     res["cta_begin"] = cb
     res["num_slots"] = int(nslot.value)
     return res
+
+
+def milo_chunk_prefix(table: HostTable) -> dict:
+    """The short-block decode's work list: entry, t0, t1 per chunk."""
+    n = ctypes.c_int32(0)
+    L = lib()
+    _check(L.milo_chunk_prefix(ctypes.byref(table.c), 0, None, None, None, ctypes.byref(n)),
+           "milo_chunk_prefix")
+    k = int(n.value)
+    out = {key: np.zeros(max(k, 1), dtype=np.int32) for key in ("entry", "t0", "t1")}
+    _check(L.milo_chunk_prefix(ctypes.byref(table.c), k, out["entry"].ctypes.data, out["t0"].ctypes.data,
+                               out["t1"].ctypes.data, None), "milo_chunk_prefix")
+    return {key: v[:k] for key, v in out.items()}
 
 
 def _stream_ptr(stream) -> Optional[int]:

@@ -175,3 +175,64 @@ def test_partition_balances_bytes(milo):
     mean = cost.mean()
     assert cost.max() <= mean * 1.15, (cost.max(), mean)
     assert (cost > 0).all()
+
+
+@pytest.mark.parametrize("shape", [
+    ([512] * 64, "choice", 4, 128),
+    ([7, 129, 1, 64, 65, 300, 1024, 2048], "rand", 2, 64),
+    ([512, 33, 1000] * 3, "rand", 3, 128),
+])
+def test_chunks_cover_every_token_once_within_budget(milo, shape):
+    """The short-block decode's work list (milo_chunk_prefix): KV-head-major,
+    then block order; every token of every entry exactly once; ranges start
+    on 32-token boundaries; each entry uses the fewest ranges whose rows fit
+    the 128 KB budget (at most 1024 tokens), and its ranges are equal up to
+    the last one's remainder."""
+    bl, law, hkv, d = shape
+    rng = np.random.default_rng(len(bl) * 11 + hkv)
+    nb = len(bl)
+    if law == "choice":
+        rk = rng.choice([16, 32, 64, 96, 128], size=nb * hkv)
+    else:
+        rk = rng.integers(0, d + 1, size=nb * hkv)
+    rv = rng.integers(0, d + 1, size=nb * hkv)
+    t = ht(milo, **table(bl, rk, rv, hkv=hkv, d=d))
+    ch = milo.milo_chunk_prefix(t)
+    r8 = lambda r: (int(r) + 7) // 8 * 8
+    # expected order: KV head g, then block b, then ascending t0
+    keys = [(int(e) % hkv, int(e) // hkv, int(t0)) for e, t0 in zip(ch["entry"], ch["t0"])]
+    assert keys == sorted(keys)
+    per_entry = {}
+    for e, t0, t1 in zip(ch["entry"], ch["t0"], ch["t1"]):
+        n = bl[int(e) // hkv]
+        assert t0 % 32 == 0 and t0 < t1 <= n
+        per_entry.setdefault(int(e), []).append((int(t0), int(t1)))
+    for b in range(nb):
+        for g in range(hkv):
+            e = b * hkv + g
+            n = bl[b]
+            ranges = per_entry.get(e, [])
+            if n == 0:
+                assert not ranges
+                continue
+            # exact cover, in order
+            assert ranges[0][0] == 0 and ranges[-1][1] == n
+            assert all(a[1] == c[0] for a, c in zip(ranges, ranges[1:]))
+            # fewest ranges within the byte budget, and equal lengths
+            row = (r8(rk[e]) + r8(rv[e])) * 2
+            most = max(32, min(1024, 131072 // row // 32 * 32))
+            assert len(ranges) == -(-n // most)
+            lens = [c - a for a, c in ranges]
+            assert all(L == lens[0] for L in lens[:-1]) and lens[-1] <= lens[0]
+            assert lens[0] <= most and lens[0] % 32 == 0 or len(lens) == 1
+
+
+def test_chunk_prefix_reports_a_short_buffer(milo):
+    t = ht(milo, **table([512] * 4, [128] * 4, [128] * 4, hkv=1, d=128))
+    L = milo.lib()
+    n = ctypes.c_int32(0)
+    assert L.milo_chunk_prefix(ctypes.byref(t.c), 0, None, None, None, ctypes.byref(n)) == 0
+    assert n.value == 8  # 512 tokens at ranks 128 + 128: two 256-token ranges per entry
+    buf = (ctypes.c_int32 * 4)()
+    assert L.milo_chunk_prefix(ctypes.byref(t.c), 4, buf, None, None, ctypes.byref(n)) == 1
+    assert n.value == 8
