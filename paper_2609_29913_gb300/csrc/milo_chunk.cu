@@ -583,44 +583,38 @@ __global__ void __launch_bounds__(kChunkThreads)
     for (int w = 0; w < kWarps; ++w) lsum += sx_l[8 * w + r4] * exp2_diff(sx_m[8 * w + r4], M);
     const uint32_t refb = sx_ref[r4];
     {
-        // v~ = sum over warps of 2^(m_w - M) v~_w, gathered in warp 0: the
-        // other warps' scaled values pass through the q~ area in turn, half
-        // of them at a time
+        // v~ = sum over warps of 2^(m_w - M) v~_w, gathered in warp 0.  The
+        // other warps' scaled values pass through a slot that is free by now:
+        // a chunk's P^V fits one piece (ranks <= d), so after its last C
+        // piece no copy targets that slot; a tail item's data is consumed.
+        static_assert((kWarps - 1) * (D / 8) * 32 * 16 <= kPieceBytes, "warp values fit a slot");
+        static_assert(L::kRanksPerPiece >= D, "P^V of any rank is one piece");
         const float sc = exp2_diff(m_w, M);
-        float4 *xv = reinterpret_cast<float4 *>(sq);
+        const int free_slot = is_tail ? 0 : ((ps.npk + ps.nc - 1) & 1);
+        float4 *xv = reinterpret_cast<float4 *>(smem + free_slot * kPieceBytes);
+        if (warp > 0) {
+#pragma unroll
+            for (int n = 0; n < NT; ++n)
+                xv[((warp - 1) * NT + n) * 32 + lane] =
+                    make_float4(sc * vacc[n][0], sc * vacc[n][1], sc * vacc[n][2], sc * vacc[n][3]);
+        }
+        __syncthreads();
         if (warp == 0) {
 #pragma unroll
             for (int n = 0; n < NT; ++n) {
-                vacc[n][0] *= sc;
-                vacc[n][1] *= sc;
-                vacc[n][2] *= sc;
-                vacc[n][3] *= sc;
-            }
-        }
-#pragma unroll 1
-        for (int w = 1; w < kWarps; ++w) {
+                float4 a = make_float4(sc * vacc[n][0], sc * vacc[n][1], sc * vacc[n][2], sc * vacc[n][3]);
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                if (warp == w) {
-#pragma unroll
-                    for (int n = 0; n < NT / 2; ++n) {
-                        const float *v = vacc[half * (NT / 2) + n];
-                        xv[n * 32 + lane] = make_float4(sc * v[0], sc * v[1], sc * v[2], sc * v[3]);
-                    }
+                for (int w = 1; w < kWarps; ++w) {
+                    const float4 o = xv[((w - 1) * NT + n) * 32 + lane];
+                    a.x += o.x;
+                    a.y += o.y;
+                    a.z += o.z;
+                    a.w += o.w;
                 }
-                __syncthreads();
-                if (warp == 0) {
-#pragma unroll
-                    for (int n = 0; n < NT / 2; ++n) {
-                        float *v = vacc[half * (NT / 2) + n];
-                        const float4 o = xv[n * 32 + lane];
-                        v[0] += o.x;
-                        v[1] += o.y;
-                        v[2] += o.z;
-                        v[3] += o.w;
-                    }
-                }
-                __syncthreads();
+                vacc[n][0] = a.x;
+                vacc[n][1] = a.y;
+                vacc[n][2] = a.z;
+                vacc[n][3] = a.w;
             }
         }
     }
