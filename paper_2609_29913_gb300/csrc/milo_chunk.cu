@@ -26,9 +26,9 @@
 // kTailTokens rows each, landing as cores [column group][token group]) and
 // runs the C steps on them with q~ = scale * log2(e) * q, a share of the
 // tokens per warp; its values are already o.  Every item then adds its result
-// into fp32 accumulators of its KV head (see add_part), and the item that
-// completes a KV head writes the normalised output.  No block waits on
-// another.
+// into fp32 accumulators of its KV head (see add_part) and exits; a small
+// finish grid chained by programmatic dependent launch (one warp per KV head)
+// writes the normalised output.  No block waits on another.
 //
 // Shared-memory cores are 8 rows x 16 bytes (rows = tokens or ranks).  Every
 // wait is bounded (~2 s) and sets MILO_ERR_TIMEOUT.
@@ -54,8 +54,8 @@ struct CLay {
     static constexpr int kQ = 2 * kPieceBytes;                  // q~ (then v~) A fragments [D/16][32 lanes][4]
     static constexpr int kZero = kQ + (D / 16) * 32 * 16;       // a zero core line
     static constexpr int kBar = kZero + 128;                    // 2 mbarriers
-    static constexpr int kX = kBar + 16;                        // warp exchange: m, l [kWarps][8], ref [8], count
-    static constexpr int kTotal = kX + ((16 * kWarps + 9) * 4 + 15) / 16 * 16;
+    static constexpr int kX = kBar + 16;                        // warp exchange: m, l [kWarps][8], ref [8]
+    static constexpr int kTotal = kX + ((16 * kWarps + 8) * 4 + 15) / 16 * 16;
     static constexpr int kRanksPerPiece = kPieceBytes / (D * 2);  // P^K / P^V rows per piece
 };
 
@@ -88,9 +88,9 @@ __device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
 // kRefMargin (compare-and-swap), and every other item reads it back.  With M
 // within kDirectMax below an item's maximum nothing overflows; an item whose
 // maximum lies further above M (a rare outlier) writes its record instead and
-// lists it.  The item that brings the count of its KV head to the total
-// divides the accumulators by the sum, folds in the listed records by the
-// log-sum-exp rule, writes the output and clears the accumulators.
+// lists it.  Once the grid is done, the finish grid divides the accumulators
+// by the sum, folds in the listed records by the log-sum-exp rule, writes the
+// output and clears the accumulators for the next call.
 constexpr float kRefMargin = 40.f;  // M = first tile maximum + this
 constexpr float kDirectMax = 60.f;  // items with m - M above this keep a record
 
@@ -112,7 +112,7 @@ __device__ __forceinline__ uint32_t publish_ref(const DecodeParams &p, int g, in
     return got;
 }
 
-// The last item of KV head g: fold the listed records into the accumulators,
+// KV head g, after every item: fold the listed records into the accumulators,
 // write the output rows, clear the accumulators.  Lane l: row l / 4, quarter
 // l % 4 of the head dimension.
 template <int D>
@@ -163,10 +163,7 @@ __device__ void finish_head(const DecodeParams &p, int g, int list_base, int lan
         __stcg(p.acc_l + ai, 0.f);
         __stcg(p.acc_m + ai, 0u);
     }
-    if (lane == 0) {
-        __stcg(p.ovf_cnt + g, 0u);
-        __stcg(p.head_cnt + g, 0u);
-    }
+    if (lane == 0) __stcg(p.ovf_cnt + g, 0u);
 }
 
 // This warp's share of an item's contribution to KV head g: head-dimension
@@ -223,7 +220,6 @@ __global__ void __launch_bounds__(kChunkThreads)
     float *sx_m = reinterpret_cast<float *>(smem + L::kX);       // [warp][row]
     float *sx_l = sx_m + 8 * kWarps;                             // [warp][row]
     uint32_t *sx_ref = reinterpret_cast<uint32_t *>(sx_l + 8 * kWarps);  // [row]
-    uint32_t *sx_cnt = sx_ref + 8;
     const uint32_t zline = smem_u32(smem + L::kZero) + mr * 16;
     const uint32_t bar0 = smem_u32(smem + L::kBar);
     const bool is_tail = (int)blockIdx.x >= p.num_chunks;
@@ -689,26 +685,23 @@ __global__ void __launch_bounds__(kChunkThreads)
         direct = add_part<D, NO>(p, g, lane, warp * NO, ov, M, lsum, refb, warp == 0, row0, nrows, rec_idx);
     }
 
-    // ---- count the item (its reductions and stores ordered before the
-    // count); the item that completes its KV head finishes it
-    const int S = p.tail_splits;
-    const int list_base = p.g_slot_begin[g] + g * p.batch * S;
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) {
-        if (!direct) {
-            const uint32_t k = atomicAdd(p.ovf_cnt + g, 1u);
-            __stcg(reinterpret_cast<int4 *>(p.ovf_list) + list_base + k, make_int4((int)rec_idx, row0, nrows, 0));
-            __threadfence();
-        }
-        *sx_cnt = atomicAdd(p.head_cnt + g, 1u);
+    // ---- an outlier's record is listed; the finish grid that follows
+    // (programmatic dependent launch) sees every reduction and record
+    if (tid == 0 && !direct) {
+        const int list_base = p.g_slot_begin[g] + g * p.batch * p.tail_splits;
+        const uint32_t k = atomicAdd(p.ovf_cnt + g, 1u);
+        __stcg(reinterpret_cast<int4 *>(p.ovf_list) + list_base + k, make_int4((int)rec_idx, row0, nrows, 0));
     }
-    __syncthreads();
-    const uint32_t total = (uint32_t)(p.g_slot_begin[g + 1] - p.g_slot_begin[g] + p.batch * S);
-    if (*sx_cnt == total - 1 && warp == 0) {
-        __threadfence();  // every other item's contribution is visible from here
-        finish_head<D>(p, g, list_base, lane);
-    }
+}
+
+// One warp per KV head: normalise the accumulators once the chunk grid is done.
+template <int D>
+__global__ void __launch_bounds__(32) finish_kernel(const __grid_constant__ DecodeParams p)
+{
+    pdl_trigger();
+    pdl_wait();  // the chunk grid's reductions and records are visible from here
+    const int g = blockIdx.x;
+    finish_head<D>(p, g, p.g_slot_begin[g] + g * p.batch * p.tail_splits, threadIdx.x);
 }
 
 }  // namespace
@@ -740,8 +733,13 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
         configured[w] = 1;
     }
     cfg.dynamicSmemBytes = (size_t)smem;
-    return w == 0 ? cudaLaunchKernelEx(&cfg, chunk_kernel<64>, p, mk, mv)
-                  : cudaLaunchKernelEx(&cfg, chunk_kernel<128>, p, mk, mv);
+    cudaError_t e = w == 0 ? cudaLaunchKernelEx(&cfg, chunk_kernel<64>, p, mk, mv)
+                           : cudaLaunchKernelEx(&cfg, chunk_kernel<128>, p, mk, mv);
+    if (e != cudaSuccess) return e;
+    cfg.gridDim = dim3(p.hkv);
+    cfg.blockDim = dim3(32);
+    cfg.dynamicSmemBytes = 0;
+    return w == 0 ? cudaLaunchKernelEx(&cfg, finish_kernel<64>, p) : cudaLaunchKernelEx(&cfg, finish_kernel<128>, p);
 }
 
 }  // namespace milo

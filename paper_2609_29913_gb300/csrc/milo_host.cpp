@@ -231,9 +231,9 @@ void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs
 }
 
 // The plan's counter buffer: CountersDev, then for the short-block decode the
-// per-KV-head item counts [H], reference maxima [8 H], list counts [H], and at
-// a 16-byte boundary the row sums [8 H] and output accumulators [8 H d].
-size_t acc_l_offset(int H) { return (sizeof(CountersDev) + sizeof(uint32_t) * 10 * (size_t)H + 15) / 16 * 16; }
+// per-KV-head reference maxima [8 H], list counts [H], and at a 16-byte
+// boundary the row sums [8 H] and output accumulators [8 H d].
+size_t acc_l_offset(int H) { return (sizeof(CountersDev) + sizeof(uint32_t) * 9 * (size_t)H + 15) / 16 * 16; }
 size_t counters_bytes(int H, int d) { return acc_l_offset(H) + sizeof(float) * 8 * (size_t)H * (1 + (size_t)d); }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -597,12 +597,11 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.rec = static_cast<float *>(workspace);
 
     prm.counters = plan->counters;
-    prm.head_cnt = reinterpret_cast<uint32_t *>(plan->counters + 1);
     {
-        // after the head counters: reference maxima, list counts, then the
-        // 16-byte aligned sums and output accumulators
+        // after CountersDev: reference maxima, list counts, then the 16-byte
+        // aligned sums and output accumulators
         const int H = plan->hkv;
-        prm.acc_m = prm.head_cnt + H;
+        prm.acc_m = reinterpret_cast<uint32_t *>(plan->counters + 1);
         prm.ovf_cnt = prm.acc_m + 8 * H;
         uint8_t *base = reinterpret_cast<uint8_t *>(plan->counters);
         prm.acc_l = reinterpret_cast<float *>(base + acc_l_offset(H));

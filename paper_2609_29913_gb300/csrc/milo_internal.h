@@ -102,7 +102,6 @@ struct DecodeParams {
     const ChunkDev *chunks;         // short-block decode: the prefix chunks (KV-head-major)
     int num_chunks;                 // 0: the persistent kernels run
     const uint16_t *tail_k, *tail_v;  // bf16 [rows, Hkv, d] dense tails (or null)
-    uint32_t *head_cnt;             // [Hkv]: chunks and tail items done per KV head
     float *acc_o;                   // [Hkv][8][d]: per-row accumulators of the short-block decode
     float *acc_l;                   // [Hkv][8]
     uint32_t *acc_m;                // [Hkv][8]: reference maxima (sign-flipped float bits; 0 = unset)
