@@ -222,12 +222,13 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
  *   out          device fp32 [batch, num_q_heads, head_dim].
  *   workspace    device, at least milo_workspace_size bytes, 256-byte aligned.
  * Asynchronous on `stream`: no host synchronisation and no allocation, so the
- * call can be captured in a CUDA graph.  Launched with programmatic dependent
- * launch: the kernel may begin streaming the plan's factors before the
- * preceding kernel on `stream` finishes, and reads q, the tails and the
- * workspace only after it has.  A plan must not be used by two calls that can
- * run concurrently (it holds per-call counters).  A query whose prefix and
- * tail are both empty yields NaN.
+ * call can be captured in a CUDA graph.  A call is two kernels launched with
+ * programmatic dependent launch: the first may begin streaming the plan's
+ * factors before the preceding kernel on `stream` finishes, and reads q, the
+ * tails and the workspace only after it has; the second combines and writes
+ * `out`.  A plan must not be used by two calls that can run concurrently (it
+ * holds per-call counters and accumulators).  A query whose prefix and tail
+ * are both empty yields NaN.
  */
 milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q,
                                int32_t batch, const void *tail_k,
