@@ -106,22 +106,25 @@ __device__ __forceinline__ uint32_t publish_ref(const DecodeParams &p, int g, in
     uint32_t got = 0u;
     if (c4 == 0 && row_ok) {
         const uint32_t mine = ref_enc(m + kRefMargin);
-        const uint32_t old = atomicCAS(p.acc_m + g * 8 + arow, 0u, mine);
+        const uint32_t old = atomicCAS(p.acc_m + (int64_t)g * p.rows_max + arow, 0u, mine);
         got = old ? old : mine;
     }
     return got;
 }
 
-// KV head g, after every item: fold the listed records into the accumulators,
-// write the output rows, clear the accumulators.  Lane l: row l / 4, quarter
-// l % 4 of the head dimension.
+// KV head g, rows 8 rg .. 8 rg + 7, after every item: fold the listed
+// records into the accumulators, write the output rows, clear the
+// accumulators and the list.  Lane l: row 8 rg + l / 4, quarter l % 4 of the
+// head dimension.
 template <int D>
-__device__ void finish_head(const DecodeParams &p, int g, int list_base, int lane)
+__device__ void finish_head(const DecodeParams &p, int g, int rg, int lane)
 {
+    const int gr = g * p.nrg + rg;  // this (KV head, row group)'s list
+    const int64_t list_base = (int64_t)gr * p.list_cap;
     constexpr int kF4 = D / 16;  // float4 columns per quarter
     const int recf = 8 * D + kRecFloatsExtra;
-    const int row = lane >> 2, qq = lane & 3;
-    const int64_t ai = (int64_t)g * 8 + row;
+    const int row = rg * 8 + (lane >> 2), qq = lane & 3;  // the KV head's query row (batch x heads)
+    const int64_t ai = (int64_t)g * p.rows_max + row;
     float4 *Oq = reinterpret_cast<float4 *>(p.acc_o + ai * D + qq * (D / 4));
     const uint32_t mb = __ldcg(p.acc_m + ai);
     float M = mb ? ref_dec(mb) : -INFINITY;
@@ -129,7 +132,7 @@ __device__ void finish_head(const DecodeParams &p, int g, int list_base, int lan
     float4 acc[kF4];
 #pragma unroll
     for (int f = 0; f < kF4; ++f) acc[f] = __ldcg(Oq + f);
-    const uint32_t nov = __ldcg(p.ovf_cnt + g);
+    const uint32_t nov = __ldcg(p.ovf_cnt + gr);
 #pragma unroll 1
     for (uint32_t k = 0; k < nov; ++k) {
         const int4 e = __ldcg(reinterpret_cast<const int4 *>(p.ovf_list) + list_base + k);
@@ -163,7 +166,7 @@ __device__ void finish_head(const DecodeParams &p, int g, int list_base, int lan
         __stcg(p.acc_l + ai, 0.f);
         __stcg(p.acc_m + ai, 0u);
     }
-    if (lane == 0) __stcg(p.ovf_cnt + g, 0u);
+    if (lane == 0) __stcg(p.ovf_cnt + gr, 0u);
 }
 
 // This warp's share of an item's contribution to KV head g: head-dimension
@@ -183,11 +186,11 @@ __device__ bool add_part(const DecodeParams &p, int g, int lane, int n0, const f
     if (direct) {
         if (row_ok && M != -INFINITY) {
             const float f = ex2_approx(M - Mref);
-            float *orow = p.acc_o + ((int64_t)g * 8 + row0 + r4) * D + 8 * n0 + 2 * c4;
+            float *orow = p.acc_o + ((int64_t)g * p.rows_max + row0 + r4) * D + 8 * n0 + 2 * c4;
 #pragma unroll
             for (int n = 0; n < NC; ++n)
                 atomicAdd(reinterpret_cast<float2 *>(orow + 8 * n), make_float2(f * ov[n][0], f * ov[n][1]));
-            if (with_l && c4 == 0) atomicAdd(p.acc_l + g * 8 + row0 + r4, f * lsum);
+            if (with_l && c4 == 0) atomicAdd(p.acc_l + (int64_t)g * p.rows_max + row0 + r4, f * lsum);
         }
     } else {
         // an outlier maximum: the item keeps a record for the final merge
@@ -222,7 +225,12 @@ __global__ void __launch_bounds__(kChunkThreads)
     uint32_t *sx_ref = reinterpret_cast<uint32_t *>(sx_l + 8 * kWarps);  // [row]
     const uint32_t zline = smem_u32(smem + L::kZero) + mr * 16;
     const uint32_t bar0 = smem_u32(smem + L::kBar);
-    const bool is_tail = (int)blockIdx.x >= p.num_chunks;
+    // blocks [0, num_chunks * nrg): chunk blockIdx / nrg for row group
+    // blockIdx % nrg (the row groups of one chunk are neighbours, so they read
+    // its pieces from L2); then the dense-tail items
+    const int nprefix = p.num_chunks * p.nrg;
+    const bool is_tail = (int)blockIdx.x >= nprefix;
+    const int rgrp = is_tail ? 0 : (int)blockIdx.x % p.nrg;
 
     pdl_trigger();
     // zero the slots, q~ and the zero line: reads past a piece's data then
@@ -234,7 +242,7 @@ __global__ void __launch_bounds__(kChunkThreads)
     Pieces ps = {};
     int g = 0, ntok = 0, nrk = 0, nrv = 0;
     if (!is_tail) {
-        ch = p.chunks[blockIdx.x];
+        ch = p.chunks[blockIdx.x / p.nrg];
         ps = pieces_of<D>(ch);
         g = ch.g;
         ntok = ch.ntok;
@@ -420,7 +428,7 @@ __global__ void __launch_bounds__(kChunkThreads)
     int qi = 0, item = 0;
     if (is_tail) {
         // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense tail
-        item = (int)blockIdx.x - p.num_chunks;
+        item = (int)blockIdx.x - nprefix;
         const int S = p.tail_splits;
         qi = item / (p.hkv * S);
         const int sp = item % S;
@@ -478,8 +486,9 @@ __global__ void __launch_bounds__(kChunkThreads)
         {
             // q rows of KV head g as the projection's B fragments (q^T)
             uint32_t qa[KD][2];
-            const bool row_ok = r4 < p.rows_g;
-            const uint16_t *qr = p.q + ((int64_t)(r4 / p.G) * p.hq + g * p.G + r4 % p.G) * D + 2 * c4;
+            const int qrow = 8 * rgrp + r4;  // the KV head's query row (batch x heads)
+            const bool row_ok = qrow < p.rows_g;
+            const uint16_t *qr = p.q + ((int64_t)(qrow / p.G) * p.hq + g * p.G + qrow % p.G) * D + 2 * c4;
 #pragma unroll
             for (int ks = 0; ks < KD; ++ks) {
                 qa[ks][0] = row_ok ? *reinterpret_cast<const uint32_t *>(qr + 16 * ks) : 0u;
@@ -556,7 +565,7 @@ __global__ void __launch_bounds__(kChunkThreads)
                              integral_constant<uint32_t, 128>{}, slot, nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
                 }
             });
-            if (k == ps.npk && warp == 0) ref = publish_ref(p, g, r4, r4 < p.rows_g, c4, m_w);
+            if (k == ps.npk && warp == 0) ref = publish_ref(p, g, 8 * rgrp + r4, 8 * rgrp + r4 < p.rows_g, c4, m_w);
             release_piece(k);
         }
     }
@@ -633,8 +642,8 @@ __global__ void __launch_bounds__(kChunkThreads)
                            : __all_sync(0xffffffffu, r4 >= nrows || !(M - (refb ? ref_dec(refb) : M) > kDirectMax));
     } else {
         rec_idx = (int64_t)blockIdx.x;
-        row0 = 0;
-        nrows = p.rows_g;
+        row0 = 8 * rgrp;
+        nrows = min(8, p.rows_g - row0);
         // warp 0 stages the merged v~ as the back-projection's A fragments (rows
         // 0-7 hi, 8-15 lo) in the q~ area, so that the rank loop below stays rolled
         if (warp == 0) {
@@ -688,20 +697,24 @@ __global__ void __launch_bounds__(kChunkThreads)
     // ---- an outlier's record is listed; the finish grid that follows
     // (programmatic dependent launch) sees every reduction and record
     if (tid == 0 && !direct) {
-        const int list_base = p.g_slot_begin[g] + g * p.batch * p.tail_splits;
-        const uint32_t k = atomicAdd(p.ovf_cnt + g, 1u);
-        __stcg(reinterpret_cast<int4 *>(p.ovf_list) + list_base + k, make_int4((int)rec_idx, row0, nrows, 0));
+        // in the list of every row group the item's rows touch
+        for (int rg = row0 / 8; rg <= (row0 + nrows - 1) / 8; ++rg) {
+            const int gr = g * p.nrg + rg;
+            const uint32_t k = atomicAdd(p.ovf_cnt + gr, 1u);
+            __stcg(reinterpret_cast<int4 *>(p.ovf_list) + (int64_t)gr * p.list_cap + k,
+                   make_int4((int)rec_idx, row0, nrows, 0));
+        }
     }
 }
 
-// One warp per KV head: normalise the accumulators once the chunk grid is done.
+// One warp per (KV head, group of 8 query rows): normalise the accumulators
+// once the chunk grid is done.
 template <int D>
 __global__ void __launch_bounds__(32) finish_kernel(const __grid_constant__ DecodeParams p)
 {
     pdl_trigger();
     pdl_wait();  // the chunk grid's reductions and records are visible from here
-    const int g = blockIdx.x;
-    finish_head<D>(p, g, p.g_slot_begin[g] + g * p.batch * p.tail_splits, threadIdx.x);
+    finish_head<D>(p, blockIdx.x / p.nrg, blockIdx.x % p.nrg, threadIdx.x);
 }
 
 }  // namespace
@@ -711,7 +724,7 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     const CUtensorMap &mk = *static_cast<const CUtensorMap *>(tmap_k);
     const CUtensorMap &mv = *static_cast<const CUtensorMap *>(tmap_v);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.num_chunks + (p.has_tail ? p.num_tail_items : 0));
+    cfg.gridDim = dim3(p.num_chunks * p.nrg + (p.has_tail ? p.num_tail_items : 0));
     cfg.blockDim = dim3(kChunkThreads);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -736,7 +749,7 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     cudaError_t e = w == 0 ? cudaLaunchKernelEx(&cfg, chunk_kernel<64>, p, mk, mv)
                            : cudaLaunchKernelEx(&cfg, chunk_kernel<128>, p, mk, mv);
     if (e != cudaSuccess) return e;
-    cfg.gridDim = dim3(p.hkv);
+    cfg.gridDim = dim3(p.hkv * p.nrg);
     cfg.blockDim = dim3(32);
     cfg.dynamicSmemBytes = 0;
     return w == 0 ? cudaLaunchKernelEx(&cfg, finish_kernel<64>, p) : cudaLaunchKernelEx(&cfg, finish_kernel<128>, p);

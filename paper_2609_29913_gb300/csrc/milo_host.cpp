@@ -231,10 +231,17 @@ void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs
 }
 
 // The plan's counter buffer: CountersDev, then for the short-block decode the
-// per-KV-head reference maxima [8 H], list counts [H], and at a 16-byte
-// boundary the row sums [8 H] and output accumulators [8 H d].
-size_t acc_l_offset(int H) { return (sizeof(CountersDev) + sizeof(uint32_t) * 9 * (size_t)H + 15) / 16 * 16; }
-size_t counters_bytes(int H, int d) { return acc_l_offset(H) + sizeof(float) * 8 * (size_t)H * (1 + (size_t)d); }
+// reference maxima [H][R] (R = 8 row groups of 8 rows), the list counts
+// [H][R / 8], and at a 16-byte boundary the row sums [H][R] and the output
+// accumulators [H][R][d].
+size_t acc_l_offset(int H, int R)
+{
+    return (sizeof(CountersDev) + sizeof(uint32_t) * (size_t)H * (R + R / 8) + 15) / 16 * 16;
+}
+size_t counters_bytes(int H, int R, int d)
+{
+    return acc_l_offset(H, R) + sizeof(float) * (size_t)H * R * (1 + (size_t)d);
+}
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
@@ -267,8 +274,8 @@ struct milo_prefix {
     int32_t *cta_seg_begin = nullptr;
     int32_t *g_slot_begin = nullptr;
     ChunkDev *chunks = nullptr;       // short-block decode: prefix chunks, KV-head-major
-    int32_t *g_chunk_begin = nullptr; // first chunk of each KV head
     int num_chunks = 0;
+    int max_head_chunks = 0;          // the most chunks of one KV head
     CountersDev *counters = nullptr;
     int32_t *status = nullptr;
 };
@@ -370,7 +377,6 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaFree(plan->cta_seg_begin);
     cudaFree(plan->g_slot_begin);
     cudaFree(plan->chunks);
-    cudaFree(plan->g_chunk_begin);
     cudaFree(plan->counters);
     cudaFree(plan->status);
     cudaSetDevice(cur);
@@ -435,6 +441,8 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     std::vector<int32_t> g_chunk;
     build_chunks(table, poffs, chunks, g_chunk);
     p->num_chunks = (int)chunks.size();
+    for (int g = 0; g < H; ++g)
+        p->max_head_chunks = std::max(p->max_head_chunks, g_chunk[(size_t)g + 1] - g_chunk[(size_t)g]);
     std::vector<SegDev> sd(segs.size());
     for (size_t i = 0; i < segs.size(); ++i) {
         sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
@@ -446,8 +454,8 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         milo_prefix_destroy(p);
         return cuda_fail(err, what);
     };
-    // + per-KV-head and per-entry counters of the short-block decode
-    const size_t cnt_bytes = counters_bytes(H, d);
+    // + the accumulators of the short-block decode (G <= 8)
+    const size_t cnt_bytes = G <= 8 ? counters_bytes(H, 8 * p->max_nrg, d) : sizeof(CountersDev);
     if ((e = cudaMalloc(&p->packed, (size_t)std::max<int64_t>(p->packed_bytes, 128))) != cudaSuccess)
         return cleanup(e, "cudaMalloc packed");
     if ((e = cudaMalloc(&p->entries, sizeof(EntryDev) * std::max<size_t>(ents.size(), 1))) != cudaSuccess)
@@ -460,14 +468,9 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         return cleanup(e, "cudaMalloc g_slot_begin");
     if ((e = cudaMalloc(&p->chunks, sizeof(ChunkDev) * std::max<size_t>(chunks.size(), 1))) != cudaSuccess)
         return cleanup(e, "cudaMalloc chunks");
-    if ((e = cudaMalloc(&p->g_chunk_begin, sizeof(int32_t) * g_chunk.size())) != cudaSuccess)
-        return cleanup(e, "cudaMalloc g_chunk_begin");
     if (!chunks.empty() && (e = cudaMemcpyAsync(p->chunks, chunks.data(), sizeof(ChunkDev) * chunks.size(),
                                                 cudaMemcpyHostToDevice, stream)) != cudaSuccess)
         return cleanup(e, "copy chunks");
-    if ((e = cudaMemcpyAsync(p->g_chunk_begin, g_chunk.data(), sizeof(int32_t) * g_chunk.size(),
-                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
-        return cleanup(e, "copy g_chunk_begin");
     if ((e = cudaMalloc(&p->counters, cnt_bytes)) != cudaSuccess) return cleanup(e, "cudaMalloc counters");
     if ((e = cudaMalloc(&p->status, sizeof(int32_t))) != cudaSuccess) return cleanup(e, "cudaMalloc status");
     if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
@@ -521,8 +524,9 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t
 namespace {
 struct CallShape {
     int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
+    bool chunked;
     int64_t records;
-    int64_t list_bytes;
+    int64_t list_cap, list_bytes;
 };
 
 CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
@@ -536,12 +540,16 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
-    // one record per prefix chunk (one row group: the short-block decode),
-    // or one per run and row group (the persistent kernel); then the tail
-    // items.  The short-block decode also lists records (an int4 per item).
-    const int64_t prefix = c.nrg == 1 ? (int64_t)p->num_chunks : (int64_t)p->num_slots * c.nrg;
+    // the short-block decode serves every call with a prefix and G <= 8
+    c.chunked = p->G <= 8 && p->num_chunks > 0;
+    // one record per prefix chunk and row group (the short-block decode), or
+    // per run and row group (the persistent kernel); then the tail items.
+    // The short-block decode also lists records: int4 [Hkv][nrg][list_cap],
+    // list_cap bounding the items whose rows meet one row group.
+    const int64_t prefix = c.chunked ? (int64_t)p->num_chunks * c.nrg : (int64_t)p->num_slots * c.nrg;
     c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
-    c.list_bytes = c.nrg == 1 ? 16 * c.records : 0;
+    c.list_cap = c.chunked ? (int64_t)p->max_head_chunks + (int64_t)batch * c.S : 0;
+    c.list_bytes = 16 * (int64_t)p->hkv * c.nrg * c.list_cap;
 
     return c;
 }
@@ -597,15 +605,16 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.rec = static_cast<float *>(workspace);
 
     prm.counters = plan->counters;
-    {
+    if (c.chunked) {
         // after CountersDev: reference maxima, list counts, then the 16-byte
         // aligned sums and output accumulators
-        const int H = plan->hkv;
+        const int H = plan->hkv, R = 8 * plan->max_nrg;
+        prm.rows_max = R;
         prm.acc_m = reinterpret_cast<uint32_t *>(plan->counters + 1);
-        prm.ovf_cnt = prm.acc_m + 8 * H;
+        prm.ovf_cnt = prm.acc_m + (size_t)H * R;
         uint8_t *base = reinterpret_cast<uint8_t *>(plan->counters);
-        prm.acc_l = reinterpret_cast<float *>(base + acc_l_offset(H));
-        prm.acc_o = prm.acc_l + 8 * H;
+        prm.acc_l = reinterpret_cast<float *>(base + acc_l_offset(H, R));
+        prm.acc_o = prm.acc_l + (size_t)H * R;
     }
     prm.status = plan->status;
     prm.batch = batch;
@@ -625,16 +634,15 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.num_tail_items = batch * plan->hkv * c.S;
     prm.has_tail = c.S > 0 ? 1 : 0;
     prm.tail_rec_base = (int64_t)plan->num_slots * c.nrg;
-    // one row group: the short-block decode
     prm.tail_k = static_cast<const uint16_t *>(tail_k);
     prm.tail_v = static_cast<const uint16_t *>(tail_v);
     prm.chunks = plan->chunks;
-    prm.num_chunks = c.nrg == 1 ? plan->num_chunks : 0;
-    if (prm.num_chunks > 0) {
-        prm.g_slot_begin = plan->g_chunk_begin;
+    prm.num_chunks = c.chunked ? plan->num_chunks : 0;
+    if (c.chunked) {
         prm.num_slots = plan->num_chunks;
-        prm.tail_rec_base = plan->num_chunks;
-        // the record list follows the records
+        prm.tail_rec_base = (int64_t)plan->num_chunks * c.nrg;
+        // the record lists follow the records
+        prm.list_cap = (int)c.list_cap;
         prm.ovf_list = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) +
                                                    (size_t)c.records * (8 * plan->d + kRecFloatsExtra) * sizeof(float));
     }

@@ -102,11 +102,13 @@ struct DecodeParams {
     const ChunkDev *chunks;         // short-block decode: the prefix chunks (KV-head-major)
     int num_chunks;                 // 0: the persistent kernels run
     const uint16_t *tail_k, *tail_v;  // bf16 [rows, Hkv, d] dense tails (or null)
-    float *acc_o;                   // [Hkv][8][d]: per-row accumulators of the short-block decode
-    float *acc_l;                   // [Hkv][8]
-    uint32_t *acc_m;                // [Hkv][8]: reference maxima (sign-flipped float bits; 0 = unset)
-    uint32_t *ovf_cnt;              // [Hkv]: records listed for the final merge
-    int32_t *ovf_list;              // int4 [chunks + tail items]: listed records (workspace)
+    int rows_max;                   // accumulator rows per KV head: 8 ceil(max_batch G / 8)
+    float *acc_o;                   // [Hkv][rows_max][d]: per-row accumulators of the short-block decode
+    float *acc_l;                   // [Hkv][rows_max]
+    uint32_t *acc_m;                // [Hkv][rows_max]: reference maxima (sign-flipped float bits; 0 = unset)
+    uint32_t *ovf_cnt;              // [Hkv][nrg]: records listed per (KV head, row group)
+    int32_t *ovf_list;              // int4 [Hkv][nrg][list_cap]: listed records (workspace)
+    int list_cap;                   // list entries per (KV head, row group)
 };
 
 // Launchers implemented in the .cu files.
@@ -121,8 +123,9 @@ cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k,
 
 int decode_smem_bytes(int head_dim, int nrg_cta);
 
-// The short-block decode grid alone (one thread block per prefix chunk and
-// per tail item); launch_decode calls it and then launches the merge.
+// The short-block decode (one thread block per prefix chunk and row group of
+// 8 query rows, and per tail item), then its finish grid; launch_decode calls
+// it when G <= 8.
 cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void *tmap_v, cudaStream_t stream);
 
 

@@ -112,6 +112,33 @@ def test_outlier_maximum_takes_the_record_path(env):
     pre.close()
 
 
+@pytest.mark.parametrize("batch,hot_tail", [(3, False), (3, True), (10, True)])
+def test_outlier_maximum_batched_row_groups(env, batch, hot_tail):
+    """The listed-record merge with several row groups of 8 query rows: GQA 7,
+    so most queries' rows straddle two row groups, whose finish warps both
+    read such an item's record.  Prefix tokens 300-309 of every KV head get
+    scores 256 times larger; with hot_tail, query 1's tail keys are scaled
+    the same way, so tail items (one per query) take the record path too."""
+    W = env["W"]
+    tails = [70 + 13 * i for i in range(batch)]
+    layer = W.build_layer(14, 2, 128, [1024, 512], [[16, 16], [64, 32]], batch=batch, tail_lengths=tails,
+                          seed=18 + batch, device="cuda")
+    A = layer.arena
+    for e in range(2):
+        r = int(layer.rank_k[e])
+        off = int(layer.off_ck[e])
+        A[off + 300 * r:off + 310 * r] *= 256.0
+    if hot_tail:
+        o0, o1 = int(layer.tail_offsets[1]), int(layer.tail_offsets[2])
+        layer.tail_k[o0:o1] *= 64.0
+    out, pre = decode(env, layer)
+    ref = env["oracle"].attention(**layer.to_numpy_bits())
+    compare(out.cpu().numpy(), ref, "batched outlier")
+    out2, _ = decode(env, layer, plan=pre)  # the accumulators and lists were cleared
+    compare(out2.cpu().numpy(), ref, "batched outlier again")
+    pre.close()
+
+
 def test_explicit_scale(env):
     layer = env["W"].make_random_case(num_q_heads=7, num_kv_heads=1, head_dim=64,
                                       block_lens=[128, 64], rank_choices=(16, 40),
@@ -211,12 +238,16 @@ def test_repeated_calls_batches_and_graph_capture(env):
     ref = env["oracle"].attention(**layer.to_numpy_bits())
     pre = milo.Prefix.from_layer(layer, max_batch=4)
     first, _ = decode(env, layer, plan=pre)
-    # warps merge their partial sums with shared-memory atomics, so repeated
-    # calls agree to fp32 rounding (not bit for bit)
+    compare(first.cpu().numpy(), ref, "repeat")
+    # Items add their scaled partial sums into fp32 accumulators with atomics
+    # in whatever order they finish, so repeated calls agree to fp32 rounding,
+    # not bit for bit: each output is a sum of some tens of partials, each
+    # addition rounding at 2^-24 of the running sum, and the running sums of
+    # signed values can exceed the final one several times over.
+    rep_tol = 2e-5 * first.abs().max().item()
     for _ in range(3):
         again, _ = decode(env, layer, plan=pre)
-        assert (again - first).abs().max().item() <= 1e-6 * first.abs().max().item()
-    compare(first.cpu().numpy(), ref, "repeat")
+        assert (again - first).abs().max().item() <= rep_tol
     # a smaller batch on the same plan (queries 0..1)
     sub = W.LayerInputs(layer.num_q_heads, layer.num_kv_heads, layer.head_dim, layer.block_len,
                         layer.rank_k, layer.rank_v, layer.off_ck, layer.off_pk, layer.off_cv,
@@ -241,7 +272,7 @@ def test_repeated_calls_batches_and_graph_capture(env):
     out.zero_()
     g.replay()
     torch.cuda.synchronize()
-    assert (out - first).abs().max().item() <= 1e-6 * first.abs().max().item()
+    assert (out - first).abs().max().item() <= rep_tol
     assert pre.status() == 0
     pre.close()
 
