@@ -378,10 +378,11 @@ def main():
     except Exception:
         traffic = None
     value = world * tokens / (ms_step * 1e-3)
-    # up to 8 query rows per KV head: the short-block grid (chunks and tail
-    # items, adding into per-KV-head accumulators) and its finish grid; more:
-    # the persistent kernel and the merge kernel
-    short = cfg.batch * (cfg.num_q_heads // cfg.num_kv_heads) <= 8
+    # up to 8 query heads per KV head: the chunk grid (a block per prefix
+    # chunk and row group of 8 query rows, and per tail item, adding into
+    # per-row accumulators) and its finish grid; more: the persistent kernel
+    # and the merge kernel
+    short = cfg.num_q_heads // cfg.num_kv_heads <= 8
     kernels_per_layer = 2
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -394,16 +395,17 @@ def main():
                    "l2": "inputs larger than L2 (step reads %.2f GB > 129 MB); no flush" % (alg_bytes / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "launch": ("one CUDA graph of %d per-layer calls, each a grid of two-warp blocks (prefix "
-                              "chunks and dense-tail items adding into per-KV-head accumulators) and a finish "
-                              "grid of one warp per KV head (programmatic dependent launch)"
+                              "chunks per row group of 8 query rows, and dense-tail items, adding into per-row "
+                              "accumulators) and a finish grid of one warp per KV head and row group "
+                              "(programmatic dependent launch)"
                               if short else
                               "one CUDA graph of %d per-layer calls, each a persistent decode and a merge "
                               "kernel (programmatic dependent launch)") % cfg.layers},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": f"{peak_kind} copy bandwidth",
-                     "kernel": ("chunk_kernel (two warps per prefix chunk, accumulator merge; finish_kernel "
-                                "chained)" if short
+                     "kernel": ("chunk_kernel (two warps per prefix chunk and row group, accumulator merge; "
+                                "finish_kernel chained)" if short
                                 else "decode_kernel (persistent rank-space split-K decode)"),
                      "per_launch_bytes": alg_bytes // cfg.layers,
                      "per_launch_us": ms_step * 1e3 / cfg.layers},
