@@ -46,16 +46,18 @@ namespace {
 
 constexpr int kPieceBytes = 32768;  // one slot
 constexpr int kTile = 32;           // tokens per tile
-constexpr int kWarps = 2;           // warps per chunk block
-constexpr int kChunkThreads = 32 * kWarps;
+constexpr int kWarps = 2;           // warps per row group of 8 query rows
 
-template <int D>
+// Shared memory of a block of RG row groups (RG x kWarps warps).
+template <int D, int RG>
 struct CLay {
-    static constexpr int kQ = 2 * kPieceBytes;                  // q~ (then v~) A fragments [D/16][32 lanes][4]
-    static constexpr int kZero = kQ + (D / 16) * 32 * 16;       // a zero core line
+    static constexpr int kQ = 2 * kPieceBytes;                  // per row group: q~ (then v~) A fragments
+    static constexpr int kQStride = (D / 16) * 32 * 16;         //   [D/16][32 lanes][4 words]
+    static constexpr int kZero = kQ + RG * kQStride;            // a zero core line
     static constexpr int kBar = kZero + 128;                    // 2 mbarriers
-    static constexpr int kX = kBar + 16;                        // warp exchange: m, l [kWarps][8], ref [8]
-    static constexpr int kTotal = kX + ((16 * kWarps + 8) * 4 + 15) / 16 * 16;
+    static constexpr int kX = kBar + 16;                        // per row group: m, l [kWarps][8], ref [8]
+    static constexpr int kXStride = 16 * kWarps + 8;            //   (words)
+    static constexpr int kTotal = kX + (RG * kXStride * 4 + 15) / 16 * 16;
     static constexpr int kRanksPerPiece = kPieceBytes / (D * 2);  // P^K / P^V rows per piece
 };
 
@@ -71,7 +73,7 @@ template <int D>
 __device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
 {
     Pieces s;
-    s.rpp = CLay<D>::kRanksPerPiece / 8;
+    s.rpp = CLay<D, 1>::kRanksPerPiece / 8;
     s.npk = (c.nrk + s.rpp - 1) / s.rpp;
     s.npv = (c.nrv + s.rpp - 1) / s.rpp;
     s.tpp = max(1, kPieceBytes / (kTile * (c.nrk + c.nrv) * 16));
@@ -206,43 +208,56 @@ __device__ bool add_part(const DecodeParams &p, int g, int lane, int n0, const f
     return direct;
 }
 
-template <int D>
-__global__ void __launch_bounds__(kChunkThreads)
+// RG row groups of 8 query rows per block, kWarps warps each: the groups
+// share every piece (RG = 2 for calls with several row groups per KV head).
+// A tail block holds RG tail items, one per group, in slot g of group g.
+template <int D, int RG>
+__global__ void __launch_bounds__(32 * kWarps * RG)
     chunk_kernel(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tmap_k,
                  const __grid_constant__ CUtensorMap tmap_v)
 {
-    static_assert(2 * (D / 8) * kTailTokens * 16 <= 2 * kPieceBytes, "a tail item fits the two slots");
-    using L = CLay<D>;
+    static_assert(RG == 1 || RG == 2, "one or two row groups per block");
+    static_assert(2 * (D / 8) * kTailTokens * 16 <= (RG == 1 ? 2 : 1) * kPieceBytes,
+                  "a group's tail item fits its slots");
+    using L = CLay<D, RG>;
+    constexpr int kThreads = 32 * kWarps * RG;
     constexpr int KD = D / 16;  // 16-wide k-steps over the head dimension
     constexpr int NT = D / 8;   // 8-wide tiles over the head dimension (and the largest rank)
     extern __shared__ __align__(128) uint8_t smem[];
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int tid = threadIdx.x, lane = tid & 31;
+    // row group of the block, warp in it
+    const int grp = RG == 1 ? 0 : (tid >> 5) / kWarps, warp = RG == 1 ? tid >> 5 : (tid >> 5) % kWarps;
     const int r4 = lane >> 2, c4 = lane & 3;  // mma fragment row and column pair
     const int mi = lane >> 3, mr = lane & 7;  // ldmatrix: matrix and row this lane addresses
-    uint4 *sq = reinterpret_cast<uint4 *>(smem + L::kQ);
-    float *sx_m = reinterpret_cast<float *>(smem + L::kX);       // [warp][row]
+    uint4 *sq = reinterpret_cast<uint4 *>(smem + L::kQ + grp * L::kQStride);
+    float *sx_m = reinterpret_cast<float *>(smem + L::kX) + grp * L::kXStride;  // [warp][row]
     float *sx_l = sx_m + 8 * kWarps;                             // [warp][row]
     uint32_t *sx_ref = reinterpret_cast<uint32_t *>(sx_l + 8 * kWarps);  // [row]
     const uint32_t zline = smem_u32(smem + L::kZero) + mr * 16;
     const uint32_t bar0 = smem_u32(smem + L::kBar);
-    // blocks [0, num_chunks * nrg): chunk blockIdx / nrg for row group
-    // blockIdx % nrg (the row groups of one chunk are neighbours, so they read
-    // its pieces from L2); then the dense-tail items
-    const int nprefix = p.num_chunks * p.nrg;
+    // blocks [0, num_chunks * nrgb): chunk blockIdx / nrgb for row groups
+    // RG (blockIdx % nrgb) + grp (the blocks of one chunk are neighbours, so
+    // they read its pieces from L2); then the dense-tail items, RG a block
+    const int nrgb = (p.nrg + RG - 1) / RG;
+    const int nprefix = p.num_chunks * nrgb;
     const bool is_tail = (int)blockIdx.x >= nprefix;
-    const int rgrp = is_tail ? 0 : (int)blockIdx.x % p.nrg;
+    const int rgrp = is_tail ? 0 : ((int)blockIdx.x % nrgb) * RG + grp;
+    const int item = is_tail ? ((int)blockIdx.x - nprefix) * RG + grp : 0;
+    // a group past the last row group or tail item only keeps the barriers
+    // (with one group per block there is none)
+    const bool active = RG == 1 || (is_tail ? item < p.num_tail_items : rgrp < p.nrg);
 
     pdl_trigger();
     // zero the slots, q~ and the zero line: reads past a piece's data then
     // see finite values (the copies below are ordered after these stores)
-    for (int i = tid; i < L::kBar / 16; i += kChunkThreads) reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
+    for (int i = tid; i < L::kBar / 16; i += kThreads) reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 
     ChunkDev ch = {};
     Pieces ps = {};
     int g = 0, ntok = 0, nrk = 0, nrv = 0;
     if (!is_tail) {
-        ch = p.chunks[blockIdx.x / p.nrg];
+        ch = p.chunks[blockIdx.x / nrgb];
         ps = pieces_of<D>(ch);
         g = ch.g;
         ntok = ch.ntok;
@@ -425,28 +440,34 @@ __global__ void __launch_bounds__(kChunkThreads)
     };
 
     uint32_t ref = 0u;  // this row's reference maximum (warp 0, lane c4 == 0), see publish_ref
-    int qi = 0, item = 0;
+    int qi = 0;
+    const bool leader = RG == 1 ? tid == 0 : warp == 0 && lane == 0;  // the group's first thread
     if (is_tail) {
-        // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense tail
-        item = (int)blockIdx.x - nprefix;
+        // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense
+        // tail, in slot grp (RG = 2) or both slots from slot 0 (RG = 1)
+        const uint32_t tbase = smem_u32(smem) + grp * kPieceBytes, tbar = bar0 + 8 * grp;
         const int S = p.tail_splits;
-        qi = item / (p.hkv * S);
-        const int sp = item % S;
-        g = (item / S) % p.hkv;
-        const int64_t o0 = p.tail_offsets[qi], o1 = p.tail_offsets[qi + 1];
-        const int T = (int)(o1 - o0);
-        if (sp == S - 1 && T > S * kTailTokens && tid == 0) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
+        int64_t o0 = 0;
+        int T = 0, sp = 0;
+        if (active) {
+            qi = item / (p.hkv * S);
+            sp = item % S;
+            g = (item / S) % p.hkv;
+            o0 = p.tail_offsets[qi];
+            T = (int)(p.tail_offsets[qi + 1] - o0);
+        }
+        if (sp == S - 1 && T > S * kTailTokens && leader) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
         const int t0 = sp * kTailTokens;
         ntok = max(0, min(t0 + kTailTokens, T) - t0);
         nrk = nrv = NT;
         // K then V: one box of kTailTokens rows x 8 columns per column group
         constexpr uint32_t kBox = kTailTokens * 16, kHalf = NT * kBox;
-        if (ntok > 0 && tid == 0) {
-            mbar_arrive_tx(bar0, 2 * kHalf);
+        if (ntok > 0 && leader) {
+            mbar_arrive_tx(tbar, 2 * kHalf);
 #pragma unroll 1
             for (int c = 0; c < NT; ++c) {
-                tma_load_3d(smem_u32(smem) + c * kBox, &tmap_k, 8 * c, g, (int)(o0 + t0), bar0);
-                tma_load_3d(smem_u32(smem) + kHalf + c * kBox, &tmap_v, 8 * c, g, (int)(o0 + t0), bar0);
+                tma_load_3d(tbase + c * kBox, &tmap_k, 8 * c, g, (int)(o0 + t0), tbar);
+                tma_load_3d(tbase + kHalf + c * kBox, &tmap_v, 8 * c, g, (int)(o0 + t0), tbar);
             }
         }
         // q~ = scale * log2(e) * q of the G heads of query qi, as score A fragments
@@ -469,15 +490,15 @@ __global__ void __launch_bounds__(kChunkThreads)
             sq[ks * 32 + lane] = f;
         }
         __syncthreads();
-        if (ntok > 0) mbar_wait(bar0, 0, p.status);
+        if (ntok > 0) mbar_wait(tbar, 0, p.status);
         // the item's tokens in units of kTailTokens / kWarps, one per warp
         constexpr int kTU = kTailTokens / kWarps;
         static_assert(kTU == 16 || kTU == 32, "tail units of 16 or 32 tokens");
         const int tb = kTU * warp;
         if (tb < ntok) {
             tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTU>{},
-                 std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{}, smem_u32(smem),
-                 128, smem_u32(smem) + kHalf, 128, tb, kTailTokens / 8, ntok);
+                 std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{}, tbase, 128,
+                 tbase + kHalf, 128, tb, kTailTokens / 8, ntok);
             if (warp == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
         }
     } else {
@@ -505,7 +526,7 @@ __global__ void __launch_bounds__(kChunkThreads)
                 const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, nrk);
                 // (a piece never holds more 16-rank steps than q~ has: ranks <= D)
                 constexpr int kNKMax = L::kRanksPerPiece / 16 < KD ? L::kRanksPerPiece / 16 : KD;
-                dispatch(std::integral_constant<int, kNKMax>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
+                if (active) dispatch(std::integral_constant<int, kNKMax>{}, (r1 - r0 + 1) / 2, [&](auto nkc) {
                     constexpr int NJ = (decltype(nkc)::value + kWarps - 1) / kWarps;  // steps per warp
                     float acc[NJ][2][4];
 #pragma unroll
@@ -549,7 +570,7 @@ __global__ void __launch_bounds__(kChunkThreads)
             const int nv = min(ps.tpp * kTile, ntok - t0);  // valid tokens of this piece
             const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;
             const uint32_t vb = slot + (uint32_t)r8 * nrk * 16;
-            dispatch(std::integral_constant<int, NT / 2>{}, r16, [&](auto r16c) {
+            if (active) dispatch(std::integral_constant<int, NT / 2>{}, r16, [&](auto r16c) {
                 using std::integral_constant;
                 if constexpr (decltype(r16c)::value <= 4) {
                     // up to 64 ranks: whole tiles round-robin over the warps
@@ -592,11 +613,14 @@ __global__ void __launch_bounds__(kChunkThreads)
         // other warps' scaled values pass through a slot that is free by now:
         // a chunk's P^V fits one piece (ranks <= d), so after its last C
         // piece no copy targets that slot; a tail item's data is consumed.
-        static_assert((kWarps - 1) * (D / 8) * 32 * 16 <= kPieceBytes, "warp values fit a slot");
+        // (A tail group's values pass through its own slot.)
+        constexpr int kXV = (kWarps - 1) * (D / 8) * 32 * 16;  // one group's exchange
+        static_assert(RG * kXV <= kPieceBytes, "warp values fit a slot");
         static_assert(L::kRanksPerPiece >= D, "P^V of any rank is one piece");
         const float sc = exp2_diff(m_w, M);
-        const int free_slot = is_tail ? 0 : ((ps.npk + ps.nc - 1) & 1);
-        float4 *xv = reinterpret_cast<float4 *>(smem + free_slot * kPieceBytes);
+        const int free_slot = (ps.npk + ps.nc - 1) & 1;
+        float4 *xv = reinterpret_cast<float4 *>(smem + (is_tail ? grp * kPieceBytes
+                                                                : free_slot * kPieceBytes + grp * kXV));
         if (warp > 0) {
 #pragma unroll
             for (int n = 0; n < NT; ++n)
@@ -631,7 +655,7 @@ __global__ void __launch_bounds__(kChunkThreads)
         // the values are already in the head dimension: o = v~ (warp 0 adds all of it)
         rec_idx = p.tail_rec_base + item;
         row0 = qi * p.G;
-        nrows = p.G;
+        nrows = active ? p.G : 0;
         float ov[NT][2];
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
@@ -641,9 +665,9 @@ __global__ void __launch_bounds__(kChunkThreads)
         direct = warp == 0 ? add_part<D, NT>(p, g, lane, 0, ov, M, lsum, refb, true, row0, nrows, rec_idx)
                            : __all_sync(0xffffffffu, r4 >= nrows || !(M - (refb ? ref_dec(refb) : M) > kDirectMax));
     } else {
-        rec_idx = (int64_t)blockIdx.x;
+        rec_idx = RG == 1 ? (int64_t)blockIdx.x : (int64_t)(blockIdx.x / nrgb) * p.nrg + rgrp;
         row0 = 8 * rgrp;
-        nrows = min(8, p.rows_g - row0);
+        nrows = active ? min(8, p.rows_g - row0) : 0;
         // warp 0 stages the merged v~ as the back-projection's A fragments (rows
         // 0-7 hi, 8-15 lo) in the q~ area, so that the rank loop below stays rolled
         if (warp == 0) {
@@ -669,7 +693,7 @@ __global__ void __launch_bounds__(kChunkThreads)
             // rank 8-groups [r0, r1) of this piece: 16-rank k-steps of v~
             const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, nrv);
 #pragma unroll 1
-            for (int ks = r0 / 2; 2 * ks < r1; ++ks) {
+            for (int ks = r0 / 2; active && 2 * ks < r1; ++ks) {
                 const uint4 a4 = sq[ks * 32 + lane];
                 const uint32_t a[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
@@ -696,7 +720,7 @@ __global__ void __launch_bounds__(kChunkThreads)
 
     // ---- an outlier's record is listed; the finish grid that follows
     // (programmatic dependent launch) sees every reduction and record
-    if (tid == 0 && !direct) {
+    if (leader && active && !direct) {
         // in the list of every row group the item's rows touch
         for (int rg = row0 / 8; rg <= (row0 + nrows - 1) / 8; ++rg) {
             const int gr = g * p.nrg + rg;
@@ -719,40 +743,51 @@ __global__ void __launch_bounds__(32) finish_kernel(const __grid_constant__ Deco
 
 }  // namespace
 
+namespace {
+template <int D, int RG>
+cudaError_t launch_chunk_grid(cudaLaunchConfig_t cfg, const DecodeParams &p, const CUtensorMap &mk,
+                              const CUtensorMap &mv)
+{
+    using L = CLay<D, RG>;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(chunk_kernel<D, RG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             L::kTotal);
+        if (e != cudaSuccess) return e;
+        // several thread blocks per SM need the largest shared-memory carveout
+        e = cudaFuncSetAttribute(chunk_kernel<D, RG>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    const int nrgb = (p.nrg + RG - 1) / RG;
+    cfg.gridDim = dim3(p.num_chunks * nrgb + (p.has_tail ? (p.num_tail_items + RG - 1) / RG : 0));
+    cfg.blockDim = dim3(32 * kWarps * RG);
+    cfg.dynamicSmemBytes = (size_t)L::kTotal;
+    return cudaLaunchKernelEx(&cfg, chunk_kernel<D, RG>, p, mk, mv);
+}
+}  // namespace
+
 cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void *tmap_v, cudaStream_t stream)
 {
     const CUtensorMap &mk = *static_cast<const CUtensorMap *>(tmap_k);
     const CUtensorMap &mv = *static_cast<const CUtensorMap *>(tmap_v);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.num_chunks * p.nrg + (p.has_tail ? p.num_tail_items : 0));
-    cfg.blockDim = dim3(kChunkThreads);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    static int configured[2] = {0, 0};
-    const int w = p.d == 64 ? 0 : 1;
-    const void *fn = w == 0 ? reinterpret_cast<const void *>(chunk_kernel<64>)
-                            : reinterpret_cast<const void *>(chunk_kernel<128>);
-    const int smem = w == 0 ? CLay<64>::kTotal : CLay<128>::kTotal;
-    if (!configured[w]) {
-        cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
-        // several thread blocks per SM need the largest shared-memory carveout
-        e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-        if (e != cudaSuccess) return e;
-        configured[w] = 1;
-    }
-    cfg.dynamicSmemBytes = (size_t)smem;
-    cudaError_t e = w == 0 ? cudaLaunchKernelEx(&cfg, chunk_kernel<64>, p, mk, mv)
-                           : cudaLaunchKernelEx(&cfg, chunk_kernel<128>, p, mk, mv);
+    // two row groups per block once a KV head has more than 8 query rows
+    const bool two = p.nrg >= 2;
+    cudaError_t e = p.d == 64 ? (two ? launch_chunk_grid<64, 2>(cfg, p, mk, mv) : launch_chunk_grid<64, 1>(cfg, p, mk, mv))
+                              : (two ? launch_chunk_grid<128, 2>(cfg, p, mk, mv)
+                                     : launch_chunk_grid<128, 1>(cfg, p, mk, mv));
     if (e != cudaSuccess) return e;
     cfg.gridDim = dim3(p.hkv * p.nrg);
     cfg.blockDim = dim3(32);
     cfg.dynamicSmemBytes = 0;
-    return w == 0 ? cudaLaunchKernelEx(&cfg, finish_kernel<64>, p) : cudaLaunchKernelEx(&cfg, finish_kernel<128>, p);
+    return p.d == 64 ? cudaLaunchKernelEx(&cfg, finish_kernel<64>, p) : cudaLaunchKernelEx(&cfg, finish_kernel<128>, p);
 }
 
 }  // namespace milo
