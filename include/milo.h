@@ -143,13 +143,14 @@ milo_status_t milo_partition_prefix(const milo_block_table_t *table,
                                     int32_t *num_slots);
 
 /*
- * Host-only: the work list of the short-block decode (calls with at most 8
- * query rows per KV head).  Every prefix entry, KV-head-major then in block
+ * Host-only: the work list of the short-block decode (plans with at most 8
+ * query heads per KV head).  Every prefix entry, KV-head-major then in block
  * order, is cut into the fewest token ranges of at most 1024 tokens whose
  * coefficient rows (C^K and C^V at ranks rounded up to 8, tokens rounded up
  * to 8, bf16) fit 128 KB, of equal length in multiples of 32 tokens (the
  * last range takes the remainder); each range is one thread block of the
- * decode grid.
+ * decode grid per row group of 8 query rows (two row groups share a block
+ * once a KV head has more than 8 rows).
  *   chunk_entry/chunk_t0/chunk_t1: host arrays of capacity `max_chunks`
  *     (entry index b * num_kv_heads + g, token range [t0, t1)); all may be
  *     NULL to query the count.

@@ -1,7 +1,9 @@
-// milo_chunk.cu -- the split-K decode of milo_decode.cu for up to 8 query rows
-// per KV head (batch x heads of one KV head <= 8): one thread block of kWarps
-// warps per chunk (three blocks per SM at head dimension 128), each chunk
-// streamed through two shared-memory slots that all its warps read.
+// milo_chunk.cu -- the split-K decode for up to 8 query heads per KV head
+// (G <= 8): one thread block of kWarps warps per chunk and row group of 8
+// query rows (batch x G rows per KV head), or of 2 kWarps warps per chunk and
+// pair of row groups once a KV head has more than 8 rows; three blocks per
+// SM at head dimension 128.  Each chunk is streamed through two
+// shared-memory slots that all the block's warps read.
 //
 // A chunk is a token range of one prefix entry (block b, KV head g).  Its
 // block walks a fixed sequence of pieces, each at most kPieceBytes and
@@ -26,9 +28,10 @@
 // kTailTokens rows each, landing as cores [column group][token group]) and
 // runs the C steps on them with q~ = scale * log2(e) * q, a share of the
 // tokens per warp; its values are already o.  Every item then adds its result
-// into fp32 accumulators of its KV head (see add_part) and exits; a small
-// finish grid chained by programmatic dependent launch (one warp per KV head)
-// writes the normalised output.  No block waits on another.
+// into fp32 accumulators of its KV head's rows (see add_part) and exits; a
+// small finish grid chained by programmatic dependent launch (one warp per KV
+// head and row group) writes the normalised output.  No block waits on
+// another.
 //
 // Shared-memory cores are 8 rows x 16 bytes (rows = tokens or ranks).  Every
 // wait is bounded (~2 s) and sets MILO_ERR_TIMEOUT.

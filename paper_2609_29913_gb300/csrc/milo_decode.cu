@@ -8,10 +8,10 @@
 // split softmax (Eq. 1 is associative over token partitions once each part
 // carries its running max and sum).
 //
-// This file holds the persistent kernel, used when a KV head has more than 8
-// query rows (several row groups share every coefficient tile read), and the
-// merge kernel.  Up to 8 rows per KV head take the short-block kernel of
-// milo_chunk.cu.
+// This file holds the persistent kernel, used when more than 8 query heads
+// share a KV head (G > 8; several row groups share every coefficient tile
+// read) or a plan has no prefix, and the merge kernel.  Every other call
+// takes the chunk grid of milo_chunk.cu.
 //
 // Persistent kernel, one thread block per SM, two roles:
 //   producer   (warp 0, one lane): turns the block's static list of prefix
