@@ -298,6 +298,20 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
             if (ps.total() > 1) issue(1);
         }
     }
+    // warm L2 with the group's q rows, the first load after the wait (a
+    // prefetch reads nothing into the block, so it may precede the wait)
+    if (warp == 0 && lane < 16 && active) {
+        const int r = lane >> 1;
+        int qrow = -1, gq = g;
+        if (is_tail) {
+            gq = (item / p.tail_splits) % p.hkv;
+            if (r < p.G) qrow = item / (p.hkv * p.tail_splits) * p.G + r;
+        } else if (8 * rgrp + r < p.rows_g) {
+            qrow = 8 * rgrp + r;
+        }
+        if (qrow >= 0)
+            prefetch_l2(p.q + ((int64_t)(qrow / p.G) * p.hq + gq * p.G + qrow % p.G) * D + (lane & 1) * (D / 2));
+    }
     __syncthreads();
     pdl_wait();  // q, the tails and the accumulators belong to the preceding grids until here
 
