@@ -190,6 +190,23 @@ def reference_arm(args, cfg, W):
     print(json.dumps(line), flush=True)
 
 
+def max_over_ranks(x, dist, device):
+    """The largest of every rank's x (a time in ms); x itself without a
+    process group.  Replicas report the slowest rank's time."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(world, tokens_per_rank, ms_step):
+    """Whole-job tokens/s: every replica attends tokens_per_rank per step, and
+    the step takes the slowest rank's ms_step."""
+    return world * tokens_per_rank / (ms_step * 1e-3)
+
+
 def pack_tensors(tensors, dev):
     """Copy device tensors (None allowed) into one byte buffer, each at a
     256-byte boundary; returns the buffer and a view of it per tensor."""
@@ -339,11 +356,7 @@ def main():
     if dist:
         dist.barrier()
     ms_total = start.elapsed_time(stop)
-    ms_step = ms_total / args.steps
-    if dist:
-        t = torch.tensor([ms_step], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_step = float(t.item())
+    ms_step = max_over_ranks(ms_total / args.steps, dist, dev)
     for p in plans:
         assert p.status() == 0, "device status word set during the timed region"
 
@@ -396,11 +409,7 @@ def main():
             e2e_step(stream)
     e1.record(stream)
     torch.cuda.synchronize()
-    e_ms = e0.elapsed_time(e1) / e_steps
-    if dist:
-        t = torch.tensor([e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e_ms = float(t.item())
+    e_ms = max_over_ranks(e0.elapsed_time(e1) / e_steps, dist, dev)
 
     # ---- CPU oracle baseline (rank 0, N = 1 only)
     cpu = None
@@ -422,7 +431,7 @@ def main():
             traffic = entry["dram_bytes_per_launch"]
     except Exception:
         traffic = None
-    value = world * tokens / (ms_step * 1e-3)
+    value = replica_throughput(world, tokens, ms_step)
     # up to 8 query heads per KV head: the chunk grid (a block per prefix
     # chunk and row group of 8 query rows, and per tail item, adding into
     # per-row accumulators) and its finish grid; more: the persistent kernel
@@ -455,7 +464,7 @@ def main():
                      "per_launch_bytes": alg_bytes // cfg.layers,
                      "per_launch_us": ms_step * 1e3 / cfg.layers},
         "cpu_baseline": cpu,
-        "e2e": {"value": world * tokens / (e_ms * 1e-3), "unit": UNIT,
+        "e2e": {"value": replica_throughput(world, tokens, e_ms), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
                 "how": "per step: every layer's q and tails copied from pinned host memory in %d copies on a "
                        "second stream, each releasing a captured graph of its layers' calls, then one copy "
