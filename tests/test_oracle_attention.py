@@ -229,6 +229,40 @@ def test_block_order_permutation_invariance(oracle):
     np.testing.assert_allclose(oracle.attention(**q), base, rtol=1e-13, atol=1e-14)
 
 
+@pytest.mark.parametrize("cut", [1, 3, 4])
+def test_block_split_invariance(oracle, cut):
+    """Cutting a block's tokens into two table entries that share its P^K and
+    P^V (the C rows split at the cut) leaves the attention unchanged: the
+    softmax of Eq. 1 does not depend on how the tokens are grouped, which is
+    what the split-K decode and its log-sum-exp merge rely on."""
+    rng = np.random.default_rng(12)
+    p = make_problem(rng, **CASES[1])
+    base = oracle.attention(**p)
+    hkv = p["num_kv_heads"]
+    b = 1  # the 5-token block
+    n = int(p["block_len"][b])
+    assert 0 < cut < n
+    lens = list(p["block_len"][:b]) + [cut, n - cut] + list(p["block_len"][b + 1:])
+    q = dict(p)
+    q["block_len"] = np.array(lens, np.int32)
+    cols = {k: [] for k in ("rank_k", "rank_v", "off_ck", "off_pk", "off_cv", "off_pv")}
+    for bb in range(len(p["block_len"])):
+        parts = [(0, cut), (cut, n)] if bb == b else [(0, int(p["block_len"][bb]))]
+        for t0, _ in parts:
+            for g in range(hkv):
+                e = bb * hkv + g
+                rk, rv = int(p["rank_k"][e]), int(p["rank_v"][e])
+                cols["rank_k"].append(rk)
+                cols["rank_v"].append(rv)
+                cols["off_ck"].append(int(p["off_ck"][e]) + t0 * rk)  # C is row-major [n][r]
+                cols["off_cv"].append(int(p["off_cv"][e]) + t0 * rv)
+                cols["off_pk"].append(int(p["off_pk"][e]))
+                cols["off_pv"].append(int(p["off_pv"][e]))
+    for k, v in cols.items():
+        q[k] = np.array(v, np.int32 if k.startswith("rank") else np.int64)
+    np.testing.assert_allclose(oracle.attention(**q), base, rtol=1e-13, atol=1e-14)
+
+
 def test_tail_equals_identity_basis_block(oracle):
     """A dense tail K, V is the same as a full-rank block with C = K, P = I."""
     rng = np.random.default_rng(12)
