@@ -178,7 +178,8 @@ __device__ void finish_head(const DecodeParams &p, int g, int rg, int lane)
 // columns 8 (n0 + n) + 2 c4, + 1 of row r4 (ov[n]), for rows arow = row0 + r4
 // with r4 < nrows.  M is the item's row maximum, lsum its row sum (used when
 // with_l), refb the row's reference (encoded; 0 = unset).  Returns whether the
-// item went to the accumulators (the same in both warps: their inputs agree);
+// item went to the accumulators (the same in every warp of the row group:
+// their inputs agree);
 // otherwise the warp wrote its columns of the item's record.
 template <int D, int NC>
 __device__ bool add_part(const DecodeParams &p, int g, int lane, int n0, const float (&ov)[NC][2], float M,
@@ -213,7 +214,9 @@ __device__ bool add_part(const DecodeParams &p, int g, int lane, int n0, const f
 
 // RG row groups of 8 query rows per block, kWarps warps each: the groups
 // share every piece (RG = 2 for calls with several row groups per KV head).
-// A tail block holds RG tail items, one per group, in slot g of group g.
+// A tail block holds RG tail items, one per group; with RG = 2 group i's
+// item sits in slot i, with RG = 1 it starts at slot 0.  "warp" below is the
+// warp's index within its row group.
 template <int D, int RG>
 __global__ void __launch_bounds__(32 * kWarps * RG)
     chunk_kernel(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tmap_k,
@@ -443,7 +446,7 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
     };
 
     const int np = ps.total();
-    // wait for piece k (both warps); afterwards release its slot and bring
+    // wait for piece k (every warp); afterwards release its slot and bring
     // piece k + 2 into it
     auto wait_piece = [&](int k) {
         mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
@@ -626,11 +629,12 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
     for (int w = 0; w < kWarps; ++w) lsum += sx_l[8 * w + r4] * exp2_diff(sx_m[8 * w + r4], M);
     const uint32_t refb = sx_ref[r4];
     {
-        // v~ = sum over warps of 2^(m_w - M) v~_w, gathered in warp 0.  The
-        // other warps' scaled values pass through a slot that is free by now:
-        // a chunk's P^V fits one piece (ranks <= d), so after its last C
-        // piece no copy targets that slot; a tail item's data is consumed.
-        // (A tail group's values pass through its own slot.)
+        // v~ = sum over the group's warps of 2^(m_w - M) v~_w, gathered in its
+        // warp 0.  The other warps' scaled values pass through a slot that is
+        // free by now: a chunk's P^V fits one piece (ranks <= d), so after its
+        // last C piece no copy targets that slot (each group has its own part
+        // of it); a tail group's values pass through its own slot, whose data
+        // it has consumed.
         constexpr int kXV = (kWarps - 1) * (D / 8) * 32 * 16;  // one group's exchange
         static_assert(RG * kXV <= kPieceBytes, "warp values fit a slot");
         static_assert(L::kRanksPerPiece >= D, "P^V of any rank is one piece");

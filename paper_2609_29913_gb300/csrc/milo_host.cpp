@@ -639,7 +639,6 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.chunks = plan->chunks;
     prm.num_chunks = c.chunked ? plan->num_chunks : 0;
     if (c.chunked) {
-        prm.num_slots = plan->num_chunks;
         prm.tail_rec_base = (int64_t)plan->num_chunks * c.nrg;
         // the record lists follow the records
         prm.list_cap = (int)c.list_cap;
