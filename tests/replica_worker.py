@@ -22,7 +22,9 @@ def main():
     ms = bench.max_over_ranks(local_ms, dist, "cpu")
     value = bench.replica_throughput(world, int(sys.argv[1]), ms)
     dist.barrier()
-    print(json.dumps({"rank": rank, "world": world, "local_ms": local_ms, "ms": ms, "value": value}), flush=True)
+    # one file per rank: the ranks' standard outputs interleave
+    with open(os.path.join(sys.argv[2], f"rank{rank}.json"), "w") as f:
+        json.dump({"rank": rank, "world": world, "local_ms": local_ms, "ms": ms, "value": value}, f)
     dist.destroy_process_group()
 
 

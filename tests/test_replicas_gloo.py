@@ -21,15 +21,18 @@ def _free_port():
         return s.getsockname()[1]
 
 
-def test_two_replicas_report_the_slowest_rank_and_all_tokens():
+def test_two_replicas_report_the_slowest_rank_and_all_tokens(tmp_path):
     tokens = 924672
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node=2",
            "--master-addr=127.0.0.1", f"--master-port={_free_port()}",
-           os.path.join(ROOT, "tests", "replica_worker.py"), str(tokens)]
+           os.path.join(ROOT, "tests", "replica_worker.py"), str(tokens), str(tmp_path)]
     env = dict(os.environ, OMP_NUM_THREADS="1")
     res = subprocess.run(cmd, capture_output=True, text=True, timeout=300, env=env, cwd=ROOT)
     assert res.returncode == 0, res.stderr[-2000:]
-    lines = [json.loads(x) for x in res.stdout.splitlines() if x.startswith("{")]
+    lines = []
+    for r in range(2):
+        with open(tmp_path / f"rank{r}.json") as f:
+            lines.append(json.load(f))
     assert sorted(d["rank"] for d in lines) == [0, 1]
     slowest = max(d["local_ms"] for d in lines)
     for d in lines:
