@@ -62,6 +62,9 @@ CASES = {
     "tail-only": (14, 2, 64, [], (8,), 2, [5, 300], False),
     "batch64-multipass": (28, 4, 128, [128, 64], (16, 128, 40), 64, [33] * 64, True),
     "batch9-odd-groups": (21, 3, 64, [96, 40], (7, 64), 9, list(range(1, 10)), True),
+    # 21 rows per KV head: 3 row groups (two-group blocks, the last half
+    # empty) and 9 tail items (two to a block, the last alone), at d = 128
+    "d128-odd-row-groups": (21, 3, 128, [512, 77, 300], (16, 64, 96, 128), 3, [5, 60, 1], True),
     "rank0": (4, 2, 64, [50, 70], (0,), 1, [3], True),
 }
 
