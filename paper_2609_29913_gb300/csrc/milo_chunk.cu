@@ -770,15 +770,16 @@ cudaError_t launch_chunk_grid(cudaLaunchConfig_t cfg, const DecodeParams &p, con
                               const CUtensorMap &mv)
 {
     using L = CLay<D, RG>;
-    static bool configured = false;
-    if (!configured) {
+    static bool configured[kMaxDevices] = {};
+    const int dev = attribute_slot();
+    if (dev < 0 || !configured[dev]) {
         cudaError_t e = cudaFuncSetAttribute(chunk_kernel<D, RG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              L::kTotal);
         if (e != cudaSuccess) return e;
         // several thread blocks per SM need the largest shared-memory carveout
         e = cudaFuncSetAttribute(chunk_kernel<D, RG>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
         if (e != cudaSuccess) return e;
-        configured = true;
+        if (dev >= 0) configured[dev] = true;
     }
     const int nrgb = (p.nrg + RG - 1) / RG;
     cfg.gridDim = dim3(p.num_chunks * nrgb + (p.has_tail ? (p.num_tail_items + RG - 1) / RG : 0));

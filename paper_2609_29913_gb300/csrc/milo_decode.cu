@@ -1031,15 +1031,16 @@ cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k, const void 
     cfg.numAttrs = 1;
     const CUtensorMap &mk = *static_cast<const CUtensorMap *>(tmap_k);
     const CUtensorMap &mv = *static_cast<const CUtensorMap *>(tmap_v);
-    static int configured[2] = {0, 0};  // largest dynamic smem size set per kernel
+    static int configured[kMaxDevices][2] = {};  // largest dynamic smem size set, per device and kernel
     const int which = p.d == 64 ? 0 : 1;
-    if (smem_bytes > configured[which]) {
+    const int dev = attribute_slot();
+    if (p.num_chunks == 0 && (dev < 0 || smem_bytes > configured[dev][which])) {
         cudaError_t e = which == 0 ? cudaFuncSetAttribute(decode_kernel<64>,
                                                           cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes)
                                    : cudaFuncSetAttribute(decode_kernel<128>,
                                                           cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
         if (e != cudaSuccess) return e;
-        configured[which] = smem_bytes;
+        if (dev >= 0) configured[dev][which] = smem_bytes;
     }
     cudaError_t e = p.num_chunks > 0 ? launch_chunks(p, tmap_k, tmap_v, stream)
                     : which == 0 ? cudaLaunchKernelEx(&cfg, decode_kernel<64>, p, mk, mv)

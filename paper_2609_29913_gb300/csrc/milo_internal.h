@@ -111,6 +111,18 @@ struct DecodeParams {
     int list_cap;                   // list entries per (KV head, row group)
 };
 
+// Kernel attributes (shared-memory size, carveout) belong to a device: the
+// launchers set them once per device, tracked in tables of kMaxDevices.
+constexpr int kMaxDevices = 64;
+// The current device, or -1 when it cannot be read or lies past the tables
+// (the caller then sets the attributes on every launch).
+inline int attribute_slot()
+{
+    int d = -1;
+    if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return -1;
+    return d;
+}
+
 // Launchers implemented in the .cu files.
 cudaError_t launch_pack(const void *arena, const EntryDev *entries_dev,
                         const int64_t *logical_offsets_dev, int num_entries,
