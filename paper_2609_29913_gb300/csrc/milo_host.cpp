@@ -545,10 +545,13 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     // one record per prefix chunk and row group (the short-block decode), or
     // per run and row group (the persistent kernel); then the tail items.
     // The short-block decode also lists records: int4 [Hkv][nrg][list_cap],
-    // list_cap bounding the items whose rows meet one row group.
+    // list_cap bounding the items whose rows meet one row group: the KV
+    // head's chunks, and the tail items of the queries whose G rows meet the
+    // group's 8 rows [8k, 8k + 8), of which there are at most 7 / G + 2.
     const int64_t prefix = c.chunked ? (int64_t)p->num_chunks * c.nrg : (int64_t)p->num_slots * c.nrg;
     c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
-    c.list_cap = c.chunked ? (int64_t)p->max_head_chunks + (int64_t)batch * c.S : 0;
+    const int64_t queries_per_group = std::min<int64_t>(batch, 7 / p->G + 2);
+    c.list_cap = c.chunked ? (int64_t)p->max_head_chunks + queries_per_group * c.S : 0;
     c.list_bytes = 16 * (int64_t)p->hkv * c.nrg * c.list_cap;
 
     return c;
