@@ -269,12 +269,15 @@ class Prefix:
         tail_offsets int64 cuda tensor [batch + 1].  Returns fp32 out."""
         import torch
         batch = int(q.shape[0])
+        made = []  # buffers allocated here, on torch's current stream
         if out is None:
             out = torch.empty((batch, self.num_q_heads, self.head_dim), device=q.device,
                               dtype=torch.float32)
+            made.append(out)
         need = self.workspace_size(batch, max_tail_tokens)
         if workspace is None:
             workspace = torch.empty(need, device=q.device, dtype=torch.uint8)
+            made.append(workspace)
         tail_rows = int(tail_k.shape[0]) if (tail_k is not None and max_tail_tokens > 0) else 0
         milo_attn_decode(self.plan, q.data_ptr(), batch,
                          tail_k.data_ptr() if tail_rows else 0,
@@ -283,6 +286,11 @@ class Prefix:
                          tail_rows, max_tail_tokens if tail_rows else 0, softmax_scale,
                          out.data_ptr(), workspace.data_ptr(), workspace.numel() * workspace.element_size(),
                          stream)
+        if isinstance(stream, torch.cuda.Stream):
+            # the call runs on `stream`: keep the caching allocator from
+            # handing these buffers out again before it has finished
+            for t in made:
+                t.record_stream(stream)
         return out
 
     def status(self, stream=None, clear=False) -> int:
