@@ -148,7 +148,8 @@ milo_status_t milo_partition_prefix(const milo_block_table_t *table,
  * order, is cut into the fewest token ranges of at most 1024 tokens whose
  * coefficient rows (C^K and C^V at ranks rounded up to 8, tokens rounded up
  * to 8, bf16) fit 128 KB, of equal length in multiples of 32 tokens (the
- * last range takes the remainder); each range is one thread block of the
+ * last range takes the remainder; an entry of rank 0 in K and V, which has
+ * no coefficient rows, is cut into 32-token ranges); each range is one thread block of the
  * decode grid per row group of 8 query rows (two row groups share a block
  * once a KV head has more than 8 rows).
  *   chunk_entry/chunk_t0/chunk_t1: host arrays of capacity `max_chunks`

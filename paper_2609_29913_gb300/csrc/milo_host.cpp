@@ -196,7 +196,11 @@ void for_each_chunk(const milo_block_table_t *t, F &&f)
             // the fewest chunks within the byte budget, then equal token
             // ranges (multiples of 32), so that an entry's chunks take
             // about equally long
-            const int most = std::max(32, std::min(kChunkMaxTok, kChunkBytes / ((rk8 + rv8) * 2) / 32 * 32));
+            // (an entry of rank 0 in K and V has no coefficient rows: its
+            // tokens go in 32-token ranges, whose pieces copy nothing)
+            const int row_bytes = (rk8 + rv8) * 2;
+            const int most = row_bytes > 0 ? std::max(32, std::min(kChunkMaxTok, kChunkBytes / row_bytes / 32 * 32))
+                                           : 32;
             const int nch = std::max(1, (n + most - 1) / most);
             const int tok = ((n + nch - 1) / nch + 31) / 32 * 32;
             for (int t0 = 0; t0 < n; t0 += tok) f(e, g, t0, std::min(n, t0 + tok));

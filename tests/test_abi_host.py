@@ -181,6 +181,7 @@ def test_partition_balances_bytes(milo):
     ([512] * 64, "choice", 4, 128),
     ([7, 129, 1, 64, 65, 300, 1024, 2048], "rand", 2, 64),
     ([512, 33, 1000] * 3, "rand", 3, 128),
+    ([50, 70, 2048, 1], "zero", 2, 64),
 ])
 def test_chunks_cover_every_token_once_within_budget(milo, shape):
     """The short-block decode's work list (milo_chunk_prefix): KV-head-major,
@@ -196,6 +197,9 @@ def test_chunks_cover_every_token_once_within_budget(milo, shape):
     else:
         rk = rng.integers(0, d + 1, size=nb * hkv)
     rv = rng.integers(0, d + 1, size=nb * hkv)
+    if law == "zero":  # entries of rank 0 in both K and V: tokens without coefficient rows
+        rk = np.zeros(nb * hkv, dtype=np.int64)
+        rv = np.zeros(nb * hkv, dtype=np.int64)
     t = ht(milo, **table(bl, rk, rv, hkv=hkv, d=d))
     ch = milo.milo_chunk_prefix(t)
     r8 = lambda r: (int(r) + 7) // 8 * 8
@@ -220,7 +224,7 @@ def test_chunks_cover_every_token_once_within_budget(milo, shape):
             assert all(a[1] == c[0] for a, c in zip(ranges, ranges[1:]))
             # fewest ranges within the byte budget, and equal lengths
             row = (r8(rk[e]) + r8(rv[e])) * 2
-            most = max(32, min(1024, 131072 // row // 32 * 32))
+            most = max(32, min(1024, 131072 // row // 32 * 32)) if row else 32
             assert len(ranges) == -(-n // most)
             lens = [c - a for a, c in ranges]
             assert all(L == lens[0] for L in lens[:-1]) and lens[-1] <= lens[0]
