@@ -69,7 +69,7 @@ CONFIGS = [
            description="28 layers, 28/4 heads, d=128, 64x512 prefix, r in {16..128}, batch 1, tail 256"),
     Config("qwen7b-28L-32k-b64", 28, 28, 4, 128, 64, 512, "choice",
            (16, 32, 64, 96, 128), batch=64, tail_len=512, seed=1002,
-           description="config 1 prefix shared by 64 queries, tail 512 each"),
+           description="the qwen7b-28L-32k-b1 prefix shared by 64 queries, tail 512 each"),
     Config("qwen14b-48L-128k-b16", 48, 40, 8, 128, 256, 512,
            "entropy_multinomial", batch=16, tail_len=1024, seed=1003,
            description="48 layers, 40/8 heads, 256x512 prefix, r 32..128 mean 64, batch 16, tail 1024"),
@@ -77,6 +77,14 @@ CONFIGS = [
            tail_law="uniform", tail_range=(128, 4096), seed=1004,
            description="1 layer, 2048x512 prefix, geometric ranks 4..128 + 5% full rank, batch 8, tails U[128,4096]"),
 ]
+
+
+def by_name(name: str) -> Config:
+    """The workload called `name` (e.g. "qwen7b-28L-32k-b1")."""
+    for cfg in CONFIGS:
+        if cfg.name == name:
+            return cfg
+    raise KeyError(name)
 
 
 def _np_rng(seed: int, layer: int) -> np.random.Generator:

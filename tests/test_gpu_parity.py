@@ -357,30 +357,31 @@ def oracle_subset(env, layer, queries, g):
     return env["oracle"].attention(**args)
 
 
-def test_config0_full(env):
+def test_qwen05b_one_layer_full(env):
     W = env["W"]
-    layer = W.make_config_layer(W.CONFIGS[0], 0, device="cuda")
+    layer = W.make_config_layer(W.by_name("qwen0.5b-1L-2k"), 0, device="cuda")
     out, _ = decode(env, layer)
-    compare(out.cpu().numpy(), env["oracle"].attention(**layer.to_numpy_bits()), "config0")
+    compare(out.cpu().numpy(), env["oracle"].attention(**layer.to_numpy_bits()), "qwen0.5b-1L-2k")
 
 
 @pytest.mark.parametrize("layer_idx", [0, 27])
-def test_config1_layers_full(env, layer_idx):
+def test_qwen7b_batch1_layers_full(env, layer_idx):
     W = env["W"]
-    layer = W.make_config_layer(W.CONFIGS[1], layer_idx, device="cuda")
+    layer = W.make_config_layer(W.by_name("qwen7b-28L-32k-b1"), layer_idx, device="cuda")
     out, _ = decode(env, layer)
-    compare(out.cpu().numpy(), env["oracle"].attention(**layer.to_numpy_bits()), f"config1 L{layer_idx}")
+    compare(out.cpu().numpy(), env["oracle"].attention(**layer.to_numpy_bits()), f"qwen7b-28L-32k-b1 L{layer_idx}")
 
 
-@pytest.mark.parametrize("cfg_idx,queries,heads", [(2, [0, 63], [0, 3]), (3, [0, 15], [0, 7]),
-                                                    (4, [0, 5], [1])])
-def test_large_configs_sampled(env, cfg_idx, queries, heads):
+@pytest.mark.parametrize("name,queries,heads", [("qwen7b-28L-32k-b64", [0, 63], [0, 3]),
+                                                ("qwen14b-48L-128k-b16", [0, 15], [0, 7]),
+                                                ("qwen7b-1L-1M-b8", [0, 5], [1])])
+def test_batched_workloads_sampled(env, name, queries, heads):
     W = env["W"]
-    layer = W.make_config_layer(W.CONFIGS[cfg_idx], 0, device="cuda")
+    layer = W.make_config_layer(W.by_name(name), 0, device="cuda")
     out, _ = decode(env, layer)
     G = layer.num_q_heads // layer.num_kv_heads
     o = out.cpu().numpy()
     assert np.isfinite(o).all()
     for g in heads:
         ref = oracle_subset(env, layer, queries, g)
-        compare(o[queries][:, g * G:(g + 1) * G], ref, f"config{cfg_idx} g{g}")
+        compare(o[queries][:, g * G:(g + 1) * G], ref, f"{name} g{g}")
