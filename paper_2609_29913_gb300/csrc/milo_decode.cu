@@ -993,7 +993,6 @@ cudaError_t static_workspace(void **ptr)
 {
     // Host code cannot use the array's name as a device address: look the
     // address up once per device, with that device current, and keep it.
-    constexpr int kMaxDevices = 64;
     static std::mutex mu;
     static void *addr[kMaxDevices] = {};
     int dev = 0;
