@@ -230,7 +230,9 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
  * tails and the workspace only after it has; the second combines and writes
  * `out`.  A plan must not be used by two calls that can run concurrently (it
  * holds per-call counters and accumulators).  A query whose prefix and tail
- * are both empty yields NaN.
+ * are both empty yields NaN.  A call with more than 2^31 - 1 work items
+ * (prefix chunks x row groups plus tail items) returns MILO_ERR_UNSUPPORTED
+ * without launching anything.
  */
 milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q,
                                int32_t batch, const void *tail_k,

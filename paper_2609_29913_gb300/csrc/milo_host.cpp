@@ -600,6 +600,11 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
 
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
+    // the kernels count thread blocks, tail items and list entries in int
+    const int64_t tail_items = (int64_t)batch * plan->hkv * c.S;
+    if (tail_items > 0x7fffffff || (int64_t)plan->num_chunks * c.nrg + tail_items > 0x7fffffff ||
+        c.list_cap > 0x7fffffff)
+        return fail(MILO_ERR_UNSUPPORTED, "call too large: more than 2^31 - 1 work items");
     DecodeParams prm{};
     prm.packed = plan->packed;
     prm.entries = plan->entries;
@@ -638,7 +643,7 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.npass_t = c.npass_t;
     prm.num_slots = plan->num_slots;
     prm.tail_splits = c.S;
-    prm.num_tail_items = batch * plan->hkv * c.S;
+    prm.num_tail_items = (int)tail_items;
     prm.has_tail = c.S > 0 ? 1 : 0;
     prm.tail_rec_base = (int64_t)plan->num_slots * c.nrg;
     prm.tail_k = static_cast<const uint16_t *>(tail_k);
