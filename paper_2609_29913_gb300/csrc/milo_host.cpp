@@ -400,6 +400,8 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     if (max_batch < 1) return fail(MILO_ERR_INVALID_ARG, "max_batch < 1");
     const int G = num_q_heads / table->num_kv_heads;
     if (G > 32) return fail(MILO_ERR_UNSUPPORTED, "more than 32 query heads per KV head");
+    // query rows per KV head are counted in int on the device
+    if ((int64_t)max_batch * G > (1 << 30)) return fail(MILO_ERR_UNSUPPORTED, "max_batch x G above 2^30");
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
 
     milo_prefix *p = new (std::nothrow) milo_prefix;
