@@ -173,6 +173,10 @@ milo_status_t milo_chunk_prefix(const milo_block_table_t *table,
  *                 h / (num_q_heads / num_kv_heads)).
  *   max_batch     largest batch any decode call on this plan will use.
  *   out_plan      receives the plan; release with milo_prefix_destroy.
+ * Errors: the table's validation status; MILO_ERR_INVALID_ARG for a bad
+ * head count or max_batch < 1; MILO_ERR_UNSUPPORTED for more than 32 query
+ * heads per KV head or max_batch x (num_q_heads / num_kv_heads) above 2^30;
+ * MILO_ERR_CUDA when an allocation, copy or the pack kernel fails.
  */
 milo_status_t milo_prefix_create(const milo_block_table_t *table,
                                  int32_t num_q_heads, int32_t max_batch,
