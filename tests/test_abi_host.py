@@ -240,3 +240,20 @@ def test_chunk_prefix_reports_a_short_buffer(milo):
     buf = (ctypes.c_int32 * 4)()
     assert L.milo_chunk_prefix(ctypes.byref(t.c), 4, buf, None, None, ctypes.byref(n)) == 1
     assert n.value == 8
+
+
+def test_calls_without_a_plan_fail_on_the_host(milo):
+    """Every per-call entry point checks its plan before touching a device:
+    a null plan is MILO_ERR_INVALID_ARG, with a message, and nothing runs."""
+    L = milo.lib()
+    size = ctypes.c_size_t(0)
+    assert L.milo_workspace_size(None, 1, 0, ctypes.byref(size)) == 1
+    assert L.milo_attn_decode(None, None, 1, None, None, None, 0, 0, ctypes.c_float(0.0), None, None, 0,
+                              None) == 1
+    assert b"null" in L.milo_last_error_message()
+    assert L.milo_attn_decode_static(None, None, 1, None, None, None, 0, 0, ctypes.c_float(0.0), None,
+                                     None) == 1
+    code = ctypes.c_int32(0)
+    assert L.milo_get_device_status(None, None, 0, ctypes.byref(code)) == 1
+    info = milo.PrefixInfoC()
+    assert L.milo_prefix_get_info(None, ctypes.byref(info)) == 1
