@@ -1,7 +1,9 @@
-"""Multi-GPU is replicas only: under torchrun every rank runs its own copy of
-the workload, the step time is the slowest rank's, and the job's throughput
-counts every rank's tokens.  These checks run that host logic as two gloo
-ranks on the CPU; nothing here touches a GPU."""
+"""bench.py's host logic, on the CPU.  Multi-GPU is replicas only: under
+torchrun every rank runs its own copy of the workload, the step time is the
+slowest rank's, and the job's throughput counts every rank's tokens; these
+checks run that logic as two gloo ranks.  The reference arm (the oracle on
+the host cores) is checked for its one contract line.  Nothing here touches
+a GPU."""
 import json
 import os
 import socket
@@ -49,3 +51,23 @@ def test_reference_arm_runs_on_rank_zero_only():
                          capture_output=True, text=True, timeout=300, env=env, cwd=ROOT)
     assert res.returncode == 0, res.stderr[-2000:]
     assert res.stdout.strip() == ""
+
+
+def test_reference_arm_prints_one_contract_line():
+    """The reference arm (the oracle on the host cores) prints one JSON line
+    with the keys the bench contract names, on the small 2k-token workload."""
+    res = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "0",
+                          "--steps", "2", "--warmup", "1"],
+                         capture_output=True, text=True, timeout=300, cwd=ROOT,
+                         env=dict(os.environ, RANK="0", WORLD_SIZE="1"))
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [x for x in res.stdout.splitlines() if x.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for key in ("impl", "metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert key in d, key
+    assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
+    assert d["config"]["workload"] == "qwen0.5b-1L-2k"
