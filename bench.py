@@ -8,13 +8,20 @@ graph; inputs are resident in HBM before timing starts.
 
 Metric: tokens-attended/s = sum over layers and queries of (prefix tokens +
 the query's tail tokens) per second (all heads of a layer count once), plus
-achieved algorithmic HBM GB/s as a fraction of the measured copy bandwidth.
+achieved algorithmic HBM GB/s as a fraction of the measured copy bandwidth
+and, where the contraction binds, algorithmic FLOP/s against the measured
+sustained bf16 tensor throughput.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--config C] [--impl milo|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config C] [--only]
+                  [--impl milo|reference]
 
-Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank runs an
-independent replica of the workload (the path has no cross-GPU exchange):
-value = all ranks' tokens / the slowest rank's time, scaling "weak".
+Prints one JSON line (rank 0).  The line's headline is workload --config
+(default 1, the 28-layer Qwen2.5-7B-shaped prefix at batch 1); unless --only
+is given, "workloads" adds a record for each of the other four workloads,
+measured in the same process with the same warm-up and step count.  Under
+torchrun (N > 1) every rank runs an independent replica of the workload (the
+path has no cross-GPU exchange): value = all ranks' tokens / the slowest
+rank's time, scaling "weak".
 """
 from __future__ import annotations
 
@@ -35,43 +42,83 @@ sys.path.insert(0, ROOT)
 METRIC = "decode tokens-attended/s over low-rank KV prefix; HBM GB/s as % of GB300 peak"
 UNIT = "tokens/s"
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
+L2_BYTES = 129 * 2 ** 20
+PARITY_ATOL, PARITY_RTOL_L2 = 1e-2, 2e-3
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--config", type=int, default=1, help="workload index 0..4 (1 = headline)")
+    ap.add_argument("--config", type=int, default=1, help="headline workload index 0..4 (1 = batch-1 7B)")
+    ap.add_argument("--only", action="store_true", help="measure the headline workload only")
     ap.add_argument("--impl", default="milo", choices=["milo", "reference"])
-    ap.add_argument("--no-check", action="store_true", help="skip the parity spot check")
+    ap.add_argument("--no-check", action="store_true", help="skip the parity checks")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU baseline sample time")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def peaks():
+    """Measured HBM copy GB/s and sustained bf16 TFLOP/s (or the fallbacks)."""
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            return float(json.load(f)["hbm_gbs"]), "measured"
+            d = json.load(f)
+        return (float(d["hbm_gbs"]), float(d.get("bf16_tflops_sustained", FALLBACK_BF16_TFLOPS_SUSTAINED)),
+                "measured")
     except Exception:
-        return FALLBACK_HBM_GBS, "fallback"
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS_SUSTAINED, "fallback"
 
 
-def algorithmic_bytes(layer) -> int:
-    """Bytes the method must move for one call: factors at their true ranks
-    (C^K, P^K, C^V, P^V), the dense tails, q reads and fp32 output writes."""
-    d = layer.head_dim
-    n = layer.block_len[np.arange(len(layer.rank_k)) // layer.num_kv_heads].astype(np.int64)
-    r = (layer.rank_k + layer.rank_v).astype(np.int64)
-    factors = int(((n + d) * r).sum()) * 2
-    tails = int(layer.tail_offsets[-1]) * layer.num_kv_heads * d * 2 * 2
-    qo = layer.batch * layer.num_q_heads * d * (2 + 4)
-    return factors + tails + qo
+# ------------------------------------------------------------ accounting
+def layer_totals(num_q_heads, num_kv_heads, head_dim, block_len, rank_k, rank_v, tail_lengths, batch):
+    """(tokens attended, algorithmic bytes, algorithmic flops) of one call.
+
+    Bytes: the factors at their true ranks (C^K, P^K, C^V, P^V), the dense
+    tails, the q reads and the fp32 output writes.  Flops (multiply-add = 2):
+    per KV head and query row, 2 (n_b + d)(r^k + r^v) per prefix entry (scores
+    and rank-space values over its n_b tokens, projection and
+    back-projection over d), and 4 d per tail token."""
+    d = int(head_dim)
+    hk = int(num_kv_heads)
+    G = int(num_q_heads) // hk
+    n = np.asarray(block_len, np.int64)[np.arange(len(rank_k)) // hk]
+    r = np.asarray(rank_k, np.int64) + np.asarray(rank_v, np.int64)
+    per_row = int((2 * (n + d) * r).sum())
+    tails = int(np.asarray(tail_lengths, np.int64).sum())
+    bytes_ = per_row + tails * hk * d * 2 * 2 + batch * num_q_heads * d * (2 + 4)
+    flops = batch * G * per_row + tails * G * hk * 4 * d
+    tokens = batch * int(np.asarray(block_len).sum()) + tails
+    return tokens, bytes_, flops
 
 
-def tokens_attended(layer) -> int:
-    return int(layer.batch * int(layer.block_len.sum()) + int(layer.tail_offsets[-1]))
+def workload_totals(cfg, W):
+    """Per-step totals of a workload from its tables alone (no factor data)."""
+    tok = byt = flo = 0
+    for l in range(cfg.layers):
+        ranks = W.draw_ranks(cfg, l).reshape(-1)
+        tl = W.draw_tail_lengths(cfg, l)
+        a, b, c = layer_totals(cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim,
+                               np.full(cfg.num_blocks, cfg.block_len), ranks, ranks, tl, cfg.batch)
+        tok, byt, flo = tok + a, byt + b, flo + c
+    return tok, byt, flo
+
+
+def shared_config(cfg, totals, world):
+    """The workload's `config` object, the same on both arms."""
+    tokens, bytes_, flops = totals
+    l2 = ("inputs larger than L2 (a step reads %.2f GB > 129 MB); no flush" % (bytes_ / 1e9)
+          if bytes_ > 2 * L2_BYTES else
+          "inputs smaller than L2 (%.2f MB): L2 flushed (a %d MB write) before each timed step" %
+          (bytes_ / 1e6, 4 * L2_BYTES >> 20))
+    return {"workload": cfg.name, "layers": cfg.layers, "batch": cfg.batch,
+            "prefix_tokens": cfg.prefix_tokens, "num_q_heads": cfg.num_q_heads,
+            "num_kv_heads": cfg.num_kv_heads, "head_dim": cfg.head_dim,
+            "tokens_per_step": tokens, "algorithmic_bytes_per_step": bytes_,
+            "algorithmic_flops_per_step": flops, "l2": l2,
+            "parallelism": "replicas" if world > 1 else "single GPU"}
 
 
 class ClockSampler:
@@ -157,15 +204,20 @@ def cpu_baseline(layers_host, target_s: float):
 
 
 def reference_arm(args, cfg, W):
-    """The oracle timed as the reference implementation (rank 0 only)."""
-    import torch  # noqa: F401
+    """The oracle timed as the reference implementation (rank 0 only).  A
+    step is one layer of the workload (a bounded sample: the whole step of
+    the GPU arm would take minutes); ms_per_step is that step's mean time and
+    value the tokens it attends per second."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
+    world = int(os.environ.get("WORLD_SIZE", "1"))
     from oracle import milo_oracle
     milo_oracle.build()
     layers = [W.make_config_layer(cfg, l, device="cpu") for l in range(min(cfg.layers, 2))]
-    host = [(L.to_numpy_bits(), tokens_attended(L)) for L in layers]
+    host = [(L.to_numpy_bits(), layer_totals(L.num_q_heads, L.num_kv_heads, L.head_dim, L.block_len,
+                                             L.rank_k, L.rank_v, np.diff(L.tail_offsets), L.batch)[0])
+            for L in layers]
     times, toks = [], []
     per = max(1, int(args.steps))
     for s in range(args.warmup + per):
@@ -177,15 +229,16 @@ def reference_arm(args, cfg, W):
             times.append(dt)
             toks.append(tk)
     value = sum(toks) / sum(times)
+    sample = (f"each step is one layer of {cfg.name} (layers 0 and 1 in turn), all queries and heads; "
+              f"{per} timed steps after {args.warmup} warm-up")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": 1e3 * sum(times) / len(times) * cfg.layers,
+            "ms_per_step": 1e3 * sum(times) / len(times),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": cfg.name, "layers": cfg.layers,
-                                            "sample": "each step is one layer of the workload"},
+            "data": "synthetic", "config": shared_config(cfg, workload_totals(cfg, W), world),
+            "step": "one layer of the workload per step (a bounded sample of the GPU arm's step)",
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": milo_oracle.max_threads(),
-                             "kind": "oracle",
-                             "sample": f"{per} single-layer calls of {cfg.name} after {args.warmup} warm-up"},
+                             "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -228,41 +281,42 @@ def pack_tensors(tensors, dev):
     return buf, views
 
 
-def main():
-    args = parse()
-    from paper_2609_29913_gb300 import workloads as W
-    cfg = W.CONFIGS[args.config]
-    if args.impl == "reference":
-        reference_arm(args, cfg, W)
-        return
+def parity_layer0(layer, out0):
+    """Layer 0's whole output [batch, Hq, d] against the oracle."""
+    from oracle import milo_oracle
+    milo_oracle.build()
+    ref = milo_oracle.attention(**layer.to_numpy_bits())
+    got = out0.double().cpu().numpy()
+    d = got.shape[-1]
+    g2, r2 = got.reshape(-1, d), ref.reshape(-1, d)
+    rows = np.linalg.norm(g2 - r2, axis=1) / np.maximum(np.linalg.norm(r2, axis=1), 1e-30)
+    err = float(np.abs(got - ref).max())
+    rel = float(np.linalg.norm(got - ref) / np.linalg.norm(ref))
+    return {"max_abs": err, "rel_l2": rel, "worst_row_rel_l2": float(rows.max()),
+            "pass": bool(err <= PARITY_ATOL and rel <= PARITY_RTOL_L2),
+            "rows": f"layer 0, every query and head ({got.shape[0]} x {got.shape[1]} rows of {d})"}
 
+
+def kernel_names(path: int, has_tail: bool) -> list:
+    """The kernels one layer call launches, for the JSON line's description."""
+    if path == 1:
+        return (["chunk_kernel (dense-tail items)"] if has_tail else []) + ["batch_tc_kernel", "finish_kernel"]
+    if path == 0:
+        return ["chunk_kernel", "finish_kernel"]
+    return ["decode_kernel", "combine_kernel"]
+
+
+def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, check=True,
+            e2e=False, cpu_seconds=0.0):
+    """Time one workload (all its layers per step) and return its record."""
     import torch
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-
-    from paper_2609_29913_gb300 import build as milo_build
-    milo_build.build()
-    from paper_2609_29913_gb300 import milo
-
-    dev = torch.device("cuda", local)
-    # ---- inputs resident in HBM, one plan per layer (logical arenas freed)
-    plans, qs, tks, tvs, toffs, metas = [], [], [], [], [], []
-    check_layer = None
+    plans, qs, tks, tvs, toffs = [], [], [], [], []
     host_layers = []
-    alg_bytes = 0
-    tokens = 0
+    check_layer = None
     max_tail = 0
     t_gen = time.perf_counter()
     for l in range(cfg.layers):
         layer = W.make_config_layer(cfg, l, device=dev)
-        alg_bytes += algorithmic_bytes(layer)
-        tokens += tokens_attended(layer)
         max_tail = max(max_tail, int(np.diff(layer.tail_offsets).max()))
         pre = milo.Prefix.from_layer(layer)
         plans.append(pre)
@@ -270,14 +324,20 @@ def main():
         tks.append(layer.tail_k)
         tvs.append(layer.tail_v)
         toffs.append(torch.as_tensor(layer.tail_offsets, device=dev))
-        if l == 0 and not args.no_check:
-            check_layer = (layer, layer.to_numpy_bits())
-        if rank == 0 and not args.no_cpu and len(host_layers) < 3:
-            host_layers.append((layer.to_numpy_bits(), tokens_attended(layer)))
-        layer.arena = None  # the packed copy in the plan is all the decode reads
+        if l == 0 and check and rank == 0:
+            check_layer = layer
+        if rank == 0 and cpu_seconds > 0 and len(host_layers) < 3:
+            host_layers.append((layer.to_numpy_bits(), layer_totals(
+                layer.num_q_heads, layer.num_kv_heads, layer.head_dim, layer.block_len, layer.rank_k,
+                layer.rank_v, np.diff(layer.tail_offsets), layer.batch)[0]))
+        if l > 0 or check_layer is None:
+            layer.arena = None  # the packed copy in the plan is all the decode reads
     torch.cuda.synchronize()
     t_gen = time.perf_counter() - t_gen
+    totals = workload_totals(cfg, W)
+    tokens, alg_bytes, alg_flops = totals
     batch = cfg.batch
+    call = milo.milo_call_info(plans[0].plan, batch, max_tail)
     ws_bytes = max(p.workspace_size(batch, max_tail) for p in plans)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
     # A step's inputs (every layer's q and dense tails, layer by layer) sit in
@@ -288,84 +348,107 @@ def main():
     qs, tks, tvs = views[0::3], views[1::3], views[2::3]
     out_buf = torch.empty((L, batch, cfg.num_q_heads, cfg.head_dim), dtype=torch.float32, device=dev)
     outs = [out_buf[l] for l in range(L)]
-
     stream = torch.cuda.Stream(device=dev)
 
     def run_step(s):
-        for l in range(cfg.layers):
-            plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws,
-                            stream=s)
+        for l in range(L):
+            plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws, stream=s)
 
-    # warm once eagerly, then capture the step in a graph
     with torch.cuda.stream(stream):
         run_step(stream)
     stream.synchronize()
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=stream):
         run_step(stream)
-    for _ in range(max(args.warmup, 3)):
+    for _ in range(max(warmup, 3)):
         graph.replay()
     torch.cuda.synchronize()
     for p in plans:
         assert p.status() == 0, "device status word set during warm-up"
 
-    # ---- parity spot check (outside the timed region): one KV head of layer 0
-    check = None
+    check = parity_layer0(check_layer, outs[0]) if check_layer is not None else None
     if check_layer is not None:
-        from oracle import milo_oracle
-        milo_oracle.build()
-        check_layer, bits = check_layer
-        hkv, G = cfg.num_kv_heads, cfg.num_q_heads // cfg.num_kv_heads
-        ent = np.arange(cfg.num_blocks) * hkv
-        qsel = list(range(min(batch, 2)))
-        sub = dict(num_kv_heads=1, head_dim=cfg.head_dim, block_len=check_layer.block_len,
-                   rank_k=check_layer.rank_k[ent], rank_v=check_layer.rank_v[ent],
-                   off_ck=check_layer.off_ck[ent], off_pk=check_layer.off_pk[ent],
-                   off_cv=check_layer.off_cv[ent], off_pv=check_layer.off_pv[ent],
-                   arena=bits["arena"], q=np.ascontiguousarray(bits["q"][qsel][:, :G]))
-        if "tail_k" in bits:
-            tk, tv, to = [], [], [0]
-            for i in qsel:
-                a, b = check_layer.tail_offsets[i], check_layer.tail_offsets[i + 1]
-                tk.append(bits["tail_k"][a:b, 0:1])
-                tv.append(bits["tail_v"][a:b, 0:1])
-                to.append(to[-1] + b - a)
-            sub.update(tail_k=np.ascontiguousarray(np.concatenate(tk)),
-                       tail_v=np.ascontiguousarray(np.concatenate(tv)), tail_offsets=np.array(to))
-        ref = milo_oracle.attention(**sub)
-        got = outs[0][qsel][:, :G].double().cpu().numpy()
-        check = {"max_abs": float(np.abs(got - ref).max()),
-                 "rel_l2": float(np.linalg.norm(got - ref) / np.linalg.norm(ref)),
-                 "rows": f"layer 0, KV head 0, queries {qsel}"}
-        check_layer = None
+        check_layer.arena = None
+    check_layer = None
 
-    # ---- timed region: K graph replays (inputs > L2: no flush needed)
-    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # ---- timed region: K graph replays.  Inputs larger than L2 need no
+    # flush; a workload that fits in L2 is timed replay by replay with a
+    # buffer larger than L2 written before each (outside the events).
+    flush = torch.empty(4 * L2_BYTES // 4, dtype=torch.float32, device=dev) if alg_bytes <= 2 * L2_BYTES else None
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    with ClockSampler(local) as clocks:
-        torch.cuda.nvtx.range_push("milo_timed")
-        start.record(stream)
-        with torch.cuda.stream(stream):
-            for _ in range(args.steps):
-                graph.replay()
-        stop.record(stream)
-        torch.cuda.synchronize()
-        torch.cuda.nvtx.range_pop()
+    with ClockSampler(dev.index if dev.index is not None else 0) as clocks:
+        if flush is None:
+            start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            start.record(stream)
+            with torch.cuda.stream(stream):
+                for _ in range(steps):
+                    graph.replay()
+            stop.record(stream)
+            torch.cuda.synchronize()
+            ms_total = start.elapsed_time(stop)
+        else:
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(steps)]
+            with torch.cuda.stream(stream):
+                for a, b in evs:
+                    flush.fill_(1.0)
+                    a.record(stream)
+                    graph.replay()
+                    b.record(stream)
+            torch.cuda.synchronize()
+            ms_total = sum(a.elapsed_time(b) for a, b in evs)
     if dist:
         dist.barrier()
-    ms_total = start.elapsed_time(stop)
-    ms_step = max_over_ranks(ms_total / args.steps, dist, dev)
+    ms_step = max_over_ranks(ms_total / steps, dist, dev)
     for p in plans:
         assert p.status() == 0, "device status word set during the timed region"
 
-    # ---- end to end through the public API with host buffers: each step
-    # copies every layer's q and tails from pinned host memory, runs the
-    # per-layer calls and reads every layer's output back.  The layers are
-    # cut into a few segments, each a captured graph whose inputs arrive by
-    # one copy on a second stream, so that later segments' copies overlap
-    # earlier segments' calls.
+    hbm, tf_sus, peak_kind = peaks()
+    achieved = alg_bytes / (ms_step * 1e-3) / 1e9
+    flops_s = alg_flops / (ms_step * 1e-3) / 1e12
+    roof_ms = max(alg_bytes / (hbm * 1e9), alg_flops / (tf_sus * 1e12)) * 1e3
+    rec = {
+        "workload": cfg.name, "ms_per_step": ms_step, "value": replica_throughput(world, tokens, ms_step),
+        "unit": UNIT, "steps": steps, "warmup": warmup,
+        "config": shared_config(cfg, totals, world),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": None,
+                     "peak_source": f"{peak_kind} copy bandwidth (hbm_gbs)"},
+        "tensor": {"achieved_tflops": flops_s, "peak_tflops": tf_sus, "frac": flops_s / tf_sus,
+                   "peak_source": f"{peak_kind} sustained cuBLAS bf16 (bf16_tflops_sustained)"},
+        "roofline_time": {"ms": roof_ms, "frac": roof_ms / ms_step,
+                          "how": "max(algorithmic bytes / hbm_gbs, algorithmic flops / bf16_tflops_sustained)"},
+        "path": {0: "chunk grid (mma.sync)", 1: "tensor-core batched grid (tcgen05)",
+                 2: "persistent grid (mma.sync)"}[call["path"]],
+        "kernels_per_layer": call["kernels"],
+        "kernels": kernel_names(call["path"], max_tail > 0),
+        "gpu_launches": call["kernels"] * L * steps,
+        "clocks": clocks.summary(), "parity_check": check, "setup_s": t_gen,
+    }
+    if e2e:
+        rec["e2e"] = measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, max_tail,
+                                 steps, dist, dev, world, tokens)
+    if cpu_seconds > 0 and rank == 0 and world == 1 and host_layers:
+        rec["cpu_baseline"] = cpu_baseline(host_layers, cpu_seconds)
+    for p in plans:
+        p.close()
+    del plans, graph, ws, in_buf, out_buf
+    torch.cuda.empty_cache()
+    return rec
+
+
+def measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, max_tail, steps, dist, dev,
+                world, tokens):
+    """The same step through the public API with host buffers: each step
+    copies every layer's q and tails from pinned host memory, runs the
+    per-layer calls and reads every layer's output back.  The layers are cut
+    into a few segments, each a captured graph whose inputs arrive by one copy
+    on a second stream, so that later segments' copies overlap earlier
+    segments' calls."""
+    import torch
+    L = len(plans)
     in_host = in_buf.cpu().pin_memory()
     out_host = torch.empty_like(out_buf, device="cpu").pin_memory()
     h2d = sum(x.numel() * x.element_size() for x in qs + tks + tvs if x is not None)
@@ -401,7 +484,7 @@ def main():
         for _ in range(2):
             e2e_step(stream)
     stream.synchronize()
-    e_steps = max(3, min(args.steps, 10))
+    e_steps = max(3, min(steps, 10))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     with torch.cuda.stream(stream):
@@ -410,74 +493,83 @@ def main():
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = max_over_ranks(e0.elapsed_time(e1) / e_steps, dist, dev)
+    return {"value": replica_throughput(world, tokens, e_ms), "unit": UNIT,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
+            "how": "per step: every layer's q and tails copied from pinned host memory in %d copies on a "
+                   "second stream, each releasing a captured graph of its layers' calls, then one copy "
+                   "of every layer's output to pinned host memory" % nseg}
 
-    # ---- CPU oracle baseline (rank 0, N = 1 only)
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu and host_layers:
-        cpu = cpu_baseline(host_layers, args.cpu_seconds)
 
-    peak, peak_kind = peaks()
-    achieved = alg_bytes / (ms_step * 1e-3) / 1e9
-    traffic = None
+def traffic_record(cfg_name):
+    """DRAM bytes per launch of the dominant kernel from profiles/traffic.json,
+    while the kernel's source still hashes to the profiled one."""
     try:
+        import hashlib
+        from paper_2609_29913_gb300 import build as b
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             tr = json.load(f)
-        from paper_2609_29913_gb300 import build as b
-        import hashlib
-        entry = tr.get(cfg.name)
-        src = entry.get("kernel_source", "milo_decode.cu") if entry else "milo_decode.cu"
-        h = hashlib.sha256(open(os.path.join(b.CSRC, src), "rb").read()).hexdigest()[:16]
-        if entry and entry.get("kernel_sha") == h:
-            traffic = entry["dram_bytes_per_launch"]
+        entry = tr.get(cfg_name)
+        if not entry:
+            return None
+        h = hashlib.sha256(open(os.path.join(b.CSRC, entry["kernel_source"]), "rb").read()).hexdigest()[:16]
+        return entry["dram_bytes_per_launch"] if entry.get("kernel_sha") == h else None
     except Exception:
-        traffic = None
-    value = replica_throughput(world, tokens, ms_step)
-    # up to 8 query heads per KV head: the chunk grid (a block per prefix
-    # chunk and row group of 8 query rows, and per tail item, adding into
-    # per-row accumulators) and its finish grid; more: the persistent kernel
-    # and the merge kernel
-    short = cfg.num_q_heads // cfg.num_kv_heads <= 8
-    kernels_per_layer = 2
+        return None
+
+
+def main():
+    args = parse()
+    from paper_2609_29913_gb300 import workloads as W
+    cfg = W.CONFIGS[args.config]
+    if args.impl == "reference":
+        reference_arm(args, cfg, W)
+        return
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2609_29913_gb300 import build as milo_build
+    milo_build.build()
+    from paper_2609_29913_gb300 import milo
+
+    dev = torch.device("cuda", local)
+    head = measure(cfg, W, milo, dev, args.steps, args.warmup, dist, rank, world, check=not args.no_check,
+                   e2e=True, cpu_seconds=0.0 if args.no_cpu else args.cpu_seconds)
+    others = []
+    if not args.only:
+        for k, other in enumerate(W.CONFIGS):
+            if k == args.config:
+                continue
+            others.append(measure(other, W, milo, dev, args.steps, args.warmup, dist, rank, world,
+                                  check=not args.no_check))
+    roof = dict(head["roofline"])
+    roof["traffic"] = traffic_record(cfg.name)
+    roof["kernel"] = ", ".join(head["kernels"])
+    roof["per_launch_bytes"] = head["config"]["algorithmic_bytes_per_step"] // cfg.layers
+    roof["per_launch_us"] = head["ms_per_step"] * 1e3 / cfg.layers
+    roof["how"] = ("algorithmic bytes of a layer call / the mean time of a layer call inside the timed "
+                   "CUDA graph (consecutive calls overlap through programmatic dependent launch)")
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": head["ms_per_step"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": cfg.name, "layers": cfg.layers, "batch": cfg.batch,
-                   "prefix_tokens": cfg.prefix_tokens, "num_q_heads": cfg.num_q_heads,
-                   "num_kv_heads": cfg.num_kv_heads, "head_dim": cfg.head_dim,
-                   "tokens_per_step": tokens, "algorithmic_bytes_per_step": alg_bytes,
-                   "l2": "inputs larger than L2 (step reads %.2f GB > 129 MB); no flush" % (alg_bytes / 1e9),
-                   "parallelism": "replicas" if world > 1 else "single GPU",
-                   "launch": ("one CUDA graph of %d per-layer calls, each a grid of two-warp blocks (prefix "
-                              "chunks per row group of 8 query rows, and dense-tail items, adding into per-row "
-                              "accumulators) and a finish grid of one warp per KV head and row group "
-                              "(programmatic dependent launch)"
-                              if short else
-                              "one CUDA graph of %d per-layer calls, each a persistent decode and a merge "
-                              "kernel (programmatic dependent launch)") % cfg.layers},
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": traffic,
-                     "peak_source": f"{peak_kind} copy bandwidth",
-                     "kernel": ("chunk_kernel (two warps per prefix chunk and row group, accumulator merge; "
-                                "finish_kernel chained)" if short
-                                else "decode_kernel (persistent rank-space split-K decode)"),
-                     "per_launch_bytes": alg_bytes // cfg.layers,
-                     "per_launch_us": ms_step * 1e3 / cfg.layers},
-        "cpu_baseline": cpu,
-        "e2e": {"value": replica_throughput(world, tokens, e_ms), "unit": UNIT,
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
-                "how": "per step: every layer's q and tails copied from pinned host memory in %d copies on a "
-                       "second stream, each releasing a captured graph of its layers' calls, then one copy "
-                       "of every layer's output to pinned host memory" % nseg},
-        "gpu_launches": kernels_per_layer * cfg.layers * args.steps,
-        "clocks": clocks.summary(),
-        "parity_check": check,
-        "setup_s": t_gen,
+        "config": head["config"],
+        "launch": "one CUDA graph of %d per-layer calls (%s per call)" % (cfg.layers, ", ".join(head["kernels"])),
+        "roofline": roof, "tensor": head["tensor"], "roofline_time": head["roofline_time"],
+        "cpu_baseline": head.get("cpu_baseline"),
+        "e2e": head["e2e"], "gpu_launches": head["gpu_launches"], "clocks": head["clocks"],
+        "parity_check": head["parity_check"], "path": head["path"], "setup_s": head["setup_s"],
+        "workloads": [{k: v for k, v in o.items() if k not in ("unit",)} for o in others],
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
-    for p in plans:
-        p.close()
     if dist:
         dist.destroy_process_group()
 

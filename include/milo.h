@@ -209,6 +209,39 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
                                   int64_t max_tail_tokens, size_t *bytes);
 
 /*
+ * How a decode call of this shape runs (host only, no device access):
+ *   path     MILO_PATH_CHUNKS (0): the chunk grid on warp-level MMA, one
+ *            thread block per prefix chunk and row group of 8 query rows
+ *            (at most 8 query heads per KV head and fewer query rows per KV
+ *            head than the tensor-core threshold);
+ *            MILO_PATH_TENSOR (1): the tensor-core grid (tcgen05, 128 query
+ *            rows per product) for the prefix, with the dense tails on the
+ *            chunk grid (at most 8 query heads per KV head and at least
+ *            milo_tensor_min_rows() query rows per KV head);
+ *            MILO_PATH_PERSISTENT (2): the persistent warp-level decode and
+ *            its merge kernel (more than 8 query heads per KV head, or no
+ *            prefix).
+ *   kernels  kernel launches of one call (each a grid).
+ *   row_tiles  tensor-core path: tiles of 128 query rows per KV head (else 0).
+ *   blocks   thread blocks of the call's main prefix grid.
+ * Errors: MILO_ERR_INVALID_ARG for a null argument, batch outside
+ * [1, max_batch] or max_tail_tokens < 0.
+ */
+typedef enum { MILO_PATH_CHUNKS = 0, MILO_PATH_TENSOR = 1, MILO_PATH_PERSISTENT = 2 } milo_path_t;
+typedef struct {
+    int32_t path;
+    int32_t kernels;
+    int32_t row_tiles;
+    int32_t blocks;
+} milo_call_info_t;
+milo_status_t milo_call_info(const milo_prefix_t *plan, int32_t batch,
+                             int64_t max_tail_tokens, milo_call_info_t *info);
+
+/* Query rows per KV head (batch x query heads per KV head) from which a
+ * call takes the tensor-core path. */
+int32_t milo_tensor_min_rows(void);
+
+/*
  * One decode-attention call for one layer (Alg. 1 Stage 2 + Eq. 1):
  * for every query i and query head h (KV head g = h / G),
  *   out[i, h] = softmax(scale * q[i,h] . [K^_1 .. K^_N, Ktail_i[:, g]]) [V^ ...].
@@ -226,7 +259,7 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
  *                in the device status word (MILO_ERR_DEVICE_BOUNDS).
  *   softmax_scale  <= 0 selects 1 / sqrt(head_dim).
  *   out          device fp32 [batch, num_q_heads, head_dim].
- *   workspace    device, at least milo_workspace_size bytes, 256-byte aligned.
+ *   workspace    device, at least milo_workspace_size bytes, 16-byte aligned.
  * Asynchronous on `stream`: no host synchronisation and no allocation, so the
  * call can be captured in a CUDA graph.  A call is two kernels launched with
  * programmatic dependent launch: the first may begin streaming the plan's

@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmilo.so")
-SOURCES = ["milo_host.cpp", "milo_pack.cu", "milo_decode.cu", "milo_chunk.cu"]
+SOURCES = ["milo_host.cpp", "milo_pack.cu", "milo_decode.cu", "milo_chunk.cu", "milo_batch.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -30,7 +30,7 @@ def nvcc() -> str:
 
 def _deps():
     files = [os.path.join(CSRC, s) for s in SOURCES]
-    files += [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".h")]
+    files += [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
     files.append(os.path.join(INCLUDE, "milo.h"))
     files.append(os.path.abspath(__file__))
     return files

@@ -42,6 +42,7 @@
 
 #include "milo.h"
 #include "milo_internal.h"
+#include "milo_merge.cuh"
 #include "milo_ptx.cuh"
 
 namespace milo {
@@ -79,42 +80,12 @@ __device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
     s.rpp = CLay<D, 1>::kRanksPerPiece / 8;
     s.npk = (c.nrk + s.rpp - 1) / s.rpp;
     s.npv = (c.nrv + s.rpp - 1) / s.rpp;
-    s.tpp = max(1, kPieceBytes / (kTile * (c.nrk + c.nrv) * 16));
+    // an entry of rank 0 in K and V has no coefficient rows: its (at most
+    // 32-token) chunk is one C piece that copies nothing
+    const int row_bytes = kTile * (c.nrk + c.nrv) * 16;
+    s.tpp = row_bytes > 0 ? max(1, kPieceBytes / row_bytes) : kChunkMaxTok / kTile;
     s.nc = (c.ntok + s.tpp * kTile - 1) / (s.tpp * kTile);
     return s;
-}
-
-// The per-KV-head merge.  Every chunk and tail item ends with (o, m, l) per
-// query row: o = sum 2^(s - m) v over its tokens, l = sum 2^(s - m) (Eq. 1 on
-// a partition of the tokens).  Rather than storing these and merging them
-// afterwards, each item adds 2^(m - M) o and 2^(m - M) l into fp32
-// accumulators of its KV head with vector reductions, for one reference M per
-// row: the first item to finish a tile sets M = its running maximum +
-// kRefMargin (compare-and-swap), and every other item reads it back.  With M
-// within kDirectMax below an item's maximum nothing overflows; an item whose
-// maximum lies further above M (a rare outlier) writes its record instead and
-// lists it.  Once the grid is done, the finish grid divides the accumulators
-// by the sum, folds in the listed records by the log-sum-exp rule, writes the
-// output and clears the accumulators for the next call.
-constexpr float kRefMargin = 40.f;  // M = first tile maximum + this
-constexpr float kDirectMax = 60.f;  // items with m - M above this keep a record
-
-// A reference maximum is stored as its float bits with the sign flipped, so
-// that 0 means "not set" (x + kRefMargin is never -0).
-__device__ __forceinline__ uint32_t ref_enc(float x) { return __float_as_uint(x) ^ 0x80000000u; }
-__device__ __forceinline__ float ref_dec(uint32_t u) { return __uint_as_float(u ^ 0x80000000u); }
-
-// Lane c4 == 0 of each valid row sets or reads the row's reference; the
-// result arrives later (it is used only at the end of the item).
-__device__ __forceinline__ uint32_t publish_ref(const DecodeParams &p, int g, int arow, bool row_ok, int c4, float m)
-{
-    uint32_t got = 0u;
-    if (c4 == 0 && row_ok) {
-        const uint32_t mine = ref_enc(m + kRefMargin);
-        const uint32_t old = atomicCAS(p.acc_m + (int64_t)g * p.rows_max + arow, 0u, mine);
-        got = old ? old : mine;
-    }
-    return got;
 }
 
 // KV head g, rows 8 rg .. 8 rg + 7, after every item: fold the listed
@@ -282,9 +253,11 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
             const int t0 = (k - ps.npk) * ps.tpp * kTile;
             const int r8 = min(t0 + ps.tpp * kTile, ch.tok8) - t0;  // rows (a multiple of 8)
             const uint32_t kb = (uint32_t)r8 * ch.nrk * 16, vb = (uint32_t)r8 * ch.nrv * 16;
+            // (a side of rank 0 copies nothing; with both, the arrival alone
+            // completes the phase)
             mbar_arrive_tx(bar, kb + vb);
-            bulk_g2s(dst, p.packed + ch.ck + (int64_t)t0 * ch.nrk * 16, kb, bar);
-            bulk_g2s(dst + kb, p.packed + ch.cv + (int64_t)t0 * ch.nrv * 16, vb, bar);
+            if (kb) bulk_g2s(dst, p.packed + ch.ck + (int64_t)t0 * ch.nrk * 16, kb, bar);
+            if (vb) bulk_g2s(dst + kb, p.packed + ch.cv + (int64_t)t0 * ch.nrv * 16, vb, bar);
         } else {
             const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, ch.nrv);
             const uint32_t b = (uint32_t)(r1 - r0) * D * 16;
@@ -806,6 +779,20 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
                               : (two ? launch_chunk_grid<128, 2>(cfg, p, mk, mv)
                                      : launch_chunk_grid<128, 1>(cfg, p, mk, mv));
     if (e != cudaSuccess) return e;
+    // the tensor-core path launches its prefix grid between the two
+    if (p.tc_ntile > 0) return cudaSuccess;
+    return launch_finish(p, stream);
+}
+
+cudaError_t launch_finish(const DecodeParams &p, cudaStream_t stream)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     cfg.gridDim = dim3(p.hkv * p.nrg);
     cfg.blockDim = dim3(32);
     cfg.dynamicSmemBytes = 0;

@@ -942,7 +942,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ De
             if (s < nsrc) {
                 const bool pre = s < nprefix;
                 const int row = pre ? k : hh % 8;
-                const float *r = pre ? p.rec + (int64_t)((gs0 + s) * p.nrg + rg) * recf
+                const float *r = pre ? p.rec + ((int64_t)(gs0 + s) * p.nrg + rg) * recf
                                      : tail0 + (int64_t)(s - nprefix) * p.nrg_t * recf;
                 mm[j] = __ldcg(r + 8 * D + row);
                 ll[j] = __ldcg(r + 8 * D + 8 + row);

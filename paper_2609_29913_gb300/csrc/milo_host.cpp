@@ -100,30 +100,55 @@ int64_t packed_layout(const milo_block_table_t *t, std::vector<int64_t> &offs)
     return cur;
 }
 
-// Static partition of the prefix over `P` thread blocks (see milo.h).
-void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::vector<int32_t> &cta_begin,
-               int &num_slots, std::vector<int32_t> *g_slot_begin)
-{
-    const int H = t->num_kv_heads, d = t->head_dim, nb = t->num_blocks;
-    constexpr int64_t kTokenOverhead = 32;  // softmax work per token, in byte-equivalents
-    auto tile_cost = [&](int e, int t8) {
+// Cost of the persistent decode's work: a token's padded coefficient bytes
+// plus kTokenOverhead (its softmax work); an entry's P^K is charged with its
+// first 32-token tile and its P^V with its last.
+struct ByteCost {
+    const milo_block_table_t *t;
+    static constexpr int64_t kTokenOverhead = 32;
+    int64_t tile(int e, int t8) const
+    {
         return (int64_t)t8 * ((r8(t->rank_k[e]) + r8(t->rank_v[e])) * 2 + kTokenOverhead);
-    };
-    auto seg_cost = [&](int e) { return (int64_t)(r8(t->rank_k[e]) + r8(t->rank_v[e])) * d * 2; };
+    }
+    int64_t first(int e) const { return (int64_t)r8(t->rank_k[e]) * t->head_dim * 2; }
+    int64_t last(int e) const { return (int64_t)r8(t->rank_v[e]) * t->head_dim * 2; }
+};
+
+// Cost of the tensor-core decode's work, in eighths of a cycle of one SM: per
+// token the softmax of a 128-row tile (~8 cycles) and the hi + lo score and
+// value products (ranks rounded up to 16: (r^k + r^v) / 8 cycles); per
+// segment the projection, back-projection and pipeline restart (~2500
+// cycles), charged with its first tile.
+struct TensorCost {
+    const milo_block_table_t *t;
+    static int r16(int r) { return (r + 15) & ~15; }
+    int64_t tile(int e, int t8) const { return (int64_t)t8 * (64 + r16(t->rank_k[e]) + r16(t->rank_v[e])); }
+    int64_t first(int) const { return 20000; }
+    int64_t last(int) const { return 0; }
+};
+constexpr int64_t kTcMinShareCost = 100000;  // in TensorCost units: ~one 512-token entry of rank 64
+
+// Static partition of the prefix over `P` shares (see milo_partition_prefix
+// in milo.h), under a cost model.
+template <class Cost>
+void partition_with(const milo_block_table_t *t, int P, const Cost &cost, std::vector<Seg> &segs,
+                    std::vector<int32_t> &cta_begin, int &num_slots, std::vector<int32_t> *g_slot_begin)
+{
+    const int H = t->num_kv_heads, nb = t->num_blocks;
     int64_t total = 0;
     for (int g = 0; g < H; ++g)
         for (int b = 0; b < nb; ++b) {
             const int e = b * H + g, n = t->block_len[b];
-            total += seg_cost(e);
-            for (int t0 = 0; t0 < n; t0 += kTileTokens) total += tile_cost(e, (std::min(n - t0, kTileTokens) + 7) & ~7);
+            total += cost.first(e) + cost.last(e);
+            for (int t0 = 0; t0 < n; t0 += kTileTokens) total += cost.tile(e, (std::min(n - t0, kTileTokens) + 7) & ~7);
         }
     segs.clear();
     cta_begin.assign((size_t)P + 1, 0);
     // Cost line: entries (KV-head-major, then block order), each charged its
-    // 64-token tiles, with P^K charged to the first tile and P^V to the last.  A tile
-    // belongs to the thread block whose share (c total/P, (c+1) total/P]
+    // 32-token tiles, with the entry's first and last charges on its first and
+    // last tile.  A tile belongs to the share (c total/P, (c+1) total/P] that
     // contains the midpoint of the tile's cost interval.  A block cut between
-    // two thread blocks is read again for its bases by the second (from L2).
+    // two shares is read again for its bases by the second (from L2).
     int cta = 0;
     int64_t pos = 0;
     for (int g = 0; g < H; ++g)
@@ -132,10 +157,8 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
             bool open = false;
             for (int t0 = 0; t0 < n; t0 += kTileTokens) {
                 const int t1 = std::min(n, t0 + kTileTokens);
-                // P^K is charged with the first tile, P^V with the last
-                const int64_t c = tile_cost(e, (t1 - t0 + 7) & ~7) +
-                                  (t0 == 0 ? (int64_t)r8(t->rank_k[e]) * d * 2 : 0) +
-                                  (t1 == n ? (int64_t)r8(t->rank_v[e]) * d * 2 : 0);
+                const int64_t c = cost.tile(e, (t1 - t0 + 7) & ~7) + (t0 == 0 ? cost.first(e) : 0) +
+                                  (t1 == n ? cost.last(e) : 0);
                 const double mid = (double)pos + 0.5 * (double)c;
                 int owner = total > 0 ? (int)(mid * P / (double)total) : 0;
                 owner = std::min(std::max(owner, cta), P - 1);
@@ -153,7 +176,7 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
             }
         }
     for (int c = cta + 1; c <= P; ++c) cta_begin[c] = (int32_t)segs.size();
-    // runs and slots: consecutive segments of one thread block with one KV head
+    // runs and slots: consecutive segments of one share with one KV head
     num_slots = 0;
     if (g_slot_begin) g_slot_begin->assign((size_t)H + 1, 0);
     std::vector<int32_t> first_slot_of_g((size_t)H, -1);
@@ -178,6 +201,12 @@ void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::
         gs[H] = num_slots;
         for (int g = H - 1; g >= 0; --g) gs[g] = first_slot_of_g[g] >= 0 ? first_slot_of_g[g] : gs[g + 1];
     }
+}
+
+void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::vector<int32_t> &cta_begin,
+               int &num_slots, std::vector<int32_t> *g_slot_begin)
+{
+    partition_with(t, P, ByteCost{t}, segs, cta_begin, num_slots, g_slot_begin);
 }
 
 // Chunks of the short-block decode: every prefix entry, KV-head-major then in
@@ -282,6 +311,28 @@ struct milo_prefix {
     int max_head_chunks = 0;          // the most chunks of one KV head
     CountersDev *counters = nullptr;
     int32_t *status = nullptr;
+    // tensor-core path: one partition per share count a call can use
+    bool tc = false;                  // calls with at least kTcMinRows rows per KV head may take it
+    struct TcPart {
+        int nshare, seg0, num_slots, max_runs;  // segments at tc_segs + seg0, shares at tc_cta + cta0
+        int cta0;
+    };
+    std::vector<TcPart> tc_parts;
+    SegDev *tc_segs = nullptr;
+    int32_t *tc_cta = nullptr;
+    int sms = 0;
+    int tc_max_shares = 0;            // shares worth at least kTcMinShareCost each
+    int tc_shares(int64_t ntile) const
+    {
+        return (int)std::max<int64_t>(1, std::min<int64_t>(sms / std::max<int64_t>(1, ntile), tc_max_shares));
+    }
+    const TcPart *tc_part(int ntile) const
+    {
+        const int ns = tc_shares(ntile);
+        for (const TcPart &t : tc_parts)
+            if (t.nshare == ns) return &t;
+        return nullptr;
+    }
 };
 
 extern "C" {
@@ -383,6 +434,8 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaFree(plan->chunks);
     cudaFree(plan->counters);
     cudaFree(plan->status);
+    cudaFree(plan->tc_segs);
+    cudaFree(plan->tc_cta);
     cudaSetDevice(cur);
     delete plan;
     return MILO_OK;
@@ -453,6 +506,49 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     for (size_t i = 0; i < segs.size(); ++i) {
         sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
     }
+    // tensor-core path: a partition for every share count sms / ntile that a
+    // call with ntile row tiles of kTcRows rows per KV head uses
+    p->sms = sms;
+    p->tc = G <= 8 && !chunks.empty() && (int64_t)max_batch * G >= kTcMinRows;
+    std::vector<SegDev> tc_sd;
+    std::vector<int32_t> tc_cb;
+    if (p->tc) {
+        // no share below about one 512-token entry of rank 64 (fewer blocks
+        // for small prefixes)
+        const TensorCost tcost{table};
+        int64_t total = 0;
+        for (int64_t x = 0; x < E; ++x) {
+            const int n = table->block_len[x / H];
+            total += tcost.first((int)x) + tcost.last((int)x);
+            for (int t0 = 0; t0 < n; t0 += kTileTokens) total += tcost.tile((int)x, (std::min(n - t0, kTileTokens) + 7) & ~7);
+        }
+        p->tc_max_shares = (int)std::max<int64_t>(1, std::min<int64_t>(sms, total / kTcMinShareCost));
+        const int64_t nt_max = ((int64_t)max_batch * G + kTcRows - 1) / kTcRows;
+        std::vector<int> counts;
+        for (int64_t nt = 1; nt <= nt_max; ++nt) {
+            const int ns = p->tc_shares(nt);
+            if (std::find(counts.begin(), counts.end(), ns) == counts.end()) counts.push_back(ns);
+            if (ns == 1) break;
+        }
+        for (int ns : counts) {
+            std::vector<Seg> ts;
+            std::vector<int32_t> cb;
+            int nslot = 0;
+            partition_with(table, ns, TensorCost{table}, ts, cb, nslot, nullptr);
+            std::vector<int> runs((size_t)H, 0);
+            for (const Seg &x : ts)
+                if (x.flags & kSegFirstOfRun) ++runs[(size_t)(x.entry % H)];
+            milo_prefix::TcPart tp;
+            tp.nshare = ns;
+            tp.seg0 = (int)tc_sd.size();
+            tp.cta0 = (int)tc_cb.size();
+            tp.num_slots = nslot;
+            tp.max_runs = *std::max_element(runs.begin(), runs.end());
+            for (const Seg &x : ts) tc_sd.push_back(SegDev{x.entry, x.t0, x.t1, x.slot, x.flags, {0, 0, 0}});
+            tc_cb.insert(tc_cb.end(), cb.begin(), cb.end());
+            p->tc_parts.push_back(tp);
+        }
+    }
 
     int64_t *loff_dev = nullptr;
     auto cleanup = [&](cudaError_t err, const char *what) {
@@ -481,6 +577,18 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     if ((e = cudaMalloc(&p->status, sizeof(int32_t))) != cudaSuccess) return cleanup(e, "cudaMalloc status");
     if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
         return cleanup(e, "cudaMalloc offsets");
+    if (p->tc) {
+        if ((e = cudaMalloc(&p->tc_segs, sizeof(SegDev) * tc_sd.size())) != cudaSuccess)
+            return cleanup(e, "cudaMalloc tensor-core segments");
+        if ((e = cudaMalloc(&p->tc_cta, sizeof(int32_t) * tc_cb.size())) != cudaSuccess)
+            return cleanup(e, "cudaMalloc tensor-core shares");
+        if ((e = cudaMemcpyAsync(p->tc_segs, tc_sd.data(), sizeof(SegDev) * tc_sd.size(), cudaMemcpyHostToDevice,
+                                 stream)) != cudaSuccess)
+            return cleanup(e, "copy tensor-core segments");
+        if ((e = cudaMemcpyAsync(p->tc_cta, tc_cb.data(), sizeof(int32_t) * tc_cb.size(), cudaMemcpyHostToDevice,
+                                 stream)) != cudaSuccess)
+            return cleanup(e, "copy tensor-core shares");
+    }
 
     if (!ents.empty() &&
         (e = cudaMemcpyAsync(p->entries, ents.data(), sizeof(EntryDev) * ents.size(), cudaMemcpyHostToDevice,
@@ -530,7 +638,10 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t
 namespace {
 struct CallShape {
     int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
-    bool chunked;
+    bool chunked;  // the chunk grid's accumulators and finish grid (paths 0 and 1)
+    int path;      // milo_path_t
+    int ntile;     // tensor-core path: row tiles per KV head
+    const milo_prefix::TcPart *part;
     int64_t records;
     int64_t list_cap, list_bytes;
 };
@@ -546,18 +657,30 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
-    // the short-block decode serves every call with a prefix and G <= 8
+    // the short-block decode serves every call with a prefix and G <= 8; its
+    // prefix part moves to the tensor cores from kTcMinRows rows per KV head
     c.chunked = p->G <= 8 && p->num_chunks > 0;
+    c.ntile = 0;
+    c.part = nullptr;
+    if (c.chunked && p->tc && c.rows_g >= kTcMinRows) {
+        c.ntile = (c.rows_g + kTcRows - 1) / kTcRows;
+        c.part = p->tc_part(c.ntile);
+    }
+    c.path = !c.chunked ? MILO_PATH_PERSISTENT : c.part ? MILO_PATH_TENSOR : MILO_PATH_CHUNKS;
+    if (!c.part) c.ntile = 0;
     // one record per prefix chunk and row group (the short-block decode), or
-    // per run and row group (the persistent kernel); then the tail items.
-    // The short-block decode also lists records: int4 [Hkv][nrg][list_cap],
-    // list_cap bounding the items whose rows meet one row group: the KV
-    // head's chunks, and the tail items of the queries whose G rows meet the
-    // group's 8 rows [8k, 8k + 8), of which there are at most 7 / G + 2.
-    const int64_t prefix = c.chunked ? (int64_t)p->num_chunks * c.nrg : (int64_t)p->num_slots * c.nrg;
+    // per run and row group (the persistent kernel and the tensor-core grid);
+    // then the tail items.  The short-block decode and the tensor-core grid
+    // also list records: int4 [Hkv][nrg][list_cap], list_cap bounding the
+    // items whose rows meet one row group: the KV head's chunks (or runs),
+    // and the tail items of the queries whose G rows meet the group's 8 rows
+    // [8k, 8k + 8), of which there are at most 7 / G + 2.
+    const int64_t prefix = c.part ? (int64_t)c.part->num_slots * c.nrg
+                           : c.chunked ? (int64_t)p->num_chunks * c.nrg : (int64_t)p->num_slots * c.nrg;
     c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
     const int64_t queries_per_group = std::min<int64_t>(batch, 7 / p->G + 2);
-    c.list_cap = c.chunked ? (int64_t)p->max_head_chunks + queries_per_group * c.S : 0;
+    const int64_t prefix_items = c.part ? (int64_t)c.part->max_runs : (int64_t)p->max_head_chunks;
+    c.list_cap = c.chunked ? prefix_items + queries_per_group * c.S : 0;
     c.list_bytes = 16 * (int64_t)p->hkv * c.nrg * c.list_cap;
 
     return c;
@@ -591,7 +714,7 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
             return fail(MILO_ERR_ALIGNMENT, "tails must be 16-byte aligned");
         if (max_tail_tokens > (int64_t)kTailTokens * (1 << 20)) return fail(MILO_ERR_INVALID_ARG, "tail too long");
     }
-    if (reinterpret_cast<uintptr_t>(q) % 4) return fail(MILO_ERR_ALIGNMENT, "q must be 4-byte aligned");
+    if (reinterpret_cast<uintptr_t>(q) % 16) return fail(MILO_ERR_ALIGNMENT, "q must be 16-byte aligned");
     if (reinterpret_cast<uintptr_t>(out) % 16) return fail(MILO_ERR_ALIGNMENT, "out must be 16-byte aligned");
     size_t need = 0;
     milo_workspace_size(plan, batch, max_tail_tokens, &need);
@@ -604,8 +727,11 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
     // the kernels count thread blocks, tail items and list entries in int
     const int64_t tail_items = (int64_t)batch * plan->hkv * c.S;
+    // (the persistent path counts record slots per row group and its merge
+    // grid's blocks per KV head, row group and float4 column in int too)
     if (tail_items > 0x7fffffff || (int64_t)plan->num_chunks * c.nrg + tail_items > 0x7fffffff ||
-        c.list_cap > 0x7fffffff)
+        c.list_cap > 0x7fffffff || (int64_t)plan->num_slots * c.nrg + tail_items * c.nrg_t > 0x7fffffff ||
+        (int64_t)plan->hkv * c.nrg * (plan->d / 4) > 0x7fffffff)
         return fail(MILO_ERR_UNSUPPORTED, "call too large: more than 2^31 - 1 work items");
     DecodeParams prm{};
     prm.packed = plan->packed;
@@ -651,9 +777,15 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     prm.tail_k = static_cast<const uint16_t *>(tail_k);
     prm.tail_v = static_cast<const uint16_t *>(tail_v);
     prm.chunks = plan->chunks;
-    prm.num_chunks = c.chunked ? plan->num_chunks : 0;
+    prm.num_chunks = c.path == MILO_PATH_CHUNKS ? plan->num_chunks : 0;
+    if (c.part) {
+        prm.tc_segs = plan->tc_segs + c.part->seg0;
+        prm.tc_cta_begin = plan->tc_cta + c.part->cta0;
+        prm.tc_ntile = c.ntile;
+        prm.tc_nshare = c.part->nshare;
+    }
     if (c.chunked) {
-        prm.tail_rec_base = (int64_t)plan->num_chunks * c.nrg;
+        prm.tail_rec_base = c.part ? (int64_t)c.part->num_slots * c.nrg : (int64_t)plan->num_chunks * c.nrg;
         // the record lists follow the records
         prm.list_cap = (int)c.list_cap;
         prm.ovf_list = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) +
@@ -683,11 +815,50 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS) return fail(MILO_ERR_CUDA, "tensor map encoding failed");
     }
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    if (c.path == MILO_PATH_TENSOR) {
+        // the dense tails on the chunk grid, then the prefix on the tensor
+        // cores, then the finish grid (each chained by programmatic
+        // dependent launch)
+        cudaError_t e = cudaSuccess;
+        if (prm.num_tail_items > 0 && (e = launch_chunks(prm, &mk, &mv, stream)) != cudaSuccess)
+            return cuda_fail(e, "tail grid launch");
+        if ((e = launch_batch_tc(prm, stream)) != cudaSuccess) return cuda_fail(e, "tensor-core grid launch");
+        if ((e = launch_finish(prm, stream)) != cudaSuccess) return cuda_fail(e, "finish grid launch");
+        return MILO_OK;
+    }
     const int smem = decode_smem_bytes(plan->d, c.nrg_cta);
-    cudaError_t e = launch_decode(prm, &mk, &mv, smem, plan->num_ctas, static_cast<cudaStream_t>(stream_));
+    cudaError_t e = launch_decode(prm, &mk, &mv, smem, plan->num_ctas, stream);
     if (e != cudaSuccess) return cuda_fail(e, "decode launch");
     return MILO_OK;
 }
+
+milo_status_t milo_call_info(const milo_prefix_t *plan, int32_t batch, int64_t max_tail_tokens,
+                             milo_call_info_t *info)
+{
+    if (!plan || !info) return fail(MILO_ERR_INVALID_ARG, "null argument");
+    if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
+    if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
+    const CallShape c = call_shape(plan, batch, max_tail_tokens);
+    info->path = c.path;
+    info->row_tiles = c.ntile;
+    if (c.path == MILO_PATH_TENSOR) {
+        info->kernels = (c.S > 0 ? 1 : 0) + 2;
+        info->blocks = c.part->nshare * c.ntile;
+    } else if (c.path == MILO_PATH_CHUNKS) {
+        info->kernels = 2;
+        const int rg = c.nrg >= 2 ? 2 : 1;
+        const int64_t tail_items = (int64_t)batch * plan->hkv * c.S;
+        info->blocks = (int32_t)std::min<int64_t>(
+            (int64_t)plan->num_chunks * ((c.nrg + rg - 1) / rg) + (tail_items + rg - 1) / rg, 0x7fffffff);
+    } else {
+        info->kernels = 2;
+        info->blocks = plan->num_ctas;
+    }
+    return MILO_OK;
+}
+
+int32_t milo_tensor_min_rows(void) { return kTcMinRows; }
 
 milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q, int32_t batch,
                                       const void *tail_k, const void *tail_v, const int64_t *tail_offsets,

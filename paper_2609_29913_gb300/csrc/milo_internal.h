@@ -65,6 +65,14 @@ struct ChunkDev {
 };
 static_assert(sizeof(ChunkDev) == 64, "chunk descriptor size");
 
+// The tensor-core prefix decode (milo_batch.cu): query rows per tile (the M
+// side of its products), tokens per score tile, bytes per ring slot, and the
+// query rows per KV head from which a call takes it.
+constexpr int kTcRows = 128;
+constexpr int kTcTok = 64;
+constexpr int kTcSlot = 32768;
+constexpr int kTcMinRows = 32;
+
 // Device-side counters owned by a plan (zero between calls).
 struct CountersDev {
     uint32_t tail_next;   // dynamic tail work counter
@@ -109,6 +117,10 @@ struct DecodeParams {
     uint32_t *ovf_cnt;              // [Hkv][nrg]: records listed per (KV head, row group)
     int32_t *ovf_list;              // int4 [Hkv][nrg][list_cap]: listed records (workspace)
     int list_cap;                   // list entries per (KV head, row group)
+    const SegDev *tc_segs;          // tensor-core path: segments of this call's partition
+    const int32_t *tc_cta_begin;    //   [tc_nshare + 1] first segment of each share
+    int tc_ntile;                   //   tiles of kTcRows query rows per KV head
+    int tc_nshare;                  //   shares (thread blocks per row tile)
 };
 
 // Kernel attributes (shared-memory size, carveout) belong to a device: the
@@ -140,6 +152,14 @@ int decode_smem_bytes(int head_dim, int nrg_cta);
 // it when G <= 8.
 cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void *tmap_v, cudaStream_t stream);
 
+
+// The tensor-core prefix grid (a thread block per share and row tile); the
+// call's tail items run on the chunk grid before it, and its finish grid
+// after it.
+cudaError_t launch_batch_tc(const DecodeParams &p, cudaStream_t stream);
+int batch_tc_smem_bytes(int head_dim);
+// The finish grid alone (one warp per KV head and row group).
+cudaError_t launch_finish(const DecodeParams &p, cudaStream_t stream);
 
 // Fixed scratch of milo_attn_decode_static (a file-scope device array).
 constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;

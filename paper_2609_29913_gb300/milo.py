@@ -31,7 +31,9 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
            "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
            "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
-           "milo_get_device_status"]
+           "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows"]
+
+PATH_NAMES = {0: "chunks", 1: "tensor", 2: "persistent"}
 
 
 class MiloError(RuntimeError):
@@ -48,6 +50,11 @@ class BlockTableC(ctypes.Structure):
                 ("off_pk", ctypes.c_void_p), ("off_cv", ctypes.c_void_p),
                 ("off_pv", ctypes.c_void_p), ("arena", ctypes.c_void_p),
                 ("arena_elems", ctypes.c_int64)]
+
+
+class CallInfoC(ctypes.Structure):
+    _fields_ = [("path", ctypes.c_int32), ("kernels", ctypes.c_int32),
+                ("row_tiles", ctypes.c_int32), ("blocks", ctypes.c_int32)]
 
 
 class PrefixInfoC(ctypes.Structure):
@@ -86,10 +93,12 @@ def lib():
                                        ctypes.c_size_t, P]
         L.milo_attn_decode_static.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
+        L.milo_call_info.argtypes = [P, i32, i64, P]
+        L.milo_tensor_min_rows.restype = i32
         for name in ("milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
                      "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
-                     "milo_get_device_status"):
+                     "milo_get_device_status", "milo_call_info"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -211,6 +220,19 @@ def milo_workspace_size(plan: int, batch: int, max_tail_tokens: int) -> int:
     _check(lib().milo_workspace_size(plan, int(batch), int(max_tail_tokens), ctypes.byref(n)),
            "milo_workspace_size")
     return int(n.value)
+
+
+def milo_call_info(plan: int, batch: int, max_tail_tokens: int) -> dict:
+    """How a call of this shape runs: path (0 chunks, 1 tensor, 2 persistent),
+    kernels per call, row tiles and main-grid blocks (host only)."""
+    info = CallInfoC()
+    _check(lib().milo_call_info(plan, int(batch), int(max_tail_tokens), ctypes.byref(info)),
+           "milo_call_info")
+    return {name: getattr(info, name) for name, _ in CallInfoC._fields_}
+
+
+def milo_tensor_min_rows() -> int:
+    return int(lib().milo_tensor_min_rows())
 
 
 def milo_attn_decode(plan: int, q_ptr: int, batch: int, tail_k_ptr: int, tail_v_ptr: int,

@@ -69,6 +69,22 @@ CASES = {
 }
 
 
+def test_rank0_entries_mixed_with_others_d128(env):
+    """Entries of rank 0 in K and V, in K only and in V only, between entries
+    of rank 16 and 128, in one plan at head dimension 128 (an entry of rank 0
+    in both has no coefficient rows: its chunk's piece copies nothing)."""
+    W = env["W"]
+    #          block:  0        1        2         3        4
+    rk = np.array([[0, 16], [0, 128], [16, 0], [128, 0], [0, 0]], dtype=np.int32)
+    rv = np.array([[0, 0], [128, 0], [0, 16], [0, 128], [16, 0]], dtype=np.int32)
+    layer = W.build_layer(14, 2, 128, [40, 512, 96, 300, 33], rk, rv, batch=2, tail_lengths=[17, 70],
+                          seed=12, device="cuda")
+    out, pre = decode(env, layer)
+    ref = env["oracle"].attention(**layer.to_numpy_bits())
+    compare(out.cpu().numpy(), ref, "rank0 mixed d128")
+    pre.close()
+
+
 @pytest.mark.parametrize("name", sorted(CASES))
 def test_small_cases_match_oracle(env, name):
     hq, hkv, d, bl, ranks, batch, tails, sep = CASES[name]
@@ -372,12 +388,37 @@ def test_qwen7b_batch1_layers_full(env, layer_idx):
     compare(out.cpu().numpy(), env["oracle"].attention(**layer.to_numpy_bits()), f"qwen7b-28L-32k-b1 L{layer_idx}")
 
 
-@pytest.mark.parametrize("name,queries,heads", [("qwen7b-28L-32k-b64", [0, 63], [0, 3]),
-                                                ("qwen14b-48L-128k-b16", [0, 15], [0, 7]),
-                                                ("qwen7b-1L-1M-b8", [0, 5], [1])])
-def test_batched_workloads_sampled(env, name, queries, heads):
+def worst_row_rel_l2(got, ref):
+    """The largest relative L2 error over the (query, head) rows."""
+    d = got.shape[-1]
+    g = np.asarray(got, np.float64).reshape(-1, d)
+    r = np.asarray(ref, np.float64).reshape(-1, d)
+    return float((np.linalg.norm(g - r, axis=1) / np.maximum(np.linalg.norm(r, axis=1), 1e-30)).max())
+
+
+@pytest.mark.parametrize("name", ["qwen7b-28L-32k-b64", "qwen14b-48L-128k-b16", "qwen7b-1L-1M-b8"])
+def test_batched_workloads_whole_layer(env, name):
+    """Layer 0 of each batched workload against the oracle over the whole
+    output tensor [batch, Hq, d] (every query, every head)."""
     W = env["W"]
     layer = W.make_config_layer(W.by_name(name), 0, device="cuda")
+    out, pre = decode(env, layer)
+    got = out.cpu().numpy()
+    ref = env["oracle"].attention(**layer.to_numpy_bits())
+    err, rel = compare(got, ref, f"{name} layer 0")
+    print(f"{name} layer 0: max-abs {err:.3e} rel-L2 {rel:.3e} "
+          f"worst (query, head) rel-L2 {worst_row_rel_l2(got, ref):.3e}")
+    pre.close()
+
+
+@pytest.mark.parametrize("name,queries,heads", [("qwen7b-28L-32k-b64", [0, 63], [0, 3]),
+                                                ("qwen14b-48L-128k-b16", [0, 15], [0, 7])])
+def test_batched_workloads_last_layer_sampled(env, name, queries, heads):
+    """The last layer of the multi-layer batched workloads on a few (query,
+    KV head) subsets, each an exact subproblem the oracle solves alone."""
+    W = env["W"]
+    cfg = W.by_name(name)
+    layer = W.make_config_layer(cfg, cfg.layers - 1, device="cuda")
     out, _ = decode(env, layer)
     G = layer.num_q_heads // layer.num_kv_heads
     o = out.cpu().numpy()
