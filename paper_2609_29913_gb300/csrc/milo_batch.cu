@@ -6,15 +6,15 @@
 // tiles of 128 rows, the M side of every product, so each product serves 128
 // rows at once (Eq. 3 substituted into Eq. 1, Alg. 1 Stage 2):
 //
-//   projection       Q~  = Q P^K^T       A = q rows (K = d),      B = P^K  (N = ranks)
-//   scores           S   = Q~ C^K^T      A = q~ hi, lo (K = ranks), B = C^K tile (N = 64 tokens)
-//   values           V~ += P C^V         A = p hi, lo (K = tokens), B = C^V tile (N = ranks)
-//   back-projection  O  += V~ P^V        A = v~ hi, lo (K = ranks), B = P^V  (N = d)
+//   projection       Q~  = Q P^K^T    A = q rows (smem, K = d)          B = P^K      (N = ranks)
+//   scores           S   = Q~ C^K^T   A = q~ hi, lo (smem, K = ranks)   B = C^K tile (N = 64 tokens)
+//   values           V~ += P C^V      A = p hi, lo (tmem, K = tokens)   B = C^V tile (N = ranks)
+//   back-projection  O  += V~ P^V     A = v~ hi, lo (tmem, K = ranks)   B = P^V      (N = d)
 //
 // q~, p and v~ are fp32 values that enter a product as two bf16 operands,
-// the value rounded to bf16 ("hi") and its rounding residual ("lo"), so they
-// keep ~16 significant bits; the factors and q are bf16 data and enter once.
-// Scores are in log2 units: q~ carries softmax scale x log2(e).
+// the value rounded to bf16 ("hi") and its residual ("lo"), so they keep ~16
+// significant bits; the factors and q are bf16 data and enter once.  Scores
+// are in log2 units: q~ carries softmax scale x log2(e).
 //
 // Work: the prefix (every entry's tokens, KV-head-major, then table order)
 // is cut on the host into near-equal shares at 32-token boundaries
@@ -29,21 +29,31 @@
 // tensor-memory columns):
 //   warp 0, lane 0   producer: bulk copies of the segment pieces (P^K, then
 //                    C^K + C^V rows of whole 64-token tiles up to 32 KB,
-//                    then P^V) into a ring of two 32 KB slots;
-//   warp 1           owns the tensor memory; lane 0 issues every MMA;
+//                    then P^V) into a ring of four 32 KB slots;
+//   warp 1           owns the tensor memory and walks the MMA schedule as a
+//                    converged warp; one elected lane issues every MMA;
 //   warps 2-5        softmax: thread t owns row t of the tile and tensor
 //                    memory lane t (warp w reaches lanes 32 (w % 4) ..).
-// Within a segment the score tile j + 1 is computed while the softmax works
-// on tile j (two score buffers in tensor memory, two p buffers in shared
-// memory).  The online softmax raises a row's reference maximum lazily (only
-// when a score passes it by kLazyTc), rescaling V~ and O in tensor memory
-// when it does.
+// Tensor memory: two score tiles (each overwritten in place by its p hi, lo
+// once read), q~ as projected, v~ (converted in place to its hi, lo at a
+// segment's end), O.  The score products run two tiles ahead of the value
+// products, so the softmax of tile j overlaps the products of tiles j - 1
+// and j + 1.  tcgen05.mma operations of one thread execute in issue order,
+// which orders a score product after the value product that read the p
+// tile it overwrites, and a segment's first value product after the
+// previous segment's back-projection.  At a segment's end the next
+// segment's projection, q~ and first score products go ahead of this
+// segment's back-projection.
 //
-// Every mbarrier wait is bounded (~2 s): a wait that gives up sets
+// The online softmax raises a row's reference maximum lazily (only when a
+// score passes it by kLazyTc), rescaling V~ and O in tensor memory when it
+// does.  Every mbarrier wait is bounded (~2 s): a wait that gives up sets
 // MILO_ERR_TIMEOUT in the status word and a shared abort flag, after which
 // every role skips its remaining work, so the block always ends.
 #include <cuda.h>
 #include <cuda_bf16.h>
+
+#include <type_traits>
 
 #include "milo.h"
 #include "milo_internal.h"
@@ -54,11 +64,11 @@ namespace milo {
 namespace {
 
 constexpr int kTcThreads = 192;
-constexpr int kTcSlots = 2;
+constexpr int kTcSlots = 4;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0;    // two score tiles of kTcTok columns
+constexpr uint32_t kColS = 0;    // two score tiles of kTcTok columns (then p hi | p lo)
 constexpr uint32_t kColQ = 128;  // projection result q~ (fp32, up to 128 ranks)
-constexpr uint32_t kColV = 256;  // rank-space values v~ (fp32, up to 128 ranks)
+constexpr uint32_t kColV = 256;  // rank-space values v~ (fp32; then v~ hi at +0, lo at +64)
 constexpr uint32_t kColO = 384;  // output O (fp32, d columns)
 constexpr float kLazyTc = 8.f;   // a row's reference maximum moves when a score passes it by this
 
@@ -70,11 +80,10 @@ enum : int {
     TB_PROJ,                        // projection done (commit)
     TB_QT,                          // q~ staged (4)
     TB_SFULL,                       // [2] score tile done (commit)
-    TB_SFREE = TB_SFULL + 2,        // [2] score tile read (4)
-    TB_PREADY = TB_SFREE + 2,       // [2] p tile staged (4)
+    TB_PREADY = TB_SFULL + 2,       // [2] p tile written (4)
     TB_PVDONE = TB_PREADY + 2,      // [2] value products of that p tile done (commit)
     TB_VDONE = TB_PVDONE + 2,       // every value product of a segment done (commit)
-    TB_VSTAGED,                     // v~ staged for the back-projection (4)
+    TB_VSTAGED,                     // v~ hi, lo written for the back-projection (4)
     TB_BPDONE,                      // back-projection done (commit)
     TB_FIN,                         // every MMA of the block done (commit)
     TB_NBAR
@@ -85,13 +94,9 @@ struct TcLay {
     static constexpr int kQ = kTcSlots * kTcSlot;                 // after the ring: q rows, cores [16 row groups][D/8]
     static constexpr int kQt = kQ + kTcRows * D * 2;              // q~ hi, then lo: cores [16][D/8] each
     static constexpr int kQtHalf = kTcRows * D * 2;
-    static constexpr int kP = kQt + 2 * kQtHalf;                  // two p tiles (hi, lo: cores [16][8] each);
-    static constexpr int kPHalf = kTcRows * kTcTok * 2;           //   v~ hi, lo at a segment's end
-    static constexpr int kPBuf = 2 * kPHalf;
-    static constexpr int kBar = kP + 2 * kPBuf;
+    static constexpr int kBar = kQt + 2 * kQtHalf;
     static constexpr int kFlag = kBar + TB_NBAR * 8;              // abort flag, tensor-memory base
     static constexpr int kTotal = kFlag + 16;
-    static_assert(2 * kQtHalf <= 2 * kPBuf, "v~ hi and lo fit the two p tiles");
     static_assert(kTotal <= 232448, "one block per SM");
 };
 
@@ -111,24 +116,51 @@ __device__ __forceinline__ uint32_t idesc(bool a_mn, bool b_mn, int n)
     return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
            ((uint32_t)(n >> 3) << 17) | ((128u >> 4) << 24);
 }
-__device__ __forceinline__ void umma(uint32_t d, uint64_t a, uint64_t b, uint32_t id, bool acc)
+// D (+)= A B with A and B in shared memory
+__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t id, bool acc)
 {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
         "l"(a), "l"(b), "r"(id), "r"((int)acc));
 }
-// n products into one accumulator: step k reads A at a + k a_step and B at
-// b + k b_step (bytes; the address is the descriptor's low field, in 16-byte
-// units); step 0 overwrites D unless acc0.
-__device__ __forceinline__ void umma_n(uint32_t d, uint64_t a, uint64_t b, uint32_t a_step, uint32_t b_step, int n,
+// D (+)= A B with A in tensor memory (row m on lane m, two bf16 a column)
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t id, bool acc)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+        "r"(a), "l"(b), "r"(id), "r"((int)acc));
+}
+// N products into one accumulator, unrolled: step k reads A at a + k a_step
+// and B at b + k b_step (descriptor units of 16 bytes; tensor-memory A: 8
+// columns = 16 bf16 a step); step 0 overwrites D unless acc0.
+template <int N>
+__device__ __forceinline__ void seq_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t a_step, uint32_t b_step,
                                        uint32_t id, bool acc0)
 {
-#pragma unroll 1
-    for (int k = 0; k < n; ++k) {
-        umma(d, a, b, id, k > 0 || acc0);
-        a += a_step >> 4;
-        b += b_step >> 4;
+#pragma unroll
+    for (int k = 0; k < N; ++k) mma_ss(d, a + (uint64_t)(k * a_step), b + (uint64_t)(k * b_step), id, k > 0 || acc0);
+}
+template <int N>
+__device__ __forceinline__ void seq_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t b_step, uint32_t id, bool acc0)
+{
+#pragma unroll
+    for (int k = 0; k < N; ++k) mma_ts(d, a + 8u * k, b + (uint64_t)(k * b_step), id, k > 0 || acc0);
+}
+// f(integral_constant<int, n>) for a runtime n in 1..8
+template <class F>
+__device__ __forceinline__ void steps(int n, F &&f)
+{
+    switch (n) {
+    case 1: f(std::integral_constant<int, 1>{}); break;
+    case 2: f(std::integral_constant<int, 2>{}); break;
+    case 3: f(std::integral_constant<int, 3>{}); break;
+    case 4: f(std::integral_constant<int, 4>{}); break;
+    case 5: f(std::integral_constant<int, 5>{}); break;
+    case 6: f(std::integral_constant<int, 6>{}); break;
+    case 7: f(std::integral_constant<int, 7>{}); break;
+    default: f(std::integral_constant<int, 8>{}); break;
     }
 }
 // mbarrier arrival once every MMA issued so far by this thread has completed
@@ -140,34 +172,53 @@ __device__ __forceinline__ void commit(uint32_t bar)
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-// 16 consecutive fp32 columns of this warp's 32 lanes (no wait)
-__device__ __forceinline__ void ld16(uint32_t taddr, float (&v)[16])
+// 16 consecutive 32-bit columns of this warp's 32 lanes (no wait)
+__device__ __forceinline__ void ld16(uint32_t taddr, uint32_t (&r)[16])
 {
-    uint32_t r[16];
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
           "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
         : "r"(taddr)
         : "memory");
+}
+__device__ __forceinline__ void ld16f(uint32_t taddr, float (&v)[16])
+{
+    uint32_t r[16];
+    ld16(taddr, r);
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 __device__ __forceinline__ void wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-__device__ __forceinline__ void st16(uint32_t taddr, const float (&v)[16])
+__device__ __forceinline__ void st8(uint32_t taddr, const uint32_t *r)
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
+                 "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+                 : "memory");
+}
+__device__ __forceinline__ void st16(uint32_t taddr, const uint32_t *r)
 {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
             taddr),
-        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
-        "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
-        "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])),
-        "r"(__float_as_uint(v[11])), "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])),
-        "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15]))
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+        "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
         : "memory");
 }
 __device__ __forceinline__ void wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 }  // namespace tc
+
+// Two fp32 values as a bf16x2 "hi" (each rounded to 8 significant bits,
+// ties away from zero, by integer arithmetic) and the bf16x2 of their
+// residuals (truncated): x = hi + lo to ~2^-17 relative.  Low half = x0.
+__device__ __forceinline__ void split2(float x0, float x1, uint32_t &hi, uint32_t &lo)
+{
+    const uint32_t h0 = (__float_as_uint(x0) + 0x8000u) & 0xffff0000u;
+    const uint32_t h1 = (__float_as_uint(x1) + 0x8000u) & 0xffff0000u;
+    const float r0 = x0 - __uint_as_float(h0), r1 = x1 - __uint_as_float(h1);
+    hi = __byte_perm(h0, h1, 0x7632);
+    lo = __byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x7632);
+}
 
 // 16 fp32 values of one row as bf16 hi + lo into two K-major cores each
 // (columns 8c .. 8c + 15 of the row): hi cores at `hi`, hi + 128, lo cores at
@@ -176,7 +227,7 @@ __device__ __forceinline__ void put16(uint8_t *hi, uint8_t *lo, const float (&x)
 {
     uint32_t h[8], l[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) split_hi_lo(x[2 * j], x[2 * j + 1], h[j], l[j]);
+    for (int j = 0; j < 8; ++j) split2(x[2 * j], x[2 * j + 1], h[j], l[j]);
     *reinterpret_cast<uint4 *>(hi) = make_uint4(h[0], h[1], h[2], h[3]);
     *reinterpret_cast<uint4 *>(hi + 128) = make_uint4(h[4], h[5], h[6], h[7]);
     *reinterpret_cast<uint4 *>(lo) = make_uint4(l[0], l[1], l[2], l[3]);
@@ -202,12 +253,13 @@ __device__ __forceinline__ bool tc_wait(uint32_t bar, uint32_t parity, int32_t *
     }
 }
 
-// What a segment (tokens [t0, t1) of one entry) needs, as both the producer
-// and the MMA issuer walk it.
+// What a segment (tokens [t0, t1) of one entry) needs, as the producer, the
+// MMA issuer and the softmax walk it.
 struct SegPlan {
     int64_t ck, pk, cv, pv;  // packed byte offsets (C at token 0 of the entry)
     int n8;                  // entry tokens rounded up to 8
     int rk, rv, rk8, rv8;    // ranks and rank 8-groups
+    int nk16, nv16;          // 16-rank steps
     int g, t0, t1;
     int ntiles, tpp, nc;     // 64-token tiles, tiles per C piece, C pieces
     bool first_of_run, last_of_run;
@@ -228,6 +280,8 @@ __device__ __forceinline__ SegPlan seg_plan(const DecodeParams &p, int s)
     q.rv = e.rv;
     q.rk8 = (e.rk + 7) / 8;
     q.rv8 = (e.rv + 7) / 8;
+    q.nk16 = (q.rk8 + 1) / 2;
+    q.nv16 = (q.rv8 + 1) / 2;
     q.g = e.g;
     q.t0 = sd.t0;
     q.t1 = sd.t1;
@@ -266,8 +320,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
     const int s_begin = p.tc_cta_begin[share], s_end = p.tc_cta_begin[share + 1];
 
     pdl_trigger();
-    // zero the ring, q rows, q~ and p areas: every later read past a piece's
-    // data (rank and token padding of the products) sees finite values
+    // zero the ring, q rows and q~: every later read past a piece's data
+    // (rank and token padding of the products) sees finite values
     for (int i = tid; i < L::kBar / 16; i += kTcThreads) reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
     if (tid == 0) {
         for (int i = 0; i < kTcSlots; ++i) {
@@ -279,7 +333,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
         mbar_init(bar(TB_QT), 4);
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(TB_SFULL + i), 1);
-            mbar_init(bar(TB_SFREE + i), 4);
             mbar_init(bar(TB_PREADY + i), 4);
             mbar_init(bar(TB_PVDONE + i), 1);
         }
@@ -349,119 +402,164 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
+        // The whole warp walks the schedule (every value warp-uniform) and
+        // one elected lane issues the products and their commits: issuing
+        // from a converged warp keeps the tensor pipe fed, where a lone
+        // lane branching between products left it idle most of the time.
         pdl_wait();
-        if (lane == 0) {
-            int n = 0;      // pieces consumed (in producer order)
-            int J = 0;      // score tiles issued (global over segments)
-            int kseg = 0;   // segments
-            int krun = 0;   // runs
-            bool o_acc = false;
-            bool ok = true;
-            auto take = [&](int &slot) {
-                slot = n % kTcSlots;
-                ok = ok && tc_wait(bar(TB_FULL + slot), (n / kTcSlots) & 1, p.status, abort_flag);
-                ++n;
-                tc::fence_after();
-                return sbase + (uint32_t)slot * kTcSlot;
-            };
-            const uint32_t q_u = sbase + L::kQ, qt_u = sbase + L::kQt, p_u = sbase + L::kP;
-            for (int s = s_begin; ok && s < s_end; ++s) {
-                const SegPlan q = seg_plan(p, s);
-                const int nk16 = (q.rk8 + 1) / 2, nv16 = (q.rv8 + 1) / 2;  // 16-rank steps
-                if (q.first_of_run) {
-                    ok = ok && tc_wait(bar(TB_QROWS), krun & 1, p.status, abort_flag);
-                    ++krun;
-                    o_acc = false;
-                    tc::fence_after();
-                }
-                // projection q~ = Q P^K^T into kColQ (N = 16 nk16 ranks, K = d)
+        int n = 0;      // pieces consumed (in producer order)
+        int krun = 0;   // runs whose q rows were waited for
+        bool ok = true;
+        auto wait = [&](int b, int parity) {
+            ok = __all_sync(0xffffffffu, ok && tc_wait(bar(b), (uint32_t)parity & 1u, p.status, abort_flag));
+            tc::fence_after();
+        };
+        // f() on one elected lane (always lane 0: the warp is converged)
+        auto on_one = [&](auto &&f) {
+            uint32_t pred;
+            asm volatile("{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\tselp.u32 %0, 1, 0, e;\n\t}" : "=r"(pred));
+            if (pred) f();
+            __syncwarp();
+        };
+        auto take = [&](int &slot) {
+            slot = n % kTcSlots;
+            wait(TB_FULL + slot, n / kTcSlots);
+            ++n;
+            return sbase + (uint32_t)slot * kTcSlot;
+        };
+        const uint32_t q_u = sbase + L::kQ, qt_u = sbase + L::kQt;
+        // projection of segment q (waits for the run's q rows first)
+        auto project = [&](const SegPlan &q) {
+            if (q.first_of_run) {
+                wait(TB_QROWS, krun);
+                ++krun;
+            }
+            int sl = 0;
+            uint32_t pk = 0;
+            if (q.rk > 0) pk = take(sl);
+            const bool go = ok;
+            on_one([&] {
                 if (q.rk > 0) {
-                    int sl;
-                    const uint32_t pk = take(sl);
-                    if (ok)
-                        tc::umma_n(tmem + kColQ, tc::sdesc(q_u, 128, DG * 128), tc::sdesc(pk, 128, DG * 128), 256, 256,
-                                   D / 16, tc::idesc(false, false, 16 * nk16), false);
+                    if (go)
+                        tc::seq_ss<D / 16>(tmem + kColQ, tc::sdesc(q_u, 128, DG * 128), tc::sdesc(pk, 128, DG * 128),
+                                           16, 16, tc::idesc(false, false, 16 * q.nk16), false);
                     tc::commit(bar(TB_EMPTY + sl));
                 }
                 tc::commit(bar(TB_PROJ));
-                ok = ok && tc_wait(bar(TB_QT), kseg & 1, p.status, abort_flag);
-                tc::fence_after();
-                // tiles: S_j is issued before the value products of tile j - 1
-                int cur_slot = -1, prev_slot = -1;
-                uint32_t cur = 0, cvb = 0, prev_cvb = 0;
-                const int J0 = J;
-                for (int j = 0; ok && j <= q.ntiles; ++j) {
-                    if (j < q.ntiles) {
-                        const int c = q.nc > 0 ? j / q.tpp : 0, jj = q.nc > 0 ? j % q.tpp : 0;
-                        if (q.nc > 0 && jj == 0) {
-                            prev_slot = cur_slot;
-                            prev_cvb = cvb;
-                            cur = take(cur_slot);
-                            int a, rows;
-                            c_piece_rows(q, c, a, rows);
-                            cvb = cur + (uint32_t)rows * q.rk8 * 16;
-                        }
-                        const int b = (J0 + j) & 1, u = (J0 + j) >> 1;
-                        if (J0 + j >= 2) ok = ok && tc_wait(bar(TB_SFREE + b), (u - 1) & 1, p.status, abort_flag);
-                        tc::fence_after();
-                        if (ok && q.rk > 0) {
-                            const uint32_t kt = cur + (uint32_t)jj * 8 * q.rk8 * 128;
-                            const uint32_t id = tc::idesc(false, false, kTcTok);
-                            tc::umma_n(tmem + kColS + kTcTok * b, tc::sdesc(qt_u, 128, DG * 128),
-                                       tc::sdesc(kt, 128, q.rk8 * 128), 256, 256, nk16, id, false);
-                            tc::umma_n(tmem + kColS + kTcTok * b, tc::sdesc(qt_u + L::kQtHalf, 128, DG * 128),
-                                       tc::sdesc(kt, 128, q.rk8 * 128), 256, 256, nk16, id, true);
-                        }
-                        tc::commit(bar(TB_SFULL + b));
-                    }
-                    if (j > 0) {
-                        // value products of tile jt = j - 1
-                        const int jt = j - 1, Jt = J0 + jt, b = Jt & 1;
-                        const int jj = q.nc > 0 ? jt % q.tpp : 0;
-                        // the tile's piece: the current one, unless tile j opened a new piece
-                        const bool in_prev = q.nc > 0 && j < q.ntiles && (j % q.tpp) == 0;
-                        const uint32_t vbase = in_prev ? prev_cvb : cvb;
-                        ok = ok && tc_wait(bar(TB_PREADY + b), (Jt >> 1) & 1, p.status, abort_flag);
-                        tc::fence_after();
-                        if (ok && q.rv > 0) {
-                            const uint32_t vt = vbase + (uint32_t)jj * 8 * q.rv8 * 128;
-                            const uint32_t id = tc::idesc(false, true, 16 * nv16);
-                            const uint32_t pa = p_u + (uint32_t)b * L::kPBuf;
-                            tc::umma_n(tmem + kColV, tc::sdesc(pa, 128, 8 * 128), tc::sdesc(vt, q.rv8 * 128, 128), 256,
-                                       2 * q.rv8 * 128, kTcTok / 16, id, jt > 0);
-                            tc::umma_n(tmem + kColV, tc::sdesc(pa + L::kPHalf, 128, 8 * 128),
-                                       tc::sdesc(vt, q.rv8 * 128, 128), 256, 2 * q.rv8 * 128, kTcTok / 16, id, true);
-                        }
-                        tc::commit(bar(TB_PVDONE + b));
-                        // the last tile of a piece releases its slot
-                        if (q.nc > 0 && (jt % q.tpp == q.tpp - 1 || jt == q.ntiles - 1))
-                            tc::commit(bar(TB_EMPTY + (in_prev ? prev_slot : cur_slot)));
-                    }
-                }
-                J = J0 + q.ntiles;
-                tc::commit(bar(TB_VDONE));
-                // back-projection O += V~ P^V (N = d, K = 16 nv16 ranks)
-                int pv_slot = -1;
-                uint32_t pvu = 0;
-                if (q.rv > 0) pvu = take(pv_slot);
-                ok = ok && tc_wait(bar(TB_VSTAGED), kseg & 1, p.status, abort_flag);
-                tc::fence_after();
-                if (ok && q.rv > 0) {
+            });
+        };
+        // the back-projection of a segment, issued once the next segment's
+        // first score products are on their way
+        SegPlan bq = {};
+        int bp_slot = -1, bp_k = 0;
+        uint32_t bp_u = 0;
+        bool o_acc = false;  // O already holds part of the run of the pending back-projection
+        auto back_project = [&]() {
+            wait(TB_VSTAGED, bp_k);
+            const bool go = ok && bq.rv > 0, acc = o_acc;
+            on_one([&] {
+                if (go) {
+                    // O += v~ P^V: A = v~ hi, then lo (tensor memory), K = 16 nv16 ranks, N = d
                     const uint32_t id = tc::idesc(false, true, D);
-                    tc::umma_n(tmem + kColO, tc::sdesc(p_u, 128, DG * 128), tc::sdesc(pvu, DG * 128, 128), 256,
-                               2 * DG * 128, nv16, id, o_acc);
-                    tc::umma_n(tmem + kColO, tc::sdesc(p_u + L::kQtHalf, 128, DG * 128), tc::sdesc(pvu, DG * 128, 128),
-                               256, 2 * DG * 128, nv16, id, true);
-                    o_acc = true;
+                    const uint64_t bd = tc::sdesc(bp_u, DG * 128, 128);
+                    tc::steps(bq.nv16, [&](auto nc) {
+                        constexpr int N = decltype(nc)::value;
+                        tc::seq_ts<N>(tmem + kColO, tmem + kColV, bd, (2 * DG * 128) >> 4, id, acc);
+                        tc::seq_ts<N>(tmem + kColO, tmem + kColV + 64, bd, (2 * DG * 128) >> 4, id, true);
+                    });
                 }
                 tc::commit(bar(TB_BPDONE));
-                if (q.rv > 0) tc::commit(bar(TB_EMPTY + pv_slot));
-                ++kseg;
+                if (bq.rv > 0) tc::commit(bar(TB_EMPTY + bp_slot));
+            });
+            if (go) o_acc = true;
+        };
+        // C pieces of the current segment, taken in order by the score
+        // products and released by the value products: at most two are live
+        // (tiles j + 1 and j + 2 once tile j's values are issued)
+        struct Piece {
+            uint32_t base, cvb;
+            int slot;
+        };
+        Piece pc[2] = {};
+        int kseg = 0, J = 0;
+        if (s_begin < s_end) project(seg_plan(p, s_begin));
+        for (int s = s_begin; ok && s < s_end; ++s, ++kseg) {
+            const SegPlan q = seg_plan(p, s);
+            const int J0 = J;
+            // the score product of tile j into buffer (J0 + j) & 1 (after the
+            // value product that read that buffer's last p tile, by issue
+            // order)
+            auto score = [&](int j) {
+                if (q.nc > 0 && j % q.tpp == 0) {
+                    const int c = j / q.tpp;
+                    Piece &x = pc[c & 1];
+                    x.base = take(x.slot);
+                    int a, rows;
+                    c_piece_rows(q, c, a, rows);
+                    x.cvb = x.base + (uint32_t)rows * q.rk8 * 16;
+                }
+                const int b = (J0 + j) & 1;
+                const bool go = ok && q.rk > 0;
+                const uint32_t kt = pc[(q.nc > 0 ? j / q.tpp : 0) & 1].base + (uint32_t)(j % q.tpp) * 8 * q.rk8 * 128;
+                on_one([&] {
+                    if (go) {
+                        const uint32_t id = tc::idesc(false, false, kTcTok);
+                        const uint64_t bd = tc::sdesc(kt, 128, q.rk8 * 128);
+                        tc::steps(q.nk16, [&](auto nc) {
+                            constexpr int N = decltype(nc)::value;
+                            tc::seq_ss<N>(tmem + kColS + kTcTok * b, tc::sdesc(qt_u, 128, DG * 128), bd, 16, 16, id,
+                                          false);
+                            tc::seq_ss<N>(tmem + kColS + kTcTok * b, tc::sdesc(qt_u + L::kQtHalf, 128, DG * 128), bd,
+                                          16, 16, id, true);
+                        });
+                    }
+                    tc::commit(bar(TB_SFULL + b));
+                });
+            };
+            // this segment's q~ is staged: its first two score products, then
+            // the previous segment's back-projection (before this segment's
+            // first value product overwrites v~)
+            wait(TB_QT, kseg);
+            if (ok) score(0);
+            if (ok && q.ntiles > 1) score(1);
+            if (kseg > 0) back_project();
+            if (q.first_of_run) o_acc = false;
+            for (int j = 0; ok && j < q.ntiles; ++j) {
+                const int Jt = J0 + j, b = Jt & 1;
+                wait(TB_PREADY + b, Jt >> 1);
+                const Piece x = pc[(q.nc > 0 ? j / q.tpp : 0) & 1];
+                const bool go = ok && q.rv > 0;
+                const bool release = q.nc > 0 && (j % q.tpp == q.tpp - 1 || j == q.ntiles - 1);
+                const uint32_t vt = x.cvb + (uint32_t)(j % q.tpp) * 8 * q.rv8 * 128;
+                on_one([&] {
+                    if (go) {
+                        // v~ += p C^V: A = p hi, then lo (tensor memory), K = 64 tokens
+                        const uint32_t id = tc::idesc(false, true, 16 * q.nv16);
+                        const uint64_t bd = tc::sdesc(vt, q.rv8 * 128, 128);
+                        const uint32_t pa = tmem + kColS + kTcTok * b;
+                        tc::seq_ts<kTcTok / 16>(tmem + kColV, pa, bd, (2 * q.rv8 * 128) >> 4, id, j > 0);
+                        tc::seq_ts<kTcTok / 16>(tmem + kColV, pa + kTcTok / 2, bd, (2 * q.rv8 * 128) >> 4, id, true);
+                    }
+                    tc::commit(bar(TB_PVDONE + b));
+                    // the last tile of a piece releases its slot
+                    if (release) tc::commit(bar(TB_EMPTY + x.slot));
+                });
+                if (ok && j + 2 < q.ntiles) score(j + 2);
             }
-            tc::commit(bar(TB_FIN));
-            mbar_wait(bar(TB_FIN), 0, p.status);
+            J = J0 + q.ntiles;
+            on_one([&] { tc::commit(bar(TB_VDONE)); });
+            // this segment's back-projection waits for the next one's
+            // projection and first score products
+            bq = q;
+            bp_k = kseg;
+            if (q.rv > 0) bp_u = take(bp_slot);
+            if (s + 1 < s_end) project(seg_plan(p, s + 1));
         }
-        __syncwarp();
+        if (ok && kseg > 0) back_project();
+        on_one([&] { tc::commit(bar(TB_FIN)); });
+        // (not given up on an abort: the tensor memory is released after it)
+        mbar_wait(bar(TB_FIN), 0, p.status);
+        tc::fence_after();
     } else {
         // ------------------------------------------------ softmax
         const int quad = warp & 3;                // tensor-memory lane quarter of this warp
@@ -469,10 +567,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
         const int row = tile * kTcRows + rl;      // the KV head's query row (batch x heads)
         const bool row_ok = row < p.rows_g;
         const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
-        uint8_t *q_s = smem + L::kQ, *qt_s = smem + L::kQt, *p_s = smem + L::kP;
+        uint8_t *q_s = smem + L::kQ, *qt_s = smem + L::kQt;
         const int rg8 = rl >> 3, r8 = rl & 7;     // core row group and row within the core
         pdl_wait();  // q and the accumulators belong to the preceding grids until here
-        int J = 0, kseg = 0;
+        int J = 0, kseg = 0, kproj = 0;
         bool ok = true;
         float m = -INFINITY, l = 0.f;
         bool o_written = false, first_tile = true;
@@ -486,13 +584,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
         auto wwait = [&](int b, int parity) {
             ok = __all_sync(0xffffffffu, ok && tc_wait(bar(b), (uint32_t)parity & 1u, p.status, abort_flag));
         };
-        for (int s = s_begin; s < s_end; ++s) {
-            const SegPlan q = seg_plan(p, s);
-            const int g = q.g;
+        // a segment's start: the run's q rows (first segment of a run) and
+        // q~ = scale log2(e) Q P^K^T as hi and lo A operands in shared memory
+        // (rank groups past the rank: zero)
+        auto prepare = [&](const SegPlan &q) {
             if (q.first_of_run) {
-                // this run's q rows as the projection's A operand
                 const uint4 *qr = reinterpret_cast<const uint4 *>(
-                    p.q + ((int64_t)(row / p.G) * p.hq + g * p.G + row % p.G) * D);
+                    p.q + ((int64_t)(row / p.G) * p.hq + q.g * p.G + row % p.G) * D);
 #pragma unroll 4
                 for (int c = 0; c < DG; ++c) {
                     const uint4 v = row_ok ? __ldcg(qr + c) : make_uint4(0u, 0u, 0u, 0u);
@@ -500,21 +598,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                 }
                 tc::fence_proxy();
                 arrive(TB_QROWS);
-                m = -INFINITY;
-                l = 0.f;
-                o_written = false;
-                first_tile = true;
             }
-            // q~ = scale log2(e) Q P^K^T as hi and lo A operands (rank groups
-            // past the rank: zero)
-            wwait(TB_PROJ, kseg);
+            wwait(TB_PROJ, kproj++);
             tc::fence_after();
-            const int nk16 = (q.rk8 + 1) / 2, nv16 = (q.rv8 + 1) / 2;
             if (ok) {
 #pragma unroll 1
-                for (int c = 0; c < nk16; ++c) {
+                for (int c = 0; c < q.nk16; ++c) {
                     float v[16];
-                    tc::ld16(tl + kColQ + 16 * c, v);
+                    tc::ld16f(tl + kColQ + 16 * c, v);
                     tc::wait_ld();
 #pragma unroll
                     for (int i = 0; i < 16; ++i) v[i] = 16 * c + i < q.rk ? v[i] * p.scale_log2 : 0.f;
@@ -525,11 +616,22 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
             tc::fence_proxy();
             tc::fence_before();
             arrive(TB_QT);
-            // tiles
+        };
+        if (s_begin < s_end) prepare(seg_plan(p, s_begin));
+        for (int s = s_begin; s < s_end; ++s, ++kseg) {
+            const SegPlan q = seg_plan(p, s);
+            const int g = q.g;
+            if (q.first_of_run) {
+                m = -INFINITY;
+                l = 0.f;
+                o_written = false;
+                first_tile = true;
+            }
             const int ntok = q.t1 - q.t0;
 #pragma unroll 1
             for (int j = 0; j < q.ntiles; ++j, ++J) {
                 const int b = J & 1;
+                const uint32_t sb = tl + kColS + kTcTok * b;
                 wwait(TB_SFULL + b, J >> 1);
                 tc::fence_after();
                 float sv[kTcTok];
@@ -537,7 +639,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
 #pragma unroll
                     for (int c = 0; c < kTcTok / 16; ++c) {
                         float v[16];
-                        tc::ld16(tl + kColS + kTcTok * b + 16 * c, v);
+                        tc::ld16f(sb + 16 * c, v);
 #pragma unroll
                         for (int i = 0; i < 16; ++i) sv[16 * c + i] = v[i];
                     }
@@ -546,15 +648,20 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
 #pragma unroll
                     for (int i = 0; i < kTcTok; ++i) sv[i] = 0.f;
                 }
-                tc::fence_before();
-                arrive(TB_SFREE + b);
                 const int nvalid = min(kTcTok, ntok - kTcTok * j);
-                float mx = -INFINITY;
+                if (nvalid < kTcTok) {
 #pragma unroll
-                for (int i = 0; i < kTcTok; ++i) {
-                    sv[i] = i < nvalid ? sv[i] : -INFINITY;
-                    mx = fmaxf(mx, sv[i]);
+                    for (int i = 0; i < kTcTok; ++i) sv[i] = i < nvalid ? sv[i] : -INFINITY;
                 }
+                // the tile maximum as a tree (no serial dependency chain)
+                float t[kTcTok / 2];
+#pragma unroll
+                for (int i = 0; i < kTcTok / 2; ++i) t[i] = fmaxf(sv[2 * i], sv[2 * i + 1]);
+#pragma unroll
+                for (int w = kTcTok / 4; w >= 1; w /= 2)
+#pragma unroll
+                    for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+                const float mx = t[0];
                 // lazy rescale: the reference moves only when a score passes it
                 // by kLazyTc; V~ and O, already summed against the old one,
                 // are multiplied by 2^(m_old - m_new) in tensor memory
@@ -570,29 +677,30 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                         tc::fence_after();
                         if (ok && q.rv > 0) {
 #pragma unroll 1
-                            for (int c = 0; c < nv16; ++c) {
-                                float v[16];
-                                tc::ld16(tl + kColV + 16 * c, v);
+                            for (int c = 0; c < q.nv16; ++c) {
+                                uint32_t r[16];
+                                tc::ld16(tl + kColV + 16 * c, r);
                                 tc::wait_ld();
 #pragma unroll
-                                for (int i = 0; i < 16; ++i) v[i] *= alpha;
-                                tc::st16(tl + kColV + 16 * c, v);
+                                for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                                tc::st16(tl + kColV + 16 * c, r);
                             }
                         }
                     }
                     if (ok && o_written) {
+                        // (every back-projection of the run is done: see the
+                        // wait at each segment's end)
 #pragma unroll 1
                         for (int c = 0; c < D / 16; ++c) {
-                            float v[16];
-                            tc::ld16(tl + kColO + 16 * c, v);
+                            uint32_t r[16];
+                            tc::ld16(tl + kColO + 16 * c, r);
                             tc::wait_ld();
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) v[i] *= alpha;
-                            tc::st16(tl + kColO + 16 * c, v);
+                            for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                            tc::st16(tl + kColO + 16 * c, r);
                         }
                     }
                     tc::wait_st();
-                    tc::fence_before();
                     l *= alpha;
                     m = mn;
                 }
@@ -600,53 +708,64 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                     ref = publish_ref(p, g, row, row_ok, 0, m);
                     first_tile = false;
                 }
-                float pr[kTcTok];
-                float ls = 0.f;
+                // p = 2^(s - m) as bf16 hi | lo over the score tile's columns
+                uint32_t ph[kTcTok / 2], pl[kTcTok / 2];
 #pragma unroll
-                for (int i = 0; i < kTcTok; ++i) {
-                    pr[i] = ex2_approx(sv[i] - m);  // a masked score gives 0
-                    ls += pr[i];
+                for (int i = 0; i < kTcTok / 2; ++i) {
+                    const float p0 = ex2_approx(sv[2 * i] - m), p1 = ex2_approx(sv[2 * i + 1] - m);  // masked: 0
+                    t[i] = p0 + p1;
+                    split2(p0, p1, ph[i], pl[i]);
                 }
-                l += ls;
-                // p tile b is free once the value products of tile J - 2 are done
-                if (j >= 2) {
-                    wwait(TB_PVDONE + b, (J - 2) >> 1);
-                    tc::fence_after();
-                }
-                uint8_t *pb = p_s + b * L::kPBuf + (rg8 * (kTcTok / 8)) * 128 + r8 * 16;
 #pragma unroll
-                for (int h = 0; h < kTcTok / 16; ++h) {
-                    float x[16];
+                for (int w = kTcTok / 4; w >= 1; w /= 2)
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) x[i] = pr[16 * h + i];
-                    put16(pb + 2 * h * 128, pb + L::kPHalf + 2 * h * 128, x);
-                }
-                tc::fence_proxy();
+                    for (int i = 0; i < w; ++i) t[i] += t[i + w];
+                l += t[0];
+                tc::st16(sb, ph);
+                tc::st16(sb + 16, ph + 16);
+                tc::st16(sb + kTcTok / 2, pl);
+                tc::st16(sb + kTcTok / 2 + 16, pl + 16);
+                tc::wait_st();
+                tc::fence_before();
                 arrive(TB_PREADY + b);
             }
-            // segment end: V~ as the back-projection's hi and lo A operands
-            // (in the p tiles, free once every value product is done)
+            // the next segment's q~ (its projection went ahead), then this
+            // segment's v~ as the back-projection's hi and lo A operands, in
+            // place in tensor memory (hi at +0, lo at +64; ranks past the
+            // rank: zero)
+            if (s + 1 < s_end) prepare(seg_plan(p, s + 1));
             wwait(TB_VDONE, kseg);
             tc::fence_after();
             if (ok && q.rv > 0) {
-#pragma unroll 1
-                for (int c = 0; c < nv16; ++c) {
-                    float v[16];
-                    tc::ld16(tl + kColV + 16 * c, v);
-                    tc::wait_ld();
+                uint32_t vh[D / 2], vl[D / 2];
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) v[i] = 16 * c + i < q.rv ? v[i] : 0.f;
-                    uint8_t *hi = p_s + (rg8 * DG + 2 * c) * 128 + r8 * 16;
-                    put16(hi, hi + L::kQtHalf, v);
+                for (int c = 0; c < D / 16; ++c) {
+                    if (c < q.nv16) {
+                        float v[16];
+                        tc::ld16f(tl + kColV + 16 * c, v);
+                        tc::wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float x0 = 16 * c + 2 * i < q.rv ? v[2 * i] : 0.f;
+                            const float x1 = 16 * c + 2 * i + 1 < q.rv ? v[2 * i + 1] : 0.f;
+                            split2(x0, x1, vh[8 * c + i], vl[8 * c + i]);
+                        }
+                    }
                 }
+#pragma unroll
+                for (int c = 0; c < D / 16; ++c) {
+                    if (c < q.nv16) {
+                        tc::st8(tl + kColV + 8 * c, vh + 8 * c);
+                        tc::st8(tl + kColV + 64 + 8 * c, vl + 8 * c);
+                    }
+                }
+                tc::wait_st();
             }
-            tc::fence_proxy();
             tc::fence_before();
             arrive(TB_VSTAGED);
             wwait(TB_BPDONE, kseg);
             tc::fence_after();
             if (q.rv > 0) o_written = true;
-            ++kseg;
             if (q.last_of_run && ok) {
                 // ---- the run's result into the accumulators of KV head g
                 // (or, for a row group with an outlier maximum, as a record)
@@ -663,7 +782,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                 for (int c = 0; c < D / 16; ++c) {
                     float o[16];
                     if (o_written) {
-                        tc::ld16(tl + kColO + 16 * c, o);
+                        tc::ld16f(tl + kColO + 16 * c, o);
                         tc::wait_ld();
                     } else {
 #pragma unroll
@@ -702,7 +821,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
         }
     }
     // every MMA is done (the issuer waited for them) and every tensor-memory
-    // read has completed: release the tensor memory
+    // access has completed: release the tensor memory
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
