@@ -12,8 +12,8 @@
 //   back-projection  O  += V~ P^V     A = v~ hi, lo (tmem, K = ranks)   B = P^V      (N = d)
 //
 // q~, p and v~ are fp32 values that enter a product as two bf16 operands,
-// the value rounded to bf16 ("hi") and its residual ("lo"), so they keep ~16
-// significant bits; the factors and q are bf16 data and enter once.  Scores
+// the value truncated to bf16 ("hi") and its residual ("lo"), so they keep
+// ~15 significant bits; the factors and q are bf16 data and enter once.  Scores
 // are in log2 units: q~ carries softmax scale x log2(e).
 //
 // Work: the prefix (every entry's tokens, KV-head-major, then table order)
@@ -25,15 +25,17 @@
 // run adds its result into the plan's per-row accumulators once, at its end
 // (the shared-reference merge of milo_merge.cuh), or lists it as records.
 //
-// A block of 192 threads, one per SM (224 KB of shared memory, all 512
+// A block of 320 threads, one per SM (227 KB of shared memory, all 512
 // tensor-memory columns):
 //   warp 0, lane 0   producer: bulk copies of the segment pieces (P^K, then
 //                    C^K + C^V rows of whole 64-token tiles up to 32 KB,
 //                    then P^V) into a ring of four 32 KB slots;
 //   warp 1           owns the tensor memory and walks the MMA schedule as a
 //                    converged warp; one elected lane issues every MMA;
-//   warps 2-5        softmax: thread t owns row t of the tile and tensor
-//                    memory lane t (warp w reaches lanes 32 (w % 4) ..).
+//   warps 2-9        softmax, two warps per tensor-memory lane quarter (warp
+//                    w reaches lanes 32 (w % 4) ..): lane t of a pair owns
+//                    row t of the quarter; the pair splits every tile's
+//                    columns.
 // Tensor memory: two score tiles (each overwritten in place by its p hi, lo
 // once read), q~ as projected, v~ (converted in place to its hi, lo at a
 // segment's end), O.  The score products run two tiles ahead of the value
@@ -63,7 +65,7 @@
 namespace milo {
 namespace {
 
-constexpr int kTcThreads = 192;
+constexpr int kTcThreads = 320;   // producer warp, MMA warp, 8 softmax warps
 constexpr int kTcSlots = 4;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColS = 0;    // two score tiles of kTcTok columns (then p hi | p lo)
@@ -76,14 +78,14 @@ constexpr float kLazyTc = 8.f;   // a row's reference maximum moves when a score
 enum : int {
     TB_FULL = 0,                    // [kTcSlots] piece landed (1 + bytes)
     TB_EMPTY = TB_FULL + kTcSlots,  // [kTcSlots] MMAs reading the piece done (commit)
-    TB_QROWS = TB_EMPTY + kTcSlots, // q rows of a run staged (4 softmax warps)
+    TB_QROWS = TB_EMPTY + kTcSlots, // q rows of a run staged (8 softmax warps)
     TB_PROJ,                        // projection done (commit)
-    TB_QT,                          // q~ staged (4)
+    TB_QT,                          // q~ staged (8)
     TB_SFULL,                       // [2] score tile done (commit)
-    TB_PREADY = TB_SFULL + 2,       // [2] p tile written (4)
+    TB_PREADY = TB_SFULL + 2,       // [2] p tile written (8)
     TB_PVDONE = TB_PREADY + 2,      // [2] value products of that p tile done (commit)
     TB_VDONE = TB_PVDONE + 2,       // every value product of a segment done (commit)
-    TB_VSTAGED,                     // v~ hi, lo written for the back-projection (4)
+    TB_VSTAGED,                     // v~ hi, lo written for the back-projection (8)
     TB_BPDONE,                      // back-projection done (commit)
     TB_FIN,                         // every MMA of the block done (commit)
     TB_NBAR
@@ -95,7 +97,8 @@ struct TcLay {
     static constexpr int kQt = kQ + kTcRows * D * 2;              // q~ hi, then lo: cores [16][D/8] each
     static constexpr int kQtHalf = kTcRows * D * 2;
     static constexpr int kBar = kQt + 2 * kQtHalf;
-    static constexpr int kFlag = kBar + TB_NBAR * 8;              // abort flag, tensor-memory base
+    static constexpr int kX = kBar + TB_NBAR * 8;                 // pair exchange: maxima float [2][4 quarters][2][32],
+    static constexpr int kFlag = kX + (2 * 4 * 2 + 4) * 32 * 4;   //   then row sums [4][32]; abort flag, tensor-memory base
     static constexpr int kTotal = kFlag + 16;
     static_assert(kTotal <= 232448, "one block per SM");
 };
@@ -208,15 +211,15 @@ __device__ __forceinline__ void st16(uint32_t taddr, const uint32_t *r)
 __device__ __forceinline__ void wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 }  // namespace tc
 
-// Two fp32 values as a bf16x2 "hi" (each rounded to 8 significant bits,
-// ties away from zero, by integer arithmetic) and the bf16x2 of their
-// residuals (truncated): x = hi + lo to ~2^-17 relative.  Low half = x0.
+// Two fp32 values as a bf16x2 "hi" (each truncated to its leading 8
+// significant bits: the top half of its bits) and the bf16x2 of their
+// residuals (truncated the same way): x = hi + lo to within 2^-15 of |x|,
+// in six integer and add operations.  Low half = x0.
 __device__ __forceinline__ void split2(float x0, float x1, uint32_t &hi, uint32_t &lo)
 {
-    const uint32_t h0 = (__float_as_uint(x0) + 0x8000u) & 0xffff0000u;
-    const uint32_t h1 = (__float_as_uint(x1) + 0x8000u) & 0xffff0000u;
-    const float r0 = x0 - __uint_as_float(h0), r1 = x1 - __uint_as_float(h1);
-    hi = __byte_perm(h0, h1, 0x7632);
+    const uint32_t u0 = __float_as_uint(x0), u1 = __float_as_uint(x1);
+    const float r0 = x0 - __uint_as_float(u0 & 0xffff0000u), r1 = x1 - __uint_as_float(u1 & 0xffff0000u);
+    hi = __byte_perm(u0, u1, 0x7632);
     lo = __byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x7632);
 }
 
@@ -266,23 +269,21 @@ struct SegPlan {
     int slot;                // run record slot
 };
 
-__device__ __forceinline__ SegPlan seg_plan(const DecodeParams &p, int s)
+__device__ __forceinline__ SegPlan seg_plan(const TcSegDev &sd)
 {
-    const SegDev sd = p.tc_segs[s];
-    const EntryDev e = p.entries[sd.entry];
     SegPlan q;
-    q.ck = e.off_ck;
-    q.pk = e.off_pk;
-    q.cv = e.off_cv;
-    q.pv = e.off_pv;
-    q.n8 = (e.n + 7) & ~7;
-    q.rk = e.rk;
-    q.rv = e.rv;
-    q.rk8 = (e.rk + 7) / 8;
-    q.rv8 = (e.rv + 7) / 8;
+    q.ck = sd.ck;
+    q.pk = sd.pk;
+    q.cv = sd.cv;
+    q.pv = sd.pv;
+    q.n8 = (sd.n + 7) & ~7;
+    q.rk = sd.rk;
+    q.rv = sd.rv;
+    q.rk8 = (sd.rk + 7) / 8;
+    q.rv8 = (sd.rv + 7) / 8;
     q.nk16 = (q.rk8 + 1) / 2;
     q.nv16 = (q.rv8 + 1) / 2;
-    q.g = e.g;
+    q.g = sd.g;
     q.t0 = sd.t0;
     q.t1 = sd.t1;
     q.ntiles = (sd.t1 - sd.t0 + kTcTok - 1) / kTcTok;
@@ -294,6 +295,28 @@ __device__ __forceinline__ SegPlan seg_plan(const DecodeParams &p, int s)
     q.slot = sd.slot;
     return q;
 }
+
+// The segments of a share, each role reading them two ahead of use (a
+// segment's record is one 64-byte load whose latency the walk hides).
+struct SegWalk {
+    const TcSegDev *segs;
+    int end;
+    TcSegDev cur, next, after;  // segments s, s + 1, s + 2 once at(s) was called
+    __device__ void start(const TcSegDev *sg, int s0, int s1)
+    {
+        segs = sg;
+        end = s1;
+        if (s0 < s1) next = segs[s0];
+        if (s0 + 1 < s1) after = segs[s0 + 1];
+    }
+    // move to segment s (called for s = s_begin, s_begin + 1, ... in order)
+    __device__ void at(int s)
+    {
+        cur = next;
+        next = after;
+        if (s + 2 < end) after = segs[s + 2];
+    }
+};
 
 // Rows of C piece c of a segment: tokens [a, a + rows) of the entry, rows a
 // multiple of 8 (the piece's tiles, the last one cut at the segment end and
@@ -328,16 +351,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
             mbar_init(bar(TB_FULL + i), 1);
             mbar_init(bar(TB_EMPTY + i), 1);
         }
-        mbar_init(bar(TB_QROWS), 4);
+        mbar_init(bar(TB_QROWS), 8);
         mbar_init(bar(TB_PROJ), 1);
-        mbar_init(bar(TB_QT), 4);
+        mbar_init(bar(TB_QT), 8);
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(TB_SFULL + i), 1);
-            mbar_init(bar(TB_PREADY + i), 4);
+            mbar_init(bar(TB_PREADY + i), 8);
             mbar_init(bar(TB_PVDONE + i), 1);
         }
         mbar_init(bar(TB_VDONE), 1);
-        mbar_init(bar(TB_VSTAGED), 4);
+        mbar_init(bar(TB_VSTAGED), 8);
         mbar_init(bar(TB_BPDONE), 1);
         mbar_init(bar(TB_FIN), 1);
         *abort_flag = 0;
@@ -371,14 +394,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                 return true;
             };
             bool ok = true;
-            for (int s = s_begin; ok && s < s_end; ++s) {
-                const SegPlan q = seg_plan(p, s);
+            // order: P^K of the first segment; then per segment the next
+            // segment's P^K (its projection goes ahead), the C pieces, P^V
+            auto issue_pk = [&](const SegPlan &q) {
                 if (q.rk > 0)
                     ok = issue([&](uint32_t dst, uint32_t b) {
                         const uint32_t bytes = (uint32_t)q.rk8 * D * 16;
                         mbar_arrive_tx(b, bytes);
                         bulk_g2s(dst, p.packed + q.pk, bytes, b);
                     });
+            };
+            SegWalk w;
+            w.start(p.tc_segs, s_begin, s_end);
+            for (int s = s_begin; ok && s < s_end; ++s) {
+                w.at(s);
+                const SegPlan q = seg_plan(w.cur);
+                if (s == s_begin) issue_pk(q);
+                if (ok && s + 1 < s_end) issue_pk(seg_plan(w.next));
                 for (int c = 0; ok && c < q.nc; ++c)
                     ok = issue([&](uint32_t dst, uint32_t b) {
                         int a, rows;
@@ -482,70 +514,87 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
         };
         Piece pc[2] = {};
         int kseg = 0, J = 0;
-        if (s_begin < s_end) project(seg_plan(p, s_begin));
+        SegWalk w;
+        w.start(p.tc_segs, s_begin, s_end);
+        if (s_begin < s_end) project(seg_plan(p.tc_segs[s_begin]));
         for (int s = s_begin; ok && s < s_end; ++s, ++kseg) {
-            const SegPlan q = seg_plan(p, s);
+            w.at(s);
+            const SegPlan q = seg_plan(w.cur);
             const int J0 = J;
-            // the score product of tile j into buffer (J0 + j) & 1 (after the
-            // value product that read that buffer's last p tile, by issue
-            // order)
-            auto score = [&](int j) {
-                if (q.nc > 0 && j % q.tpp == 0) {
-                    const int c = j / q.tpp;
-                    Piece &x = pc[c & 1];
-                    x.base = take(x.slot);
-                    int a, rows;
-                    c_piece_rows(q, c, a, rows);
-                    x.cvb = x.base + (uint32_t)rows * q.rk8 * 16;
-                }
-                const int b = (J0 + j) & 1;
-                const bool go = ok && q.rk > 0;
-                const uint32_t kt = pc[(q.nc > 0 ? j / q.tpp : 0) & 1].base + (uint32_t)(j % q.tpp) * 8 * q.rk8 * 128;
-                on_one([&] {
-                    if (go) {
-                        const uint32_t id = tc::idesc(false, false, kTcTok);
-                        const uint64_t bd = tc::sdesc(kt, 128, q.rk8 * 128);
-                        tc::steps(q.nk16, [&](auto nc) {
-                            constexpr int N = decltype(nc)::value;
-                            tc::seq_ss<N>(tmem + kColS + kTcTok * b, tc::sdesc(qt_u, 128, DG * 128), bd, 16, 16, id,
-                                          false);
-                            tc::seq_ss<N>(tmem + kColS + kTcTok * b, tc::sdesc(qt_u + L::kQtHalf, 128, DG * 128), bd,
-                                          16, 16, id, true);
-                        });
-                    }
-                    tc::commit(bar(TB_SFULL + b));
-                });
-            };
-            // this segment's q~ is staged: its first two score products, then
-            // the previous segment's back-projection (before this segment's
-            // first value product overwrites v~)
+            // this segment's q~ is staged: the next segment's projection (its
+            // q rows and P^K come first)
             wait(TB_QT, kseg);
-            if (ok) score(0);
-            if (ok && q.ntiles > 1) score(1);
-            if (kseg > 0) back_project();
-            if (q.first_of_run) o_acc = false;
-            for (int j = 0; ok && j < q.ntiles; ++j) {
-                const int Jt = J0 + j, b = Jt & 1;
-                wait(TB_PREADY + b, Jt >> 1);
-                const Piece x = pc[(q.nc > 0 ? j / q.tpp : 0) & 1];
-                const bool go = ok && q.rv > 0;
-                const bool release = q.nc > 0 && (j % q.tpp == q.tpp - 1 || j == q.ntiles - 1);
-                const uint32_t vt = x.cvb + (uint32_t)(j % q.tpp) * 8 * q.rv8 * 128;
-                on_one([&] {
-                    if (go) {
-                        // v~ += p C^V: A = p hi, then lo (tensor memory), K = 64 tokens
-                        const uint32_t id = tc::idesc(false, true, 16 * q.nv16);
-                        const uint64_t bd = tc::sdesc(vt, q.rv8 * 128, 128);
-                        const uint32_t pa = tmem + kColS + kTcTok * b;
-                        tc::seq_ts<kTcTok / 16>(tmem + kColV, pa, bd, (2 * q.rv8 * 128) >> 4, id, j > 0);
-                        tc::seq_ts<kTcTok / 16>(tmem + kColV, pa + kTcTok / 2, bd, (2 * q.rv8 * 128) >> 4, id, true);
+            if (ok && s + 1 < s_end) project(seg_plan(w.next));
+            // per-segment constants of the products (descriptors without
+            // their address field; a 64-token tile of C^K and of C^V)
+            const uint32_t kstride = 8u * q.rk8 * 128, vstride = 8u * q.rv8 * 128;
+            const uint64_t bdS = tc::sdesc(0, 128, q.rk8 * 128), bdV = tc::sdesc(0, q.rv8 * 128, 128);
+            const uint64_t aS_hi = tc::sdesc(qt_u, 128, DG * 128), aS_lo = tc::sdesc(qt_u + L::kQtHalf, 128, DG * 128);
+            const uint32_t idS = tc::idesc(false, false, kTcTok), idV = tc::idesc(false, true, 16 * q.nv16);
+            const uint32_t vkstep = (2u * q.rv8 * 128) >> 4;
+            // pieces by counters: the score side opens them (tile s_in of
+            // piece s_piece), the value side releases them (v_in of v_piece)
+            int s_piece = -1, s_in = q.tpp - 1, v_piece = 0, v_in = 0;
+            // the whole tile loop for a compile-time count of 16-rank score
+            // steps (no per-tile dispatch)
+            tc::steps(q.nk16, [&](auto nkc) {
+                constexpr int NK = decltype(nkc)::value;
+                // the score product of tile j into buffer (J0 + j) & 1 (after
+                // the value product that read that buffer's last p tile, by
+                // issue order)
+                auto score = [&](int j) {
+                    if (q.nc > 0 && ++s_in == q.tpp) {
+                        s_in = 0;
+                        ++s_piece;
+                        Piece &x = pc[s_piece & 1];
+                        x.base = take(x.slot);
+                        int a, rows;
+                        c_piece_rows(q, s_piece, a, rows);
+                        x.cvb = x.base + (uint32_t)rows * q.rk8 * 16;
                     }
-                    tc::commit(bar(TB_PVDONE + b));
-                    // the last tile of a piece releases its slot
-                    if (release) tc::commit(bar(TB_EMPTY + x.slot));
-                });
-                if (ok && j + 2 < q.ntiles) score(j + 2);
-            }
+                    const int b = (J0 + j) & 1;
+                    const bool go = ok && q.rk > 0;
+                    const uint64_t bd = bdS | (uint64_t)(((pc[s_piece & 1].base + (uint32_t)s_in * kstride) >> 4) & 0x3FFF);
+                    on_one([&] {
+                        if (go) {
+                            tc::seq_ss<NK>(tmem + kColS + kTcTok * b, aS_hi, bd, 16, 16, idS, false);
+                            tc::seq_ss<NK>(tmem + kColS + kTcTok * b, aS_lo, bd, 16, 16, idS, true);
+                        }
+                        tc::commit(bar(TB_SFULL + b));
+                    });
+                };
+                // this segment's first two score products, then the previous
+                // segment's back-projection (before this segment's first value
+                // product overwrites v~)
+                if (ok) score(0);
+                if (ok && q.ntiles > 1) score(1);
+                if (kseg > 0) back_project();
+                if (q.first_of_run) o_acc = false;
+                for (int j = 0; ok && j < q.ntiles; ++j) {
+                    const int Jt = J0 + j, b = Jt & 1;
+                    wait(TB_PREADY + b, Jt >> 1);
+                    const Piece x = pc[v_piece & 1];
+                    const bool go = ok && q.rv > 0;
+                    const bool release = q.nc > 0 && (v_in == q.tpp - 1 || j == q.ntiles - 1);
+                    const uint64_t bd = bdV | (uint64_t)(((x.cvb + (uint32_t)v_in * vstride) >> 4) & 0x3FFF);
+                    on_one([&] {
+                        if (go) {
+                            // v~ += p C^V: A = p hi, then lo (tensor memory), K = 64 tokens
+                            const uint32_t pa = tmem + kColS + kTcTok * b;
+                            tc::seq_ts<kTcTok / 16>(tmem + kColV, pa, bd, vkstep, idV, j > 0);
+                            tc::seq_ts<kTcTok / 16>(tmem + kColV, pa + kTcTok / 2, bd, vkstep, idV, true);
+                        }
+                        tc::commit(bar(TB_PVDONE + b));
+                        // the last tile of a piece releases its slot
+                        if (release) tc::commit(bar(TB_EMPTY + x.slot));
+                    });
+                    if (++v_in == q.tpp) {
+                        v_in = 0;
+                        ++v_piece;
+                    }
+                    if (ok && j + 2 < q.ntiles) score(j + 2);
+                }
+            });
             J = J0 + q.ntiles;
             on_one([&] { tc::commit(bar(TB_VDONE)); });
             // this segment's back-projection waits for the next one's
@@ -553,7 +602,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
             bq = q;
             bp_k = kseg;
             if (q.rv > 0) bp_u = take(bp_slot);
-            if (s + 1 < s_end) project(seg_plan(p, s + 1));
         }
         if (ok && kseg > 0) back_project();
         on_one([&] { tc::commit(bar(TB_FIN)); });
@@ -562,48 +610,66 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
         tc::fence_after();
     } else {
         // ------------------------------------------------ softmax
-        const int quad = warp & 3;                // tensor-memory lane quarter of this warp
+        // Warps 2..9, two per tensor-memory lane quarter: the pair (half 0
+        // and 1) shares the quarter's 32 rows and splits every tile's 64
+        // columns, every rank chunk and the head dimension; a pair meets
+        // through a named barrier once per tile (the row maximum).
+        const int quad = warp & 3, half = (warp - 2) >> 2;
         const int rl = 32 * quad + lane;          // row within the tile
         const int row = tile * kTcRows + rl;      // the KV head's query row (batch x heads)
         const bool row_ok = row < p.rows_g;
         const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
         uint8_t *q_s = smem + L::kQ, *qt_s = smem + L::kQt;
+        float *xch = reinterpret_cast<float *>(smem + L::kX);  // maxima [2][4][2][32], row sums [4][32]
         const int rg8 = rl >> 3, r8 = rl & 7;     // core row group and row within the core
+        constexpr int kHalfTok = kTcTok / 2;      // columns of a tile per warp
         pdl_wait();  // q and the accumulators belong to the preceding grids until here
-        int J = 0, kseg = 0, kproj = 0;
+        int J = 0, kseg = 0, kproj = 0, bp_waited = 0;
         bool ok = true;
-        float m = -INFINITY, l = 0.f;
+        float m = -INFINITY, l = 0.f;             // l: this warp's columns only
         bool o_written = false, first_tile = true;
         uint32_t ref = 0u;
         auto arrive = [&](int b) {
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(b));
         };
+        auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory"); };
         // the warp-collective tensor-memory accesses after a wait need every
         // lane to agree on its outcome
         auto wwait = [&](int b, int parity) {
             ok = __all_sync(0xffffffffu, ok && tc_wait(bar(b), (uint32_t)parity & 1u, p.status, abort_flag));
-        };
-        // a segment's start: the run's q rows (first segment of a run) and
-        // q~ = scale log2(e) Q P^K^T as hi and lo A operands in shared memory
-        // (rank groups past the rank: zero)
-        auto prepare = [&](const SegPlan &q) {
-            if (q.first_of_run) {
-                const uint4 *qr = reinterpret_cast<const uint4 *>(
-                    p.q + ((int64_t)(row / p.G) * p.hq + q.g * p.G + row % p.G) * D);
-#pragma unroll 4
-                for (int c = 0; c < DG; ++c) {
-                    const uint4 v = row_ok ? __ldcg(qr + c) : make_uint4(0u, 0u, 0u, 0u);
-                    *reinterpret_cast<uint4 *>(q_s + (rg8 * DG + c) * 128 + r8 * 16) = v;
-                }
-                tc::fence_proxy();
-                arrive(TB_QROWS);
-            }
-            wwait(TB_PROJ, kproj++);
             tc::fence_after();
+        };
+        // back-projections done up to segment k (in phase order)
+        auto wait_bp_upto = [&](int k) {
+            while (bp_waited <= k) {
+                wwait(TB_BPDONE, bp_waited);
+                ++bp_waited;
+            }
+        };
+        // a run's q rows as the projection's A operand (this warp's half of
+        // the columns)
+        auto write_qrows = [&](const SegPlan &q) {
+            const uint4 *qr = reinterpret_cast<const uint4 *>(
+                p.q + ((int64_t)(row / p.G) * p.hq + q.g * p.G + row % p.G) * D);
+#pragma unroll 4
+            for (int c = half * (DG / 2); c < (half + 1) * (DG / 2); ++c) {
+                const uint4 v = row_ok ? __ldcg(qr + c) : make_uint4(0u, 0u, 0u, 0u);
+                *reinterpret_cast<uint4 *>(q_s + (rg8 * DG + c) * 128 + r8 * 16) = v;
+            }
+            tc::fence_proxy();
+            arrive(TB_QROWS);
+        };
+        // segment s's q~ = scale log2(e) Q P^K^T as hi and lo A operands in
+        // shared memory (rank chunks of this warp's parity; ranks past the
+        // rank: zero), then the next run's q rows if segment s + 1 starts one
+        // (its projection is issued as soon as q~ is staged)
+        auto prepare = [&](int s, const TcSegDev &sd, const TcSegDev &sd_next) {
+            const SegPlan q = seg_plan(sd);
+            wwait(TB_PROJ, kproj++);
             if (ok) {
 #pragma unroll 1
-                for (int c = 0; c < q.nk16; ++c) {
+                for (int c = half; c < q.nk16; c += 2) {
                     float v[16];
                     tc::ld16f(tl + kColQ + 16 * c, v);
                     tc::wait_ld();
@@ -616,10 +682,21 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
             tc::fence_proxy();
             tc::fence_before();
             arrive(TB_QT);
+            if (s + 1 < s_end) {
+                const SegPlan qn = seg_plan(sd_next);
+                if (qn.first_of_run) write_qrows(qn);
+            }
         };
-        if (s_begin < s_end) prepare(seg_plan(p, s_begin));
+        SegWalk w;
+        w.start(p.tc_segs, s_begin, s_end);
+        if (s_begin < s_end) {
+            const TcSegDev first = p.tc_segs[s_begin];
+            write_qrows(seg_plan(first));
+            prepare(s_begin, first, s_begin + 1 < s_end ? p.tc_segs[s_begin + 1] : first);
+        }
         for (int s = s_begin; s < s_end; ++s, ++kseg) {
-            const SegPlan q = seg_plan(p, s);
+            w.at(s);
+            const SegPlan q = seg_plan(w.cur);
             const int g = q.g;
             if (q.first_of_run) {
                 m = -INFINITY;
@@ -633,38 +710,45 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                 const int b = J & 1;
                 const uint32_t sb = tl + kColS + kTcTok * b;
                 wwait(TB_SFULL + b, J >> 1);
-                tc::fence_after();
-                float sv[kTcTok];
+                float sv[kHalfTok];
                 if (ok && q.rk > 0) {
-#pragma unroll
-                    for (int c = 0; c < kTcTok / 16; ++c) {
-                        float v[16];
-                        tc::ld16f(sb + 16 * c, v);
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) sv[16 * c + i] = v[i];
-                    }
+                    float v0[16], v1[16];
+                    tc::ld16f(sb + kHalfTok * half, v0);
+                    tc::ld16f(sb + kHalfTok * half + 16, v1);
                     tc::wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        sv[i] = v0[i];
+                        sv[16 + i] = v1[i];
+                    }
                 } else {
 #pragma unroll
-                    for (int i = 0; i < kTcTok; ++i) sv[i] = 0.f;
+                    for (int i = 0; i < kHalfTok; ++i) sv[i] = 0.f;
                 }
-                const int nvalid = min(kTcTok, ntok - kTcTok * j);
-                if (nvalid < kTcTok) {
+                const int nvalid = min(kTcTok, ntok - kTcTok * j) - kHalfTok * half;  // this warp's valid columns
+                if (nvalid < kHalfTok) {
 #pragma unroll
-                    for (int i = 0; i < kTcTok; ++i) sv[i] = i < nvalid ? sv[i] : -INFINITY;
+                    for (int i = 0; i < kHalfTok; ++i) sv[i] = i < nvalid ? sv[i] : -INFINITY;
                 }
-                // the tile maximum as a tree (no serial dependency chain)
-                float t[kTcTok / 2];
+                // the row maximum of the tile: a tree over this warp's columns,
+                // then the pair's two halves through shared memory (both
+                // warps have read their scores before either overwrites the
+                // tile with p)
+                float t[kHalfTok / 2];
 #pragma unroll
-                for (int i = 0; i < kTcTok / 2; ++i) t[i] = fmaxf(sv[2 * i], sv[2 * i + 1]);
+                for (int i = 0; i < kHalfTok / 2; ++i) t[i] = fmaxf(sv[2 * i], sv[2 * i + 1]);
 #pragma unroll
-                for (int w = kTcTok / 4; w >= 1; w /= 2)
+                for (int w = kHalfTok / 4; w >= 1; w /= 2)
 #pragma unroll
                     for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
-                const float mx = t[0];
+                float *xb = xch + ((J & 1) * 4 + quad) * 64;
+                xb[half * 32 + lane] = t[0];
+                pair_sync();
+                const float mx = fmaxf(t[0], xb[(1 - half) * 32 + lane]);
                 // lazy rescale: the reference moves only when a score passes it
                 // by kLazyTc; V~ and O, already summed against the old one,
-                // are multiplied by 2^(m_old - m_new) in tensor memory
+                // are multiplied by 2^(m_old - m_new) in tensor memory (the
+                // pair splits the rank and head-dimension chunks)
                 const bool need = mx > m + kLazyTc;
                 if (__any_sync(0xffffffffu, need)) {
                     const float mn = need ? mx : m;
@@ -674,10 +758,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                         // product) must be done
                         const int Jp = J - 1;
                         wwait(TB_PVDONE + (Jp & 1), Jp >> 1);
-                        tc::fence_after();
                         if (ok && q.rv > 0) {
 #pragma unroll 1
-                            for (int c = 0; c < q.nv16; ++c) {
+                            for (int c = half; c < q.nv16; c += 2) {
                                 uint32_t r[16];
                                 tc::ld16(tl + kColV + 16 * c, r);
                                 tc::wait_ld();
@@ -687,17 +770,18 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                             }
                         }
                     }
-                    if (ok && o_written) {
-                        // (every back-projection of the run is done: see the
-                        // wait at each segment's end)
+                    if (o_written) {
+                        wait_bp_upto(kseg - 1);  // every back-projection of the run is done
+                        if (ok) {
 #pragma unroll 1
-                        for (int c = 0; c < D / 16; ++c) {
-                            uint32_t r[16];
-                            tc::ld16(tl + kColO + 16 * c, r);
-                            tc::wait_ld();
+                            for (int c = half; c < D / 16; c += 2) {
+                                uint32_t r[16];
+                                tc::ld16(tl + kColO + 16 * c, r);
+                                tc::wait_ld();
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-                            tc::st16(tl + kColO + 16 * c, r);
+                                for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                                tc::st16(tl + kColO + 16 * c, r);
+                            }
                         }
                     }
                     tc::wait_st();
@@ -708,23 +792,22 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                     ref = publish_ref(p, g, row, row_ok, 0, m);
                     first_tile = false;
                 }
-                // p = 2^(s - m) as bf16 hi | lo over the score tile's columns
-                uint32_t ph[kTcTok / 2], pl[kTcTok / 2];
+                // p = 2^(s - m) of this warp's columns as bf16 hi | lo over the
+                // score tile (hi in columns [0, 32), lo in [32, 64))
+                uint32_t ph[kHalfTok / 2], pl[kHalfTok / 2];
 #pragma unroll
-                for (int i = 0; i < kTcTok / 2; ++i) {
+                for (int i = 0; i < kHalfTok / 2; ++i) {
                     const float p0 = ex2_approx(sv[2 * i] - m), p1 = ex2_approx(sv[2 * i + 1] - m);  // masked: 0
                     t[i] = p0 + p1;
                     split2(p0, p1, ph[i], pl[i]);
                 }
 #pragma unroll
-                for (int w = kTcTok / 4; w >= 1; w /= 2)
+                for (int w = kHalfTok / 4; w >= 1; w /= 2)
 #pragma unroll
                     for (int i = 0; i < w; ++i) t[i] += t[i + w];
                 l += t[0];
-                tc::st16(sb, ph);
-                tc::st16(sb + 16, ph + 16);
-                tc::st16(sb + kTcTok / 2, pl);
-                tc::st16(sb + kTcTok / 2 + 16, pl + 16);
+                tc::st16(sb + (kHalfTok / 2) * half, ph);
+                tc::st16(sb + kTcTok / 2 + (kHalfTok / 2) * half, pl);
                 tc::wait_st();
                 tc::fence_before();
                 arrive(TB_PREADY + b);
@@ -732,15 +815,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
             // the next segment's q~ (its projection went ahead), then this
             // segment's v~ as the back-projection's hi and lo A operands, in
             // place in tensor memory (hi at +0, lo at +64; ranks past the
-            // rank: zero)
-            if (s + 1 < s_end) prepare(seg_plan(p, s + 1));
+            // rank: zero): both warps of the pair read their chunks before
+            // either writes
+            if (s + 1 < s_end) prepare(s + 1, w.next, w.after);
             wwait(TB_VDONE, kseg);
-            tc::fence_after();
-            if (ok && q.rv > 0) {
-                uint32_t vh[D / 2], vl[D / 2];
+            if (q.rv > 0) {
+                // (the pair barrier runs in both warps whatever ok says)
+                uint32_t vh[D / 4], vl[D / 4];
 #pragma unroll
-                for (int c = 0; c < D / 16; ++c) {
-                    if (c < q.nv16) {
+                for (int k = 0; k < D / 32; ++k) {
+                    const int c = 2 * k + half;
+                    if (ok && c < q.nv16) {
                         float v[16];
                         tc::ld16f(tl + kColV + 16 * c, v);
                         tc::wait_ld();
@@ -748,27 +833,36 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                         for (int i = 0; i < 8; ++i) {
                             const float x0 = 16 * c + 2 * i < q.rv ? v[2 * i] : 0.f;
                             const float x1 = 16 * c + 2 * i + 1 < q.rv ? v[2 * i + 1] : 0.f;
-                            split2(x0, x1, vh[8 * c + i], vl[8 * c + i]);
+                            split2(x0, x1, vh[8 * k + i], vl[8 * k + i]);
                         }
                     }
                 }
+                pair_sync();
 #pragma unroll
-                for (int c = 0; c < D / 16; ++c) {
-                    if (c < q.nv16) {
-                        tc::st8(tl + kColV + 8 * c, vh + 8 * c);
-                        tc::st8(tl + kColV + 64 + 8 * c, vl + 8 * c);
+                for (int k = 0; k < D / 32; ++k) {
+                    const int c = 2 * k + half;
+                    if (ok && c < q.nv16) {
+                        tc::st8(tl + kColV + 8 * c, vh + 8 * k);
+                        tc::st8(tl + kColV + 64 + 8 * c, vl + 8 * k);
                     }
                 }
                 tc::wait_st();
             }
             tc::fence_before();
+            // the previous segment's back-projection is done before this
+            // one's can be (the phase order of its barrier)
+            wait_bp_upto(kseg - 1);
             arrive(TB_VSTAGED);
-            wwait(TB_BPDONE, kseg);
-            tc::fence_after();
             if (q.rv > 0) o_written = true;
-            if (q.last_of_run && ok) {
+            if (q.last_of_run) {
+                wait_bp_upto(kseg);
                 // ---- the run's result into the accumulators of KV head g
-                // (or, for a row group with an outlier maximum, as a record)
+                // (or, for a row group with an outlier maximum, as a record);
+                // the pair adds its row sums, each warp its half of O
+                float *xl = xch + 2 * 4 * 2 * 32 + quad * 32;
+                if (half == 1) xl[lane] = l;
+                pair_sync();
+                const float lsum = half == 0 ? l + xl[lane] : 0.f;  // used by half 0
                 const float Mref = ref ? ref_dec(ref) : m;
                 const bool outlier = row_ok && m - Mref > kDirectMax;
                 const uint32_t votes = __ballot_sync(0xffffffffu, outlier);
@@ -778,43 +872,45 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                 float *rec = p.rec + rec_idx * (8 * D + kRecFloatsExtra);
                 const float f = row_ok && direct ? ex2_approx(m - Mref) : 0.f;
                 float *arow = p.acc_o + ((int64_t)g * p.rows_max + row) * D;
+                if (ok) {
 #pragma unroll 1
-                for (int c = 0; c < D / 16; ++c) {
-                    float o[16];
-                    if (o_written) {
-                        tc::ld16f(tl + kColO + 16 * c, o);
-                        tc::wait_ld();
-                    } else {
+                    for (int c = half; c < D / 16; c += 2) {
+                        float o[16];
+                        if (o_written) {
+                            tc::ld16f(tl + kColO + 16 * c, o);
+                            tc::wait_ld();
+                        } else {
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) o[i] = 0.f;
-                    }
-                    if (!row_ok) continue;
-                    if (direct) {
+                            for (int i = 0; i < 16; ++i) o[i] = 0.f;
+                        }
+                        if (!row_ok) continue;
+                        if (direct) {
 #pragma unroll
-                        for (int i = 0; i < 16; i += 4)
-                            atomicAdd(reinterpret_cast<float4 *>(arow + 16 * c + i),
-                                      make_float4(f * o[i], f * o[i + 1], f * o[i + 2], f * o[i + 3]));
-                    } else {
+                            for (int i = 0; i < 16; i += 4)
+                                atomicAdd(reinterpret_cast<float4 *>(arow + 16 * c + i),
+                                          make_float4(f * o[i], f * o[i + 1], f * o[i + 2], f * o[i + 3]));
+                        } else {
 #pragma unroll
-                        for (int i = 0; i < 16; i += 4)
-                            __stcg(reinterpret_cast<float4 *>(rec + r8 * D + 16 * c + i),
-                                   make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+                            for (int i = 0; i < 16; i += 4)
+                                __stcg(reinterpret_cast<float4 *>(rec + r8 * D + 16 * c + i),
+                                       make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+                        }
                     }
-                }
-                if (row_ok) {
-                    if (direct) {
-                        atomicAdd(p.acc_l + (int64_t)g * p.rows_max + row, f * l);
-                    } else {
-                        __stcg(rec + 8 * D + r8, m);
-                        __stcg(rec + 8 * D + 8 + r8, l);
+                    if (row_ok && half == 0) {
+                        if (direct) {
+                            atomicAdd(p.acc_l + (int64_t)g * p.rows_max + row, f * lsum);
+                        } else {
+                            __stcg(rec + 8 * D + r8, m);
+                            __stcg(rec + 8 * D + 8 + r8, lsum);
+                        }
                     }
-                }
-                // one lane per row group lists an outlier record
-                if (!direct && r8 == 0 && row_ok) {
-                    const int gr = g * p.nrg + rgg;
-                    const uint32_t k = atomicAdd(p.ovf_cnt + gr, 1u);
-                    __stcg(reinterpret_cast<int4 *>(p.ovf_list) + (int64_t)gr * p.list_cap + k,
-                           make_int4((int)rec_idx, 8 * rgg, min(8, p.rows_g - 8 * rgg), 0));
+                    // one lane per row group lists an outlier record
+                    if (!direct && half == 0 && r8 == 0 && row_ok) {
+                        const int gr = g * p.nrg + rgg;
+                        const uint32_t k = atomicAdd(p.ovf_cnt + gr, 1u);
+                        __stcg(reinterpret_cast<int4 *>(p.ovf_list) + (int64_t)gr * p.list_cap + k,
+                               make_int4((int)rec_idx, 8 * rgg, min(8, p.rows_g - 8 * rgg), 0));
+                    }
                 }
                 tc::fence_before();
             }

@@ -318,7 +318,7 @@ struct milo_prefix {
         int cta0;
     };
     std::vector<TcPart> tc_parts;
-    SegDev *tc_segs = nullptr;
+    TcSegDev *tc_segs = nullptr;
     int32_t *tc_cta = nullptr;
     int sms = 0;
     int tc_max_shares = 0;            // shares worth at least kTcMinShareCost each
@@ -510,7 +510,7 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     // call with ntile row tiles of kTcRows rows per KV head uses
     p->sms = sms;
     p->tc = G <= 8 && !chunks.empty() && (int64_t)max_batch * G >= kTcMinRows;
-    std::vector<SegDev> tc_sd;
+    std::vector<TcSegDev> tc_sd;
     std::vector<int32_t> tc_cb;
     if (p->tc) {
         // no share below about one 512-token entry of rank 64 (fewer blocks
@@ -544,7 +544,11 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
             tp.cta0 = (int)tc_cb.size();
             tp.num_slots = nslot;
             tp.max_runs = *std::max_element(runs.begin(), runs.end());
-            for (const Seg &x : ts) tc_sd.push_back(SegDev{x.entry, x.t0, x.t1, x.slot, x.flags, {0, 0, 0}});
+            for (const Seg &x : ts) {
+                const EntryDev &en = ents[(size_t)x.entry];
+                tc_sd.push_back(TcSegDev{en.off_ck, en.off_pk, en.off_cv, en.off_pv, x.t0, x.t1, en.n, en.rk, en.rv,
+                                         en.g, x.slot, x.flags});
+            }
             tc_cb.insert(tc_cb.end(), cb.begin(), cb.end());
             p->tc_parts.push_back(tp);
         }
@@ -578,11 +582,11 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
         return cleanup(e, "cudaMalloc offsets");
     if (p->tc) {
-        if ((e = cudaMalloc(&p->tc_segs, sizeof(SegDev) * tc_sd.size())) != cudaSuccess)
+        if ((e = cudaMalloc(&p->tc_segs, sizeof(TcSegDev) * tc_sd.size())) != cudaSuccess)
             return cleanup(e, "cudaMalloc tensor-core segments");
         if ((e = cudaMalloc(&p->tc_cta, sizeof(int32_t) * tc_cb.size())) != cudaSuccess)
             return cleanup(e, "cudaMalloc tensor-core shares");
-        if ((e = cudaMemcpyAsync(p->tc_segs, tc_sd.data(), sizeof(SegDev) * tc_sd.size(), cudaMemcpyHostToDevice,
+        if ((e = cudaMemcpyAsync(p->tc_segs, tc_sd.data(), sizeof(TcSegDev) * tc_sd.size(), cudaMemcpyHostToDevice,
                                  stream)) != cudaSuccess)
             return cleanup(e, "copy tensor-core segments");
         if ((e = cudaMemcpyAsync(p->tc_cta, tc_cb.data(), sizeof(int32_t) * tc_cb.size(), cudaMemcpyHostToDevice,

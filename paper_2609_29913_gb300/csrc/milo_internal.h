@@ -73,6 +73,16 @@ constexpr int kTcTok = 64;
 constexpr int kTcSlot = 32768;
 constexpr int kTcMinRows = 32;
 
+// A segment of the tensor-core decode's partition, with what it needs of its
+// entry (one 64-byte load, no dependent loads).
+struct TcSegDev {
+    int64_t ck, pk, cv, pv;     // packed byte offsets of the entry's factors
+    int32_t t0, t1;             // tokens [t0, t1) of the entry
+    int32_t n, rk, rv, g;       // entry tokens, ranks, KV head
+    int32_t slot, flags;        // run record slot, kSegFirstOfRun / kSegLastOfRun
+};
+static_assert(sizeof(TcSegDev) == 64, "tensor-core segment size");
+
 // Device-side counters owned by a plan (zero between calls).
 struct CountersDev {
     uint32_t tail_next;   // dynamic tail work counter
@@ -117,7 +127,7 @@ struct DecodeParams {
     uint32_t *ovf_cnt;              // [Hkv][nrg]: records listed per (KV head, row group)
     int32_t *ovf_list;              // int4 [Hkv][nrg][list_cap]: listed records (workspace)
     int list_cap;                   // list entries per (KV head, row group)
-    const SegDev *tc_segs;          // tensor-core path: segments of this call's partition
+    const TcSegDev *tc_segs;        // tensor-core path: segments of this call's partition
     const int32_t *tc_cta_begin;    //   [tc_nshare + 1] first segment of each share
     int tc_ntile;                   //   tiles of kTcRows query rows per KV head
     int tc_nshare;                  //   shares (thread blocks per row tile)
