@@ -1,0 +1,58 @@
+"""Run decode calls on the first layers of a named workload, for profilers.
+
+  python -m paper_2609_29913_gb300.profile_layer --workload qwen7b-1L-1M-b8 \
+      [--layers 1] [--calls 3]
+
+Builds the plans of layers 0 .. layers-1 of the workload (seeded synthetic
+inputs, as the benchmark draws them), then makes `calls` rounds of one
+decode call per layer on the current stream, synchronises and checks every
+plan's device status word.  Each call launches the kernels milo_call_info
+names, so a profiler can select them by name and count (e.g. ncu -k
+regex:batch_tc -s 1 -c 1 skips the first round's launch).  It keeps the
+device footprint to the chosen layers, well under the full workload's.
+"""
+from __future__ import annotations
+
+import argparse
+import sys
+
+import numpy as np
+
+
+def main(argv=None) -> int:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--workload", required=True)
+    ap.add_argument("--layers", type=int, default=1)
+    ap.add_argument("--calls", type=int, default=3)
+    args = ap.parse_args(argv)
+
+    import torch
+    from . import build, milo, workloads
+
+    build.build()
+    cfg = workloads.by_name(args.workload)
+    plans, layers = [], []
+    for l in range(min(args.layers, cfg.layers)):
+        layer = workloads.make_config_layer(cfg, l, device="cuda")
+        plans.append(milo.Prefix.from_layer(layer))
+        layers.append(layer)
+    toffs = [torch.as_tensor(L.tail_offsets, device="cuda") for L in layers]
+    max_tail = max(int(np.diff(L.tail_offsets).max()) for L in layers)
+    for _ in range(args.calls):
+        for L, pre, toff in zip(layers, plans, toffs):
+            pre.decode(L.q, L.tail_k, L.tail_v, toff, max_tail)
+    torch.cuda.synchronize()
+    for pre in plans:
+        if pre.status() != 0:
+            print("device status word set", file=sys.stderr)
+            return 1
+    info = milo.milo_call_info(plans[0].plan, cfg.batch, max_tail)
+    print(f"{cfg.name}: {len(plans)} layer(s) x {args.calls} call(s), path {milo.PATH_NAMES[info['path']]}, "
+          f"{info['kernels']} kernels per call, {info['blocks']} blocks in the prefix grid")
+    for pre in plans:
+        pre.close()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
