@@ -427,6 +427,10 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
         "gpu_launches": call["kernels"] * L * steps,
         "clocks": clocks.summary(), "parity_check": check, "setup_s": t_gen,
     }
+    rec["roofline"]["traffic"] = traffic_record(cfg.name)
+    rec["roofline"]["traffic_of"] = (
+        "DRAM bytes per launch of the tensor-core prefix grid (the prefix only), from profiles/traffic.json"
+        if call["path"] == 1 else "DRAM bytes per launch of chunk_kernel, from profiles/traffic.json")
     if e2e:
         rec["e2e"] = measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, max_tail,
                                  steps, dist, dev, world, tokens)
@@ -550,7 +554,6 @@ def main():
             others.append(measure(other, W, milo, dev, args.steps, args.warmup, dist, rank, world,
                                   check=not args.no_check))
     roof = dict(head["roofline"])
-    roof["traffic"] = traffic_record(cfg.name)
     roof["kernel"] = ", ".join(head["kernels"])
     roof["per_launch_bytes"] = head["config"]["algorithmic_bytes_per_step"] // cfg.layers
     roof["per_launch_us"] = head["ms_per_step"] * 1e3 / cfg.layers
