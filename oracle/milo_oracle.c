@@ -13,6 +13,12 @@
  *                             of every stored block (Eq. 3 with Sigma folded
  *                             into C), followed by exact softmax attention
  *                             (Eq. 1) over [blocks..., query's own tail].
+ *   - mo_attention_dense_rope: the same, for factors of pre-RoPE keys (the
+ *                             observation of Sec. 3: keys are compressed
+ *                             before the rotary position embedding), so every
+ *                             reconstructed prefix key is rotated to its
+ *                             position before the scores.
+ *   - mo_rope_rotate:         that rotation of a set of rows.
  *   - mo_attention_rankspace: the same attention written in rank space,
  *                             q.K^_b^T = (q P_b^T) C_b^T and
  *                             p V^_b   = (p C_b) P_b.  A second, independent
@@ -32,7 +38,11 @@
  * the allocation maximises Eq. 6 (Alg. 1 prints argmin); the softmax scale is
  * 1/sqrt(head_dim); query head h reads KV head h / (Hq / Hkv); a query attends
  * to every stored block in table order and then to all of its own tail
- * tokens, with no mask.
+ * tokens, with no mask.  RoPE (where asked for): dimension i pairs with
+ * i + d/2 (the half-split form of the Qwen2.5 models), pair i turns by the
+ * angle pos * theta^(-2i/d) counter-clockwise, block b's token t sits at
+ * position block_pos[b] + t (by default the block's start in the
+ * concatenated prefix), and q and the dense tails arrive already rotated.
  *
  * Parity status: every function here is pinned by CPU tests (brute force,
  * closed forms, invariants, numpy.linalg.svd, exhaustive search).
@@ -105,6 +115,8 @@ typedef struct {
     const void *arena, *q, *tk, *tv;
     const int64_t *toff;
     double scale;
+    double rope_theta;        /* > 0: prefix keys are pre-RoPE (rotate them) */
+    const int64_t *block_pos; /* [nblk] first position of each block, or NULL */
 } mo_problem;
 
 static int check_problem(const mo_problem *p, int64_t *n_prefix, int64_t *t_max)
@@ -132,6 +144,12 @@ static int check_problem(const mo_problem *p, int64_t *n_prefix, int64_t *t_max)
         if (t > tm) tm = t;
     }
     if (tm > 0 && (!p->tk || !p->tv)) return MO_ERR_ARG;
+    if (p->rope_theta > 0.0) {
+        if (p->d % 2 != 0) return MO_ERR_ARG;
+        if (p->block_pos)
+            for (int b = 0; b < p->nblk; ++b)
+                if (p->block_pos[b] < 0) return MO_ERR_ARG;
+    }
     *n_prefix = np;
     *t_max = tm;
     return MO_OK;
@@ -155,6 +173,28 @@ static void reconstruct(const double *C, const double *P, int n, int r, int d,
             double a = C[(int64_t)t * r + j];
             const double *pr = P + (int64_t)j * d;
             for (int c = 0; c < d; ++c) o[c] += a * pr[c];
+        }
+    }
+}
+
+/* Rotary position embedding of n rows of width d (row t at position
+ * pos0 + t, or pos[t] when pos is given): pair (i, i + d/2) turns by the
+ * angle position * theta^(-2i/d),
+ *   x_i       <- x_i cos a - x_{i+d/2} sin a
+ *   x_{i+d/2} <- x_{i+d/2} cos a + x_i sin a. */
+static void rope_rows(double *X, int n, int d, int64_t pos0, const int64_t *pos,
+                      double theta)
+{
+    const int h = d / 2;
+    for (int t = 0; t < n; ++t) {
+        const double where = (double)(pos ? pos[t] : pos0 + t);
+        double *x = X + (int64_t)t * d;
+        for (int i = 0; i < h; ++i) {
+            const double a = where * pow(theta, -2.0 * i / d);
+            const double c = cos(a), s = sin(a);
+            const double x0 = x[i], x1 = x[i + h];
+            x[i] = x0 * c - x1 * s;
+            x[i + h] = x1 * c + x0 * s;
         }
     }
 }
@@ -224,6 +264,9 @@ static int attention_dense(const mo_problem *p, double *out, double *weights,
             fetch(p->dtype, p->arena, p->ock[e], (int64_t)n * r, C);
             fetch(p->dtype, p->arena, p->opk[e], (int64_t)r * d, P);
             reconstruct(C, P, n, r, d, K);
+            if (p->rope_theta > 0.0)
+                rope_rows(K, n, d, p->block_pos ? p->block_pos[b] : pos[b], NULL,
+                          p->rope_theta);
             for (int row = 0; row < rows; ++row)
                 for (int t = 0; t < n; ++t)
                     S[(int64_t)row * ncol + pos[b] + t] =
@@ -437,6 +480,38 @@ int mo_attention_dense(int dtype, int batch, int num_q_heads, int num_kv_heads,
                     off_cv, off_pv, arena, q, tail_k, tail_v, tail_offsets,
                     scale > 0.0 ? scale : 1.0 / sqrt((double)head_dim)};
     return attention_dense(&p, out, weights, wstride);
+}
+
+/* Pre-RoPE factors: as mo_attention_dense, with every reconstructed prefix
+ * key rotated (rope_theta > 0; head_dim even) to its position block_pos[b]
+ * + t (block_pos NULL: the block's start in the concatenated prefix). */
+int mo_attention_dense_rope(int dtype, int batch, int num_q_heads, int num_kv_heads,
+                            int head_dim, int num_blocks, const int32_t *block_len,
+                            const int32_t *rank_k, const int32_t *rank_v,
+                            const int64_t *off_ck, const int64_t *off_pk,
+                            const int64_t *off_cv, const int64_t *off_pv,
+                            const void *arena, const void *q, const void *tail_k,
+                            const void *tail_v, const int64_t *tail_offsets,
+                            double scale, double rope_theta, const int64_t *block_pos,
+                            double *out, double *weights, int64_t wstride)
+{
+    if (!(rope_theta > 0.0)) return MO_ERR_ARG;
+    mo_problem p = {dtype, batch, num_q_heads, num_kv_heads, head_dim,
+                    num_blocks, block_len, rank_k, rank_v, off_ck, off_pk,
+                    off_cv, off_pv, arena, q, tail_k, tail_v, tail_offsets,
+                    scale > 0.0 ? scale : 1.0 / sqrt((double)head_dim),
+                    rope_theta, block_pos};
+    return attention_dense(&p, out, weights, wstride);
+}
+
+/* The rotation alone, in place, on n fp64 rows of width d: row t at
+ * position pos[t]. */
+int mo_rope_rotate(int n, int d, double *X, const int64_t *pos, double theta)
+{
+    if (n < 0 || d <= 0 || d % 2 != 0 || !(theta > 0.0) || (n > 0 && (!X || !pos)))
+        return MO_ERR_ARG;
+    rope_rows(X, n, d, 0, pos, theta);
+    return MO_OK;
 }
 
 int mo_attention_rankspace(int dtype, int batch, int num_q_heads,

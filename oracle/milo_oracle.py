@@ -11,6 +11,9 @@ may be ``float64`` or ``uint16`` holding bf16 bit patterns (widened exactly).
 Functions and the passage of the paper each follows:
   attention(..., form="dense")      Alg. 1 Stage 2 reconstruction + Eq. 1
   attention(..., form="rankspace")  the same attention in rank space (Eq. 1 + Eq. 3)
+  attention(..., rope_theta=...)    pre-RoPE factors (Sec. 3): reconstructed prefix
+                                    keys rotated to their positions, then Eq. 1
+  rope_rotate(X, pos, theta)        that rotation of the rows of X
   svd(X)                            Eq. 3, one-sided Jacobi SVD of one block
   spectral_information(sigma, r)    Eq. 5
   allocate_ranks(...)               Eq. 6 solved by the greedy rule of Eq. 7
@@ -58,6 +61,10 @@ def lib():
         i32, i64, dbl = ctypes.c_int, ctypes.c_int64, ctypes.c_double
         L.mo_attention_dense.argtypes = [i32] * 6 + [P] * 7 + [P] * 4 + [P, dbl, P, P, i64]
         L.mo_attention_dense.restype = i32
+        L.mo_attention_dense_rope.argtypes = [i32] * 6 + [P] * 7 + [P] * 4 + [P, dbl, dbl, P, P, P, i64]
+        L.mo_attention_dense_rope.restype = i32
+        L.mo_rope_rotate.argtypes = [i32, i32, P, P, dbl]
+        L.mo_rope_rotate.restype = i32
         L.mo_attention_rankspace.argtypes = [i32] * 6 + [P] * 7 + [P] * 4 + [P, dbl, P]
         L.mo_attention_rankspace.restype = i32
         L.mo_svd_jacobi.argtypes = [i32, i32, P, P, P, P, P]
@@ -103,9 +110,17 @@ def max_threads() -> int:
 
 def attention(*, num_kv_heads, head_dim, block_len, rank_k, rank_v, off_ck,
               off_pk, off_cv, off_pv, arena, q, tail_k=None, tail_v=None,
-              tail_offsets=None, scale=None, form="dense", weights=False):
+              tail_offsets=None, scale=None, form="dense", weights=False,
+              rope_theta=None, block_pos=None):
     """Exact decode attention of queries ``q`` [batch, Hq, d] over a low-rank
     block prefix followed by each query's dense tail.
+
+    With ``rope_theta`` the factors are those of pre-RoPE keys: every
+    reconstructed prefix key is rotated to its position (block b's token t at
+    ``block_pos[b] + t``; by default the block's start in the concatenated
+    prefix) before the scores; q and the tails are taken as already rotated.
+    Only the dense form does this (rank space cannot hold a per-position
+    rotation).
 
     Returns fp64 ``out`` [batch, Hq, d] (and, with ``weights=True`` and the
     dense form, the normalised softmax weights [batch, Hq, N_prefix + T_max],
@@ -139,6 +154,17 @@ def attention(*, num_kv_heads, head_dim, block_len, rank_k, rank_v, off_ck,
             _ptr(rv), _ptr(ock), _ptr(opk), _ptr(ocv), _ptr(opv), _ptr(arena),
             _ptr(q), _ptr(tk), _ptr(tv), _ptr(toff), sc, _ptr(out))
     L = lib()
+    if rope_theta is not None:
+        if form != "dense":
+            raise ValueError("pre-RoPE factors need the dense form")
+        bpos = None if block_pos is None else i64(block_pos)
+        if bpos is not None and bpos.shape != (nblk,):
+            raise ValueError("block_pos must hold one position per block")
+        wstride = int(blen.sum()) + tmax
+        w = np.zeros((batch, hq, wstride), dtype=np.float64) if weights else None
+        _check(L.mo_attention_dense_rope(*args[:-1], float(rope_theta), _ptr(bpos), args[-1],
+                                         _ptr(w), wstride), "attention")
+        return (out, w) if weights else out
     if form == "dense":
         wstride = int(blen.sum()) + tmax
         w = np.zeros((batch, hq, wstride), dtype=np.float64) if weights else None
@@ -150,6 +176,23 @@ def attention(*, num_kv_heads, head_dim, block_len, rank_k, rank_v, off_ck,
         _check(L.mo_attention_rankspace(*args), "attention")
         return out
     raise ValueError(form)
+
+
+def rope_rotate(X, pos, theta: float) -> np.ndarray:
+    """Rows of X ([n, d] or [..., n, d], fp64) rotated by the rotary position
+    embedding, row t to position pos[t] (the rotation the pre-RoPE attention
+    applies to reconstructed keys)."""
+    X = np.array(X, dtype=np.float64, copy=True)
+    d = X.shape[-1]
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    flat = np.ascontiguousarray(X.reshape(-1, d))
+    n_rows = flat.shape[0]
+    if pos.size == X.shape[-2] and flat.shape[0] != pos.size:
+        pos = np.broadcast_to(pos, X.shape[:-1]).reshape(-1).copy()
+    if pos.size != n_rows:
+        raise ValueError("one position per row")
+    _check(lib().mo_rope_rotate(n_rows, d, _ptr(flat), _ptr(pos), float(theta)), "rope_rotate")
+    return flat.reshape(X.shape)
 
 
 def svd(X: np.ndarray):
