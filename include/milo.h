@@ -203,7 +203,8 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan,
 /*
  * Workspace a decode call needs (device memory the caller provides): the
  * split-softmax partial results (running max, sum and output per partition
- * of the tokens, Eq. 1 split over token ranges).  `bytes` receives the size.
+ * of the tokens, Eq. 1 split over token ranges).  `bytes` receives the size,
+ * enough for milo_attn_decode and milo_attn_decode_reconstruct alike.
  */
 milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
                                   int64_t max_tail_tokens, size_t *bytes);
@@ -261,11 +262,14 @@ int32_t milo_tensor_min_rows(void);
  *   out          device fp32 [batch, num_q_heads, head_dim].
  *   workspace    device, at least milo_workspace_size bytes, 16-byte aligned.
  * Asynchronous on `stream`: no host synchronisation and no allocation, so the
- * call can be captured in a CUDA graph.  A call is two kernels launched with
- * programmatic dependent launch: the first may begin streaming the plan's
- * factors before the preceding kernel on `stream` finishes, and reads q, the
- * tails and the workspace only after it has; the second combines and writes
- * `out`.  A plan must not be used by two calls that can run concurrently (it
+ * call can be captured in a CUDA graph.  A call is two or three kernels
+ * (milo_call_info) launched with programmatic dependent launch: the prefix
+ * grid may begin streaming the plan's factors before the preceding kernel on
+ * `stream` finishes, and reads q, the tails and the workspace only after it
+ * has; the last combines and writes `out`.  A plan holding pre-RoPE factors
+ * (milo_prefix_set_rope) is refused with MILO_ERR_UNSUPPORTED: rank-space
+ * scoring cannot apply a per-position rotation.  A plan must not be used by
+ * two calls that can run concurrently (it
  * holds per-call counters and accumulators).  A query whose prefix and tail
  * are both empty yields NaN.  A call with more than 2^31 - 1 work items
  * (prefix chunks x row groups plus tail items) returns MILO_ERR_UNSUPPORTED
@@ -304,6 +308,55 @@ milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q,
                                       int64_t tail_rows, int64_t max_tail_tokens,
                                       float softmax_scale, float *out,
                                       void *stream);
+
+/*
+ * The same decode call by reconstruct-then-attend, the paper's own inference
+ * path (Alg. 1 Stage 2 with the fused reconstruction of Sec. 3.5): every
+ * prefix token's key and value are rebuilt densely, K^ = C^K P^K and
+ * V^ = C^V P^V, in fp16 tiles in shared memory (the paper's fp16 KV buffer)
+ * and attended by flash decoding, instead of being scored in rank space.  It
+ * is the comparison for the rank-space path and the path for pre-RoPE
+ * factors.
+ *   Arguments, layouts, ownership, workspace and errors are those of
+ *   milo_attn_decode, and a plan's per-call state is shared between the two
+ *   (calls on one plan must not overlap).  It needs a prefix and at most 8
+ *   query heads per KV head (else MILO_ERR_UNSUPPORTED).  q, the
+ *   reconstructed keys and values must lie inside the fp16 range (|x| < 65504).
+ *   Three kernels at most: the tails' chunk grid (when there are tails), the
+ *   reconstructing prefix grid (one block of 4 warps per chunk of up to 256
+ *   tokens of one entry and group of up to 64 query rows), the finish grid.
+ */
+milo_status_t milo_attn_decode_reconstruct(const milo_prefix_t *plan, const void *q,
+                                           int32_t batch, const void *tail_k,
+                                           const void *tail_v,
+                                           const int64_t *tail_offsets,
+                                           int64_t tail_rows, int64_t max_tail_tokens,
+                                           float softmax_scale, float *out,
+                                           void *workspace, size_t workspace_bytes,
+                                           void *stream);
+
+/*
+ * Declare the plan's factors to be those of pre-RoPE keys (Sec. 3: keys are
+ * compressed before the rotary position embedding).  milo_attn_decode_reconstruct
+ * then rotates every reconstructed prefix key to its position before scoring:
+ * dimension i pairs with i + head_dim/2, and pair i turns counter-clockwise by
+ * position * rope_theta^(-2i/head_dim); block b's token t sits at position
+ * block_pos[b] + t.  q and the dense tails are taken as already rotated (as a
+ * KV cache stores them); values are not rotated.
+ *   rope_theta  > 0: the rotary base (e.g. 1e6 for the Qwen2.5 models);
+ *               0 clears the setting (the factors are the keys as scored).
+ *   block_pos   host int64 [num_blocks], each in [0, 2^40], read during the
+ *               call only; NULL places the blocks at their starts in the
+ *               concatenated prefix (0, n_0, n_0 + n_1, ...).  A retrieval
+ *               subset of blocks passes their original positions.
+ * Builds the rotation tables on the plan's device: allocates, synchronises
+ * the device and copies, so it must not be called during stream capture or
+ * while a call on the plan may be running.  Errors: MILO_ERR_INVALID_ARG
+ * (null plan, rope_theta negative or not finite, a position out of range,
+ * another device current), MILO_ERR_UNSUPPORTED (no prefix), MILO_ERR_CUDA.
+ */
+milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta,
+                                   const int64_t *block_pos);
 
 /*
  * Read (and optionally clear) the plan's sticky device status word, which the

@@ -779,8 +779,9 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
                               : (two ? launch_chunk_grid<128, 2>(cfg, p, mk, mv)
                                      : launch_chunk_grid<128, 1>(cfg, p, mk, mv));
     if (e != cudaSuccess) return e;
-    // the tensor-core path launches its prefix grid between the two
-    if (p.tc_ntile > 0) return cudaSuccess;
+    // the tensor-core and reconstruct-then-attend calls launch their prefix
+    // grid between the two
+    if (p.tc_ntile > 0 || p.rc_chunks) return cudaSuccess;
     return launch_finish(p, stream);
 }
 

@@ -322,6 +322,12 @@ struct milo_prefix {
     int32_t *tc_cta = nullptr;
     int sms = 0;
     int tc_max_shares = 0;            // shares worth at least kTcMinShareCost each
+    // reconstruct-then-attend: chunks of at most kRcChunkTiles tiles of one entry
+    int4 *rc_chunks = nullptr;
+    int rc_num_chunks = 0, rc_max_head_chunks = 0;
+    // pre-RoPE factors (milo_prefix_set_rope): rotation tables, or null
+    float2 *rope_tile = nullptr, *rope_off = nullptr;
+    int32_t *rope_tile_base = nullptr;
     int tc_shares(int64_t ntile) const
     {
         return (int)std::max<int64_t>(1, std::min<int64_t>(sms / std::max<int64_t>(1, ntile), tc_max_shares));
@@ -436,6 +442,10 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaFree(plan->status);
     cudaFree(plan->tc_segs);
     cudaFree(plan->tc_cta);
+    cudaFree(plan->rc_chunks);
+    cudaFree(plan->rope_tile);
+    cudaFree(plan->rope_off);
+    cudaFree(plan->rope_tile_base);
     cudaSetDevice(cur);
     delete plan;
     return MILO_OK;
@@ -502,6 +512,20 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     p->num_chunks = (int)chunks.size();
     for (int g = 0; g < H; ++g)
         p->max_head_chunks = std::max(p->max_head_chunks, g_chunk[(size_t)g + 1] - g_chunk[(size_t)g]);
+    // reconstruct-then-attend chunks, in entry order
+    std::vector<int4> rc;
+    {
+        std::vector<int> per_head((size_t)H, 0);
+        for (int64_t x = 0; x < E; ++x) {
+            const int tiles = (table->block_len[x / H] + kRcTok - 1) / kRcTok;
+            for (int t0 = 0; t0 < tiles; t0 += kRcChunkTiles) {
+                rc.push_back(make_int4((int)x, t0, std::min(kRcChunkTiles, tiles - t0), 0));
+                ++per_head[(size_t)(x % H)];
+            }
+        }
+        p->rc_num_chunks = (int)rc.size();
+        for (int g = 0; g < H; ++g) p->rc_max_head_chunks = std::max(p->rc_max_head_chunks, per_head[(size_t)g]);
+    }
     std::vector<SegDev> sd(segs.size());
     for (size_t i = 0; i < segs.size(); ++i) {
         sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
@@ -577,6 +601,13 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     if (!chunks.empty() && (e = cudaMemcpyAsync(p->chunks, chunks.data(), sizeof(ChunkDev) * chunks.size(),
                                                 cudaMemcpyHostToDevice, stream)) != cudaSuccess)
         return cleanup(e, "copy chunks");
+    if (!rc.empty()) {
+        if ((e = cudaMalloc(&p->rc_chunks, sizeof(int4) * rc.size())) != cudaSuccess)
+            return cleanup(e, "cudaMalloc reconstruction chunks");
+        if ((e = cudaMemcpyAsync(p->rc_chunks, rc.data(), sizeof(int4) * rc.size(), cudaMemcpyHostToDevice,
+                                 stream)) != cudaSuccess)
+            return cleanup(e, "copy reconstruction chunks");
+    }
     if ((e = cudaMalloc(&p->counters, cnt_bytes)) != cudaSuccess) return cleanup(e, "cudaMalloc counters");
     if ((e = cudaMalloc(&p->status, sizeof(int32_t))) != cudaSuccess) return cleanup(e, "cudaMalloc status");
     if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
@@ -648,6 +679,9 @@ struct CallShape {
     const milo_prefix::TcPart *part;
     int64_t records;
     int64_t list_cap, list_bytes;
+    // reconstruct-then-attend calls (the same accumulators and finish grid):
+    // one record per chunk and row group, then the tail items'
+    int64_t records_rc, list_cap_rc, list_bytes_rc;
 };
 
 CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
@@ -686,6 +720,10 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     const int64_t prefix_items = c.part ? (int64_t)c.part->max_runs : (int64_t)p->max_head_chunks;
     c.list_cap = c.chunked ? prefix_items + queries_per_group * c.S : 0;
     c.list_bytes = 16 * (int64_t)p->hkv * c.nrg * c.list_cap;
+    const int64_t tail_records = (int64_t)batch * p->hkv * c.S * c.nrg_t;
+    c.records_rc = (int64_t)p->rc_num_chunks * c.nrg + tail_records;
+    c.list_cap_rc = c.chunked ? (int64_t)p->rc_max_head_chunks + queries_per_group * c.S : 0;
+    c.list_bytes_rc = 16 * (int64_t)p->hkv * c.nrg * c.list_cap_rc;
 
     return c;
 }
@@ -697,17 +735,24 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch, int6
     if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
     if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
-    *bytes = (size_t)std::max<int64_t>(c.records, 1) * (8 * plan->d + kRecFloatsExtra) * sizeof(float) +
-             (size_t)c.list_bytes;
+    const size_t rec_bytes = (8 * plan->d + kRecFloatsExtra) * sizeof(float);
+    // enough for milo_attn_decode and milo_attn_decode_reconstruct alike
+    const size_t a = (size_t)std::max<int64_t>(c.records, 1) * rec_bytes + (size_t)c.list_bytes;
+    const size_t b = (size_t)std::max<int64_t>(c.records_rc, 1) * rec_bytes + (size_t)c.list_bytes_rc;
+    *bytes = std::max(a, b);
     return MILO_OK;
 }
 
-milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t batch, const void *tail_k,
-                               const void *tail_v, const int64_t *tail_offsets, int64_t tail_rows,
-                               int64_t max_tail_tokens, float softmax_scale, float *out, void *workspace,
-                               size_t workspace_bytes, void *stream_)
+namespace {
+// One decode call: the rank-space paths, or (recon) reconstruct-then-attend.
+milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batch, const void *tail_k,
+                          const void *tail_v, const int64_t *tail_offsets, int64_t tail_rows, int64_t max_tail_tokens,
+                          float softmax_scale, float *out, void *workspace, size_t workspace_bytes, void *stream_,
+                          bool recon)
 {
     if (!plan || !q || !out) return fail(MILO_ERR_INVALID_ARG, "null plan, q or out");
+    if (!recon && plan->rope_tile)
+        return fail(MILO_ERR_UNSUPPORTED, "the plan holds pre-RoPE factors: use milo_attn_decode_reconstruct");
     if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
     if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
     if (plan->nb == 0 && max_tail_tokens == 0) return fail(MILO_ERR_INVALID_ARG, "no prefix and no tail");
@@ -729,6 +774,11 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
 
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
+    if (recon && (!c.chunked || plan->rc_num_chunks == 0))
+        return fail(MILO_ERR_UNSUPPORTED, "reconstruct-then-attend needs a prefix and at most 8 query heads per KV head");
+    if (recon && ((int64_t)plan->rc_num_chunks * c.nrg > 0x7fffffff || c.list_cap_rc > 0x7fffffff ||
+                  (int64_t)plan->rc_num_chunks * ((c.rows_g + kRcRows - 1) / kRcRows) > 0x7fffffff))
+        return fail(MILO_ERR_UNSUPPORTED, "call too large: more than 2^31 - 1 work items");
     // the kernels count thread blocks, tail items and list entries in int
     const int64_t tail_items = (int64_t)batch * plan->hkv * c.S;
     // (the persistent path counts record slots per row group and its merge
@@ -820,6 +870,29 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
         if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS) return fail(MILO_ERR_CUDA, "tensor map encoding failed");
     }
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    if (recon) {
+        // the dense tails on the chunk grid, then the reconstructing prefix
+        // grid, then the finish grid (each chained by programmatic dependent
+        // launch); records: the chunks' first, then the tail items'
+        prm.num_chunks = 0;
+        prm.tc_ntile = 0;
+        prm.rc_chunks = plan->rc_chunks;
+        prm.rope_tile = plan->rope_tile;
+        prm.rope_off = plan->rope_off;
+        prm.rope_tile_base = plan->rope_tile_base;
+        prm.tail_rec_base = (int64_t)plan->rc_num_chunks * c.nrg;
+        prm.list_cap = (int)c.list_cap_rc;
+        prm.ovf_list = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(workspace) +
+                                                   (size_t)std::max<int64_t>(c.records_rc, 1) *
+                                                       (8 * plan->d + kRecFloatsExtra) * sizeof(float));
+        cudaError_t e = cudaSuccess;
+        if (prm.num_tail_items > 0 && (e = launch_chunks(prm, &mk, &mv, stream)) != cudaSuccess)
+            return cuda_fail(e, "tail grid launch");
+        if ((e = launch_recon(prm, plan->rc_num_chunks, stream)) != cudaSuccess)
+            return cuda_fail(e, "reconstruction grid launch");
+        if ((e = launch_finish(prm, stream)) != cudaSuccess) return cuda_fail(e, "finish grid launch");
+        return MILO_OK;
+    }
     if (c.path == MILO_PATH_TENSOR) {
         // the dense tails on the chunk grid, then the prefix on the tensor
         // cores, then the finish grid (each chained by programmatic
@@ -834,6 +907,100 @@ milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t
     const int smem = decode_smem_bytes(plan->d, c.nrg_cta);
     cudaError_t e = launch_decode(prm, &mk, &mv, smem, plan->num_ctas, stream);
     if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    return MILO_OK;
+}
+}  // namespace
+
+milo_status_t milo_attn_decode(const milo_prefix_t *plan, const void *q, int32_t batch, const void *tail_k,
+                               const void *tail_v, const int64_t *tail_offsets, int64_t tail_rows,
+                               int64_t max_tail_tokens, float softmax_scale, float *out, void *workspace,
+                               size_t workspace_bytes, void *stream)
+{
+    return decode_call(plan, q, batch, tail_k, tail_v, tail_offsets, tail_rows, max_tail_tokens, softmax_scale, out,
+                       workspace, workspace_bytes, stream, false);
+}
+
+milo_status_t milo_attn_decode_reconstruct(const milo_prefix_t *plan, const void *q, int32_t batch,
+                                           const void *tail_k, const void *tail_v, const int64_t *tail_offsets,
+                                           int64_t tail_rows, int64_t max_tail_tokens, float softmax_scale,
+                                           float *out, void *workspace, size_t workspace_bytes, void *stream)
+{
+    return decode_call(plan, q, batch, tail_k, tail_v, tail_offsets, tail_rows, max_tail_tokens, softmax_scale, out,
+                       workspace, workspace_bytes, stream, true);
+}
+
+milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta, const int64_t *block_pos)
+{
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    if (!(rope_theta >= 0.0) || std::isinf(rope_theta)) return fail(MILO_ERR_INVALID_ARG, "rope_theta must be finite and >= 0");
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
+    cudaError_t e = cudaDeviceSynchronize();  // no call may be reading the old tables
+    if (e != cudaSuccess) return cuda_fail(e, "synchronize before the rotation tables change");
+    cudaFree(plan->rope_tile);
+    cudaFree(plan->rope_off);
+    cudaFree(plan->rope_tile_base);
+    plan->rope_tile = plan->rope_off = nullptr;
+    plan->rope_tile_base = nullptr;
+    if (rope_theta == 0.0) return MILO_OK;
+    const int d = plan->d, h = d / 2, nb = plan->nb;
+    if (!plan->rc_chunks) return fail(MILO_ERR_UNSUPPORTED, "no prefix to rotate");
+    // block positions (default: the blocks' starts in the concatenated prefix)
+    std::vector<int32_t> len((size_t)nb);
+    std::vector<int32_t> base((size_t)nb + 1, 0);
+    {
+        std::vector<EntryDev> ents((size_t)nb * plan->hkv);
+        if ((e = cudaMemcpy(ents.data(), plan->entries, sizeof(EntryDev) * ents.size(), cudaMemcpyDeviceToHost)) !=
+            cudaSuccess)
+            return cuda_fail(e, "read the plan's entries");
+        for (int b = 0; b < nb; ++b) len[(size_t)b] = ents[(size_t)b * plan->hkv].n;
+    }
+    std::vector<int64_t> pos((size_t)nb);
+    int64_t cum = 0;
+    for (int b = 0; b < nb; ++b) {
+        pos[(size_t)b] = block_pos ? block_pos[b] : cum;
+        if (pos[(size_t)b] < 0 || pos[(size_t)b] > ((int64_t)1 << 40))
+            return fail(MILO_ERR_INVALID_ARG, "block position outside [0, 2^40]");
+        cum += len[(size_t)b];
+        base[(size_t)b + 1] = base[(size_t)b] + (len[(size_t)b] + kRcTok - 1) / kRcTok;
+    }
+    // frequency of pair i, and the (cos, sin) tables, in fp64 then rounded
+    std::vector<double> th((size_t)h);
+    for (int i = 0; i < h; ++i) th[(size_t)i] = std::pow(rope_theta, -2.0 * i / d);
+    std::vector<float2> off((size_t)kRcTok * h), tile((size_t)base[(size_t)nb] * h);
+    for (int u = 0; u < kRcTok; ++u)
+        for (int i = 0; i < h; ++i) {
+            const double a = u * th[(size_t)i];
+            off[(size_t)u * h + i] = make_float2((float)std::cos(a), (float)std::sin(a));
+        }
+    for (int b = 0; b < nb; ++b)
+        for (int k = 0; k < base[(size_t)b + 1] - base[(size_t)b]; ++k)
+            for (int i = 0; i < h; ++i) {
+                const double a = (double)(pos[(size_t)b] + (int64_t)k * kRcTok) * th[(size_t)i];
+                tile[((size_t)base[(size_t)b] + k) * h + i] = make_float2((float)std::cos(a), (float)std::sin(a));
+            }
+    auto undo = [&](cudaError_t err, const char *what) {
+        cudaFree(plan->rope_tile);
+        cudaFree(plan->rope_off);
+        cudaFree(plan->rope_tile_base);
+        plan->rope_tile = plan->rope_off = nullptr;
+        plan->rope_tile_base = nullptr;
+        return cuda_fail(err, what);
+    };
+    if ((e = cudaMalloc(&plan->rope_tile, sizeof(float2) * std::max<size_t>(tile.size(), 1))) != cudaSuccess)
+        return undo(e, "cudaMalloc rotation table");
+    if ((e = cudaMalloc(&plan->rope_off, sizeof(float2) * off.size())) != cudaSuccess)
+        return undo(e, "cudaMalloc rotation table");
+    if ((e = cudaMalloc(&plan->rope_tile_base, sizeof(int32_t) * base.size())) != cudaSuccess)
+        return undo(e, "cudaMalloc rotation table");
+    if ((e = cudaMemcpy(plan->rope_tile, tile.data(), sizeof(float2) * tile.size(), cudaMemcpyHostToDevice)) !=
+            cudaSuccess ||
+        (e = cudaMemcpy(plan->rope_off, off.data(), sizeof(float2) * off.size(), cudaMemcpyHostToDevice)) !=
+            cudaSuccess ||
+        (e = cudaMemcpy(plan->rope_tile_base, base.data(), sizeof(int32_t) * base.size(), cudaMemcpyHostToDevice)) !=
+            cudaSuccess)
+        return undo(e, "copy rotation tables");
     return MILO_OK;
 }
 

@@ -83,6 +83,13 @@ struct TcSegDev {
 };
 static_assert(sizeof(TcSegDev) == 64, "tensor-core segment size");
 
+// Reconstruct-then-attend (milo_recon.cu): tokens per reconstructed tile,
+// query rows per thread block, and tiles per chunk (a chunk is a thread
+// block's token range of one entry: int4 {entry, first tile, tiles, 0}).
+constexpr int kRcTok = 64;
+constexpr int kRcRows = 64;
+constexpr int kRcChunkTiles = 4;
+
 // Device-side counters owned by a plan (zero between calls).
 struct CountersDev {
     uint32_t tail_next;   // dynamic tail work counter
@@ -131,6 +138,10 @@ struct DecodeParams {
     const int32_t *tc_cta_begin;    //   [tc_nshare + 1] first segment of each share
     int tc_ntile;                   //   tiles of kTcRows query rows per KV head
     int tc_nshare;                  //   shares (thread blocks per row tile)
+    const int4 *rc_chunks;          // reconstruct-then-attend: the prefix chunks (or null)
+    const float2 *rope_tile;        //   pre-RoPE factors: (cos, sin) of each tile start's angle, [tile][d/2]
+    const float2 *rope_off;         //   (cos, sin) of u theta_i for u < kRcTok, [u][d/2]
+    const int32_t *rope_tile_base;  //   first tile of each block in rope_tile
 };
 
 // Kernel attributes (shared-memory size, carveout) belong to a device: the
@@ -170,6 +181,10 @@ cudaError_t launch_batch_tc(const DecodeParams &p, cudaStream_t stream);
 int batch_tc_smem_bytes(int head_dim);
 // The finish grid alone (one warp per KV head and row group).
 cudaError_t launch_finish(const DecodeParams &p, cudaStream_t stream);
+// The reconstruct-then-attend prefix grid (a thread block per chunk and group
+// of kRcRows query rows); like the tensor-core grid it sits between the tail
+// items' chunk grid and the finish grid.
+cudaError_t launch_recon(const DecodeParams &p, int num_chunks, cudaStream_t stream);
 
 // Fixed scratch of milo_attn_decode_static (a file-scope device array).
 constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;

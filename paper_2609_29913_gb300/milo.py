@@ -31,7 +31,8 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
            "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
            "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
-           "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows"]
+           "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows",
+           "milo_attn_decode_reconstruct", "milo_prefix_set_rope"]
 
 PATH_NAMES = {0: "chunks", 1: "tensor", 2: "persistent"}
 
@@ -92,13 +93,17 @@ def lib():
         L.milo_attn_decode.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P,
                                        ctypes.c_size_t, P]
         L.milo_attn_decode_static.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P]
+        L.milo_attn_decode_reconstruct.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P,
+                                                   ctypes.c_size_t, P]
+        L.milo_prefix_set_rope.argtypes = [P, ctypes.c_double, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         L.milo_call_info.argtypes = [P, i32, i64, P]
         L.milo_tensor_min_rows.restype = i32
         for name in ("milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
                      "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
-                     "milo_get_device_status", "milo_call_info"):
+                     "milo_get_device_status", "milo_call_info", "milo_attn_decode_reconstruct",
+                     "milo_prefix_set_rope"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -255,6 +260,27 @@ def milo_attn_decode_static(plan: int, q_ptr: int, batch: int, tail_k_ptr: int, 
                                          out_ptr, _stream_ptr(stream)), "milo_attn_decode_static")
 
 
+def milo_attn_decode_reconstruct(plan: int, q_ptr: int, batch: int, tail_k_ptr: int, tail_v_ptr: int,
+                                 tail_offsets_ptr: int, tail_rows: int, max_tail_tokens: int,
+                                 softmax_scale: float, out_ptr: int, workspace_ptr: int,
+                                 workspace_bytes: int, stream=None) -> None:
+    """The same call by reconstruct-then-attend (the paper's own path)."""
+    _check(lib().milo_attn_decode_reconstruct(plan, q_ptr, int(batch), tail_k_ptr or None, tail_v_ptr or None,
+                                              tail_offsets_ptr or None, int(tail_rows), int(max_tail_tokens),
+                                              float(softmax_scale), out_ptr, workspace_ptr,
+                                              int(workspace_bytes), _stream_ptr(stream)),
+           "milo_attn_decode_reconstruct")
+
+
+def milo_prefix_set_rope(plan: int, rope_theta: float, block_pos=None) -> None:
+    """Declare the plan's factors pre-RoPE (rope_theta > 0) or not (0);
+    block_pos: one int64 position per block, or None for the concatenated
+    prefix."""
+    pos = None if block_pos is None else _arr(block_pos, np.int64)
+    _check(lib().milo_prefix_set_rope(plan, float(rope_theta), None if pos is None else pos.ctypes.data),
+           "milo_prefix_set_rope")
+
+
 def milo_get_device_status(plan: int, stream=None, clear: bool = False) -> int:
     code = ctypes.c_int32(0)
     _check(lib().milo_get_device_status(plan, _stream_ptr(stream), int(bool(clear)),
@@ -285,8 +311,19 @@ class Prefix:
     def workspace_size(self, batch: int, max_tail_tokens: int) -> int:
         return milo_workspace_size(self.plan, batch, max_tail_tokens)
 
+    def set_rope(self, rope_theta: float, block_pos=None) -> None:
+        """The factors are those of pre-RoPE keys (see milo_prefix_set_rope);
+        decode_reconstruct then rotates the reconstructed keys."""
+        milo_prefix_set_rope(self.plan, rope_theta, block_pos)
+
+    def decode_reconstruct(self, q, tail_k=None, tail_v=None, tail_offsets=None, max_tail_tokens=0,
+                           softmax_scale: float = 0.0, out=None, workspace=None, stream=None):
+        """``decode`` by reconstruct-then-attend (milo_attn_decode_reconstruct)."""
+        return self.decode(q, tail_k, tail_v, tail_offsets, max_tail_tokens, softmax_scale, out, workspace,
+                           stream, _call=milo_attn_decode_reconstruct)
+
     def decode(self, q, tail_k=None, tail_v=None, tail_offsets=None, max_tail_tokens=0,
-               softmax_scale: float = 0.0, out=None, workspace=None, stream=None):
+               softmax_scale: float = 0.0, out=None, workspace=None, stream=None, _call=None):
         """q: bf16 [batch, Hq, d] cuda tensor; tails bf16 [rows, Hkv, d];
         tail_offsets int64 cuda tensor [batch + 1].  Returns fp32 out."""
         import torch
@@ -301,13 +338,13 @@ class Prefix:
             workspace = torch.empty(need, device=q.device, dtype=torch.uint8)
             made.append(workspace)
         tail_rows = int(tail_k.shape[0]) if (tail_k is not None and max_tail_tokens > 0) else 0
-        milo_attn_decode(self.plan, q.data_ptr(), batch,
-                         tail_k.data_ptr() if tail_rows else 0,
-                         tail_v.data_ptr() if tail_rows else 0,
-                         tail_offsets.data_ptr() if tail_rows else 0,
-                         tail_rows, max_tail_tokens if tail_rows else 0, softmax_scale,
-                         out.data_ptr(), workspace.data_ptr(), workspace.numel() * workspace.element_size(),
-                         stream)
+        (_call or milo_attn_decode)(self.plan, q.data_ptr(), batch,
+                                    tail_k.data_ptr() if tail_rows else 0,
+                                    tail_v.data_ptr() if tail_rows else 0,
+                                    tail_offsets.data_ptr() if tail_rows else 0,
+                                    tail_rows, max_tail_tokens if tail_rows else 0, softmax_scale,
+                                    out.data_ptr(), workspace.data_ptr(),
+                                    workspace.numel() * workspace.element_size(), stream)
         if isinstance(stream, torch.cuda.Stream):
             # the call runs on `stream`: keep the caching allocator from
             # handing these buffers out again before it has finished
