@@ -45,6 +45,11 @@ FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
 L2_BYTES = 129 * 2 ** 20
 PARITY_ATOL, PARITY_RTOL_L2 = 1e-2, 2e-3
+# workloads on which the reconstruct-then-attend path and its pre-RoPE
+# variant are timed beside the rank-space path; the rotary base of the
+# Qwen2.5 models
+RECON_WORKLOADS = ("qwen7b-28L-32k-b1", "qwen7b-28L-32k-b64")
+ROPE_THETA = 1e6
 
 
 def parse(argv=None):
@@ -58,6 +63,8 @@ def parse(argv=None):
     ap.add_argument("--no-check", action="store_true", help="skip the parity checks")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU baseline sample time")
+    ap.add_argument("--no-recon", action="store_true",
+                    help="skip timing the reconstruct-then-attend path beside the rank-space path")
     return ap.parse_args(argv)
 
 
@@ -281,11 +288,13 @@ def pack_tensors(tensors, dev):
     return buf, views
 
 
-def parity_layer0(layer, out0):
-    """Layer 0's whole output [batch, Hq, d] against the oracle."""
-    from oracle import milo_oracle
-    milo_oracle.build()
-    ref = milo_oracle.attention(**layer.to_numpy_bits())
+def parity_layer0(layer, out0, ref=None):
+    """Layer 0's whole output [batch, Hq, d] against the oracle (ref: the
+    oracle's output, when already computed)."""
+    if ref is None:
+        from oracle import milo_oracle
+        milo_oracle.build()
+        ref = milo_oracle.attention(**layer.to_numpy_bits())
     got = out0.double().cpu().numpy()
     d = got.shape[-1]
     g2, r2 = got.reshape(-1, d), ref.reshape(-1, d)
@@ -306,8 +315,42 @@ def kernel_names(path: int, has_tail: bool) -> list:
     return ["decode_kernel", "combine_kernel"]
 
 
+def time_graph(step, stream, steps, warmup, flush):
+    """Capture step(stream) in a CUDA graph, replay it `warmup` times, then
+    time `steps` replays with CUDA events on `stream` (replay by replay after
+    writing `flush`, when given).  Returns the total ms."""
+    import torch
+    with torch.cuda.stream(stream):
+        step(stream)
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step(stream)
+    for _ in range(max(warmup, 3)):
+        graph.replay()
+    torch.cuda.synchronize()
+    if flush is None:
+        start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        with torch.cuda.stream(stream):
+            for _ in range(steps):
+                graph.replay()
+        stop.record(stream)
+        torch.cuda.synchronize()
+        return start.elapsed_time(stop), graph
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    with torch.cuda.stream(stream):
+        for a, b in evs:
+            flush.fill_(1.0)
+            a.record(stream)
+            graph.replay()
+            b.record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs), graph
+
+
 def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, check=True,
-            e2e=False, cpu_seconds=0.0):
+            e2e=False, cpu_seconds=0.0, recon=False):
     """Time one workload (all its layers per step) and return its record."""
     import torch
     plans, qs, tks, tvs, toffs = [], [], [], [], []
@@ -366,10 +409,12 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
     for p in plans:
         assert p.status() == 0, "device status word set during warm-up"
 
-    check = parity_layer0(check_layer, outs[0]) if check_layer is not None else None
+    ref0 = None
     if check_layer is not None:
-        check_layer.arena = None
-    check_layer = None
+        from oracle import milo_oracle
+        milo_oracle.build()
+        ref0 = milo_oracle.attention(**check_layer.to_numpy_bits())
+    check = parity_layer0(check_layer, outs[0], ref0) if check_layer is not None else None
 
     # ---- timed region: K graph replays.  Inputs larger than L2 need no
     # flush; a workload that fits in L2 is timed replay by replay with a
@@ -427,6 +472,13 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
         "gpu_launches": call["kernels"] * L * steps,
         "clocks": clocks.summary(), "parity_check": check, "setup_s": t_gen,
     }
+    if recon:
+        rec["reconstruct_then_attend"] = measure_recon(cfg, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream,
+                                                      steps, warmup, flush, dist, dev, world, tokens, ms_step,
+                                                      check_layer, ref0)
+    if check_layer is not None:
+        check_layer.arena = None
+    check_layer = None
     rec["roofline"]["traffic"] = traffic_record(cfg.name)
     rec["roofline"]["traffic_of"] = (
         "DRAM bytes per launch of the tensor-core prefix grid (the prefix only), from profiles/traffic.json"
@@ -441,6 +493,57 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
     del plans, graph, ws, in_buf, out_buf
     torch.cuda.empty_cache()
     return rec
+
+
+def measure_recon(cfg, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup, flush, dist, dev,
+                  world, tokens, ms_rank_space, check_layer, ref0):
+    """The same step by reconstruct-then-attend (the paper's own path: dense
+    keys and values rebuilt from the factors, then attended), on the same
+    plans and inputs; then the pre-RoPE variant (every reconstructed prefix
+    key rotated to its position, rotary base ROPE_THETA).  Each is timed like
+    the rank-space step and checked on layer 0 against the oracle."""
+    L = len(plans)
+    kernels = (1 if max_tail > 0 else 0) + 2
+
+    def step(s):
+        for l in range(L):
+            plans[l].decode_reconstruct(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws,
+                                        stream=s)
+
+    def one(label):
+        ms_total, _ = time_graph(step, stream, steps, warmup, flush)
+        for p in plans:
+            assert p.status() == 0, f"device status word set during the {label} timing"
+        ms = max_over_ranks(ms_total / steps, dist, dev)
+        return {"ms_per_step": ms, "value": replica_throughput(world, tokens, ms), "unit": UNIT,
+                "gpu_launches": kernels * L * steps,
+                "kernels": (["chunk_kernel (dense-tail items)"] if max_tail > 0 else []) +
+                           ["recon_kernel", "finish_kernel"]}
+
+    out = one("reconstruct")
+    out["rank_space_ms_per_step"] = ms_rank_space
+    out["rank_space_speedup"] = out["ms_per_step"] / ms_rank_space
+    out["how"] = ("the same graph of per-layer calls through milo_attn_decode_reconstruct: per tile of 64 "
+                  "tokens, K^ = C^K P^K and V^ = C^V P^V rebuilt in fp16 in shared memory, then flash "
+                  "decoding; rank_space_speedup = this ms / the rank-space ms on the same inputs")
+    if check_layer is not None:
+        out["parity_check"] = parity_layer0(check_layer, outs[0], ref0)
+    for p in plans:
+        p.set_rope(ROPE_THETA)
+    try:
+        rope = one("pre-RoPE")
+        rope["rope_theta"] = ROPE_THETA
+        rope["how"] = ("reconstruct-then-attend over pre-RoPE factors: every reconstructed prefix key turns "
+                       "to its position (the blocks' starts in the concatenated prefix) before scoring")
+        if check_layer is not None:
+            from oracle import milo_oracle
+            ref_rope = milo_oracle.attention(**check_layer.to_numpy_bits(), rope_theta=ROPE_THETA)
+            rope["parity_check"] = parity_layer0(check_layer, outs[0], ref_rope)
+        out["pre_rope"] = rope
+    finally:
+        for p in plans:
+            p.set_rope(0.0)
+    return out
 
 
 def measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, max_tail, steps, dist, dev,
@@ -545,14 +648,16 @@ def main():
 
     dev = torch.device("cuda", local)
     head = measure(cfg, W, milo, dev, args.steps, args.warmup, dist, rank, world, check=not args.no_check,
-                   e2e=True, cpu_seconds=0.0 if args.no_cpu else args.cpu_seconds)
+                   e2e=True, cpu_seconds=0.0 if args.no_cpu else args.cpu_seconds,
+                   recon=not args.no_recon and cfg.name in RECON_WORKLOADS)
     others = []
     if not args.only:
         for k, other in enumerate(W.CONFIGS):
             if k == args.config:
                 continue
             others.append(measure(other, W, milo, dev, args.steps, args.warmup, dist, rank, world,
-                                  check=not args.no_check))
+                                  check=not args.no_check,
+                                  recon=not args.no_recon and other.name in RECON_WORKLOADS))
     roof = dict(head["roofline"])
     roof["kernel"] = ", ".join(head["kernels"])
     roof["per_launch_bytes"] = head["config"]["algorithmic_bytes_per_step"] // cfg.layers
@@ -569,6 +674,7 @@ def main():
         "cpu_baseline": head.get("cpu_baseline"),
         "e2e": head["e2e"], "gpu_launches": head["gpu_launches"], "clocks": head["clocks"],
         "parity_check": head["parity_check"], "path": head["path"], "setup_s": head["setup_s"],
+        "reconstruct_then_attend": head.get("reconstruct_then_attend"),
         "workloads": [{k: v for k, v in o.items() if k not in ("unit",)} for o in others],
     }
     if rank == 0:
