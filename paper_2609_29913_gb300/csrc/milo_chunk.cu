@@ -24,9 +24,9 @@
 //                merged; each warp produces a share of the head dimension.
 //
 // A dense-tail item (one query's tail split for one KV head, kTailTokens
-// tokens) brings its K and V rows with 3-D TMA boxes (8 head dimensions x
-// kTailTokens rows each, landing as cores [column group][token group]) and
-// runs the C steps on them with q~ = scale * log2(e) * q, a share of the
+// tokens) brings its K and V rows with 3-D TMA boxes (64 head dimensions x
+// kTailTokens rows each, 128-byte rows with the 128-byte swizzle: few, wide
+// requests) and runs the C steps on them with q~ = scale * log2(e) * q, a share of the
 // tokens per warp; its values are already o.  Every item then adds its result
 // into fp32 accumulators of its KV head's rows (see add_part) and exits; a
 // small finish grid chained by programmatic dependent launch (one warp per KV
@@ -298,7 +298,9 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
     for (int n = 0; n < NT; ++n) vacc[n][0] = vacc[n][1] = vacc[n][2] = vacc[n][3] = 0.f;
 
     // One tile of TT (16 or 32) tokens at token tb of the tile data: C^K core
-    // (tg, rg) at kb + tg * ktg + rg * KRG, C^V core at vb + tg * vtg + rg * VRG;
+    // (tg, rg) at kb + tg * ktg + rg * KRG, C^V core at vb + tg * vtg + rg * VRG
+    // (SWZ: a dense-tail item, whose core (tg, cg) row r lies in TMA box
+    // cg / 8 at row 8 tg + r, 16-byte chunk (cg % 8) ^ r, boxes KRG apart);
     // tg8 token groups present, tokens < nv valid, at least one of them in
     // this tile.  R16 (at least both ranks / 16) fixes the 16-rank steps;
     // R16, TT, KRG and VRG are compile-time constants, so that the body is one
@@ -308,21 +310,34 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
     // the slots are zeroed at start, and the furthest such read ends inside
     // the q~ area): for scores their q~ is 0, and the rank-space values they
     // give are never back-projected.
-    auto tile = [&](auto r16c, auto ttc, auto krgc, auto vrgc, uint32_t kb, uint32_t ktg, uint32_t vb,
+    auto tile = [&](auto r16c, auto ttc, auto krgc, auto vrgc, auto swzc, uint32_t kb, uint32_t ktg, uint32_t vb,
                     uint32_t vtg, int tb, int tg8, int nv) {
         constexpr int R16 = decltype(r16c)::value;
         constexpr int NH = decltype(ttc)::value / 16;  // 16-token halves
         constexpr uint32_t KRG = decltype(krgc)::value, VRG = decltype(vrgc)::value;
+        constexpr bool SWZ = decltype(swzc)::value;
         // per half h: this lane's ldmatrix row address at rank step 0
         uint32_t kh[NH], vh[NH];
+        // swizzled: the 16-byte chunk of column group 2k + b in row r is
+        // (2 (k % 4) ^ (r & 6)) | ((b ^ r) & 1): the first part per k % 4
+        uint32_t sw[4] = {0u, 0u, 0u, 0u};
+        if constexpr (SWZ) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) sw[j] = (uint32_t)((2 * j) ^ (mr & 6)) << 4;
+        }
 #pragma unroll
         for (int h = 0; h < NH; ++h) {
             // scores, matrices (tg0, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks), (tg0 + 1, 2ks + 1)
             const int tgk = min(tb / 8 + 2 * h + (mi >> 1), tg8 - 1);
-            kh[h] = kb + tgk * ktg + (mi & 1) * KRG + mr * 16;
             // values (transposed), matrices (tg0, 2jp), (tg0 + 1, 2jp), (tg0, 2jp + 1), (tg0 + 1, 2jp + 1)
             const int tgv = min(tb / 8 + 2 * h + (mi & 1), tg8 - 1);
-            vh[h] = vb + tgv * vtg + (mi >> 1) * VRG + mr * 16;
+            if constexpr (SWZ) {
+                kh[h] = kb + tgk * 1024 + mr * 128 + ((((mi & 1) ^ mr) & 1) << 4);
+                vh[h] = vb + tgv * 1024 + mr * 128 + ((((mi >> 1) ^ mr) & 1) << 4);
+            } else {
+                kh[h] = kb + tgk * ktg + (mi & 1) * KRG + mr * 16;
+                vh[h] = vb + tgv * vtg + (mi >> 1) * VRG + mr * 16;
+            }
         }
         float s4[2 * NH][4];
 #pragma unroll
@@ -334,7 +349,7 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
 #pragma unroll
             for (int h = 0; h < NH; ++h) {
                 uint32_t b0, b1, b2, b3;
-                ldsm_x4(kh[h] + 2 * ks * KRG, b0, b1, b2, b3);
+                ldsm_x4(SWZ ? kh[h] + (ks >> 2) * KRG + sw[ks & 3] : kh[h] + 2 * ks * KRG, b0, b1, b2, b3);
                 mma16816(s4[2 * h], qa, b0, b1);
                 mma16816(s4[2 * h + 1], qa, b2, b3);
             }
@@ -395,7 +410,7 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
 #pragma unroll
             for (int h = 0; h < NH; ++h) {
                 uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(vh[h] + 2 * jp * VRG, b0, b1, b2, b3);
+                ldsm_x4_t(SWZ ? vh[h] + (jp >> 2) * VRG + sw[jp & 3] : vh[h] + 2 * jp * VRG, b0, b1, b2, b3);
                 mma16816(vacc[2 * jp], pa[h], b0, b1);
                 mma16816(vacc[2 * jp + 1], pa[h], b2, b3);
             }
@@ -453,14 +468,22 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
         const int t0 = sp * kTailTokens;
         ntok = max(0, min(t0 + kTailTokens, T) - t0);
         nrk = nrv = NT;
-        // K then V: one box of kTailTokens rows x 8 columns per column group
-        constexpr uint32_t kBox = kTailTokens * 16, kHalf = NT * kBox;
+        // K then V: one box of kTailTokens rows x 64 columns (128-byte rows,
+        // 128-byte swizzle) per 64 columns; a box starts on a 1024-byte line
+        constexpr uint32_t kBox = kTailTokens * 128, kHalf = (D / 64) * kBox;
+        static_assert(kPieceBytes % 1024 == 0 && kHalf % 1024 == 0, "swizzled boxes on 1024-byte lines");
+        if (ntok > 0 && (tbase & 1023u)) {
+            // (cannot happen: the dynamic shared memory starts on a 1024-byte
+            // line) the item is dropped and the call reports a bounds error
+            if (leader) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
+            ntok = 0;
+        }
         if (ntok > 0 && leader) {
             mbar_arrive_tx(tbar, 2 * kHalf);
-#pragma unroll 1
-            for (int c = 0; c < NT; ++c) {
-                tma_load_3d(tbase + c * kBox, &tmap_k, 8 * c, g, (int)(o0 + t0), tbar);
-                tma_load_3d(tbase + kHalf + c * kBox, &tmap_v, 8 * c, g, (int)(o0 + t0), tbar);
+#pragma unroll
+            for (int c = 0; c < D / 64; ++c) {
+                tma_load_3d(tbase + c * kBox, &tmap_k, 64 * c, g, (int)(o0 + t0), tbar);
+                tma_load_3d(tbase + kHalf + c * kBox, &tmap_v, 64 * c, g, (int)(o0 + t0), tbar);
             }
         }
         // q~ = scale * log2(e) * q of the G heads of query qi, as score A fragments
@@ -490,8 +513,8 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
         const int tb = kTU * warp;
         if (tb < ntok) {
             tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTU>{},
-                 std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{}, tbase, 128,
-                 tbase + kHalf, 128, tb, kTailTokens / 8, ntok);
+                 std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{},
+                 std::true_type{}, tbase, 1024, tbase + kHalf, 1024, tb, kTailTokens / 8, ntok);
             if (warp == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
         }
     } else {
@@ -570,13 +593,15 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
 #pragma unroll 1
                     for (int tb = kTile * warp; tb < nv; tb += kWarps * kTile)
                         tile(r16c, integral_constant<int, kTile>{}, integral_constant<uint32_t, 128>{},
-                             integral_constant<uint32_t, 128>{}, slot, nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
+                             integral_constant<uint32_t, 128>{}, std::false_type{}, slot, nrk * 128, vb, nrv * 128,
+                             tb, r8 / 8, nv);
                 } else {
                     // above: 16-token halves of the tiles round-robin over the warps
 #pragma unroll 1
                     for (int tb = 16 * warp; tb < nv; tb += kWarps * 16)
                         tile(r16c, integral_constant<int, 16>{}, integral_constant<uint32_t, 128>{},
-                             integral_constant<uint32_t, 128>{}, slot, nrk * 128, vb, nrv * 128, tb, r8 / 8, nv);
+                             integral_constant<uint32_t, 128>{}, std::false_type{}, slot, nrk * 128, vb, nrv * 128,
+                             tb, r8 / 8, nv);
                 }
             });
             if (k == ps.npk && warp == 0) ref = publish_ref(p, g, 8 * rgrp + r4, 8 * rgrp + r4 < p.rows_g, c4, m_w);

@@ -857,16 +857,21 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
         if (!enc) return fail(MILO_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
         const cuuint64_t dims[3] = {(cuuint64_t)plan->d, (cuuint64_t)plan->hkv, (cuuint64_t)tail_rows};
         const cuuint64_t strides[2] = {(cuuint64_t)plan->d * 2, (cuuint64_t)plan->hkv * plan->d * 2};
-        // boxes of one 16-byte column chunk: a tail item lands in shared memory as
-        // 8x8 cores [column group][token group], like a packed coefficient tile
-        const cuuint32_t box[3] = {8, 1, (cuuint32_t)kTailTokens};
+        // the chunk grid (its tail items, for every call with at most 8 query
+        // heads per KV head): boxes of 64 columns (128-byte rows, 128-byte
+        // swizzle), few wide requests; the persistent kernel: boxes of one
+        // 16-byte column chunk, landing as 8x8 cores [column group][token
+        // group] like a packed coefficient tile
+        const bool wide = c.chunked;
+        const cuuint32_t box[3] = {wide ? 64u : 8u, 1, (cuuint32_t)kTailTokens};
         const cuuint32_t estr[3] = {1, 1, 1};
+        const CUtensorMapSwizzle swz = wide ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE;
         CUresult r1 = enc(&mk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(tail_k), dims, strides, box,
-                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         CUresult r2 = enc(&mv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(tail_v), dims, strides, box,
-                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS) return fail(MILO_ERR_CUDA, "tensor map encoding failed");
     }
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
