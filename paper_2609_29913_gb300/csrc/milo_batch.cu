@@ -211,14 +211,61 @@ __device__ __forceinline__ void st16(uint32_t taddr, const uint32_t *r)
 __device__ __forceinline__ void wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 }  // namespace tc
 
+// Packed fp32 pairs (one 64-bit register pair; x in the low half): the
+// paired add and subtract round each lane as the scalar instructions do.
+__device__ __forceinline__ uint64_t f2(float x, float y)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+    return r;
+}
+__device__ __forceinline__ void f2get(uint64_t r, float &x, float &y) { asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(r)); }
+__device__ __forceinline__ uint64_t f2add(uint64_t a, uint64_t b)
+{
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2sub(uint64_t a, uint64_t b)
+{
+    uint64_t r;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c)
+{
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+// The maximum of N values by a tree of three-input maxima.
+template <int N>
+__device__ __forceinline__ float max_tree(const float *v)
+{
+    if constexpr (N == 1) {
+        return v[0];
+    } else if constexpr (N == 2) {
+        return fmaxf(v[0], v[1]);
+    } else {
+        constexpr int M = (N + 2) / 3;
+        float t[M];
+#pragma unroll
+        for (int i = 0; i < N / 3; ++i) t[i] = max3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+        if constexpr (N % 3 == 2) t[M - 1] = fmaxf(v[N - 2], v[N - 1]);
+        if constexpr (N % 3 == 1) t[M - 1] = v[N - 1];
+        return max_tree<M>(t);
+    }
+}
+
 // Two fp32 values as a bf16x2 "hi" (each truncated to its leading 8
 // significant bits: the top half of its bits) and the bf16x2 of their
 // residuals (truncated the same way): x = hi + lo to within 2^-15 of |x|,
-// in six integer and add operations.  Low half = x0.
+// in five integer and paired-add operations.  Low half = x0.
 __device__ __forceinline__ void split2(float x0, float x1, uint32_t &hi, uint32_t &lo)
 {
     const uint32_t u0 = __float_as_uint(x0), u1 = __float_as_uint(x1);
-    const float r0 = x0 - __uint_as_float(u0 & 0xffff0000u), r1 = x1 - __uint_as_float(u1 & 0xffff0000u);
+    float r0, r1;
+    f2get(f2sub(f2(x0, x1), f2(__uint_as_float(u0 & 0xffff0000u), __uint_as_float(u1 & 0xffff0000u))), r0, r1);
     hi = __byte_perm(u0, u1, 0x7632);
     lo = __byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x7632);
 }
@@ -734,17 +781,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                 // then the pair's two halves through shared memory (both
                 // warps have read their scores before either overwrites the
                 // tile with p)
-                float t[kHalfTok / 2];
-#pragma unroll
-                for (int i = 0; i < kHalfTok / 2; ++i) t[i] = fmaxf(sv[2 * i], sv[2 * i + 1]);
-#pragma unroll
-                for (int w = kHalfTok / 4; w >= 1; w /= 2)
-#pragma unroll
-                    for (int i = 0; i < w; ++i) t[i] = fmaxf(t[i], t[i + w]);
+                const float tmax = max_tree<kHalfTok>(sv);
                 float *xb = xch + ((J & 1) * 4 + quad) * 64;
-                xb[half * 32 + lane] = t[0];
+                xb[half * 32 + lane] = tmax;
                 pair_sync();
-                const float mx = fmaxf(t[0], xb[(1 - half) * 32 + lane]);
+                const float mx = fmaxf(tmax, xb[(1 - half) * 32 + lane]);
                 // lazy rescale: the reference moves only when a score passes it
                 // by kLazyTc; V~ and O, already summed against the old one,
                 // are multiplied by 2^(m_old - m_new) in tensor memory (the
@@ -795,17 +836,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
                 // p = 2^(s - m) of this warp's columns as bf16 hi | lo over the
                 // score tile (hi in columns [0, 32), lo in [32, 64))
                 uint32_t ph[kHalfTok / 2], pl[kHalfTok / 2];
+                uint64_t t2[kHalfTok / 2];  // pairs of p, then their pairwise sums
+                const uint64_t m2 = f2(m, m);
 #pragma unroll
                 for (int i = 0; i < kHalfTok / 2; ++i) {
-                    const float p0 = ex2_approx(sv[2 * i] - m), p1 = ex2_approx(sv[2 * i + 1] - m);  // masked: 0
-                    t[i] = p0 + p1;
+                    float d0, d1;
+                    f2get(f2sub(f2(sv[2 * i], sv[2 * i + 1]), m2), d0, d1);
+                    const float p0 = ex2_approx(d0), p1 = ex2_approx(d1);  // masked: 0
+                    t2[i] = f2(p0, p1);
                     split2(p0, p1, ph[i], pl[i]);
                 }
 #pragma unroll
                 for (int w = kHalfTok / 4; w >= 1; w /= 2)
 #pragma unroll
-                    for (int i = 0; i < w; ++i) t[i] += t[i + w];
-                l += t[0];
+                    for (int i = 0; i < w; ++i) t2[i] = f2add(t2[i], t2[i + w]);
+                {
+                    float a, c;
+                    f2get(t2[0], a, c);
+                    l += a + c;
+                }
                 tc::st16(sb + (kHalfTok / 2) * half, ph);
                 tc::st16(sb + kTcTok / 2 + (kHalfTok / 2) * half, pl);
                 tc::wait_st();

@@ -226,8 +226,11 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
 
     pdl_trigger();
     // zero the slots, q~ and the zero line: reads past a piece's data then
-    // see finite values (the copies below are ordered after these stores)
-    for (int i = tid; i < L::kBar / 16; i += kThreads) reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
+    // see finite values (the copies below are ordered after these stores).
+    // A tail block reads only the rows its boxes write (out-of-range rows
+    // arrive as zeros) and no rank padding, so its slots stay as they are.
+    for (int i = tid + (is_tail ? L::kQ / 16 : 0); i < L::kBar / 16; i += kThreads)
+        reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0u, 0u, 0u, 0u);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 
     ChunkDev ch = {};
