@@ -323,8 +323,8 @@ milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q,
  *   query heads per KV head (else MILO_ERR_UNSUPPORTED).  q, the
  *   reconstructed keys and values must lie inside the fp16 range (|x| < 65504).
  *   Three kernels at most: the tails' chunk grid (when there are tails), the
- *   reconstructing prefix grid (one block of 4 warps per chunk of up to 256
- *   tokens of one entry and group of up to 64 query rows), the finish grid.
+ *   reconstructing prefix grid (one block of 8 warps per chunk of up to 256
+ *   tokens of one entry and group of up to 128 query rows), the finish grid.
  */
 milo_status_t milo_attn_decode_reconstruct(const milo_prefix_t *plan, const void *q,
                                            int32_t batch, const void *tail_k,

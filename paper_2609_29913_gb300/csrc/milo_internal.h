@@ -87,7 +87,7 @@ static_assert(sizeof(TcSegDev) == 64, "tensor-core segment size");
 // query rows per thread block, and tiles per chunk (a chunk is a thread
 // block's token range of one entry: int4 {entry, first tile, tiles, 0}).
 constexpr int kRcTok = 64;
-constexpr int kRcRows = 64;
+constexpr int kRcRows = 128;
 constexpr int kRcChunkTiles = 4;
 
 // Device-side counters owned by a plan (zero between calls).

@@ -6,18 +6,20 @@
 //
 // Work: the prefix is cut on the host into chunks of at most kRcChunkTiles
 // tiles of kRcTok tokens of one entry (block b, KV head g); one thread block
-// of 4 warps per (chunk, group of up to kRcRows query rows of KV head g).  Per
+// of 8 warps per (chunk, group of up to kRcRows query rows of KV head g).  Per
 // tile the block
 //   1. reconstructs the dense keys and values of the tile's tokens,
 //        K^ = C^K P^K,  V^ = C^V P^V        (Eq. 3 with Sigma folded into C)
-//      with mma.sync (bf16 factors, fp32 sums; warp w makes tokens 16w..16w+15),
-//      rotates each key to its position when the plan holds pre-RoPE factors,
-//      and stores both tiles in shared memory as fp16, as the paper's kernel
-//      fills its fp16 KV buffer;
+//      with mma.sync (bf16 factors, fp32 sums; warp w makes tokens
+//      16 (w % 4) .. + 15 and half of the columns: the pairs (i, i + d/2) of
+//      its half), rotates each key to its position when the plan holds
+//      pre-RoPE factors, and stores both tiles in shared memory as fp16, as
+//      the paper's kernel fills its fp16 KV buffer;
 //   2. runs flash decoding over them (Eq. 1): scores q K^T, an online
-//      softmax in log2 units, o += p V^ (fp16 operands, fp32 sums).  A warp
-//      owns 16 query rows; with fewer than 64 rows in the group the warps of
-//      a 16-row fragment split the tile's tokens and merge at the end.
+//      softmax in log2 units, o += p V^ (fp16 operands, fp32 sums).  Each
+//      16-row fragment of the group has W warps (4, 4, 2 or 1 for groups of
+//      up to 16, 32, 64 or 128 rows), which split the tile's tokens and merge
+//      at the end.
 // Each (chunk, row group) then adds its (o, m, l) into the per-row
 // accumulators of KV head g by the shared-reference merge of milo_merge.cuh
 // (or lists a record for an outlier maximum), like every other item of a
@@ -40,7 +42,8 @@
 namespace milo {
 namespace {
 
-constexpr int kRcThreads = 128;
+constexpr int kRcWarps = 8;
+constexpr int kRcThreads = 32 * kRcWarps;
 constexpr int kRcRing = 3;
 
 template <int D>
@@ -58,8 +61,8 @@ struct RcLay {
     // after the last tile the ring holds the warps' merge records:
     // [warp][D/8 column tiles][32 lanes] float4, then [warp][32 lanes] float4 (m0, m1, l0, l1)
     static constexpr int kXO = kC;
-    static constexpr int kXM = kXO + 4 * (D / 8) * 32 * 16;
-    static_assert(kXM + 4 * 32 * 16 <= kC + kRcRing * kCBuf, "merge records fit the ring");
+    static constexpr int kXM = kXO + kRcWarps * (D / 8) * 32 * 16;
+    static_assert(kXM + kRcWarps * 32 * 16 <= kC + kRcRing * kCBuf, "merge records fit the ring");
     static_assert(kTotal <= 232448, "one block per SM");
 };
 
@@ -86,34 +89,45 @@ __device__ __forceinline__ uint32_t bf2_to_h2(uint32_t x)
     return pack_half2(lo, hi);
 }
 
-// One fp32 tile of 16 tokens x D columns (warp-fragment layout: n-tile j,
-// elements 0,1 row r4, columns 8j + 2c4 + {0,1}; elements 2,3 row r4 + 8)
-// = C (16 tokens x rank, cores [token group][rank group], nr = rank groups)
-// times P (rank x D, cores [rank group][column group]), over ks16 16-rank
-// steps.  Rank groups past the rank read a zero core line of P.
+// The 8-column tiles of a warp's half h of the head dimension: local tile
+// i < D/32 is column tile h D/32 + i, and local tile i + D/32 its rotary
+// partner (the same columns + D/2).
 template <int D>
-__device__ __forceinline__ void reconstruct16(float (&acc)[D / 8][4], uint32_t c_base, int tg0, int nr, int ks16,
-                                              uint32_t p_base, int mi, int mr)
+__device__ __forceinline__ int col_tile(int h, int i)
+{
+    return i < D / 32 ? h * (D / 32) + i : D / 16 + h * (D / 32) + (i - D / 32);
+}
+
+// One fp32 tile of 16 tokens x half the columns (warp-fragment layout: local
+// tile i, elements 0,1 row r4, columns 8 col_tile(h, i) + 2c4 + {0,1};
+// elements 2,3 row r4 + 8) = C (16 tokens x rank, cores [token group][rank
+// group], nr = rank groups) times P (rank x D, cores [rank group][column
+// group]), over ks16 16-rank steps.  Rank groups past the rank read the
+// zeroed rows of P.
+template <int D>
+__device__ __forceinline__ void reconstruct16(float (&acc)[D / 16][4], uint32_t c_base, int tg0, int nr, int ks16,
+                                              uint32_t p_base, int h, int mi, int mr)
 {
 #pragma unroll
-    for (int j = 0; j < D / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+    for (int i = 0; i < D / 16; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
 #pragma unroll 1
     for (int ks = 0; ks < ks16; ++ks) {
         uint32_t a[4];
         // matrices (tg0, 2ks), (tg0 + 1, 2ks), (tg0, 2ks + 1), (tg0 + 1, 2ks + 1)
         ldsm_x4(c_base + ((tg0 + (mi & 1)) * nr + 2 * ks + (mi >> 1)) * 128 + mr * 16, a[0], a[1], a[2], a[3]);
 #pragma unroll
-        for (int jp = 0; jp < D / 16; ++jp) {
-            // transposed: (2ks, 2jp), (2ks + 1, 2jp), (2ks, 2jp + 1), (2ks + 1, 2jp + 1)
+        for (int ip = 0; ip < D / 32; ++ip) {
+            // transposed: (2ks, j), (2ks + 1, j), (2ks, j + 1), (2ks + 1, j + 1), j = col_tile(2 ip)
+            const int j = col_tile<D>(h, 2 * ip);
             uint32_t b0, b1, b2, b3;
-            ldsm_x4_t(p_base + ((2 * ks + (mi & 1)) * (D / 8) + 2 * jp + (mi >> 1)) * 128 + mr * 16, b0, b1, b2, b3);
-            mma16816(acc[2 * jp], a, b0, b1);
-            mma16816(acc[2 * jp + 1], a, b2, b3);
+            ldsm_x4_t(p_base + ((2 * ks + (mi & 1)) * (D / 8) + j + (mi >> 1)) * 128 + mr * 16, b0, b1, b2, b3);
+            mma16816(acc[2 * ip], a, b0, b1);
+            mma16816(acc[2 * ip + 1], a, b2, b3);
         }
     }
 }
 
-// W warps per 16-row fragment (4, 2 or 1: groups of at most 16, 32 or 64
+// W warps per 16-row fragment (4, 2 or 1: groups of at most 32, 64 or 128
 // rows); ROPE: the keys are pre-RoPE and turn to their positions.
 template <int D, int W, bool ROPE>
 __global__ void __launch_bounds__(kRcThreads, 1) recon_kernel(const __grid_constant__ DecodeParams p)
@@ -128,8 +142,8 @@ __global__ void __launch_bounds__(kRcThreads, 1) recon_kernel(const __grid_const
     const uint32_t bar_p = sbase + L::kBar;
     auto bar_c = [&](int k) { return bar_p + 8 * (1 + k % kRcRing); };
 
-    const int nrg64 = (p.rows_g + kRcRows - 1) / kRcRows;
-    const int chunk = (int)blockIdx.x / nrg64, rg64 = (int)blockIdx.x % nrg64;
+    const int nrgb = (p.rows_g + kRcRows - 1) / kRcRows;
+    const int chunk = (int)blockIdx.x / nrgb, rgb = (int)blockIdx.x % nrgb;
     const int4 ck = p.rc_chunks[chunk];  // entry, first tile, tiles
     const EntryDev en = p.entries[ck.x];
     const int g = en.g, n = en.n;
@@ -167,7 +181,7 @@ __global__ void __launch_bounds__(kRcThreads, 1) recon_kernel(const __grid_const
 
     // this warp's fragment (16 rows) and token slice
     const int frag = warp / W, slice = warp % W;
-    const int rbase = rg64 * kRcRows + 16 * frag;  // first row of the fragment within KV head g
+    const int rbase = rgb * kRcRows + 16 * frag;  // first row of the fragment within KV head g
     const bool frag_ok = rbase < p.rows_g;
     const int row0 = rbase + r4, row1 = row0 + 8;
     const bool ok0 = row0 < p.rows_g, ok1 = row1 < p.rows_g;
@@ -209,39 +223,43 @@ __global__ void __launch_bounds__(kRcThreads, 1) recon_kernel(const __grid_const
         const uint32_t cb = sbase + L::kC + (k % kRcRing) * L::kCBuf;
         const int nv = min(kRcTok, n - (tile0 + k) * kRcTok);  // valid tokens of the tile
 
-        // ---- 1. reconstruct 16 tokens (warp) x D of K^ and V^ into fp16 tiles
+        // ---- 1. reconstruct 16 tokens x half of the columns (warp) of K^ and
+        // V^ into fp16 tiles
         {
-            float acc[D / 8][4];
-            reconstruct16<D>(acc, cb, 2 * warp, nrk, (nrk + 1) >> 1, sbase + L::kPK, mi, mr);
+            const int mt = warp & 3, hh = warp >> 2;  // token 16-group, column half
+            float acc[D / 16][4];
+            reconstruct16<D>(acc, cb, 2 * mt, nrk, (nrk + 1) >> 1, sbase + L::kPK, hh, mi, mr);
             if constexpr (ROPE) {
-                // pair (i, i + D/2) = column tiles (j, j + D/16), same registers;
+                // pair (i, i + D/2) = local tiles (t, t + D/32), same registers;
                 // angle = (tile start + u) theta_i from the plan's tables
                 const float2 *tab_t = p.rope_tile + ((int64_t)p.rope_tile_base[b] + tile0 + k) * (D / 2);
 #pragma unroll
-                for (int j = 0; j < D / 16; ++j)
+                for (int t = 0; t < D / 32; ++t)
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const int i = 8 * j + 2 * c4 + (e & 1);
-                        const int u = 16 * warp + r4 + (e >> 1) * 8;
+                        const int i = 8 * col_tile<D>(hh, t) + 2 * c4 + (e & 1);
+                        const int u = 16 * mt + r4 + (e >> 1) * 8;
                         const float2 a = __ldg(tab_t + i), c = __ldg(p.rope_off + u * (D / 2) + i);
                         const float cs = a.x * c.x - a.y * c.y, sn = a.y * c.x + a.x * c.y;
-                        const float x0 = acc[j][e], x1 = acc[j + D / 16][e];
-                        acc[j][e] = x0 * cs - x1 * sn;
-                        acc[j + D / 16][e] = x1 * cs + x0 * sn;
+                        const float x0 = acc[t][e], x1 = acc[t + D / 32][e];
+                        acc[t][e] = x0 * cs - x1 * sn;
+                        acc[t + D / 32][e] = x1 * cs + x0 * sn;
                     }
             }
             uint32_t *kk = reinterpret_cast<uint32_t *>(smem + L::kK);
 #pragma unroll
-            for (int j = 0; j < D / 8; ++j) {
-                kk[((2 * warp) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[j][0], acc[j][1]);
-                kk[((2 * warp + 1) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[j][2], acc[j][3]);
+            for (int t = 0; t < D / 16; ++t) {
+                const int j = col_tile<D>(hh, t);
+                kk[((2 * mt) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[t][0], acc[t][1]);
+                kk[((2 * mt + 1) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[t][2], acc[t][3]);
             }
-            reconstruct16<D>(acc, cb + L::kCSide, 2 * warp, nrv, (nrv + 1) >> 1, sbase + L::kPV, mi, mr);
+            reconstruct16<D>(acc, cb + L::kCSide, 2 * mt, nrv, (nrv + 1) >> 1, sbase + L::kPV, hh, mi, mr);
             uint32_t *vv = reinterpret_cast<uint32_t *>(smem + L::kV);
 #pragma unroll
-            for (int j = 0; j < D / 8; ++j) {
-                vv[((2 * warp) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[j][0], acc[j][1]);
-                vv[((2 * warp + 1) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[j][2], acc[j][3]);
+            for (int t = 0; t < D / 16; ++t) {
+                const int j = col_tile<D>(hh, t);
+                vv[((2 * mt) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[t][0], acc[t][1]);
+                vv[((2 * mt + 1) * (D / 8) + j) * 32 + r4 * 4 + c4] = pack_half2(acc[t][2], acc[t][3]);
             }
         }
         __syncthreads();
@@ -467,10 +485,10 @@ cudaError_t launch_recon(const DecodeParams &p, int num_chunks, cudaStream_t str
 {
     const int64_t blocks = (int64_t)num_chunks * ((p.rows_g + kRcRows - 1) / kRcRows);
     if (blocks < 1 || blocks > 0x7fffffff) return cudaErrorInvalidValue;
-    // warps per 16-row fragment: the 4 warps split the rows of a group of up
-    // to 16, 32 or 64 rows
+    // warps per 16-row fragment: groups of up to 32 rows (one or two
+    // fragments) give each fragment 4 warps, of up to 64 rows 2, else 1
     const int f = ((p.rows_g < kRcRows ? p.rows_g : kRcRows) + 15) / 16;
-    const int w = f == 1 ? 4 : f == 2 ? 2 : 1;
+    const int w = f <= 2 ? 4 : f <= 4 ? 2 : 1;
     const bool rope = p.rope_tile != nullptr;
     if (p.d == 64) return rope ? launch_d<64, true>(p, (int)blocks, w, stream) : launch_d<64, false>(p, (int)blocks, w, stream);
     return rope ? launch_d<128, true>(p, (int)blocks, w, stream) : launch_d<128, false>(p, (int)blocks, w, stream);

@@ -3,9 +3,9 @@ paper's own inference path: dense keys and values rebuilt from the factors,
 then attended) and of its pre-RoPE variant, against the fp64 oracle, through
 the C ABI.
 
-The cases cover the three ways the 4 warps of a block share rows (groups of
-up to 16, 32 and 64 query rows, and more than one group), head dimensions 64
-and 128, ragged blocks (1 to 600 tokens: partial tiles and several chunks),
+The cases cover the ways the 8 warps of a block share rows (4 warps per
+16-row fragment in groups of up to 32 query rows, 2 up to 64, 1 up to 128,
+and more than one group), head dimensions 64 and 128, ragged blocks (1 to 600 tokens: partial tiles and several chunks),
 ranks 0 (K, V or both) next to full ranks, a peaked softmax, outlier scores
 that force the listed-record merge, calls without tails, rotation tables for
 the default and for explicit block positions, the refusal of the rank-space
@@ -57,16 +57,18 @@ def compare(got, ref, what=""):
 
 CASES = {
     # name: (hq, hkv, d, block_lens, rank_choices, batch, tail_lengths, separate_kv)
-    # 7 rows per KV head: one fragment, the 4 warps split each tile's tokens
+    # 7 rows per KV head: one fragment, 4 warps split each tile's tokens
     "b1-g7-d128": (28, 4, 128, [512, 300, 64, 65, 1], (16, 32, 64, 96, 128), 1, [256], True),
-    # 28 rows: two fragments, two warps each
+    # 28 rows: two fragments, four warps each
     "b4-g7-d128": (28, 4, 128, [200, 600, 7], (8, 40, 96, 128), 4, [5, 64, 0, 130], True),
-    # 70 rows: two groups of up to 64 rows, a warp per fragment
+    # 70 rows: one group, a warp per fragment
     "b10-g7-d128": (14, 2, 128, [512, 129], (16, 64, 128), 10, [(37 * i) % 90 for i in range(10)], False),
-    # head dimension 64, ragged blocks, ranks 1 .. 64, 48 rows (three fragments)
+    # 140 rows: two groups (128 + 12 rows)
+    "b20-g7-d128": (28, 4, 128, [256, 77], (16, 64, 128), 20, [(41 * i) % 70 for i in range(20)], True),
+    # head dimension 64, ragged blocks, ranks 1 .. 64, 48 rows (three fragments, two warps each)
     "d64-ragged": (8, 2, 64, [1, 7, 129, 64, 200], (1, 4, 7, 8, 13, 64), 12,
                    [(7 * i) % 50 for i in range(12)], True),
-    # G = 5, 80 rows (one group of 64 and one of 16), long tails
+    # G = 5, 80 rows (five fragments), long tails
     "g5-b16": (40, 8, 128, [512, 256], (32, 77, 128), 16, [1024 - 50 * i for i in range(16)], True),
     # G = 1 and no tails
     "g1-notail": (4, 4, 128, [300, 64, 100], (16, 128), 3, [0, 0, 0], True),
