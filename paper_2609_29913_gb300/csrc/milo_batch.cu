@@ -209,6 +209,43 @@ __device__ __forceinline__ void st16(uint32_t taddr, const uint32_t *r)
         : "memory");
 }
 __device__ __forceinline__ void wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// The 16-lane shapes: threads 0-15 access lanes base .. base + 15 at the
+// address's column, threads 16-31 the same lanes OFF columns further.
+template <int OFF>
+__device__ __forceinline__ void ld16x2(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], %17;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr), "n"(OFF)
+        : "memory");
+}
+template <int OFF>
+__device__ __forceinline__ void ld16x2f(uint32_t taddr, float (&v)[16])
+{
+    uint32_t r[16];
+    ld16x2<OFF>(taddr, r);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+template <int OFF>
+__device__ __forceinline__ void st8x2(uint32_t taddr, const uint32_t *r)
+{
+    asm volatile("tcgen05.st.sync.aligned.16x32bx2.x8.b32 [%0], %9, {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
+                 "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "n"(OFF)
+                 : "memory");
+}
+template <int OFF>
+__device__ __forceinline__ void st16x2(uint32_t taddr, const uint32_t *r)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x32bx2.x16.b32 [%0], %17, {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+            taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+        "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "n"(OFF)
+        : "memory");
+}
 }  // namespace tc
 
 // Packed fp32 pairs (one 64-bit register pair; x in the low half): the
@@ -658,312 +695,363 @@ __global__ void __launch_bounds__(kTcThreads, 1) batch_tc_kernel(const __grid_co
     } else {
         // ------------------------------------------------ softmax
         // Warps 2..9, two per tensor-memory lane quarter: the pair (half 0
-        // and 1) shares the quarter's 32 rows and splits every tile's 64
+        // and 1) shares the quarter's rows and splits every tile's 64
         // columns, every rank chunk and the head dimension; a pair meets
-        // through a named barrier once per tile (the row maximum).
-        const int quad = warp & 3, half = (warp - 2) >> 2;
-        const int rl = 32 * quad + lane;          // row within the tile
-        const int row = tile * kTcRows + rl;      // the KV head's query row (batch x heads)
-        const bool row_ok = row < p.rows_g;
-        const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
-        uint8_t *q_s = smem + L::kQ, *qt_s = smem + L::kQt;
-        float *xch = reinterpret_cast<float *>(smem + L::kX);  // maxima [2][4][2][32], row sums [4][32]
-        const int rg8 = rl >> 3, r8 = rl & 7;     // core row group and row within the core
-        constexpr int kHalfTok = kTcTok / 2;      // columns of a tile per warp
+        // through a named barrier once per tile (the row maximum).  A tile
+        // of at most 64 rows is spread 16 rows per quarter (row r on lane
+        // 32 (r / 16) + r % 16, the other lanes hold zero rows), so that
+        // all four sub-partitions share its softmax: a warp then reaches its
+        // 16 lanes with the 16-lane shapes, threads 16-31 taking the second
+        // half of the warp's columns.  Only a call of one such tile spreads:
+        // beside full tiles of the same shares (which read the same pieces)
+        // a spread tile gained nothing and the full ones slowed down (76 to
+        // 81 us a block on the batch-64 layer, against 421 to 377 us for the
+        // one tile of the 56-row, 1M-token layer).
         pdl_wait();  // q and the accumulators belong to the preceding grids until here
-        int J = 0, kseg = 0, kproj = 0, bp_waited = 0;
-        bool ok = true;
-        float m = -INFINITY, l = 0.f;             // l: this warp's columns only
-        bool o_written = false, first_tile = true;
-        uint32_t ref = 0u;
-        auto arrive = [&](int b) {
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(b));
-        };
-        auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory"); };
-        // the warp-collective tensor-memory accesses after a wait need every
-        // lane to agree on its outcome
-        auto wwait = [&](int b, int parity) {
-            ok = __all_sync(0xffffffffu, ok && tc_wait(bar(b), (uint32_t)parity & 1u, p.status, abort_flag));
-            tc::fence_after();
-        };
-        // back-projections done up to segment k (in phase order)
-        auto wait_bp_upto = [&](int k) {
-            while (bp_waited <= k) {
-                wwait(TB_BPDONE, bp_waited);
-                ++bp_waited;
-            }
-        };
-        // a run's q rows as the projection's A operand (this warp's half of
-        // the columns)
-        auto write_qrows = [&](const SegPlan &q) {
-            const uint4 *qr = reinterpret_cast<const uint4 *>(
-                p.q + ((int64_t)(row / p.G) * p.hq + q.g * p.G + row % p.G) * D);
-#pragma unroll 4
-            for (int c = half * (DG / 2); c < (half + 1) * (DG / 2); ++c) {
-                const uint4 v = row_ok ? __ldcg(qr + c) : make_uint4(0u, 0u, 0u, 0u);
-                *reinterpret_cast<uint4 *>(q_s + (rg8 * DG + c) * 128 + r8 * 16) = v;
-            }
-            tc::fence_proxy();
-            arrive(TB_QROWS);
-        };
-        // segment s's q~ = scale log2(e) Q P^K^T as hi and lo A operands in
-        // shared memory (rank chunks of this warp's parity; ranks past the
-        // rank: zero), then the next run's q rows if segment s + 1 starts one
-        // (its projection is issued as soon as q~ is staged)
-        auto prepare = [&](int s, const TcSegDev &sd, const TcSegDev &sd_next) {
-            const SegPlan q = seg_plan(sd);
-            wwait(TB_PROJ, kproj++);
-            if (ok) {
-#pragma unroll 1
-                for (int c = half; c < q.nk16; c += 2) {
-                    float v[16];
-                    tc::ld16f(tl + kColQ + 16 * c, v);
-                    tc::wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) v[i] = 16 * c + i < q.rk ? v[i] * p.scale_log2 : 0.f;
-                    uint8_t *hi = qt_s + (rg8 * DG + 2 * c) * 128 + r8 * 16;
-                    put16(hi, hi + L::kQtHalf, v);
+        const bool spread = p.tc_ntile == 1 && p.rows_g <= kTcRows / 2;
+        auto role = [&](auto spc) {
+            constexpr bool SP = decltype(spc)::value;
+            const int quad = warp & 3, half = (warp - 2) >> 2;
+            const int u = SP ? lane >> 4 : 0;           // SP: which 16 of the warp's 32 columns
+            const int ts = SP ? lane & 15 : lane;       // the thread's row within the quarter
+            const int rl = (SP ? 16 : 32) * quad + ts;  // row within the tile
+            const int pos = 32 * quad + ts;             // its tensor-memory lane (and A-operand row)
+            const int row = tile * kTcRows + rl;        // the KV head's query row (batch x heads)
+            const bool row_ok = row < p.rows_g;
+            const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
+            uint8_t *q_s = smem + L::kQ, *qt_s = smem + L::kQt;
+            float *xch = reinterpret_cast<float *>(smem + L::kX);  // maxima [2][4][2][32], row sums [4][32]
+            const int rg8 = pos >> 3, r8 = pos & 7;     // core row group and row within the core (r8 = row % 8)
+            constexpr int kHalfTok = kTcTok / 2;        // columns of a tile per warp
+            constexpr int kCols = SP ? kHalfTok / 2 : kHalfTok;  // ... per thread
+            int J = 0, kseg = 0, kproj = 0, bp_waited = 0;
+            bool ok = true;
+            float m = -INFINITY, l = 0.f;             // l: this warp's columns only
+            bool o_written = false, first_tile = true;
+            uint32_t ref = 0u;
+            auto arrive = [&](int b) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(b));
+            };
+            auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + quad) : "memory"); };
+            // the warp-collective tensor-memory accesses after a wait need every
+            // lane to agree on its outcome
+            auto wwait = [&](int b, int parity) {
+                ok = __all_sync(0xffffffffu, ok && tc_wait(bar(b), (uint32_t)parity & 1u, p.status, abort_flag));
+                tc::fence_after();
+            };
+            // back-projections done up to segment k (in phase order)
+            auto wait_bp_upto = [&](int k) {
+                while (bp_waited <= k) {
+                    wwait(TB_BPDONE, bp_waited);
+                    ++bp_waited;
                 }
-            }
-            tc::fence_proxy();
-            tc::fence_before();
-            arrive(TB_QT);
-            if (s + 1 < s_end) {
-                const SegPlan qn = seg_plan(sd_next);
-                if (qn.first_of_run) write_qrows(qn);
-            }
-        };
-        SegWalk w;
-        w.start(p.tc_segs, s_begin, s_end);
-        if (s_begin < s_end) {
-            const TcSegDev first = p.tc_segs[s_begin];
-            write_qrows(seg_plan(first));
-            prepare(s_begin, first, s_begin + 1 < s_end ? p.tc_segs[s_begin + 1] : first);
-        }
-        for (int s = s_begin; s < s_end; ++s, ++kseg) {
-            w.at(s);
-            const SegPlan q = seg_plan(w.cur);
-            const int g = q.g;
-            if (q.first_of_run) {
-                m = -INFINITY;
-                l = 0.f;
-                o_written = false;
-                first_tile = true;
-            }
-            const int ntok = q.t1 - q.t0;
-#pragma unroll 1
-            for (int j = 0; j < q.ntiles; ++j, ++J) {
-                const int b = J & 1;
-                const uint32_t sb = tl + kColS + kTcTok * b;
-                wwait(TB_SFULL + b, J >> 1);
-                float sv[kHalfTok];
-                if (ok && q.rk > 0) {
-                    float v0[16], v1[16];
-                    tc::ld16f(sb + kHalfTok * half, v0);
-                    tc::ld16f(sb + kHalfTok * half + 16, v1);
-                    tc::wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        sv[i] = v0[i];
-                        sv[16 + i] = v1[i];
+            };
+            // a run's q rows as the projection's A operand (this thread's share
+            // of the columns)
+            auto write_qrows = [&](const SegPlan &q) {
+                const uint4 *qr = reinterpret_cast<const uint4 *>(
+                    p.q + ((int64_t)(row / p.G) * p.hq + q.g * p.G + row % p.G) * D);
+                constexpr int kParts = SP ? 4 : 2;
+                const int part = SP ? 2 * half + u : half;
+    #pragma unroll 4
+                for (int c = part * (DG / kParts); c < (part + 1) * (DG / kParts); ++c) {
+                    const uint4 v = row_ok ? __ldcg(qr + c) : make_uint4(0u, 0u, 0u, 0u);
+                    *reinterpret_cast<uint4 *>(q_s + (rg8 * DG + c) * 128 + r8 * 16) = v;
+                }
+                tc::fence_proxy();
+                arrive(TB_QROWS);
+            };
+            // segment s's q~ = scale log2(e) Q P^K^T as hi and lo A operands in
+            // shared memory (rank chunks of this warp's parity; ranks past the
+            // rank: zero), then the next run's q rows if segment s + 1 starts one
+            // (its projection is issued as soon as q~ is staged)
+            auto prepare = [&](int s, const TcSegDev &sd, const TcSegDev &sd_next) {
+                const SegPlan q = seg_plan(sd);
+                wwait(TB_PROJ, kproj++);
+                if (ok) {
+                    // rank chunks of 16: SP, chunk pair cp (of this warp's
+                    // parity) gives the thread chunk 2 cp + u
+    #pragma unroll 1
+                    for (int cc = half; (SP ? 2 * cc : cc) < q.nk16; cc += 2) {
+                        float v[16];
+                        int c = cc;
+                        if constexpr (SP) {
+                            tc::ld16x2f<16>(tl + kColQ + 32 * cc, v);
+                            c = 2 * cc + u;
+                        } else {
+                            tc::ld16f(tl + kColQ + 16 * cc, v);
+                        }
+                        tc::wait_ld();
+    #pragma unroll
+                        for (int i = 0; i < 16; ++i) v[i] = 16 * c + i < q.rk ? v[i] * p.scale_log2 : 0.f;
+                        uint8_t *hi = qt_s + (rg8 * DG + 2 * c) * 128 + r8 * 16;
+                        put16(hi, hi + L::kQtHalf, v);
                     }
-                } else {
-#pragma unroll
-                    for (int i = 0; i < kHalfTok; ++i) sv[i] = 0.f;
                 }
-                const int nvalid = min(kTcTok, ntok - kTcTok * j) - kHalfTok * half;  // this warp's valid columns
-                if (nvalid < kHalfTok) {
-#pragma unroll
-                    for (int i = 0; i < kHalfTok; ++i) sv[i] = i < nvalid ? sv[i] : -INFINITY;
+                tc::fence_proxy();
+                tc::fence_before();
+                arrive(TB_QT);
+                if (s + 1 < s_end) {
+                    const SegPlan qn = seg_plan(sd_next);
+                    if (qn.first_of_run) write_qrows(qn);
                 }
-                // the row maximum of the tile: a tree over this warp's columns,
-                // then the pair's two halves through shared memory (both
-                // warps have read their scores before either overwrites the
-                // tile with p)
-                const float tmax = max_tree<kHalfTok>(sv);
-                float *xb = xch + ((J & 1) * 4 + quad) * 64;
-                xb[half * 32 + lane] = tmax;
-                pair_sync();
-                const float mx = fmaxf(tmax, xb[(1 - half) * 32 + lane]);
-                // lazy rescale: the reference moves only when a score passes it
-                // by kLazyTc; V~ and O, already summed against the old one,
-                // are multiplied by 2^(m_old - m_new) in tensor memory (the
-                // pair splits the rank and head-dimension chunks)
-                const bool need = mx > m + kLazyTc;
-                if (__any_sync(0xffffffffu, need)) {
-                    const float mn = need ? mx : m;
-                    const float alpha = need ? exp2_diff(m, mn) : 1.f;
-                    if (j > 0) {
-                        // the value products of tile j - 1 (and every earlier
-                        // product) must be done
-                        const int Jp = J - 1;
-                        wwait(TB_PVDONE + (Jp & 1), Jp >> 1);
-                        if (ok && q.rv > 0) {
-#pragma unroll 1
-                            for (int c = half; c < q.nv16; c += 2) {
-                                uint32_t r[16];
-                                tc::ld16(tl + kColV + 16 * c, r);
-                                tc::wait_ld();
-#pragma unroll
-                                for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-                                tc::st16(tl + kColV + 16 * c, r);
+            };
+            SegWalk w;
+            w.start(p.tc_segs, s_begin, s_end);
+            if (s_begin < s_end) {
+                const TcSegDev first = p.tc_segs[s_begin];
+                write_qrows(seg_plan(first));
+                prepare(s_begin, first, s_begin + 1 < s_end ? p.tc_segs[s_begin + 1] : first);
+            }
+            for (int s = s_begin; s < s_end; ++s, ++kseg) {
+                w.at(s);
+                const SegPlan q = seg_plan(w.cur);
+                const int g = q.g;
+                if (q.first_of_run) {
+                    m = -INFINITY;
+                    l = 0.f;
+                    o_written = false;
+                    first_tile = true;
+                }
+                const int ntok = q.t1 - q.t0;
+    #pragma unroll 1
+                for (int j = 0; j < q.ntiles; ++j, ++J) {
+                    const int b = J & 1;
+                    const uint32_t sb = tl + kColS + kTcTok * b;
+                    wwait(TB_SFULL + b, J >> 1);
+                    float sv[kCols];
+                    if (ok && q.rk > 0) {
+                        if constexpr (SP) {
+                            tc::ld16x2f<16>(sb + kHalfTok * half, sv);
+                            tc::wait_ld();
+                        } else {
+                            float v0[16], v1[16];
+                            tc::ld16f(sb + kHalfTok * half, v0);
+                            tc::ld16f(sb + kHalfTok * half + 16, v1);
+                            tc::wait_ld();
+    #pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                sv[i] = v0[i];
+                                sv[16 + i] = v1[i];
+                            }
+                        }
+                    } else {
+    #pragma unroll
+                        for (int i = 0; i < kCols; ++i) sv[i] = 0.f;
+                    }
+                    // this thread's valid columns
+                    const int nvalid = min(kTcTok, ntok - kTcTok * j) - kHalfTok * half - kCols * u;
+                    if (nvalid < kCols) {
+    #pragma unroll
+                        for (int i = 0; i < kCols; ++i) sv[i] = i < nvalid ? sv[i] : -INFINITY;
+                    }
+                    // the row maximum of the tile: a tree over this warp's columns,
+                    // then the pair's two halves through shared memory (both
+                    // warps have read their scores before either overwrites the
+                    // tile with p)
+                    float tmax = max_tree<kCols>(sv);
+                    if constexpr (SP) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
+                    float *xb = xch + ((J & 1) * 4 + quad) * 64;
+                    xb[half * 32 + ts] = tmax;
+                    pair_sync();
+                    const float mx = fmaxf(tmax, xb[(1 - half) * 32 + ts]);
+                    // lazy rescale: the reference moves only when a score passes it
+                    // by kLazyTc; V~ and O, already summed against the old one,
+                    // are multiplied by 2^(m_old - m_new) in tensor memory (the
+                    // pair splits the rank and head-dimension chunks)
+                    const bool need = mx > m + kLazyTc;
+                    if (__any_sync(0xffffffffu, need)) {
+                        const float mn = need ? mx : m;
+                        const float alpha = need ? exp2_diff(m, mn) : 1.f;
+                        if (j > 0) {
+                            // the value products of tile j - 1 (and every earlier
+                            // product) must be done
+                            const int Jp = J - 1;
+                            wwait(TB_PVDONE + (Jp & 1), Jp >> 1);
+                            if (ok && q.rv > 0) {
+    #pragma unroll 1
+                                for (int c = half; (SP ? 2 * c : c) < q.nv16; c += 2) {
+                                    uint32_t r[16];
+                                    if constexpr (SP) tc::ld16x2<16>(tl + kColV + 32 * c, r); else tc::ld16(tl + kColV + 16 * c, r);
+                                    tc::wait_ld();
+    #pragma unroll
+                                    for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                                    if constexpr (SP) tc::st16x2<16>(tl + kColV + 32 * c, r); else tc::st16(tl + kColV + 16 * c, r);
+                                }
+                            }
+                        }
+                        if (o_written) {
+                            wait_bp_upto(kseg - 1);  // every back-projection of the run is done
+                            if (ok) {
+    #pragma unroll 1
+                                for (int c = half; c < (SP ? D / 32 : D / 16); c += 2) {
+                                    uint32_t r[16];
+                                    if constexpr (SP) tc::ld16x2<16>(tl + kColO + 32 * c, r); else tc::ld16(tl + kColO + 16 * c, r);
+                                    tc::wait_ld();
+    #pragma unroll
+                                    for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                                    if constexpr (SP) tc::st16x2<16>(tl + kColO + 32 * c, r); else tc::st16(tl + kColO + 16 * c, r);
+                                }
+                            }
+                        }
+                        tc::wait_st();
+                        l *= alpha;
+                        m = mn;
+                    }
+                    if (first_tile) {
+                        ref = publish_ref(p, g, row, row_ok, u, m);  // (SP: the thread with u = 0)
+                        if constexpr (SP) ref = __shfl_sync(0xffffffffu, ref, ts);
+                        first_tile = false;
+                    }
+                    // p = 2^(s - m) of this warp's columns as bf16 hi | lo over the
+                    // score tile (hi in columns [0, 32), lo in [32, 64))
+                    uint32_t ph[kCols / 2], pl[kCols / 2];
+                    uint64_t t2[kCols / 2];  // pairs of p, then their pairwise sums
+                    const uint64_t m2 = f2(m, m);
+    #pragma unroll
+                    for (int i = 0; i < kCols / 2; ++i) {
+                        float d0, d1;
+                        f2get(f2sub(f2(sv[2 * i], sv[2 * i + 1]), m2), d0, d1);
+                        const float p0 = ex2_approx(d0), p1 = ex2_approx(d1);  // masked: 0
+                        t2[i] = f2(p0, p1);
+                        split2(p0, p1, ph[i], pl[i]);
+                    }
+    #pragma unroll
+                    for (int w = kCols / 4; w >= 1; w /= 2)
+    #pragma unroll
+                        for (int i = 0; i < w; ++i) t2[i] = f2add(t2[i], t2[i + w]);
+                    {
+                        float a, c;
+                        f2get(t2[0], a, c);
+                        l += a + c;
+                    }
+                    if constexpr (SP) {
+                        tc::st8x2<8>(sb + (kHalfTok / 2) * half, ph);
+                        tc::st8x2<8>(sb + kTcTok / 2 + (kHalfTok / 2) * half, pl);
+                    } else {
+                        tc::st16(sb + (kHalfTok / 2) * half, ph);
+                        tc::st16(sb + kTcTok / 2 + (kHalfTok / 2) * half, pl);
+                    }
+                    tc::wait_st();
+                    tc::fence_before();
+                    arrive(TB_PREADY + b);
+                }
+                // the next segment's q~ (its projection went ahead), then this
+                // segment's v~ as the back-projection's hi and lo A operands, in
+                // place in tensor memory (hi at +0, lo at +64; ranks past the
+                // rank: zero): both warps of the pair read their chunks before
+                // either writes
+                if (s + 1 < s_end) prepare(s + 1, w.next, w.after);
+                wwait(TB_VDONE, kseg);
+                if (q.rv > 0) {
+                    // (the pair barrier runs in both warps whatever ok says)
+                    // rank chunks of 16 (SP: chunk pairs, the thread's chunk 2 cc + u)
+                    constexpr int kNC = SP ? D / 64 : D / 32;  // chunks (SP: pairs) per warp
+                    uint32_t vh[8 * kNC], vl[8 * kNC];
+    #pragma unroll
+                    for (int k = 0; k < kNC; ++k) {
+                        const int cc = 2 * k + half, c = SP ? 2 * cc + u : cc;
+                        if (ok && (SP ? 2 * cc : cc) < q.nv16) {
+                            float v[16];
+                            if constexpr (SP) tc::ld16x2f<16>(tl + kColV + 32 * cc, v); else tc::ld16f(tl + kColV + 16 * cc, v);
+                            tc::wait_ld();
+    #pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const float x0 = 16 * c + 2 * i < q.rv ? v[2 * i] : 0.f;
+                                const float x1 = 16 * c + 2 * i + 1 < q.rv ? v[2 * i + 1] : 0.f;
+                                split2(x0, x1, vh[8 * k + i], vl[8 * k + i]);
                             }
                         }
                     }
-                    if (o_written) {
-                        wait_bp_upto(kseg - 1);  // every back-projection of the run is done
-                        if (ok) {
-#pragma unroll 1
-                            for (int c = half; c < D / 16; c += 2) {
-                                uint32_t r[16];
-                                tc::ld16(tl + kColO + 16 * c, r);
-                                tc::wait_ld();
-#pragma unroll
-                                for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-                                tc::st16(tl + kColO + 16 * c, r);
+                    pair_sync();
+    #pragma unroll
+                    for (int k = 0; k < kNC; ++k) {
+                        const int cc = 2 * k + half;
+                        if (ok && (SP ? 2 * cc : cc) < q.nv16) {
+                            if constexpr (SP) {
+                                tc::st8x2<8>(tl + kColV + 16 * cc, vh + 8 * k);
+                                tc::st8x2<8>(tl + kColV + 64 + 16 * cc, vl + 8 * k);
+                            } else {
+                                tc::st8(tl + kColV + 8 * cc, vh + 8 * k);
+                                tc::st8(tl + kColV + 64 + 8 * cc, vl + 8 * k);
                             }
                         }
                     }
                     tc::wait_st();
-                    l *= alpha;
-                    m = mn;
-                }
-                if (first_tile) {
-                    ref = publish_ref(p, g, row, row_ok, 0, m);
-                    first_tile = false;
-                }
-                // p = 2^(s - m) of this warp's columns as bf16 hi | lo over the
-                // score tile (hi in columns [0, 32), lo in [32, 64))
-                uint32_t ph[kHalfTok / 2], pl[kHalfTok / 2];
-                uint64_t t2[kHalfTok / 2];  // pairs of p, then their pairwise sums
-                const uint64_t m2 = f2(m, m);
-#pragma unroll
-                for (int i = 0; i < kHalfTok / 2; ++i) {
-                    float d0, d1;
-                    f2get(f2sub(f2(sv[2 * i], sv[2 * i + 1]), m2), d0, d1);
-                    const float p0 = ex2_approx(d0), p1 = ex2_approx(d1);  // masked: 0
-                    t2[i] = f2(p0, p1);
-                    split2(p0, p1, ph[i], pl[i]);
-                }
-#pragma unroll
-                for (int w = kHalfTok / 4; w >= 1; w /= 2)
-#pragma unroll
-                    for (int i = 0; i < w; ++i) t2[i] = f2add(t2[i], t2[i + w]);
-                {
-                    float a, c;
-                    f2get(t2[0], a, c);
-                    l += a + c;
-                }
-                tc::st16(sb + (kHalfTok / 2) * half, ph);
-                tc::st16(sb + kTcTok / 2 + (kHalfTok / 2) * half, pl);
-                tc::wait_st();
-                tc::fence_before();
-                arrive(TB_PREADY + b);
-            }
-            // the next segment's q~ (its projection went ahead), then this
-            // segment's v~ as the back-projection's hi and lo A operands, in
-            // place in tensor memory (hi at +0, lo at +64; ranks past the
-            // rank: zero): both warps of the pair read their chunks before
-            // either writes
-            if (s + 1 < s_end) prepare(s + 1, w.next, w.after);
-            wwait(TB_VDONE, kseg);
-            if (q.rv > 0) {
-                // (the pair barrier runs in both warps whatever ok says)
-                uint32_t vh[D / 4], vl[D / 4];
-#pragma unroll
-                for (int k = 0; k < D / 32; ++k) {
-                    const int c = 2 * k + half;
-                    if (ok && c < q.nv16) {
-                        float v[16];
-                        tc::ld16f(tl + kColV + 16 * c, v);
-                        tc::wait_ld();
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            const float x0 = 16 * c + 2 * i < q.rv ? v[2 * i] : 0.f;
-                            const float x1 = 16 * c + 2 * i + 1 < q.rv ? v[2 * i + 1] : 0.f;
-                            split2(x0, x1, vh[8 * k + i], vl[8 * k + i]);
-                        }
-                    }
-                }
-                pair_sync();
-#pragma unroll
-                for (int k = 0; k < D / 32; ++k) {
-                    const int c = 2 * k + half;
-                    if (ok && c < q.nv16) {
-                        tc::st8(tl + kColV + 8 * c, vh + 8 * k);
-                        tc::st8(tl + kColV + 64 + 8 * c, vl + 8 * k);
-                    }
-                }
-                tc::wait_st();
-            }
-            tc::fence_before();
-            // the previous segment's back-projection is done before this
-            // one's can be (the phase order of its barrier)
-            wait_bp_upto(kseg - 1);
-            arrive(TB_VSTAGED);
-            if (q.rv > 0) o_written = true;
-            if (q.last_of_run) {
-                wait_bp_upto(kseg);
-                // ---- the run's result into the accumulators of KV head g
-                // (or, for a row group with an outlier maximum, as a record);
-                // the pair adds its row sums, each warp its half of O
-                float *xl = xch + 2 * 4 * 2 * 32 + quad * 32;
-                if (half == 1) xl[lane] = l;
-                pair_sync();
-                const float lsum = half == 0 ? l + xl[lane] : 0.f;  // used by half 0
-                const float Mref = ref ? ref_dec(ref) : m;
-                const bool outlier = row_ok && m - Mref > kDirectMax;
-                const uint32_t votes = __ballot_sync(0xffffffffu, outlier);
-                const bool direct = ((votes >> (lane & ~7)) & 0xffu) == 0u;
-                const int rgg = row >> 3;
-                const int64_t rec_idx = (int64_t)q.slot * p.nrg + rgg;
-                float *rec = p.rec + rec_idx * (8 * D + kRecFloatsExtra);
-                const float f = row_ok && direct ? ex2_approx(m - Mref) : 0.f;
-                float *arow = p.acc_o + ((int64_t)g * p.rows_max + row) * D;
-                if (ok) {
-#pragma unroll 1
-                    for (int c = half; c < D / 16; c += 2) {
-                        float o[16];
-                        if (o_written) {
-                            tc::ld16f(tl + kColO + 16 * c, o);
-                            tc::wait_ld();
-                        } else {
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) o[i] = 0.f;
-                        }
-                        if (!row_ok) continue;
-                        if (direct) {
-#pragma unroll
-                            for (int i = 0; i < 16; i += 4)
-                                atomicAdd(reinterpret_cast<float4 *>(arow + 16 * c + i),
-                                          make_float4(f * o[i], f * o[i + 1], f * o[i + 2], f * o[i + 3]));
-                        } else {
-#pragma unroll
-                            for (int i = 0; i < 16; i += 4)
-                                __stcg(reinterpret_cast<float4 *>(rec + r8 * D + 16 * c + i),
-                                       make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
-                        }
-                    }
-                    if (row_ok && half == 0) {
-                        if (direct) {
-                            atomicAdd(p.acc_l + (int64_t)g * p.rows_max + row, f * lsum);
-                        } else {
-                            __stcg(rec + 8 * D + r8, m);
-                            __stcg(rec + 8 * D + 8 + r8, lsum);
-                        }
-                    }
-                    // one lane per row group lists an outlier record
-                    if (!direct && half == 0 && r8 == 0 && row_ok) {
-                        const int gr = g * p.nrg + rgg;
-                        const uint32_t k = atomicAdd(p.ovf_cnt + gr, 1u);
-                        __stcg(reinterpret_cast<int4 *>(p.ovf_list) + (int64_t)gr * p.list_cap + k,
-                               make_int4((int)rec_idx, 8 * rgg, min(8, p.rows_g - 8 * rgg), 0));
-                    }
                 }
                 tc::fence_before();
+                // the previous segment's back-projection is done before this
+                // one's can be (the phase order of its barrier)
+                wait_bp_upto(kseg - 1);
+                arrive(TB_VSTAGED);
+                if (q.rv > 0) o_written = true;
+                if (q.last_of_run) {
+                    wait_bp_upto(kseg);
+                    // ---- the run's result into the accumulators of KV head g
+                    // (or, for a row group with an outlier maximum, as a record);
+                    // the pair adds its row sums, each warp its half of O
+                    float *xl = xch + 2 * 4 * 2 * 32 + quad * 32;
+                    float lw = l;
+                    if constexpr (SP) lw += __shfl_xor_sync(0xffffffffu, lw, 16);
+                    if (half == 1) xl[ts] = lw;
+                    pair_sync();
+                    const float lsum = half == 0 ? lw + xl[ts] : 0.f;  // used by half 0
+                    const float Mref = ref ? ref_dec(ref) : m;
+                    const bool outlier = row_ok && m - Mref > kDirectMax;
+                    const uint32_t votes = __ballot_sync(0xffffffffu, outlier);
+                    const bool direct = ((votes >> (ts & ~7)) & 0xffu) == 0u;  // the row's group of 8
+                    const int rgg = row >> 3;
+                    const int64_t rec_idx = (int64_t)q.slot * p.nrg + rgg;
+                    float *rec = p.rec + rec_idx * (8 * D + kRecFloatsExtra);
+                    const float f = row_ok && direct ? ex2_approx(m - Mref) : 0.f;
+                    float *arow = p.acc_o + ((int64_t)g * p.rows_max + row) * D;
+                    if (ok) {
+    #pragma unroll 1
+                        for (int cc = half; cc < (SP ? D / 32 : D / 16); cc += 2) {
+                            float o[16];
+                            const int c = SP ? 2 * cc + u : cc;  // this thread's 16 columns
+                            if (o_written) {
+                                if constexpr (SP) tc::ld16x2f<16>(tl + kColO + 32 * cc, o); else tc::ld16f(tl + kColO + 16 * cc, o);
+                                tc::wait_ld();
+                            } else {
+    #pragma unroll
+                                for (int i = 0; i < 16; ++i) o[i] = 0.f;
+                            }
+                            if (!row_ok) continue;
+                            if (direct) {
+    #pragma unroll
+                                for (int i = 0; i < 16; i += 4)
+                                    atomicAdd(reinterpret_cast<float4 *>(arow + 16 * c + i),
+                                              make_float4(f * o[i], f * o[i + 1], f * o[i + 2], f * o[i + 3]));
+                            } else {
+    #pragma unroll
+                                for (int i = 0; i < 16; i += 4)
+                                    __stcg(reinterpret_cast<float4 *>(rec + r8 * D + 16 * c + i),
+                                           make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+                            }
+                        }
+                        if (row_ok && half == 0 && u == 0) {
+                            if (direct) {
+                                atomicAdd(p.acc_l + (int64_t)g * p.rows_max + row, f * lsum);
+                            } else {
+                                __stcg(rec + 8 * D + r8, m);
+                                __stcg(rec + 8 * D + 8 + r8, lsum);
+                            }
+                        }
+                        // one lane per row group lists an outlier record
+                        if (!direct && half == 0 && u == 0 && r8 == 0 && row_ok) {
+                            const int gr = g * p.nrg + rgg;
+                            const uint32_t k = atomicAdd(p.ovf_cnt + gr, 1u);
+                            __stcg(reinterpret_cast<int4 *>(p.ovf_list) + (int64_t)gr * p.list_cap + k,
+                                   make_int4((int)rec_idx, 8 * rgg, min(8, p.rows_g - 8 * rgg), 0));
+                        }
+                    }
+                    tc::fence_before();
+                }
             }
-        }
+        };
+        if (spread) role(std::true_type{}); else role(std::false_type{});
     }
     // every MMA is done (the issuer waited for them) and every tensor-memory
     // access has completed: release the tensor memory

@@ -3,7 +3,8 @@ milo_tensor_min_rows() query rows per KV head and at most 8 query heads per
 KV head) against the fp64 oracle, through the C ABI.
 
 The cases put the row count at the path's threshold and across a 128-row
-tile boundary, and cover head dimensions 64 and 128, ragged blocks, ranks 0
+tile boundary, run calls of one tile of at most 64 rows (spread 16 per
+tensor-memory lane quarter) and fuller ones, and cover head dimensions 64 and 128, ragged blocks, ranks 0
 (K, V or both) next to full ranks, separate K and V ranks, a peaked softmax,
 late outlier scores that force the listed-record merge, calls without tails,
 shares that cross KV heads, and repeated and graph-captured calls.
@@ -68,6 +69,8 @@ CASES = {
     "g5-b16": (40, 8, 128, [512, 512], (32, 77, 128), 16, [1024 - 50 * i for i in range(16)], True),
     # many short blocks: shares hold many segments and cross KV heads
     "many-blocks": (28, 4, 128, [96] * 40, (4, 8, 16, 24, 128), 8, [0] * 8, True),
+    # head dimension 64 with 48 rows (one spread tile) and ranks up to 64
+    "d64-spread": (8, 2, 64, [300, 7, 129], (4, 16, 33, 64), 12, [(11 * i) % 90 for i in range(12)], True),
 }
 
 
@@ -83,32 +86,36 @@ def test_tensor_path_matches_oracle(env, name):
     pre.close()
 
 
-def test_tensor_path_rank0_entries(env):
+@pytest.mark.parametrize("batch", [10, 8])
+def test_tensor_path_rank0_entries(env, batch):
     """Entries of rank 0 in K and V, in K only and in V only, next to ranks 16
-    and 128, over 70 query rows per KV head."""
+    and 128, over 70 (a full tile) and 56 (a spread tile) query rows per KV
+    head."""
     W = env["W"]
     rk = np.array([[0, 16], [0, 128], [16, 0], [128, 0], [0, 0]], dtype=np.int32)
     rv = np.array([[0, 0], [128, 0], [0, 16], [0, 128], [16, 0]], dtype=np.int32)
-    layer = W.build_layer(14, 2, 128, [40, 512, 96, 300, 33], rk, rv, batch=10,
-                          tail_lengths=[17 * i for i in range(10)], seed=13, device="cuda")
+    layer = W.build_layer(14, 2, 128, [40, 512, 96, 300, 33], rk, rv, batch=batch,
+                          tail_lengths=[17 * i for i in range(batch)], seed=13, device="cuda")
     out, pre = run(env, layer)
     compare(out.cpu().numpy(), env["oracle"].attention(**layer.to_numpy_bits()), "tensor rank0")
     pre.close()
 
 
-def test_tensor_path_peaked_softmax(env):
+@pytest.mark.parametrize("batch", [10, 8])
+def test_tensor_path_peaked_softmax(env, batch):
     """q scaled by 30: scores spread over tens of log2 units, so the rows'
-    reference maxima move and V~ and O are rescaled in tensor memory."""
+    reference maxima move and V~ and O are rescaled in tensor memory (full
+    and spread tiles)."""
     layer = env["W"].make_random_case(num_q_heads=14, num_kv_heads=2, head_dim=128,
                                       block_lens=[512, 77, 512, 300], rank_choices=(16, 64, 128),
-                                      batch=10, tail_lengths=[40 * i for i in range(10)], seed=3,
+                                      batch=batch, tail_lengths=[40 * i for i in range(batch)], seed=3,
                                       device="cuda", q_scale=30.0)
     out, pre = run(env, layer)
     compare(out.cpu().numpy(), env["oracle"].attention(**layer.to_numpy_bits()), "tensor peaked")
     pre.close()
 
 
-@pytest.mark.parametrize("batch", [10, 20])
+@pytest.mark.parametrize("batch", [8, 10, 20])
 def test_tensor_path_outlier_records(env, batch):
     """Prefix tokens 300-309 of block 0 get scores 256 times larger, far above
     the reference each row took from its first tile: the runs holding them
