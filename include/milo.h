@@ -359,6 +359,20 @@ milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta,
                                    const int64_t *block_pos);
 
 /*
+ * Check of the failure reporting: one warp waits, through the bounded
+ * mbarrier wait every kernel of the library uses, on an mbarrier that nothing
+ * completes (arrive = 0) or that the warp completes first (arrive != 0), with
+ * a limit of limit_ns nanoseconds (in [1e6, 1e10]).  A wait that runs out sets
+ * MILO_ERR_TIMEOUT in the plan's status word (milo_get_device_status reads
+ * it) and the kernel returns: the failure is reported without faulting or
+ * hanging the GPU, and the context stays usable.  Asynchronous on `stream`.
+ * Errors: MILO_ERR_INVALID_ARG (null plan, limit out of range, another
+ * device current), MILO_ERR_CUDA.
+ */
+milo_status_t milo_check_bounded_wait(const milo_prefix_t *plan, int64_t limit_ns,
+                                      int32_t arrive, void *stream);
+
+/*
  * Read (and optionally clear) the plan's sticky device status word, which the
  * kernels set on a timed-out wait (MILO_ERR_TIMEOUT) or a failed device-side
  * index check (MILO_ERR_DEVICE_BOUNDS).  Synchronises `stream`.

@@ -1056,6 +1056,18 @@ milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q, 
                             softmax_scale, out, ws, kStaticWorkspaceBytes, stream);
 }
 
+milo_status_t milo_check_bounded_wait(const milo_prefix_t *plan, int64_t limit_ns, int32_t arrive, void *stream)
+{
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    if (limit_ns < 1000000 || limit_ns > 10000000000LL) return fail(MILO_ERR_INVALID_ARG, "limit_ns outside [1e6, 1e10]");
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
+    cudaError_t e = launch_wait_check(plan->status, (uint64_t)limit_ns, arrive ? 1 : 0, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "wait check launch");
+    return MILO_OK;
+}
+
 milo_status_t milo_get_device_status(const milo_prefix_t *plan, void *stream, int32_t clear, int32_t *code)
 {
     if (!plan || !code) return fail(MILO_ERR_INVALID_ARG, "null argument");

@@ -185,6 +185,9 @@ cudaError_t launch_finish(const DecodeParams &p, cudaStream_t stream);
 // of kRcRows query rows); like the tensor-core grid it sits between the tail
 // items' chunk grid and the finish grid.
 cudaError_t launch_recon(const DecodeParams &p, int num_chunks, cudaStream_t stream);
+// One warp's bounded wait on an mbarrier that nothing completes (arrive = 0)
+// or that it completes first (arrive = 1), against a status word.
+cudaError_t launch_wait_check(int32_t *status, uint64_t limit_ns, int arrive, cudaStream_t stream);
 
 // Fixed scratch of milo_attn_decode_static (a file-scope device array).
 constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;

@@ -67,8 +67,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
     return ok != 0;
 }
 
-// Bounded wait: false (and the status word set) once kTimeoutNs has passed.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status)
+// Bounded wait: false (and the status word set) once limit_ns has passed.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status,
+                                          uint64_t limit_ns = kTimeoutNs)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
@@ -76,7 +77,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t
 #pragma unroll 1
         for (int i = 0; i < 32; ++i)
             if (mbar_try_wait(bar, parity)) return true;
-        if (globaltimer() - t0 > kTimeoutNs) {
+        if (globaltimer() - t0 > limit_ns) {
             atomicCAS(status, 0, (int32_t)MILO_ERR_TIMEOUT);
             return false;
         }

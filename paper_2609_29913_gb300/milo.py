@@ -32,7 +32,7 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
            "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
            "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows",
-           "milo_attn_decode_reconstruct", "milo_prefix_set_rope"]
+           "milo_attn_decode_reconstruct", "milo_prefix_set_rope", "milo_check_bounded_wait"]
 
 PATH_NAMES = {0: "chunks", 1: "tensor", 2: "persistent"}
 
@@ -96,6 +96,7 @@ def lib():
         L.milo_attn_decode_reconstruct.argtypes = [P, P, i32, P, P, P, i64, i64, ctypes.c_float, P, P,
                                                    ctypes.c_size_t, P]
         L.milo_prefix_set_rope.argtypes = [P, ctypes.c_double, P]
+        L.milo_check_bounded_wait.argtypes = [P, i64, i32, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         L.milo_call_info.argtypes = [P, i32, i64, P]
         L.milo_tensor_min_rows.restype = i32
@@ -103,7 +104,7 @@ def lib():
                      "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
                      "milo_get_device_status", "milo_call_info", "milo_attn_decode_reconstruct",
-                     "milo_prefix_set_rope"):
+                     "milo_prefix_set_rope", "milo_check_bounded_wait"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -279,6 +280,14 @@ def milo_prefix_set_rope(plan: int, rope_theta: float, block_pos=None) -> None:
     pos = None if block_pos is None else _arr(block_pos, np.int64)
     _check(lib().milo_prefix_set_rope(plan, float(rope_theta), None if pos is None else pos.ctypes.data),
            "milo_prefix_set_rope")
+
+
+def milo_check_bounded_wait(plan: int, limit_ns: int, arrive: bool, stream=None) -> None:
+    """One warp's bounded wait on an mbarrier nothing completes (arrive=False)
+    or that it completes itself; a wait that runs out sets MILO_ERR_TIMEOUT in
+    the plan's status word."""
+    _check(lib().milo_check_bounded_wait(plan, int(limit_ns), int(bool(arrive)), _stream_ptr(stream)),
+           "milo_check_bounded_wait")
 
 
 def milo_get_device_status(plan: int, stream=None, clear: bool = False) -> int:

@@ -426,3 +426,30 @@ def test_batched_workloads_last_layer_sampled(env, name, queries, heads):
     for g in heads:
         ref = oracle_subset(env, layer, queries, g)
         compare(o[queries][:, g * G:(g + 1) * G], ref, f"{name} g{g}")
+
+
+def test_bounded_wait_runs_out_and_reports(env):
+    """The bounded mbarrier wait of the kernels, on a barrier nothing
+    completes (a 50 ms limit): the status word reads MILO_ERR_TIMEOUT, the
+    kernel ends, and the same plan then decodes correctly.  A wait on a
+    completed barrier reports nothing."""
+    milo, W = env["milo"], env["W"]
+    layer = W.make_random_case(num_q_heads=14, num_kv_heads=2, head_dim=128, block_lens=[256, 64],
+                               rank_choices=(16, 64), batch=2, tail_lengths=[10, 30], seed=5, device="cuda")
+    pre = milo.Prefix.from_layer(layer)
+    assert pre.status(clear=True) == 0
+    milo.milo_check_bounded_wait(pre.plan, 50_000_000, True)
+    assert pre.status() == 0
+    milo.milo_check_bounded_wait(pre.plan, 50_000_000, False)
+    assert pre.status(clear=True) == 6  # MILO_ERR_TIMEOUT
+    assert pre.status() == 0
+    toff = torch.as_tensor(layer.tail_offsets, device="cuda")
+    out = pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, 30)
+    torch.cuda.synchronize()
+    assert pre.status() == 0
+    ref = env["oracle"].attention(**layer.to_numpy_bits())
+    got = out.cpu().numpy().astype(np.float64)
+    assert np.abs(got - ref).max() <= 1e-2
+    with pytest.raises(milo.MiloError):
+        milo.milo_check_bounded_wait(pre.plan, 10, False)
+    pre.close()
