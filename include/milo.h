@@ -359,6 +359,72 @@ milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta,
                                    const int64_t *block_pos);
 
 /*
+ * The compression stage (Alg. 1 Stage 1) on the GPU.  For every block b and
+ * KV head g of a prefix, the SVD of its keys and of its values (Eq. 3; from
+ * the eigen-decomposition of X^T X by Jacobi rotations, fp32), the ranks of
+ * each (KV head, K) and (KV head, V) group by the greedy of Eq. 7 for the
+ * budget problem of Eq. 6 (every block first gets min(r_min, n_b, d) units,
+ * then the remaining budget goes one unit at a time to the block whose next
+ * singular value has the largest gain log(1 + sigma^2 / eps^2), ties to the
+ * lowest block index, never above min(r_max, n_b, d)), and the factors
+ * C = A Sigma (n_b x r, row-major) and P = B^T (r x d, row-major) in bf16.
+ *   num_blocks, num_kv_heads   the prefix's blocks and KV heads.
+ *   head_dim                   64 or 128.
+ *   block_len                  host [num_blocks], each in [1, 65536].
+ *   r_min, r_max               0 <= r_min <= r_max.
+ *   budget_k, budget_v         R_tot of every (KV head, K) and (KV head, V)
+ *                              group; at least sum_b min(r_min, n_b, d).
+ */
+typedef struct {
+    int32_t num_blocks;
+    int32_t num_kv_heads;
+    int32_t head_dim;
+    const int32_t *block_len;
+    int32_t r_min, r_max;
+    int64_t budget_k, budget_v;
+} milo_encode_params_t;
+
+/*
+ * The arena milo_encode fills: offsets, host [num_blocks * num_kv_heads * 4]
+ * element offsets of C^K, P^K, C^V, P^V of entry b * num_kv_heads + g (each
+ * region sized for min(r_max, n_b, d) ranks, 8-element aligned), and
+ * *arena_elems the bf16 elements it spans.  With the ranks milo_encode
+ * returns, these offsets form a milo_block_table_t.  Either output may be
+ * NULL.  Errors: MILO_ERR_INVALID_ARG, MILO_ERR_BAD_TABLE (a block length),
+ * MILO_ERR_UNSUPPORTED (head_dim).
+ */
+milo_status_t milo_encode_layout(const milo_encode_params_t *params, int64_t *offsets,
+                                 int64_t *arena_elems);
+
+/* Device workspace milo_encode needs (256-byte aligned): per key and value
+ * matrix the singular values and the d x d eigenvectors (8 d^2 + O(d) bytes
+ * per block and KV head). */
+milo_status_t milo_encode_workspace_size(const milo_encode_params_t *params, size_t *bytes);
+
+/*
+ * Compress a prefix.
+ *   k, v       device bf16 [sum n_b, num_kv_heads, head_dim] (token-major, as a
+ *              KV cache holds them; block b is tokens n_0 + .. + n_{b-1} on),
+ *              16-byte aligned.  For pre-RoPE factors pass the keys before
+ *              the rotary embedding.
+ *   arena      device bf16, at least milo_encode_layout's count, 16-byte
+ *              aligned: receives the factors at its offsets.
+ *   rank_k/v   device int32 [num_blocks * num_kv_heads]: the ranks.
+ *   sigma      device fp32 [2 * num_blocks * num_kv_heads * head_dim] or NULL:
+ *              the singular values (row 2e keys, 2e + 1 values of entry e),
+ *              non-increasing.
+ *   workspace  device, milo_encode_workspace_size bytes, 256-byte aligned.
+ * It copies its small tables to the device and waits for that copy; the
+ * three grids then run asynchronously on `stream` (not for stream capture).
+ * Errors: those of milo_encode_layout, MILO_ERR_ALIGNMENT, MILO_ERR_WORKSPACE,
+ * MILO_ERR_INVALID_ARG (a budget below the starting ranks, an arena too
+ * small, a null pointer), MILO_ERR_CUDA.
+ */
+milo_status_t milo_encode(const milo_encode_params_t *params, const void *k, const void *v,
+                          void *arena, int64_t arena_elems, int32_t *rank_k, int32_t *rank_v,
+                          float *sigma, void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * Check of the failure reporting: one warp waits, through the bounded
  * mbarrier wait every kernel of the library uses, on an mbarrier that nothing
  * completes (arrive = 0) or that the warp completes first (arrive != 0), with

@@ -1056,6 +1056,114 @@ milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q, 
                             softmax_scale, out, ws, kStaticWorkspaceBytes, stream);
 }
 
+namespace {
+// Checks of an encode request; on success the starting ranks fit both budgets.
+milo_status_t check_encode(const milo_encode_params_t *q)
+{
+    if (!q || !q->block_len) return fail(MILO_ERR_INVALID_ARG, "null encode parameters");
+    if (q->num_blocks < 1 || q->num_kv_heads < 1) return fail(MILO_ERR_INVALID_ARG, "no blocks or no KV heads");
+    if (q->head_dim != 64 && q->head_dim != 128) return fail(MILO_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
+    if (q->r_min < 0 || q->r_max < q->r_min) return fail(MILO_ERR_INVALID_ARG, "need 0 <= r_min <= r_max");
+    if ((int64_t)q->num_blocks * q->num_kv_heads * 2 > 0x7fffffff) return fail(MILO_ERR_UNSUPPORTED, "too many blocks");
+    int64_t start = 0;
+    for (int b = 0; b < q->num_blocks; ++b) {
+        const int n = q->block_len[b];
+        if (n < 1 || n > 65536) return fail(MILO_ERR_BAD_TABLE, "block length outside [1, 65536]");
+        start += std::min(q->r_min, std::min(n, q->head_dim));
+    }
+    if (q->budget_k < start || q->budget_v < start)
+        return fail(MILO_ERR_INVALID_ARG, "a budget is below the starting ranks sum(min(r_min, n_b, d))");
+    return MILO_OK;
+}
+// Workspace of an encode: block starts and lengths, the layout, the status
+// word, the singular values and the eigenvectors.
+struct EncodeWs {
+    size_t tok0, blen, offs, status, sigma, vt, total;
+};
+EncodeWs encode_ws(const milo_encode_params_t *q)
+{
+    const int64_t nb = q->num_blocks, E = nb * q->num_kv_heads, d = q->head_dim;
+    EncodeWs w;
+    size_t cur = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = cur;
+        cur = (cur + bytes + 255) / 256 * 256;
+        return at;
+    };
+    w.tok0 = take(8 * nb);
+    w.blen = take(4 * nb);
+    w.offs = take(8 * 4 * E);
+    w.status = take(16);
+    w.sigma = take(4 * 2 * E * d);
+    w.vt = take(4 * 2 * E * d * d);
+    w.total = cur;
+    return w;
+}
+}  // namespace
+
+milo_status_t milo_encode_layout(const milo_encode_params_t *params, int64_t *offsets, int64_t *arena_elems)
+{
+    milo_status_t s = check_encode(params);
+    if (s != MILO_OK) return s;
+    const int64_t n = encode_layout(params->num_blocks, params->num_kv_heads, params->head_dim, params->block_len,
+                                    params->r_max, offsets);
+    if (arena_elems) *arena_elems = n;
+    return MILO_OK;
+}
+
+milo_status_t milo_encode_workspace_size(const milo_encode_params_t *params, size_t *bytes)
+{
+    if (!bytes) return fail(MILO_ERR_INVALID_ARG, "null argument");
+    milo_status_t s = check_encode(params);
+    if (s != MILO_OK) return s;
+    *bytes = encode_ws(params).total;
+    return MILO_OK;
+}
+
+milo_status_t milo_encode(const milo_encode_params_t *params, const void *k, const void *v, void *arena,
+                          int64_t arena_elems, int32_t *rank_k, int32_t *rank_v, float *sigma, void *workspace,
+                          size_t workspace_bytes, void *stream_)
+{
+    milo_status_t s = check_encode(params);
+    if (s != MILO_OK) return s;
+    if (!k || !v || !arena || !rank_k || !rank_v || !workspace) return fail(MILO_ERR_INVALID_ARG, "null pointer");
+    if (reinterpret_cast<uintptr_t>(k) % 16 || reinterpret_cast<uintptr_t>(v) % 16 ||
+        reinterpret_cast<uintptr_t>(arena) % 16 || reinterpret_cast<uintptr_t>(workspace) % 256)
+        return fail(MILO_ERR_ALIGNMENT, "k, v and arena must be 16-byte aligned, the workspace 256-byte aligned");
+    const EncodeWs w = encode_ws(params);
+    if (workspace_bytes < w.total) return fail(MILO_ERR_WORKSPACE, "workspace too small");
+    const int nb = params->num_blocks, H = params->num_kv_heads, d = params->head_dim;
+    std::vector<int64_t> tok0((size_t)nb), offs((size_t)nb * H * 4);
+    int64_t cum = 0;
+    for (int b = 0; b < nb; ++b) {
+        tok0[(size_t)b] = cum;
+        cum += params->block_len[b];
+    }
+    if (cum * H * d > ((int64_t)1 << 40)) return fail(MILO_ERR_UNSUPPORTED, "prefix too long");
+    const int64_t need = encode_layout(nb, H, d, params->block_len, params->r_max, offs.data());
+    if (arena_elems < need) return fail(MILO_ERR_INVALID_ARG, "arena smaller than milo_encode_layout's count");
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(ws + w.tok0, tok0.data(), 8 * tok0.size(), cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(ws + w.blen, params->block_len, 4 * (size_t)nb, cudaMemcpyHostToDevice, stream)) !=
+            cudaSuccess ||
+        (e = cudaMemcpyAsync(ws + w.offs, offs.data(), 8 * offs.size(), cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
+        (e = cudaMemsetAsync(ws + w.status, 0, 16, stream)) != cudaSuccess)
+        return cuda_fail(e, "stage encode tables");
+    // (the copies read host memory that lives until this function returns:
+    // wait for them)
+    if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "synchronize encode tables");
+    float *sg = sigma ? sigma : reinterpret_cast<float *>(ws + w.sigma);
+    e = launch_encode(static_cast<const uint16_t *>(k), static_cast<const uint16_t *>(v),
+                      reinterpret_cast<const int64_t *>(ws + w.tok0), reinterpret_cast<const int32_t *>(ws + w.blen),
+                      reinterpret_cast<const int64_t *>(ws + w.offs), static_cast<uint16_t *>(arena), rank_k, rank_v, sg,
+                      reinterpret_cast<float *>(ws + w.vt), reinterpret_cast<int32_t *>(ws + w.status), nb, H, d,
+                      params->r_min, params->r_max, params->budget_k, params->budget_v, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "encode launch");
+    return MILO_OK;
+}
+
 milo_status_t milo_check_bounded_wait(const milo_prefix_t *plan, int64_t limit_ns, int32_t arrive, void *stream)
 {
     if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");

@@ -189,6 +189,16 @@ cudaError_t launch_recon(const DecodeParams &p, int num_chunks, cudaStream_t str
 // or that it completes first (arrive = 1), against a status word.
 cudaError_t launch_wait_check(int32_t *status, uint64_t limit_ns, int arrive, cudaStream_t stream);
 
+// The compression stage (milo_encode.cu): the arena layout of its output
+// (element offsets [E][4] of C^K, P^K, C^V, P^V, each region sized for
+// min(r_max, n_b, d) ranks and 8-element aligned; returns the element
+// count), and the launch of its three grids.
+int64_t encode_layout(int nb, int hkv, int d, const int32_t *blen, int r_max, int64_t *offs);
+cudaError_t launch_encode(const uint16_t *k, const uint16_t *v, const int64_t *tok0, const int32_t *blen,
+                          const int64_t *offs, uint16_t *arena, int32_t *rank_k, int32_t *rank_v, float *sigma,
+                          float *vt, int32_t *status, int nb, int hkv, int d, int r_min, int r_max,
+                          int64_t budget_k, int64_t budget_v, cudaStream_t stream);
+
 // Fixed scratch of milo_attn_decode_static (a file-scope device array).
 constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;
 // Device address of that array on the current device (looked up once per

@@ -32,7 +32,8 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
            "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
            "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows",
-           "milo_attn_decode_reconstruct", "milo_prefix_set_rope", "milo_check_bounded_wait"]
+           "milo_attn_decode_reconstruct", "milo_prefix_set_rope", "milo_check_bounded_wait",
+           "milo_encode_layout", "milo_encode_workspace_size", "milo_encode"]
 
 PATH_NAMES = {0: "chunks", 1: "tensor", 2: "persistent"}
 
@@ -56,6 +57,13 @@ class BlockTableC(ctypes.Structure):
 class CallInfoC(ctypes.Structure):
     _fields_ = [("path", ctypes.c_int32), ("kernels", ctypes.c_int32),
                 ("row_tiles", ctypes.c_int32), ("blocks", ctypes.c_int32)]
+
+
+class EncodeParamsC(ctypes.Structure):
+    _fields_ = [("num_blocks", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("block_len", ctypes.c_void_p),
+                ("r_min", ctypes.c_int32), ("r_max", ctypes.c_int32),
+                ("budget_k", ctypes.c_int64), ("budget_v", ctypes.c_int64)]
 
 
 class PrefixInfoC(ctypes.Structure):
@@ -97,6 +105,9 @@ def lib():
                                                    ctypes.c_size_t, P]
         L.milo_prefix_set_rope.argtypes = [P, ctypes.c_double, P]
         L.milo_check_bounded_wait.argtypes = [P, i64, i32, P]
+        L.milo_encode_layout.argtypes = [P, P, P]
+        L.milo_encode_workspace_size.argtypes = [P, P]
+        L.milo_encode.argtypes = [P, P, P, P, i64, P, P, P, P, ctypes.c_size_t, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         L.milo_call_info.argtypes = [P, i32, i64, P]
         L.milo_tensor_min_rows.restype = i32
@@ -104,7 +115,8 @@ def lib():
                      "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
                      "milo_get_device_status", "milo_call_info", "milo_attn_decode_reconstruct",
-                     "milo_prefix_set_rope", "milo_check_bounded_wait"):
+                     "milo_prefix_set_rope", "milo_check_bounded_wait", "milo_encode_layout",
+                     "milo_encode_workspace_size", "milo_encode"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -288,6 +300,66 @@ def milo_check_bounded_wait(plan: int, limit_ns: int, arrive: bool, stream=None)
     the plan's status word."""
     _check(lib().milo_check_bounded_wait(plan, int(limit_ns), int(bool(arrive)), _stream_ptr(stream)),
            "milo_check_bounded_wait")
+
+
+def _encode_params(block_len, num_kv_heads, head_dim, r_min, r_max, budget_k, budget_v):
+    bl = _arr(block_len, np.int32)
+    c = EncodeParamsC(int(bl.shape[0]), int(num_kv_heads), int(head_dim), bl.ctypes.data if bl.size else None,
+                      int(r_min), int(r_max), int(budget_k), int(budget_v))
+    return c, bl
+
+
+def milo_encode_layout(block_len, num_kv_heads, head_dim, r_max, r_min=0, budget_k=None, budget_v=None):
+    """Element offsets [E][4] of C^K, P^K, C^V, P^V and the element count of
+    the arena milo_encode fills."""
+    big = 1 << 62
+    c, bl = _encode_params(block_len, num_kv_heads, head_dim, r_min, r_max,
+                           big if budget_k is None else budget_k, big if budget_v is None else budget_v)
+    E = int(bl.shape[0]) * int(num_kv_heads)
+    offs = np.zeros((max(E, 1), 4), dtype=np.int64)
+    n = ctypes.c_int64(0)
+    _check(lib().milo_encode_layout(ctypes.byref(c), offs.ctypes.data, ctypes.byref(n)), "milo_encode_layout")
+    return offs[:E], int(n.value)
+
+
+def encode(k, v, block_len, *, r_min, r_max, budget_k, budget_v, stream=None):
+    """Compress a prefix on the GPU (milo_encode).  k, v: bf16 cuda tensors
+    [sum(block_len), Hkv, d].  Returns a dict: ``arena`` (bf16 cuda tensor),
+    ``rank_k``, ``rank_v`` (numpy int32 [E]), the four offset arrays,
+    ``sigma`` (fp32 cuda tensor [2E, d]) and the table arguments, ready for
+    :class:`HostTable` (``HostTable(**table_args(result))``)."""
+    import torch
+    N, hkv, d = (int(x) for x in k.shape)
+    bl = _arr(block_len, np.int32)
+    if int(bl.sum()) != N or tuple(v.shape) != tuple(k.shape):
+        raise ValueError("k, v must be [sum(block_len), Hkv, d]")
+    c, bl = _encode_params(bl, hkv, d, r_min, r_max, budget_k, budget_v)
+    E = int(bl.shape[0]) * hkv
+    offs, n = milo_encode_layout(bl, hkv, d, r_max, r_min, budget_k, budget_v)
+    wsb = ctypes.c_size_t(0)
+    L = lib()
+    _check(L.milo_encode_workspace_size(ctypes.byref(c), ctypes.byref(wsb)), "milo_encode_workspace_size")
+    dev = k.device
+    arena = torch.zeros(max(n, 8), dtype=torch.bfloat16, device=dev)
+    ranks = torch.zeros((2, max(E, 1)), dtype=torch.int32, device=dev)
+    sigma = torch.zeros((2 * E, d), dtype=torch.float32, device=dev)
+    ws = torch.empty(int(wsb.value) + 256, dtype=torch.uint8, device=dev)
+    wp = (ws.data_ptr() + 255) // 256 * 256
+    _check(L.milo_encode(ctypes.byref(c), k.data_ptr(), v.data_ptr(), arena.data_ptr(), int(arena.numel()),
+                         ranks[0].data_ptr(), ranks[1].data_ptr(), sigma.data_ptr(), wp, int(wsb.value),
+                         _stream_ptr(stream)), "milo_encode")
+    rk = ranks.cpu().numpy()
+    return dict(arena=arena, rank_k=rk[0, :E].copy(), rank_v=rk[1, :E].copy(), off_ck=offs[:, 0].copy(),
+                off_pk=offs[:, 1].copy(), off_cv=offs[:, 2].copy(), off_pv=offs[:, 3].copy(), sigma=sigma,
+                block_len=bl.copy(), num_kv_heads=hkv, head_dim=d)
+
+
+def table_args(enc: dict) -> dict:
+    """HostTable arguments of an :func:`encode` result."""
+    return dict(num_kv_heads=enc["num_kv_heads"], head_dim=enc["head_dim"], block_len=enc["block_len"],
+                rank_k=enc["rank_k"], rank_v=enc["rank_v"], off_ck=enc["off_ck"], off_pk=enc["off_pk"],
+                off_cv=enc["off_cv"], off_pv=enc["off_pv"], arena_ptr=enc["arena"].data_ptr(),
+                arena_elems=int(enc["arena"].numel()))
 
 
 def milo_get_device_status(plan: int, stream=None, clear: bool = False) -> int:

@@ -318,3 +318,42 @@ def make_random_case(*, num_q_heads, num_kv_heads, head_dim, block_lens,
                        batch=batch, tail_lengths=tail_lengths, seed=seed,
                        device=device, q_scale=q_scale, basis=basis,
                        poison_gaps=poison_gaps)
+
+
+def make_dense_kv(block_lens, num_kv_heads: int, head_dim: int, *, seed: int = 0,
+                  device="cpu", noise: float = 0.0, zero_blocks=()):
+    """Dense keys and values of a prefix, the input of the compression stage:
+    bf16 [sum(block_lens), num_kv_heads, head_dim] each (token-major, as a KV
+    cache holds them).
+
+    Recipe: for every block b and KV head g, independently for K and V,
+    X = Z diag(s) Q + noise W with Z, W standard Gaussian [n_b, d], s_j =
+    j^(-1/2) (variance 1/j, the decay law of the factor workloads) and Q an
+    orthonormal d x d matrix (drawn and factorised on the host), so that X's
+    singular values decay like sqrt(n_b / j).  Blocks listed in
+    ``zero_blocks`` are all zeros (every singular value 0)."""
+    bl = np.asarray(block_lens, dtype=np.int64).reshape(-1)
+    nb, hk, d = int(bl.shape[0]), int(num_kv_heads), int(head_dim)
+    gen = _torch_gen(device, seed, 7777)
+    gen_cpu = _torch_gen("cpu", seed + 104_729, 7777)
+    N = int(bl.sum())
+    out = []
+    s = torch.arange(1, d + 1, dtype=torch.float32, device=device).rsqrt()
+    for _side in range(2):
+        X = torch.empty((N, hk, d), dtype=torch.float32, device=device)
+        Q = _orthonormal_rows(nb * hk, d, d, gen_cpu, device)  # [nb * hk, d, d]
+        t0 = 0
+        for b in range(nb):
+            n = int(bl[b])
+            for g in range(hk):
+                if b in zero_blocks:
+                    X[t0:t0 + n, g] = 0.0
+                    continue
+                Z = torch.randn((n, d), generator=gen, device=device)
+                x = (Z * s) @ Q[b * hk + g]
+                if noise:
+                    x = x + noise * torch.randn((n, d), generator=gen, device=device)
+                X[t0:t0 + n, g] = x
+            t0 += n
+        out.append(X.to(torch.bfloat16))
+    return out[0], out[1]

@@ -257,3 +257,27 @@ def test_calls_without_a_plan_fail_on_the_host(milo):
     assert L.milo_get_device_status(None, None, 0, ctypes.byref(code)) == 1
     info = milo.PrefixInfoC()
     assert L.milo_prefix_get_info(None, ctypes.byref(info)) == 1
+
+
+def test_encode_layout_host(milo):
+    """The compression stage's arena layout (host only): regions sized for
+    min(r_max, n_b, d) ranks, 8-element aligned, in entry order, disjoint;
+    the error cases."""
+    bl = [512, 7, 130]
+    offs, n = milo.milo_encode_layout(bl, 2, 128, r_max=96)
+    assert offs.shape == (6, 4)
+    cur = 0
+    for b, nb in enumerate(bl):
+        cap = min(96, nb, 128)
+        for g in range(2):
+            e = b * 2 + g
+            for f, size in enumerate((nb * cap, cap * 128, nb * cap, cap * 128)):
+                assert offs[e, f] == cur and offs[e, f] % 8 == 0
+                cur += (size + 7) // 8 * 8
+    assert n == cur
+    with pytest.raises(milo.MiloError):
+        milo.milo_encode_layout(bl, 2, 96, r_max=8)            # head_dim
+    with pytest.raises(milo.MiloError):
+        milo.milo_encode_layout([0, 4], 1, 64, r_max=8)        # empty block
+    with pytest.raises(milo.MiloError):
+        milo.milo_encode_layout(bl, 1, 64, r_max=8, r_min=9)   # r_min > r_max
