@@ -155,10 +155,16 @@ __global__ void __launch_bounds__(kEncThreads, 1) spectrum_kernel(const EncParam
                 for (int c = 0; c < T; ++c) acc[a][c] = fmaf(xa[a], xb[c], acc[a][c]);
         }
     }
+    // G, and a copy of it in this matrix's eigenvector slot (the eigenvalues
+    // are read off at the end as Rayleigh quotients against it)
+    float *g0 = p.vt + (int64_t)m * D * D;
 #pragma unroll
     for (int a = 0; a < T; ++a)
 #pragma unroll
-        for (int c = 0; c < T; ++c) G[(T * ti + a) * L::kLd + T * tj + c] = acc[a][c];
+        for (int c = 0; c < T; ++c) {
+            G[(T * ti + a) * L::kLd + T * tj + c] = acc[a][c];
+            g0[(T * ti + a) * D + T * tj + c] = acc[a][c];
+        }
     for (int x = tid; x < D * D; x += kEncThreads) V[(x / D) * L::kLd + x % D] = (x / D == x % D) ? 1.f : 0.f;
     __syncthreads();
 
@@ -233,33 +239,72 @@ __global__ void __launch_bounds__(kEncThreads, 1) spectrum_kernel(const EncParam
             __syncthreads();
         }
     }
-    // ---- eigenvalues (the diagonal) in descending order, ties by index:
-    // rank of each value by counting, then sigma and the eigenvector rows
+    // ---- eigenvalues: the Rayleigh quotients lambda_i = v_i^T G0 v_i / v_i^T v_i
+    // of the accumulated rotation columns against the original G (the
+    // rotated diagonal carries the rounding of every rotation, ~1e-5 of the
+    // largest eigenvalue; the quotient ~1e-7), in a fixed summation order
     int *order = reinterpret_cast<int *>(X);  // [D]: position -> eigen index
+    float *nrm = X + D;                       // [D]: v_i^T v_i
+    float *lam = X + 2 * D;                   // [D]
+    float *part = X + 3 * D;                  // [16][D]: partial quotients by row tile
     for (int i = tid; i < D; i += kEncThreads) {
-        const float li = G[i * L::kLd + i];
+        float nn = 0.f;
+        for (int r = 0; r < D; ++r) nn = fmaf(V[r * L::kLd + i], V[r * L::kLd + i], nn);
+        nrm[i] = nn;
+    }
+    {
+        // thread (ti, tj): W[a][i] = sum_b G0[a][b] V[b][i] for its T x T tile,
+        // then sum_a V[a][i] W[a][i] over its rows
+        float w[T][T];
+#pragma unroll
+        for (int a = 0; a < T; ++a)
+#pragma unroll
+            for (int c = 0; c < T; ++c) w[a][c] = 0.f;
+        for (int bb = 0; bb < D; ++bb) {
+            float ga[T], vb[T];
+#pragma unroll
+            for (int a = 0; a < T; ++a) {
+                ga[a] = g0[(T * ti + a) * D + bb];
+                vb[a] = V[bb * L::kLd + T * tj + a];
+            }
+#pragma unroll
+            for (int a = 0; a < T; ++a)
+#pragma unroll
+                for (int c = 0; c < T; ++c) w[a][c] = fmaf(ga[a], vb[c], w[a][c]);
+        }
+#pragma unroll
+        for (int c = 0; c < T; ++c) {
+            float sacc = 0.f;
+#pragma unroll
+            for (int a = 0; a < T; ++a) sacc = fmaf(V[(T * ti + a) * L::kLd + T * tj + c], w[a][c], sacc);
+            part[ti * D + T * tj + c] = sacc;
+        }
+    }
+    __syncthreads();
+    for (int i = tid; i < D; i += kEncThreads) {
+        float q = 0.f;
+        for (int t = 0; t < 16; ++t) q += part[t * D + i];
+        lam[i] = q / nrm[i];
+    }
+    __syncthreads();
+    // descending order, ties by index
+    for (int i = tid; i < D; i += kEncThreads) {
+        const float li = lam[i];
         int pos = 0;
         for (int j = 0; j < D; ++j) {
-            const float lj = G[j * L::kLd + j];
+            const float lj = lam[j];
             pos += (lj > li) || (lj == li && j < i);
         }
         order[pos] = i;
     }
     __syncthreads();
     float *sg = p.sigma + (int64_t)m * D;
-    float *vt = p.vt + (int64_t)m * D * D;
-    float *inv = X + D;  // [D]: 1 / norm of each accumulated column of V
-    for (int x = tid; x < D; x += kEncThreads) {
-        const int i = order[x];
-        sg[x] = sqrtf(fmaxf(G[i * L::kLd + i], 0.f));
-        float nn = 0.f;
-        for (int r = 0; r < D; ++r) nn = fmaf(V[r * L::kLd + i], V[r * L::kLd + i], nn);
-        inv[x] = 1.f / sqrtf(nn);
-    }
-    __syncthreads();
+    float *vt = p.vt + (int64_t)m * D * D;  // (G0 is no longer read)
+    for (int x = tid; x < D; x += kEncThreads) sg[x] = sqrtf(fmaxf(lam[order[x]], 0.f));
     for (int x = tid; x < D * D; x += kEncThreads) {
         const int j = x / D, c = x % D;  // row j of B^T = column order[j] of V, unit length
-        vt[x] = V[c * L::kLd + order[j]] * inv[j];
+        const int i = order[j];
+        vt[x] = V[c * L::kLd + i] / sqrtf(nrm[i]);
     }
 }
 
