@@ -65,6 +65,7 @@ def parse(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU baseline sample time")
     ap.add_argument("--no-recon", action="store_true",
                     help="skip timing the reconstruct-then-attend path beside the rank-space path")
+    ap.add_argument("--no-encode", action="store_true", help="skip timing the compression stage")
     return ap.parse_args(argv)
 
 
@@ -546,6 +547,68 @@ def measure_recon(cfg, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, s
     return out
 
 
+def measure_encode(cfg, W, milo, dev, reps=5, cpu_seconds=0.0):
+    """The compression stage (milo_encode, Alg. 1 Stage 1) on one layer of
+    the workload's shape: dense keys and values drawn with a decaying
+    spectrum, budgets of a mean rank of d/2 (the paper's 50% rank budget),
+    r_min 16, r_max d.  Timed end to end per call (host staging included) on
+    the device; checked against the oracle's greedy on the GPU's singular
+    values and the oracle's SVD of one block; the oracle's own compression
+    timed on a bounded sample of blocks on the host."""
+    import torch
+    bl = [cfg.block_len] * cfg.num_blocks
+    hkv, d = cfg.num_kv_heads, cfg.head_dim
+    k, v = W.make_dense_kv(bl, hkv, d, seed=cfg.seed, device=dev)
+    budget = (d // 2) * cfg.num_blocks
+    kw = dict(r_min=16, r_max=d, budget_k=budget, budget_v=budget)
+    enc = milo.encode(k, v, bl, **kw)  # warm-up
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        enc = milo.encode(k, v, bl, **kw)
+        torch.cuda.synchronize()
+        times.append(time.perf_counter() - t0)
+    ms = 1e3 * statistics.median(times)
+    tokens = int(sum(bl))
+    rec = {"ms_per_layer": ms, "value": tokens / (ms * 1e-3), "unit": "prefix tokens encoded/s (all KV heads)",
+           "matrices_per_layer": 2 * cfg.num_blocks * hkv, "mean_rank_k": float(enc["rank_k"].mean()),
+           "mean_rank_v": float(enc["rank_v"].mean()),
+           "how": "median of %d milo_encode calls on one %d x %d-token layer, %d KV heads, d %d (three grids: "
+                  "Gram + Jacobi eigen-decomposition, allocation, factors)" % (reps, cfg.num_blocks,
+                                                                                 cfg.block_len, hkv, d)}
+    from oracle import milo_oracle
+    milo_oracle.build()
+    sig = enc["sigma"].cpu().numpy().astype(np.float64)
+    gsig = [sig[2 * (b * hkv)][:min(cfg.block_len, d)] for b in range(cfg.num_blocks)]
+    want = milo_oracle.allocate_ranks(gsig, kw["r_min"], kw["r_max"], budget, 1e-6)
+    got = np.array([enc["rank_k"][b * hkv] for b in range(cfg.num_blocks)])
+    X = (k[:cfg.block_len, 0, :].float().cpu().numpy()).astype(np.float64)
+    t0 = time.perf_counter()
+    s_ref = milo_oracle.svd(X)[0]
+    t_svd = time.perf_counter() - t0
+    rec["parity_check"] = {
+        "ranks_equal_oracle_greedy_on_gpu_sigma": bool(np.array_equal(got, want)),
+        "sigma2_max_err_over_sigma1_2_block0": float(np.abs(sig[0][:len(s_ref)] ** 2 - s_ref ** 2).max() / s_ref[0] ** 2),
+        "what": "KV head 0 keys: the oracle's greedy (Eq. 7) fed the GPU's singular values gives the GPU's ranks; "
+                "block 0's singular values against the oracle's fp64 Jacobi SVD"}
+    if cpu_seconds > 0:
+        # the oracle's compression (SVD of K and V of each block, then the
+        # greedy) of as many blocks of KV head 0 as fit the time
+        Kh = k[:, 0, :].float().cpu().numpy().astype(np.float64)
+        Vh = v[:, 0, :].float().cpu().numpy().astype(np.float64)
+        nb = max(1, min(cfg.num_blocks, int(cpu_seconds / max(2 * t_svd, 1e-3))))
+        n = cfg.block_len
+        t0 = time.perf_counter()
+        milo_oracle.compress_blocks([Kh[i * n:(i + 1) * n] for i in range(nb)], [Vh[i * n:(i + 1) * n] for i in range(nb)],
+                                    R_tot_k=(d // 2) * nb, R_tot_v=(d // 2) * nb, r_min=16, r_max=d)
+        dt = time.perf_counter() - t0
+        rec["cpu_baseline"] = {"value": nb * n / dt, "unit": "prefix tokens encoded/s (one KV head)",
+                               "cores": milo_oracle.max_threads(), "kind": "oracle",
+                               "sample": f"{nb} blocks of {n} tokens of one KV head (keys and values), {dt:.1f} s"}
+    return rec
+
+
 def measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, max_tail, steps, dist, dev,
                 world, tokens):
     """The same step through the public API with host buffers: each step
@@ -658,6 +721,8 @@ def main():
             others.append(measure(other, W, milo, dev, args.steps, args.warmup, dist, rank, world,
                                   check=not args.no_check,
                                   recon=not args.no_recon and other.name in RECON_WORKLOADS))
+    if not args.no_encode and rank == 0:
+        head["encode"] = measure_encode(cfg, W, milo, dev, cpu_seconds=0.0 if args.no_cpu else 4.0)
     roof = dict(head["roofline"])
     roof["kernel"] = ", ".join(head["kernels"])
     roof["per_launch_bytes"] = head["config"]["algorithmic_bytes_per_step"] // cfg.layers
@@ -675,6 +740,7 @@ def main():
         "e2e": head["e2e"], "gpu_launches": head["gpu_launches"], "clocks": head["clocks"],
         "parity_check": head["parity_check"], "path": head["path"], "setup_s": head["setup_s"],
         "reconstruct_then_attend": head.get("reconstruct_then_attend"),
+        "encode": head.get("encode"),
         "workloads": [{k: v for k, v in o.items() if k not in ("unit",)} for o in others],
     }
     if rank == 0:
