@@ -216,7 +216,9 @@ __global__ void __launch_bounds__(kEncThreads, 1) spectrum_kernel(const EncParam
                 rot[tid] = make_float4(c, s, __int_as_float(pp), __int_as_float(qq));
             }
             __syncthreads();
-            // rows p, q of G: G <- R^T G
+            // rows p, q of G: G <- R^T G (unrolled: the updates are
+            // independent, so their shared-memory round trips overlap)
+#pragma unroll 8
             for (int x = tid; x < (D / 2) * D; x += kEncThreads) {
                 const float4 rr = rot[x / D];
                 const int col = x % D, pp = __float_as_int(rr.z), qq = __float_as_int(rr.w);
@@ -226,6 +228,7 @@ __global__ void __launch_bounds__(kEncThreads, 1) spectrum_kernel(const EncParam
             }
             __syncthreads();
             // columns p, q of G and of V: G <- G R, V <- V R
+#pragma unroll 8
             for (int x = tid; x < (D / 2) * D; x += kEncThreads) {
                 const float4 rr = rot[x / D];
                 const int row = x % D, pp = __float_as_int(rr.z), qq = __float_as_int(rr.w);
@@ -349,17 +352,18 @@ __global__ void __launch_bounds__(kEncThreads) allocate_kernel(const EncParams p
         if (tid == 0) atomicCAS(p.status, 0, (int32_t)MILO_ERR_INVALID_ARG);
         return;
     }
-    // candidates above a value (bits of a non-negative float order like the value)
+    // candidates above a value (bits of a non-negative float order like the
+    // value), over the flattened (block, j) space so that the loads are
+    // independent and coalesced
     auto count_above = [&](uint32_t bits, bool or_equal) {
         long long c = 0;
-        for (int b = 0; b < p.nb; ++b) {
+        for (int64_t x = tid; x < (int64_t)p.nb * p.d; x += kEncThreads) {
+            const int b = (int)(x / p.d), j = (int)(x % p.d);
             int r0, cap;
             group_caps(p, b, r0, cap);
-            const float *sg = p.sigma + (int64_t)(2 * (b * p.hkv + g) + side) * p.d;
-            for (int j = r0 + tid; j < cap; j += kEncThreads) {
-                const uint32_t u = __float_as_uint(sg[j]);
-                c += or_equal ? (u >= bits) : (u > bits);
-            }
+            if (j < r0 || j >= cap) continue;
+            const uint32_t u = __float_as_uint(p.sigma[(int64_t)(2 * (b * p.hkv + g) + side) * p.d + j]);
+            c += or_equal ? (u >= bits) : (u > bits);
         }
         return block_sum(c);
     };
