@@ -66,6 +66,7 @@ def parse(argv=None):
     ap.add_argument("--no-recon", action="store_true",
                     help="skip timing the reconstruct-then-attend path beside the rank-space path")
     ap.add_argument("--no-encode", action="store_true", help="skip timing the compression stage")
+    ap.add_argument("--no-offload", action="store_true", help="skip timing the offloaded prefix")
     return ap.parse_args(argv)
 
 
@@ -351,7 +352,7 @@ def time_graph(step, stream, steps, warmup, flush):
 
 
 def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, check=True,
-            e2e=False, cpu_seconds=0.0, recon=False):
+            e2e=False, cpu_seconds=0.0, recon=False, offload=False):
     """Time one workload (all its layers per step) and return its record."""
     import torch
     plans, qs, tks, tvs, toffs = [], [], [], [], []
@@ -477,6 +478,7 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
         rec["reconstruct_then_attend"] = measure_recon(cfg, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream,
                                                       steps, warmup, flush, dist, dev, world, tokens, ms_step,
                                                       check_layer, ref0)
+    offload_check = check_layer
     if check_layer is not None:
         check_layer.arena = None
     check_layer = None
@@ -487,6 +489,9 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
     if e2e:
         rec["e2e"] = measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, max_tail,
                                  steps, dist, dev, world, tokens)
+    if offload:  # (last: it moves the plans' arenas to host memory)
+        rec["offload"] = measure_offload(plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup,
+                                         dist, dev, world, tokens, ms_step, offload_check, ref0, milo)
     if cpu_seconds > 0 and rank == 0 and world == 1 and host_layers:
         rec["cpu_baseline"] = cpu_baseline(host_layers, cpu_seconds)
     for p in plans:
@@ -545,6 +550,68 @@ def measure_recon(cfg, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, s
         for p in plans:
             p.set_rope(0.0)
     return out
+
+
+def measure_offload(plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup, dist, dev, world, tokens,
+                    ms_resident, check_layer, ref0, milo=None):
+    """The same step with every layer's packed factors in pinned host memory
+    (milo_prefix_offload): layer l is copied into device buffer l % 2 on a
+    copy stream (milo_prefix_stage) while the decode stream runs layer l - 1;
+    the copy into a buffer waits for the decode two layers back.  One CUDA
+    graph per step.  The interconnect's copy rate is measured in the same run
+    (one pinned host-to-device copy of the step's bytes)."""
+    import torch
+    L = len(plans)
+    for p in plans:
+        p.offload()
+    nbytes = max(int(p.info["packed_bytes"]) for p in plans)
+    total_bytes = sum(int(p.info["packed_bytes"]) for p in plans)
+    bufs = [torch.empty(nbytes + 128, dtype=torch.uint8, device=dev) for _ in range(2)]
+    copy = torch.cuda.Stream(device=dev)
+    staged = [torch.cuda.Event() for _ in range(L)]
+    done = [torch.cuda.Event() for _ in range(L)]
+    fork = torch.cuda.Event()
+
+    def step(s):
+        fork.record(s)
+        copy.wait_event(fork)
+        for l in range(L):
+            if l >= 2:
+                copy.wait_event(done[l - 2])
+            plans[l].stage(bufs[l % 2], stream=copy)
+            staged[l].record(copy)
+            s.wait_event(staged[l])
+            plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws, stream=s)
+            done[l].record(s)
+        s.wait_stream(copy)
+
+    ms_total, _ = time_graph(step, stream, steps, warmup, None)
+    for p in plans:
+        assert p.status() == 0, "device status word set during the offloaded timing"
+    ms = max_over_ranks(ms_total / steps, dist, dev)
+    # the host-to-device copy rate of the same bytes, one copy
+    host = torch.empty(total_bytes, dtype=torch.uint8).pin_memory()
+    dst = torch.empty(total_bytes, dtype=torch.uint8, device=dev)
+    dst.copy_(host, non_blocking=True)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(3):
+        dst.copy_(host, non_blocking=True)
+    b.record()
+    torch.cuda.synchronize()
+    h2d = 3 * total_bytes / (a.elapsed_time(b) * 1e-3) / 1e9
+    achieved = total_bytes / (ms * 1e-3) / 1e9
+    rec = {"ms_per_step": ms, "value": replica_throughput(world, tokens, ms), "unit": UNIT,
+           "resident_ms_per_step": ms_resident,
+           "interconnect": {"achieved": achieved, "peak": h2d, "unit": "GB/s", "frac": achieved / h2d,
+                            "peak_source": "pinned host-to-device copy of the step's bytes, measured in this run"},
+           "gpu_launches": sum(1 for _ in plans) * steps * milo.milo_call_info(plans[0].plan, qs[0].shape[0], max_tail)["kernels"],
+           "how": "packed arenas in pinned host memory; per layer one cudaMemcpyAsync into one of two device "
+                  "buffers on a copy stream, overlapped with the previous layer's decode; one CUDA graph a step"}
+    if check_layer is not None:
+        rec["parity_check"] = parity_layer0(check_layer, outs[0], ref0)
+    return rec
 
 
 def measure_encode(cfg, W, milo, dev, reps=5, cpu_seconds=0.0):
@@ -712,7 +779,7 @@ def main():
     dev = torch.device("cuda", local)
     head = measure(cfg, W, milo, dev, args.steps, args.warmup, dist, rank, world, check=not args.no_check,
                    e2e=True, cpu_seconds=0.0 if args.no_cpu else args.cpu_seconds,
-                   recon=not args.no_recon and cfg.name in RECON_WORKLOADS)
+                   recon=not args.no_recon and cfg.name in RECON_WORKLOADS, offload=not args.no_offload)
     others = []
     if not args.only:
         for k, other in enumerate(W.CONFIGS):
@@ -741,6 +808,7 @@ def main():
         "parity_check": head["parity_check"], "path": head["path"], "setup_s": head["setup_s"],
         "reconstruct_then_attend": head.get("reconstruct_then_attend"),
         "encode": head.get("encode"),
+        "offload": head.get("offload"),
         "workloads": [{k: v for k, v in o.items() if k not in ("unit",)} for o in others],
     }
     if rank == 0:

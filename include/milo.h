@@ -194,7 +194,8 @@ typedef struct {
     int64_t prefix_tokens;        /* sum of block lengths                     */
     int64_t logical_factor_bytes; /* bytes of C^K,P^K,C^V,P^V at true ranks   */
     int64_t packed_bytes;         /* bytes of the packed arena (with padding) */
-    const void *packed_arena;     /* device pointer to the packed arena       */
+    const void *packed_arena;     /* device pointer to the packed arena (an   */
+                                  /* offloaded plan: the staged copy, or NULL) */
 } milo_prefix_info_t;
 
 milo_status_t milo_prefix_get_info(const milo_prefix_t *plan,
@@ -357,6 +358,27 @@ milo_status_t milo_attn_decode_reconstruct(const milo_prefix_t *plan, const void
  */
 milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta,
                                    const int64_t *block_pos);
+
+/*
+ * The offloaded prefix (the paper's throughput setting: factors held in CPU
+ * memory and brought to the GPU per step).  milo_prefix_offload moves the
+ * plan's packed arena to pinned host memory (on GB300: Grace memory, read
+ * over NVLink-C2C) and frees its device copy; it synchronises the device.
+ * milo_prefix_stage then enqueues, on `stream`, the copy of that arena into a
+ * caller-owned device buffer (at least milo_prefix_get_info's packed_bytes,
+ * 128-byte aligned) and points the plan at it: the plan's decode calls from
+ * then on read that buffer, which must hold the copy until they are done
+ * (order them after the copy: the same stream, or an event).  Two buffers
+ * let the copy of the next layer overlap the decode of this one.  A decode
+ * call on an offloaded plan that was never staged returns
+ * MILO_ERR_INVALID_ARG.  Staging is an ordinary asynchronous copy and can be
+ * captured in a CUDA graph.  Errors: MILO_ERR_INVALID_ARG (null arguments,
+ * a plan not (or already) offloaded, a buffer too small, another device
+ * current), MILO_ERR_ALIGNMENT, MILO_ERR_CUDA.
+ */
+milo_status_t milo_prefix_offload(milo_prefix_t *plan);
+milo_status_t milo_prefix_stage(milo_prefix_t *plan, void *device_buffer, size_t bytes,
+                                void *stream);
 
 /*
  * The compression stage (Alg. 1 Stage 1) on the GPU.  For every block b and

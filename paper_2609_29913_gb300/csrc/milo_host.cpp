@@ -301,7 +301,8 @@ struct milo_prefix {
     int nb = 0, hkv = 0, hq = 0, d = 0, G = 0, max_batch = 0;
     int num_ctas = 0, num_segments = 0, num_slots = 0, max_nrg = 0;
     int64_t prefix_tokens = 0, logical_bytes = 0, packed_bytes = 0;
-    uint8_t *packed = nullptr;
+    uint8_t *packed = nullptr;        // the arena the kernels read (an offloaded plan: the staged copy)
+    uint8_t *packed_host = nullptr;   // offloaded plans: the arena in pinned host memory
     EntryDev *entries = nullptr;
     SegDev *segs = nullptr;
     int32_t *cta_seg_begin = nullptr;
@@ -432,7 +433,8 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaGetDevice(&cur);
     cudaSetDevice(plan->device);
     cudaDeviceSynchronize();
-    cudaFree(plan->packed);
+    if (plan->packed_host) cudaFreeHost(plan->packed_host);  // (a staged copy belongs to the caller)
+    else cudaFree(plan->packed);
     cudaFree(plan->entries);
     cudaFree(plan->segs);
     cudaFree(plan->cta_seg_begin);
@@ -753,6 +755,7 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
     if (!plan || !q || !out) return fail(MILO_ERR_INVALID_ARG, "null plan, q or out");
     if (!recon && plan->rope_tile)
         return fail(MILO_ERR_UNSUPPORTED, "the plan holds pre-RoPE factors: use milo_attn_decode_reconstruct");
+    if (!plan->packed) return fail(MILO_ERR_INVALID_ARG, "the plan's arena is offloaded: stage it first (milo_prefix_stage)");
     if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
     if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
     if (plan->nb == 0 && max_tail_tokens == 0) return fail(MILO_ERR_INVALID_ARG, "no prefix and no tail");
@@ -1161,6 +1164,45 @@ milo_status_t milo_encode(const milo_encode_params_t *params, const void *k, con
                       reinterpret_cast<float *>(ws + w.vt), reinterpret_cast<int32_t *>(ws + w.status), nb, H, d,
                       params->r_min, params->r_max, params->budget_k, params->budget_v, stream);
     if (e != cudaSuccess) return cuda_fail(e, "encode launch");
+    return MILO_OK;
+}
+
+milo_status_t milo_prefix_offload(milo_prefix_t *plan)
+{
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    if (plan->packed_host) return fail(MILO_ERR_INVALID_ARG, "the plan is already offloaded");
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "synchronize before offloading");
+    const size_t bytes = (size_t)std::max<int64_t>(plan->packed_bytes, 128);
+    uint8_t *host = nullptr;
+    if ((e = cudaHostAlloc(reinterpret_cast<void **>(&host), bytes, cudaHostAllocDefault)) != cudaSuccess)
+        return cuda_fail(e, "cudaHostAlloc for the offloaded arena");
+    if ((e = cudaMemcpy(host, plan->packed, bytes, cudaMemcpyDeviceToHost)) != cudaSuccess) {
+        cudaFreeHost(host);
+        return cuda_fail(e, "copy the arena to host memory");
+    }
+    cudaFree(plan->packed);
+    plan->packed = nullptr;
+    plan->packed_host = host;
+    return MILO_OK;
+}
+
+milo_status_t milo_prefix_stage(milo_prefix_t *plan, void *device_buffer, size_t bytes, void *stream)
+{
+    if (!plan || !device_buffer) return fail(MILO_ERR_INVALID_ARG, "null plan or buffer");
+    if (!plan->packed_host) return fail(MILO_ERR_INVALID_ARG, "the plan is not offloaded");
+    if ((int64_t)bytes < plan->packed_bytes) return fail(MILO_ERR_INVALID_ARG, "staging buffer smaller than the arena");
+    if (reinterpret_cast<uintptr_t>(device_buffer) % 128) return fail(MILO_ERR_ALIGNMENT, "staging buffer not 128-byte aligned");
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
+    cudaError_t e = cudaMemcpyAsync(device_buffer, plan->packed_host, (size_t)plan->packed_bytes, cudaMemcpyHostToDevice,
+                                    static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "stage the arena");
+    plan->packed = static_cast<uint8_t *>(device_buffer);
     return MILO_OK;
 }
 

@@ -33,7 +33,8 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
            "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows",
            "milo_attn_decode_reconstruct", "milo_prefix_set_rope", "milo_check_bounded_wait",
-           "milo_encode_layout", "milo_encode_workspace_size", "milo_encode"]
+           "milo_encode_layout", "milo_encode_workspace_size", "milo_encode",
+           "milo_prefix_offload", "milo_prefix_stage"]
 
 PATH_NAMES = {0: "chunks", 1: "tensor", 2: "persistent"}
 
@@ -108,6 +109,8 @@ def lib():
         L.milo_encode_layout.argtypes = [P, P, P]
         L.milo_encode_workspace_size.argtypes = [P, P]
         L.milo_encode.argtypes = [P, P, P, P, i64, P, P, P, P, ctypes.c_size_t, P]
+        L.milo_prefix_offload.argtypes = [P]
+        L.milo_prefix_stage.argtypes = [P, P, ctypes.c_size_t, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         L.milo_call_info.argtypes = [P, i32, i64, P]
         L.milo_tensor_min_rows.restype = i32
@@ -116,7 +119,7 @@ def lib():
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
                      "milo_get_device_status", "milo_call_info", "milo_attn_decode_reconstruct",
                      "milo_prefix_set_rope", "milo_check_bounded_wait", "milo_encode_layout",
-                     "milo_encode_workspace_size", "milo_encode"):
+                     "milo_encode_workspace_size", "milo_encode", "milo_prefix_offload", "milo_prefix_stage"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -432,6 +435,18 @@ class Prefix:
             for t in made:
                 t.record_stream(stream)
         return out
+
+    def offload(self) -> None:
+        """Move the packed arena to pinned host memory (milo_prefix_offload)."""
+        _check(lib().milo_prefix_offload(self.plan), "milo_prefix_offload")
+        self.info = milo_prefix_get_info(self.plan)
+
+    def stage(self, buffer, stream=None) -> None:
+        """Enqueue the copy of the offloaded arena into ``buffer`` (a cuda
+        uint8 tensor of at least info['packed_bytes'] bytes) on ``stream``;
+        the following decode calls read it there."""
+        _check(lib().milo_prefix_stage(self.plan, buffer.data_ptr(), buffer.numel() * buffer.element_size(),
+                                       _stream_ptr(stream)), "milo_prefix_stage")
 
     def status(self, stream=None, clear=False) -> int:
         return milo_get_device_status(self.plan, stream, clear)
