@@ -360,8 +360,8 @@ milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta,
                                    const int64_t *block_pos);
 
 /*
- * The offloaded prefix (the paper's throughput setting: factors held in CPU
- * memory and brought to the GPU per step).  milo_prefix_offload moves the
+ * The offloaded prefix (the paper's throughput setting, Sec. 5.2: factors
+ * held in CPU memory and brought to the GPU per step).  milo_prefix_offload moves the
  * plan's packed arena to pinned host memory (on GB300: Grace memory, read
  * over NVLink-C2C) and frees its device copy; it synchronises the device.
  * milo_prefix_stage then enqueues, on `stream`, the copy of that arena into a
@@ -379,6 +379,57 @@ milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta,
 milo_status_t milo_prefix_offload(milo_prefix_t *plan);
 milo_status_t milo_prefix_stage(milo_prefix_t *plan, void *device_buffer, size_t bytes,
                                 void *stream);
+
+/*
+ * INT8 storage of the factors (Sec. 5.3, Table 2, "MILO + INT8": asymmetric
+ * INT8 quantisation on top of the low-rank cache).  The group is one 8x8
+ * bf16 core of a packed arena (128 bytes: 8 tokens x 8 ranks of C, or 8
+ * ranks x 8 columns of P).  Per group: m = the smallest value (+0 for a
+ * zero), s = (largest - m) / 255 in fp32 rounded up to bf16, the 64 codes
+ * c = rint((x - m) * (1 / s)) clamped to [0, 255] (0 when s = 0 or 1 / s
+ * overflows fp32), and the
+ * value read back bf16(m + s c) (fp32 arithmetic, one rounding to nearest
+ * even for the sum, one to bf16).  Layout for an arena of `bytes` bytes
+ * (a multiple of 128), group g at bytes [128 g, 128 g + 128):
+ *   codes    bytes / 2 bytes; group g's 64 codes at [64 g, 64 g + 64), in
+ *            the core's element order; 8-byte aligned.
+ *   params   bytes / 32 bytes; one little-endian 32-bit word per group, the
+ *            bf16 bits of m in its low half and of s in its high half;
+ *            4-byte aligned.
+ * Stored bytes: 68 per 128-byte core (1.88x fewer than bf16).  Values must
+ * be finite with (largest - smallest) below the largest finite float.
+ *
+ * milo_quantize_int8 / milo_dequantize_int8: one stream-ordered kernel each
+ * over any packed arena, group by group (padding included: a group's zero
+ * padding takes part in its minimum and maximum, and reads back as m + s c).  The pointers are device pointers, or (dequantise's
+ * codes and params) mapped pinned host memory.  Errors: MILO_ERR_INVALID_ARG
+ * (null pointer, bytes negative or not a multiple of 128), MILO_ERR_ALIGNMENT
+ * (packed not 16-byte aligned, codes not 8, params not 4), MILO_ERR_CUDA.
+ */
+milo_status_t milo_quantize_int8(const void *packed, int64_t bytes, void *codes, void *params,
+                                 void *stream);
+milo_status_t milo_dequantize_int8(const void *codes, const void *params, int64_t bytes,
+                                   void *packed, void *stream);
+
+/*
+ * milo_prefix_quantize_int8 replaces a plan's resident bf16 arena with its
+ * INT8 form (codes then params in one allocation: device memory when
+ * to_host = 0, mapped pinned host memory when to_host = 1, the offloaded
+ * INT8 prefix) and frees the bf16 arena; it synchronises the device.  The
+ * plan's decode calls then need milo_prefix_stage: for an INT8 plan it
+ * enqueues on `stream` one kernel that reads the codes (over NVLink-C2C for
+ * host storage) and writes the bf16 values read back, with every factor's
+ * padding (ranks past r, tokens past n_b) set to 0, into the caller's
+ * buffer (as for an offloaded plan: at least packed_bytes, 128-byte
+ * aligned, held until the decode calls that read it are done).  Decode
+ * calls then compute attention over those values.  milo_prefix_storage_bytes
+ * gives the bytes the plan's arena occupies at rest (bf16 or INT8, wherever
+ * it is).  Errors: MILO_ERR_INVALID_ARG (null plan, the plan already
+ * offloaded or quantised, another device current), MILO_ERR_CUDA.
+ */
+milo_status_t milo_prefix_quantize_int8(milo_prefix_t *plan, int32_t to_host);
+milo_status_t milo_prefix_storage_bytes(const milo_prefix_t *plan, int64_t *bytes,
+                                        int32_t *int8, int32_t *on_host);
 
 /*
  * The compression stage (Alg. 1 Stage 1) on the GPU.  For every block b and

@@ -303,6 +303,11 @@ struct milo_prefix {
     int64_t prefix_tokens = 0, logical_bytes = 0, packed_bytes = 0;
     uint8_t *packed = nullptr;        // the arena the kernels read (an offloaded plan: the staged copy)
     uint8_t *packed_host = nullptr;   // offloaded plans: the arena in pinned host memory
+    // INT8 plans (milo_prefix_quantize_int8): codes then parameters in one
+    // allocation, device memory or mapped pinned host memory
+    uint8_t *int8_store = nullptr;    // the allocation (cudaFree / cudaFreeHost)
+    const uint8_t *int8_dev = nullptr;  // its address as the kernels see it
+    bool int8_host = false;
     EntryDev *entries = nullptr;
     SegDev *segs = nullptr;
     int32_t *cta_seg_begin = nullptr;
@@ -433,8 +438,12 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
     cudaGetDevice(&cur);
     cudaSetDevice(plan->device);
     cudaDeviceSynchronize();
-    if (plan->packed_host) cudaFreeHost(plan->packed_host);  // (a staged copy belongs to the caller)
-    else cudaFree(plan->packed);
+    // (a staged copy belongs to the caller)
+    if (plan->packed_host) cudaFreeHost(plan->packed_host);
+    else if (plan->int8_store) {
+        if (plan->int8_host) cudaFreeHost(plan->int8_store);
+        else cudaFree(plan->int8_store);
+    } else cudaFree(plan->packed);
     cudaFree(plan->entries);
     cudaFree(plan->segs);
     cudaFree(plan->cta_seg_begin);
@@ -1171,6 +1180,7 @@ milo_status_t milo_prefix_offload(milo_prefix_t *plan)
 {
     if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
     if (plan->packed_host) return fail(MILO_ERR_INVALID_ARG, "the plan is already offloaded");
+    if (plan->int8_store) return fail(MILO_ERR_INVALID_ARG, "the plan's arena is held as INT8");
     int cur = -1;
     cudaGetDevice(&cur);
     if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
@@ -1193,16 +1203,107 @@ milo_status_t milo_prefix_offload(milo_prefix_t *plan)
 milo_status_t milo_prefix_stage(milo_prefix_t *plan, void *device_buffer, size_t bytes, void *stream)
 {
     if (!plan || !device_buffer) return fail(MILO_ERR_INVALID_ARG, "null plan or buffer");
-    if (!plan->packed_host) return fail(MILO_ERR_INVALID_ARG, "the plan is not offloaded");
+    if (!plan->packed_host && !plan->int8_store) return fail(MILO_ERR_INVALID_ARG, "the plan is not offloaded");
     if ((int64_t)bytes < plan->packed_bytes) return fail(MILO_ERR_INVALID_ARG, "staging buffer smaller than the arena");
     if (reinterpret_cast<uintptr_t>(device_buffer) % 128) return fail(MILO_ERR_ALIGNMENT, "staging buffer not 128-byte aligned");
     int cur = -1;
     cudaGetDevice(&cur);
     if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
-    cudaError_t e = cudaMemcpyAsync(device_buffer, plan->packed_host, (size_t)plan->packed_bytes, cudaMemcpyHostToDevice,
-                                    static_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return cuda_fail(e, "stage the arena");
+    cudaError_t e;
+    if (plan->int8_store) {
+        const uint8_t *codes = plan->int8_dev;
+        e = launch_dequant_plan_int8(plan->entries, plan->nb * plan->hkv, plan->d, codes, codes + plan->packed_bytes / 2,
+                                     device_buffer, static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "stage the INT8 arena");
+    } else {
+        e = cudaMemcpyAsync(device_buffer, plan->packed_host, (size_t)plan->packed_bytes, cudaMemcpyHostToDevice,
+                            static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "stage the arena");
+    }
     plan->packed = static_cast<uint8_t *>(device_buffer);
+    return MILO_OK;
+}
+
+namespace {
+milo_status_t check_int8_args(const void *a, const void *b, const void *c, int64_t bytes)
+{
+    if (!a || !b || !c) return fail(MILO_ERR_INVALID_ARG, "null pointer");
+    if (bytes < 0 || bytes % 128) return fail(MILO_ERR_INVALID_ARG, "bytes negative or not a multiple of 128");
+    return MILO_OK;
+}
+}  // namespace
+
+milo_status_t milo_quantize_int8(const void *packed, int64_t bytes, void *codes, void *params, void *stream)
+{
+    milo_status_t s = check_int8_args(packed, codes, params, bytes);
+    if (s != MILO_OK) return s;
+    if (reinterpret_cast<uintptr_t>(packed) % 16 || reinterpret_cast<uintptr_t>(codes) % 8 ||
+        reinterpret_cast<uintptr_t>(params) % 4)
+        return fail(MILO_ERR_ALIGNMENT, "packed not 16-byte, codes not 8-byte or params not 4-byte aligned");
+    cudaError_t e = launch_quant_int8(packed, bytes / 128, codes, params, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? MILO_OK : cuda_fail(e, "quantise launch");
+}
+
+milo_status_t milo_dequantize_int8(const void *codes, const void *params, int64_t bytes, void *packed, void *stream)
+{
+    milo_status_t s = check_int8_args(codes, params, packed, bytes);
+    if (s != MILO_OK) return s;
+    if (reinterpret_cast<uintptr_t>(packed) % 16 || reinterpret_cast<uintptr_t>(codes) % 8 ||
+        reinterpret_cast<uintptr_t>(params) % 4)
+        return fail(MILO_ERR_ALIGNMENT, "packed not 16-byte, codes not 8-byte or params not 4-byte aligned");
+    cudaError_t e = launch_dequant_int8(codes, params, bytes / 128, packed, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? MILO_OK : cuda_fail(e, "dequantise launch");
+}
+
+milo_status_t milo_prefix_quantize_int8(milo_prefix_t *plan, int32_t to_host)
+{
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    if (plan->packed_host) return fail(MILO_ERR_INVALID_ARG, "the plan is offloaded");
+    if (plan->int8_store) return fail(MILO_ERR_INVALID_ARG, "the plan is already held as INT8");
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "synchronize before quantising");
+    const int64_t nbytes = plan->packed_bytes;
+    const size_t store = (size_t)std::max<int64_t>(nbytes / 2 + nbytes / 32, 128);
+    uint8_t *mem = nullptr;
+    void *dev = nullptr;
+    if (to_host) {
+        if ((e = cudaHostAlloc(reinterpret_cast<void **>(&mem), store, cudaHostAllocMapped)) != cudaSuccess)
+            return cuda_fail(e, "cudaHostAlloc for the INT8 arena");
+        if ((e = cudaHostGetDevicePointer(&dev, mem, 0)) != cudaSuccess) {
+            cudaFreeHost(mem);
+            return cuda_fail(e, "device address of the INT8 arena");
+        }
+    } else {
+        if ((e = cudaMalloc(reinterpret_cast<void **>(&mem), store)) != cudaSuccess)
+            return cuda_fail(e, "cudaMalloc for the INT8 arena");
+        dev = mem;
+    }
+    uint8_t *codes = static_cast<uint8_t *>(dev);
+    e = launch_quant_int8(plan->packed, nbytes / 128, codes, codes + nbytes / 2, nullptr);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        if (to_host) cudaFreeHost(mem);
+        else cudaFree(mem);
+        return cuda_fail(e, "quantise the arena");
+    }
+    cudaFree(plan->packed);
+    plan->packed = nullptr;
+    plan->int8_store = mem;
+    plan->int8_dev = codes;
+    plan->int8_host = to_host != 0;
+    return MILO_OK;
+}
+
+milo_status_t milo_prefix_storage_bytes(const milo_prefix_t *plan, int64_t *bytes, int32_t *int8, int32_t *on_host)
+{
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    const int64_t nb = plan->packed_bytes;
+    if (bytes) *bytes = plan->int8_store ? nb / 2 + nb / 32 : nb;
+    if (int8) *int8 = plan->int8_store ? 1 : 0;
+    if (on_host) *on_host = (plan->packed_host || (plan->int8_store && plan->int8_host)) ? 1 : 0;
     return MILO_OK;
 }
 

@@ -199,6 +199,15 @@ cudaError_t launch_encode(const uint16_t *k, const uint16_t *v, const int64_t *t
                           float *vt, int32_t *status, int nb, int hkv, int d, int r_min, int r_max,
                           int64_t budget_k, int64_t budget_v, cudaStream_t stream);
 
+// INT8 storage of a packed arena (milo_int8.cu): `groups` 128-byte cores,
+// 64 codes and one parameter word each.
+cudaError_t launch_quant_int8(const void *packed, int64_t groups, void *codes, void *params, cudaStream_t stream);
+cudaError_t launch_dequant_int8(const void *codes, const void *params, int64_t groups, void *packed,
+                                cudaStream_t stream);
+// The same for a plan's arena, with the padding of every factor read back as 0.
+cudaError_t launch_dequant_plan_int8(const EntryDev *entries, int num_entries, int head_dim, const void *codes,
+                                     const void *params, void *packed, cudaStream_t stream);
+
 // Fixed scratch of milo_attn_decode_static (a file-scope device array).
 constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;
 // Device address of that array on the current device (looked up once per

@@ -34,7 +34,8 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows",
            "milo_attn_decode_reconstruct", "milo_prefix_set_rope", "milo_check_bounded_wait",
            "milo_encode_layout", "milo_encode_workspace_size", "milo_encode",
-           "milo_prefix_offload", "milo_prefix_stage"]
+           "milo_prefix_offload", "milo_prefix_stage", "milo_quantize_int8", "milo_dequantize_int8",
+           "milo_prefix_quantize_int8", "milo_prefix_storage_bytes"]
 
 PATH_NAMES = {0: "chunks", 1: "tensor", 2: "persistent"}
 
@@ -111,6 +112,10 @@ def lib():
         L.milo_encode.argtypes = [P, P, P, P, i64, P, P, P, P, ctypes.c_size_t, P]
         L.milo_prefix_offload.argtypes = [P]
         L.milo_prefix_stage.argtypes = [P, P, ctypes.c_size_t, P]
+        L.milo_quantize_int8.argtypes = [P, i64, P, P, P]
+        L.milo_dequantize_int8.argtypes = [P, P, i64, P, P]
+        L.milo_prefix_quantize_int8.argtypes = [P, i32]
+        L.milo_prefix_storage_bytes.argtypes = [P, P, P, P]
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         L.milo_call_info.argtypes = [P, i32, i64, P]
         L.milo_tensor_min_rows.restype = i32
@@ -119,7 +124,9 @@ def lib():
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
                      "milo_get_device_status", "milo_call_info", "milo_attn_decode_reconstruct",
                      "milo_prefix_set_rope", "milo_check_bounded_wait", "milo_encode_layout",
-                     "milo_encode_workspace_size", "milo_encode", "milo_prefix_offload", "milo_prefix_stage"):
+                     "milo_encode_workspace_size", "milo_encode", "milo_prefix_offload", "milo_prefix_stage",
+                     "milo_quantize_int8", "milo_dequantize_int8", "milo_prefix_quantize_int8",
+                     "milo_prefix_storage_bytes"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -365,6 +372,32 @@ def table_args(enc: dict) -> dict:
                 arena_elems=int(enc["arena"].numel()))
 
 
+def milo_quantize_int8(packed, codes, params, stream=None) -> None:
+    """INT8 codes and group parameters of a packed arena (cuda uint8 tensors:
+    ``packed`` of B bytes, ``codes`` of B/2, ``params`` of B/32)."""
+    nbytes = packed.numel() * packed.element_size()
+    if codes.numel() * codes.element_size() < nbytes // 2 or params.numel() * params.element_size() < nbytes // 32:
+        raise ValueError("codes or params too small")
+    _check(lib().milo_quantize_int8(packed.data_ptr(), nbytes, codes.data_ptr(), params.data_ptr(),
+                                    _stream_ptr(stream)), "milo_quantize_int8")
+
+
+def milo_dequantize_int8(codes, params, packed, stream=None) -> None:
+    """The bf16 values read back from INT8 codes into ``packed`` (B bytes)."""
+    nbytes = packed.numel() * packed.element_size()
+    if codes.numel() * codes.element_size() < nbytes // 2 or params.numel() * params.element_size() < nbytes // 32:
+        raise ValueError("codes or params too small")
+    _check(lib().milo_dequantize_int8(codes.data_ptr(), params.data_ptr(), nbytes, packed.data_ptr(),
+                                      _stream_ptr(stream)), "milo_dequantize_int8")
+
+
+def milo_prefix_storage_bytes(plan: int) -> dict:
+    b, q, h = ctypes.c_int64(0), ctypes.c_int32(0), ctypes.c_int32(0)
+    _check(lib().milo_prefix_storage_bytes(plan, ctypes.byref(b), ctypes.byref(q), ctypes.byref(h)),
+           "milo_prefix_storage_bytes")
+    return {"bytes": b.value, "int8": bool(q.value), "on_host": bool(h.value)}
+
+
 def milo_get_device_status(plan: int, stream=None, clear: bool = False) -> int:
     code = ctypes.c_int32(0)
     _check(lib().milo_get_device_status(plan, _stream_ptr(stream), int(bool(clear)),
@@ -441,10 +474,21 @@ class Prefix:
         _check(lib().milo_prefix_offload(self.plan), "milo_prefix_offload")
         self.info = milo_prefix_get_info(self.plan)
 
+    def quantize_int8(self, to_host: bool = False) -> None:
+        """Hold the arena as INT8 codes (milo_prefix_quantize_int8), in device
+        memory or, with ``to_host``, in mapped pinned host memory."""
+        _check(lib().milo_prefix_quantize_int8(self.plan, int(bool(to_host))), "milo_prefix_quantize_int8")
+        self.info = milo_prefix_get_info(self.plan)
+
+    def storage(self) -> dict:
+        """Bytes of the arena at rest, whether INT8, whether on the host."""
+        return milo_prefix_storage_bytes(self.plan)
+
     def stage(self, buffer, stream=None) -> None:
-        """Enqueue the copy of the offloaded arena into ``buffer`` (a cuda
-        uint8 tensor of at least info['packed_bytes'] bytes) on ``stream``;
-        the following decode calls read it there."""
+        """Enqueue the copy (an offloaded plan) or the dequantisation (an INT8
+        plan) of the arena into ``buffer`` (a cuda uint8 tensor of at least
+        info['packed_bytes'] bytes) on ``stream``; the following decode calls
+        read it there."""
         _check(lib().milo_prefix_stage(self.plan, buffer.data_ptr(), buffer.numel() * buffer.element_size(),
                                        _stream_ptr(stream)), "milo_prefix_stage")
 

@@ -22,7 +22,7 @@ def milo():
 def declared_functions():
     text = open(os.path.join(ROOT, "include", "milo.h")).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(milo_[a-z_]+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(milo_[a-z0-9_]+)\s*\(", text)))
 
 
 def test_exports_every_declared_symbol(milo):
@@ -281,3 +281,21 @@ def test_encode_layout_host(milo):
         milo.milo_encode_layout([0, 4], 1, 64, r_max=8)        # empty block
     with pytest.raises(milo.MiloError):
         milo.milo_encode_layout(bl, 1, 64, r_max=8, r_min=9)   # r_min > r_max
+
+
+def test_int8_entry_points_check_arguments_on_the_host(milo):
+    """The INT8 entry points reject bad arguments before any device work:
+    null pointers and partial groups (MILO_ERR_INVALID_ARG), misaligned
+    pointers (MILO_ERR_ALIGNMENT), a null plan."""
+    L = milo.lib()
+    a16, a8, a4 = 1 << 20, (1 << 20) + 8, (1 << 20) + 4   # never dereferenced: the checks fail first
+    assert L.milo_quantize_int8(None, 128, a8, a4, None) == 1
+    assert L.milo_quantize_int8(a16, 200, a8, a4, None) == 1
+    assert L.milo_quantize_int8(a16, -128, a8, a4, None) == 1
+    assert L.milo_quantize_int8(a16 + 8, 128, a8, a4, None) == 3
+    assert L.milo_quantize_int8(a16, 128, a8 + 4, a4, None) == 3
+    assert L.milo_dequantize_int8(a8, a4 + 2, 128, a16, None) == 3
+    assert L.milo_dequantize_int8(a8, a4, 128, None, None) == 1
+    assert L.milo_prefix_quantize_int8(None, 0) == 1
+    b = ctypes.c_int64(0)
+    assert L.milo_prefix_storage_bytes(None, ctypes.byref(b), None, None) == 1
