@@ -60,59 +60,70 @@ def tiles(F_bits, rows: int, cols: int) -> np.ndarray:
     return P.reshape(r8 // TILE, TILE, c8 // TILE, TILE).transpose(0, 2, 1, 3).copy()
 
 
-def quantize_group(x_bits):
-    """One group (any shape, 64 values of bf16 bits) -> (codes uint8 of the
-    same shape, m bits, s bits)."""
-    x = bf16_to_f32(x_bits).astype(np.float32)
+def quantize_groups(x_bits):
+    """Groups of 64 values (bf16 bits, shape [..., 8, 8] or [..., 64]: the
+    last axes hold one group) -> (codes uint8 of the same shape, m bits [...],
+    s bits [...])."""
+    x_bits = np.asarray(x_bits, dtype=np.uint16)
+    shape = x_bits.shape
+    lead = shape[:-2] if shape[-2:] == (TILE, TILE) else shape[:-1]
+    x = bf16_to_f32(x_bits).reshape(lead + (GROUP,)).astype(np.float32)
     zero = np.float32(0.0)
-    lo = np.float32(x.min()) + zero           # + 0 turns -0 into +0
-    hi = np.float32(x.max()) + zero
-    span = np.float32(hi - lo)
-    s_bits = f32_to_bf16_up(np.float32(span / np.float32(255.0)))
-    s = bf16_to_f32(s_bits)[()]
-    m_bits = f32_to_bf16_rne(lo)              # exact: lo is one of the bf16 values (or +0)
+    lo = (x.min(axis=-1) + zero).astype(np.float32)      # + 0 turns -0 into +0
+    hi = (x.max(axis=-1) + zero).astype(np.float32)
+    span = (hi - lo).astype(np.float32)
+    s_bits = f32_to_bf16_up((span / np.float32(255.0)).astype(np.float32))
+    s = bf16_to_f32(s_bits)
+    m_bits = f32_to_bf16_rne(lo)                          # exact: lo is one of the bf16 values (or +0)
     with np.errstate(over="ignore", divide="ignore"):
-        inv = np.float32(np.float32(1.0) / s) if s > 0 else np.float32(np.inf)
-    if not np.isfinite(inv):                  # s = 0, or 1 / s beyond fp32: every code 0
-        codes = np.zeros(x.shape, dtype=np.uint8)
-    else:
-        t = x - lo                            # fp32 subtraction
-        c = np.rint((t * inv).astype(np.float32))
-        codes = np.clip(c, 0, 255).astype(np.uint8)
-    return codes, int(m_bits), int(s_bits)
+        inv = (np.float32(1.0) / np.where(s > 0, s, np.float32(1.0))).astype(np.float32)
+    inv = np.where((s > 0) & np.isfinite(inv), inv, np.float32(0.0)).astype(np.float32)
+    # s = 0, or 1 / s beyond fp32: inv = 0 and every code 0
+    t = (x - lo[..., None]).astype(np.float32)            # fp32 subtraction
+    c = np.rint((t * inv[..., None]).astype(np.float32))  # fp32 product, nearest even
+    codes = np.clip(c, 0, 255).astype(np.uint8).reshape(shape)
+    return codes, m_bits, s_bits
+
+
+def quantize_group(x_bits):
+    """One group (64 values of bf16 bits, any shape) -> (codes uint8 of the
+    same shape, m bits, s bits)."""
+    x_bits = np.asarray(x_bits, dtype=np.uint16)
+    codes, m, s = quantize_groups(x_bits.reshape(GROUP))
+    return codes.reshape(x_bits.shape), int(m), int(s)
+
+
+def dequantize_groups(codes, m_bits, s_bits) -> np.ndarray:
+    """Codes of groups ([..., 8, 8] or [..., 64]) with their m and s bits
+    ([...]) -> bf16 bits of m + s c (fp32: s c exact, one rounding for the
+    sum; then to bf16, nearest even)."""
+    codes = np.asarray(codes, dtype=np.uint8)
+    shape = codes.shape
+    m = bf16_to_f32(np.asarray(m_bits, dtype=np.uint16))
+    s = bf16_to_f32(np.asarray(s_bits, dtype=np.uint16))
+    c = codes.reshape(m.shape + (GROUP,)).astype(np.float32)
+    prod = (s[..., None] * c).astype(np.float32)          # exact
+    return f32_to_bf16_rne((m[..., None] + prod).astype(np.float32)).reshape(shape)
 
 
 def dequantize_group(codes, m_bits: int, s_bits: int) -> np.ndarray:
-    """Codes of one group -> bf16 bits of m + s c (fp32, then bf16)."""
-    m = bf16_to_f32(np.uint16(m_bits))[()]
-    s = bf16_to_f32(np.uint16(s_bits))[()]
-    prod = np.float32(s) * np.asarray(codes, dtype=np.float32)   # exact
-    return f32_to_bf16_rne((np.float32(m) + prod).astype(np.float32))
+    """Codes of one group -> bf16 bits of m + s c."""
+    codes = np.asarray(codes, dtype=np.uint8)
+    return dequantize_groups(codes.reshape(GROUP), np.uint16(m_bits), np.uint16(s_bits)).reshape(codes.shape)
 
 
 def quantize_matrix(F_bits, rows: int, cols: int):
     """All tiles of one factor matrix.  Returns codes [R, Cg, 8, 8] uint8 and
     m, s bits [R, Cg] (R = rows8/8, Cg = cols8/8)."""
-    T = tiles(F_bits, rows, cols)
-    R, Cg = T.shape[:2]
-    codes = np.zeros(T.shape, dtype=np.uint8)
-    m = np.zeros((R, Cg), dtype=np.uint16)
-    s = np.zeros((R, Cg), dtype=np.uint16)
-    for i in range(R):
-        for j in range(Cg):
-            codes[i, j], m[i, j], s[i, j] = quantize_group(T[i, j])
-    return codes, m, s
+    return quantize_groups(tiles(F_bits, rows, cols))
 
 
 def dequantize_matrix(codes, m, s, rows: int, cols: int) -> np.ndarray:
     """Inverse of quantize_matrix up to the quantisation error: bf16 bits
     [rows, cols] (the padding dropped)."""
     R, Cg = codes.shape[:2]
-    out = np.zeros((R * TILE, Cg * TILE), dtype=np.uint16)
-    for i in range(R):
-        for j in range(Cg):
-            out[TILE * i:TILE * (i + 1), TILE * j:TILE * (j + 1)] = dequantize_group(codes[i, j], m[i, j], s[i, j])
-    return out[:rows, :cols]
+    T = dequantize_groups(codes, m, s)
+    return T.transpose(0, 2, 1, 3).reshape(R * TILE, Cg * TILE)[:rows, :cols]
 
 
 def factor_shapes(*, num_kv_heads, head_dim, block_len, rank_k, rank_v, off_ck, off_pk, off_cv, off_pv):

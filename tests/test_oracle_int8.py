@@ -161,3 +161,23 @@ def test_stored_bytes_double_the_reduction():
         ntiles = b16 // 128
         assert b8 - 4 * ntiles == b16 // 2
         assert Fraction(b16, b8) == Fraction(128, 68)
+
+
+def test_matrix_form_is_the_group_rule_tile_by_tile():
+    """quantize_matrix / dequantize_matrix apply the one-group rule to every
+    tile (checked tile by tile against quantize_group / dequantize_group)."""
+    rng = np.random.default_rng(11)
+    rows, cols = 37, 21
+    F = (rng.standard_normal((rows, cols)) * np.logspace(0, -3, cols)[None, :]).astype(np.float32)
+    Fb = Q.f32_to_bf16_rne(F)
+    codes, m, s = Q.quantize_matrix(Fb, rows, cols)
+    T = Q.tiles(Fb, rows, cols)
+    back = Q.dequantize_matrix(codes, m, s, rows, cols)
+    for i in range(T.shape[0]):
+        for j in range(T.shape[1]):
+            c1, m1, s1 = Q.quantize_group(T[i, j])
+            assert np.array_equal(codes[i, j], c1) and m[i, j] == m1 and s[i, j] == s1
+            d1 = Q.dequantize_group(c1, m1, s1)
+            r0, c0 = 8 * i, 8 * j
+            blk = back[r0:r0 + 8, c0:c0 + 8]
+            assert np.array_equal(blk, d1[:blk.shape[0], :blk.shape[1]])
