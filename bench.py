@@ -67,6 +67,7 @@ def parse(argv=None):
                     help="skip timing the reconstruct-then-attend path beside the rank-space path")
     ap.add_argument("--no-encode", action="store_true", help="skip timing the compression stage")
     ap.add_argument("--no-offload", action="store_true", help="skip timing the offloaded prefix")
+    ap.add_argument("--no-int8", action="store_true", help="skip timing the INT8-stored factors")
     return ap.parse_args(argv)
 
 
@@ -352,7 +353,7 @@ def time_graph(step, stream, steps, warmup, flush):
 
 
 def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, check=True,
-            e2e=False, cpu_seconds=0.0, recon=False, offload=False):
+            e2e=False, cpu_seconds=0.0, recon=False, offload=False, int8=False):
     """Time one workload (all its layers per step) and return its record."""
     import torch
     plans, qs, tks, tvs, toffs = [], [], [], [], []
@@ -492,6 +493,14 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
     if offload:  # (last: it moves the plans' arenas to host memory)
         rec["offload"] = measure_offload(plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup,
                                          dist, dev, world, tokens, ms_step, offload_check, ref0, milo)
+    if int8:
+        for p in plans:
+            p.close()
+        plans = []
+        torch.cuda.empty_cache()
+        rec["int8"] = measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup,
+                                   dist, dev, world, tokens, ms_step, rec.get("offload"), offload_check is not None,
+                                   ref0)
     if cpu_seconds > 0 and rank == 0 and world == 1 and host_layers:
         rec["cpu_baseline"] = cpu_baseline(host_layers, cpu_seconds)
     for p in plans:
@@ -611,6 +620,110 @@ def measure_offload(plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, step
                   "buffers on a copy stream, overlapped with the previous layer's decode; one CUDA graph a step"}
     if check_layer is not None:
         rec["parity_check"] = parity_layer0(check_layer, outs[0], ref0)
+    return rec
+
+
+def measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup, dist, dev, world,
+                 tokens, ms_resident, offload_rec, check, ref0):
+    """The same step with every layer's factors held as INT8 (Sec. 5.3,
+    Table 2; milo_prefix_quantize_int8), in two placements, each on plans
+    built afresh from the same layers:
+      offloaded: codes in mapped pinned host memory; per layer one staging
+        kernel reads them over the chip-to-chip link and writes the bf16
+        read-back into device buffer l % 2 on a copy stream, overlapped with
+        the previous layer's decode (the structure of the bf16 offloaded step);
+      resident: codes in device memory, staged the same way from HBM.
+    One CUDA graph per step.  Parity: layer 0 against the oracle's attention
+    over the oracle's INT8 read-back of the same factors; the distance to the
+    bf16 result is the quantisation's effect."""
+    import torch
+    from oracle import milo_int8, milo_oracle
+    L = cfg.layers
+    rec = {"what": "MILO + INT8 (asymmetric, one bf16 minimum and step per 8x8 tile of a factor)"}
+    layer0_bits = None
+    for mode, to_host in (("offloaded", True), ("resident", False)):
+        plans = []
+        for l in range(L):
+            layer = W.make_config_layer(cfg, l, device=dev)
+            if l == 0 and check and layer0_bits is None:
+                layer0_bits = layer.to_numpy_bits()
+            pre = milo.Prefix.from_layer(layer)
+            pre.quantize_int8(to_host=to_host)
+            plans.append(pre)
+            layer.arena = None
+        torch.cuda.synchronize()
+        nbytes = max(int(p.info["packed_bytes"]) for p in plans)
+        stored = sum(p.storage()["bytes"] for p in plans)
+        bf16_bytes = sum(int(p.info["packed_bytes"]) for p in plans)
+        bufs = [torch.empty(nbytes + 128, dtype=torch.uint8, device=dev) for _ in range(2)]
+        copy = torch.cuda.Stream(device=dev)
+        staged = [torch.cuda.Event() for _ in range(L)]
+        done = [torch.cuda.Event() for _ in range(L)]
+        fork = torch.cuda.Event()
+
+        def step(s):
+            fork.record(s)
+            copy.wait_event(fork)
+            for l in range(L):
+                if l >= 2:
+                    copy.wait_event(done[l - 2])
+                plans[l].stage(bufs[l % 2], stream=copy)
+                staged[l].record(copy)
+                s.wait_event(staged[l])
+                plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws, stream=s)
+                done[l].record(s)
+            s.wait_stream(copy)
+
+        ms_total, graph = time_graph(step, stream, steps, warmup, None)
+        for p in plans:
+            assert p.status() == 0, "device status word set during the INT8 timing"
+        ms = max_over_ranks(ms_total / steps, dist, dev)
+        r = {"ms_per_step": ms, "value": replica_throughput(world, tokens, ms), "unit": UNIT,
+             "stored_bytes_per_step": stored, "bf16_bytes_per_step": bf16_bytes,
+             "gpu_launches": L * steps * (1 + milo.milo_call_info(plans[0].plan, qs[0].shape[0], max_tail)["kernels"])}
+        # the staging kernel alone: every layer staged into one buffer, on one stream
+        def stage_only(s):
+            for l in range(L):
+                plans[l].stage(bufs[0], stream=s)
+        ms_stage, _ = time_graph(stage_only, stream, max(steps // 4, 5), warmup, None)
+        ms_stage /= max(steps // 4, 5)
+        if to_host:
+            ach = stored / (ms * 1e-3) / 1e9
+            r["interconnect"] = {"achieved": ach, "peak": offload_rec["interconnect"]["peak"] if offload_rec else None,
+                                 "unit": "GB/s", "bytes": "INT8 codes and group parameters of every layer"}
+            if offload_rec:
+                r["interconnect"]["frac"] = ach / offload_rec["interconnect"]["peak"]
+                r["speedup_vs_bf16_offloaded"] = offload_rec["ms_per_step"] / ms
+            r["stage_kernel"] = {"us_per_layer": 1e3 * ms_stage / L,
+                                 "link_gbs": stored / (ms_stage * 1e-3) / 1e9,
+                                 "how": "dequant_plan_kernel reading mapped host memory, all layers back to back"}
+        else:
+            hbm = (stored + bf16_bytes) / (ms_stage * 1e-3) / 1e9
+            peak_gbs, _, peak_kind = peaks()
+            r["stage_kernel"] = {"us_per_layer": 1e3 * ms_stage / L, "achieved_gbs": hbm,
+                                 "peak_gbs": peak_gbs, "frac": hbm / peak_gbs, "peak_source": peak_kind,
+                                 "how": "dequant_plan_kernel from device memory: reads codes and parameters "
+                                        "(68 B per 128 B core), writes the bf16 core; all layers back to back"}
+            r["vs_bf16_resident"] = ms_resident / ms
+        if mode == "offloaded" and layer0_bits is not None:
+            milo_oracle.build()
+            deq, _ = milo_int8.quantize_arena(arena=layer0_bits["arena"], **{
+                k: layer0_bits[k] for k in ("num_kv_heads", "head_dim", "block_len", "rank_k", "rank_v",
+                                            "off_ck", "off_pk", "off_cv", "off_pv")})
+            bits = dict(layer0_bits, arena=deq)
+            ref_q = milo_oracle.attention(**bits)
+            pc = parity_layer0(None, outs[0], ref_q)
+            if ref0 is not None:
+                got = outs[0].double().cpu().numpy()
+                pc["rel_l2_vs_bf16_factors"] = float(np.linalg.norm(got - ref0) / np.linalg.norm(ref0))
+            pc["what"] = "against the oracle's attention over its own INT8 read-back of layer 0's factors"
+            r["parity_check"] = pc
+        rec[mode] = r
+        for p in plans:
+            p.close()
+        del plans, graph, bufs
+        torch.cuda.empty_cache()
+    rec["reduction_vs_bf16_factors"] = rec["offloaded"]["bf16_bytes_per_step"] / rec["offloaded"]["stored_bytes_per_step"]
     return rec
 
 
@@ -779,7 +892,8 @@ def main():
     dev = torch.device("cuda", local)
     head = measure(cfg, W, milo, dev, args.steps, args.warmup, dist, rank, world, check=not args.no_check,
                    e2e=True, cpu_seconds=0.0 if args.no_cpu else args.cpu_seconds,
-                   recon=not args.no_recon and cfg.name in RECON_WORKLOADS, offload=not args.no_offload)
+                   recon=not args.no_recon and cfg.name in RECON_WORKLOADS, offload=not args.no_offload,
+                   int8=not args.no_int8)
     others = []
     if not args.only:
         for k, other in enumerate(W.CONFIGS):
@@ -809,6 +923,7 @@ def main():
         "reconstruct_then_attend": head.get("reconstruct_then_attend"),
         "encode": head.get("encode"),
         "offload": head.get("offload"),
+        "int8": head.get("int8"),
         "workloads": [{k: v for k, v in o.items() if k not in ("unit",)} for o in others],
     }
     if rank == 0:

@@ -308,6 +308,7 @@ struct milo_prefix {
     uint8_t *int8_store = nullptr;    // the allocation (cudaFree / cudaFreeHost)
     const uint8_t *int8_dev = nullptr;  // its address as the kernels see it
     bool int8_host = false;
+    int64_t max_factor_groups = 0;    // the most 8x8 cores of one factor
     EntryDev *entries = nullptr;
     SegDev *segs = nullptr;
     int32_t *cta_seg_begin = nullptr;
@@ -510,6 +511,11 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         en.rk = table->rank_k[x];
         en.rv = table->rank_v[x];
         en.g = (int)(x % H);
+        {   // the most 8x8 cores of one factor (the INT8 staging grid's extent)
+            const int64_t n8 = (en.n + 7) / 8, d8 = table->head_dim / 8;
+            const int64_t k8 = (en.rk + 7) / 8, v8 = (en.rv + 7) / 8;
+            p->max_factor_groups = std::max({p->max_factor_groups, n8 * k8, n8 * v8, k8 * d8, v8 * d8});
+        }
         loffs[(size_t)x * 4 + 0] = table->off_ck[x];
         loffs[(size_t)x * 4 + 1] = table->off_pk[x];
         loffs[(size_t)x * 4 + 2] = table->off_cv[x];
@@ -1212,7 +1218,8 @@ milo_status_t milo_prefix_stage(milo_prefix_t *plan, void *device_buffer, size_t
     cudaError_t e;
     if (plan->int8_store) {
         const uint8_t *codes = plan->int8_dev;
-        e = launch_dequant_plan_int8(plan->entries, plan->nb * plan->hkv, plan->d, codes, codes + plan->packed_bytes / 2,
+        e = launch_dequant_plan_int8(plan->entries, plan->nb * plan->hkv, plan->d, plan->max_factor_groups, codes,
+                                     codes + plan->packed_bytes / 2,
                                      device_buffer, static_cast<cudaStream_t>(stream));
         if (e != cudaSuccess) return cuda_fail(e, "stage the INT8 arena");
     } else {

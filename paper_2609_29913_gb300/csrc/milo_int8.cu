@@ -113,11 +113,15 @@ __global__ void __launch_bounds__(kInt8Threads) dequant_kernel(const uint2 *__re
     if (g < groups) dst[g * 8 + row] = dequant_row(codes[g * 8 + row], params[g]);
 }
 
-// The read-back of a plan's arena: one block per factor of an entry (grid
-// E x 4: C^K, P^K, C^V, P^V), so each core knows which of its rows and
-// columns are padding (ranks past r, tokens past n) and writes 0 there
-// instead of m + s c: the staged arena then holds exactly the zero-padded
-// read-back factors the decode kernels expect.
+// The read-back of a plan's arena: blocks over (entry, factor, slice of
+// kPlanGroups cores) (grid E x 4 x slices: C^K, P^K, C^V, P^V), so each core
+// knows which of its rows and columns are padding (ranks past r, tokens past
+// n) and writes 0 there instead of m + s c: the staged arena then holds
+// exactly the zero-padded read-back factors the decode kernels expect.  Each
+// lane issues the loads of its four cores before converting any of them.
+constexpr int kPlanUnroll = 4;
+constexpr int kPlanGroups = (kInt8Threads / 8) * kPlanUnroll;   // cores per block
+
 __global__ void __launch_bounds__(kInt8Threads) dequant_plan_kernel(const EntryDev *__restrict__ entries, int head_dim,
                                                                     const uint2 *__restrict__ codes,
                                                                     const uint32_t *__restrict__ params,
@@ -127,19 +131,33 @@ __global__ void __launch_bounds__(kInt8Threads) dequant_plan_kernel(const EntryD
     const EntryDev ent = entries[blockIdx.x];
     const int r = (f < 2) ? ent.rk : ent.rv;
     const int r8 = (r + 7) & ~7;
-    if (r8 == 0) return;
-    const int64_t off = (f == 0) ? ent.off_ck : (f == 1) ? ent.off_pk : (f == 2) ? ent.off_cv : ent.off_pv;
     // C: rows = tokens (n), columns = ranks (r); P: rows = ranks (r), columns = head_dim
-    const int rows = (f & 1) ? r : ent.n;
-    const int cols = (f & 1) ? head_dim : r;
     const int cgs = ((f & 1) ? head_dim : r8) / 8;
     const int rgs = ((f & 1) ? r8 : ((ent.n + 7) & ~7)) / 8;
+    const int total = rgs * cgs;
+    const int base = blockIdx.z * kPlanGroups;
+    if (base >= total) return;
+    const int rows = (f & 1) ? r : ent.n;
+    const int cols = (f & 1) ? head_dim : r;
+    const int64_t off = (f == 0) ? ent.off_ck : (f == 1) ? ent.off_pk : (f == 2) ? ent.off_cv : ent.off_pv;
     const int64_t g0 = off / 128;
-    const int row = threadIdx.x & 7;
-    for (int t = threadIdx.x >> 3; t < rgs * cgs; t += kInt8Threads / 8) {
-        const int tr = t / cgs, tc = t % cgs;
-        const int64_t g = g0 + t;
-        uint4 v = dequant_row(codes[g * 8 + row], params[g]);
+    const int row = threadIdx.x & 7, team = threadIdx.x >> 3;
+    uint2 c[kPlanUnroll];
+    uint32_t pw[kPlanUnroll];
+#pragma unroll
+    for (int u = 0; u < kPlanUnroll; ++u) {
+        const int t = base + team + u * (kInt8Threads / 8);
+        if (t < total) {
+            c[u] = codes[(g0 + t) * 8 + row];
+            pw[u] = params[g0 + t];
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kPlanUnroll; ++u) {
+        const int t = base + team + u * (kInt8Threads / 8);
+        if (t >= total) break;
+        const int tr = t / cgs, tc = t - tr * cgs;
+        uint4 v = dequant_row(c[u], pw[u]);
         const int valid = (8 * tr + row < rows) ? min(8, cols - 8 * tc) : 0;
         if (valid < 8) {
             uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -148,7 +166,7 @@ __global__ void __launch_bounds__(kInt8Threads) dequant_plan_kernel(const EntryD
                 if (i >= valid) w[i >> 1] &= (i & 1) ? 0x0000FFFFu : 0xFFFF0000u;
             v = make_uint4(w[0], w[1], w[2], w[3]);
         }
-        dst[g * 8 + row] = v;
+        dst[(g0 + t) * 8 + row] = v;
     }
 }
 
@@ -181,11 +199,12 @@ cudaError_t launch_dequant_int8(const void *codes, const void *params, int64_t g
     return cudaGetLastError();
 }
 
-cudaError_t launch_dequant_plan_int8(const EntryDev *entries, int num_entries, int head_dim, const void *codes,
-                                     const void *params, void *packed, cudaStream_t stream)
+cudaError_t launch_dequant_plan_int8(const EntryDev *entries, int num_entries, int head_dim, int64_t max_factor_groups,
+                                     const void *codes, const void *params, void *packed, cudaStream_t stream)
 {
-    if (num_entries <= 0) return cudaSuccess;
-    dequant_plan_kernel<<<dim3(num_entries, 4), kInt8Threads, 0, stream>>>(
+    if (num_entries <= 0 || max_factor_groups <= 0) return cudaSuccess;
+    const int slices = (int)((max_factor_groups + kPlanGroups - 1) / kPlanGroups);
+    dequant_plan_kernel<<<dim3(num_entries, 4, slices), kInt8Threads, 0, stream>>>(
         entries, head_dim, static_cast<const uint2 *>(codes), static_cast<const uint32_t *>(params),
         static_cast<uint4 *>(packed));
     return cudaGetLastError();

@@ -205,8 +205,9 @@ cudaError_t launch_quant_int8(const void *packed, int64_t groups, void *codes, v
 cudaError_t launch_dequant_int8(const void *codes, const void *params, int64_t groups, void *packed,
                                 cudaStream_t stream);
 // The same for a plan's arena, with the padding of every factor read back as 0.
-cudaError_t launch_dequant_plan_int8(const EntryDev *entries, int num_entries, int head_dim, const void *codes,
-                                     const void *params, void *packed, cudaStream_t stream);
+// max_factor_groups: the most 8x8 cores of one factor (C^K, P^K, C^V or P^V).
+cudaError_t launch_dequant_plan_int8(const EntryDev *entries, int num_entries, int head_dim, int64_t max_factor_groups,
+                                     const void *codes, const void *params, void *packed, cudaStream_t stream);
 
 // Fixed scratch of milo_attn_decode_static (a file-scope device array).
 constexpr size_t kStaticWorkspaceBytes = size_t(8) << 20;
