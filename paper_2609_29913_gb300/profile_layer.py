@@ -1,7 +1,7 @@
 """Run decode calls on the first layers of a named workload, for profilers.
 
   python -m paper_2609_29913_gb300.profile_layer --workload qwen7b-1L-1M-b8 \
-      [--layers 1] [--calls 3] [--reconstruct [--rope-theta 1e6]]
+      [--layers 1] [--calls 3] [--reconstruct [--rope-theta 1e6]] [--int8 device|host]
 
 Builds the plans of layers 0 .. layers-1 of the workload (seeded synthetic
 inputs, as the benchmark draws them), then makes `calls` rounds of one
@@ -10,7 +10,10 @@ plan's device status word.  Each call launches the kernels milo_call_info
 names, so a profiler can select them by name and count (e.g. ncu -k
 regex:batch_tc -s 1 -c 1 skips the first round's launch).  With
 --reconstruct the calls go through milo_attn_decode_reconstruct (kernel
-recon_kernel), with --rope-theta over pre-RoPE factors.  It keeps the device
+recon_kernel), with --rope-theta over pre-RoPE factors.  With --int8 the
+plans hold their factors as INT8 codes (device memory or mapped host
+memory) and every call is preceded by its staging kernel
+(dequant_plan_kernel) into one device buffer.  It keeps the device
 footprint to the chosen layers, well under the full workload's.
 """
 from __future__ import annotations
@@ -28,6 +31,7 @@ def main(argv=None) -> int:
     ap.add_argument("--calls", type=int, default=3)
     ap.add_argument("--reconstruct", action="store_true")
     ap.add_argument("--rope-theta", type=float, default=0.0)
+    ap.add_argument("--int8", choices=("device", "host"), default=None)
     args = ap.parse_args(argv)
 
     import torch
@@ -44,9 +48,16 @@ def main(argv=None) -> int:
     if args.rope_theta > 0:
         for pre in plans:
             pre.set_rope(args.rope_theta)
+    buf = None
+    if args.int8:
+        for pre in plans:
+            pre.quantize_int8(to_host=args.int8 == "host")
+        buf = torch.empty(max(int(p.info["packed_bytes"]) for p in plans) + 128, dtype=torch.uint8, device="cuda")
     max_tail = max(int(np.diff(L.tail_offsets).max()) for L in layers)
     for _ in range(args.calls):
         for L, pre, toff in zip(layers, plans, toffs):
+            if buf is not None:
+                pre.stage(buf)
             (pre.decode_reconstruct if args.reconstruct else pre.decode)(L.q, L.tail_k, L.tail_v, toff, max_tail)
     torch.cuda.synchronize()
     for pre in plans:
