@@ -794,32 +794,30 @@ def measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, m
     """The same step through the public API with host buffers: each step
     copies every layer's q and tails from pinned host memory, runs the
     per-layer calls and reads every layer's output back.  The layers are cut
-    into a few segments, each a captured graph whose inputs arrive by one copy
-    on a second stream, so that later segments' copies overlap earlier
-    segments' calls."""
+    into segments, each a captured graph whose inputs arrive by one copy on
+    a second stream and whose outputs leave by one copy on a third, so that
+    later segments' input copies and earlier segments' output copies overlap
+    the calls in between."""
     import torch
     L = len(plans)
     in_host = in_buf.cpu().pin_memory()
     out_host = torch.empty_like(out_buf, device="cpu").pin_memory()
     h2d = sum(x.numel() * x.element_size() for x in qs + tks + tvs if x is not None)
     d2h = out_host.numel() * out_host.element_size()
+    # four segments: more (or segments of 1, 2, 4, ... layers) measured no
+    # better, each cross-stream edge costing the calls their chaining
     nseg = min(4, L)
     cuts = [round(k * L / nseg) for k in range(nseg + 1)]
     base = in_buf.data_ptr()
     seg_bytes = [qs[a].data_ptr() - base for a in cuts[:-1]] + [in_buf.numel()]
-    seg_graphs = []
-    for a, b in zip(cuts, cuts[1:]):
-        gs = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(gs, stream=stream):
-            for l in range(a, b):
-                plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws,
-                                stream=stream)
-        seg_graphs.append(gs)
     copy_stream = torch.cuda.Stream(device=dev)
+    out_stream = torch.cuda.Stream(device=dev)
     seg_done = [torch.cuda.Event() for _ in range(nseg)]
+    seg_out = [torch.cuda.Event() for _ in range(nseg)]
 
-    def e2e_step(s):
+    def body(s):
         copy_stream.wait_stream(s)  # the previous step's calls have read their inputs
+        out_stream.wait_stream(s)
         with torch.cuda.stream(copy_stream):
             for k in range(nseg):
                 lo, hi = seg_bytes[k], seg_bytes[k + 1]
@@ -827,8 +825,25 @@ def measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, m
                 seg_done[k].record(copy_stream)
         for k in range(nseg):
             s.wait_event(seg_done[k])
-            seg_graphs[k].replay()
-        out_host.copy_(out_buf, non_blocking=True)
+            for l in range(cuts[k], cuts[k + 1]):
+                plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws, stream=s)
+            seg_out[k].record(s)
+            out_stream.wait_event(seg_out[k])
+            with torch.cuda.stream(out_stream):
+                out_host[cuts[k]:cuts[k + 1]].copy_(out_buf[cuts[k]:cuts[k + 1]], non_blocking=True)
+        s.wait_stream(out_stream)  # the step ends when its last output is on the host
+
+    # the whole step (copies, calls, event edges) is one CUDA graph, so the
+    # host issues one launch a step
+    with torch.cuda.stream(stream):
+        body(stream)
+    stream.synchronize()
+    step_graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(step_graph, stream=stream):
+        body(stream)
+
+    def e2e_step(s):
+        step_graph.replay()
 
     with torch.cuda.stream(stream):
         for _ in range(2):
@@ -845,9 +860,11 @@ def measure_e2e(plans, stream, in_buf, out_buf, qs, tks, tvs, toffs, outs, ws, m
     e_ms = max_over_ranks(e0.elapsed_time(e1) / e_steps, dist, dev)
     return {"value": replica_throughput(world, tokens, e_ms), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
-            "how": "per step: every layer's q and tails copied from pinned host memory in %d copies on a "
-                   "second stream, each releasing a captured graph of its layers' calls, then one copy "
-                   "of every layer's output to pinned host memory" % nseg}
+            "segments": nseg,
+            "how": "one CUDA graph a step: every layer's q and tails copied from pinned host memory in %d "
+                   "copies on a second stream, each releasing its layers' calls, whose outputs are copied to "
+                   "pinned host memory on a third stream; the step ends when the last output copy is done"
+                   % nseg}
 
 
 def traffic_record(cfg_name):
