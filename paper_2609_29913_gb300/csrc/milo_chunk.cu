@@ -455,9 +455,12 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
     const bool leader = RG == 1 ? tid == 0 : warp == 0 && lane == 0;  // the group's first thread
     if (is_tail) {
         // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense
-        // tail, in slot grp (RG = 2) or both slots from slot 0 (RG = 1)
-        const uint32_t tbase = smem_u32(smem) + grp * kPieceBytes, tbar = bar0 + 8 * grp;
-        const int S = p.tail_splits;
+        // tail in pieces of kTailTokens.  With one group a block (RG = 1) an
+        // item holds up to p.tail_pieces pieces, streamed through the two
+        // slots (piece k in slot k & 1, requested when piece k - 2 is
+        // consumed); with two groups each group's item is one piece in the
+        // group's slot.
+        const int S = p.tail_splits, P = RG == 1 ? p.tail_pieces : 1;
         int64_t o0 = 0;
         int T = 0, sp = 0;
         if (active) {
@@ -467,27 +470,36 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
             o0 = p.tail_offsets[qi];
             T = (int)(p.tail_offsets[qi + 1] - o0);
         }
-        if (sp == S - 1 && T > S * kTailTokens && leader) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
-        const int t0 = sp * kTailTokens;
-        ntok = max(0, min(t0 + kTailTokens, T) - t0);
+        if (sp == S - 1 && T > S * P * kTailTokens && leader)
+            atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
+        const int t0 = sp * P * kTailTokens;
+        ntok = max(0, min(t0 + P * kTailTokens, T) - t0);
+        const int npieces = (ntok + kTailTokens - 1) / kTailTokens;
         nrk = nrv = NT;
         // K then V: one box of kTailTokens rows x 64 columns (128-byte rows,
         // 128-byte swizzle) per 64 columns; a box starts on a 1024-byte line
         constexpr uint32_t kBox = kTailTokens * 128, kHalf = (D / 64) * kBox;
         static_assert(kPieceBytes % 1024 == 0 && kHalf % 1024 == 0, "swizzled boxes on 1024-byte lines");
-        if (ntok > 0 && (tbase & 1023u)) {
+        auto tslot = [&](int k) { return (uint32_t)(RG == 1 ? (k & 1) : grp); };
+        if (npieces > 0 && (smem_u32(smem) & 1023u)) {
             // (cannot happen: the dynamic shared memory starts on a 1024-byte
             // line) the item is dropped and the call reports a bounds error
             if (leader) atomicCAS(p.status, 0, (int32_t)MILO_ERR_DEVICE_BOUNDS);
             ntok = 0;
         }
-        if (ntok > 0 && leader) {
-            mbar_arrive_tx(tbar, 2 * kHalf);
+        const int np_t = ntok > 0 ? npieces : 0;
+        auto tail_issue = [&](int k) {
+            const uint32_t base = smem_u32(smem) + tslot(k) * kPieceBytes, b = bar0 + 8 * tslot(k);
+            mbar_arrive_tx(b, 2 * kHalf);
 #pragma unroll
             for (int c = 0; c < D / 64; ++c) {
-                tma_load_3d(tbase + c * kBox, &tmap_k, 64 * c, g, (int)(o0 + t0), tbar);
-                tma_load_3d(tbase + kHalf + c * kBox, &tmap_v, 64 * c, g, (int)(o0 + t0), tbar);
+                tma_load_3d(base + c * kBox, &tmap_k, 64 * c, g, (int)(o0 + t0 + k * kTailTokens), b);
+                tma_load_3d(base + kHalf + c * kBox, &tmap_v, 64 * c, g, (int)(o0 + t0 + k * kTailTokens), b);
             }
+        };
+        if (leader) {
+            if (np_t > 0) tail_issue(0);
+            if (np_t > 1) tail_issue(1);
         }
         // q~ = scale * log2(e) * q of the G heads of query qi, as score A fragments
         // (k-steps split between the warps)
@@ -509,16 +521,27 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
             sq[ks * 32 + lane] = f;
         }
         __syncthreads();
-        if (ntok > 0) mbar_wait(tbar, 0, p.status);
-        // the item's tokens in units of kTailTokens / kWarps, one per warp
+        // each piece's tokens in units of kTailTokens / kWarps, one per warp
         constexpr int kTU = kTailTokens / kWarps;
         static_assert(kTU == 16 || kTU == 32, "tail units of 16 or 32 tokens");
         const int tb = kTU * warp;
-        if (tb < ntok) {
-            tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTU>{},
-                 std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{},
-                 std::true_type{}, tbase, 1024, tbase + kHalf, 1024, tb, kTailTokens / 8, ntok);
-            if (warp == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
+#pragma unroll 1
+        for (int k = 0; k < np_t; ++k) {
+            const uint32_t base = smem_u32(smem) + tslot(k) * kPieceBytes;
+            mbar_wait(bar0 + 8 * tslot(k), (k >> 1) & 1, p.status);
+            const int nk = min(kTailTokens, ntok - k * kTailTokens);
+            if (tb < nk) {
+                tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTU>{},
+                     std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{},
+                     std::true_type{}, base, 1024, base + kHalf, 1024, tb, kTailTokens / 8, nk);
+                if (k == 0 && warp == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
+            }
+            if (k + 2 < np_t) {
+                // (RG = 1 here: P > 1) the slot's reads before its next copy
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncthreads();
+                if (leader) tail_issue(k + 2);
+            }
         }
     } else {
         // P^K pieces (the loops over the piece kinds keep each kind's
@@ -802,7 +825,8 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     // two row groups per block once a KV head has more than 8 query rows
-    const bool two = p.nrg >= 2;
+    // (one when the grid holds long tail items alone)
+    const bool two = p.nrg >= 2 && p.tail_pieces <= 1;
     cudaError_t e = p.d == 64 ? (two ? launch_chunk_grid<64, 2>(cfg, p, mk, mv) : launch_chunk_grid<64, 1>(cfg, p, mk, mv))
                               : (two ? launch_chunk_grid<128, 2>(cfg, p, mk, mv)
                                      : launch_chunk_grid<128, 1>(cfg, p, mk, mv));

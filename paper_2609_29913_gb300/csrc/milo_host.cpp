@@ -690,6 +690,7 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t
 namespace {
 struct CallShape {
     int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
+    int P;         // kTailTokens pieces per tail item
     bool chunked;  // the chunk grid's accumulators and finish grid (paths 0 and 1)
     int path;      // milo_path_t
     int ntile;     // tensor-core path: row tiles per KV head
@@ -711,7 +712,6 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.nrg_t = (p->G + 7) / 8;
     c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
-    c.S = max_tail > 0 ? (int)((max_tail + kTailTokens - 1) / kTailTokens) : 0;
     // the short-block decode serves every call with a prefix and G <= 8; its
     // prefix part moves to the tensor cores from kTcMinRows rows per KV head
     c.chunked = p->G <= 8 && p->num_chunks > 0;
@@ -723,6 +723,12 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     }
     c.path = !c.chunked ? MILO_PATH_PERSISTENT : c.part ? MILO_PATH_TENSOR : MILO_PATH_CHUNKS;
     if (!c.part) c.ntile = 0;
+    // tail items: on the tensor-core path the chunk grid holds the tails
+    // alone, and each item streams up to kTailPiecesLong pieces (fewer items,
+    // each merged once); beside prefix chunks, or in the persistent kernel,
+    // an item is one piece
+    c.P = c.path == MILO_PATH_TENSOR ? kTailPiecesLong : 1;
+    c.S = max_tail > 0 ? (int)((max_tail + (int64_t)c.P * kTailTokens - 1) / ((int64_t)c.P * kTailTokens)) : 0;
     // one record per prefix chunk and row group (the short-block decode), or
     // per run and row group (the persistent kernel and the tensor-core grid);
     // then the tail items.  The short-block decode and the tensor-core grid
@@ -843,6 +849,7 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
     prm.npass_t = c.npass_t;
     prm.num_slots = plan->num_slots;
     prm.tail_splits = c.S;
+    prm.tail_pieces = c.P;
     prm.num_tail_items = (int)tail_items;
     prm.has_tail = c.S > 0 ? 1 : 0;
     prm.tail_rec_base = (int64_t)plan->num_slots * c.nrg;

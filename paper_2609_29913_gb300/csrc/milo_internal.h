@@ -14,7 +14,8 @@ constexpr int kThreads = 32 * (1 + kMmaWarps);  // + one producer warp
 constexpr int kSlots = 5;            // ring depth (fills in flight)
 constexpr int kSlotBytes = 32768;    // bytes per ring slot (one fill)
 constexpr int kHdrInts = 32;         // fill header (ints)
-constexpr int kTailTokens = 64;      // tokens per dense-tail work item
+constexpr int kTailTokens = 64;      // tokens per dense-tail work item (per piece of one)
+constexpr int kTailPiecesLong = 8;   // pieces per tail item when the chunk grid holds tails alone
 constexpr int kRecFloatsExtra = 16;  // m[8], l[8] after o[8][d] in a record
 
 // fill flags: a fill carries, in processing order, the previous segment's
@@ -118,7 +119,8 @@ struct DecodeParams {
     int ngrp_t;                     // tail row groups per pass (1 or 2)
     int npass_t;                    // ceil(nrg_t / ngrp_t)
     int num_slots;                  // prefix record slots
-    int tail_splits;                // S
+    int tail_splits;                // S: tail items per (query, KV head)
+    int tail_pieces;                // kTailTokens pieces per tail item (the chunk grid)
     int num_tail_items;             // batch * Hkv * S
     int has_tail;
     int64_t tail_rec_base;          // first tail record index

@@ -280,3 +280,40 @@ def test_int8_argument_errors(env):
     with pytest.raises(milo.MiloError) as ei:
         milo.milo_dequantize_int8(x[1:129], x, x[:128])   # codes not 8-byte aligned
     assert ei.value.status == 3
+
+
+def test_int8_plan_on_the_reconstruct_path_with_pre_rope(env):
+    """An INT8 plan in host memory with pre-RoPE factors, staged, decoded by
+    reconstruct-then-attend: the oracle's pre-RoPE attention over its INT8
+    read-back (and the static no-workspace call on the rank-space path of a
+    second INT8 plan)."""
+    milo, W, oracle = env["milo"], env["W"], env["oracle"]
+    layer = W.make_random_case(num_q_heads=14, num_kv_heads=2, head_dim=128, block_lens=[512, 200, 65],
+                               rank_choices=(8, 32, 128), batch=3, tail_lengths=[5, 40, 0], seed=91,
+                               device="cuda")
+    bits = layer.to_numpy_bits()
+    deq, _ = Q.quantize_arena(arena=bits["arena"], **layer.table_arrays())
+    ref = oracle.attention(**dict(bits, arena=deq), rope_theta=1e6)
+    pre = milo.Prefix.from_layer(layer)
+    pre.quantize_int8(to_host=True)
+    pre.set_rope(1e6)
+    buf = torch.empty(int(pre.info["packed_bytes"]) + 128, dtype=torch.uint8, device="cuda")
+    pre.stage(buf)
+    toff = torch.as_tensor(layer.tail_offsets, device="cuda")
+    out = pre.decode_reconstruct(layer.q, layer.tail_k, layer.tail_v, toff, 40)
+    torch.cuda.synchronize()
+    assert pre.status() == 0
+    compare(out.cpu().numpy(), ref, "int8 pre-RoPE reconstruct")
+    pre.close()
+
+    ref_rs = oracle.attention(**dict(bits, arena=deq))
+    pre = milo.Prefix.from_layer(layer)
+    pre.quantize_int8()
+    pre.stage(buf)
+    out = torch.full((3, 14, 128), float("nan"), device="cuda")
+    milo.milo_attn_decode_static(pre.plan, layer.q.data_ptr(), 3, layer.tail_k.data_ptr(), layer.tail_v.data_ptr(),
+                                 toff.data_ptr(), int(layer.tail_k.shape[0]), 40, 0.0, out.data_ptr())
+    torch.cuda.synchronize()
+    assert pre.status() == 0
+    compare(out.cpu().numpy(), ref_rs, "int8 static call")
+    pre.close()

@@ -78,7 +78,7 @@ def test_static_scratch_rejects_oversized_call(env):
     """A call needing more scratch than the built-in array is refused on the
     host with MILO_ERR_WORKSPACE and launches nothing (the output stays)."""
     milo, W = env["milo"], env["W"]
-    batch, tail = 64, 2048
+    batch, tail = 4, 8192   # 28 rows per KV head (the chunk grid): 128 tail items per (query, KV head)
     layer = W.make_random_case(num_q_heads=28, num_kv_heads=4, head_dim=128, block_lens=[64],
                                rank_choices=(16,), batch=batch, tail_lengths=[tail] * batch,
                                seed=11, device="cuda")
