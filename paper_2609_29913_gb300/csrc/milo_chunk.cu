@@ -1,7 +1,7 @@
 // milo_chunk.cu -- the split-K decode for up to 8 query heads per KV head
-// (G <= 8): one thread block of kWarps warps per chunk and row group of 8
-// query rows (batch x G rows per KV head), or of 2 kWarps warps per chunk and
-// pair of row groups once a KV head has more than 8 rows; three blocks per
+// (G <= 8): one thread block of four warps per chunk and row group of 8
+// query rows (batch x G rows per KV head), or of two warps per row group and
+// a pair of row groups once a KV head has more than 8 rows; three blocks per
 // SM at head dimension 128.  Each chunk is streamed through two
 // shared-memory slots that all the block's warps read.
 //
@@ -50,9 +50,13 @@ namespace {
 
 constexpr int kPieceBytes = 32768;  // one slot
 constexpr int kTile = 32;           // tokens per tile
-constexpr int kWarps = 2;           // warps per row group of 8 query rows
+// warps per row group of 8 query rows: four when a block holds one row
+// group (more warps in flight on each SM's three blocks), two when it holds
+// two (their exchange areas share one slot)
+template <int RG>
+constexpr int kWarpsOf = RG == 1 ? 4 : 2;
 
-// Shared memory of a block of RG row groups (RG x kWarps warps).
+// Shared memory of a block of RG row groups (RG x kWarpsOf<RG> warps).
 template <int D, int RG>
 struct CLay {
     static constexpr int kQ = 2 * kPieceBytes;                  // per row group: q~ (then v~) A fragments
@@ -60,7 +64,7 @@ struct CLay {
     static constexpr int kZero = kQ + RG * kQStride;            // a zero core line
     static constexpr int kBar = kZero + 128;                    // 2 mbarriers
     static constexpr int kX = kBar + 16;                        // per row group: m, l [kWarps][8], ref [8]
-    static constexpr int kXStride = 16 * kWarps + 8;            //   (words)
+    static constexpr int kXStride = 16 * kWarpsOf<RG> + 8;      //   (words)
     static constexpr int kTotal = kX + (RG * kXStride * 4 + 15) / 16 * 16;
     static constexpr int kRanksPerPiece = kPieceBytes / (D * 2);  // P^K / P^V rows per piece
 };
@@ -183,13 +187,13 @@ __device__ bool add_part(const DecodeParams &p, int g, int lane, int n0, const f
     return direct;
 }
 
-// RG row groups of 8 query rows per block, kWarps warps each: the groups
+// RG row groups of 8 query rows per block, kWarpsOf<RG> warps each: the groups
 // share every piece (RG = 2 for calls with several row groups per KV head).
 // A tail block holds RG tail items, one per group; with RG = 2 group i's
-// item sits in slot i, with RG = 1 it starts at slot 0.  "warp" below is the
+// item sits in slot i, with RG = 1 its pieces alternate between the slots.  "warp" below is the
 // warp's index within its row group.
 template <int D, int RG>
-__global__ void __launch_bounds__(32 * kWarps * RG)
+__global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     chunk_kernel(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tmap_k,
                  const __grid_constant__ CUtensorMap tmap_v)
 {
@@ -197,6 +201,7 @@ __global__ void __launch_bounds__(32 * kWarps * RG)
     static_assert(2 * (D / 8) * kTailTokens * 16 <= (RG == 1 ? 2 : 1) * kPieceBytes,
                   "a group's tail item fits its slots");
     using L = CLay<D, RG>;
+    constexpr int kWarps = kWarpsOf<RG>;
     constexpr int kThreads = 32 * kWarps * RG;
     constexpr int KD = D / 16;  // 16-wide k-steps over the head dimension
     constexpr int NT = D / 8;   // 8-wide tiles over the head dimension (and the largest rank)
@@ -807,7 +812,7 @@ cudaError_t launch_chunk_grid(cudaLaunchConfig_t cfg, const DecodeParams &p, con
     }
     const int nrgb = (p.nrg + RG - 1) / RG;
     cfg.gridDim = dim3(p.num_chunks * nrgb + (p.has_tail ? (p.num_tail_items + RG - 1) / RG : 0));
-    cfg.blockDim = dim3(32 * kWarps * RG);
+    cfg.blockDim = dim3(32 * kWarpsOf<RG> * RG);
     cfg.dynamicSmemBytes = (size_t)L::kTotal;
     return cudaLaunchKernelEx(&cfg, chunk_kernel<D, RG>, p, mk, mv);
 }
