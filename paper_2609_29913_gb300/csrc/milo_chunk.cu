@@ -23,10 +23,12 @@
 //                (Alg. 1 Stage 2's back-projection), after the warps' v~ are
 //                merged; each warp produces a share of the head dimension.
 //
-// A dense-tail item (one query's tail split for one KV head, kTailTokens
-// tokens) brings its K and V rows with 3-D TMA boxes (64 head dimensions x
-// kTailTokens rows each, 128-byte rows with the 128-byte swizzle: few, wide
-// requests) and runs the C steps on them with q~ = scale * log2(e) * q, a share of the
+// A dense-tail item (one query's tail split for one KV head, in pieces of
+// kTailTokens tokens: one piece beside prefix chunks, up to
+// DecodeParams::tail_pieces when the grid holds tails alone) brings each
+// piece's K and V rows with 3-D TMA boxes (64 head dimensions x kTailTokens
+// rows each, 128-byte rows with the 128-byte swizzle: few, wide requests)
+// and runs the C steps on them with q~ = scale * log2(e) * q, a share of the
 // tokens per warp; its values are already o.  Every item then adds its result
 // into fp32 accumulators of its KV head's rows (see add_part) and exits; a
 // small finish grid chained by programmatic dependent launch (one warp per KV
