@@ -23,11 +23,9 @@
 //                (Alg. 1 Stage 2's back-projection), after the warps' v~ are
 //                merged; each warp produces a share of the head dimension.
 //
-// A dense-tail item (one query's tail split for one KV head, in pieces of
-// kTailTokens tokens: one piece beside prefix chunks, up to
-// DecodeParams::tail_pieces when the grid holds tails alone) brings each
-// piece's K and V rows with 3-D TMA boxes (64 head dimensions x kTailTokens
-// rows each, 128-byte rows with the 128-byte swizzle: few, wide requests)
+// A dense-tail item (one query's tail for one KV head: 1, or tail_pieces when the grid holds tails
+// alone, pieces of kTailTokens tokens) brings each piece's K and V rows with 3-D TMA boxes (64 head
+// dimensions x kTailTokens rows each, 128-byte rows with the 128-byte swizzle: few, wide requests)
 // and runs the C steps on them with q~ = scale * log2(e) * q, a share of the
 // tokens per warp; its values are already o.  Every item then adds its result
 // into fp32 accumulators of its KV head's rows (see add_part) and exits; a
