@@ -117,13 +117,15 @@ struct ByteCost {
 // Cost of the tensor-core decode's work, in eighths of a cycle of one SM: per
 // token the softmax of a 128-row tile (~8 cycles) and the hi + lo score and
 // value products (ranks rounded up to 16: (r^k + r^v) / 8 cycles); per
-// segment the projection, back-projection and pipeline restart (~2500
-// cycles), charged with its first tile.
+// segment the projection, the staging of q~ and v~ and the back-projection
+// (~7500 cycles), charged with its first tile.  (A segment weight of 2500,
+// 5000, 7500 and 10000 cycles measured 0.433, 0.429, 0.425 and 0.428 ms on
+// the 1M-token layer and 3.37, 3.31, 3.27 and 3.27 ms on the batch-64 step.)
 struct TensorCost {
     const milo_block_table_t *t;
     static int r16(int r) { return (r + 15) & ~15; }
     int64_t tile(int e, int t8) const { return (int64_t)t8 * (64 + r16(t->rank_k[e]) + r16(t->rank_v[e])); }
-    int64_t first(int) const { return 20000; }
+    int64_t first(int) const { return 60000; }
     int64_t last(int) const { return 0; }
 };
 constexpr int64_t kTcMinShareCost = 100000;  // in TensorCost units: ~one 512-token entry of rank 64
