@@ -142,10 +142,13 @@ __global__ void __launch_bounds__(kInt8Threads) dequant_kernel(const uint2 *__re
 // n) and writes 0 there instead of m + s c: the staged arena then holds
 // exactly the zero-padded read-back factors the decode kernels expect.  Each
 // lane issues the loads of its four cores before converting any of them.
+// (128-thread blocks: small enough in registers to run beside the decode
+// grid's blocks of the layer before, which the staging overlaps)
+constexpr int kPlanThreads = 128;
 constexpr int kPlanUnroll = 4;
-constexpr int kPlanGroups = (kInt8Threads / 8) * kPlanUnroll;   // cores per block
+constexpr int kPlanGroups = (kPlanThreads / 8) * kPlanUnroll;   // cores per block
 
-__global__ void __launch_bounds__(kInt8Threads) dequant_plan_kernel(const EntryDev *__restrict__ entries, int head_dim,
+__global__ void __launch_bounds__(kPlanThreads) dequant_plan_kernel(const EntryDev *__restrict__ entries, int head_dim,
                                                                     const uint2 *__restrict__ codes,
                                                                     const uint32_t *__restrict__ params,
                                                                     uint4 *__restrict__ dst)
@@ -170,7 +173,7 @@ __global__ void __launch_bounds__(kInt8Threads) dequant_plan_kernel(const EntryD
     uint32_t pw[kPlanUnroll];
 #pragma unroll
     for (int u = 0; u < kPlanUnroll; ++u) {
-        const int t = base + team + u * (kInt8Threads / 8);
+        const int t = base + team + u * (kPlanThreads / 8);
         if (t < total) {
             c[u] = codes[(g0 + t) * 8 + row];
             pw[u] = params[g0 + t];
@@ -178,7 +181,7 @@ __global__ void __launch_bounds__(kInt8Threads) dequant_plan_kernel(const EntryD
     }
 #pragma unroll
     for (int u = 0; u < kPlanUnroll; ++u) {
-        const int t = base + team + u * (kInt8Threads / 8);
+        const int t = base + team + u * (kPlanThreads / 8);
         if (t >= total) break;
         uint4 v = dequant_row(c[u], pw[u]);
         int valid = 8;
@@ -231,7 +234,7 @@ cudaError_t launch_dequant_plan_int8(const EntryDev *entries, int num_entries, i
 {
     if (num_entries <= 0 || max_factor_groups <= 0) return cudaSuccess;
     const int slices = (int)((max_factor_groups + kPlanGroups - 1) / kPlanGroups);
-    dequant_plan_kernel<<<dim3(num_entries, 4, slices), kInt8Threads, 0, stream>>>(
+    dequant_plan_kernel<<<dim3(num_entries, 4, slices), kPlanThreads, 0, stream>>>(
         entries, head_dim, static_cast<const uint2 *>(codes), static_cast<const uint32_t *>(params),
         static_cast<uint4 *>(packed));
     return cudaGetLastError();
