@@ -288,8 +288,9 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
         const int r = lane >> 1;
         int qrow = -1, gq = g;
         if (is_tail) {
-            gq = (item / p.tail_splits) % p.hkv;
-            if (r < p.G) qrow = item / (p.hkv * p.tail_splits) * p.G + r;
+            const int rq = (item / p.tail_splits) % p.nrg_t;
+            gq = (item / (p.tail_splits * p.nrg_t)) % p.hkv;
+            if (8 * rq + r < p.G) qrow = item / (p.hkv * p.tail_splits * p.nrg_t) * p.G + 8 * rq + r;
         } else if (8 * rgrp + r < p.rows_g) {
             qrow = 8 * rgrp + r;
         }
@@ -456,7 +457,7 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     };
 
     uint32_t ref = 0u;  // this row's reference maximum (warp 0, lane c4 == 0), see publish_ref
-    int qi = 0;
+    int qi = 0, rq = 0;  // tail item: query, and group of 8 of its G heads
     const bool leader = RG == 1 ? tid == 0 : warp == 0 && lane == 0;  // the group's first thread
     if (is_tail) {
         // tail item: query qi, KV head g, tokens [t0, t0 + ntok) of qi's dense
@@ -469,9 +470,11 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
         int64_t o0 = 0;
         int T = 0, sp = 0;
         if (active) {
-            qi = item / (p.hkv * S);
+            // item = ((qi * Hkv + g) * nrg_t + rq) * S + sp: rows [8 rq, 8 rq + 8) of qi's G heads
             sp = item % S;
-            g = (item / S) % p.hkv;
+            rq = (item / S) % p.nrg_t;
+            g = (item / (S * p.nrg_t)) % p.hkv;
+            qi = item / (S * p.nrg_t * p.hkv);
             o0 = p.tail_offsets[qi];
             T = (int)(p.tail_offsets[qi + 1] - o0);
         }
@@ -511,8 +514,8 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
 #pragma unroll 1
         for (int ks = warp; ks < KD; ks += kWarps) {
             float x[4] = {0.f, 0.f, 0.f, 0.f};
-            if (r4 < p.G) {
-                const uint16_t *qr = p.q + ((int64_t)qi * p.hq + g * p.G + r4) * D + 16 * ks + 2 * c4;
+            if (8 * rq + r4 < p.G) {
+                const uint16_t *qr = p.q + ((int64_t)qi * p.hq + g * p.G + 8 * rq + r4) * D + 16 * ks + 2 * c4;
                 const __nv_bfloat162 a2 = *reinterpret_cast<const __nv_bfloat162 *>(qr);
                 const __nv_bfloat162 b2 = *reinterpret_cast<const __nv_bfloat162 *>(qr + 8);
                 x[0] = __low2float(a2) * p.scale_log2;
@@ -539,7 +542,8 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
                 tile(std::integral_constant<int, NT / 2>{}, std::integral_constant<int, kTU>{},
                      std::integral_constant<uint32_t, kBox>{}, std::integral_constant<uint32_t, kBox>{},
                      std::true_type{}, base, 1024, base + kHalf, 1024, tb, kTailTokens / 8, nk);
-                if (k == 0 && warp == 0) ref = publish_ref(p, g, qi * p.G + r4, r4 < p.G, c4, m_w);
+                if (k == 0 && warp == 0)
+                    ref = publish_ref(p, g, qi * p.G + 8 * rq + r4, 8 * rq + r4 < p.G, c4, m_w);
             }
             if (k + 2 < np_t) {
                 // (RG = 1 here: P > 1) the slot's reads before its next copy
@@ -704,8 +708,8 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     if (is_tail) {
         // the values are already in the head dimension: o = v~ (warp 0 adds all of it)
         rec_idx = p.tail_rec_base + item;
-        row0 = qi * p.G;
-        nrows = active ? p.G : 0;
+        row0 = qi * p.G + 8 * rq;
+        nrows = active ? min(8, p.G - 8 * rq) : 0;
         float ov[NT][2];
 #pragma unroll
         for (int n = 0; n < NT; ++n) {

@@ -552,7 +552,7 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     // tensor-core path: a partition for every share count sms / ntile that a
     // call with ntile row tiles of kTcRows rows per KV head uses
     p->sms = sms;
-    p->tc = G <= 8 && !chunks.empty() && (int64_t)max_batch * G >= kTcMinRows;
+    p->tc = !chunks.empty() && (int64_t)max_batch * G >= kTcMinRows;
     std::vector<TcSegDev> tc_sd;
     std::vector<int32_t> tc_cb;
     if (p->tc) {
@@ -603,8 +603,8 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         milo_prefix_destroy(p);
         return cuda_fail(err, what);
     };
-    // + the accumulators of the short-block decode (G <= 8)
-    const size_t cnt_bytes = G <= 8 ? counters_bytes(H, 8 * p->max_nrg, d) : sizeof(CountersDev);
+    // + the accumulators of the chunk grid's calls
+    const size_t cnt_bytes = counters_bytes(H, 8 * p->max_nrg, d);
     if ((e = cudaMalloc(&p->packed, (size_t)std::max<int64_t>(p->packed_bytes, 128))) != cudaSuccess)
         return cleanup(e, "cudaMalloc packed");
     if ((e = cudaMalloc(&p->entries, sizeof(EntryDev) * std::max<size_t>(ents.size(), 1))) != cudaSuccess)
@@ -714,9 +714,10 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     c.nrg_t = (p->G + 7) / 8;
     c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
     c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
-    // the short-block decode serves every call with a prefix and G <= 8; its
-    // prefix part moves to the tensor cores from kTcMinRows rows per KV head
-    c.chunked = p->G <= 8 && p->num_chunks > 0;
+    // the chunk grid serves every call (a call without a prefix holds tail
+    // items alone); its prefix part moves to the tensor cores from
+    // kTcMinRows rows per KV head
+    c.chunked = true;
     c.ntile = 0;
     c.part = nullptr;
     if (c.chunked && p->tc && c.rows_g >= kTcMinRows) {
@@ -741,7 +742,12 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     const int64_t prefix = c.part ? (int64_t)c.part->num_slots * c.nrg
                            : c.chunked ? (int64_t)p->num_chunks * c.nrg : (int64_t)p->num_slots * c.nrg;
     c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
-    const int64_t queries_per_group = std::min<int64_t>(batch, 7 / p->G + 2);
+    // tail items (per split) whose 8 rows meet one row group: with G <= 8 an
+    // item is one query's G rows, at most 7 / G + 2 queries meet 8 rows; with
+    // G > 8 an item is 8 (or fewer, the query's last) of a query's rows, and
+    // at most three such spans meet 8 rows
+    const int64_t queries_per_group =
+        p->G <= 8 ? std::min<int64_t>(batch, 7 / p->G + 2) : std::min<int64_t>((int64_t)batch * c.nrg_t, 3);
     const int64_t prefix_items = c.part ? (int64_t)c.part->max_runs : (int64_t)p->max_head_chunks;
     c.list_cap = c.chunked ? prefix_items + queries_per_group * c.S : 0;
     c.list_bytes = 16 * (int64_t)p->hkv * c.nrg * c.list_cap;
@@ -801,12 +807,12 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
 
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
     if (recon && (!c.chunked || plan->rc_num_chunks == 0))
-        return fail(MILO_ERR_UNSUPPORTED, "reconstruct-then-attend needs a prefix and at most 8 query heads per KV head");
+        return fail(MILO_ERR_UNSUPPORTED, "reconstruct-then-attend needs a prefix");
     if (recon && ((int64_t)plan->rc_num_chunks * c.nrg > 0x7fffffff || c.list_cap_rc > 0x7fffffff ||
                   (int64_t)plan->rc_num_chunks * ((c.rows_g + kRcRows - 1) / kRcRows) > 0x7fffffff))
         return fail(MILO_ERR_UNSUPPORTED, "call too large: more than 2^31 - 1 work items");
     // the kernels count thread blocks, tail items and list entries in int
-    const int64_t tail_items = (int64_t)batch * plan->hkv * c.S;
+    const int64_t tail_items = (int64_t)batch * plan->hkv * c.S * (c.chunked ? c.nrg_t : 1);
     // (the persistent path counts record slots per row group and its merge
     // grid's blocks per KV head, row group and float4 column in int too)
     if (tail_items > 0x7fffffff || (int64_t)plan->num_chunks * c.nrg + tail_items > 0x7fffffff ||
@@ -936,6 +942,13 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
         if ((e = launch_finish(prm, stream)) != cudaSuccess) return cuda_fail(e, "finish grid launch");
         return MILO_OK;
     }
+    if (c.path == MILO_PATH_CHUNKS) {
+        // the prefix chunks and the tail items in one grid (tail items alone
+        // without a prefix), then the finish grid
+        cudaError_t e = launch_chunks(prm, &mk, &mv, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "chunk grid launch");
+        return MILO_OK;
+    }
     const int smem = decode_smem_bytes(plan->d, c.nrg_cta);
     cudaError_t e = launch_decode(prm, &mk, &mv, smem, plan->num_ctas, stream);
     if (e != cudaSuccess) return cuda_fail(e, "decode launch");
@@ -1051,7 +1064,7 @@ milo_status_t milo_call_info(const milo_prefix_t *plan, int32_t batch, int64_t m
     } else if (c.path == MILO_PATH_CHUNKS) {
         info->kernels = 2;
         const int rg = c.nrg >= 2 ? 2 : 1;
-        const int64_t tail_items = (int64_t)batch * plan->hkv * c.S;
+        const int64_t tail_items = (int64_t)batch * plan->hkv * c.S * (c.chunked ? c.nrg_t : 1);
         info->blocks = (int32_t)std::min<int64_t>(
             (int64_t)plan->num_chunks * ((c.nrg + rg - 1) / rg) + (tail_items + rg - 1) / rg, 0x7fffffff);
     } else {
