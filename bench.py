@@ -313,9 +313,7 @@ def kernel_names(path: int, has_tail: bool) -> list:
     """The kernels one layer call launches, for the JSON line's description."""
     if path == 1:
         return (["chunk_kernel (dense-tail items)"] if has_tail else []) + ["batch_tc_kernel", "finish_kernel"]
-    if path == 0:
-        return ["chunk_kernel", "finish_kernel"]
-    return ["decode_kernel", "combine_kernel"]
+    return ["chunk_kernel", "finish_kernel"]
 
 
 def time_graph(step, stream, steps, warmup, flush):
@@ -468,8 +466,7 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
                    "peak_source": f"{peak_kind} sustained cuBLAS bf16 (bf16_tflops_sustained)"},
         "roofline_time": {"ms": roof_ms, "frac": roof_ms / ms_step,
                           "how": "max(algorithmic bytes / hbm_gbs, algorithmic flops / bf16_tflops_sustained)"},
-        "path": {0: "chunk grid (mma.sync)", 1: "tensor-core batched grid (tcgen05)",
-                 2: "persistent grid (mma.sync)"}[call["path"]],
+        "path": {0: "chunk grid (mma.sync)", 1: "tensor-core batched grid (tcgen05)"}[call["path"]],
         "kernels_per_layer": call["kernels"],
         "kernels": kernel_names(call["path"], max_tail > 0),
         "gpu_launches": call["kernels"] * L * steps,

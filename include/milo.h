@@ -89,7 +89,7 @@ typedef struct {
     int64_t arena_elems;
 } milo_block_table_t;
 
-/* Opaque per-layer plan: packed factors, static work partition, counters. */
+/* Opaque per-layer plan: packed factors, the work lists, accumulators. */
 typedef struct milo_prefix milo_prefix_t;
 
 /*
@@ -119,32 +119,37 @@ milo_status_t milo_packed_layout(const milo_block_table_t *table,
                                  int64_t *packed_offsets, int64_t *total_bytes);
 
 /*
- * Static prefix work partition the decode kernel uses, computed on the host.
- * The prefix (every entry's tokens, KV-head-major, then block order) is cut
- * at 32-token boundaries into segments so that each of `num_ctas` thread
- * blocks receives a near-equal share of the cost line, where a token costs its
- * padded coefficient bytes plus 32 (the softmax work), a block's P^K is charged
- * with its first 32-token tile and its P^V with its last; a tile goes to the
- * thread block whose share holds the midpoint of the tile's cost.  Consecutive segments
- * of one thread block with the same KV head form a "run" whose partial result
- * occupies one slot.
+ * Host-only: the static partition of the prefix over `num_shares` thread
+ * blocks of the tensor-core grid (Alg. 1 Stage 2 split over token ranges,
+ * merged by Eq. 1).  The prefix (every entry's tokens, KV-head-major, then
+ * block order) is laid on a cost line in 32-token tiles, a tile of t8 tokens
+ * (rounded up to 8) costing t8 x (64 + r16(r^k) + r16(r^v)) (r16 = rank
+ * rounded up to 16: the softmax of a 128-row tile and the hi and lo score and
+ * value products) and each entry's first tile 60000 more (its projection,
+ * staging and back-projection); a tile goes to the share of the line,
+ * (c T / num_shares, (c + 1) T / num_shares], that holds the midpoint of the
+ * tile's cost, so no share costs more than T / num_shares plus one tile.
+ * Consecutive tiles of one entry in one share form a segment; consecutive
+ * segments of one share with the same KV head form a "run" whose partial
+ * result occupies one slot (slots numbered in order, hence by KV head).
  *   seg_entry/seg_t0/seg_t1/seg_slot: host arrays of capacity `max_segments`
- *     (entry index, token range [t0, t1), slot); may be NULL to query count.
- *   cta_begin: host [num_ctas + 1] first segment of each thread block; may
- *     be NULL.
+ *     (entry index b * num_kv_heads + g, token range [t0, t1), slot); all may
+ *     be NULL to query the count.
+ *   share_begin: host [num_shares + 1] first segment of each share; may be
+ *     NULL.
  *   num_segments/num_slots: outputs (either may be NULL).
- * Returns MILO_ERR_INVALID_ARG if max_segments is too small.
+ * Returns the table's validation status, MILO_ERR_INVALID_ARG for
+ * num_shares < 1, or (after setting the outputs) if max_segments is too small.
  */
 milo_status_t milo_partition_prefix(const milo_block_table_t *table,
-                                    int32_t num_ctas, int32_t max_segments,
+                                    int32_t num_shares, int32_t max_segments,
                                     int32_t *seg_entry, int32_t *seg_t0,
                                     int32_t *seg_t1, int32_t *seg_slot,
-                                    int32_t *cta_begin, int32_t *num_segments,
+                                    int32_t *share_begin, int32_t *num_segments,
                                     int32_t *num_slots);
 
 /*
- * Host-only: the work list of the short-block decode (plans with at most 8
- * query heads per KV head).  Every prefix entry, KV-head-major then in block
+ * Host-only: the work list of the chunk grid.  Every prefix entry, KV-head-major then in block
  * order, is cut into the fewest token ranges of at most 1024 tokens whose
  * coefficient rows (C^K and C^V at ranks rounded up to 8, tokens rounded up
  * to 8, bf16) fit 128 KB, of equal length in multiples of 32 tokens (the
@@ -167,15 +172,15 @@ milo_status_t milo_chunk_prefix(const milo_block_table_t *table,
 /*
  * Build a plan for one layer on the current device: validate the table,
  * allocate and fill the packed arena (a pack kernel on `stream`, then a
- * stream synchronisation), build the work partition and the device-side
- * counters.  The logical arena may be freed after this call returns.
+ * stream synchronisation), build the work lists and the device-side
+ * accumulators.  The logical arena may be freed after this call returns.
  *   num_q_heads   multiple of num_kv_heads (query head h reads KV head
  *                 h / (num_q_heads / num_kv_heads)).
  *   max_batch     largest batch any decode call on this plan will use.
  *   out_plan      receives the plan; release with milo_prefix_destroy.
  * Errors: the table's validation status; MILO_ERR_INVALID_ARG for a bad
- * head count or max_batch < 1; MILO_ERR_UNSUPPORTED for more than 32 query
- * heads per KV head or max_batch x (num_q_heads / num_kv_heads) above 2^30;
+ * head count or max_batch < 1; MILO_ERR_UNSUPPORTED for
+ * max_batch x (num_q_heads / num_kv_heads) above 2^30;
  * MILO_ERR_CUDA when an allocation, copy or the pack kernel fails.
  */
 milo_status_t milo_prefix_create(const milo_block_table_t *table,
@@ -188,9 +193,6 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan);
 /* Plan facts for accounting and tests. */
 typedef struct {
     int32_t num_blocks, num_kv_heads, num_q_heads, head_dim, max_batch;
-    int32_t num_ctas;             /* thread blocks of the decode kernel       */
-    int32_t num_segments;         /* prefix segments of the partition         */
-    int32_t num_slots;            /* prefix partial slots (runs)              */
     int64_t prefix_tokens;        /* sum of block lengths                     */
     int64_t logical_factor_bytes; /* bytes of C^K,P^K,C^V,P^V at true ranks   */
     int64_t packed_bytes;         /* bytes of the packed arena (with padding) */
@@ -214,22 +216,19 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
  * How a decode call of this shape runs (host only, no device access):
  *   path     MILO_PATH_CHUNKS (0): the chunk grid on warp-level MMA, one
  *            thread block per prefix chunk and row group of 8 query rows
- *            (at most 8 query heads per KV head and fewer query rows per KV
- *            head than the tensor-core threshold);
+ *            (fewer query rows per KV head than the tensor-core threshold,
+ *            or no prefix: then the grid holds the tail items alone);
  *            MILO_PATH_TENSOR (1): the tensor-core grid (tcgen05, 128 query
  *            rows per product) for the prefix, with the dense tails on the
- *            chunk grid (at most 8 query heads per KV head and at least
- *            milo_tensor_min_rows() query rows per KV head);
- *            MILO_PATH_PERSISTENT (2): the persistent warp-level decode and
- *            its merge kernel (more than 8 query heads per KV head, or no
- *            prefix).
+ *            chunk grid (at least milo_tensor_min_rows() query rows per KV
+ *            head).
  *   kernels  kernel launches of one call (each a grid).
  *   row_tiles  tensor-core path: tiles of 128 query rows per KV head (else 0).
  *   blocks   thread blocks of the call's main prefix grid.
  * Errors: MILO_ERR_INVALID_ARG for a null argument, batch outside
  * [1, max_batch] or max_tail_tokens < 0.
  */
-typedef enum { MILO_PATH_CHUNKS = 0, MILO_PATH_TENSOR = 1, MILO_PATH_PERSISTENT = 2 } milo_path_t;
+typedef enum { MILO_PATH_CHUNKS = 0, MILO_PATH_TENSOR = 1 } milo_path_t;
 typedef struct {
     int32_t path;
     int32_t kernels;
@@ -271,7 +270,7 @@ int32_t milo_tensor_min_rows(void);
  * (milo_prefix_set_rope) is refused with MILO_ERR_UNSUPPORTED: rank-space
  * scoring cannot apply a per-position rotation.  A plan must not be used by
  * two calls that can run concurrently (it
- * holds per-call counters and accumulators).  A query whose prefix and tail
+ * holds per-call accumulators).  A query whose prefix and tail
  * are both empty yields NaN.  A call with more than 2^31 - 1 work items
  * (prefix chunks x row groups plus tail items) returns MILO_ERR_UNSUPPORTED
  * without launching anything.

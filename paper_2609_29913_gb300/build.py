@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmilo.so")
-SOURCES = ["milo_host.cpp", "milo_pack.cu", "milo_decode.cu", "milo_chunk.cu", "milo_batch.cu", "milo_recon.cu", "milo_check.cu", "milo_encode.cu", "milo_int8.cu"]
+SOURCES = ["milo_host.cpp", "milo_pack.cu", "milo_scratch.cu", "milo_chunk.cu", "milo_batch.cu", "milo_recon.cu", "milo_check.cu", "milo_encode.cu", "milo_int8.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

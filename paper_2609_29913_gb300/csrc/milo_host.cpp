@@ -100,20 +100,6 @@ int64_t packed_layout(const milo_block_table_t *t, std::vector<int64_t> &offs)
     return cur;
 }
 
-// Cost of the persistent decode's work: a token's padded coefficient bytes
-// plus kTokenOverhead (its softmax work); an entry's P^K is charged with its
-// first 32-token tile and its P^V with its last.
-struct ByteCost {
-    const milo_block_table_t *t;
-    static constexpr int64_t kTokenOverhead = 32;
-    int64_t tile(int e, int t8) const
-    {
-        return (int64_t)t8 * ((r8(t->rank_k[e]) + r8(t->rank_v[e])) * 2 + kTokenOverhead);
-    }
-    int64_t first(int e) const { return (int64_t)r8(t->rank_k[e]) * t->head_dim * 2; }
-    int64_t last(int e) const { return (int64_t)r8(t->rank_v[e]) * t->head_dim * 2; }
-};
-
 // Cost of the tensor-core decode's work, in eighths of a cycle of one SM: per
 // token the softmax of a 128-row tile (~8 cycles) and the hi + lo score and
 // value products (ranks rounded up to 16: (r^k + r^v) / 8 cycles); per
@@ -130,11 +116,13 @@ struct TensorCost {
 };
 constexpr int64_t kTcMinShareCost = 100000;  // in TensorCost units: ~one 512-token entry of rank 64
 
-// Static partition of the prefix over `P` shares (see milo_partition_prefix
-// in milo.h), under a cost model.
+// Static partition of the prefix over `P` shares of the tensor-core grid,
+// under a cost model: segments (entry, token range) listed share by share
+// (share c holds segs[cta_begin[c] .. cta_begin[c + 1])), each share's
+// segments grouped in runs of one KV head, one accumulator slot per run.
 template <class Cost>
 void partition_with(const milo_block_table_t *t, int P, const Cost &cost, std::vector<Seg> &segs,
-                    std::vector<int32_t> &cta_begin, int &num_slots, std::vector<int32_t> *g_slot_begin)
+                    std::vector<int32_t> &cta_begin, int &num_slots)
 {
     const int H = t->num_kv_heads, nb = t->num_blocks;
     int64_t total = 0;
@@ -180,8 +168,6 @@ void partition_with(const milo_block_table_t *t, int P, const Cost &cost, std::v
     for (int c = cta + 1; c <= P; ++c) cta_begin[c] = (int32_t)segs.size();
     // runs and slots: consecutive segments of one share with one KV head
     num_slots = 0;
-    if (g_slot_begin) g_slot_begin->assign((size_t)H + 1, 0);
-    std::vector<int32_t> first_slot_of_g((size_t)H, -1);
     for (int c = 0; c < P; ++c) {
         int prev_g = -1;
         for (int s = cta_begin[c]; s < cta_begin[c + 1]; ++s) {
@@ -189,7 +175,6 @@ void partition_with(const milo_block_table_t *t, int P, const Cost &cost, std::v
             if (g != prev_g) {
                 segs[s].flags |= kSegFirstOfRun;
                 if (s > cta_begin[c]) segs[s - 1].flags |= kSegLastOfRun;
-                if (first_slot_of_g[g] < 0) first_slot_of_g[g] = num_slots;
                 ++num_slots;
                 prev_g = g;
             }
@@ -197,21 +182,10 @@ void partition_with(const milo_block_table_t *t, int P, const Cost &cost, std::v
         }
         if (cta_begin[c + 1] > cta_begin[c]) segs[cta_begin[c + 1] - 1].flags |= kSegLastOfRun;
     }
-    if (g_slot_begin) {
-        // slots are numbered in KV-head order, so each head's slots are contiguous
-        auto &gs = *g_slot_begin;
-        gs[H] = num_slots;
-        for (int g = H - 1; g >= 0; --g) gs[g] = first_slot_of_g[g] >= 0 ? first_slot_of_g[g] : gs[g + 1];
-    }
 }
 
-void partition(const milo_block_table_t *t, int P, std::vector<Seg> &segs, std::vector<int32_t> &cta_begin,
-               int &num_slots, std::vector<int32_t> *g_slot_begin)
-{
-    partition_with(t, P, ByteCost{t}, segs, cta_begin, num_slots, g_slot_begin);
-}
 
-// Chunks of the short-block decode: every prefix entry, KV-head-major then in
+// Chunks of the chunk grid: every prefix entry, KV-head-major then in
 // block order, cut into the fewest token ranges of at most kChunkMaxTok tokens
 // whose coefficient rows (C^K and C^V, rounded up to 8 tokens) fit
 // kChunkBytes, of about equal length; a range starts at a multiple of 32
@@ -265,15 +239,14 @@ void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs
     for (int g = 1; g <= H; ++g) g_begin[(size_t)g] = std::max(g_begin[(size_t)g], g_begin[(size_t)g - 1]);
 }
 
-// The plan's counter buffer: CountersDev, then for the short-block decode the
-// reference maxima [H][R] (R = 8 row groups of 8 rows), the list counts
-// [H][R / 8], and at a 16-byte boundary the row sums [H][R] and the output
-// accumulators [H][R][d].
+// The plan's accumulator buffer: the reference maxima [H][R] (R = 8 x the
+// row groups of 8 rows), the list counts [H][R / 8], and at a 16-byte
+// boundary the row sums [H][R] and the output accumulators [H][R][d].
 size_t acc_l_offset(int H, int R)
 {
-    return (sizeof(CountersDev) + sizeof(uint32_t) * (size_t)H * (R + R / 8) + 15) / 16 * 16;
+    return (sizeof(uint32_t) * (size_t)H * (R + R / 8) + 15) / 16 * 16;
 }
-size_t counters_bytes(int H, int R, int d)
+size_t acc_bytes(int H, int R, int d)
 {
     return acc_l_offset(H, R) + sizeof(float) * (size_t)H * R * (1 + (size_t)d);
 }
@@ -301,7 +274,7 @@ EncodeTiledFn encode_fn()
 struct milo_prefix {
     int device = 0;
     int nb = 0, hkv = 0, hq = 0, d = 0, G = 0, max_batch = 0;
-    int num_ctas = 0, num_segments = 0, num_slots = 0, max_nrg = 0;
+    int max_nrg = 0;
     int64_t prefix_tokens = 0, logical_bytes = 0, packed_bytes = 0;
     uint8_t *packed = nullptr;        // the arena the kernels read (an offloaded plan: the staged copy)
     uint8_t *packed_host = nullptr;   // offloaded plans: the arena in pinned host memory
@@ -312,13 +285,10 @@ struct milo_prefix {
     bool int8_host = false;
     int64_t max_factor_groups = 0;    // the most 8x8 cores of one factor
     EntryDev *entries = nullptr;
-    SegDev *segs = nullptr;
-    int32_t *cta_seg_begin = nullptr;
-    int32_t *g_slot_begin = nullptr;
-    ChunkDev *chunks = nullptr;       // short-block decode: prefix chunks, KV-head-major
+    ChunkDev *chunks = nullptr;       // the chunk grid's prefix chunks, KV-head-major
     int num_chunks = 0;
     int max_head_chunks = 0;          // the most chunks of one KV head
-    CountersDev *counters = nullptr;
+    uint8_t *acc = nullptr;            // the chunk grid's per-row accumulators (zero between calls)
     int32_t *status = nullptr;
     // tensor-core path: one partition per share count a call can use
     bool tc = false;                  // calls with at least kTcMinRows rows per KV head may take it
@@ -385,20 +355,20 @@ milo_status_t milo_packed_layout(const milo_block_table_t *table, int64_t *packe
     return MILO_OK;
 }
 
-milo_status_t milo_partition_prefix(const milo_block_table_t *table, int32_t num_ctas, int32_t max_segments,
+milo_status_t milo_partition_prefix(const milo_block_table_t *table, int32_t num_shares, int32_t max_segments,
                                     int32_t *seg_entry, int32_t *seg_t0, int32_t *seg_t1, int32_t *seg_slot,
-                                    int32_t *cta_begin, int32_t *num_segments, int32_t *num_slots)
+                                    int32_t *share_begin, int32_t *num_segments, int32_t *num_slots)
 {
     milo_status_t s = validate(table);
     if (s != MILO_OK) return s;
-    if (num_ctas < 1) return fail(MILO_ERR_INVALID_ARG, "num_ctas < 1");
+    if (num_shares < 1) return fail(MILO_ERR_INVALID_ARG, "num_shares < 1");
     std::vector<Seg> segs;
     std::vector<int32_t> cb;
     int ns = 0;
-    partition(table, num_ctas, segs, cb, ns, nullptr);
+    partition_with(table, num_shares, TensorCost{table}, segs, cb, ns);
     if (num_segments) *num_segments = (int32_t)segs.size();
     if (num_slots) *num_slots = ns;
-    if (cta_begin) std::memcpy(cta_begin, cb.data(), cb.size() * sizeof(int32_t));
+    if (share_begin) std::memcpy(share_begin, cb.data(), cb.size() * sizeof(int32_t));
     if (seg_entry || seg_t0 || seg_t1 || seg_slot) {
         if ((int64_t)segs.size() > max_segments) return fail(MILO_ERR_INVALID_ARG, "max_segments too small");
         for (size_t i = 0; i < segs.size(); ++i) {
@@ -448,11 +418,8 @@ milo_status_t milo_prefix_destroy(milo_prefix_t *plan)
         else cudaFree(plan->int8_store);
     } else cudaFree(plan->packed);
     cudaFree(plan->entries);
-    cudaFree(plan->segs);
-    cudaFree(plan->cta_seg_begin);
-    cudaFree(plan->g_slot_begin);
     cudaFree(plan->chunks);
-    cudaFree(plan->counters);
+    cudaFree(plan->acc);
     cudaFree(plan->status);
     cudaFree(plan->tc_segs);
     cudaFree(plan->tc_cta);
@@ -476,7 +443,6 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         return fail(MILO_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
     if (max_batch < 1) return fail(MILO_ERR_INVALID_ARG, "max_batch < 1");
     const int G = num_q_heads / table->num_kv_heads;
-    if (G > 32) return fail(MILO_ERR_UNSUPPORTED, "more than 32 query heads per KV head");
     // query rows per KV head are counted in int on the device
     if ((int64_t)max_batch * G > (1 << 30)) return fail(MILO_ERR_UNSUPPORTED, "max_batch x G above 2^30");
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
@@ -490,15 +456,10 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     if (e != cudaSuccess) { delete p; return cuda_fail(e, "cudaDeviceGetAttribute"); }
     const int H = table->num_kv_heads, d = table->head_dim, nb = table->num_blocks;
     p->nb = nb; p->hkv = H; p->hq = num_q_heads; p->d = d; p->G = G; p->max_batch = max_batch;
-    p->num_ctas = sms;
     p->max_nrg = (max_batch * G + 7) / 8;
 
     std::vector<int64_t> poffs;
     p->packed_bytes = packed_layout(table, poffs);
-    std::vector<Seg> segs;
-    std::vector<int32_t> cta_begin, g_slot;
-    partition(table, p->num_ctas, segs, cta_begin, p->num_slots, &g_slot);
-    p->num_segments = (int)segs.size();
 
     const int64_t E = (int64_t)nb * H;
     std::vector<EntryDev> ents((size_t)E);
@@ -545,10 +506,6 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         p->rc_num_chunks = (int)rc.size();
         for (int g = 0; g < H; ++g) p->rc_max_head_chunks = std::max(p->rc_max_head_chunks, per_head[(size_t)g]);
     }
-    std::vector<SegDev> sd(segs.size());
-    for (size_t i = 0; i < segs.size(); ++i) {
-        sd[i] = SegDev{segs[i].entry, segs[i].t0, segs[i].t1, segs[i].slot, segs[i].flags, {0, 0, 0}};
-    }
     // tensor-core path: a partition for every share count sms / ntile that a
     // call with ntile row tiles of kTcRows rows per KV head uses
     p->sms = sms;
@@ -577,7 +534,7 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
             std::vector<Seg> ts;
             std::vector<int32_t> cb;
             int nslot = 0;
-            partition_with(table, ns, TensorCost{table}, ts, cb, nslot, nullptr);
+            partition_with(table, ns, TensorCost{table}, ts, cb, nslot);
             std::vector<int> runs((size_t)H, 0);
             for (const Seg &x : ts)
                 if (x.flags & kSegFirstOfRun) ++runs[(size_t)(x.entry % H)];
@@ -604,17 +561,11 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         return cuda_fail(err, what);
     };
     // + the accumulators of the chunk grid's calls
-    const size_t cnt_bytes = counters_bytes(H, 8 * p->max_nrg, d);
+    const size_t cnt_bytes = acc_bytes(H, 8 * p->max_nrg, d);
     if ((e = cudaMalloc(&p->packed, (size_t)std::max<int64_t>(p->packed_bytes, 128))) != cudaSuccess)
         return cleanup(e, "cudaMalloc packed");
     if ((e = cudaMalloc(&p->entries, sizeof(EntryDev) * std::max<size_t>(ents.size(), 1))) != cudaSuccess)
         return cleanup(e, "cudaMalloc entries");
-    if ((e = cudaMalloc(&p->segs, sizeof(SegDev) * std::max<size_t>(sd.size(), 1))) != cudaSuccess)
-        return cleanup(e, "cudaMalloc segs");
-    if ((e = cudaMalloc(&p->cta_seg_begin, sizeof(int32_t) * cta_begin.size())) != cudaSuccess)
-        return cleanup(e, "cudaMalloc cta_seg_begin");
-    if ((e = cudaMalloc(&p->g_slot_begin, sizeof(int32_t) * g_slot.size())) != cudaSuccess)
-        return cleanup(e, "cudaMalloc g_slot_begin");
     if ((e = cudaMalloc(&p->chunks, sizeof(ChunkDev) * std::max<size_t>(chunks.size(), 1))) != cudaSuccess)
         return cleanup(e, "cudaMalloc chunks");
     if (!chunks.empty() && (e = cudaMemcpyAsync(p->chunks, chunks.data(), sizeof(ChunkDev) * chunks.size(),
@@ -627,7 +578,7 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
                                  stream)) != cudaSuccess)
             return cleanup(e, "copy reconstruction chunks");
     }
-    if ((e = cudaMalloc(&p->counters, cnt_bytes)) != cudaSuccess) return cleanup(e, "cudaMalloc counters");
+    if ((e = cudaMalloc(&p->acc, cnt_bytes)) != cudaSuccess) return cleanup(e, "cudaMalloc accumulators");
     if ((e = cudaMalloc(&p->status, sizeof(int32_t))) != cudaSuccess) return cleanup(e, "cudaMalloc status");
     if ((e = cudaMalloc(&loff_dev, sizeof(int64_t) * std::max<size_t>(loffs.size(), 1))) != cudaSuccess)
         return cleanup(e, "cudaMalloc offsets");
@@ -648,19 +599,10 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
         (e = cudaMemcpyAsync(p->entries, ents.data(), sizeof(EntryDev) * ents.size(), cudaMemcpyHostToDevice,
                              stream)) != cudaSuccess)
         return cleanup(e, "copy entries");
-    if (!sd.empty() && (e = cudaMemcpyAsync(p->segs, sd.data(), sizeof(SegDev) * sd.size(), cudaMemcpyHostToDevice,
-                                            stream)) != cudaSuccess)
-        return cleanup(e, "copy segs");
-    if ((e = cudaMemcpyAsync(p->cta_seg_begin, cta_begin.data(), sizeof(int32_t) * cta_begin.size(),
-                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
-        return cleanup(e, "copy cta_seg_begin");
-    if ((e = cudaMemcpyAsync(p->g_slot_begin, g_slot.data(), sizeof(int32_t) * g_slot.size(),
-                             cudaMemcpyHostToDevice, stream)) != cudaSuccess)
-        return cleanup(e, "copy g_slot_begin");
     if (!loffs.empty() && (e = cudaMemcpyAsync(loff_dev, loffs.data(), sizeof(int64_t) * loffs.size(),
                                                cudaMemcpyHostToDevice, stream)) != cudaSuccess)
         return cleanup(e, "copy offsets");
-    if ((e = cudaMemsetAsync(p->counters, 0, cnt_bytes, stream)) != cudaSuccess) return cleanup(e, "memset counters");
+    if ((e = cudaMemsetAsync(p->acc, 0, cnt_bytes, stream)) != cudaSuccess) return cleanup(e, "memset accumulators");
     if ((e = cudaMemsetAsync(p->status, 0, sizeof(int32_t), stream)) != cudaSuccess) return cleanup(e, "memset status");
     if ((e = launch_pack(table->arena, p->entries, loff_dev, (int)E, d, p->packed, p->packed_bytes, stream)) !=
         cudaSuccess)
@@ -679,9 +621,6 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t
     info->num_q_heads = plan->hq;
     info->head_dim = plan->d;
     info->max_batch = plan->max_batch;
-    info->num_ctas = plan->num_ctas;
-    info->num_segments = plan->num_segments;
-    info->num_slots = plan->num_slots;
     info->prefix_tokens = plan->prefix_tokens;
     info->logical_factor_bytes = plan->logical_bytes;
     info->packed_bytes = plan->packed_bytes;
@@ -691,9 +630,8 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t
 
 namespace {
 struct CallShape {
-    int rows_g, nrg, nrg_cta, npass, nrg_t, ngrp_t, npass_t, S;
+    int rows_g, nrg, nrg_t, S;  // query rows and row groups per KV head, row groups per query, tail splits
     int P;         // kTailTokens pieces per tail item
-    bool chunked;  // the chunk grid's accumulators and finish grid (paths 0 and 1)
     int path;      // milo_path_t
     int ntile;     // tensor-core path: row tiles per KV head
     const milo_prefix::TcPart *part;
@@ -709,38 +647,29 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     CallShape c;
     c.rows_g = batch * p->G;
     c.nrg = (c.rows_g + 7) / 8;
-    c.nrg_cta = c.nrg >= 2 ? 2 : 1;
-    c.npass = (c.nrg + c.nrg_cta - 1) / c.nrg_cta;
     c.nrg_t = (p->G + 7) / 8;
-    c.ngrp_t = c.nrg_t >= 2 ? 2 : 1;
-    c.npass_t = (c.nrg_t + c.ngrp_t - 1) / c.ngrp_t;
     // the chunk grid serves every call (a call without a prefix holds tail
     // items alone); its prefix part moves to the tensor cores from
     // kTcMinRows rows per KV head
-    c.chunked = true;
     c.ntile = 0;
     c.part = nullptr;
-    if (c.chunked && p->tc && c.rows_g >= kTcMinRows) {
+    if (p->tc && c.rows_g >= kTcMinRows) {
         c.ntile = (c.rows_g + kTcRows - 1) / kTcRows;
         c.part = p->tc_part(c.ntile);
     }
-    c.path = !c.chunked ? MILO_PATH_PERSISTENT : c.part ? MILO_PATH_TENSOR : MILO_PATH_CHUNKS;
+    c.path = c.part ? MILO_PATH_TENSOR : MILO_PATH_CHUNKS;
     if (!c.part) c.ntile = 0;
     // tail items: on the tensor-core path the chunk grid holds the tails
     // alone, and each item streams up to kTailPiecesLong pieces (fewer items,
-    // each merged once); beside prefix chunks, or in the persistent kernel,
-    // an item is one piece
+    // each merged once); beside prefix chunks an item is one piece
     c.P = c.path == MILO_PATH_TENSOR ? kTailPiecesLong : 1;
     c.S = max_tail > 0 ? (int)((max_tail + (int64_t)c.P * kTailTokens - 1) / ((int64_t)c.P * kTailTokens)) : 0;
-    // one record per prefix chunk and row group (the short-block decode), or
-    // per run and row group (the persistent kernel and the tensor-core grid);
-    // then the tail items.  The short-block decode and the tensor-core grid
-    // also list records: int4 [Hkv][nrg][list_cap], list_cap bounding the
+    // one record per prefix chunk and row group (the chunk grid), or per run
+    // and row group (the tensor-core grid); then the tail items.  Outlier
+    // records are listed: int4 [Hkv][nrg][list_cap], list_cap bounding the
     // items whose rows meet one row group: the KV head's chunks (or runs),
-    // and the tail items of the queries whose G rows meet the group's 8 rows
-    // [8k, 8k + 8), of which there are at most 7 / G + 2.
-    const int64_t prefix = c.part ? (int64_t)c.part->num_slots * c.nrg
-                           : c.chunked ? (int64_t)p->num_chunks * c.nrg : (int64_t)p->num_slots * c.nrg;
+    // and the tail items below.
+    const int64_t prefix = c.part ? (int64_t)c.part->num_slots * c.nrg : (int64_t)p->num_chunks * c.nrg;
     c.records = prefix + (int64_t)batch * p->hkv * c.S * c.nrg_t;
     // tail items (per split) whose 8 rows meet one row group: with G <= 8 an
     // item is one query's G rows, at most 7 / G + 2 queries meet 8 rows; with
@@ -749,11 +678,11 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     const int64_t queries_per_group =
         p->G <= 8 ? std::min<int64_t>(batch, 7 / p->G + 2) : std::min<int64_t>((int64_t)batch * c.nrg_t, 3);
     const int64_t prefix_items = c.part ? (int64_t)c.part->max_runs : (int64_t)p->max_head_chunks;
-    c.list_cap = c.chunked ? prefix_items + queries_per_group * c.S : 0;
+    c.list_cap = prefix_items + queries_per_group * c.S;
     c.list_bytes = 16 * (int64_t)p->hkv * c.nrg * c.list_cap;
     const int64_t tail_records = (int64_t)batch * p->hkv * c.S * c.nrg_t;
     c.records_rc = (int64_t)p->rc_num_chunks * c.nrg + tail_records;
-    c.list_cap_rc = c.chunked ? (int64_t)p->rc_max_head_chunks + queries_per_group * c.S : 0;
+    c.list_cap_rc = (int64_t)p->rc_max_head_chunks + queries_per_group * c.S;
     c.list_bytes_rc = 16 * (int64_t)p->hkv * c.nrg * c.list_cap_rc;
 
     return c;
@@ -806,40 +735,32 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
     if (cur != plan->device) return fail(MILO_ERR_INVALID_ARG, "plan belongs to another device");
 
     const CallShape c = call_shape(plan, batch, max_tail_tokens);
-    if (recon && (!c.chunked || plan->rc_num_chunks == 0))
+    if (recon && plan->rc_num_chunks == 0)
         return fail(MILO_ERR_UNSUPPORTED, "reconstruct-then-attend needs a prefix");
     if (recon && ((int64_t)plan->rc_num_chunks * c.nrg > 0x7fffffff || c.list_cap_rc > 0x7fffffff ||
                   (int64_t)plan->rc_num_chunks * ((c.rows_g + kRcRows - 1) / kRcRows) > 0x7fffffff))
         return fail(MILO_ERR_UNSUPPORTED, "call too large: more than 2^31 - 1 work items");
     // the kernels count thread blocks, tail items and list entries in int
-    const int64_t tail_items = (int64_t)batch * plan->hkv * c.S * (c.chunked ? c.nrg_t : 1);
-    // (the persistent path counts record slots per row group and its merge
-    // grid's blocks per KV head, row group and float4 column in int too)
+    const int64_t tail_items = (int64_t)batch * plan->hkv * c.S * c.nrg_t;
     if (tail_items > 0x7fffffff || (int64_t)plan->num_chunks * c.nrg + tail_items > 0x7fffffff ||
-        c.list_cap > 0x7fffffff || (int64_t)plan->num_slots * c.nrg + tail_items * c.nrg_t > 0x7fffffff ||
-        (int64_t)plan->hkv * c.nrg * (plan->d / 4) > 0x7fffffff)
+        c.list_cap > 0x7fffffff || (int64_t)plan->hkv * c.nrg > 0x7fffffff)
         return fail(MILO_ERR_UNSUPPORTED, "call too large: more than 2^31 - 1 work items");
     DecodeParams prm{};
     prm.packed = plan->packed;
     prm.entries = plan->entries;
-    prm.segs = plan->segs;
-    prm.cta_seg_begin = plan->cta_seg_begin;
-    prm.g_slot_begin = plan->g_slot_begin;
     prm.q = static_cast<const uint16_t *>(q);
     prm.tail_offsets = tail_offsets;
     prm.out = out;
     prm.rec = static_cast<float *>(workspace);
 
-    prm.counters = plan->counters;
-    if (c.chunked) {
-        // after CountersDev: reference maxima, list counts, then the 16-byte
-        // aligned sums and output accumulators
+    {
+        // reference maxima, list counts, then the 16-byte aligned sums and
+        // output accumulators
         const int H = plan->hkv, R = 8 * plan->max_nrg;
         prm.rows_max = R;
-        prm.acc_m = reinterpret_cast<uint32_t *>(plan->counters + 1);
+        prm.acc_m = reinterpret_cast<uint32_t *>(plan->acc);
         prm.ovf_cnt = prm.acc_m + (size_t)H * R;
-        uint8_t *base = reinterpret_cast<uint8_t *>(plan->counters);
-        prm.acc_l = reinterpret_cast<float *>(base + acc_l_offset(H, R));
+        prm.acc_l = reinterpret_cast<float *>(plan->acc + acc_l_offset(H, R));
         prm.acc_o = prm.acc_l + (size_t)H * R;
     }
     prm.status = plan->status;
@@ -850,17 +771,11 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
     prm.d = plan->d;
     prm.rows_g = c.rows_g;
     prm.nrg = c.nrg;
-    prm.nrg_cta = c.nrg_cta;
-    prm.npass = c.npass;
     prm.nrg_t = c.nrg_t;
-    prm.ngrp_t = c.ngrp_t;
-    prm.npass_t = c.npass_t;
-    prm.num_slots = plan->num_slots;
     prm.tail_splits = c.S;
     prm.tail_pieces = c.P;
     prm.num_tail_items = (int)tail_items;
     prm.has_tail = c.S > 0 ? 1 : 0;
-    prm.tail_rec_base = (int64_t)plan->num_slots * c.nrg;
     prm.tail_k = static_cast<const uint16_t *>(tail_k);
     prm.tail_v = static_cast<const uint16_t *>(tail_v);
     prm.chunks = plan->chunks;
@@ -871,7 +786,7 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
         prm.tc_ntile = c.ntile;
         prm.tc_nshare = c.part->nshare;
     }
-    if (c.chunked) {
+    {
         prm.tail_rec_base = c.part ? (int64_t)c.part->num_slots * c.nrg : (int64_t)plan->num_chunks * c.nrg;
         // the record lists follow the records
         prm.list_cap = (int)c.list_cap;
@@ -880,7 +795,6 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
     }
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)plan->d);
     prm.scale_log2 = scale * 1.4426950408889634f;
-    prm.num_ctas = plan->num_ctas;
 
     alignas(64) CUtensorMap mk, mv;
     std::memset(&mk, 0, sizeof mk);
@@ -890,15 +804,11 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
         if (!enc) return fail(MILO_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
         const cuuint64_t dims[3] = {(cuuint64_t)plan->d, (cuuint64_t)plan->hkv, (cuuint64_t)tail_rows};
         const cuuint64_t strides[2] = {(cuuint64_t)plan->d * 2, (cuuint64_t)plan->hkv * plan->d * 2};
-        // the chunk grid (its tail items, for every call with at most 8 query
-        // heads per KV head): boxes of 64 columns (128-byte rows, 128-byte
-        // swizzle), few wide requests; the persistent kernel: boxes of one
-        // 16-byte column chunk, landing as 8x8 cores [column group][token
-        // group] like a packed coefficient tile
-        const bool wide = c.chunked;
-        const cuuint32_t box[3] = {wide ? 64u : 8u, 1, (cuuint32_t)kTailTokens};
+        // the chunk grid's tail items: boxes of 64 columns (128-byte rows,
+        // 128-byte swizzle), few wide requests
+        const cuuint32_t box[3] = {64u, 1, (cuuint32_t)kTailTokens};
         const cuuint32_t estr[3] = {1, 1, 1};
-        const CUtensorMapSwizzle swz = wide ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE;
+        const CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B;
         CUresult r1 = enc(&mk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(tail_k), dims, strides, box,
                           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -942,16 +852,10 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
         if ((e = launch_finish(prm, stream)) != cudaSuccess) return cuda_fail(e, "finish grid launch");
         return MILO_OK;
     }
-    if (c.path == MILO_PATH_CHUNKS) {
-        // the prefix chunks and the tail items in one grid (tail items alone
-        // without a prefix), then the finish grid
-        cudaError_t e = launch_chunks(prm, &mk, &mv, stream);
-        if (e != cudaSuccess) return cuda_fail(e, "chunk grid launch");
-        return MILO_OK;
-    }
-    const int smem = decode_smem_bytes(plan->d, c.nrg_cta);
-    cudaError_t e = launch_decode(prm, &mk, &mv, smem, plan->num_ctas, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    // MILO_PATH_CHUNKS: the prefix chunks and the tail items in one grid
+    // (tail items alone without a prefix), then the finish grid
+    cudaError_t e = launch_chunks(prm, &mk, &mv, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "chunk grid launch");
     return MILO_OK;
 }
 }  // namespace
@@ -1061,15 +965,12 @@ milo_status_t milo_call_info(const milo_prefix_t *plan, int32_t batch, int64_t m
     if (c.path == MILO_PATH_TENSOR) {
         info->kernels = (c.S > 0 ? 1 : 0) + 2;
         info->blocks = c.part->nshare * c.ntile;
-    } else if (c.path == MILO_PATH_CHUNKS) {
-        info->kernels = 2;
-        const int rg = c.nrg >= 2 ? 2 : 1;
-        const int64_t tail_items = (int64_t)batch * plan->hkv * c.S * (c.chunked ? c.nrg_t : 1);
-        info->blocks = (int32_t)std::min<int64_t>(
-            (int64_t)plan->num_chunks * ((c.nrg + rg - 1) / rg) + (tail_items + rg - 1) / rg, 0x7fffffff);
     } else {
         info->kernels = 2;
-        info->blocks = plan->num_ctas;
+        const int rg = c.nrg >= 2 ? 2 : 1;
+        const int64_t tail_items = (int64_t)batch * plan->hkv * c.S * c.nrg_t;
+        info->blocks = (int32_t)std::min<int64_t>(
+            (int64_t)plan->num_chunks * ((c.nrg + rg - 1) / rg) + (tail_items + rg - 1) / rg, 0x7fffffff);
     }
     return MILO_OK;
 }

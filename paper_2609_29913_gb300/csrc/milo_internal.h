@@ -7,34 +7,10 @@
 
 namespace milo {
 
-constexpr int kTileTokens = 32;      // tokens per coefficient tile (and partition cut granularity)
-constexpr int kMmaWarps = 7;         // compute warps per decode thread block (8 warps in all:
-                                     // at most two per SM sub-partition, 255 registers each)
-constexpr int kThreads = 32 * (1 + kMmaWarps);  // + one producer warp
-constexpr int kSlots = 5;            // ring depth (fills in flight)
-constexpr int kSlotBytes = 32768;    // bytes per ring slot (one fill)
-constexpr int kHdrInts = 32;         // fill header (ints)
+constexpr int kTileTokens = 32;      // tokens per partition cut (the tensor-core grid's segments)
 constexpr int kTailTokens = 64;      // tokens per dense-tail work item (per piece of one)
 constexpr int kTailPiecesLong = 8;   // pieces per tail item when the chunk grid holds tails alone
 constexpr int kRecFloatsExtra = 16;  // m[8], l[8] after o[8][d] in a record
-
-// fill flags: a fill carries, in processing order, the previous segment's
-// P^V, up to two bases P^K of coming segments, the start of a segment, its
-// coefficient tiles, a tail item, the end marker
-enum : int { kHasPv = 1, kHasPk0 = 2, kHasPk1 = 4, kSegStart = 8, kHasC = 16, kTailFill = 32, kEndFill = 64 };
-// fill header words
-enum : int {
-    H_FLAGS,
-    H_PV_G, H_PV_RV8, H_PV_REC, H_PV_RUN, H_PV_PASS, H_PV_OFF,
-    H_PK_J, H_PK_G, H_PK_RK8, H_PK_PASS, H_PK_OFF,  // P^K part 0; part 1 follows with the same layout
-    H_PK1_J = H_PK_J + 5,
-    H_SS_J = H_PK1_J + 5, H_SS_PASS, H_SS_RK8,
-    H_C_OFF, H_T0, H_T1, H_RK8, H_RV8, H_TOK8,
-    H_QI, H_G, H_ITEM,
-    H_PV_SEG,
-    H_WORDS
-};
-static_assert(H_WORDS <= kHdrInts, "fill header size");
 
 // Per-(block, KV head) entry of the packed arena.
 struct EntryDev {
@@ -44,17 +20,10 @@ struct EntryDev {
     int32_t g;                               // KV head
 };
 
-// Prefix segment of the static partition.
+// Flags of a segment of the tensor-core grid's partition.
 enum : int32_t { kSegFirstOfRun = 1, kSegLastOfRun = 2 };
-struct SegDev {
-    int32_t entry;
-    int32_t t0, t1;    // token range within the block
-    int32_t slot;      // partial slot (run)
-    int32_t flags;
-    int32_t pad[3];
-};
 
-// One chunk of the short-block decode: tokens [t0, t1) of a prefix entry.
+// One chunk of the chunk grid: tokens [t0, t1) of a prefix entry.
 constexpr int kChunkBytes = 131072;   // coefficient bytes (C^K + C^V rows) per chunk
 constexpr int kChunkMaxTok = 1024;   // tokens per chunk
 struct ChunkDev {
@@ -91,46 +60,29 @@ constexpr int kRcTok = 64;
 constexpr int kRcRows = 128;
 constexpr int kRcChunkTiles = 4;
 
-// Device-side counters owned by a plan (zero between calls).
-struct CountersDev {
-    uint32_t tail_next;   // dynamic tail work counter
-    uint32_t ctas_done;   // thread blocks finished (resets tail_next)
-    uint32_t pad[30];
-};
-
 struct DecodeParams {
     const uint8_t *packed;
     const EntryDev *entries;
-    const SegDev *segs;
-    const int32_t *cta_seg_begin;   // [num_ctas + 1]
-    const int32_t *g_slot_begin;    // [Hkv + 1]
     const uint16_t *q;              // bf16 [batch, Hq, d]
     const int64_t *tail_offsets;    // [batch + 1] or null
     float *out;                     // [batch, Hq, d]
     float *rec;                     // workspace records
-    CountersDev *counters;
     int32_t *status;
     int batch, hq, hkv, G, d;
     int rows_g;                     // batch * G
     int nrg;                        // ceil(rows_g / 8)
-    int nrg_cta;                    // prefix row groups per pass (1 or 2)
-    int npass;                      // ceil(nrg / nrg_cta)
     int nrg_t;                      // tail row groups per query: ceil(G / 8)
-    int ngrp_t;                     // tail row groups per pass (1 or 2)
-    int npass_t;                    // ceil(nrg_t / ngrp_t)
-    int num_slots;                  // prefix record slots
     int tail_splits;                // S: tail items per (query, KV head)
     int tail_pieces;                // kTailTokens pieces per tail item (the chunk grid)
-    int num_tail_items;             // batch * Hkv * S
+    int num_tail_items;             // batch * Hkv * S * nrg_t
     int has_tail;
     int64_t tail_rec_base;          // first tail record index
     float scale_log2;               // softmax scale * log2(e)
-    int num_ctas;
-    const ChunkDev *chunks;         // short-block decode: the prefix chunks (KV-head-major)
-    int num_chunks;                 // 0: the persistent kernels run
+    const ChunkDev *chunks;         // the chunk grid's prefix chunks (KV-head-major)
+    int num_chunks;                 // prefix chunks in this call's chunk grid (0: tail items alone)
     const uint16_t *tail_k, *tail_v;  // bf16 [rows, Hkv, d] dense tails (or null)
     int rows_max;                   // accumulator rows per KV head: 8 ceil(max_batch G / 8)
-    float *acc_o;                   // [Hkv][rows_max][d]: per-row accumulators of the short-block decode
+    float *acc_o;                   // [Hkv][rows_max][d]: per-row accumulators of the call
     float *acc_l;                   // [Hkv][rows_max]
     uint32_t *acc_m;                // [Hkv][rows_max]: reference maxima (sign-flipped float bits; 0 = unset)
     uint32_t *ovf_cnt;              // [Hkv][nrg]: records listed per (KV head, row group)
@@ -164,15 +116,8 @@ cudaError_t launch_pack(const void *arena, const EntryDev *entries_dev,
                         int head_dim, uint8_t *packed, int64_t packed_bytes,
                         cudaStream_t stream);
 
-cudaError_t launch_decode(const DecodeParams &p, const void *tmap_k,
-                          const void *tmap_v, int smem_bytes, int num_ctas,
-                          cudaStream_t stream);
-
-int decode_smem_bytes(int head_dim, int nrg_cta);
-
-// The short-block decode (one thread block per prefix chunk and row group of
-// 8 query rows, and per tail item), then its finish grid; launch_decode calls
-// it when G <= 8.
+// The chunk grid (one thread block per prefix chunk and row group of 8 query
+// rows, and per tail item), then its finish grid.
 cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void *tmap_v, cudaStream_t stream);
 
 

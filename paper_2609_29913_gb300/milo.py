@@ -37,7 +37,7 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_prefix_offload", "milo_prefix_stage", "milo_quantize_int8", "milo_dequantize_int8",
            "milo_prefix_quantize_int8", "milo_prefix_storage_bytes"]
 
-PATH_NAMES = {0: "chunks", 1: "tensor", 2: "persistent"}
+PATH_NAMES = {0: "chunks", 1: "tensor"}
 
 
 class MiloError(RuntimeError):
@@ -71,8 +71,7 @@ class EncodeParamsC(ctypes.Structure):
 class PrefixInfoC(ctypes.Structure):
     _fields_ = [("num_blocks", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
                 ("num_q_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
-                ("max_batch", ctypes.c_int32), ("num_ctas", ctypes.c_int32),
-                ("num_segments", ctypes.c_int32), ("num_slots", ctypes.c_int32),
+                ("max_batch", ctypes.c_int32),
                 ("prefix_tokens", ctypes.c_int64), ("logical_factor_bytes", ctypes.c_int64),
                 ("packed_bytes", ctypes.c_int64), ("packed_arena", ctypes.c_void_p)]
 
@@ -185,27 +184,29 @@ def milo_packed_layout(table: HostTable):
     return offs[:table.num_entries * 4].reshape(-1, 4), int(total.value)
 
 
-def milo_partition_prefix(table: HostTable, num_ctas: int) -> dict:
+def milo_partition_prefix(table: HostTable, num_shares: int) -> dict:
+    """The tensor-core grid's partition over num_shares shares: entry, t0, t1,
+    slot per segment, share_begin, num_slots."""
     nseg, nslot = ctypes.c_int32(0), ctypes.c_int32(0)
     L = lib()
-    _check(L.milo_partition_prefix(ctypes.byref(table.c), int(num_ctas), 0, None, None, None,
+    _check(L.milo_partition_prefix(ctypes.byref(table.c), int(num_shares), 0, None, None, None,
                                    None, None, ctypes.byref(nseg), ctypes.byref(nslot)),
            "milo_partition_prefix")
     n = int(nseg.value)
     out = {k: np.zeros(max(n, 1), dtype=np.int32) for k in ("entry", "t0", "t1", "slot")}
-    cb = np.zeros(int(num_ctas) + 1, dtype=np.int32)
-    _check(L.milo_partition_prefix(ctypes.byref(table.c), int(num_ctas), n,
+    sb = np.zeros(int(num_shares) + 1, dtype=np.int32)
+    _check(L.milo_partition_prefix(ctypes.byref(table.c), int(num_shares), n,
                                    out["entry"].ctypes.data, out["t0"].ctypes.data,
                                    out["t1"].ctypes.data, out["slot"].ctypes.data,
-                                   cb.ctypes.data, None, None), "milo_partition_prefix")
+                                   sb.ctypes.data, None, None), "milo_partition_prefix")
     res = {k: v[:n] for k, v in out.items()}
-    res["cta_begin"] = cb
+    res["share_begin"] = sb
     res["num_slots"] = int(nslot.value)
     return res
 
 
 def milo_chunk_prefix(table: HostTable) -> dict:
-    """The short-block decode's work list: entry, t0, t1 per chunk."""
+    """The chunk grid's work list: entry, t0, t1 per chunk."""
     n = ctypes.c_int32(0)
     L = lib()
     _check(L.milo_chunk_prefix(ctypes.byref(table.c), 0, None, None, None, ctypes.byref(n)),
@@ -251,7 +252,7 @@ def milo_workspace_size(plan: int, batch: int, max_tail_tokens: int) -> int:
 
 
 def milo_call_info(plan: int, batch: int, max_tail_tokens: int) -> dict:
-    """How a call of this shape runs: path (0 chunks, 1 tensor, 2 persistent),
+    """How a call of this shape runs: path (0 chunks, 1 tensor),
     kernels per call, row tiles and main-grid blocks (host only)."""
     info = CallInfoC()
     _check(lib().milo_call_info(plan, int(batch), int(max_tail_tokens), ctypes.byref(info)),

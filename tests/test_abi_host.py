@@ -108,15 +108,18 @@ def test_packed_layout_sizes_and_alignment(milo):
     assert total - (flat[-1] + sizes[-1]) < 128
 
 
-@pytest.mark.parametrize("ctas", [1, 3, 7, 152, 1000])
+@pytest.mark.parametrize("shares", [1, 3, 7, 152, 1000])
 @pytest.mark.parametrize("shape", [
     ([512] * 64, "choice", 4, 128),
     ([7, 129, 1, 64, 65, 300], "rand", 2, 64),
     ([512] * 8, "rand", 1, 128),
 ])
-def test_partition_covers_every_token_once(milo, ctas, shape):
+def test_partition_covers_every_token_once(milo, shares, shape):
+    """The tensor-core grid's partition: every token of every entry in exactly
+    one segment, cut at 32-token boundaries; one slot per (share, KV-head
+    run), slots numbered in KV-head order."""
     bl, law, hkv, d = shape
-    rng = np.random.default_rng(len(bl) * 7 + ctas)
+    rng = np.random.default_rng(len(bl) * 7 + shares)
     nb = len(bl)
     if law == "choice":
         rk = rng.choice([16, 32, 64, 96, 128], size=nb * hkv)
@@ -124,7 +127,7 @@ def test_partition_covers_every_token_once(milo, ctas, shape):
         rk = rng.integers(0, d + 1, size=nb * hkv)
     rv = rng.integers(0, d + 1, size=nb * hkv)
     t = ht(milo, **table(bl, rk, rv, hkv=hkv, d=d))
-    part = milo.milo_partition_prefix(t, ctas)
+    part = milo.milo_partition_prefix(t, shares)
     cover = {}
     for e, t0, t1 in zip(part["entry"], part["t0"], part["t1"]):
         assert t0 % 32 == 0 and t0 < t1 <= bl[e // hkv]
@@ -134,14 +137,13 @@ def test_partition_covers_every_token_once(milo, ctas, shape):
             assert key not in cover
             cover[key] = 1
     assert len(cover) == sum(bl) * hkv
-    cb = part["cta_begin"]
-    assert cb[0] == 0 and cb[-1] == len(part["entry"]) and (np.diff(cb) >= 0).all()
-    # slots: one per (thread block, KV-head run), numbered in KV-head order
+    sb = part["share_begin"]
+    assert sb[0] == 0 and sb[-1] == len(part["entry"]) and (np.diff(sb) >= 0).all()
     slots = part["slot"]
     heads_of_slot = {}
-    for c in range(ctas):
+    for c in range(shares):
         prev = None
-        for s in range(cb[c], cb[c + 1]):
+        for s in range(sb[c], sb[c + 1]):
             g = int(part["entry"][s]) % hkv
             heads_of_slot.setdefault(int(slots[s]), set()).add(g)
             if prev is not None and g == prev[0]:
@@ -153,27 +155,37 @@ def test_partition_covers_every_token_once(milo, ctas, shape):
     assert part["num_slots"] == len(heads_of_slot)
 
 
-def test_partition_balances_bytes(milo):
+@pytest.mark.parametrize("shares", [19, 152])
+def test_partition_balances_cost(milo, shares):
+    """Each share's cost under the header's model (per 32-token tile of t8
+    tokens t8 x (64 + r16(r^k) + r16(r^v)), plus 60000 on an entry's first
+    tile), recounted from the segments, is at most total / shares plus the
+    largest single tile: a tile goes to the share holding its midpoint."""
     rng = np.random.default_rng(5)
     nb, hkv, d = 64, 4, 128
     rk = rng.choice([16, 32, 64, 96, 128], size=nb * hkv)
-    t = ht(milo, **table([512] * nb, rk, rk, hkv=hkv, d=d))
-    ctas = 152
-    part = milo.milo_partition_prefix(t, ctas)
-    r8 = lambda r: (r + 7) // 8 * 8
-    cost = np.zeros(ctas)
-    cb = part["cta_begin"]
-    for c in range(ctas):
-        for s in range(cb[c], cb[c + 1]):
-            e = part["entry"][s]
-            tok = part["t1"][s] - part["t0"][s]
-            # the header's cost model: factor bytes + 32 per token for the softmax;
-            # bases count once per block (a cut block's second reader hits L2)
-            cost[c] += tok * (r8(rk[e]) * 4 + 32)
-            cost[c] += r8(rk[e]) * d * 2 if part["t0"][s] == 0 else 0      # P^K
-            cost[c] += r8(rk[e]) * d * 2 if part["t1"][s] == 512 else 0    # P^V
-    mean = cost.mean()
-    assert cost.max() <= mean * 1.15, (cost.max(), mean)
+    rv = rng.choice([16, 32, 64, 96, 128], size=nb * hkv)
+    bl = [512] * nb
+    t = ht(milo, **table(bl, rk, rv, hkv=hkv, d=d))
+    part = milo.milo_partition_prefix(t, shares)
+    r16 = lambda r: (r + 15) // 16 * 16
+
+    def tile_cost(e, t0, n):
+        t8 = (min(n - t0, 32) + 7) // 8 * 8
+        return t8 * (64 + r16(rk[e]) + r16(rv[e])) + (60000 if t0 == 0 else 0)
+
+    cost = np.zeros(shares)
+    sb = part["share_begin"]
+    for c in range(shares):
+        for s in range(sb[c], sb[c + 1]):
+            e = int(part["entry"][s])
+            n = bl[e // hkv]
+            for t0 in range(int(part["t0"][s]), int(part["t1"][s]), 32):
+                cost[c] += tile_cost(e, t0, n)
+    total = sum(tile_cost(e, t0, bl[e // hkv]) for e in range(nb * hkv) for t0 in range(0, bl[e // hkv], 32))
+    assert cost.sum() == total
+    biggest = max(tile_cost(e, 0, 512) for e in range(nb * hkv))
+    assert cost.max() <= total / shares + biggest, (cost.max(), total / shares)
     assert (cost > 0).all()
 
 
@@ -184,7 +196,7 @@ def test_partition_balances_bytes(milo):
     ([50, 70, 2048, 1], "zero", 2, 64),
 ])
 def test_chunks_cover_every_token_once_within_budget(milo, shape):
-    """The short-block decode's work list (milo_chunk_prefix): KV-head-major,
+    """The chunk grid's work list (milo_chunk_prefix): KV-head-major,
     then block order; every token of every entry exactly once; ranges start
     on 32-token boundaries; each entry uses the fewest ranges whose rows fit
     the 128 KB budget (at most 1024 tokens), and its ranges are equal up to

@@ -66,6 +66,13 @@ CASES = {
     # empty) and 9 tail items (two to a block, the last alone), at d = 128
     "d128-odd-row-groups": (21, 3, 128, [512, 77, 300], (16, 64, 96, 128), 3, [5, 60, 1], True),
     "rank0": (4, 2, 64, [50, 70], (0,), 1, [3], True),
+    # G = 10 at batch 2 (20 rows, chunk grid): tail items of 8 and 2 rows
+    "g10-b2": (20, 2, 128, [130, 512, 7], (8, 64, 128), 2, [70, 129], True),
+    # G = 12 at batch 3 (36 rows: the tensor-core grid) with long tail items
+    # of 8 and 4 rows
+    "g12-b3-tensor": (24, 2, 64, [256, 300], (16, 33, 64), 3, [600, 0, 65], True),
+    # G = 12 without a prefix: a chunk grid of tail items alone
+    "g12-tail-only": (12, 1, 128, [], (8,), 2, [1, 200], False),
 }
 
 

@@ -50,8 +50,8 @@ def call_static(milo, pre, layer, toff, max_tail, out):
     # 32 query rows per KV head: the prefix on the tensor-core grid, whose run
     # records sit in the built-in scratch
     (16, 2, 128, [512, 300], (16, 64, 128), 4, [5, 64, 0, 130]),
-    # 20 query heads per KV head: the persistent decode and merge kernels,
-    # whose records also sit in the built-in scratch
+    # 20 query heads per KV head: three row groups per query on the chunk
+    # grid, whose records and lists also sit in the built-in scratch
     (40, 2, 128, [200, 64, 130], (16, 64, 128), 1, [70]),
 ])
 def test_static_scratch_matches_workspace_call(env, shape):
