@@ -497,7 +497,7 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
         torch.cuda.empty_cache()
         rec["int8"] = measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup,
                                    dist, dev, world, tokens, ms_step, rec.get("offload"), offload_check is not None,
-                                   ref0)
+                                   ref0, alg_bytes)
     if cpu_seconds > 0 and rank == 0 and world == 1 and host_layers:
         rec["cpu_baseline"] = cpu_baseline(host_layers, cpu_seconds)
     for p in plans:
@@ -621,7 +621,7 @@ def measure_offload(plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, step
 
 
 def measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup, dist, dev, world,
-                 tokens, ms_resident, offload_rec, check, ref0):
+                 tokens, ms_resident, offload_rec, check, ref0, alg_bytes):
     """The same step with every layer's factors held as INT8 (Sec. 5.3,
     Table 2; milo_prefix_quantize_int8), in two placements, each on plans
     built afresh from the same layers:
@@ -629,7 +629,9 @@ def measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, 
         kernel reads them over the chip-to-chip link and writes the bf16
         read-back into device buffer l % 2 on a copy stream, overlapped with
         the previous layer's decode (the structure of the bf16 offloaded step);
-      resident: codes in device memory, staged the same way from HBM.
+      resident: codes in device memory, staged the same way from HBM;
+      resident_direct: the same plans unstaged, the chunk grid reading the
+        codes itself (one decode per layer, half the factor bytes).
     One CUDA graph per step.  Parity: layer 0 against the oracle's attention
     over the oracle's INT8 read-back of the same factors; the distance to the
     bf16 result is the quantisation's effect."""
@@ -638,6 +640,7 @@ def measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, 
     L = cfg.layers
     rec = {"what": "MILO + INT8 (asymmetric, one bf16 minimum and step per 8x8 tile of a factor)"}
     layer0_bits = None
+    ref_q = None
     for mode, to_host in (("offloaded", True), ("resident", False)):
         plans = []
         for l in range(L):
@@ -702,6 +705,9 @@ def measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, 
                                  "how": "dequant_plan_kernel from device memory: reads codes and parameters "
                                         "(68 B per 128 B core), writes the bf16 core; all layers back to back"}
             r["vs_bf16_resident"] = ms_resident / ms
+            rec["resident_direct"] = measure_int8_direct(milo, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream,
+                                                         steps, warmup, dist, dev, world, tokens, ms_resident,
+                                                         alg_bytes, stored, ref_q, ref0)
         if mode == "offloaded" and layer0_bits is not None:
             milo_oracle.build()
             deq, _ = milo_int8.quantize_arena(arena=layer0_bits["arena"], **{
@@ -722,6 +728,52 @@ def measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, 
         torch.cuda.empty_cache()
     rec["reduction_vs_bf16_factors"] = rec["offloaded"]["bf16_bytes_per_step"] / rec["offloaded"]["stored_bytes_per_step"]
     return rec
+
+
+def measure_int8_direct(milo, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup, dist, dev,
+                        world, tokens, ms_resident, alg_bytes, stored, ref_q, ref0):
+    """The resident INT8 plans unstaged (milo_prefix_stage with no buffer):
+    each layer's decode is one chunk grid that reads the codes and group
+    parameters (68 B per 128-byte core) and reads them back in shared memory.
+    Algorithmic bytes: the bf16 step's, with the factors' true-rank bf16
+    bytes replaced by the INT8 bytes stored."""
+    import torch
+    L = len(plans)
+    for p in plans:
+        p.stage(None)
+    need = max(p.workspace_size(qs[0].shape[0], max_tail) for p in plans)
+    if ws.numel() < need:
+        ws = torch.empty(need, dtype=torch.uint8, device=dev)
+
+    def step(s):
+        for l in range(L):
+            plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=ws, stream=s)
+
+    ms_total, _ = time_graph(step, stream, steps, warmup, None)
+    for p in plans:
+        assert p.status() == 0, "device status word set during the INT8 direct timing"
+    ms = max_over_ranks(ms_total / steps, dist, dev)
+    logical = sum(int(p.info["logical_factor_bytes"]) for p in plans)
+    nbytes = alg_bytes - logical + stored
+    ach = nbytes / (ms * 1e-3) / 1e9
+    peak_gbs, _, peak_kind = peaks()
+    call = milo.milo_call_info(plans[0].plan, qs[0].shape[0], max_tail)
+    r = {"ms_per_step": ms, "value": replica_throughput(world, tokens, ms), "unit": UNIT,
+         "vs_bf16_resident": ms_resident / ms,
+         "path": "chunk grid reading INT8 codes (%s)" % milo.PATH_NAMES[call["path"]],
+         "gpu_launches": call["kernels"] * L * steps,
+         "roofline": {"bound": "hbm", "achieved": ach, "peak": peak_gbs, "unit": "GB/s", "frac": ach / peak_gbs,
+                      "peak_source": f"{peak_kind} copy bandwidth (hbm_gbs)", "bytes_per_step": nbytes,
+                      "how": "the bf16 step's algorithmic bytes with the factors' true-rank bf16 bytes "
+                             "replaced by the INT8 codes and parameters stored"}}
+    if ref_q is not None:
+        pc = parity_layer0(None, outs[0], ref_q)
+        if ref0 is not None:
+            got = outs[0].double().cpu().numpy()
+            pc["rel_l2_vs_bf16_factors"] = float(np.linalg.norm(got - ref0) / np.linalg.norm(ref0))
+        pc["what"] = "against the oracle's attention over its own INT8 read-back of layer 0's factors"
+        r["parity_check"] = pc
+    return r
 
 
 def measure_encode(cfg, W, milo, dev, reps=5, cpu_seconds=0.0):

@@ -41,6 +41,7 @@
 #include <type_traits>
 
 #include "milo.h"
+#include "milo_int8.cuh"
 #include "milo_internal.h"
 #include "milo_merge.cuh"
 #include "milo_ptx.cuh"
@@ -66,6 +67,11 @@ struct CLay {
     static constexpr int kX = kBar + 16;                        // per row group: m, l [kWarps][8], ref [8]
     static constexpr int kXStride = 16 * kWarpsOf<RG> + 8;      //   (words)
     static constexpr int kTotal = kX + (RG * kXStride * 4 + 15) / 16 * 16;
+    // reading an INT8 plan: per slot, a piece's parameter words (at most 256
+    // cores and 12 words of alignment)
+    static constexpr int kPrm = kTotal;
+    static constexpr int kPrmSlot = 1088;
+    static constexpr int kTotalQ8 = kPrm + 2 * kPrmSlot;
     static constexpr int kRanksPerPiece = kPieceBytes / (D * 2);  // P^K / P^V rows per piece
 };
 
@@ -90,6 +96,51 @@ __device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
     s.tpp = row_bytes > 0 ? max(1, kPieceBytes / row_bytes) : kChunkMaxTok / kTile;
     s.nc = (c.ntok + s.tpp * kTile - 1) / (s.tpp * kTile);
     return s;
+}
+
+// A piece of an INT8 plan read directly: up to two runs of consecutive cores
+// (a C piece: the C^K rows, then the C^V rows).  Each run's 64-byte code
+// groups land at the end of the slot, in order, and its parameter words in
+// the slot's parameter area, copied in aligned groups of four (the run's
+// first word at index core0 % 4 of its copy; run 1's copy follows run 0's).
+struct Q8Piece {
+    int64_t core0[2];  // first core of each run (packed byte offset / 128)
+    int n[2];          // cores of each run
+    int words[2];      // parameter words copied for each run (multiples of 4)
+    int rg0, rlim;     // P pieces: first rank group, and the rank from which rows read back 0
+};
+
+template <int D>
+__device__ __forceinline__ Q8Piece q8_piece(const ChunkDev &ch, const Pieces &ps, int k)
+{
+    Q8Piece q;
+    q.core0[1] = 0;
+    q.n[1] = 0;
+    q.rg0 = 0;
+    q.rlim = 1 << 30;  // C pieces: nothing to clear
+    if (k < ps.npk) {
+        const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, ch.nrk);
+        q.core0[0] = ch.pk / 128 + (int64_t)r0 * (D / 8);
+        q.n[0] = (r1 - r0) * (D / 8);
+        q.rg0 = r0;
+        q.rlim = ch.rk;
+    } else if (k < ps.npk + ps.nc) {
+        const int t0 = (k - ps.npk) * ps.tpp * kTile;
+        const int tg = (min(t0 + ps.tpp * kTile, ch.tok8) - t0) / 8;  // token groups
+        q.core0[0] = ch.ck / 128 + (int64_t)(t0 / 8) * ch.nrk;
+        q.n[0] = tg * ch.nrk;
+        q.core0[1] = ch.cv / 128 + (int64_t)(t0 / 8) * ch.nrv;
+        q.n[1] = tg * ch.nrv;
+    } else {
+        const int r0 = (k - ps.npk - ps.nc) * ps.rpp, r1 = min(r0 + ps.rpp, ch.nrv);
+        q.core0[0] = ch.pv / 128 + (int64_t)r0 * (D / 8);
+        q.n[0] = (r1 - r0) * (D / 8);
+        q.rg0 = r0;
+        q.rlim = ch.rv;
+    }
+#pragma unroll
+    for (int j = 0; j < 2; ++j) q.words[j] = q.n[j] ? ((int)(q.core0[j] & 3) + q.n[j] + 3) & ~3 : 0;
+    return q;
 }
 
 // KV head g, rows 8 rg .. 8 rg + 7, after every item: fold the listed
@@ -191,8 +242,9 @@ __device__ bool add_part(const DecodeParams &p, int g, int lane, int n0, const f
 // share every piece (RG = 2 for calls with several row groups per KV head).
 // A tail block holds RG tail items, one per group; with RG = 2 group i's
 // item sits in slot i, with RG = 1 its pieces alternate between the slots.  "warp" below is the
-// warp's index within its row group.
-template <int D, int RG>
+// warp's index within its row group.  Q8: the plan is held as INT8 codes,
+// read directly (p.q8_codes, p.q8_params).
+template <int D, int RG, bool Q8>
 __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     chunk_kernel(const __grid_constant__ DecodeParams p, const __grid_constant__ CUtensorMap tmap_k,
                  const __grid_constant__ CUtensorMap tmap_v)
@@ -252,6 +304,22 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     // piece k into slot k & 1 (thread 0)
     auto issue = [&](int k) {
         const uint32_t bar = bar0 + 8 * (k & 1), dst = smem_u32(smem) + (k & 1) * kPieceBytes;
+        if constexpr (Q8) {
+            // an INT8 plan: codes at the slot's end, parameters in its parameter area
+            const Q8Piece q = q8_piece<D>(ch, ps, k);
+            const uint32_t n = (uint32_t)(q.n[0] + q.n[1]);
+            const uint32_t cdst = dst + kPieceBytes - 64u * n;
+            const uint32_t pdst = smem_u32(smem) + L::kPrm + (k & 1) * L::kPrmSlot;
+            mbar_arrive_tx(bar, 64u * n + 4u * (uint32_t)(q.words[0] + q.words[1]));
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                if (q.n[j] == 0) continue;
+                bulk_g2s(cdst + (j ? 64u * q.n[0] : 0u), p.q8_codes + q.core0[j] * 64, 64u * q.n[j], bar);
+                bulk_g2s(pdst + (j ? 4u * q.words[0] : 0u), p.q8_params + (q.core0[j] & ~(int64_t)3),
+                         4u * q.words[j], bar);
+            }
+            return;
+        }
         if (k < ps.npk) {
             const int r0 = k * ps.rpp, r1 = min(r0 + ps.rpp, ch.nrk);
             const uint32_t b = (uint32_t)(r1 - r0) * D * 16;
@@ -443,10 +511,63 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     };
 
     const int np = ps.total();
+    // An INT8 piece in slot k & 1 becomes the bf16 cores the bf16 piece would
+    // be (every thread): core i at byte 128 i of the slot, its values read
+    // back as the staging kernel reads them (milo_int8.cuh), P rows past the
+    // rank set to 0 (C padding stays as read back: it meets q~ = 0 or p = 0
+    // only).  Eight neighbouring threads take the eight rows of a core (8
+    // code bytes in, 16 bytes out: no bank conflicts), kQ8Cores cores a
+    // round, each thread loading its rows' codes before the round's barrier
+    // and writing their values after it: the codes sit at the slot's end (64
+    // bytes per core, at most 256 cores), so a round's writes reach only
+    // codes of its own or earlier rounds.
+    auto q8_read = [&](int k) {
+        constexpr int kU = 4;                          // rows a thread takes per round
+        constexpr int kQ8Cores = kU * kThreads / 8;    // cores per round
+        const Q8Piece q = q8_piece<D>(ch, ps, k);
+        const int n = q.n[0] + q.n[1];
+        uint8_t *sb = smem + (k & 1) * kPieceBytes;
+        const int in0 = kPieceBytes - 64 * n;
+        const uint32_t *prm = reinterpret_cast<const uint32_t *>(smem + L::kPrm + (k & 1) * L::kPrmSlot);
+        const int pa = (int)(q.core0[0] & 3), pb = q.words[0] + (int)(q.core0[1] & 3) - q.n[0];
+        const int row = tid & 7;
+#pragma unroll 1
+        for (int b = 0; b < n; b += kQ8Cores) {
+            uint2 c[kU];
+            uint32_t pw[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int i = b + (tid >> 3) + u * (kThreads / 8);
+                if (i < n) {
+                    c[u] = *reinterpret_cast<const uint2 *>(sb + in0 + 64 * i + 8 * row);
+                    pw[u] = prm[i < q.n[0] ? pa + i : pb + i];
+                }
+            }
+            __syncthreads();
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int i = b + (tid >> 3) + u * (kThreads / 8);
+                if (i < n) {
+                    uint4 v = dequant_row(c[u], pw[u]);
+                    // P pieces: rank 8 (rg0 + i / (D / 8)) + row
+                    if (8 * (q.rg0 + i / (D / 8)) + row >= q.rlim) v = make_uint4(0u, 0u, 0u, 0u);
+                    *reinterpret_cast<uint4 *>(sb + 128 * i + 16 * row) = v;
+                }
+            }
+        }
+        // codes left past the values, within the 2 KB that a tile's reads
+        // can pass the data by, are cleared (two code bytes read as one bf16
+        // may be a NaN)
+        const int z1 = min(kPieceBytes, 128 * n + 4096);
+        for (int o = max(128 * n, in0) + 16 * tid; o < z1; o += 16 * kThreads)
+            *reinterpret_cast<uint4 *>(sb + o) = make_uint4(0u, 0u, 0u, 0u);
+        __syncthreads();
+    };
     // wait for piece k (every warp); afterwards release its slot and bring
     // piece k + 2 into it
     auto wait_piece = [&](int k) {
         mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
+        if constexpr (Q8) q8_read(k);
         return smem_u32(smem) + (k & 1) * kPieceBytes;
     };
     auto release_piece = [&](int k) {
@@ -798,27 +919,38 @@ __global__ void __launch_bounds__(32) finish_kernel(const __grid_constant__ Deco
 }  // namespace
 
 namespace {
-template <int D, int RG>
+template <int D, int RG, bool Q8>
 cudaError_t launch_chunk_grid(cudaLaunchConfig_t cfg, const DecodeParams &p, const CUtensorMap &mk,
                               const CUtensorMap &mv)
 {
     using L = CLay<D, RG>;
+    constexpr int kSmem = Q8 ? L::kTotalQ8 : L::kTotal;
     static bool configured[kMaxDevices] = {};
     const int dev = attribute_slot();
     if (dev < 0 || !configured[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(chunk_kernel<D, RG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             L::kTotal);
+        cudaError_t e = cudaFuncSetAttribute(chunk_kernel<D, RG, Q8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSmem);
         if (e != cudaSuccess) return e;
         // several thread blocks per SM need the largest shared-memory carveout
-        e = cudaFuncSetAttribute(chunk_kernel<D, RG>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        e = cudaFuncSetAttribute(chunk_kernel<D, RG, Q8>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
         if (e != cudaSuccess) return e;
         if (dev >= 0) configured[dev] = true;
     }
     const int nrgb = (p.nrg + RG - 1) / RG;
     cfg.gridDim = dim3(p.num_chunks * nrgb + (p.has_tail ? (p.num_tail_items + RG - 1) / RG : 0));
     cfg.blockDim = dim3(32 * kWarpsOf<RG> * RG);
-    cfg.dynamicSmemBytes = (size_t)L::kTotal;
-    return cudaLaunchKernelEx(&cfg, chunk_kernel<D, RG>, p, mk, mv);
+    cfg.dynamicSmemBytes = (size_t)kSmem;
+    return cudaLaunchKernelEx(&cfg, chunk_kernel<D, RG, Q8>, p, mk, mv);
+}
+
+template <int D, bool Q8>
+cudaError_t launch_chunk_grid_d(cudaLaunchConfig_t cfg, const DecodeParams &p, const CUtensorMap &mk,
+                                const CUtensorMap &mv)
+{
+    // two row groups per block once a KV head has more than 8 query rows
+    // (one when the grid holds long tail items alone)
+    const bool two = p.nrg >= 2 && p.tail_pieces <= 1;
+    return two ? launch_chunk_grid<D, 2, Q8>(cfg, p, mk, mv) : launch_chunk_grid<D, 1, Q8>(cfg, p, mk, mv);
 }
 }  // namespace
 
@@ -833,12 +965,12 @@ cudaError_t launch_chunks(const DecodeParams &p, const void *tmap_k, const void 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    // two row groups per block once a KV head has more than 8 query rows
-    // (one when the grid holds long tail items alone)
-    const bool two = p.nrg >= 2 && p.tail_pieces <= 1;
-    cudaError_t e = p.d == 64 ? (two ? launch_chunk_grid<64, 2>(cfg, p, mk, mv) : launch_chunk_grid<64, 1>(cfg, p, mk, mv))
-                              : (two ? launch_chunk_grid<128, 2>(cfg, p, mk, mv)
-                                     : launch_chunk_grid<128, 1>(cfg, p, mk, mv));
+    // (an INT8 plan read directly: the INT8 variant; its tail items are bf16)
+    const bool q8 = p.q8_codes != nullptr;
+    cudaError_t e = p.d == 64 ? (q8 ? launch_chunk_grid_d<64, true>(cfg, p, mk, mv)
+                                    : launch_chunk_grid_d<64, false>(cfg, p, mk, mv))
+                              : (q8 ? launch_chunk_grid_d<128, true>(cfg, p, mk, mv)
+                                    : launch_chunk_grid_d<128, false>(cfg, p, mk, mv));
     if (e != cudaSuccess) return e;
     // the tensor-core and reconstruct-then-attend calls launch their prefix
     // grid between the two

@@ -232,6 +232,8 @@ void build_chunks(const milo_block_table_t *t, const std::vector<int64_t> &poffs
         c.nrk = rk8 / 8;
         c.nrv = rv8 / 8;
         c.g = g;
+        c.rk = t->rank_k[e];
+        c.rv = t->rank_v[e];
         chunks.push_back(c);
         g_begin[(size_t)g + 1] = (int32_t)chunks.size();
     });
@@ -629,6 +631,10 @@ milo_status_t milo_prefix_get_info(const milo_prefix_t *plan, milo_prefix_info_t
 }
 
 namespace {
+// An INT8 plan in device memory that is not staged: the chunk grid reads its
+// codes directly.
+bool reads_int8(const milo_prefix_t *p) { return !p->packed && p->int8_store && !p->int8_host; }
+
 struct CallShape {
     int rows_g, nrg, nrg_t, S;  // query rows and row groups per KV head, row groups per query, tail splits
     int P;         // kTailTokens pieces per tail item
@@ -653,7 +659,7 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     // kTcMinRows rows per KV head
     c.ntile = 0;
     c.part = nullptr;
-    if (p->tc && c.rows_g >= kTcMinRows) {
+    if (p->tc && c.rows_g >= kTcMinRows && !reads_int8(p)) {
         c.ntile = (c.rows_g + kTcRows - 1) / kTcRows;
         c.part = p->tc_part(c.ntile);
     }
@@ -713,7 +719,8 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
     if (!plan || !q || !out) return fail(MILO_ERR_INVALID_ARG, "null plan, q or out");
     if (!recon && plan->rope_tile)
         return fail(MILO_ERR_UNSUPPORTED, "the plan holds pre-RoPE factors: use milo_attn_decode_reconstruct");
-    if (!plan->packed) return fail(MILO_ERR_INVALID_ARG, "the plan's arena is offloaded: stage it first (milo_prefix_stage)");
+    if (!plan->packed && !(reads_int8(plan) && !recon))
+        return fail(MILO_ERR_INVALID_ARG, "the plan's arena is offloaded: stage it first (milo_prefix_stage)");
     if (batch < 1 || batch > plan->max_batch) return fail(MILO_ERR_INVALID_ARG, "batch outside [1, max_batch]");
     if (max_tail_tokens < 0) return fail(MILO_ERR_INVALID_ARG, "max_tail_tokens < 0");
     if (plan->nb == 0 && max_tail_tokens == 0) return fail(MILO_ERR_INVALID_ARG, "no prefix and no tail");
@@ -747,6 +754,10 @@ milo_status_t decode_call(const milo_prefix_t *plan, const void *q, int32_t batc
         return fail(MILO_ERR_UNSUPPORTED, "call too large: more than 2^31 - 1 work items");
     DecodeParams prm{};
     prm.packed = plan->packed;
+    if (reads_int8(plan)) {
+        prm.q8_codes = plan->int8_dev;
+        prm.q8_params = reinterpret_cast<const uint32_t *>(plan->int8_dev + plan->packed_bytes / 2);
+    }
     prm.entries = plan->entries;
     prm.q = static_cast<const uint16_t *>(q);
     prm.tail_offsets = tail_offsets;
@@ -1131,7 +1142,14 @@ milo_status_t milo_prefix_offload(milo_prefix_t *plan)
 
 milo_status_t milo_prefix_stage(milo_prefix_t *plan, void *device_buffer, size_t bytes, void *stream)
 {
-    if (!plan || !device_buffer) return fail(MILO_ERR_INVALID_ARG, "null plan or buffer");
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    if (!device_buffer) {
+        // an INT8 plan in device memory goes back to reading its codes
+        if (!plan->int8_store || plan->int8_host)
+            return fail(MILO_ERR_INVALID_ARG, "null buffer (only an INT8 plan in device memory reads without one)");
+        plan->packed = nullptr;
+        return MILO_OK;
+    }
     if (!plan->packed_host && !plan->int8_store) return fail(MILO_ERR_INVALID_ARG, "the plan is not offloaded");
     if ((int64_t)bytes < plan->packed_bytes) return fail(MILO_ERR_INVALID_ARG, "staging buffer smaller than the arena");
     if (reinterpret_cast<uintptr_t>(device_buffer) % 128) return fail(MILO_ERR_ALIGNMENT, "staging buffer not 128-byte aligned");
@@ -1196,7 +1214,9 @@ milo_status_t milo_prefix_quantize_int8(milo_prefix_t *plan, int32_t to_host)
     cudaError_t e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return cuda_fail(e, "synchronize before quantising");
     const int64_t nbytes = plan->packed_bytes;
-    const size_t store = (size_t)std::max<int64_t>(nbytes / 2 + nbytes / 32, 128);
+    // (+16: the chunk grid copies parameter words in aligned groups of four,
+    // which may reach up to three words past the last)
+    const size_t store = (size_t)std::max<int64_t>(nbytes / 2 + nbytes / 32, 128) + 16;
     uint8_t *mem = nullptr;
     void *dev = nullptr;
     if (to_host) {

@@ -31,7 +31,8 @@ struct ChunkDev {
     int32_t ntok, tok8;         // tokens, and rows copied (rounded up to 8 within the entry)
     int32_t nrk, nrv;           // rank 8-groups of K and V
     int32_t g;                  // KV head
-    int32_t pad[3];
+    int32_t rk, rv;             // true ranks (the INT8 read zeroes P rows past them)
+    int32_t pad;
 };
 static_assert(sizeof(ChunkDev) == 64, "chunk descriptor size");
 
@@ -79,6 +80,8 @@ struct DecodeParams {
     int64_t tail_rec_base;          // first tail record index
     float scale_log2;               // softmax scale * log2(e)
     const ChunkDev *chunks;         // the chunk grid's prefix chunks (KV-head-major)
+    const uint8_t *q8_codes;        // INT8 plan read directly (packed is then null): core i's 64 codes
+    const uint32_t *q8_params;      //   at q8_codes + 64 i, its parameter word at q8_params[i]
     int num_chunks;                 // prefix chunks in this call's chunk grid (0: tail items alone)
     const uint16_t *tail_k, *tail_v;  // bf16 [rows, Hkv, d] dense tails (or null)
     int rows_max;                   // accumulator rows per KV head: 8 ceil(max_batch G / 8)

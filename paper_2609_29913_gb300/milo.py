@@ -489,7 +489,12 @@ class Prefix:
         """Enqueue the copy (an offloaded plan) or the dequantisation (an INT8
         plan) of the arena into ``buffer`` (a cuda uint8 tensor of at least
         info['packed_bytes'] bytes) on ``stream``; the following decode calls
-        read it there."""
+        read it there.  ``buffer`` None: an INT8 plan in device memory goes
+        back to reading its codes directly."""
+        if buffer is None:
+            _check(lib().milo_prefix_stage(self.plan, None, 0, _stream_ptr(stream)), "milo_prefix_stage")
+            self.info = milo_prefix_get_info(self.plan)
+            return
         _check(lib().milo_prefix_stage(self.plan, buffer.data_ptr(), buffer.numel() * buffer.element_size(),
                                        _stream_ptr(stream)), "milo_prefix_stage")
 

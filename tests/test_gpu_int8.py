@@ -5,6 +5,9 @@ INT8"), through the C ABI:
   and group parameters of the oracle's quantiser applied to the same factors
   (8 x 8 tiles of the logical C and P matrices, zero-padded), and
   milo_dequantize_int8 gives the oracle's read-back values bit for bit;
+- a plan held as INT8 in device memory decodes from its codes directly (the
+  chunk grid) like the oracle's attention over the read-back factors, and
+  like its staged decode;
 - a plan held as INT8 (device memory, or mapped pinned host memory read over
   the chip-to-chip link) and staged decodes like the oracle's attention over
   the read-back factors (max-abs 1e-2, relative L2 2e-3: the decode bar), on
@@ -179,8 +182,17 @@ def test_int8_plan_decodes_like_oracle(env, name, to_host):
     st = pre.storage()
     assert st == {"bytes": nbytes // 2 + nbytes // 32, "int8": True, "on_host": to_host}
     assert pre.info["packed_arena"] is None
-    with pytest.raises(milo.MiloError):
-        pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt)
+    if to_host:
+        # codes over the link are read only by the staging kernel
+        with pytest.raises(milo.MiloError):
+            pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt)
+    else:
+        # codes in device memory: the chunk grid reads them directly
+        assert env["milo"].milo_call_info(pre.plan, layer.batch, mt)["path"] == 0
+        direct = pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt)
+        torch.cuda.synchronize()
+        assert pre.status() == 0
+        compare(direct.cpu().numpy(), ref, f"{name} int8 read directly")
     buf = torch.full((nbytes + 256,), 0x7F, dtype=torch.uint8, device="cuda")
     pre.stage(buf)
     out = pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt)
@@ -188,6 +200,72 @@ def test_int8_plan_decodes_like_oracle(env, name, to_host):
     assert pre.status() == 0
     np.testing.assert_array_equal(buf[:nbytes].cpu().numpy().view(np.uint16), want)
     compare(out.cpu().numpy(), ref, f"{name} int8 host={to_host}")
+    if not to_host:
+        # the direct read gives the staged values: the same attention up to
+        # the order of the fp32 reductions
+        np.testing.assert_allclose(direct.cpu().numpy(), out.cpu().numpy(), rtol=1e-5, atol=1e-5)
+        pre.stage(None)
+        again = pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt)
+        torch.cuda.synchronize()
+        assert milo.milo_prefix_get_info(pre.plan)["packed_arena"] is None and pre.status() == 0
+        np.testing.assert_allclose(again.cpu().numpy(), direct.cpu().numpy(), rtol=1e-5, atol=1e-5)
+    else:
+        with pytest.raises(milo.MiloError):
+            pre.stage(None)                 # host codes are never read directly
+    pre.close()
+
+
+DIRECT = {
+    # name: (hq, hkv, d, block_lens, rank_choices, batch, tails)
+    # ranks 100 and 128 on both sides: full 32 KB pieces of 256 cores (codes
+    # left past the values are cleared), P rows past ranks 1, 13 and 100
+    "d128-full-pieces": (28, 4, 128, [512, 300, 64, 7, 1024], (0, 1, 13, 64, 100, 128), 2, [37, 0]),
+    # G = 12 over 36 rows (the tensor-core grid for a bf16 plan), d = 64
+    "d64-g12": (24, 2, 64, [129, 1, 65, 600], (1, 7, 8, 33, 64), 3, [5, 0, 90]),
+    # one query, no tail
+    "d128-b1-no-tail": (7, 1, 128, [2048, 33], (16, 96), 1, [0]),
+}
+
+
+@pytest.mark.parametrize("name", sorted(DIRECT))
+def test_int8_read_directly_matches_staged(env, name):
+    """An INT8 plan in device memory decoded by the chunk grid straight from
+    its codes (no staging) gives the oracle's attention over the read-back
+    factors, and the staged decode's output up to the order of the fp32
+    reductions; eager and graph-captured."""
+    milo = env["milo"]
+    hq, hkv, d, bl, ranks, batch, tails = DIRECT[name]
+    layer = env["W"].make_random_case(num_q_heads=hq, num_kv_heads=hkv, head_dim=d, block_lens=bl,
+                                      rank_choices=ranks, batch=batch, tail_lengths=tails, seed=31,
+                                      device="cuda", separate_kv_ranks=True)
+    ref = oracle_reference(env, layer)
+    pre = milo.Prefix.from_layer(layer)
+    toff = torch.as_tensor(layer.tail_offsets, device="cuda")
+    mt = int(np.diff(layer.tail_offsets).max())
+    pre.quantize_int8()
+    direct = pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt)
+    torch.cuda.synchronize()
+    assert pre.status() == 0
+    compare(direct.cpu().numpy(), ref, f"{name} read directly")
+    nbytes = int(pre.info["packed_bytes"])
+    buf = torch.full((nbytes + 256,), 0x7F, dtype=torch.uint8, device="cuda")
+    pre.stage(buf)
+    staged = pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt)
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(direct.cpu().numpy(), staged.cpu().numpy(), rtol=1e-5, atol=1e-5)
+    pre.stage(None)
+    out = torch.full_like(direct, float("nan"))
+    ws = torch.empty(pre.workspace_size(batch, mt), dtype=torch.uint8, device="cuda")
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt, out=out, workspace=ws, stream=s)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    assert pre.status() == 0
+    np.testing.assert_allclose(out.cpu().numpy(), direct.cpu().numpy(), rtol=1e-5, atol=1e-5)
     pre.close()
 
 
@@ -254,9 +332,13 @@ def test_int8_argument_errors(env):
     layer = W.make_random_case(num_q_heads=14, num_kv_heads=2, head_dim=128, block_lens=[128, 64],
                                rank_choices=(16, 32), batch=1, tail_lengths=[5], seed=3, device="cuda")
     pre = milo.Prefix.from_layer(layer)
+    with pytest.raises(milo.MiloError):
+        pre.stage(None)                     # a resident bf16 plan
     pre.offload()
     with pytest.raises(milo.MiloError):
         pre.quantize_int8()                 # offloaded bf16 plan
+    with pytest.raises(milo.MiloError):
+        pre.stage(None)                     # offloaded bf16 plans need a buffer
     pre.close()
     pre = milo.Prefix.from_layer(layer)
     pre.quantize_int8()
