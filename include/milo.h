@@ -371,9 +371,12 @@ milo_status_t milo_prefix_set_rope(milo_prefix_t *plan, double rope_theta,
  * let the copy of the next layer overlap the decode of this one.  A decode
  * call on an offloaded plan that was never staged returns
  * MILO_ERR_INVALID_ARG.  Staging is an ordinary asynchronous copy and can be
- * captured in a CUDA graph.  Errors: MILO_ERR_INVALID_ARG (null arguments,
- * a plan not (or already) offloaded, a buffer too small, another device
- * current), MILO_ERR_ALIGNMENT, MILO_ERR_CUDA.
+ * captured in a CUDA graph.  device_buffer NULL (bytes ignored): an INT8
+ * plan in device memory stops reading a staged buffer and reads its codes
+ * directly again (see milo_prefix_quantize_int8).  Errors:
+ * MILO_ERR_INVALID_ARG (null plan, a plan not offloaded, a buffer too small,
+ * a NULL buffer for any other plan, another device current),
+ * MILO_ERR_ALIGNMENT, MILO_ERR_CUDA.
  */
 milo_status_t milo_prefix_offload(milo_prefix_t *plan);
 milo_status_t milo_prefix_stage(milo_prefix_t *plan, void *device_buffer, size_t bytes,
@@ -414,14 +417,19 @@ milo_status_t milo_dequantize_int8(const void *codes, const void *params, int64_
  * milo_prefix_quantize_int8 replaces a plan's resident bf16 arena with its
  * INT8 form (codes then params in one allocation: device memory when
  * to_host = 0, mapped pinned host memory when to_host = 1, the offloaded
- * INT8 prefix) and frees the bf16 arena; it synchronises the device.  The
- * plan's decode calls then need milo_prefix_stage: for an INT8 plan it
+ * INT8 prefix) and frees the bf16 arena; it synchronises the device.
+ * With the codes in device memory, milo_attn_decode reads them directly:
+ * the chunk grid (MILO_PATH_CHUNKS, whatever the batch) copies each piece's
+ * codes and parameters and reads them back in shared memory, as the
+ * staging kernel below would (milo_attn_decode_reconstruct needs a staged
+ * plan).  Any INT8 plan can instead be staged with milo_prefix_stage: it
  * enqueues on `stream` one kernel that reads the codes (over NVLink-C2C for
  * host storage) and writes the bf16 values read back, with every factor's
  * padding (ranks past r, tokens past n_b) set to 0, into the caller's
  * buffer (as for an offloaded plan: at least packed_bytes, 128-byte
- * aligned, held until the decode calls that read it are done).  Decode
- * calls then compute attention over those values.  milo_prefix_storage_bytes
+ * aligned, held until the decode calls that read it are done); decode
+ * calls then compute attention over those values on any path.  Host-held
+ * codes are read only by staging.  milo_prefix_storage_bytes
  * gives the bytes the plan's arena occupies at rest (bf16 or INT8, wherever
  * it is).  Errors: MILO_ERR_INVALID_ARG (null plan, the plan already
  * offloaded or quantised, another device current), MILO_ERR_CUDA.

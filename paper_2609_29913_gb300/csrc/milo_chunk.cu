@@ -1,9 +1,9 @@
-// milo_chunk.cu -- the split-K decode for up to 8 query heads per KV head
-// (G <= 8): one thread block of four warps per chunk and row group of 8
-// query rows (batch x G rows per KV head), or of two warps per row group and
-// a pair of row groups once a KV head has more than 8 rows; three blocks per
-// SM at head dimension 128.  Each chunk is streamed through two
-// shared-memory slots that all the block's warps read.
+// milo_chunk.cu -- the chunk grid: the split-K decode with one thread block
+// of four warps per chunk and row group of 8 query rows (8 of the batch x G
+// rows of a KV head), or of two warps per row group and a pair of row groups
+// once a KV head has more than 8 rows; three blocks per SM at head dimension
+// 128.  Each chunk is streamed through two shared-memory slots that all the
+// block's warps read.
 //
 // A chunk is a token range of one prefix entry (block b, KV head g).  Its
 // block walks a fixed sequence of pieces, each at most kPieceBytes and
@@ -23,7 +23,12 @@
 //                (Alg. 1 Stage 2's back-projection), after the warps' v~ are
 //                merged; each warp produces a share of the head dimension.
 //
-// A dense-tail item (one query's tail for one KV head: 1, or tail_pieces when the grid holds tails
+// A plan held as INT8 codes in device memory is read directly by a variant
+// (Q8) that copies each piece's codes and group parameters and reads them
+// back into bf16 cores in shared memory before the steps above.
+//
+// A dense-tail item (the tail of one query and KV head for the query's G
+// rows, or 8 of them when G > 8: 1, or tail_pieces when the grid holds tails
 // alone, pieces of kTailTokens tokens) brings each piece's K and V rows with 3-D TMA boxes (64 head
 // dimensions x kTailTokens rows each, 128-byte rows with the 128-byte swizzle: few, wide requests)
 // and runs the C steps on them with q~ = scale * log2(e) * q, a share of the
@@ -50,6 +55,7 @@ namespace milo {
 namespace {
 
 constexpr int kPieceBytes = 32768;  // one slot
+constexpr int kQ8Raw = 16384;       // reading an INT8 plan: one piece's codes (at most 256 cores)
 constexpr int kTile = 32;           // tokens per tile
 // warps per row group of 8 query rows: four when a block holds one row
 // group (more warps in flight on each SM's three blocks), two when it holds
@@ -100,7 +106,7 @@ __device__ __forceinline__ Pieces pieces_of(const ChunkDev &c)
 
 // A piece of an INT8 plan read directly: up to two runs of consecutive cores
 // (a C piece: the C^K rows, then the C^V rows).  Each run's 64-byte code
-// groups land at the end of the slot, in order, and its parameter words in
+// groups land in the piece's raw slot, in order, and its parameter words in
 // the slot's parameter area, copied in aligned groups of four (the run's
 // first word at index core0 % 4 of its copy; run 1's copy follows run 0's).
 struct Q8Piece {
@@ -305,12 +311,11 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     auto issue = [&](int k) {
         const uint32_t bar = bar0 + 8 * (k & 1), dst = smem_u32(smem) + (k & 1) * kPieceBytes;
         if constexpr (Q8) {
-            // an INT8 plan: codes at the slot's end, parameters in its parameter area
+            // an INT8 plan: codes in raw slot k & 1, parameters in its parameter area
             const Q8Piece q = q8_piece<D>(ch, ps, k);
-            const uint32_t n = (uint32_t)(q.n[0] + q.n[1]);
-            const uint32_t cdst = dst + kPieceBytes - 64u * n;
+            const uint32_t cdst = smem_u32(smem) + (k & 1) * kQ8Raw;
             const uint32_t pdst = smem_u32(smem) + L::kPrm + (k & 1) * L::kPrmSlot;
-            mbar_arrive_tx(bar, 64u * n + 4u * (uint32_t)(q.words[0] + q.words[1]));
+            mbar_arrive_tx(bar, 64u * (uint32_t)(q.n[0] + q.n[1]) + 4u * (uint32_t)(q.words[0] + q.words[1]));
 #pragma unroll
             for (int j = 0; j < 2; ++j) {
                 if (q.n[j] == 0) continue;
@@ -511,66 +516,54 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
     };
 
     const int np = ps.total();
-    // An INT8 piece in slot k & 1 becomes the bf16 cores the bf16 piece would
-    // be (every thread): core i at byte 128 i of the slot, its values read
+    // Reading an INT8 plan (Q8), shared memory holds two raw slots of
+    // kQ8Raw bytes at the start (the codes of pieces k & 1) and one bf16
+    // slot after them, where each piece becomes the bf16 cores the bf16
+    // piece would be (every thread): core i at byte 128 i, its values read
     // back as the staging kernel reads them (milo_int8.cuh), P rows past the
     // rank set to 0 (C padding stays as read back: it meets q~ = 0 or p = 0
     // only).  Eight neighbouring threads take the eight rows of a core (8
-    // code bytes in, 16 bytes out: no bank conflicts), kQ8Cores cores a
-    // round, each thread loading its rows' codes before the round's barrier
-    // and writing their values after it: the codes sit at the slot's end (64
-    // bytes per core, at most 256 cores), so a round's writes reach only
-    // codes of its own or earlier rounds.
+    // code bytes in, 16 bytes out: no bank conflicts).  The raw slot is free
+    // again once the piece is read back, so piece k + 2 is requested then,
+    // before the tiles run.  A tile's reads past the values (at most 2 KB)
+    // land in the q~ area that follows the bf16 slot.
     auto q8_read = [&](int k) {
-        constexpr int kU = 4;                          // rows a thread takes per round
-        constexpr int kQ8Cores = kU * kThreads / 8;    // cores per round
         const Q8Piece q = q8_piece<D>(ch, ps, k);
         const int n = q.n[0] + q.n[1];
-        uint8_t *sb = smem + (k & 1) * kPieceBytes;
-        const int in0 = kPieceBytes - 64 * n;
+        const uint8_t *raw = smem + (k & 1) * kQ8Raw;
+        uint8_t *vals = smem + kPieceBytes;
         const uint32_t *prm = reinterpret_cast<const uint32_t *>(smem + L::kPrm + (k & 1) * L::kPrmSlot);
         const int pa = (int)(q.core0[0] & 3), pb = q.words[0] + (int)(q.core0[1] & 3) - q.n[0];
         const int row = tid & 7;
-#pragma unroll 1
-        for (int b = 0; b < n; b += kQ8Cores) {
-            uint2 c[kU];
-            uint32_t pw[kU];
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                const int i = b + (tid >> 3) + u * (kThreads / 8);
-                if (i < n) {
-                    c[u] = *reinterpret_cast<const uint2 *>(sb + in0 + 64 * i + 8 * row);
-                    pw[u] = prm[i < q.n[0] ? pa + i : pb + i];
-                }
-            }
-            __syncthreads();
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                const int i = b + (tid >> 3) + u * (kThreads / 8);
-                if (i < n) {
-                    uint4 v = dequant_row(c[u], pw[u]);
-                    // P pieces: rank 8 (rg0 + i / (D / 8)) + row
-                    if (8 * (q.rg0 + i / (D / 8)) + row >= q.rlim) v = make_uint4(0u, 0u, 0u, 0u);
-                    *reinterpret_cast<uint4 *>(sb + 128 * i + 16 * row) = v;
-                }
-            }
+#pragma unroll 4
+        for (int i = tid >> 3; i < n; i += kThreads / 8) {
+            const uint2 c = *reinterpret_cast<const uint2 *>(raw + 64 * i + 8 * row);
+            uint4 v = dequant_row(c, prm[i < q.n[0] ? pa + i : pb + i]);
+            // P pieces: rank 8 (rg0 + i / (D / 8)) + row
+            if (8 * (q.rg0 + i / (D / 8)) + row >= q.rlim) v = make_uint4(0u, 0u, 0u, 0u);
+            *reinterpret_cast<uint4 *>(vals + 128 * i + 16 * row) = v;
         }
-        // codes left past the values, within the 2 KB that a tile's reads
-        // can pass the data by, are cleared (two code bytes read as one bf16
-        // may be a NaN)
-        const int z1 = min(kPieceBytes, 128 * n + 4096);
-        for (int o = max(128 * n, in0) + 16 * tid; o < z1; o += 16 * kThreads)
-            *reinterpret_cast<uint4 *>(sb + o) = make_uint4(0u, 0u, 0u, 0u);
+        // the raw slot's reads before its next copy (async proxy), the values
+        // before the tiles
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncthreads();
+        if (tid == 0 && k + 2 < np) issue(k + 2);
     };
     // wait for piece k (every warp); afterwards release its slot and bring
     // piece k + 2 into it
     auto wait_piece = [&](int k) {
         mbar_wait(bar0 + 8 * (k & 1), (k >> 1) & 1, p.status);
-        if constexpr (Q8) q8_read(k);
+        if constexpr (Q8) {
+            q8_read(k);
+            return smem_u32(smem) + (uint32_t)kPieceBytes;
+        }
         return smem_u32(smem) + (k & 1) * kPieceBytes;
     };
     auto release_piece = [&](int k) {
+        if constexpr (Q8) {
+            __syncthreads();  // the bf16 slot's reads before the next read-back
+            return;
+        }
         // the slot's reads are ordered before the async-proxy write
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncthreads();
@@ -793,7 +786,9 @@ __global__ void __launch_bounds__(32 * kWarpsOf<RG> * RG, 3)
         static_assert(RG * kXV <= kPieceBytes, "warp values fit a slot");
         static_assert(L::kRanksPerPiece >= D, "P^V of any rank is one piece");
         const float sc = exp2_diff(m_w, M);
-        const int free_slot = (ps.npk + ps.nc - 1) & 1;
+        // (reading an INT8 plan: the bf16 slot, whose next read-back, of
+        // P^V, comes after the exchange)
+        const int free_slot = Q8 ? 1 : (ps.npk + ps.nc - 1) & 1;
         float4 *xv = reinterpret_cast<float4 *>(smem + (is_tail ? grp * kPieceBytes
                                                                 : free_slot * kPieceBytes + grp * kXV));
         if (warp > 0) {
