@@ -1,6 +1,7 @@
 """GPU parity of the tensor-core path (calls with at least
-milo_tensor_min_rows() query rows per KV head and at most 8 query heads per
-KV head) against the fp64 oracle, through the C ABI.
+milo_tensor_min_rows() query rows per KV head) against the fp64 oracle,
+through the C ABI.  (Its cases with more than 8 query heads per KV head,
+G = 12 and 32, sit in test_gpu_parity.py.)
 
 The cases put the row count at the path's threshold and across a 128-row
 tile boundary, run calls of one tile of at most 64 rows (spread 16 per
