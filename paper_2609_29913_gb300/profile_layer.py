@@ -1,7 +1,7 @@
 """Run decode calls on the first layers of a named workload, for profilers.
 
   python -m paper_2609_29913_gb300.profile_layer --workload qwen7b-1L-1M-b8 \
-      [--layers 1] [--calls 3] [--reconstruct [--rope-theta 1e6]] [--int8 device|host]
+      [--layers 1] [--calls 3] [--reconstruct [--rope-theta 1e6]] [--int8 device|host|direct]
 
 Builds the plans of layers 0 .. layers-1 of the workload (seeded synthetic
 inputs, as the benchmark draws them), then makes `calls` rounds of one
@@ -13,7 +13,9 @@ regex:batch_tc -s 1 -c 1 skips the first round's launch).  With
 recon_kernel), with --rope-theta over pre-RoPE factors.  With --int8 the
 plans hold their factors as INT8 codes (device memory or mapped host
 memory) and every call is preceded by its staging kernel
-(dequant_plan_kernel) into one device buffer.  It keeps the device
+(dequant_plan_kernel) into one device buffer; with --int8 direct the codes
+stay in device memory and the chunk grid reads them itself (chunk_kernel's
+INT8 variant, no staging).  It keeps the device
 footprint to the chosen layers, well under the full workload's.
 """
 from __future__ import annotations
@@ -31,7 +33,7 @@ def main(argv=None) -> int:
     ap.add_argument("--calls", type=int, default=3)
     ap.add_argument("--reconstruct", action="store_true")
     ap.add_argument("--rope-theta", type=float, default=0.0)
-    ap.add_argument("--int8", choices=("device", "host"), default=None)
+    ap.add_argument("--int8", choices=("device", "host", "direct"), default=None)
     args = ap.parse_args(argv)
 
     import torch
@@ -52,7 +54,9 @@ def main(argv=None) -> int:
     if args.int8:
         for pre in plans:
             pre.quantize_int8(to_host=args.int8 == "host")
-        buf = torch.empty(max(int(p.info["packed_bytes"]) for p in plans) + 128, dtype=torch.uint8, device="cuda")
+        if args.int8 != "direct":
+            buf = torch.empty(max(int(p.info["packed_bytes"]) for p in plans) + 128, dtype=torch.uint8,
+                              device="cuda")
     max_tail = max(int(np.diff(L.tail_offsets).max()) for L in layers)
     for _ in range(args.calls):
         for L, pre, toff in zip(layers, plans, toffs):

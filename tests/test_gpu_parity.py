@@ -105,6 +105,23 @@ def test_small_cases_match_oracle(env, name):
     pre.close()
 
 
+@pytest.mark.parametrize("batch", [1, 5])
+def test_longest_block(env, batch):
+    """A block of 65536 tokens (the longest a table accepts) at ranks 128 and
+    16 beside a 3-token block, at batch 1 (7 rows: the chunk grid, the long
+    entry cut into chunks of at most 1024 tokens) and batch 5 (35 rows: the
+    tensor-core grid, the entry cut at 32-token boundaries over the shares)."""
+    milo, W = env["milo"], env["W"]
+    layer = W.build_layer(7, 1, 128, [65536, 3], [[128], [8]], [[16], [5]], batch=batch,
+                          tail_lengths=[70 + 3 * i for i in range(batch)], seed=65, device="cuda")
+    out, pre = decode(env, layer)
+    mt = int(np.diff(layer.tail_offsets).max())
+    assert milo.milo_call_info(pre.plan, batch, mt)["path"] == (0 if batch == 1 else 1)
+    ref = env["oracle"].attention(**layer.to_numpy_bits())
+    compare(out.cpu().numpy(), ref, f"longest block, batch {batch}")
+    pre.close()
+
+
 def test_peaked_softmax(env):
     layer = env["W"].make_random_case(num_q_heads=14, num_kv_heads=2, head_dim=128,
                                       block_lens=[512, 77, 512], rank_choices=(16, 64, 128),
