@@ -66,6 +66,8 @@ def parse(argv=None):
     ap.add_argument("--no-recon", action="store_true",
                     help="skip timing the reconstruct-then-attend path beside the rank-space path")
     ap.add_argument("--no-encode", action="store_true", help="skip timing the compression stage")
+    ap.add_argument("--no-paths", action="store_true",
+                    help="skip timing each workload on the other decode path (chunk grid / tensor-core grid)")
     ap.add_argument("--no-offload", action="store_true", help="skip timing the offloaded prefix")
     ap.add_argument("--no-int8", action="store_true", help="skip timing the INT8-stored factors")
     return ap.parse_args(argv)
@@ -351,7 +353,7 @@ def time_graph(step, stream, steps, warmup, flush):
 
 
 def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, check=True,
-            e2e=False, cpu_seconds=0.0, recon=False, offload=False, int8=False):
+            e2e=False, cpu_seconds=0.0, recon=False, offload=False, int8=False, paths=False):
     """Time one workload (all its layers per step) and return its record."""
     import torch
     plans, qs, tks, tvs, toffs = [], [], [], [], []
@@ -472,6 +474,9 @@ def measure(cfg, W, milo, dev, steps, warmup, dist=None, rank=0, world=1, *, che
         "gpu_launches": call["kernels"] * L * steps,
         "clocks": clocks.summary(), "parity_check": check, "setup_s": t_gen,
     }
+    if paths:
+        rec["other_path"] = measure_other_path(milo, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps,
+                                               warmup, flush, dist, dev, world, tokens, ms_step, call["path"], ref0)
     if recon:
         rec["reconstruct_then_attend"] = measure_recon(cfg, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream,
                                                       steps, warmup, flush, dist, dev, world, tokens, ms_step,
@@ -730,6 +735,44 @@ def measure_int8(cfg, W, milo, qs, tks, tvs, toffs, outs, ws, max_tail, stream, 
     return rec
 
 
+def measure_other_path(milo, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup, flush, dist,
+                       dev, world, tokens, ms_default, path_default, ref0):
+    """The same step on the other decode path, chosen per plan with
+    milo_prefix_set_tensor_min_rows (the chunk grid for a workload that takes
+    the tensor-core grid, and the reverse), timed the same way; the plans go
+    back to the default threshold afterwards."""
+    import torch
+    other = 1 - path_default
+    for p in plans:
+        p.set_tensor_min_rows(1 if other == 1 else 1 << 30)
+    try:
+        batch = qs[0].shape[0]
+        need = max(p.workspace_size(batch, max_tail) for p in plans)
+        wsx = ws if ws.numel() >= need else torch.empty(need, dtype=torch.uint8, device=dev)
+        L = len(plans)
+
+        def step(s):
+            for l in range(L):
+                plans[l].decode(qs[l], tks[l], tvs[l], toffs[l], max_tail, out=outs[l], workspace=wsx, stream=s)
+
+        ms_total, _ = time_graph(step, stream, steps, warmup, flush)
+        for p in plans:
+            assert p.status() == 0, "device status word set on the other path"
+        ms = max_over_ranks(ms_total / steps, dist, dev)
+        call = milo.milo_call_info(plans[0].plan, batch, max_tail)
+        assert call["path"] == other
+        r = {"path": {0: "chunk grid (mma.sync)", 1: "tensor-core batched grid (tcgen05)"}[other],
+             "ms_per_step": ms, "value": replica_throughput(world, tokens, ms), "unit": UNIT,
+             "default_speedup": ms / ms_default, "gpu_launches": call["kernels"] * L * steps,
+             "how": "milo_prefix_set_tensor_min_rows on every plan, one CUDA graph a step as for the default path"}
+        if ref0 is not None:
+            r["parity_check"] = parity_layer0(None, outs[0], ref0)
+        return r
+    finally:
+        for p in plans:
+            p.set_tensor_min_rows(milo.milo_tensor_min_rows())
+
+
 def measure_int8_direct(milo, plans, qs, tks, tvs, toffs, outs, ws, max_tail, stream, steps, warmup, dist, dev,
                         world, tokens, ms_resident, alg_bytes, stored, ref_q, ref0):
     """The resident INT8 plans unstaged (milo_prefix_stage with no buffer):
@@ -959,7 +1002,7 @@ def main():
     head = measure(cfg, W, milo, dev, args.steps, args.warmup, dist, rank, world, check=not args.no_check,
                    e2e=True, cpu_seconds=0.0 if args.no_cpu else args.cpu_seconds,
                    recon=not args.no_recon and cfg.name in RECON_WORKLOADS, offload=not args.no_offload,
-                   int8=not args.no_int8)
+                   int8=not args.no_int8, paths=not args.no_paths)
     others = []
     if not args.only:
         for k, other in enumerate(W.CONFIGS):
@@ -967,7 +1010,8 @@ def main():
                 continue
             others.append(measure(other, W, milo, dev, args.steps, args.warmup, dist, rank, world,
                                   check=not args.no_check,
-                                  recon=not args.no_recon and other.name in RECON_WORKLOADS))
+                                  recon=not args.no_recon and other.name in RECON_WORKLOADS,
+                                  paths=not args.no_paths))
     if not args.no_encode and rank == 0:
         head["encode"] = measure_encode(cfg, W, milo, dev, cpu_seconds=0.0 if args.no_cpu else 4.0)
     roof = dict(head["roofline"])
@@ -986,6 +1030,7 @@ def main():
         "cpu_baseline": head.get("cpu_baseline"),
         "e2e": head["e2e"], "gpu_launches": head["gpu_launches"], "clocks": head["clocks"],
         "parity_check": head["parity_check"], "path": head["path"], "setup_s": head["setup_s"],
+        "other_path": head.get("other_path"),
         "reconstruct_then_attend": head.get("reconstruct_then_attend"),
         "encode": head.get("encode"),
         "offload": head.get("offload"),

@@ -220,8 +220,8 @@ milo_status_t milo_workspace_size(const milo_prefix_t *plan, int32_t batch,
  *            or no prefix: then the grid holds the tail items alone);
  *            MILO_PATH_TENSOR (1): the tensor-core grid (tcgen05, 128 query
  *            rows per product) for the prefix, with the dense tails on the
- *            chunk grid (at least milo_tensor_min_rows() query rows per KV
- *            head).
+ *            chunk grid (at least the plan's threshold of query rows per KV
+ *            head: milo_tensor_min_rows() unless set, see below).
  *   kernels  kernel launches of one call (each a grid).
  *   row_tiles  tensor-core path: tiles of 128 query rows per KV head (else 0).
  *   blocks   thread blocks of the call's main prefix grid.
@@ -239,8 +239,21 @@ milo_status_t milo_call_info(const milo_prefix_t *plan, int32_t batch,
                              int64_t max_tail_tokens, milo_call_info_t *info);
 
 /* Query rows per KV head (batch x query heads per KV head) from which a
- * call takes the tensor-core path. */
+ * call takes the tensor-core path, by default. */
 int32_t milo_tensor_min_rows(void);
+
+/*
+ * Set a plan's threshold (host only): its calls with at least `rows` query
+ * rows per KV head take the tensor-core path, the others the chunk grid
+ * (rows = 1: every call with a prefix on the tensor cores; a value above
+ * max_batch x G: never).  Both paths compute the same attention; the
+ * threshold only chooses the faster, so it is a tuning and testing knob.
+ * It applies to calls enqueued after it returns, and milo_workspace_size
+ * and milo_call_info follow it (the workspace a call needs depends on its
+ * path).  An INT8 plan read directly always takes the chunk grid.
+ * Errors: MILO_ERR_INVALID_ARG for a null plan or rows < 1.
+ */
+milo_status_t milo_prefix_set_tensor_min_rows(milo_prefix_t *plan, int32_t rows);
 
 /*
  * One decode-attention call for one layer (Alg. 1 Stage 2 + Eq. 1):

@@ -293,7 +293,8 @@ struct milo_prefix {
     uint8_t *acc = nullptr;            // the chunk grid's per-row accumulators (zero between calls)
     int32_t *status = nullptr;
     // tensor-core path: one partition per share count a call can use
-    bool tc = false;                  // calls with at least kTcMinRows rows per KV head may take it
+    bool tc = false;                  // the tensor-core partitions exist (a plan with a prefix)
+    int tc_min_rows = kTcMinRows;     // calls with at least this many rows per KV head take them
     struct TcPart {
         int nshare, seg0, num_slots, max_runs;  // segments at tc_segs + seg0, shares at tc_cta + cta0
         int cta0;
@@ -511,7 +512,7 @@ milo_status_t milo_prefix_create(const milo_block_table_t *table, int32_t num_q_
     // tensor-core path: a partition for every share count sms / ntile that a
     // call with ntile row tiles of kTcRows rows per KV head uses
     p->sms = sms;
-    p->tc = !chunks.empty() && (int64_t)max_batch * G >= kTcMinRows;
+    p->tc = !chunks.empty();
     std::vector<TcSegDev> tc_sd;
     std::vector<int32_t> tc_cb;
     if (p->tc) {
@@ -659,7 +660,7 @@ CallShape call_shape(const milo_prefix_t *p, int batch, int64_t max_tail)
     // kTcMinRows rows per KV head
     c.ntile = 0;
     c.part = nullptr;
-    if (p->tc && c.rows_g >= kTcMinRows && !reads_int8(p)) {
+    if (p->tc && c.rows_g >= p->tc_min_rows && !reads_int8(p)) {
         c.ntile = (c.rows_g + kTcRows - 1) / kTcRows;
         c.part = p->tc_part(c.ntile);
     }
@@ -987,6 +988,14 @@ milo_status_t milo_call_info(const milo_prefix_t *plan, int32_t batch, int64_t m
 }
 
 int32_t milo_tensor_min_rows(void) { return kTcMinRows; }
+
+milo_status_t milo_prefix_set_tensor_min_rows(milo_prefix_t *plan, int32_t rows)
+{
+    if (!plan) return fail(MILO_ERR_INVALID_ARG, "null plan");
+    if (rows < 1) return fail(MILO_ERR_INVALID_ARG, "rows < 1");
+    plan->tc_min_rows = rows;
+    return MILO_OK;
+}
 
 milo_status_t milo_attn_decode_static(const milo_prefix_t *plan, const void *q, int32_t batch,
                                       const void *tail_k, const void *tail_v, const int64_t *tail_offsets,

@@ -32,6 +32,7 @@ EXPORTS = ["milo_status_string", "milo_version", "milo_last_error_message",
            "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
            "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
            "milo_get_device_status", "milo_call_info", "milo_tensor_min_rows",
+           "milo_prefix_set_tensor_min_rows",
            "milo_attn_decode_reconstruct", "milo_prefix_set_rope", "milo_check_bounded_wait",
            "milo_encode_layout", "milo_encode_workspace_size", "milo_encode",
            "milo_prefix_offload", "milo_prefix_stage", "milo_quantize_int8", "milo_dequantize_int8",
@@ -118,10 +119,12 @@ def lib():
         L.milo_get_device_status.argtypes = [P, P, i32, P]
         L.milo_call_info.argtypes = [P, i32, i64, P]
         L.milo_tensor_min_rows.restype = i32
+        L.milo_prefix_set_tensor_min_rows.argtypes = [P, i32]
         for name in ("milo_validate_table", "milo_packed_layout", "milo_partition_prefix",
                      "milo_chunk_prefix", "milo_prefix_create", "milo_prefix_destroy", "milo_prefix_get_info",
                      "milo_workspace_size", "milo_attn_decode", "milo_attn_decode_static",
                      "milo_get_device_status", "milo_call_info", "milo_attn_decode_reconstruct",
+                     "milo_prefix_set_tensor_min_rows",
                      "milo_prefix_set_rope", "milo_check_bounded_wait", "milo_encode_layout",
                      "milo_encode_workspace_size", "milo_encode", "milo_prefix_offload", "milo_prefix_stage",
                      "milo_quantize_int8", "milo_dequantize_int8", "milo_prefix_quantize_int8",
@@ -469,6 +472,11 @@ class Prefix:
             for t in made:
                 t.record_stream(stream)
         return out
+
+    def set_tensor_min_rows(self, rows: int) -> None:
+        """Calls with at least ``rows`` query rows per KV head take the
+        tensor-core path (milo_prefix_set_tensor_min_rows)."""
+        _check(lib().milo_prefix_set_tensor_min_rows(self.plan, int(rows)), "milo_prefix_set_tensor_min_rows")
 
     def offload(self) -> None:
         """Move the packed arena to pinned host memory (milo_prefix_offload)."""

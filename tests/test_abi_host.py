@@ -311,3 +311,12 @@ def test_int8_entry_points_check_arguments_on_the_host(milo):
     assert L.milo_prefix_quantize_int8(None, 0) == 1
     b = ctypes.c_int64(0)
     assert L.milo_prefix_storage_bytes(None, ctypes.byref(b), None, None) == 1
+
+
+def test_tensor_threshold_setter_rejects_bad_arguments(milo):
+    """milo_prefix_set_tensor_min_rows: a null plan is an argument error
+    (a plan needs a device, so the rest is tested on the GPU)."""
+    L = milo.lib()
+    assert L.milo_prefix_set_tensor_min_rows(None, 1) == 1
+    assert L.milo_prefix_set_tensor_min_rows(None, 0) == 1
+    assert L.milo_tensor_min_rows() == 32

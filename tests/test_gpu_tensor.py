@@ -173,6 +173,38 @@ def test_tensor_path_repeated_and_graph_captured(env):
     pre.close()
 
 
+@pytest.mark.parametrize("shape", [
+    # (hq, hkv, d, block_lens, rank_choices, batch, tails)
+    (28, 4, 128, [512, 300, 7], (0, 16, 64, 128), 1, [256]),    # 7 rows: the chunk grid by default
+    (8, 8, 64, [129, 64], (1, 33, 64), 1, [5]),                  # 1 row per KV head (G = 1)
+    (24, 2, 64, [200, 65], (8, 40, 64), 2, [70, 0]),             # G = 12: 24 rows, 8-row tail items
+    (28, 4, 128, [128, 64], (16, 128), 64, [33] * 64),           # 448 rows: the tensor-core grid by default
+])
+def test_forced_paths_match_oracle_and_each_other(env, shape):
+    """The same call on both paths (milo_prefix_set_tensor_min_rows): the
+    chunk grid and the tensor-core grid each match the oracle, and each
+    other, whatever the row count."""
+    milo, W = env["milo"], env["W"]
+    hq, hkv, d, bl, ranks, batch, tails = shape
+    layer = W.make_random_case(num_q_heads=hq, num_kv_heads=hkv, head_dim=d, block_lens=bl, rank_choices=ranks,
+                               batch=batch, tail_lengths=tails, seed=zlib.crc32(repr(shape).encode()) % 1000,
+                               device="cuda", separate_kv_ranks=True)
+    ref = env["oracle"].attention(**layer.to_numpy_bits())
+    pre = milo.Prefix.from_layer(layer)
+    toff = torch.as_tensor(layer.tail_offsets, device="cuda")
+    mt = int(np.diff(layer.tail_offsets).max())
+    outs = {}
+    for path, rows in ((0, 1 << 30), (1, 1)):
+        pre.set_tensor_min_rows(rows)
+        assert milo.milo_call_info(pre.plan, batch, mt)["path"] == path
+        outs[path] = pre.decode(layer.q, layer.tail_k, layer.tail_v, toff, mt).cpu().numpy()
+        torch.cuda.synchronize()
+        assert pre.status(clear=True) == 0
+        compare(outs[path], ref, f"{shape} path {path}")
+    np.testing.assert_allclose(outs[0], outs[1], rtol=0, atol=1e-4)
+    pre.close()
+
+
 def test_call_paths(env):
     """The path milo_call_info reports for each row count of one plan."""
     milo, W = env["milo"], env["W"]
