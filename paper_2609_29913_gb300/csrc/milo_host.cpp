@@ -341,7 +341,7 @@ const char *milo_status_string(int32_t s)
     }
 }
 
-int32_t milo_version(void) { return 100; }
+int32_t milo_version(void) { return 200; }
 
 const char *milo_last_error_message(void) { return g_last_error.c_str(); }
 
