@@ -197,7 +197,8 @@ typedef struct {
     int64_t logical_factor_bytes; /* bytes of C^K,P^K,C^V,P^V at true ranks   */
     int64_t packed_bytes;         /* bytes of the packed arena (with padding) */
     const void *packed_arena;     /* device pointer to the packed arena (an   */
-                                  /* offloaded plan: the staged copy, or NULL) */
+                                  /* offloaded or INT8 plan: the staged copy, */
+                                  /* or NULL)                                 */
 } milo_prefix_info_t;
 
 milo_status_t milo_prefix_get_info(const milo_prefix_t *plan,
@@ -281,9 +282,11 @@ milo_status_t milo_prefix_set_tensor_min_rows(milo_prefix_t *plan, int32_t rows)
  * `stream` finishes, and reads q, the tails and the workspace only after it
  * has; the last combines and writes `out`.  A plan holding pre-RoPE factors
  * (milo_prefix_set_rope) is refused with MILO_ERR_UNSUPPORTED: rank-space
- * scoring cannot apply a per-position rotation.  A plan must not be used by
- * two calls that can run concurrently (it
- * holds per-call accumulators).  A query whose prefix and tail
+ * scoring cannot apply a per-position rotation.  An offloaded plan must be
+ * staged first (MILO_ERR_INVALID_ARG otherwise); an INT8 plan in device
+ * memory that is not staged is read from its codes (milo_prefix_quantize_int8).
+ * A plan must not be used by two calls that can run concurrently (it holds
+ * per-call accumulators).  A query whose prefix and tail
  * are both empty yields NaN.  A call with more than 2^31 - 1 work items
  * (prefix chunks x row groups plus tail items) returns MILO_ERR_UNSUPPORTED
  * without launching anything.
