@@ -82,3 +82,16 @@ def test_damaged_files_are_refused(tmp_path):
             store.load_prefix(damaged(tmp_path, L, _raw=raw))
     with pytest.raises(ValueError):
         store.save_prefix(tmp_path / "x.npz", **L.table_arrays(), arena=np.zeros(8, dtype=np.float32))
+
+
+def test_empty_prefix_round_trip(tmp_path):
+    """A table without blocks (a call that attends to tails only) saves and
+    loads as empty arrays of the right types."""
+    path = tmp_path / "empty.npz"
+    z32, z64 = np.zeros(0, np.int32), np.zeros(0, np.int64)
+    store.save_prefix(path, num_kv_heads=2, head_dim=128, block_len=z32, rank_k=z32, rank_v=z32, off_ck=z64,
+                      off_pk=z64, off_cv=z64, off_pv=z64, arena=np.zeros(0, np.uint16))
+    got = store.load_prefix(path)
+    assert got["num_kv_heads"] == 2 and got["head_dim"] == 128
+    assert got["block_len"].dtype == np.int32 and got["off_pv"].dtype == np.int64
+    assert all(got[k].size == 0 for k in ("block_len", "rank_k", "off_ck", "arena"))
