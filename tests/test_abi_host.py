@@ -320,3 +320,54 @@ def test_tensor_threshold_setter_rejects_bad_arguments(milo):
     assert L.milo_prefix_set_tensor_min_rows(None, 1) == 1
     assert L.milo_prefix_set_tensor_min_rows(None, 0) == 1
     assert L.milo_tensor_min_rows() == 32
+
+
+def covers_exactly(entries, t0s, t1s, bl, hkv, cut):
+    """Every entry's tokens [0, n) covered once by the ranges of that entry,
+    in order, each starting on a multiple of `cut` (the last ends at n)."""
+    by = {}
+    for e, a, b in zip(entries, t0s, t1s):
+        by.setdefault(int(e), []).append((int(a), int(b)))
+    assert set(by) == set(range(len(bl) * hkv))
+    for e, rs in by.items():
+        n = bl[e // hkv]
+        assert rs[0][0] == 0 and rs[-1][1] == n, (e, rs[:2], rs[-1])
+        for (a0, b0), (a1, b1) in zip(rs, rs[1:]):
+            assert b0 == a1 and a0 < b0
+        assert all(a % cut == 0 and a < b for a, b in rs)
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_work_lists_of_random_tables(milo, seed):
+    """Random tables (1 to 12 blocks of 1 to 2000 tokens, 1 to 4 KV heads,
+    d = 64 or 128, ranks 0 to d, K and V apart): the chunk grid's list and
+    the tensor-core partition for a random share count both cover every
+    token of every entry exactly once, in KV-head-major order, cut at
+    32-token boundaries; no share costs more than its part of the cost line
+    plus one tile."""
+    rng = np.random.default_rng(1000 + seed)
+    nb, hkv, d = int(rng.integers(1, 13)), int(rng.integers(1, 5)), int(rng.choice([64, 128]))
+    bl = [int(x) for x in rng.integers(1, 2001, size=nb)]
+    rk = rng.integers(0, d + 1, size=nb * hkv)
+    rv = rng.integers(0, d + 1, size=nb * hkv)
+    t = ht(milo, **table(bl, rk, rv, hkv=hkv, d=d))
+    ch = milo.milo_chunk_prefix(t)
+    covers_exactly(ch["entry"], ch["t0"], ch["t1"], bl, hkv, 32)
+    heads = np.asarray(ch["entry"]) % hkv
+    assert np.all(np.diff(heads) >= 0)                      # KV-head-major
+    shares = int(rng.integers(1, 200))
+    part = milo.milo_partition_prefix(t, shares)
+    covers_exactly(part["entry"], part["t0"], part["t1"], bl, hkv, 32)
+    r16 = lambda r: (int(r) + 15) // 16 * 16
+    cost = np.zeros(shares)
+    sb = part["share_begin"]
+    biggest = 0
+    for c in range(shares):
+        for s in range(sb[c], sb[c + 1]):
+            e = int(part["entry"][s])
+            n = bl[e // hkv]
+            for a in range(int(part["t0"][s]), int(part["t1"][s]), 32):
+                tc = ((min(n - a, 32) + 7) // 8 * 8) * (64 + r16(rk[e]) + r16(rv[e])) + (60000 if a == 0 else 0)
+                cost[c] += tc
+                biggest = max(biggest, tc)
+    assert cost.max() <= cost.sum() / shares + biggest
