@@ -85,5 +85,8 @@ def prefix_from_file(path, num_q_heads: int, max_batch: int, stream=None):
     arena = torch.from_numpy(d.pop("arena").view(np.int16)).to("cuda").view(torch.bfloat16)
     table = milo.HostTable(**d, arena_ptr=arena.data_ptr(), arena_elems=int(arena.numel()))
     pre = milo.Prefix(table, num_q_heads, max_batch, stream)
+    # the plan holds its packed copy; the table no longer points at the arena
+    table.c.arena = None
+    table.c.arena_elems = 0
     del arena
     return pre
